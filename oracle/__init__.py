@@ -1,0 +1,206 @@
+"""CPU oracle for the integer-only quantized linear layer (MobileQuant, arXiv 2408.13933).
+
+TEST INFRASTRUCTURE ONLY: the test suite, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline leg are the only callers.  The product path (the CUDA
+library and its Python binding) never imports this package.
+
+The arithmetic lives in plain C (``mq_oracle.c``); this module compiles it
+with gcc and marshals numpy arrays through ctypes.  Function-by-function
+citations of the paper are in ``mq_oracle.h``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "mq_oracle.c")
+_HDR = os.path.join(_HERE, "mq_oracle.h")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+OK, EINVAL, EOVERFLOW = 0, 1, 2
+
+
+def build(force: bool = False) -> str:
+    """Compile liboracle.so with gcc (-O2, no vectorisation flags, one thread)."""
+    newest = max(os.path.getmtime(_SRC), os.path.getmtime(_HDR))
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < newest:
+        tmp = _LIB + ".tmp.%d" % os.getpid()
+        subprocess.check_call(
+            ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-Wall", "-Wextra",
+             "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _bind(lib):
+    p = ctypes.c_void_p
+    i32, i64, f32, ci = ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_int
+    lib.oracle_requant_params.argtypes = [f32, p, ci, f32, p, p]
+    lib.oracle_pack.argtypes = [p, ci, ci, ci, p, p]
+    lib.oracle_unpack.argtypes = [p, ci, ci, ci, p]
+    lib.oracle_linear.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci, p]
+    lib.oracle_linear_points.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci, p, p]
+    lib.oracle_requant_one.argtypes = [i64, i32, i32, i32]
+    lib.oracle_requant_one.restype = i32
+    lib.oracle_residual_add.argtypes = [p, p, i64, p]
+    lib.oracle_residual_add.restype = None
+    return lib
+
+
+def _ptr(a: np.ndarray):
+    assert a.flags["C_CONTIGUOUS"], "oracle arrays must be C-contiguous"
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def _check(rc: int, what: str):
+    if rc != OK:
+        raise OracleError(f"{what} failed with oracle code {rc}")
+
+
+class Oracle:
+    """numpy front end over one compiled copy of the C oracle."""
+
+    def __init__(self, lib_path: str):
+        self.lib = _bind(ctypes.CDLL(lib_path))
+
+    def requant_params(self, sx: float, sw: np.ndarray, sy: float):
+        """Per-channel (M0, shift) with M0 * 2^-shift ~= sx*sw[n]/sy (see header)."""
+        sw = np.ascontiguousarray(sw, dtype=np.float32)
+        n = sw.shape[0]
+        m0 = np.zeros(n, np.int32)
+        sh = np.zeros(n, np.int32)
+        _check(self.lib.oracle_requant_params(float(sx), _ptr(sw), n, float(sy), _ptr(m0),
+                                              _ptr(sh)), "oracle_requant_params")
+        return m0, sh
+
+    def pack(self, w: np.ndarray, bits: int):
+        """Pack int8 values [N, K] -> (packed uint8, colsum int32)."""
+        w = np.ascontiguousarray(w, dtype=np.int8)
+        n, k = w.shape
+        packed = np.zeros((n, k if bits == 8 else k // 2), np.uint8)
+        colsum = np.zeros(n, np.int32)
+        _check(self.lib.oracle_pack(_ptr(w), n, k, bits, _ptr(packed), _ptr(colsum)),
+               "oracle_pack")
+        return packed, colsum
+
+    def unpack(self, packed: np.ndarray, n: int, k: int, bits: int) -> np.ndarray:
+        packed = np.ascontiguousarray(packed, dtype=np.uint8)
+        w = np.zeros((n, k), np.int8)
+        _check(self.lib.oracle_unpack(_ptr(packed), n, k, bits, _ptr(w)), "oracle_unpack")
+        return w
+
+    def linear(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
+               m0: np.ndarray, shift: np.ndarray, zy: int, want_acc: bool = False):
+        """Full integer linear layer: returns y int8 [M, N] (and acc int32 [M, N])."""
+        x = np.ascontiguousarray(x, dtype=np.int8)
+        m, k = x.shape
+        packed = np.ascontiguousarray(packed, dtype=np.uint8)
+        m0 = np.ascontiguousarray(m0, dtype=np.int32)
+        shift = np.ascontiguousarray(shift, dtype=np.int32)
+        y = np.zeros((m, n), np.int8)
+        acc = np.zeros((m, n), np.int32) if want_acc else None
+        _check(self.lib.oracle_linear(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
+                                      _ptr(m0), _ptr(shift), int(zy), _ptr(y), n,
+                                      _ptr(acc) if acc is not None else None),
+               "oracle_linear")
+        return (y, acc) if want_acc else y
+
+    def linear_points(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
+                      m0: np.ndarray, shift: np.ndarray, zy: int, pts: np.ndarray):
+        """The layer at listed (m, n) coordinates only: returns (y[i], acc[i])."""
+        x = np.ascontiguousarray(x, dtype=np.int8)
+        m, k = x.shape
+        pts = np.ascontiguousarray(pts, dtype=np.int64).reshape(-1, 2)
+        cnt = pts.shape[0]
+        y = np.zeros(cnt, np.int8)
+        acc = np.zeros(cnt, np.int32)
+        packed = np.ascontiguousarray(packed, dtype=np.uint8)
+        m0 = np.ascontiguousarray(m0, dtype=np.int32)
+        shift = np.ascontiguousarray(shift, dtype=np.int32)
+        _check(self.lib.oracle_linear_points(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
+                                             _ptr(m0), _ptr(shift), int(zy), _ptr(pts), cnt,
+                                             _ptr(y), _ptr(acc)),
+               "oracle_linear_points")
+        return y, acc
+
+    def requant_one(self, acc: int, m0: int, shift: int, zy: int) -> int:
+        return int(self.lib.oracle_requant_one(int(acc), int(m0), int(shift), int(zy)))
+
+    def residual_add(self, a: np.ndarray, b: np.ndarray) -> np.ndarray:
+        a = np.ascontiguousarray(a, dtype=np.int8)
+        b = np.ascontiguousarray(b, dtype=np.int8)
+        assert a.shape == b.shape
+        out = np.zeros_like(a)
+        self.lib.oracle_residual_add(_ptr(a), _ptr(b), a.size, _ptr(out))
+        return out
+
+
+def _default() -> Oracle:
+    global _lib
+    with _lock:
+        if _lib is None:
+            build()
+            _lib = Oracle(_LIB)
+    return _lib
+
+
+def requant_params(sx, sw, sy):
+    return _default().requant_params(sx, sw, sy)
+
+
+def pack(w, bits):
+    return _default().pack(w, bits)
+
+
+def unpack(packed, n, k, bits):
+    return _default().unpack(packed, n, k, bits)
+
+
+def linear(x, zx, packed, bits, n, m0, shift, zy, want_acc=False):
+    return _default().linear(x, zx, packed, bits, n, m0, shift, zy, want_acc)
+
+
+def linear_points(x, zx, packed, bits, n, m0, shift, zy, pts):
+    return _default().linear_points(x, zx, packed, bits, n, m0, shift, zy, pts)
+
+
+def requant_one(acc, m0, shift, zy):
+    return _default().requant_one(acc, m0, shift, zy)
+
+
+def residual_add(a, b):
+    return _default().residual_add(a, b)
+
+
+def compile_variant(src_text: str, out_path: str) -> str:
+    """Compile a (test-modified) copy of the oracle source to out_path."""
+    d = os.path.dirname(out_path)
+    c_path = os.path.join(d, "mq_oracle_variant.c")
+    with open(c_path, "w") as f:
+        f.write(src_text)
+    import shutil
+    shutil.copy(_HDR, os.path.join(d, "mq_oracle.h"))
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-o", out_path,
+                           c_path, "-lm"])
+    return out_path
+
+
+def source() -> str:
+    with open(_SRC) as f:
+        return f.read()
+
+
+def raw():
+    """The ctypes handle (for tests that probe argument validation)."""
+    return _default().lib

@@ -1,0 +1,113 @@
+/*
+ * mq_oracle.h -- plain, slow, single-threaded CPU oracle for the integer-only
+ * quantized linear layer of MobileQuant (arXiv 2408.13933).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may include, link,
+ * load or call this code: only the test suite, the smoke check and the
+ * benchmark's CPU-baseline leg do.  It shares no header, helper, table or
+ * constant with the CUDA library; it is written from the paper's definitions:
+ *
+ *   - Sec. 3.1 (mobile-friendly design choices): integer (fixed-point) weights
+ *     and activations, per-tensor/per-channel static quantization, int8 x int8.
+ *   - Sec. 4.2, eqs. 2-4: the asymmetric uniform quantizer
+ *       q_max = 2^bw - 1, alpha = (f_max - f_min)/q_max, beta = f_min/alpha,
+ *       X_int = min(max(round(X/alpha) - beta, 0), q_max).
+ *     Applied to the layer output with a static (alpha, beta) it is the
+ *     requantization below; shifted by -128 to signed int8 its offset is the
+ *     output zero point zy (reading R1 of the design notes).
+ *   - Sec. 5.1 and Appendix A: symmetric per-output-channel weights (int8, or
+ *     int4 in [-8, 7]), so the weight zero point is 0.
+ *
+ * Conventions: M tokens, K input features, N output features.  x is int8
+ * [M][ldx], weights are int8 [N][K] (K contiguous) or int4 packed two per byte
+ * [N][K/2] with the low nibble holding the even k.  Output y is int8 [M][ldy].
+ *
+ * Every accumulation is done in int64 and every rounding is done on exact
+ * integers (__int128), so the oracle's result is the mathematical definition.
+ *
+ * Parity status of each function is stated beside it.
+ */
+#ifndef MQ_ORACLE_H
+#define MQ_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Return codes of the oracle (its own, not the library's). */
+#define ORACLE_OK 0
+#define ORACLE_EINVAL 1    /* bad argument */
+#define ORACLE_EOVERFLOW 2 /* an accumulator left the int32 range */
+
+/*
+ * Fixed-point multiplier for the per-channel real scale
+ *     M[n] = (sx * sw[n]) / sy          (double, in that order)
+ * written as M[n] ~= M0[n] * 2^-shift[n] with M0 in [2^30, 2^31) and
+ * shift in [1, 62].  Multipliers below 2^-32 (whose product with any int32
+ * accumulator is under 1/2 in magnitude) are returned as M0 = 0, shift = 1.
+ * Multipliers >= 2^30 are rejected (shift would be < 1).
+ * Follows the fixed-point statement of Sec. 3.1 / Sec. 1 (all operations in
+ * fixed point) with the rounding reading R4 of the design notes.
+ * Pinned by: power-of-two closed forms, relative-error bound 2^-31.
+ */
+int oracle_requant_params(float sx, const float *sw, int N, float sy,
+                          int32_t *M0, int32_t *shift);
+
+/*
+ * Pack int8 weight values w[N][K] for `bits` = 8 (copy) or 4 (two's-complement
+ * nibbles, low nibble = even k; values must lie in [-8, 7]) and compute
+ * colsum[n] = sum_k w[n][k] in int32.  Pinned by: round trip, golden bytes,
+ * brute-force sums.
+ */
+int oracle_pack(const int8_t *w, int N, int K, int bits, uint8_t *packed,
+                int32_t *colsum);
+
+/* Inverse of oracle_pack: packed -> int8 values [N][K]. */
+int oracle_unpack(const uint8_t *packed, int N, int K, int bits, int8_t *w);
+
+/*
+ * The integer-only linear layer, straight from its definition:
+ *   acc[m][n] = sum_k (x[m][k] - zx) * w[n][k]                (int64)
+ *   v         = acc * M0[n]                                    (exact)
+ *   q         = floor(v / 2^s + 1/2)     (round half up, s = shift[n])
+ *   y[m][n]   = clamp(zy + q, -128, 127)
+ * acc_out (may be NULL) receives acc as int32 [M][N] (row stride N).
+ * Returns ORACLE_EOVERFLOW if any |acc| >= 2^31.
+ * Pinned by: exhaustive K=1 brute force, zero-point identity, exact
+ * dequantization invariant, closed-form requant and exact-rational ties.
+ */
+int oracle_linear(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                  const uint8_t *packed, int bits, int N, const int32_t *M0,
+                  const int32_t *shift, int32_t zy, int8_t *y, int ldy,
+                  int32_t *acc_out);
+
+/*
+ * The same layer evaluated only at the listed output coordinates
+ * (m = pts[2i], n = pts[2i+1]); y_out[i] / acc_out[i] receive the results.
+ * Used to check full-size problems on a sample of outputs.
+ */
+int oracle_linear_points(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                         const uint8_t *packed, int bits, int N,
+                         const int32_t *M0, const int32_t *shift, int32_t zy,
+                         const int64_t *pts, int count, int8_t *y_out,
+                         int32_t *acc_out);
+
+/*
+ * Requantize one accumulator: clamp(zy + floor(acc*M0 / 2^s + 1/2), -128, 127).
+ * Exposed so that tests can sweep accumulators around rounding ties.
+ */
+int32_t oracle_requant_one(int64_t acc, int32_t M0, int32_t shift, int32_t zy);
+
+/*
+ * Saturating int8 residual add, out[i] = clamp(a[i] + b[i], -128, 127): the
+ * glue between chained layers of the 22-layer stack (reading R8).
+ */
+void oracle_residual_add(const int8_t *a, const int8_t *b, int64_t n,
+                         int8_t *out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,209 @@
+"""Seeded synthetic inputs shaped like the paper's workloads.
+
+This module is shared by the CUDA path's tests/benchmark and by the oracle's
+tests.  It holds none of the integer layer's arithmetic: it draws float data,
+quantizes it to int8/int4 codes (the data-synthesis step the workloads are
+defined by) and picks static output ranges from the *float* layer, the way a
+calibration set would (Sec. 3.1, "static quantization statistics ... computed
+on a holdout calibration set").  It never computes an integer accumulator,
+a zero-point correction or a fixed-point requantization.
+
+Value recipe (reading R5/R6/R9 of the design notes):
+  * activations: N(0, 1) floats, 4 seeded input channels scaled x20 (outliers),
+    quantized per tensor, asymmetric: sx = (max - min) / 255,
+    zx = clamp(rint(-128 - min / sx), -128, 127), x = clamp(rint(x / sx) + zx).
+  * weights: N(0, 0.02) (optionally 1% of output rows drawn as 0.02 * t(3)),
+    symmetric per output channel: int8 sw = max|w_n| / 127, w in [-127, 127];
+    int4 sw = max|w_n| / 7, w in [-8, 7].
+  * output range: min/max of the float layer (dequantized activations times
+    float weights) over calibration rows -> sy = (max - min) / 255 and
+    zy = clamp(rint(-128 - min / sy), -128, 127).
+Seeds: numpy PCG64 seeded with SeedSequence([1234, config, layer, linear, role]).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+BASE_SEED = 1234
+ROLE_X, ROLE_W, ROLE_OUTLIER, ROLE_TROWS, ROLE_RES = 0, 1, 2, 3, 4
+
+# Decoder-block linear shapes (name, K, N), TinyLlama-1.1B (hidden 2048,
+# 32 heads, 4 KV heads x 64, FFN 5632) and Gemma-2B (hidden 2048, 8 heads x 256,
+# 1 KV head, FFN 16384).
+TINYLLAMA_LINEARS = [
+    ("q", 2048, 2048), ("k", 2048, 256), ("v", 2048, 256), ("o", 2048, 2048),
+    ("gate", 2048, 5632), ("up", 2048, 5632), ("down", 5632, 2048),
+]
+TINYLLAMA_HEAD = ("head", 2048, 32000)
+GEMMA_LINEARS = [
+    ("q", 2048, 2048), ("k", 2048, 256), ("v", 2048, 256), ("o", 2048, 2048),
+    ("gate", 2048, 16384), ("up", 2048, 16384), ("down", 16384, 2048),
+]
+GEMMA_HEAD = ("head", 2048, 256000)
+
+
+def rng_for(config: int, layer: int, linear: int, role: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(
+        np.random.SeedSequence([BASE_SEED, config, layer, linear, role])))
+
+
+def rint_clip(v: np.ndarray, lo: int, hi: int) -> np.ndarray:
+    return np.clip(np.rint(v), lo, hi)
+
+
+def float_activations(rng: np.random.Generator, m: int, k: int, n_outliers: int = 4,
+                      outlier_scale: float = 20.0, orng: np.random.Generator | None = None):
+    xf = rng.standard_normal((m, k), dtype=np.float32)
+    orng = orng if orng is not None else rng
+    if n_outliers and k:
+        ch = orng.choice(k, size=min(n_outliers, k), replace=False)
+        xf[:, ch] *= outlier_scale
+    return xf
+
+
+def quantize_per_tensor(xf: np.ndarray):
+    """Asymmetric per-tensor int8 codes (eqs. 2-4, shifted to signed int8)."""
+    lo = float(min(xf.min(), 0.0)) if xf.size else -1.0
+    hi = float(max(xf.max(), 0.0)) if xf.size else 1.0
+    if hi - lo <= 0:
+        hi = lo + 1.0
+    s = np.float32((hi - lo) / 255.0)
+    z = int(rint_clip(np.array(-128.0 - lo / float(s)), -128, 127))
+    q = rint_clip(xf / s + z, -128, 127).astype(np.int8)
+    return q, float(s), z
+
+
+def float_weights(rng: np.random.Generator, n: int, k: int, std: float = 0.02,
+                  t_rows_frac: float = 0.0, trng: np.random.Generator | None = None):
+    wf = rng.standard_normal((n, k), dtype=np.float32) * np.float32(std)
+    if t_rows_frac > 0 and n:
+        trng = trng if trng is not None else rng
+        nrows = max(1, int(round(n * t_rows_frac)))
+        rows = trng.choice(n, size=nrows, replace=False)
+        wf[rows] = (trng.standard_t(3.0, size=(nrows, k)) * std).astype(np.float32)
+    return wf
+
+
+def quantize_per_channel_symmetric(wf: np.ndarray, bits: int):
+    qmax = 127 if bits == 8 else 7
+    qmin = -127 if bits == 8 else -8
+    amax = np.abs(wf).max(axis=1) if wf.size else np.zeros(wf.shape[0], np.float32)
+    amax = np.where(amax > 0, amax, np.float32(1e-8)).astype(np.float32)
+    sw = (amax / np.float32(qmax)).astype(np.float32)
+    q = rint_clip(wf / sw[:, None], qmin, qmax).astype(np.int8)
+    return q, sw
+
+
+def output_range(yf: np.ndarray):
+    """Static output (sy, zy) from the float layer's min/max (calibration)."""
+    return quantize_params_from_range(float(yf.min()) if yf.size else -1.0,
+                                      float(yf.max()) if yf.size else 1.0)
+
+
+def quantize_params_from_range(lo: float, hi: float):
+    lo, hi = min(lo, 0.0), max(hi, 0.0)
+    if hi - lo <= 0:
+        hi = lo + 1.0
+    s = np.float32((hi - lo) / 255.0)
+    z = int(rint_clip(np.array(-128.0 - lo / float(s)), -128, 127))
+    return float(s), z
+
+
+@dataclass
+class LinearCase:
+    """One quantized linear problem: int8 x [M,K], int weights [N,K], scales."""
+    name: str
+    x: np.ndarray          # int8 [M, K]
+    zx: int
+    sx: float
+    w: np.ndarray          # int8 values [N, K] (int4 range if bits == 4)
+    sw: np.ndarray         # float32 [N]
+    bits: int
+    sy: float
+    zy: int
+    residual: np.ndarray | None = None   # optional int8 [M, N]
+    meta: dict = field(default_factory=dict)
+
+    @property
+    def M(self): return self.x.shape[0]
+
+    @property
+    def K(self): return self.x.shape[1]
+
+    @property
+    def N(self): return self.w.shape[0]
+
+
+def make_linear(config: int, layer: int, linear: int, name: str, m: int, k: int, n: int,
+                bits: int, t_rows_frac: float = 0.0, calib_rows: int = 64,
+                x: tuple | None = None) -> LinearCase:
+    """A seeded linear problem.  `x` may pass (x_int8, sx, zx) to reuse inputs."""
+    if x is None:
+        xf = float_activations(rng_for(config, layer, linear, ROLE_X), m, k,
+                               orng=rng_for(config, layer, linear, ROLE_OUTLIER))
+        xq, sx, zx = quantize_per_tensor(xf)
+    else:
+        xq, sx, zx = x
+    wf = float_weights(rng_for(config, layer, linear, ROLE_W), n, k, t_rows_frac=t_rows_frac,
+                       trng=rng_for(config, layer, linear, ROLE_TROWS))
+    wq, sw = quantize_per_channel_symmetric(wf, bits)
+    rows = min(m, calib_rows)
+    # Float layer on the calibration rows: dequantized activations times the
+    # float weights (the unquantized model's output), for static output ranges.
+    xdq = (xq[:rows].astype(np.float32) - np.float32(zx)) * np.float32(sx)
+    yf = xdq @ wf.T if rows and n else np.zeros((0, n), np.float32)
+    sy, zy = output_range(yf)
+    return LinearCase(name, xq, zx, sx, wq, sw, bits, sy, zy)
+
+
+def block_linears(config: int, m: int, bits: int, shapes=TINYLLAMA_LINEARS, layer: int = 0,
+                  t_rows_frac: float = 0.0, shared_input: bool = False):
+    """All linears of one decoder block, each with its own seeded input
+    (or, with shared_input, q/k/v/gate/up reading one x of width 2048)."""
+    out = []
+    shared = None
+    for j, (name, k, n) in enumerate(shapes):
+        xin = None
+        if shared_input and name in ("q", "k", "v", "gate", "up"):
+            if shared is None:
+                xf = float_activations(rng_for(config, layer, 99, ROLE_X), m, k,
+                                       orng=rng_for(config, layer, 99, ROLE_OUTLIER))
+                shared = quantize_per_tensor(xf)
+            xin = shared
+        out.append(make_linear(config, layer, j, name, m, k, n, bits,
+                               t_rows_frac=t_rows_frac, x=xin))
+    return out
+
+
+def residual_codes(config: int, layer: int, m: int, n: int, scale: float = 8.0) -> np.ndarray:
+    """Seeded fixed int8 residual for the chained stack (reading R8)."""
+    r = rng_for(config, layer, 0, ROLE_RES).standard_normal((m, n), dtype=np.float32) * scale
+    return rint_clip(r, -128, 127).astype(np.int8)
+
+
+def random_case(seed: int, m: int, k: int, n: int, bits: int, extreme: str | None = None) -> LinearCase:
+    """Small seeded problem for parity tests, optionally with extreme values:
+    'min' (all codes at the most negative value), 'max', or 'mixed'."""
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([BASE_SEED, 7, seed])))
+    wlo, whi = (-128, 127) if bits == 8 else (-8, 7)
+    x = rng.integers(-128, 128, size=(m, k), dtype=np.int16).astype(np.int8)
+    w = rng.integers(wlo, whi + 1, size=(n, k), dtype=np.int16).astype(np.int8)
+    zx = int(rng.integers(-128, 128))
+    if extreme == "min":
+        x[:] = -128
+        w[:] = wlo
+        zx = 127
+    elif extreme == "max":
+        x[:] = 127
+        w[:] = whi
+        zx = -128
+    elif extreme == "mixed":
+        x[:] = np.where(rng.random((m, k)) < 0.5, -128, 127).astype(np.int8)
+        w[:] = np.where(rng.random((n, k)) < 0.5, wlo, whi).astype(np.int8)
+    sx = float(np.float32(rng.uniform(0.005, 0.05)))
+    sw = rng.uniform(1e-4, 3e-3, size=n).astype(np.float32)
+    sy = float(np.float32(rng.uniform(0.02, 0.2)))
+    zy = int(rng.integers(-128, 128))
+    return LinearCase(f"rand{seed}", x, zx, sx, w, sw, bits, sy, zy)

@@ -1,0 +1,366 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself.
+
+Each check ties the oracle to something independent of its code:
+  * hand-derived worked examples (tests/golden/tiny_linear.json);
+  * exhaustive brute force (K = 1 over every int8 x, w and zero point);
+  * the zero-point identity sum((x - zx) w) = sum(x w) - zx colsum(w), with the
+    right side from numpy's int64 matmul;
+  * the exact dequantization invariant: with power-of-two scales the float64
+    matmul of dequantized operands equals acc * sx * sw exactly;
+  * closed-form requantization (multiplier 2^-t is a rounding right shift) and
+    exact-rational rounding at ties (fractions.Fraction);
+  * eq. 4's quantizer with the real multiplier, to within one step at near-ties;
+  * the requant parameters' 2^-31 relative error bound.
+A mutation test plants typical mistakes in a copy of the oracle and checks
+that the battery above rejects every one of them.
+"""
+import json
+import os
+import random
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import Oracle
+from paper_2408_13933_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "tiny_linear.json")
+
+
+def load_golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+# ----------------------------------------------------------------------------
+# Pin battery: each returns None on success and raises AssertionError on a
+# mismatch.  They take an Oracle so that the mutation test can reuse them.
+# ----------------------------------------------------------------------------
+
+def pin_golden(orc: Oracle):
+    g = load_golden()
+    for c in g["cases"]:
+        w = np.array(c["w"], np.int8)
+        packed, colsum = orc.pack(w, c["bits"])
+        assert colsum.tolist() == c["colsum"], c["name"]
+        if "packed" in c:
+            assert packed.tolist() == c["packed"], c["name"]
+        y, acc = orc.linear(np.array(c["x"], np.int8), c["zx"], packed, c["bits"], w.shape[0],
+                            np.array(c["M0"], np.int32), np.array(c["shift"], np.int32),
+                            c["zy"], want_acc=True)
+        assert acc.tolist() == c["acc"], c["name"]
+        assert y.tolist() == c["y"], c["name"]
+    rq = g["requant_one"]
+    for r in rq["rows"]:
+        assert orc.requant_one(r["acc"], rq["M0"], rq["shift"], r["zy"]) == r["y"], r
+    rp = g["requant_params"]
+    m0, sh = orc.requant_params(rp["sx"], np.array(rp["sw"], np.float32), rp["sy"])
+    assert m0.tolist() == rp["M0"] and sh.tolist() == rp["shift"]
+
+
+def pin_k1_exhaustive(orc: Oracle, zxs=range(-128, 128)):
+    xs = np.arange(-128, 128, dtype=np.int16).astype(np.int8).reshape(256, 1)
+    ws = np.arange(-128, 128, dtype=np.int16).astype(np.int8).reshape(256, 1)
+    packed, _ = orc.pack(ws, 8)
+    m0 = np.full(256, 1 << 30, np.int32)
+    sh = np.full(256, 31, np.int32)
+    for zx in zxs:
+        _, acc = orc.linear(xs, zx, packed, 8, 256, m0, sh, 0, want_acc=True)
+        ref = np.outer(xs[:, 0].astype(np.int64) - zx, ws[:, 0].astype(np.int64))
+        assert np.array_equal(acc.astype(np.int64), ref), zx
+
+
+def pin_int4_exhaustive_pairs(orc: Oracle):
+    # every pair of int4 weights against a spread of activations (K = 2)
+    ws = np.array([[a, b] for a in range(-8, 8) for b in range(-8, 8)], np.int8)
+    xs = np.array([[a, b] for a in (-128, -77, -1, 0, 1, 64, 127) for b in (-128, -3, 0, 5, 127)],
+                  np.int8)
+    packed, colsum = orc.pack(ws, 4)
+    assert np.array_equal(colsum, ws.astype(np.int32).sum(1))
+    m0 = np.full(ws.shape[0], 1 << 30, np.int32)
+    sh = np.full(ws.shape[0], 31, np.int32)
+    for zx in (-128, -5, 0, 3, 127):
+        _, acc = orc.linear(xs, zx, packed, 4, ws.shape[0], m0, sh, 0, want_acc=True)
+        ref = (xs.astype(np.int64) - zx) @ ws.astype(np.int64).T
+        assert np.array_equal(acc.astype(np.int64), ref), zx
+
+
+def pin_zero_point_identity(orc: Oracle, seeds=(1, 2, 3)):
+    for seed in seeds:
+        for bits in (8, 4):
+            for extreme in (None, "min", "max", "mixed"):
+                c = synth.random_case(seed, 7, 96, 13, bits, extreme)
+                packed, colsum = orc.pack(c.w, bits)
+                m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+                _, acc = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True)
+                xw = c.x.astype(np.int64) @ c.w.astype(np.int64).T
+                ref = xw - c.zx * c.w.astype(np.int64).sum(1)[None, :]
+                assert np.array_equal(acc.astype(np.int64), ref), (seed, bits, extreme)
+                assert np.array_equal(colsum.astype(np.int64), c.w.astype(np.int64).sum(1))
+
+
+def pin_exact_dequant(orc: Oracle):
+    rng = np.random.default_rng(5)
+    for bits in (8, 4):
+        c = synth.random_case(11, 9, 160, 17, bits)
+        a = 7
+        b = rng.integers(3, 12, size=c.N)
+        sx = 2.0 ** -a
+        sw = (2.0 ** -b.astype(np.float64))
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(1.0, np.ones(c.N, np.float32), 1.0)
+        _, acc = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, 0, want_acc=True)
+        xd = (c.x.astype(np.float64) - c.zx) * sx
+        wd = c.w.astype(np.float64) * sw[:, None]
+        yf = xd @ wd.T            # float64 BLAS; every partial sum is exact
+        assert np.array_equal(yf, acc.astype(np.float64) * sx * sw[None, :])
+
+
+def _round_half_up_frac(fr: Fraction) -> int:
+    import math
+    return math.floor(fr + Fraction(1, 2))
+
+
+def pin_requant_closed_form(orc: Oracle):
+    rng = random.Random(3)
+    for t in (1, 2, 5, 8, 13, 20, 30):
+        for _ in range(300):
+            acc = rng.randint(-(1 << 31) + 1, (1 << 31) - 1) if rng.random() < 0.5 \
+                else rng.randint(-4 << t, 4 << t)
+            zy = rng.randint(-128, 127)
+            q = (acc + (1 << (t - 1))) >> t      # Python >> floors: round half up
+            want = max(-128, min(127, zy + q))
+            assert orc.requant_one(acc, 1 << 30, 30 + t, zy) == want, (t, acc, zy)
+
+
+def pin_requant_ties(orc: Oracle):
+    rng = random.Random(4)
+    for _ in range(400):
+        s = rng.randint(1, 62)
+        m0 = rng.randint(1 << 30, (1 << 31) - 1)
+        # accumulators just around the tie points j + 1/2 of acc*m0/2^s
+        j = rng.randint(-200, 200)
+        centre = int(Fraction(2 * j + 1, 2) * Fraction(1 << s, m0))
+        for acc in range(centre - 2, centre + 3):
+            if not -(1 << 31) < acc < (1 << 31):
+                continue
+            q = _round_half_up_frac(Fraction(acc * m0, 1 << s))
+            want = max(-128, min(127, q))
+            assert orc.requant_one(acc, m0, s, 0) == want, (acc, m0, s)
+    # exact ties for small shifts, both signs
+    for s in range(1, 9):
+        for acc in range(-300, 301):
+            q = _round_half_up_frac(Fraction(acc * (1 << 30), 1 << s))
+            assert orc.requant_one(acc, 1 << 30, s, 0) == max(-128, min(127, q)), (acc, s)
+
+
+def pin_requant_vs_eq4(orc: Oracle):
+    """Requantization with the fixed-point multiplier against eq. 4 applied to
+    the real-valued layer output (float64): equal except at near-ties."""
+    c = synth.make_linear(0, 0, 0, "q", 64, 256, 96, 8)
+    packed, _ = orc.pack(c.w, 8)
+    m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+    y, acc = orc.linear(c.x, c.zx, packed, 8, c.N, m0, sh, c.zy, want_acc=True)
+    yf = acc.astype(np.float64) * (c.sx * c.sw.astype(np.float64))[None, :]
+    # eq. 4 with alpha = sy and beta = -(zy + 128), shifted to signed int8
+    ref = np.clip(np.floor(yf / c.sy + 0.5) + c.zy, -128, 127)
+    diff = np.abs(y.astype(np.int64) - ref)
+    assert diff.max() <= 1
+    assert (diff != 0).mean() < 1e-3
+    # the calibration must leave most outputs unsaturated for the check to bite
+    assert np.mean(np.abs(y.astype(np.int64)) < 127) > 0.9
+
+
+def pin_requant_params_bound(orc: Oracle):
+    rng = np.random.default_rng(9)
+    for _ in range(20):
+        sx = np.float32(rng.uniform(1e-3, 1.0))
+        sy = np.float32(rng.uniform(1e-3, 1.0))
+        sw = rng.uniform(1e-5, 1e-1, size=64).astype(np.float32)
+        m0, sh = orc.requant_params(float(sx), sw, float(sy))
+        for n in range(64):
+            exact = Fraction(float(sx)) * Fraction(float(sw[n])) / Fraction(float(sy))
+            got = Fraction(int(m0[n]), 1 << int(sh[n]))
+            assert (1 << 30) <= int(m0[n]) < (1 << 31)
+            assert 1 <= int(sh[n]) <= 62
+            assert abs(got - exact) / exact <= Fraction(1, 1 << 31) + Fraction(1, 1 << 52)
+    # powers of two are exact
+    for t in range(0, 30):
+        m0, sh = orc.requant_params(1.0, np.array([2.0 ** -t], np.float32), 1.0)
+        # 2^-t = 0.5 * 2^(1-t): M0 = 0.5 * 2^31, shift = 31 - (1 - t)
+        assert (int(m0[0]), int(sh[0])) == (1 << 30, 30 + t)
+
+
+PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zero_point_identity,
+               pin_exact_dequant, pin_requant_closed_form, pin_requant_ties, pin_requant_vs_eq4,
+               pin_requant_params_bound]
+
+
+# ----------------------------------------------------------------------------
+# Tests
+# ----------------------------------------------------------------------------
+
+@pytest.fixture(scope="module")
+def O():
+    oracle.build()
+    return oracle._default()
+
+
+def test_golden_worked_examples(O):
+    pin_golden(O)
+
+
+def test_k1_exhaustive_all_zero_points(O):
+    pin_k1_exhaustive(O)
+
+
+def test_int4_pairs_exhaustive(O):
+    pin_int4_exhaustive_pairs(O)
+
+
+def test_zero_point_identity(O):
+    pin_zero_point_identity(O)
+
+
+def test_exact_dequantization_invariant(O):
+    pin_exact_dequant(O)
+
+
+def test_requant_closed_form_shift(O):
+    pin_requant_closed_form(O)
+
+
+def test_requant_exact_ties(O):
+    pin_requant_ties(O)
+
+
+def test_requant_matches_eq4_quantizer(O):
+    pin_requant_vs_eq4(O)
+
+
+def test_requant_params_error_bound(O):
+    pin_requant_params_bound(O)
+
+
+def test_bruteforce_small_k(O):
+    rng = np.random.default_rng(1)
+    for k in (1, 2, 3):
+        for bits in (8, 4):
+            lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+            if bits == 4 and k % 2:
+                continue
+            x = rng.integers(-128, 128, size=(5, k)).astype(np.int8)
+            w = rng.integers(lo, hi + 1, size=(6, k)).astype(np.int8)
+            zx = int(rng.integers(-128, 128))
+            packed, _ = O.pack(w, bits)
+            m0, sh = O.requant_params(0.02, np.full(6, 0.01, np.float32), 0.05)
+            y, acc = O.linear(x, zx, packed, bits, 6, m0, sh, 3, want_acc=True)
+            for m in range(5):
+                for n in range(6):
+                    a = sum((int(x[m, kk]) - zx) * int(w[n, kk]) for kk in range(k))
+                    assert acc[m, n] == a
+                    q = _round_half_up_frac(Fraction(a * int(m0[n]), 1 << int(sh[n])))
+                    assert y[m, n] == max(-128, min(127, 3 + q))
+
+
+def test_requant_params_special_cases(O):
+    m0, sh = O.requant_params(2.0 ** -20, np.array([2.0 ** -20], np.float32), 1.0)
+    assert (int(m0[0]), int(sh[0])) == (0, 1)          # below 2^-32: output is zy
+    m0, sh = O.requant_params(2.0 ** 15, np.array([2.0 ** 14], np.float32), 1.0)
+    assert (int(m0[0]), int(sh[0])) == (1 << 30, 1)    # 2^29: smallest legal shift
+    with pytest.raises(oracle.OracleError):
+        O.requant_params(2.0 ** 15, np.array([2.0 ** 15], np.float32), 1.0)  # 2^30
+    for bad in (0.0, -1.0, float("nan"), float("inf")):
+        with pytest.raises(oracle.OracleError):
+            O.requant_params(bad, np.array([0.1], np.float32), 1.0)
+        with pytest.raises(oracle.OracleError):
+            O.requant_params(0.1, np.array([bad], np.float32), 1.0)
+
+
+def test_pack_roundtrip_and_range(O):
+    rng = np.random.default_rng(2)
+    for bits, lo, hi in ((8, -128, 127), (4, -8, 7)):
+        w = rng.integers(lo, hi + 1, size=(33, 64)).astype(np.int8)
+        packed, colsum = O.pack(w, bits)
+        assert np.array_equal(O.unpack(packed, 33, 64, bits), w)
+        assert np.array_equal(colsum, w.astype(np.int64).sum(1))
+    with pytest.raises(oracle.OracleError):
+        O.pack(np.array([[8, 0]], np.int8), 4)
+    with pytest.raises(oracle.OracleError):
+        O.pack(np.array([[-9, 0]], np.int8), 4)
+
+
+def test_accumulator_overflow_detected(O):
+    k_ok, k_bad = 65536, 65794
+    for k, ok in ((k_ok, True), (k_bad, False)):
+        x = np.full((1, k), -128, np.int8)
+        w = np.full((1, k), -128, np.int8)
+        packed, _ = O.pack(w, 8)
+        m0 = np.array([1 << 30], np.int32)
+        sh = np.array([62], np.int32)
+        if ok:
+            _, acc = O.linear(x, 127, packed, 8, 1, m0, sh, 0, want_acc=True)
+            assert int(acc[0, 0]) == 255 * 128 * k
+        else:
+            with pytest.raises(oracle.OracleError):
+                O.linear(x, 127, packed, 8, 1, m0, sh, 0)
+
+
+def test_linear_points_agree_with_full(O):
+    c = synth.random_case(21, 11, 64, 19, 4)
+    packed, _ = O.pack(c.w, 4)
+    m0, sh = O.requant_params(c.sx, c.sw, c.sy)
+    y, acc = O.linear(c.x, c.zx, packed, 4, c.N, m0, sh, c.zy, want_acc=True)
+    pts = np.array([(m, n) for m in range(11) for n in range(19)], np.int64)
+    yp, ap = O.linear_points(c.x, c.zx, packed, 4, c.N, m0, sh, c.zy, pts)
+    assert np.array_equal(yp, y.reshape(-1)) and np.array_equal(ap, acc.reshape(-1))
+
+
+def test_residual_add_saturates(O):
+    a = np.array([-128, -100, 0, 100, 127, 127, -1], np.int8)
+    b = np.array([-1, -100, 5, 100, 1, -128, 1], np.int8)
+    assert O.residual_add(a, b).tolist() == [-128, -128, 5, 127, 127, -1, 0]
+
+
+MUTATIONS = [
+    ("zero point sign", "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - zx;",
+     "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] + zx;"),
+    ("nibble order", "int nibble = (k % 2 == 0) ? (byte & 0x0F) : (byte >> 4);",
+     "int nibble = (k % 2 == 0) ? (byte >> 4) : (byte & 0x0F);"),
+    ("int4 sign extension", "return nibble >= 8 ? nibble - 16 : nibble;", "return nibble;"),
+    ("round half down", "__int128 q = oracle_floor_div(2 * v + two_s, 2 * two_s);",
+     "__int128 q = oracle_floor_div(2 * v + two_s - 1, 2 * two_s);"),
+    ("truncating division", "if (r != 0 && a < 0) q -= 1;", "(void)r;"),
+    ("dropped rounding term", "__int128 q = oracle_floor_div(2 * v + two_s, 2 * two_s);",
+     "__int128 q = oracle_floor_div(2 * v, 2 * two_s);"),
+    ("multiplier exponent off by one", "int s = 31 - e;", "int s = 30 - e;"),
+    ("mantissa rounding", "long long m0 = llround(ldexp(f, 31));",
+     "long long m0 = (long long)(ldexp(f, 31));"),
+    ("missing zero point", "y[(size_t)m * (size_t)ldy + (size_t)n] =\n                    (int8_t)oracle_requant_one(acc, M0[n], shift[n], zy);",
+     "y[(size_t)m * (size_t)ldy + (size_t)n] =\n                    (int8_t)oracle_requant_one(acc, M0[n], shift[n], 0);"),
+    ("dropped last k", "for (int k = 0; k < K; ++k) {\n        int64_t xv",
+     "for (int k = 0; k < K - 1; ++k) {\n        int64_t xv"),
+    ("colsum of first row only", "if (colsum) colsum[n] = (int32_t)sum;",
+     "if (colsum) colsum[n] = (int32_t)(n == 0 ? sum : 0);"),
+    ("saturation bound", "if (out > 127) out = 127;", "if (out > 126) out = 126;"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_pins_reject_planted_mistake(tmp_path, name, old, new):
+    src = oracle.source()
+    assert old in src, f"mutation anchor for '{name}' not found"
+    lib = oracle.compile_variant(src.replace(old, new, 1), str(tmp_path / "libmut.so"))
+    mutant = Oracle(lib)
+    failures = 0
+    for pin in PIN_BATTERY:
+        try:
+            if pin is pin_k1_exhaustive:
+                pin(mutant, zxs=(-128, -1, 0, 1, 127))
+            else:
+                pin(mutant)
+        except (AssertionError, oracle.OracleError):
+            failures += 1
+    assert failures > 0, f"no pin caught the planted mistake '{name}'"
