@@ -1,0 +1,178 @@
+/*
+ * mq.h -- C ABI of libmq, the GB300 (sm_103a) integer-only quantized linear
+ * layer of MobileQuant (arXiv 2408.13933).
+ *
+ * The layer (Sec. 3.1; Sec. 4.2 eqs. 2-4; Sec. 5.1 and Appendix A):
+ *   x  : int8 activations [M][ldx], static per-tensor scale sx and zero point zx
+ *   w  : int8 or int4 weights [N][K], symmetric per output channel (scale sw[n],
+ *        zero point 0), the learned equivalent transform already folded in
+ *   acc[m][n] = sum_k (x[m][k] - zx) * w[n][k]
+ *             = sum_k x[m][k] w[n][k] - zx * colsum[n]            (int32)
+ *   y[m][n]   = clamp(zy + round_half_up(acc * M0[n] * 2^-shift[n]), -128, 127)
+ *   optionally y[m][n] = clamp(y[m][n] + residual[m][n], -128, 127)
+ * with M0[n] * 2^-shift[n] ~= sx * sw[n] / sy the fixed-point form of the
+ * output quantizer of eq. 4 (alpha = sy, offset zy).
+ *
+ * Conventions for every call:
+ *   - Every function returns an int status (mq_status); 0 is MQ_OK.  Nothing
+ *     throws or aborts across the ABI.
+ *   - All buffers belong to the caller.  The library allocates no memory.
+ *   - "device" pointers are CUDA device addresses on the current device; "host"
+ *     pointers are ordinary CPU memory.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Kernel launches are asynchronous on that stream; argument
+ *     errors are reported before anything is launched.
+ *   - Kernels never spin forever: every device-side wait has a time limit.  A
+ *     kernel that hits it records MQ_ERR_DEVICE_TIMEOUT in a device status
+ *     word, abandons its work and exits; mq_check_device_status() reports it.
+ *   - Indices: M tokens, K input features, N output features.  All int8
+ *     matrices are row-major with the feature index contiguous.
+ */
+#ifndef MQ_H
+#define MQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MQ_OK = 0,
+    MQ_ERR_INVALID_ARG = 1,       /* null pointer, bad range, bad bits, bad scale */
+    MQ_ERR_UNSUPPORTED_SHAPE = 2, /* a dimension outside the supported range */
+    MQ_ERR_K_OVERFLOW = 3,        /* K > MQ_MAX_K: int32 accumulator could overflow */
+    MQ_ERR_ALIGNMENT = 4,         /* K, ldx or a pointer violates the 16-byte rule */
+    MQ_ERR_CUDA = 5,              /* a CUDA runtime call failed */
+    MQ_ERR_DEVICE_TIMEOUT = 6,    /* a kernel gave up on a bounded wait */
+    MQ_ERR_WORKSPACE = 7          /* workspace missing or too small */
+} mq_status;
+
+/* |acc| <= 255 * 128 * K < 2^31 holds for every input when K <= 65536. */
+#define MQ_MAX_K 65536
+/* Largest number of linears in one mq_linear_batch call. */
+#define MQ_MAX_BATCH 256
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *mq_status_string(int status);
+
+/*
+ * Fixed-point requantization parameters (Sec. 3.1: fixed-point operators;
+ * eq. 4: output quantizer with static scale sy).  For each output channel n
+ * the real multiplier M = (sx * sw[n]) / sy (IEEE double, in that order) is
+ * written M = f * 2^e with f in [0.5, 1); then
+ *     M0[n] = round_half_away(f * 2^31)   (if that equals 2^31: 2^30 and e+1)
+ *     shift[n] = 31 - e                   (must lie in [1, 62])
+ * so M0[n] * 2^-shift[n] = M within a relative 2^-31.  M < 2^-32 gives
+ * M0 = 0, shift = 1 (output == zy).  M >= 2^30 is MQ_ERR_INVALID_ARG.
+ *   sw    : host float [N], each finite and > 0
+ *   sx, sy: finite and > 0
+ *   M0, shift: host int32 [N], written by the call
+ * Errors: MQ_ERR_INVALID_ARG (null pointer, N < 0, bad scale, M >= 2^30).
+ */
+int mq_requant_params(const float *sw, int N, float sx, float sy, int32_t *M0,
+                      int32_t *shift);
+
+/* Bytes of the packed weight buffer: N*K for bits 8, N*K/2 for bits 4.
+ * Errors: MQ_ERR_INVALID_ARG (negative size, bits not 4/8, odd K for 4). */
+int mq_packed_size(int N, int K, int bits, size_t *bytes);
+
+/*
+ * Pack weight values and compute colsum (the zero-point correction term of
+ * the identity sum((x-zx)w) = sum(xw) - zx*colsum(w); eq. 4's offset applied
+ * to the input).
+ *   w      : int8 [N][K] values; for bits 4 each must lie in [-8, 7]
+ *   bits   : 8 -> packed is an int8 copy [N][K];
+ *            4 -> packed is uint8 [N][K/2], byte j of row n holds k = 2j in
+ *                 bits 0-3 and k = 2j+1 in bits 4-7 (two's complement)
+ *   packed : mq_packed_size bytes, written
+ *   colsum : int32 [N], written: colsum[n] = sum_k w[n][k]
+ *   on_device = 0: w, packed, colsum are host pointers; the call is synchronous.
+ *   on_device = 1: they are device pointers; a kernel runs on `stream` and the
+ *                  call waits for it (to report out-of-range int4 values).
+ * Errors: MQ_ERR_INVALID_ARG (null, bad bits, odd K for int4, int4 value out
+ * of range -- packed/colsum contents are then unspecified), MQ_ERR_CUDA.
+ */
+int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed,
+                    int32_t *colsum, int on_device, void *stream);
+
+/* Device workspace bytes a mq_linear_* call of this shape needs (0 for every
+ * shape in this version; kept so that callers need not change when a kernel
+ * starts to use one).  Errors: MQ_ERR_INVALID_ARG. */
+int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes);
+
+/*
+ * One quantized linear layer, int8 activations x int8 weights (W8A8).
+ *   x        : device int8 [M][ldx], ldx >= K
+ *   zx       : input zero point in [-128, 127]
+ *   packed   : device, from mq_pack_weights(bits = 8)
+ *   colsum   : device int32 [N]
+ *   M0, shift: device int32 [N], from mq_requant_params
+ *   zy       : output zero point in [-128, 127]
+ *   y        : device int8 [M][ldy], ldy >= N, written
+ *   workspace: device, ws_bytes >= mq_workspace_size (may be NULL when 0)
+ * Requirements: 0 <= M, N; 0 <= K <= MQ_MAX_K; K % 16 == 0; ldx % 16 == 0;
+ * x and packed 16-byte aligned.  With K == 0 (every output is requant(0),
+ * i.e. zy) x and packed are not read and may be NULL.  M <= 16 runs the
+ * weight-streaming decode kernel, larger M the tcgen05 tensor-core kernel;
+ * both are bit-exact.
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_K_OVERFLOW, MQ_ERR_ALIGNMENT,
+ * MQ_ERR_WORKSPACE, MQ_ERR_CUDA (launch failure).
+ */
+int mq_linear_w8a8(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                   const void *packed, const int32_t *colsum, int N,
+                   const int32_t *M0, const int32_t *shift, int32_t zy,
+                   int8_t *y, int ldy, void *workspace, size_t ws_bytes,
+                   void *stream);
+
+/* The same layer with int4 weights (W4A8; Sec. 5.1 W4A8 setting and the
+ * symmetric per-channel scheme of Appendix A).  `packed` comes from
+ * mq_pack_weights(bits = 4).  Requires K % 32 == 0 (16-byte weight rows);
+ * other requirements and errors as mq_linear_w8a8. */
+int mq_linear_w4a8(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                   const void *packed, const int32_t *colsum, int N,
+                   const int32_t *M0, const int32_t *shift, int32_t zy,
+                   int8_t *y, int ldy, void *workspace, size_t ws_bytes,
+                   void *stream);
+
+/*
+ * Several independent linears in as few launches as possible (one per kernel
+ * family): a decoder block's projections that read the same activations, or
+ * a whole step's worth of small decode GEMVs.  Each descriptor has the
+ * meaning and requirements of one mq_linear_w8a8 / mq_linear_w4a8 call; in
+ * addition `residual` (device int8 [M][ldy], may be NULL) is added to the
+ * requantized output with int8 saturation, the int8 residual glue between
+ * chained layers.  Descriptors must not write overlapping outputs.
+ *   descs : host array of `count` descriptors (1 <= count <= MQ_MAX_BATCH)
+ * Errors: as the single calls; the index of the first bad descriptor is not
+ * reported, nothing is launched when any descriptor is invalid.
+ */
+typedef struct mq_linear_desc {
+    const int8_t *x;
+    const void *packed;
+    const int32_t *colsum;
+    const int32_t *M0;
+    const int32_t *shift;
+    const int8_t *residual; /* may be NULL */
+    int8_t *y;
+    int32_t M, N, K, ldx, ldy;
+    int32_t zx, zy;
+    int32_t bits; /* 8 or 4 */
+} mq_linear_desc;
+
+int mq_linear_batch(const mq_linear_desc *descs, int count, void *workspace,
+                    size_t ws_bytes, void *stream);
+
+/*
+ * Wait for `stream` and report device-side failures recorded by this
+ * library's kernels since the previous call: MQ_ERR_DEVICE_TIMEOUT if a
+ * bounded wait expired, MQ_ERR_CUDA if the stream reports a CUDA error,
+ * MQ_OK otherwise.  Clears the recorded status.
+ */
+int mq_check_device_status(void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MQ_H */

@@ -1,0 +1,50 @@
+// mq_internal.h -- definitions shared by libmq's host code and its kernels.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include "../../include/mq.h"
+
+// Bits of the device status word (a __device__ int owned by libmq).
+#define MQ_DEVICE_STATUS_TIMEOUT 1
+#define MQ_DEVICE_STATUS_PACK_RANGE 2
+
+namespace mq {
+
+// One linear problem as the kernels see it (validated by the host).
+struct Problem {
+    const int8_t *x;
+    const uint8_t *w;
+    const int32_t *colsum;
+    const int32_t *M0;
+    const int32_t *shift;
+    const int8_t *residual;
+    int8_t *y;
+    int32_t M, N, K, ldx, ldy;
+    int32_t zx, zy;
+    int32_t bits;
+    int32_t tile_begin;  // first global tile / block index of this problem
+    int32_t tiles_m;     // prefill: number of 128-row tiles
+};
+
+// Largest M served by the weight-streaming decode kernel.
+constexpr int DECODE_MAX_M = 16;
+
+// Problems per kernel launch (kernel parameter space).
+constexpr int PREFILL_MAX_PROBLEMS = 32;
+constexpr int DECODE_MAX_PROBLEMS = 128;
+
+// Device status words (__device__ ints owned by libmq, addresses cached per
+// device): kernels atomicOr MQ_DEVICE_STATUS_* bits into them.  The pack
+// kernel reports out-of-range int4 values in a word of its own.
+int *device_status_ptr();
+int *pack_status_ptr();
+
+// Launchers (asynchronous on `stream`); return MQ_OK or MQ_ERR_CUDA.
+int launch_prefill(const Problem *probs, int count, void *stream);
+int launch_decode(const Problem *probs, int count, void *stream);
+int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
+                int *status, void *stream);
+
+}  // namespace mq

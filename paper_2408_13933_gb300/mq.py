@@ -1,0 +1,179 @@
+"""Thin ctypes binding of libmq (include/mq.h): argument marshalling only.
+
+Every computation runs in libmq's CUDA kernels (or, for the host-side calls
+mq_requant_params / mq_pack_weights(on_device=0), in its C++ host code).
+Importing this module loads libmq.so and raises ImportError if it has not
+been built -- there is no fallback.
+
+Tensors are torch tensors (device memory and streams come from PyTorch);
+numpy arrays are accepted where the C call takes host memory.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+_LIB_PATH = _build.LIB
+if not os.path.exists(_LIB_PATH):
+    raise ImportError(
+        f"libmq.so not found at {_LIB_PATH}: build it first "
+        "(python -m paper_2408_13933_gb300.build, or __graft_entry__.build())")
+lib = ctypes.CDLL(_LIB_PATH)
+
+MQ_OK = 0
+MQ_ERR_INVALID_ARG = 1
+MQ_ERR_UNSUPPORTED_SHAPE = 2
+MQ_ERR_K_OVERFLOW = 3
+MQ_ERR_ALIGNMENT = 4
+MQ_ERR_CUDA = 5
+MQ_ERR_DEVICE_TIMEOUT = 6
+MQ_ERR_WORKSPACE = 7
+MQ_MAX_K = 65536
+MQ_MAX_BATCH = 256
+
+EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_weights",
+            "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
+            "mq_check_device_status"]
+
+_vp, _i32, _int, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int, ctypes.c_size_t
+
+
+class LinearDesc(ctypes.Structure):
+    """Mirror of mq_linear_desc."""
+    _fields_ = [("x", _vp), ("packed", _vp), ("colsum", _vp), ("M0", _vp), ("shift", _vp),
+                ("residual", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
+                ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32)]
+
+
+lib.mq_status_string.argtypes = [_int]
+lib.mq_status_string.restype = ctypes.c_char_p
+lib.mq_requant_params.argtypes = [_vp, _int, ctypes.c_float, ctypes.c_float, _vp, _vp]
+lib.mq_packed_size.argtypes = [_int, _int, _int, ctypes.POINTER(_sz)]
+lib.mq_pack_weights.argtypes = [_vp, _int, _int, _int, _vp, _vp, _int, _vp]
+lib.mq_workspace_size.argtypes = [_int, _int, _int, _int, ctypes.POINTER(_sz)]
+_linear_args = [_vp, _int, _int, _int, _i32, _vp, _vp, _int, _vp, _vp, _i32, _vp, _int, _vp,
+                _sz, _vp]
+lib.mq_linear_w8a8.argtypes = _linear_args
+lib.mq_linear_w4a8.argtypes = _linear_args
+lib.mq_linear_batch.argtypes = [ctypes.POINTER(LinearDesc), _int, _vp, _sz, _vp]
+lib.mq_check_device_status.argtypes = [_vp]
+for _f in EXPORTED:
+    if _f != "mq_status_string":
+        getattr(lib, _f).restype = _int
+
+
+class MQError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {status_string(code)} ({code})")
+
+
+def status_string(code: int) -> str:
+    return lib.mq_status_string(int(code)).decode()
+
+
+def _check(code: int, where: str):
+    if code != MQ_OK:
+        raise MQError(code, where)
+
+
+def _ptr(t) -> int | None:
+    """Address of a torch tensor's or numpy array's data (None for None)."""
+    if t is None:
+        return None
+    if isinstance(t, np.ndarray):
+        assert t.flags["C_CONTIGUOUS"]
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return stream if isinstance(stream, int) else stream.cuda_stream
+
+
+def requant_params(sw: np.ndarray, sx: float, sy: float):
+    """mq_requant_params on host arrays: returns (M0, shift) int32 [N]."""
+    sw = np.ascontiguousarray(sw, dtype=np.float32)
+    n = sw.shape[0]
+    m0 = np.zeros(n, np.int32)
+    sh = np.zeros(n, np.int32)
+    _check(lib.mq_requant_params(_ptr(sw), n, float(sx), float(sy), _ptr(m0), _ptr(sh)),
+           "mq_requant_params")
+    return m0, sh
+
+
+def packed_size(n: int, k: int, bits: int) -> int:
+    out = _sz(0)
+    _check(lib.mq_packed_size(n, k, bits, ctypes.byref(out)), "mq_packed_size")
+    return out.value
+
+
+def workspace_size(m: int, n: int, k: int, bits: int) -> int:
+    out = _sz(0)
+    _check(lib.mq_workspace_size(m, n, k, bits, ctypes.byref(out)), "mq_workspace_size")
+    return out.value
+
+
+def pack_weights(w, bits: int, stream=None):
+    """mq_pack_weights.  `w` int8 [N, K]: a numpy array (host path) or a CUDA
+    torch tensor (device path).  Returns (packed, colsum) on the same side."""
+    n, k = w.shape
+    size = packed_size(n, k, bits)
+    if isinstance(w, np.ndarray):
+        w = np.ascontiguousarray(w, dtype=np.int8)
+        packed = np.zeros(size, np.uint8)
+        colsum = np.zeros(n, np.int32)
+        _check(lib.mq_pack_weights(_ptr(w), n, k, bits, _ptr(packed), _ptr(colsum), 0, None),
+               "mq_pack_weights(host)")
+        return packed.reshape(n, -1) if n else packed, colsum
+    import torch
+    assert w.is_cuda and w.dtype == torch.int8 and w.is_contiguous()
+    packed = torch.empty(size, dtype=torch.uint8, device=w.device)
+    colsum = torch.empty(n, dtype=torch.int32, device=w.device)
+    _check(lib.mq_pack_weights(_ptr(w), n, k, bits, _ptr(packed), _ptr(colsum), 1,
+                               _stream(stream)), "mq_pack_weights(device)")
+    return packed.view(n, -1) if n else packed, colsum
+
+
+def linear(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y, bits: int,
+           ldx: int | None = None, ldy: int | None = None, m: int | None = None,
+           k: int | None = None, stream=None, workspace=None, ws_bytes: int = 0) -> int:
+    """mq_linear_w8a8 / mq_linear_w4a8 on CUDA tensors; returns the status code."""
+    m = x.shape[0] if m is None else m
+    k = x.shape[1] if k is None else k
+    ldx = x.stride(0) if ldx is None else ldx
+    ldy = y.stride(0) if ldy is None else ldy
+    fn = lib.mq_linear_w8a8 if bits == 8 else lib.mq_linear_w4a8
+    return fn(_ptr(x), m, k, ldx, int(zx), _ptr(packed), _ptr(colsum), n, _ptr(m0), _ptr(shift),
+              int(zy), _ptr(y), ldy, _ptr(workspace), ws_bytes, _stream(stream))
+
+
+def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
+              ldx=None, ldy=None, m=None, k=None) -> LinearDesc:
+    d = LinearDesc()
+    d.x, d.packed, d.colsum = _ptr(x), _ptr(packed), _ptr(colsum)
+    d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
+    d.M = x.shape[0] if m is None else m
+    d.K = x.shape[1] if k is None else k
+    d.N = n
+    d.ldx = x.stride(0) if ldx is None else ldx
+    d.ldy = y.stride(0) if ldy is None else ldy
+    d.zx, d.zy, d.bits = int(zx), int(zy), int(bits)
+    return d
+
+
+def linear_batch(descs, stream=None, workspace=None, ws_bytes: int = 0) -> int:
+    """mq_linear_batch over a list of LinearDesc; returns the status code."""
+    arr = (LinearDesc * len(descs))(*descs)
+    return lib.mq_linear_batch(arr, len(descs), _ptr(workspace), ws_bytes, _stream(stream))
+
+
+def check_device_status(stream=None) -> int:
+    return lib.mq_check_device_status(_stream(stream))

@@ -1,0 +1,143 @@
+"""Host-side checks of libmq that need no GPU.
+
+* the shared library loads and exports every function declared in include/mq.h;
+* mq_requant_params agrees with the oracle's independent implementation;
+* host-side mq_pack_weights agrees with the oracle's packing and colsum;
+* argument validation rejects bad calls before anything is launched.
+Every call made here either is host-only or fails validation, so nothing
+touches a GPU.
+"""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2408_13933_gb300 import build, synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def mq():
+    build.build()
+    from paper_2408_13933_gb300 import mq as _mq
+    return _mq
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "mq.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(mq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol(mq):
+    names = declared_functions()
+    assert len(names) >= 9
+    for name in names:
+        assert hasattr(mq.lib, name), name
+    assert set(names) == set(mq.EXPORTED)
+
+
+def test_status_strings(mq):
+    for code in range(8):
+        assert mq.status_string(code).startswith("MQ_")
+    assert mq.status_string(99) == "MQ_ERR_UNKNOWN"
+
+
+def test_requant_params_match_oracle(mq):
+    rng = np.random.default_rng(1)
+    for _ in range(50):
+        sx = float(np.float32(rng.uniform(1e-4, 2.0)))
+        sy = float(np.float32(rng.uniform(1e-4, 2.0)))
+        sw = np.exp(rng.uniform(-14, 2, size=257)).astype(np.float32)
+        try:
+            ref = oracle.requant_params(sx, sw, sy)
+        except oracle.OracleError:
+            with pytest.raises(mq.MQError):
+                mq.requant_params(sw, sx, sy)
+            continue
+        got = mq.requant_params(sw, sx, sy)
+        assert np.array_equal(got[0], ref[0]) and np.array_equal(got[1], ref[1])
+
+
+def test_requant_params_edge_cases(mq):
+    cases = [(0.5, [0.25, 0.75, 1.0], 2.0), (2.0 ** -20, [2.0 ** -20], 1.0),
+             (2.0 ** 15, [2.0 ** 14], 1.0), (1.0, [1.0 - 2.0 ** -24], 1.0),
+             (3.0, [1.0 / 3.0], 1.0), (1e-30, [1e-30], 1.0)]
+    for sx, sw, sy in cases:
+        sw = np.array(sw, np.float32)
+        ref = oracle.requant_params(sx, sw, sy)
+        got = mq.requant_params(sw, sx, sy)
+        assert got[0].tolist() == ref[0].tolist() and got[1].tolist() == ref[1].tolist()
+    for sx, sw, sy in [(2.0 ** 15, [2.0 ** 15], 1.0), (0.0, [1.0], 1.0), (1.0, [-1.0], 1.0),
+                       (1.0, [float("nan")], 1.0), (1.0, [1.0], float("inf"))]:
+        with pytest.raises(mq.MQError) as e:
+            mq.requant_params(np.array(sw, np.float32), sx, sy)
+        assert e.value.code == mq.MQ_ERR_INVALID_ARG
+
+
+def test_host_pack_matches_oracle(mq):
+    for bits in (8, 4):
+        for (n, k) in ((1, 2), (7, 64), (33, 130), (0, 16)):
+            c = synth.random_case(3, 1, k, max(n, 1), bits)
+            w = c.w[:n]
+            packed, colsum = mq.pack_weights(w, bits)
+            rp, rc = oracle.pack(w, bits)
+            assert np.array_equal(packed.reshape(-1), rp.reshape(-1))
+            assert np.array_equal(colsum, rc)
+
+
+def test_host_pack_rejects_int4_out_of_range(mq):
+    with pytest.raises(mq.MQError):
+        mq.pack_weights(np.array([[0, 8]], np.int8), 4)
+    with pytest.raises(mq.MQError):
+        mq.pack_weights(np.array([[0, 1, 2]], np.int8), 4)  # odd K
+
+
+def test_packed_and_workspace_sizes(mq):
+    assert mq.packed_size(3, 64, 8) == 192
+    assert mq.packed_size(3, 64, 4) == 96
+    assert mq.workspace_size(1024, 2048, 2048, 8) == 0
+    with pytest.raises(mq.MQError):
+        mq.packed_size(3, 63, 4)
+    with pytest.raises(mq.MQError):
+        mq.packed_size(-1, 64, 8)
+
+
+FAKE = 1 << 20  # a non-null, 16-byte aligned address; never dereferenced here
+
+
+def _call(mq, bits=8, x=FAKE, M=32, K=64, ldx=64, zx=0, packed=FAKE, colsum=FAKE, N=32,
+          m0=FAKE, shift=FAKE, zy=0, y=FAKE, ldy=32):
+    fn = mq.lib.mq_linear_w8a8 if bits == 8 else mq.lib.mq_linear_w4a8
+    return fn(x, M, K, ldx, zx, packed, colsum, N, m0, shift, zy, y, ldy, None, 0, None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(x=None), 1), (dict(packed=None), 1), (dict(colsum=None), 1), (dict(m0=None), 1),
+    (dict(shift=None), 1), (dict(y=None), 1), (dict(M=-1), 1), (dict(N=-1), 1),
+    (dict(K=-16), 1), (dict(zx=128), 1), (dict(zx=-129), 1), (dict(zy=200), 1),
+    (dict(ldx=32), 1), (dict(ldy=16), 1), (dict(K=65552, ldx=65552), 3),
+    (dict(K=24, ldx=32), 4), (dict(ldx=72), 4), (dict(x=FAKE + 8), 4),
+    (dict(packed=FAKE + 4), 4), (dict(bits=4, K=48, ldx=48), 4),
+])
+def test_linear_validation_rejects_before_launch(mq, kw, code):
+    assert _call(mq, **kw) == code
+
+
+def test_linear_bad_bits_and_batch_args(mq):
+    d = mq.LinearDesc()
+    d.bits = 3
+    assert mq.lib.mq_linear_batch((mq.LinearDesc * 1)(d), 1, None, 0, None) == 1
+    assert mq.lib.mq_linear_batch(None, 1, None, 0, None) == 1
+    assert mq.lib.mq_linear_batch((mq.LinearDesc * 1)(), 0, None, 0, None) == 1
+    assert mq.lib.mq_linear_batch((mq.LinearDesc * 1)(), mq.MQ_MAX_BATCH + 1, None, 0, None) == 1
+
+
+def test_empty_problems_launch_nothing(mq):
+    # M == 0 or N == 0 is valid and returns without touching the device
+    assert _call(mq, M=0) == 0
+    assert _call(mq, N=0) == 0
