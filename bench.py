@@ -1,0 +1,486 @@
+#!/usr/bin/env python
+"""Benchmark of the integer-only quantized linear layer (MobileQuant W8A8 / W4A8).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mq|reference]
+
+Headline workload: the seven W8A8 linears of one TinyLlama-1.1B-shaped decoder
+block at prefill M = 1024 tokens (q 2048->2048, k/v 2048->256, o 2048->2048,
+gate/up 2048->5632, down 5632->2048; q/k/v/gate/up share one input), with the
+seeded int8 residual added to down's output.  One step = one pass over the
+block = one batched libmq launch (mq_linear_batch) of the tcgen05 prefill
+kernel.  Steps rotate over three layers' weights and activations (216 MB,
+more than the 129 MB L2), so no step reads another's data from L2.
+
+Reported beside it, measured in the same run: W4A8 decode of the same block's
+linears at M = 1, 4, 16 (weight GB/s), rotating over 12 layers (264 MB).
+
+Multi-GPU (torchrun, one rank per GPU): replicas only -- every rank runs the
+same workload on its own GPU, no collective on the data path; value is the
+total over ranks divided by the slowest rank's time.
+
+--impl reference runs the CPU oracle (oracle/, plain C, one thread) on a
+bounded sample of the same workload: each step is one token row of the block.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2408_13933_gb300 import synth  # noqa: E402
+
+METRIC = "W8A8 prefill int8 TOPS (% of tensor peak); W4A8 decode weight GB/s (% HBM)"
+PREFILL_M = 1024
+PREFILL_LAYERS = 3
+DECODE_LAYERS = 12
+DECODE_MS = (1, 4, 16)
+CONFIG_ID_PREFILL = 1
+CONFIG_ID_DECODE = 2
+WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
+
+
+def block_ops(m: int) -> int:
+    return sum(2 * m * k * n for _, k, n in synth.TINYLLAMA_LINEARS)
+
+
+def block_weight_bytes(bits: int) -> int:
+    return sum(k * n * bits // 8 for _, k, n in synth.TINYLLAMA_LINEARS)
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+# --------------------------------------------------------------------------- dist
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+class Dist:
+    def __init__(self, world: int, rank: int, local: int):
+        self.world, self.rank, self.local = world, rank, local
+        self.pg = None
+        if world > 1:
+            import torch
+            import torch.distributed as dist
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg is not None:
+            self.pg.barrier()
+
+    def max(self, v: float) -> float:
+        if self.pg is None:
+            return v
+        import torch
+        t = torch.tensor([v], dtype=torch.float64, device="cuda")
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg is not None:
+            self.pg.destroy_process_group()
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling (every 100 ms) while the timed region runs."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.t0 = self.t1 = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu=timestamp,{self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def start(self):
+        self.t0 = time.time()
+
+    def stop(self):
+        self.t1 = time.time()
+
+    def result(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=5)
+        rows = []
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[3:]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if self.t0 - 1 <= r[0] <= self.t1 + 1]
+        use = inside if inside else rows
+        if not use:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in use for i, v in enumerate(r[3][2:6])
+                          if v.strip().lower() == "active"})
+        return {"sm_mhz": statistics.median(r[1] for r in use),
+                "sm_max_mhz": max(r[2] for r in use), "reasons": reasons,
+                "samples": len(use), "samples_in_region": len(inside)}
+
+
+# --------------------------------------------------------------------------- workload
+class PrefillBlock:
+    """Device-resident operands of one layer's seven W8A8 linears at M tokens."""
+
+    def __init__(self, mq, torch, layer: int, m: int):
+        self.cases = synth.block_linears(CONFIG_ID_PREFILL, m, 8, layer=layer, shared_input=True)
+        down = self.cases[-1]
+        down.residual = synth.residual_codes(CONFIG_ID_PREFILL, layer, m, down.N)
+        dev = "cuda"
+        # distinct inputs: the shared x (q/k/v/gate/up), o's input, down's input
+        self.x_host = {}
+        self.x_dev = {}
+        for c in self.cases:
+            key = id(c.x)
+            if key not in self.x_dev:
+                self.x_host[key] = torch.from_numpy(c.x).pin_memory()
+                self.x_dev[key] = torch.empty(c.x.shape, dtype=torch.int8, device=dev)
+                self.x_dev[key].copy_(self.x_host[key])
+        self.descs, self.y, self.keep = [], [], []
+        for c in self.cases:
+            packed, colsum = mq.pack_weights(c.w, 8)
+            m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
+            t = [torch.from_numpy(a).to(dev) for a in (packed, colsum, m0, sh)]
+            y = torch.empty((m, c.N), dtype=torch.int8, device=dev)
+            res = torch.from_numpy(c.residual).to(dev) if c.residual is not None else None
+            self.keep += t + ([res] if res is not None else [])
+            self.y.append(y)
+            self.descs.append(mq.make_desc(self.x_dev[id(c.x)], c.zx, t[0], t[1], c.N, t[2], t[3],
+                                           c.zy, y, 8, residual=res))
+        self.arr = (mq.LinearDesc * len(self.descs))(*self.descs)
+        self.y_host = [torch.empty(y.shape, dtype=torch.int8).pin_memory() for y in self.y]
+        self.h2d_bytes = sum(v.numel() for v in self.x_host.values())
+        self.d2h_bytes = sum(y.numel() for y in self.y)
+
+
+class DecodeLayer:
+    """One layer's seven W4A8 linears, uploaded once; descriptors for each
+    decode width M use the first M rows of a 16-row seeded input."""
+
+    def __init__(self, mq, torch, layer: int):
+        cases = synth.block_linears(CONFIG_ID_DECODE, max(DECODE_MS), 4, layer=layer)
+        self.arr, self.keep = {}, []
+        dev = []
+        for c in cases:
+            packed, colsum = mq.pack_weights(c.w, 4)
+            m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
+            t = [torch.from_numpy(a).cuda() for a in (c.x, packed, colsum, m0, sh)]
+            self.keep += t
+            dev.append((c, t))
+        for m in DECODE_MS:
+            descs = []
+            for c, t in dev:
+                y = torch.empty((m, c.N), dtype=torch.int8, device="cuda")
+                self.keep.append(y)
+                descs.append(mq.make_desc(t[0], c.zx, t[1], t[2], c.N, t[3], t[4], c.zy, y, 4,
+                                          m=m))
+            self.arr[m] = (mq.LinearDesc * len(descs))(*descs)
+        self.count = len(cases)
+
+
+def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
+    blocks = [PrefillBlock(mq, torch, layer, PREFILL_M) for layer in range(PREFILL_LAYERS)]
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    call = mq.lib.mq_linear_batch
+
+    def step(i):
+        b = blocks[i % len(blocks)]
+        rc = call(b.arr, len(b.descs), None, 0, sp)
+        if rc:
+            raise RuntimeError(f"mq_linear_batch failed: {mq.status_string(rc)}")
+
+    for i in range(warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error after warm-up")
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    clocks = ClockSampler(dist.local)
+    time.sleep(0.3)
+    dist.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    clocks.start()
+    t_start.record(stream)
+    for i in range(steps):
+        ev[i][0].record(stream)
+        step(i)
+        ev[i][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clocks.stop()
+    dist.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    kernel_ms = [a.elapsed_time(b) for a, b in ev]
+    status = mq.check_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {mq.status_string(status)} after timed region")
+    max_total_ms = dist.max(total_ms)
+
+    # end to end through the public API: pinned host inputs in, outputs back out
+    e2e_steps = min(steps, 50)
+    torch.cuda.synchronize()
+    dist.barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_steps):
+        b = blocks[i % len(blocks)]
+        for key, xh in b.x_host.items():
+            b.x_dev[key].copy_(xh, non_blocking=True)
+        step(i)
+        for y, yh in zip(b.y, b.y_host):
+            yh.copy_(y, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = dist.max(e0.elapsed_time(e1))
+    return {
+        "blocks": blocks, "total_ms": max_total_ms, "kernel_ms_mean": statistics.mean(kernel_ms),
+        "kernel_ms_median": statistics.median(kernel_ms), "clocks": clocks.result(),
+        "e2e_ms": e2e_ms, "e2e_steps": e2e_steps,
+        "h2d": blocks[0].h2d_bytes, "d2h": blocks[0].d2h_bytes,
+    }
+
+
+def run_decode(mq, torch, steps_per_m: int = 240):
+    """Weight GB/s of the W4A8 block linears at M = 1, 4, 16 (one batched
+    launch per layer, 12 layers in rotation), timed with CUDA events per launch
+    (kernel) and over a captured CUDA graph of back-to-back launches (stream)."""
+    out = {}
+    wbytes = block_weight_bytes(4)
+    stream = torch.cuda.current_stream()
+    layers = [DecodeLayer(mq, torch, layer) for layer in range(DECODE_LAYERS)]
+    call = mq.lib.mq_linear_batch
+    sp = stream.cuda_stream
+    for m in DECODE_MS:
+        for L in layers * 2:
+            assert call(L.arr[m], L.count, None, 0, sp) == 0
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps_per_m)]
+        for i in range(steps_per_m):
+            L = layers[i % len(layers)]
+            ev[i][0].record(stream)
+            call(L.arr[m], L.count, None, 0, sp)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        kms = statistics.median(a.elapsed_time(b) for a, b in ev)
+        # back-to-back launches from a CUDA graph (no host launch gaps)
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(g, stream=side):
+                for L in layers:
+                    call(L.arr[m], L.count, None, 0, side.cuda_stream)
+        stream.wait_stream(side)
+        g.replay()
+        torch.cuda.synchronize()
+        reps = max(1, steps_per_m // len(layers))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        gms = e0.elapsed_time(e1) / (reps * len(layers))
+        assert mq.check_device_status() == 0
+        out[f"m{m}"] = {"kernel_us": round(kms * 1e3, 2), "kernel_gbs": round(wbytes / kms / 1e6, 1),
+                        "stream_us": round(gms * 1e3, 2), "stream_gbs": round(wbytes / gms / 1e6, 1)}
+        del g
+    return out
+
+
+# --------------------------------------------------------------------------- CPU oracle
+def oracle_sample(blocks_cases, rows: range, col_frac: float = 1.0):
+    """Run the oracle on `rows` of every linear of one block; returns
+    (int8 ops done, seconds, {linear index: y})."""
+    import oracle
+    ops = 0
+    outs = {}
+    t0 = time.perf_counter()
+    for j, c in enumerate(blocks_cases):
+        n = max(1, int(round(c.N * col_frac)))
+        packed, _ = oracle.pack(c.w[:n], c.bits)
+        m0, sh = oracle.requant_params(c.sx, c.sw[:n], c.sy)
+        x = np.ascontiguousarray(c.x[rows.start:rows.stop])
+        y = oracle.linear(x, c.zx, packed, c.bits, n, m0, sh, c.zy)
+        if c.residual is not None:
+            y = oracle.residual_add(y, np.ascontiguousarray(c.residual[rows.start:rows.stop, :n]))
+        outs[j] = y
+        ops += 2 * x.shape[0] * c.K * n
+    return ops, time.perf_counter() - t0, outs
+
+
+def cpu_baseline(blocks, torch, rows: int = 192):
+    cases = blocks[0].cases
+    import oracle
+    oracle.build()
+    t_pack = time.perf_counter()
+    ops, secs, outs = oracle_sample(cases, range(0, rows))
+    # the GPU's outputs for the same rows of layer 0 (last written by the
+    # e2e loop, which ran layer 0's block at least once)
+    torch.cuda.synchronize()
+    checked = mism = 0
+    for j, y in outs.items():
+        got = blocks[0].y[j][:rows].cpu().numpy()
+        checked += y.size
+        mism += int(np.count_nonzero(got != y))
+    _ = t_pack
+    return {"value": round(ops / secs / 1e12, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
+            "sample": f"rows 0..{rows - 1} of all 7 linears of layer 0 (+ residual): "
+                      f"{ops / 1e9:.1f} GOP of the {block_ops(PREFILL_M) / 1e9:.1f} GOP block",
+            "seconds": round(secs, 2),
+            "parity_sample": {"outputs": checked, "mismatches": mism}}
+
+
+def run_reference(args, dist: Dist):
+    """Reference arm: the CPU oracle timed on this host, one token row of the
+    block per step (a bounded sample of the same workload)."""
+    if dist.rank != 0:
+        return
+    import oracle
+    oracle.build()
+    cases = synth.block_linears(CONFIG_ID_PREFILL, PREFILL_M, 8, layer=0, shared_input=True)
+    cases[-1].residual = synth.residual_codes(CONFIG_ID_PREFILL, 0, PREFILL_M, cases[-1].N)
+    # size the per-step sample so that warm-up + steps take about 90 s at most
+    _, t_row, _ = oracle_sample(cases, range(0, 1))
+    budget = 90.0
+    frac = min(1.0, budget / max(1e-9, (args.steps + args.warmup) * t_row))
+    for i in range(args.warmup):
+        oracle_sample(cases, range(i % PREFILL_M, i % PREFILL_M + 1), frac)
+    ops = 0
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        r = (args.warmup + i) % PREFILL_M
+        o, _, _ = oracle_sample(cases, range(r, r + 1), frac)
+        ops += o
+    secs = time.perf_counter() - t0
+    value = ops / secs / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": dist.world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs * 1e3 / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "tokens": PREFILL_M, "layers_rotated": 1,
+                   "sample_per_step": f"1 token row x {frac:.3f} of the output columns of "
+                                      "all 7 linears"},
+        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1, "kind": "oracle",
+                         "sample": "one token row of the block per step"},
+        "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawTextHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["mq", "reference"], default="mq")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    world, rank, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, Dist(1, rank, local))
+        return
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = Dist(world, rank, local)
+    from paper_2408_13933_gb300 import build
+    build.build()
+    from paper_2408_13933_gb300 import mq
+
+    pre = run_prefill(mq, torch, dist, args.steps, args.warmup)
+    decode = run_decode(mq, torch)
+    peaks = measured_peaks()
+
+    ops = block_ops(PREFILL_M)
+    ms_per_step = pre["total_ms"] / args.steps
+    value = ops * args.steps * world / (pre["total_ms"] * 1e-3) / 1e12
+    kern_tflops = ops / (pre["kernel_ms_mean"] * 1e-3) / 1e12
+    e2e_value = ops * pre["e2e_steps"] * world / (pre["e2e_ms"] * 1e-3) / 1e12
+    hbm = peaks["hbm_gbs"]
+    for v in decode.values():
+        v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
+
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int8",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "tokens": PREFILL_M,
+                   "linears": [f"{n} {k}->{nn}" for n, k, nn in synth.TINYLLAMA_LINEARS],
+                   "int8_ops_per_step": ops, "launches_per_step": 1,
+                   "l2": f"{PREFILL_LAYERS} layers rotated per step "
+                         f"({PREFILL_LAYERS * 72} MB > 129 MB L2)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "tensor", "achieved": round(kern_tflops, 1),
+                     "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                     "frac": round(kern_tflops / peaks["bf16_tflops"], 3), "traffic": None,
+                     "kernel": "mq::prefill::prefill_kernel",
+                     "peak_note": f"dense f16 tensor peak = bf16 burst ({peaks['source']}), "
+                                  "int8 ops run as exact f16 MMAs"},
+        "clocks": pre["clocks"],
+        "e2e": {"value": round(e2e_value, 2), "unit": "TOPS", "h2d_bytes_per_step": pre["h2d"],
+                "d2h_bytes_per_step": pre["d2h"]},
+        "gpu_launches": args.steps,
+        "decode_w4a8": {"unit": "GB/s of int4 weights", "weight_bytes_per_block":
+                        block_weight_bytes(4), "layers_rotated": DECODE_LAYERS,
+                        "hbm_peak_gbs": hbm, **decode},
+    }
+    if rank == 0 and world == 1:
+        line["cpu_baseline"] = cpu_baseline(pre["blocks"], torch)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -71,8 +71,11 @@ def quantize_per_tensor(xf: np.ndarray):
         hi = lo + 1.0
     s = np.float32((hi - lo) / 255.0)
     z = int(rint_clip(np.array(-128.0 - lo / float(s)), -128, 127))
-    q = rint_clip(xf / s + z, -128, 127).astype(np.int8)
-    return q, float(s), z
+    t = xf / s
+    t += np.float32(z)
+    np.rint(t, out=t)
+    np.clip(t, -128, 127, out=t)
+    return t.astype(np.int8), float(s), z
 
 
 def float_weights(rng: np.random.Generator, n: int, k: int, std: float = 0.02,
@@ -86,14 +89,21 @@ def float_weights(rng: np.random.Generator, n: int, k: int, std: float = 0.02,
     return wf
 
 
-def quantize_per_channel_symmetric(wf: np.ndarray, bits: int):
+def quantize_per_channel_symmetric(wf: np.ndarray, bits: int, inplace: bool = False):
+    """Symmetric per-output-channel codes; with inplace=True wf is overwritten."""
     qmax = 127 if bits == 8 else 7
     qmin = -127 if bits == 8 else -8
-    amax = np.abs(wf).max(axis=1) if wf.size else np.zeros(wf.shape[0], np.float32)
+    if wf.size:
+        amax = np.maximum(wf.max(axis=1), -wf.min(axis=1))
+    else:
+        amax = np.zeros(wf.shape[0], np.float32)
     amax = np.where(amax > 0, amax, np.float32(1e-8)).astype(np.float32)
     sw = (amax / np.float32(qmax)).astype(np.float32)
-    q = rint_clip(wf / sw[:, None], qmin, qmax).astype(np.int8)
-    return q, sw
+    t = wf if inplace else wf.copy()
+    np.divide(t, sw[:, None], out=t)
+    np.rint(t, out=t)
+    np.clip(t, qmin, qmax, out=t)
+    return t.astype(np.int8), sw
 
 
 def output_range(yf: np.ndarray):
@@ -148,13 +158,13 @@ def make_linear(config: int, layer: int, linear: int, name: str, m: int, k: int,
         xq, sx, zx = x
     wf = float_weights(rng_for(config, layer, linear, ROLE_W), n, k, t_rows_frac=t_rows_frac,
                        trng=rng_for(config, layer, linear, ROLE_TROWS))
-    wq, sw = quantize_per_channel_symmetric(wf, bits)
     rows = min(m, calib_rows)
     # Float layer on the calibration rows: dequantized activations times the
     # float weights (the unquantized model's output), for static output ranges.
     xdq = (xq[:rows].astype(np.float32) - np.float32(zx)) * np.float32(sx)
     yf = xdq @ wf.T if rows and n else np.zeros((0, n), np.float32)
     sy, zy = output_range(yf)
+    wq, sw = quantize_per_channel_symmetric(wf, bits, inplace=True)
     return LinearCase(name, xq, zx, sx, wq, sw, bits, sy, zy)
 
 
