@@ -22,6 +22,7 @@ Seeds: numpy PCG64 seeded with SeedSequence([1234, config, layer, linear, role])
 """
 from __future__ import annotations
 
+import os
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -78,9 +79,32 @@ def quantize_per_tensor(xf: np.ndarray):
     return t.astype(np.int8), float(s), z
 
 
+_POOL = None
+ROW_BLOCK = 256
+
+
+def _pool():
+    global _POOL
+    if _POOL is None:
+        from concurrent.futures import ThreadPoolExecutor
+        _POOL = ThreadPoolExecutor(max_workers=max(1, min(16, os.cpu_count() or 1)))
+    return _POOL
+
+
 def float_weights(rng: np.random.Generator, n: int, k: int, std: float = 0.02,
                   t_rows_frac: float = 0.0, trng: np.random.Generator | None = None):
-    wf = rng.standard_normal((n, k), dtype=np.float32) * np.float32(std)
+    """N(0, std) weights; rows are drawn in blocks of ROW_BLOCK, block b from a
+    generator seeded by (rng's first draw, b), in parallel threads."""
+    wf = np.empty((n, k), np.float32)
+    base = int(rng.integers(0, 2**63 - 1))
+
+    def fill(b):
+        r = np.random.Generator(np.random.PCG64(np.random.SeedSequence([base, b])))
+        lo, hi = b * ROW_BLOCK, min(n, (b + 1) * ROW_BLOCK)
+        r.standard_normal((hi - lo, k), dtype=np.float32, out=wf[lo:hi])
+        wf[lo:hi] *= np.float32(std)
+
+    list(_pool().map(fill, range((n + ROW_BLOCK - 1) // ROW_BLOCK)))
     if t_rows_frac > 0 and n:
         trng = trng if trng is not None else rng
         nrows = max(1, int(round(n * t_rows_frac)))
@@ -217,3 +241,68 @@ def random_case(seed: int, m: int, k: int, n: int, bits: int, extreme: str | Non
     sy = float(np.float32(rng.uniform(0.02, 0.2)))
     zy = int(rng.integers(-128, 128))
     return LinearCase(f"rand{seed}", x, zx, sx, w, sw, bits, sy, zy)
+
+
+def _quantize_with(yf: np.ndarray, s: float, z: int) -> np.ndarray:
+    t = yf / np.float32(s)
+    t += np.float32(z)
+    np.rint(t, out=t)
+    np.clip(t, -128, 127, out=t)
+    return t.astype(np.int8)
+
+
+@dataclass
+class ChainLayer:
+    """One layer of the chained stack: seven linears (q, k, v, o, gate, up,
+    down), the seeded residual r and the input/output scales of each linear."""
+    cases: list          # LinearCase per linear, x left empty (filled by the chain)
+    residual: np.ndarray  # int8 [M, hidden]
+
+
+def chain_stack(config: int, m: int, layers: int, shapes=TINYLLAMA_LINEARS, head=TINYLLAMA_HEAD,
+                calib_rows: int = 32, t_rows_frac: float = 0.0):
+    """Seeded 22-layer-style W8A8 stack (reading R8 of the design notes).
+
+    Layer l: q/k/v/gate/up read x_l; o reads q's int8 output (stand-in for the
+    attention output); down reads up's int8 output (stand-in for SiLU(gate) *
+    up); x_{l+1} = sat8(y_down + r_l).  Static output ranges come from a float
+    shadow of the chain on the first `calib_rows` rows (dequantized codes times
+    float weights, quantized with the chosen ranges -- the calibration pass).
+    Returns (x0, sx0, zx0, [ChainLayer], head LinearCase with empty x)."""
+    hidden = shapes[0][1]
+    xf = float_activations(rng_for(config, 0, 99, ROLE_X), m, hidden,
+                           orng=rng_for(config, 0, 99, ROLE_OUTLIER))
+    x0, sx0, zx0 = quantize_per_tensor(xf)
+    c = min(m, calib_rows)
+    cur_codes, cur_s, cur_z = x0[:c], sx0, zx0
+    out_layers = []
+    for layer in range(layers):
+        cases = []
+        produced = {}
+        for j, (name, k, n) in enumerate(shapes):
+            if name == "o":
+                in_codes, in_s, in_z = produced["q"]
+            elif name == "down":
+                in_codes, in_s, in_z = produced["up"]
+            else:
+                in_codes, in_s, in_z = cur_codes, cur_s, cur_z
+            wf = float_weights(rng_for(config, layer, j, ROLE_W), n, k, t_rows_frac=t_rows_frac,
+                               trng=rng_for(config, layer, j, ROLE_TROWS))
+            xin = (in_codes.astype(np.float32) - np.float32(in_z)) * np.float32(in_s)
+            yf = xin @ wf.T
+            sy, zy = output_range(yf)
+            produced[name] = (_quantize_with(yf, sy, zy), sy, zy)
+            wq, sw = quantize_per_channel_symmetric(wf, 8, inplace=True)
+            cases.append(LinearCase(name, np.zeros((0, k), np.int8), in_z, in_s, wq, sw, 8, sy, zy))
+        r = residual_codes(config, layer, m, hidden)
+        dcodes, ds, dz = produced["down"]
+        nxt = np.clip(dcodes.astype(np.int16) + r[:c], -128, 127).astype(np.int8)
+        out_layers.append(ChainLayer(cases, r))
+        cur_codes, cur_s, cur_z = nxt, ds, dz
+    name, k, n = head
+    wf = float_weights(rng_for(config, layers, 0, ROLE_W), n, k)
+    xin = (cur_codes.astype(np.float32) - np.float32(cur_z)) * np.float32(cur_s)
+    sy, zy = output_range(xin @ wf.T)
+    wq, sw = quantize_per_channel_symmetric(wf, 8, inplace=True)
+    head_case = LinearCase(name, np.zeros((0, k), np.int8), cur_z, cur_s, wq, sw, 8, sy, zy)
+    return x0, sx0, zx0, out_layers, head_case
