@@ -3,7 +3,7 @@
 //
 // At M <= 16 the layer reads each weight once and does at most 16 MACs with
 // it, so its speed is the weight stream (the paper notes that autoregressive
-// generation is memory-bound, Sec. 5.4 and Appendix A.2).  Each warp streams
+// generation is memory-bound, Sec. 5.6 and Appendix A.2).  Each warp streams
 // 16-row weight tiles straight from HBM into registers with 128-bit loads,
 // widens them in registers to f16 (exact for int8 and int4), and multiplies
 // with legacy warp-level mma.sync m16n8k16 (f16 x f16 -> f32): the weights
