@@ -3,28 +3,46 @@
 //
 // At M <= 16 the layer reads each weight once and does at most 16 MACs with
 // it, so its speed is the weight stream (the paper notes that autoregressive
-// generation is memory-bound, Sec. 5.6 and Appendix A.2).  Each warp streams
-// 16-row weight tiles straight from HBM into registers with 128-bit loads,
-// widens them in registers to f16 (exact for int8 and int4), and multiplies
-// with legacy warp-level mma.sync m16n8k16 (f16 x f16 -> f32): the weights
-// are the 16-row A operand, the (zero-padded) tokens the 8-column B operand.
-// Register-resident operands keep the weight stream out of shared memory;
-// on sm_103a the f16 mma.sync rate is 4x its int8 rate.
+// generation is memory-bound, Sec. 5.6 and Appendix A.2).
 //
-// Exactness: every product is an integer of magnitude <= 2^14 (int8) or
-// 2^10 (int4); a warp converts its f32 accumulators to int32 every 1024
-// (int8) or 16384 (int4) values of k, so no f32 partial sum exceeds 2^24.
+// Data path.  A persistent grid of CTAs (two per SM) walks 64-row units of
+// up to DECODE_MAX_PROBLEMS linears.  In each CTA one producer thread streams
+// the weight rows of its units with TMA into an 8-stage shared-memory ring,
+// continuing across unit boundaries.  A stage holds 64 weight rows x 128
+// bytes and the matching k slice of the 16 (zero-padded) token rows of x,
+// both 128-byte swizzled, so up to 64 KB of weights per CTA are in flight and
+// the activation fragments come from shared memory without bank conflicts.
+// Eight consumer warps read the ring, widen weights in registers to f16 and multiply with warp-level
+// mma.sync m16n8k16 (f16 x f16 -> f32): weights are the 16-row A operand, the
+// (zero-padded) tokens the 8-column B operand.  Warp w of the consumers owns
+// the 16-byte chunk w of every row of a stage (conflict-free under the
+// swizzle) for all four 16-row tiles of the unit, so one activation fragment
+// serves four weight tiles.
 //
-// The reduction order over k inside one mma is free, so the k index of each
-// fragment slot is permuted to whatever the cheapest in-register unpacking
-// yields (int4: nibble pairs (p, p+4) of a 32-bit word), and the activation
-// fragments use the same permutation.
+// Widening.  A weight code is made unsigned (u = w + 8 for int4, u = w + 128
+// for int8) and placed unchanged in the low mantissa bits of an f16 whose
+// exponent field is zero: that is the f16 subnormal u * 2^-24, exact, made by
+// one LOP3 per two weights.  int4 nibbles at bits 4-7 of a half become
+// 16 u * 2^-24; they are multiplied with activations scaled by 1/16 (exact in
+// f16), so every product lands on the common scale 2^-24.  The accumulator
+// holds S = sum(u x) * 2^-24 exactly while |sum(u x)| < 2^24 (int4: 8738
+// values of k per warp, int8: 514); int8 partials are flushed to int32 every
+// 512 values of k per warp, int4 never needs a flush (a warp sees at most
+// MQ_MAX_K / 8 = 8192 values of k).  The bias is removed exactly in the
+// epilogue with the token's activation sum: sum(w x) = sum(u x) - 8 sum(x)
+// (int4) or - 128 sum(x) (int8).
 //
-// CTA = 8 warps on one 32-row block of one problem; the warps split K
-// (step-cyclic) and reduce their int32 partials in shared memory; the
-// epilogue subtracts zx * colsum, requantizes (round half up), saturates,
-// adds the optional residual and stores int8.
+// The reduction order over k inside one mma is free, so each fragment slot's
+// k index is whatever the unpacking yields; the activation fragments use the
+// same assignment.
+//
+// Epilogue (per unit): the eight warps' int32 partials and activation sums
+// meet in shared memory; acc = sum(u x) - bias sum(x) - zx colsum[n], then
+// fixed-point requant (round half up), saturation, optional residual, store.
+// All mbarrier waits are bounded (mq_wait_parity).
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
 #include "mq_internal.h"
 #include "mq_ptx.cuh"
@@ -32,288 +50,403 @@
 namespace mq {
 namespace decode {
 
-constexpr int WARPS = 8;
-constexpr int THREADS = WARPS * 32;
-constexpr int R = 2;              // 16-row mma tiles per warp (rows per CTA = 16 * R)
-constexpr int ROWS = 16 * R;
+constexpr int CONS_WARPS = 8;
+constexpr int CONS_THREADS = CONS_WARPS * 32;
+constexpr int PROD_WARP = CONS_WARPS;  // warp 8
+constexpr int THREADS = CONS_THREADS + 32;
+constexpr int UNIT_ROWS = 64;          // four 16-row mma tiles
+constexpr int ROW_BYTES = 128;         // weight bytes per row per stage
+constexpr int W_BYTES = UNIT_ROWS * ROW_BYTES;  // 8 KB of weights
+constexpr int X_BOX = 16 * 128;                 // one x box: 16 tokens x 128 k
+constexpr int STAGE_BYTES = W_BYTES + 2 * X_BOX;
+constexpr int STAGES = 8;
+constexpr int CONS_BARRIER = 1;        // named barrier among the consumer warps
 
 struct Params {
+    CUtensorMap tmap_w[DECODE_MAX_PROBLEMS];  // weight bytes [N][K*bits/8], box 128 x 64, 128B swizzle
+    CUtensorMap tmap_x[DECODE_MAX_PROBLEMS];  // x [M][ldx], box 128 x 16, 128B swizzle
     Problem p[DECODE_MAX_PROBLEMS];
     int count;
-    int total_blocks;
+    int total_units;
     int *status;
 };
 
-__device__ __forceinline__ uint4 ldg16(const void *p) {
-    uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
-    return v;
+struct Smem {
+    uint8_t ring[STAGES][STAGE_BYTES];
+    uint64_t full[STAGES];
+    uint64_t empty[STAGES];
+    int32_t red[UNIT_ROWS][16];   // per (row, token) int32 partial sums
+    int32_t xsum[16];             // per token activation sum over K
+    int abort;
+};
+
+constexpr size_t SMEM_BYTES = sizeof(Smem) + 1024;
+
+__device__ __forceinline__ void cons_sync() {
+    asm volatile("bar.sync %0, %1;" ::"n"(CONS_BARRIER), "n"(CONS_THREADS) : "memory");
 }
 
-__device__ __forceinline__ uint4 ldg16_keep(const void *p) {
-    uint4 v;
-    asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
-    return v;
-}
-
-__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
+__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
     asm volatile(
         "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
         "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Activation int8 words (k0..k3) and (k4..k7) -> f16 pairs (k0,k4) (k1,k5)
-// (k2,k6) (k3,k7), matching the int4 weight pairs below.
-__device__ __forceinline__ void x8_pairs_int4order(uint32_t a, uint32_t b, uint32_t (&o)[4]) {
-    const uint32_t ua = a ^ 0x80808080u, ub = b ^ 0x80808080u;
-    const uint32_t u = prmt(ua, ub, 0x5140u);  // a0 b0 a1 b1
-    const uint32_t v = prmt(ua, ub, 0x7362u);  // a2 b2 a3 b3
-    o[0] = hsub2(prmt(u, 0x64646464u, 0x4140u), F16X2_1152);
-    o[1] = hsub2(prmt(u, 0x64646464u, 0x4342u), F16X2_1152);
-    o[2] = hsub2(prmt(v, 0x64646464u, 0x4140u), F16X2_1152);
-    o[3] = hsub2(prmt(v, 0x64646464u, 0x4342u), F16X2_1152);
+__device__ __forceinline__ int dp4a_sum(uint32_t w, int acc) {
+    return __dp4a((int)w, 0x01010101, acc);
 }
 
-// int4 word (nibble p = k offset p) -> f16 pairs (k0,k4) (k1,k5) (k2,k6) (k3,k7).
-// Pair (p, p+4) sits at bits 4p and 16+4p.  Even p: mantissa = nibble, value
-// 1024 + (e + 8), minus 1032.  Odd p: mantissa = 16 * nibble, value
-// 1024 + 16 (e + 8), times 1/16 minus 72.
-__device__ __forceinline__ void w4_pairs(uint32_t w, uint32_t (&o)[4]) {
-    const uint32_t F16X2_1032 = 0x64086408u;
-    const uint32_t SCALE16 = 0x2C002C00u;  // (1/16, 1/16)
-    const uint32_t OFF72 = 0xD480D480u;    // (-72, -72)
-    const uint32_t w2 = w >> 8;
-    o[0] = hsub2(lop3_sel_xor(w, 0x000F000Fu, 0x64086408u), F16X2_1032);
-    o[1] = hfma2(lop3_sel_xor(w, 0x00F000F0u, 0x64806480u), SCALE16, OFF72);
-    o[2] = hsub2(lop3_sel_xor(w2, 0x000F000Fu, 0x64086408u), F16X2_1032);
-    o[3] = hfma2(lop3_sel_xor(w2, 0x00F000F0u, 0x64806480u), SCALE16, OFF72);
+__device__ __forceinline__ uint32_t lds32(const uint8_t *p) {
+    return *reinterpret_cast<const uint32_t *>(p);
+}
+
+// Two chosen activation bytes of the word pair (a, b) -> an exact f16 pair:
+// byte ^ 0x80 = x + 128 as mantissa of 1024, minus 1152.  `scaled` gives
+// (x/16) instead: (1024 + x + 128)/16 - 72.
+__device__ __forceinline__ uint32_t x_pair(uint32_t a, uint32_t b, uint32_t sel, bool scaled) {
+    const uint32_t t = prmt(a ^ 0x80808080u, b ^ 0x80808080u, sel);  // bytes [p, q, ., .]
+    const uint32_t h = prmt(t, 0x64646464u, 0x5140u);                // bytes [p, 64, q, 64]
+    return scaled ? hfma2(h, 0x2C002C00u, 0xD480D480u) : hsub2(h, F16X2_1152);
 }
 
 template <int BITS>
 struct Cfg;
 template <>
 struct Cfg<4> {
-    static constexpr int KSTEP = 128;       // k per warp step (4 threads x 32)
-    static constexpr int KTHREAD = 32;      // k per thread per step
-    static constexpr int CHUNK_STEPS = 128; // 16384 k between f32 -> int32 flushes
-    static constexpr int MMAS = 8;          // mma k16 per step
+    static constexpr int KSTAGE = 256;       // k per stage (128 bytes per row)
+    static constexpr int KWARP = 32;         // k per consumer warp per stage
+    static constexpr bool FLUSH = false;     // 15 * 128 * 8192 < 2^24
+    static constexpr int FLUSH_STAGES = 1;
+    static constexpr int BIAS = 8;
 };
 template <>
 struct Cfg<8> {
-    static constexpr int KSTEP = 64;
-    static constexpr int KTHREAD = 16;
-    static constexpr int CHUNK_STEPS = 16;  // 1024 k
-    static constexpr int MMAS = 4;
+    static constexpr int KSTAGE = 128;
+    static constexpr int KWARP = 16;
+    static constexpr bool FLUSH = true;
+    static constexpr int FLUSH_STAGES = 32;  // 512 k per warp: 255 * 128 * 512 < 2^24
+    static constexpr int BIAS = 128;
 };
 
-template <int BITS, int NT>
-struct StepRegs {
-    uint4 w[R][2];                     // rows g and g+8 of each 16-row tile
-    uint4 x[NT][BITS == 4 ? 2 : 1];    // this thread's k segment of token g (+8)
-};
-
-template <int BITS, int NT>
-__device__ __forceinline__ void load_step(const Problem &p, int n_base, int step, int g, int t,
-                                          StepRegs<BITS, NT> &r) {
-    using C = Cfg<BITS>;
-    const int k = step * C::KSTEP + t * C::KTHREAD;
-    const bool kin = k < p.K;
-    const size_t row_bytes = (size_t)p.K * BITS / 8;
-    const size_t kbyte = (size_t)k * BITS / 8;
-#pragma unroll
-    for (int rr = 0; rr < R; ++rr)
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int n = n_base + rr * 16 + h * 8 + g;
-            r.w[rr][h] = (kin && n < p.N) ? ldg16(p.w + (size_t)n * row_bytes + kbyte)
-                                          : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-        const int m = nt * 8 + g;
-        const bool ok = kin && m < p.M;
-        const int8_t *src = p.x + (size_t)m * (size_t)p.ldx + k;
-#pragma unroll
-        for (int q = 0; q < (BITS == 4 ? 2 : 1); ++q)
-            r.x[nt][q] = ok ? ldg16_keep(src + 16 * q) : make_uint4(0, 0, 0, 0);
-    }
+__device__ __forceinline__ void unit_at(const Params &P, int u, int &pi, int &rb) {
+    pi = 0;
+    while (pi + 1 < P.count && u >= P.p[pi + 1].tile_begin) ++pi;
+    rb = u - P.p[pi].tile_begin;
 }
 
 template <int BITS, int NT>
-__device__ __forceinline__ void compute_step(const StepRegs<BITS, NT> &r,
-                                             float (&acc)[R][NT][4]) {
-    if constexpr (BITS == 4) {
-        // x: 32 int8 per token = words x0..x7 (k 0..31); word pair (2j, 2j+1)
-        // holds k 8j..8j+7.
+__global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constant__ Params P) {
+    using C = Cfg<BITS>;
+    extern __shared__ uint8_t smem_raw[];
+    Smem &s = *reinterpret_cast<Smem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < STAGES; ++i) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], CONS_WARPS);
+        }
+        s.abort = 0;
+        fence_mbar_init();
+    }
+    for (int i = threadIdx.x; i < UNIT_ROWS * 16; i += THREADS) (&s.red[0][0])[i] = 0;
+    if (threadIdx.x < 16) s.xsum[threadIdx.x] = 0;
+    __syncthreads();
+
+    if (warp == PROD_WARP) {
+        // ------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            for (int i = 0; i < P.count; ++i)
+                if (P.p[i].K > 0) {
+                    prefetch_tensormap(&P.tmap_w[i]);
+                    prefetch_tensormap(&P.tmap_x[i]);
+                }
+            constexpr int XBOXES = C::KSTAGE / 128;  // x boxes per stage (int4: 2, int8: 1)
+            uint32_t it = 0;
+            bool ok = true;
+            for (int u = blockIdx.x; ok && u < P.total_units; u += gridDim.x) {
+                int pi, rb;
+                unit_at(P, u, pi, rb);
+                const int nst = (P.p[pi].K + C::KSTAGE - 1) / C::KSTAGE;
+                for (int j = 0; j < nst; ++j, ++it) {
+                    const int slot = it % STAGES;
+                    if (!mq_wait_parity(&s.empty[slot], ((it / STAGES) & 1) ^ 1, &s.abort,
+                                        P.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&s.full[slot], W_BYTES + XBOXES * X_BOX);
+                    tma_load_2d(s.ring[slot], &P.tmap_w[pi], j * ROW_BYTES, rb * UNIT_ROWS,
+                                &s.full[slot]);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            uint32_t xb[NT][4];
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const uint4 &lo = r.x[nt][j >> 1];
-                const uint32_t wa = (j & 1) ? lo.z : lo.x;
-                const uint32_t wb = (j & 1) ? lo.w : lo.y;
-                x8_pairs_int4order(wa, wb, xb[nt]);
-            }
-#pragma unroll
-            for (int rr = 0; rr < R; ++rr) {
-                const uint32_t w0 = j == 0 ? r.w[rr][0].x : j == 1 ? r.w[rr][0].y
-                                  : j == 2 ? r.w[rr][0].z : r.w[rr][0].w;
-                const uint32_t w1 = j == 0 ? r.w[rr][1].x : j == 1 ? r.w[rr][1].y
-                                  : j == 2 ? r.w[rr][1].z : r.w[rr][1].w;
-                uint32_t pg[4], ph[4];
-                w4_pairs(w0, pg);
-                w4_pairs(w1, ph);
-                const uint32_t a0[4] = {pg[0], ph[0], pg[1], ph[1]};
-                const uint32_t a1[4] = {pg[2], ph[2], pg[3], ph[3]};
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt) {
-                    mma16816(acc[rr][nt], a0, xb[nt][0], xb[nt][1]);
-                    mma16816(acc[rr][nt], a1, xb[nt][2], xb[nt][3]);
+                    for (int h = 0; h < XBOXES; ++h)
+                        tma_load_2d(s.ring[slot] + W_BYTES + h * X_BOX, &P.tmap_x[pi],
+                                    j * C::KSTAGE + h * 128, 0, &s.full[slot]);
                 }
             }
         }
+        __syncwarp();
     } else {
-        // int8: word j of the 16-byte segment holds k 4j..4j+3 (natural pairs).
+        // ------------------------------------------------------ consumers
+        const int g = lane >> 2, t = lane & 3;
+        uint32_t it = 0;
+        bool ok = true;  // after a failed wait the warp still walks the barriers
+        for (int u = blockIdx.x; u < P.total_units; u += gridDim.x) {
+            int pi, rb;
+            unit_at(P, u, pi, rb);
+            const Problem &p = P.p[pi];
+            const int nst = (p.K + C::KSTAGE - 1) / C::KSTAGE;
+            float acc[4][NT][4];
+            int32_t iacc[4][NT][4];
+            int xs[NT];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            uint32_t xb[NT][2];
+            for (int rt = 0; rt < 4; ++rt)
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const uint4 &v = r.x[nt][0];
-                const uint32_t xw = j == 0 ? v.x : j == 1 ? v.y : j == 2 ? v.z : v.w;
-                i8x4_to_f16x4(xw, xb[nt][0], xb[nt][1]);
+                for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        acc[rt][nt][i] = 0.f;
+                        iacc[rt][nt][i] = 0;
+                    }
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) xs[nt] = 0;
+            for (int j = 0; ok && j < nst; ++j, ++it) {
+                const int slot = it % STAGES;
+                bool got = true;
+                if (lane == 0)
+                    got = mq_wait_parity(&s.full[slot], (it / STAGES) & 1, &s.abort, P.status);
+                if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) {
+                    ok = false;
+                    break;
+                }
+                // activation fragment of this warp's k range, token g (+8): the
+                // bytes at stage offset warp * KWARP + t * KWARP/4 of token row m
+                // (zero outside M and K: TMA fill)
+                uint32_t xa[NT], xb[NT];
+                {
+                    const int off = warp * C::KWARP + t * (C::KWARP / 4);
+                    const uint8_t *xbox = s.ring[slot] + W_BYTES + (off >> 7) * X_BOX;
+                    const int c = (off & 127) >> 4, inner = off & 15;
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) {
+                        const int m = nt * 8 + g;
+                        const uint8_t *src = xbox + m * 128 + ((c ^ (m & 7)) << 4) + inner;
+                        if (BITS == 4) {
+                            const uint2 v = *reinterpret_cast<const uint2 *>(src);
+                            xa[nt] = v.x;
+                            xb[nt] = v.y;
+                        } else {
+                            xa[nt] = lds32(src);
+                            xb[nt] = 0u;
+                        }
+                    }
+                }
+                // weight word t of chunk `warp` of rows g and g+8 of the four tiles
+                uint32_t wv[4][2];
+                const uint8_t *ring = s.ring[slot];
+#pragma unroll
+                for (int rt = 0; rt < 4; ++rt)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int row = rt * 16 + h * 8 + g;
+                        wv[rt][h] = lds32(ring + row * ROW_BYTES + ((warp ^ (row & 7)) << 4) + t * 4);
+                    }
+                if constexpr (BITS == 4) {
+                    // x bytes k0..k7 = xa (k0..k3), xb (k4..k7): pairs (k0,k4) (k2,k6)
+                    // at scale 1, (k1,k5) (k3,k7) at scale 1/16
+                    uint32_t b04[NT], b26[NT], b15[NT], b37[NT];
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) {
+                        b04[nt] = x_pair(xa[nt], xb[nt], 0x0040u, false);
+                        b26[nt] = x_pair(xa[nt], xb[nt], 0x0062u, false);
+                        b15[nt] = x_pair(xa[nt], xb[nt], 0x0051u, true);
+                        b37[nt] = x_pair(xa[nt], xb[nt], 0x0073u, true);
+                        xs[nt] = dp4a_sum(xa[nt], dp4a_sum(xb[nt], xs[nt]));
+                    }
+#pragma unroll
+                    for (int rt = 0; rt < 4; ++rt) {
+                        uint32_t pa0[2], pa1[2], pb0[2], pb1[2];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const uint32_t w = wv[rt][h], w2 = w >> 8;
+                            pa0[h] = lop3_sel_xor(w, 0x000F000Fu, 0x00080008u);   // u0, u4
+                            pb0[h] = lop3_sel_xor(w, 0x00F000F0u, 0x00800080u);   // 16 u1, 16 u5
+                            pa1[h] = lop3_sel_xor(w2, 0x000F000Fu, 0x00080008u);  // u2, u6
+                            pb1[h] = lop3_sel_xor(w2, 0x00F000F0u, 0x00800080u);  // 16 u3, 16 u7
+                        }
+#pragma unroll
+                        for (int nt = 0; nt < NT; ++nt) {
+                            mma16816(acc[rt][nt], pa0[0], pa0[1], pa1[0], pa1[1], b04[nt], b26[nt]);
+                            mma16816(acc[rt][nt], pb0[0], pb0[1], pb1[0], pb1[1], b15[nt], b37[nt]);
+                        }
+                    }
+                } else {
+                    // x bytes k0..k3: pairs (k0,k2), (k1,k3)
+                    uint32_t b02[NT], b13[NT];
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) {
+                        b02[nt] = x_pair(xa[nt], xa[nt], 0x0020u, false);
+                        b13[nt] = x_pair(xa[nt], xa[nt], 0x0031u, false);
+                        xs[nt] = dp4a_sum(xa[nt], xs[nt]);
+                    }
+#pragma unroll
+                    for (int rt = 0; rt < 4; ++rt) {
+                        uint32_t pa[2], pb[2];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const uint32_t w = wv[rt][h];
+                            pa[h] = lop3_sel_xor(w, 0x00FF00FFu, 0x00800080u);       // u0, u2
+                            pb[h] = lop3_sel_xor(w >> 8, 0x00FF00FFu, 0x00800080u);  // u1, u3
+                        }
+#pragma unroll
+                        for (int nt = 0; nt < NT; ++nt)
+                            mma16816(acc[rt][nt], pa[0], pa[1], pb[0], pb[1], b02[nt], b13[nt]);
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s.empty[slot]);
+                if constexpr (C::FLUSH) {
+                    if ((j + 1) % C::FLUSH_STAGES == 0) {
+#pragma unroll
+                        for (int rt = 0; rt < 4; ++rt)
+#pragma unroll
+                            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) {
+                                    iacc[rt][nt][i] +=
+                                        __float2int_rn(acc[rt][nt][i] * 16777216.0f);
+                                    acc[rt][nt][i] = 0.f;
+                                }
+                    }
+                }
             }
+            // ---- reduce the eight warps' partials: fragment element i of tile
+            // (rt, nt) is row rt*16 + g (+8 for i >= 2), token nt*8 + 2t + (i & 1)
+            if (ok) {
 #pragma unroll
-            for (int rr = 0; rr < R; ++rr) {
-                const uint32_t w0 = j == 0 ? r.w[rr][0].x : j == 1 ? r.w[rr][0].y
-                                  : j == 2 ? r.w[rr][0].z : r.w[rr][0].w;
-                const uint32_t w1 = j == 0 ? r.w[rr][1].x : j == 1 ? r.w[rr][1].y
-                                  : j == 2 ? r.w[rr][1].z : r.w[rr][1].w;
-                uint32_t g0, g1, h0, h1;
-                i8x4_to_f16x4(w0, g0, g1);
-                i8x4_to_f16x4(w1, h0, h1);
-                const uint32_t a[4] = {g0, h0, g1, h1};
+                for (int rt = 0; rt < 4; ++rt)
 #pragma unroll
-                for (int nt = 0; nt < NT; ++nt) mma16816(acc[rr][nt], a, xb[nt][0], xb[nt][1]);
+                    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const int row = rt * 16 + g + (i >= 2 ? 8 : 0);
+                            const int tok = nt * 8 + 2 * t + (i & 1);
+                            int32_t v = __float2int_rn(acc[rt][nt][i] * 16777216.0f);
+                            if constexpr (C::FLUSH) v += iacc[rt][nt][i];
+                            if (tok < p.M) atomicAdd(&s.red[row][tok], v);
+                        }
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                    int v = xs[nt];
+                    v += __shfl_xor_sync(0xffffffffu, v, 1);
+                    v += __shfl_xor_sync(0xffffffffu, v, 2);
+                    if (t == 0 && nt * 8 + g < p.M) atomicAdd(&s.xsum[nt * 8 + g], v);
+                }
             }
+            cons_sync();
+            if (ok) {
+                for (int idx = threadIdx.x; idx < UNIT_ROWS * p.M; idx += CONS_THREADS) {
+                    const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
+                    const int n = rb * UNIT_ROWS + row;
+                    const int32_t sum = s.red[row][tok];
+                    s.red[row][tok] = 0;
+                    if (n >= p.N) continue;
+                    const int32_t cs = __ldg(p.colsum + n);
+                    const int32_t m0 = __ldg(p.M0 + n);
+                    const int32_t sh = __ldg(p.shift + n);
+                    // sum(w x) = sum(u x) - bias * sum(x); acc = sum(w x) - zx colsum
+                    // (two's-complement wrap is exact: the result fits in int32)
+                    const int32_t a = (int32_t)((uint32_t)sum -
+                                                (uint32_t)(C::BIAS * s.xsum[tok]) -
+                                                (uint32_t)(p.zx * cs));
+                    const int64_t v = (int64_t)a * (int64_t)m0;
+                    const int64_t q = (v + ((int64_t)1 << (sh - 1))) >> sh;
+                    int64_t yv = (int64_t)p.zy + q;
+                    yv = yv < -128 ? -128 : (yv > 127 ? 127 : yv);
+                    if (p.residual) {
+                        yv += (int64_t)p.residual[(size_t)tok * (size_t)p.ldy + n];
+                        yv = yv < -128 ? -128 : (yv > 127 ? 127 : yv);
+                    }
+                    p.y[(size_t)tok * (size_t)p.ldy + n] = (int8_t)yv;
+                }
+            }
+            cons_sync();  // every read of red / xsum of this unit is done
+            if (threadIdx.x < 16) s.xsum[threadIdx.x] = 0;
+            cons_sync();
         }
     }
+    __syncthreads();
 }
 
-template <int BITS, int NT>
-__device__ __forceinline__ void flush(float (&acc)[R][NT][4], int32_t (&iacc)[R][NT][4]) {
-#pragma unroll
-    for (int rr = 0; rr < R; ++rr)
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                iacc[rr][nt][i] += __float2int_rn(acc[rr][nt][i]);
-                acc[rr][nt][i] = 0.f;
-            }
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    }
+    return fn;
 }
 
-template <int BITS, int NT>
-__global__ void __launch_bounds__(THREADS) decode_kernel(const __grid_constant__ Params P) {
-    using C = Cfg<BITS>;
-    __shared__ int32_t red[ROWS][16];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = lane >> 2, t = lane & 3;
-
-    int pi = 0;
-    while (pi + 1 < P.count && (int)blockIdx.x >= P.p[pi + 1].tile_begin) ++pi;
-    const Problem &p = P.p[pi];
-    const int n_base = ((int)blockIdx.x - p.tile_begin) * ROWS;
-
-    for (int i = threadIdx.x; i < ROWS * 16; i += THREADS) (&red[0][0])[i] = 0;
-    __syncthreads();
-
-    float acc[R][NT][4];
-    int32_t iacc[R][NT][4];
-#pragma unroll
-    for (int rr = 0; rr < R; ++rr)
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                acc[rr][nt][i] = 0.f;
-                iacc[rr][nt][i] = 0;
-            }
-
-    const int nsteps = (p.K + C::KSTEP - 1) / C::KSTEP;
-    StepRegs<BITS, NT> cur, nxt;
-    int step = warp;
-    if (step < nsteps) load_step<BITS, NT>(p, n_base, step, g, t, nxt);
-    int local = 0;
-    while (step < nsteps) {
-        cur = nxt;
-        const int next = step + WARPS;
-        if (next < nsteps) load_step<BITS, NT>(p, n_base, next, g, t, nxt);
-        compute_step<BITS, NT>(cur, acc);
-        if (++local == C::CHUNK_STEPS) {
-            flush<BITS, NT>(acc, iacc);
-            local = 0;
-        }
-        step = next;
-    }
-    flush<BITS, NT>(acc, iacc);
-
-    // cross-warp reduction of the int32 partials: fragment element i of tile
-    // (rr, nt) is row rr*16 + g (+8 for i >= 2), token nt*8 + 2t + (i & 1)
-#pragma unroll
-    for (int rr = 0; rr < R; ++rr)
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int row = rr * 16 + g + (i >= 2 ? 8 : 0);
-                const int tok = nt * 8 + 2 * t + (i & 1);
-                if (tok < p.M) atomicAdd(&red[row][tok], iacc[rr][nt][i]);
-            }
-    __syncthreads();
-
-    for (int idx = threadIdx.x; idx < ROWS * p.M; idx += THREADS) {
-        const int row = idx % ROWS, tok = idx / ROWS;
-        const int n = n_base + row;
-        if (n >= p.N) continue;
-        const int32_t cs = __ldg(p.colsum + n);
-        const int32_t m0 = __ldg(p.M0 + n);
-        const int32_t sh = __ldg(p.shift + n);
-        const int32_t a = (int32_t)((uint32_t)red[row][tok] - (uint32_t)(p.zx * cs));
-        const int64_t v = (int64_t)a * (int64_t)m0;
-        const int64_t q = (v + ((int64_t)1 << (sh - 1))) >> sh;
-        int64_t yv = (int64_t)p.zy + q;
-        yv = yv < -128 ? -128 : (yv > 127 ? 127 : yv);
-        if (p.residual) {
-            yv += (int64_t)p.residual[(size_t)tok * (size_t)p.ldy + n];
-            yv = yv < -128 ? -128 : (yv > 127 ? 127 : yv);
-        }
-        p.y[(size_t)tok * (size_t)p.ldy + n] = (int8_t)yv;
-    }
+// uint8 tensor [rows][cols] with row pitch `pitch`, box 128 x box_rows, 128-byte swizzle.
+bool encode_sw128(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows,
+                  uint64_t pitch, uint32_t box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {pitch};
+    const cuuint32_t box[2] = {ROW_BYTES, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
 }
 
 template <int BITS, int NT>
 int launch_t(const Problem *probs, int count, cudaStream_t stream) {
+    auto kern = decode_kernel<BITS, NT>;
+    static int attr_done = -1;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
+    if (attr_done != dev) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)SMEM_BYTES) != cudaSuccess)
+            return MQ_ERR_CUDA;
+        attr_done = dev;
+    }
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return MQ_ERR_CUDA;
     for (int begin = 0; begin < count; begin += DECODE_MAX_PROBLEMS) {
         const int n = count - begin < DECODE_MAX_PROBLEMS ? count - begin : DECODE_MAX_PROBLEMS;
         Params P{};
-        int blocks = 0;
+        int units = 0;
         for (int i = 0; i < n; ++i) {
-            P.p[i] = probs[begin + i];
-            P.p[i].tile_begin = blocks;
-            blocks += (P.p[i].N + ROWS - 1) / ROWS;
+            Problem &q = P.p[i];
+            q = probs[begin + i];
+            q.tile_begin = units;
+            units += (q.N + UNIT_ROWS - 1) / UNIT_ROWS;
+            const uint64_t wcols = (uint64_t)q.K * BITS / 8;
+            if (q.K > 0 &&
+                (!encode_sw128(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, wcols, UNIT_ROWS) ||
+                 !encode_sw128(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M, (uint64_t)q.ldx,
+                               16)))
+                return MQ_ERR_CUDA;
         }
         P.count = n;
-        P.total_blocks = blocks;
+        P.total_units = units;
         P.status = device_status_ptr();
-        if (blocks == 0) continue;
-        decode_kernel<BITS, NT><<<blocks, THREADS, 0, stream>>>(P);
+        if (units == 0) continue;
+        const int grid = units < 2 * sms ? units : 2 * sms;
+        kern<<<grid, THREADS, SMEM_BYTES, stream>>>(P);
         if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;

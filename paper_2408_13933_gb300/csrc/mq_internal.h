@@ -33,7 +33,7 @@ constexpr int DECODE_MAX_M = 16;
 
 // Problems per kernel launch (kernel parameter space).
 constexpr int PREFILL_MAX_PROBLEMS = 32;
-constexpr int DECODE_MAX_PROBLEMS = 128;
+constexpr int DECODE_MAX_PROBLEMS = 64;
 
 // Device status words (__device__ ints owned by libmq, addresses cached per
 // device): kernels atomicOr MQ_DEVICE_STATUS_* bits into them.  The pack
