@@ -293,7 +293,11 @@ def run_decode(mq, torch, steps_per_m: int = 240):
     wbytes = block_weight_bytes(4)
     stream = torch.cuda.current_stream()
     layers = [DecodeLayer(mq, torch, layer) for layer in range(DECODE_LAYERS)]
-    call = mq.lib.mq_linear_batch
+    ws = mq.workspace()
+    wsp, wsn = ws.data_ptr(), ws.numel()
+
+    def call(arr, count, _ws, _n, strm):
+        return mq.lib.mq_linear_batch(arr, count, wsp, wsn, strm)
     sp = stream.cuda_stream
     for m in DECODE_MS:
         for L in layers * 2:

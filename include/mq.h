@@ -97,9 +97,20 @@ int mq_packed_size(int N, int K, int bits, size_t *bytes);
 int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed,
                     int32_t *colsum, int on_device, void *stream);
 
-/* Device workspace bytes a mq_linear_* call of this shape needs (0 for every
- * shape in this version; kept so that callers need not change when a kernel
- * starts to use one).  Errors: MQ_ERR_INVALID_ARG. */
+/*
+ * Device workspace bytes a mq_linear_* call of this shape needs: 0 for the
+ * tensor-core path (M > 16); for the decode path (1 <= M <= 16) a fixed size
+ * (about 1.3 MB) holding per-CTA int32 partial sums and counters, used to
+ * combine 64-row units whose K range is split among CTAs.  For
+ * mq_linear_batch the workspace must hold the largest size of its
+ * descriptors.
+ * Workspace contract: device memory, 16-byte aligned, zero-filled before its
+ * first use; every call that completes leaves it zero-filled again, so it can
+ * be reused by later calls on the same stream.  Calls that may run
+ * concurrently (different streams) need different workspaces.  After
+ * MQ_ERR_DEVICE_TIMEOUT the workspace must be zero-filled again.
+ * Errors: MQ_ERR_INVALID_ARG.
+ */
 int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes);
 
 /*
@@ -111,14 +122,16 @@ int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes);
  *   M0, shift: device int32 [N], from mq_requant_params
  *   zy       : output zero point in [-128, 127]
  *   y        : device int8 [M][ldy], ldy >= N, written
- *   workspace: device, ws_bytes >= mq_workspace_size (may be NULL when 0)
+ *   workspace: device, ws_bytes >= mq_workspace_size (may be NULL when 0);
+ *              see the workspace contract at mq_workspace_size
  * Requirements: 0 <= M, N; 0 <= K <= MQ_MAX_K; K % 16 == 0; ldx % 16 == 0;
  * x and packed 16-byte aligned.  With K == 0 (every output is requant(0),
  * i.e. zy) x and packed are not read and may be NULL.  M <= 16 runs the
  * weight-streaming decode kernel, larger M the tcgen05 tensor-core kernel;
  * both are bit-exact.
  * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_K_OVERFLOW, MQ_ERR_ALIGNMENT,
- * MQ_ERR_WORKSPACE, MQ_ERR_CUDA (launch failure).
+ * MQ_ERR_WORKSPACE (decode shape without a large enough workspace),
+ * MQ_ERR_CUDA (launch failure).
  */
 int mq_linear_w8a8(const int8_t *x, int M, int K, int ldx, int32_t zx,
                    const void *packed, const int32_t *colsum, int N,

@@ -5,10 +5,18 @@
 // it, so its speed is the weight stream (the paper notes that autoregressive
 // generation is memory-bound, Sec. 5.6 and Appendix A.2).
 //
-// Data path.  A persistent grid of CTAs (two per SM) walks 64-row units of
-// up to DECODE_MAX_PROBLEMS linears.  In each CTA one producer thread streams
-// the weight rows of its units with TMA into an 8-stage shared-memory ring,
-// continuing across unit boundaries.  A stage holds 64 weight rows x 128
+// Schedule (stream-K).  The work of up to DECODE_MAX_PROBLEMS linears is cut
+// into 64-row units and each unit into stages of KSTAGE values of k; the
+// global sequence of stages is split evenly among the CTAs of a persistent
+// grid (two per SM), so every SM streams the same number of weight bytes no
+// matter how the linears' sizes differ.  A unit whose stages fall to several
+// CTAs is combined in the caller's workspace: each contributor adds its int32
+// partial sums with atomics and counts itself in; the last one requantizes,
+// stores, and leaves the slot and counter zero again.
+//
+// Data path.  In each CTA one producer thread streams the weight rows of its
+// stages with TMA into an 8-stage shared-memory ring, continuing across unit
+// boundaries.  A stage holds 64 weight rows x 128
 // bytes and the matching k slice of the 16 (zero-padded) token rows of x,
 // both 128-byte swizzled, so up to 64 KB of weights per CTA are in flight and
 // the activation fragments come from shared memory without bank conflicts.
@@ -65,9 +73,11 @@ constexpr int CONS_BARRIER = 1;        // named barrier among the consumer warps
 struct Params {
     CUtensorMap tmap_w[DECODE_MAX_PROBLEMS];  // weight bytes [N][K*bits/8], box 128 x 64, 128B swizzle
     CUtensorMap tmap_x[DECODE_MAX_PROBLEMS];  // x [M][ldx], box 128 x 16, 128B swizzle
-    Problem p[DECODE_MAX_PROBLEMS];
+    Problem p[DECODE_MAX_PROBLEMS];  // tile_begin = first global stage, tiles_m = stages per unit
     int count;
-    int total_units;
+    int total_stages;
+    int32_t *ws_count;   // [gridDim.x] contributor counters (zero between calls)
+    int32_t *ws_sum;     // [gridDim.x][UNIT_ROWS][16] partial sums (zero between calls)
     int *status;
 };
 
@@ -76,7 +86,12 @@ struct Smem {
     uint64_t full[STAGES];
     uint64_t empty[STAGES];
     int32_t red[UNIT_ROWS][16];   // per (row, token) int32 partial sums
-    int32_t xsum[16];             // per token activation sum over K
+    int32_t xsum[2][16];          // per token activation sum, by piece parity
+    int32_t row_corr[UNIT_ROWS];  // zx * colsum[n] of the current unit's rows
+    int32_t row_m0[UNIT_ROWS];
+    int32_t row_shift[UNIT_ROWS];
+    Problem prob[DECODE_MAX_PROBLEMS];  // the kernel's problem table, read once
+    int last[2];                  // this CTA completes a split unit, by piece parity
     int abort;
 };
 
@@ -131,10 +146,128 @@ struct Cfg<8> {
     static constexpr int BIAS = 128;
 };
 
-__device__ __forceinline__ void unit_at(const Params &P, int u, int &pi, int &rb) {
-    pi = 0;
-    while (pi + 1 < P.count && u >= P.p[pi + 1].tile_begin) ++pi;
-    rb = u - P.p[pi].tile_begin;
+// First global stage of CTA c when S stages are split among G CTAs.
+__device__ __forceinline__ int range_begin(int c, int S, int G) {
+    return (int)(((long long)c * S) / G);
+}
+
+// The CTA whose range holds global stage s.
+__device__ __forceinline__ int cta_of(int s, int S, int G) {
+    int c = (int)(((long long)s * G) / S);
+    while (c + 1 < G && range_begin(c + 1, S, G) <= s) ++c;
+    while (c > 0 && range_begin(c, S, G) > s) --c;
+    return c;
+}
+
+// Problem holding global stage s, searching forward from `pi` (stages are
+// visited in increasing order, so the walk is amortized O(1)).
+__device__ __forceinline__ int problem_from(const Smem &sm, int count, int pi, int s) {
+    while (pi + 1 < count && s >= sm.prob[pi + 1].tile_begin) ++pi;
+    return pi;
+}
+
+// Requantize one output of tile row `row` (global row n, token tok) from
+// sum(w x): acc = sum(w x) - zx colsum[n], fixed point, saturate, optional
+// residual.
+__device__ __forceinline__ void store_out(const Problem &p, const Smem &sm, int row, int n,
+                                          int tok, int32_t sum_wx) {
+    // two's-complement wrap is exact: the true value fits in int32
+    const int32_t a = (int32_t)((uint32_t)sum_wx - (uint32_t)sm.row_corr[row]);
+    int32_t y = mq_requant(a, sm.row_m0[row], sm.row_shift[row], p.zy);
+    if (p.residual)
+        y = min(127, max(-128, y + (int32_t)p.residual[(size_t)tok * (size_t)p.ldy + n]));
+    p.y[(size_t)tok * (size_t)p.ldy + n] = (int8_t)y;
+}
+
+// One stage of one warp: activation fragment and weight words from the ring
+// slot, widening, mma.  Returns nothing; accumulates into acc and xs.
+template <int BITS, int NT>
+__device__ __forceinline__ void compute_stage(const uint8_t *ring, int warp, int g, int t,
+                                              float (&acc)[4][NT][4], int (&xs)[NT]) {
+    using C = Cfg<BITS>;
+    // activation fragment of this warp's k range, token g (+8): the bytes at
+    // stage offset warp * KWARP + t * KWARP/4 of token row m (zero outside M
+    // and K: TMA fill)
+    uint32_t xa[NT], xb[NT];
+    {
+        const int off = warp * C::KWARP + t * (C::KWARP / 4);
+        const uint8_t *xbox = ring + W_BYTES + (off >> 7) * X_BOX;
+        const int c = (off & 127) >> 4, inner = off & 15;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            const int m = nt * 8 + g;
+            const uint8_t *src = xbox + m * 128 + ((c ^ (m & 7)) << 4) + inner;
+            if (BITS == 4) {
+                const uint2 v = *reinterpret_cast<const uint2 *>(src);
+                xa[nt] = v.x;
+                xb[nt] = v.y;
+            } else {
+                xa[nt] = lds32(src);
+                xb[nt] = 0u;
+            }
+        }
+    }
+    // weight word t of chunk `warp` of rows g and g+8 of the four tiles
+    uint32_t wv[4][2];
+#pragma unroll
+    for (int rt = 0; rt < 4; ++rt)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int row = rt * 16 + h * 8 + g;
+            wv[rt][h] = lds32(ring + row * ROW_BYTES + ((warp ^ (row & 7)) << 4) + t * 4);
+        }
+    if constexpr (BITS == 4) {
+        // x bytes k0..k7 = xa (k0..k3), xb (k4..k7): pairs (k0,k4) (k2,k6) at
+        // scale 1, (k1,k5) (k3,k7) at scale 1/16
+        uint32_t b04[NT], b26[NT], b15[NT], b37[NT];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            b04[nt] = x_pair(xa[nt], xb[nt], 0x0040u, false);
+            b26[nt] = x_pair(xa[nt], xb[nt], 0x0062u, false);
+            b15[nt] = x_pair(xa[nt], xb[nt], 0x0051u, true);
+            b37[nt] = x_pair(xa[nt], xb[nt], 0x0073u, true);
+            xs[nt] = dp4a_sum(xa[nt], dp4a_sum(xb[nt], xs[nt]));
+        }
+#pragma unroll
+        for (int rt = 0; rt < 4; ++rt) {
+            uint32_t pa0[2], pa1[2], pb0[2], pb1[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const uint32_t w = wv[rt][h], w2 = w >> 8;
+                pa0[h] = lop3_sel_xor(w, 0x000F000Fu, 0x00080008u);   // u0, u4
+                pb0[h] = lop3_sel_xor(w, 0x00F000F0u, 0x00800080u);   // 16 u1, 16 u5
+                pa1[h] = lop3_sel_xor(w2, 0x000F000Fu, 0x00080008u);  // u2, u6
+                pb1[h] = lop3_sel_xor(w2, 0x00F000F0u, 0x00800080u);  // 16 u3, 16 u7
+            }
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                mma16816(acc[rt][nt], pa0[0], pa0[1], pa1[0], pa1[1], b04[nt], b26[nt]);
+                mma16816(acc[rt][nt], pb0[0], pb0[1], pb1[0], pb1[1], b15[nt], b37[nt]);
+            }
+        }
+    } else {
+        // x bytes k0..k3: pairs (k0,k2), (k1,k3)
+        uint32_t b02[NT], b13[NT];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            b02[nt] = x_pair(xa[nt], xa[nt], 0x0020u, false);
+            b13[nt] = x_pair(xa[nt], xa[nt], 0x0031u, false);
+            xs[nt] = dp4a_sum(xa[nt], xs[nt]);
+        }
+#pragma unroll
+        for (int rt = 0; rt < 4; ++rt) {
+            uint32_t pa[2], pb[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const uint32_t w = wv[rt][h];
+                pa[h] = lop3_sel_xor(w, 0x00FF00FFu, 0x00800080u);       // u0, u2
+                pb[h] = lop3_sel_xor(w >> 8, 0x00FF00FFu, 0x00800080u);  // u1, u3
+            }
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+                mma16816(acc[rt][nt], pa[0], pa[1], pb[0], pb[1], b02[nt], b13[nt]);
+        }
+    }
 }
 
 template <int BITS, int NT>
@@ -144,6 +277,8 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
     Smem &s = *reinterpret_cast<Smem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int S = P.total_stages, G = gridDim.x, cta = blockIdx.x;
+    const int s_begin = range_begin(cta, S, G), s_end = range_begin(cta + 1, S, G);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
@@ -151,11 +286,14 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             mbar_init(&s.empty[i], CONS_WARPS);
         }
         s.abort = 0;
+        s.last[0] = s.last[1] = 0;
         fence_mbar_init();
     }
     for (int i = threadIdx.x; i < UNIT_ROWS * 16; i += THREADS) (&s.red[0][0])[i] = 0;
-    if (threadIdx.x < 16) s.xsum[threadIdx.x] = 0;
+    if (threadIdx.x < 32) (&s.xsum[0][0])[threadIdx.x] = 0;
+    for (int i = threadIdx.x; i < P.count; i += THREADS) s.prob[i] = P.p[i];
     __syncthreads();
+    const int count = P.count;
 
     if (warp == PROD_WARP) {
         // ------------------------------------------------------ TMA producer
@@ -167,26 +305,26 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                 }
             constexpr int XBOXES = C::KSTAGE / 128;  // x boxes per stage (int4: 2, int8: 1)
             uint32_t it = 0;
-            bool ok = true;
-            for (int u = blockIdx.x; ok && u < P.total_units; u += gridDim.x) {
-                int pi, rb;
-                unit_at(P, u, pi, rb);
-                const int nst = (P.p[pi].K + C::KSTAGE - 1) / C::KSTAGE;
-                for (int j = 0; j < nst; ++j, ++it) {
-                    const int slot = it % STAGES;
-                    if (!mq_wait_parity(&s.empty[slot], ((it / STAGES) & 1) ^ 1, &s.abort,
-                                        P.status)) {
-                        ok = false;
-                        break;
-                    }
-                    mbar_arrive_expect_tx(&s.full[slot], W_BYTES + XBOXES * X_BOX);
-                    tma_load_2d(s.ring[slot], &P.tmap_w[pi], j * ROW_BYTES, rb * UNIT_ROWS,
-                                &s.full[slot]);
-#pragma unroll
-                    for (int h = 0; h < XBOXES; ++h)
-                        tma_load_2d(s.ring[slot] + W_BYTES + h * X_BOX, &P.tmap_x[pi],
-                                    j * C::KSTAGE + h * 128, 0, &s.full[slot]);
+            int pi = 0;
+            for (int gs = s_begin; gs < s_end; ++gs, ++it) {
+                pi = problem_from(s, count, pi, gs);
+                const Problem &p = s.prob[pi];
+                const int local = gs - p.tile_begin;
+                const int rb = local / p.tiles_m, j = local % p.tiles_m;
+                const int slot = it % STAGES;
+                if (!mq_wait_parity(&s.empty[slot], ((it / STAGES) & 1) ^ 1, &s.abort, P.status))
+                    break;
+                if (p.K == 0) {  // an empty stage: nothing to load
+                    mbar_arrive(&s.full[slot]);
+                    continue;
                 }
+                mbar_arrive_expect_tx(&s.full[slot], W_BYTES + XBOXES * X_BOX);
+                tma_load_2d(s.ring[slot], &P.tmap_w[pi], j * ROW_BYTES, rb * UNIT_ROWS,
+                            &s.full[slot]);
+#pragma unroll
+                for (int h = 0; h < XBOXES; ++h)
+                    tma_load_2d(s.ring[slot] + W_BYTES + h * X_BOX, &P.tmap_x[pi],
+                                j * C::KSTAGE + h * 128, 0, &s.full[slot]);
             }
         }
         __syncwarp();
@@ -194,12 +332,31 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
         // ------------------------------------------------------ consumers
         const int g = lane >> 2, t = lane & 3;
         uint32_t it = 0;
-        bool ok = true;  // after a failed wait the warp still walks the barriers
-        for (int u = blockIdx.x; u < P.total_units; u += gridDim.x) {
-            int pi, rb;
-            unit_at(P, u, pi, rb);
-            const Problem &p = P.p[pi];
-            const int nst = (p.K + C::KSTAGE - 1) / C::KSTAGE;
+        bool ok = true;  // after a failed wait the warps still walk the barriers
+        int gs = s_begin;
+        int pi = 0;
+        int par = 0;  // piece parity: selects xsum / last buffers
+        while (gs < s_end) {
+            // the piece [gs, piece_end) of one unit that this CTA owns
+            pi = problem_from(s, count, pi, gs);
+            const Problem &p = s.prob[pi];
+            const int nst = p.tiles_m;
+            const int local = gs - p.tile_begin;
+            const int rb = local / nst;
+            const int u_begin = p.tile_begin + rb * nst, u_end = u_begin + nst;
+            const int piece_end = u_end < s_end ? u_end : s_end;
+            // requant parameters of the unit's rows: loaded now, published to
+            // shared memory when the piece is done, so the loads overlap the
+            // stage loop instead of stalling the warp here
+            int32_t prm_cs = 0, prm_m0 = 0, prm_sh = 33;
+            if (threadIdx.x < UNIT_ROWS) {
+                const int n = rb * UNIT_ROWS + threadIdx.x;
+                if (n < p.N) {
+                    prm_cs = __ldg(p.colsum + n);
+                    prm_m0 = __ldg(p.M0 + n);
+                    prm_sh = __ldg(p.shift + n);
+                }
+            }
             float acc[4][NT][4];
             int32_t iacc[4][NT][4];
             int xs[NT];
@@ -214,7 +371,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     }
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) xs[nt] = 0;
-            for (int j = 0; ok && j < nst; ++j, ++it) {
+            for (int q = gs; ok && q < piece_end; ++q, ++it) {
                 const int slot = it % STAGES;
                 bool got = true;
                 if (lane == 0)
@@ -223,94 +380,11 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     ok = false;
                     break;
                 }
-                // activation fragment of this warp's k range, token g (+8): the
-                // bytes at stage offset warp * KWARP + t * KWARP/4 of token row m
-                // (zero outside M and K: TMA fill)
-                uint32_t xa[NT], xb[NT];
-                {
-                    const int off = warp * C::KWARP + t * (C::KWARP / 4);
-                    const uint8_t *xbox = s.ring[slot] + W_BYTES + (off >> 7) * X_BOX;
-                    const int c = (off & 127) >> 4, inner = off & 15;
-#pragma unroll
-                    for (int nt = 0; nt < NT; ++nt) {
-                        const int m = nt * 8 + g;
-                        const uint8_t *src = xbox + m * 128 + ((c ^ (m & 7)) << 4) + inner;
-                        if (BITS == 4) {
-                            const uint2 v = *reinterpret_cast<const uint2 *>(src);
-                            xa[nt] = v.x;
-                            xb[nt] = v.y;
-                        } else {
-                            xa[nt] = lds32(src);
-                            xb[nt] = 0u;
-                        }
-                    }
-                }
-                // weight word t of chunk `warp` of rows g and g+8 of the four tiles
-                uint32_t wv[4][2];
-                const uint8_t *ring = s.ring[slot];
-#pragma unroll
-                for (int rt = 0; rt < 4; ++rt)
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const int row = rt * 16 + h * 8 + g;
-                        wv[rt][h] = lds32(ring + row * ROW_BYTES + ((warp ^ (row & 7)) << 4) + t * 4);
-                    }
-                if constexpr (BITS == 4) {
-                    // x bytes k0..k7 = xa (k0..k3), xb (k4..k7): pairs (k0,k4) (k2,k6)
-                    // at scale 1, (k1,k5) (k3,k7) at scale 1/16
-                    uint32_t b04[NT], b26[NT], b15[NT], b37[NT];
-#pragma unroll
-                    for (int nt = 0; nt < NT; ++nt) {
-                        b04[nt] = x_pair(xa[nt], xb[nt], 0x0040u, false);
-                        b26[nt] = x_pair(xa[nt], xb[nt], 0x0062u, false);
-                        b15[nt] = x_pair(xa[nt], xb[nt], 0x0051u, true);
-                        b37[nt] = x_pair(xa[nt], xb[nt], 0x0073u, true);
-                        xs[nt] = dp4a_sum(xa[nt], dp4a_sum(xb[nt], xs[nt]));
-                    }
-#pragma unroll
-                    for (int rt = 0; rt < 4; ++rt) {
-                        uint32_t pa0[2], pa1[2], pb0[2], pb1[2];
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            const uint32_t w = wv[rt][h], w2 = w >> 8;
-                            pa0[h] = lop3_sel_xor(w, 0x000F000Fu, 0x00080008u);   // u0, u4
-                            pb0[h] = lop3_sel_xor(w, 0x00F000F0u, 0x00800080u);   // 16 u1, 16 u5
-                            pa1[h] = lop3_sel_xor(w2, 0x000F000Fu, 0x00080008u);  // u2, u6
-                            pb1[h] = lop3_sel_xor(w2, 0x00F000F0u, 0x00800080u);  // 16 u3, 16 u7
-                        }
-#pragma unroll
-                        for (int nt = 0; nt < NT; ++nt) {
-                            mma16816(acc[rt][nt], pa0[0], pa0[1], pa1[0], pa1[1], b04[nt], b26[nt]);
-                            mma16816(acc[rt][nt], pb0[0], pb0[1], pb1[0], pb1[1], b15[nt], b37[nt]);
-                        }
-                    }
-                } else {
-                    // x bytes k0..k3: pairs (k0,k2), (k1,k3)
-                    uint32_t b02[NT], b13[NT];
-#pragma unroll
-                    for (int nt = 0; nt < NT; ++nt) {
-                        b02[nt] = x_pair(xa[nt], xa[nt], 0x0020u, false);
-                        b13[nt] = x_pair(xa[nt], xa[nt], 0x0031u, false);
-                        xs[nt] = dp4a_sum(xa[nt], xs[nt]);
-                    }
-#pragma unroll
-                    for (int rt = 0; rt < 4; ++rt) {
-                        uint32_t pa[2], pb[2];
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            const uint32_t w = wv[rt][h];
-                            pa[h] = lop3_sel_xor(w, 0x00FF00FFu, 0x00800080u);       // u0, u2
-                            pb[h] = lop3_sel_xor(w >> 8, 0x00FF00FFu, 0x00800080u);  // u1, u3
-                        }
-#pragma unroll
-                        for (int nt = 0; nt < NT; ++nt)
-                            mma16816(acc[rt][nt], pa[0], pa[1], pb[0], pb[1], b02[nt], b13[nt]);
-                    }
-                }
+                if (p.K > 0) compute_stage<BITS, NT>(s.ring[slot], warp, g, t, acc, xs);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&s.empty[slot]);
                 if constexpr (C::FLUSH) {
-                    if ((j + 1) % C::FLUSH_STAGES == 0) {
+                    if ((q - gs + 1) % C::FLUSH_STAGES == 0) {
 #pragma unroll
                         for (int rt = 0; rt < 4; ++rt)
 #pragma unroll
@@ -324,7 +398,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     }
                 }
             }
-            // ---- reduce the eight warps' partials: fragment element i of tile
+            // ---- this CTA's partial of the unit: fragment element i of tile
             // (rt, nt) is row rt*16 + g (+8 for i >= 2), token nt*8 + 2t + (i & 1)
             if (ok) {
 #pragma unroll
@@ -344,39 +418,77 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     int v = xs[nt];
                     v += __shfl_xor_sync(0xffffffffu, v, 1);
                     v += __shfl_xor_sync(0xffffffffu, v, 2);
-                    if (t == 0 && nt * 8 + g < p.M) atomicAdd(&s.xsum[nt * 8 + g], v);
+                    if (t == 0 && nt * 8 + g < p.M) atomicAdd(&s.xsum[par][nt * 8 + g], v);
                 }
             }
+            if (threadIdx.x < UNIT_ROWS) {
+                s.row_corr[threadIdx.x] = p.zx * prm_cs;
+                s.row_m0[threadIdx.x] = prm_m0;
+                s.row_shift[threadIdx.x] = prm_sh;
+            }
             cons_sync();
-            if (ok) {
-                for (int idx = threadIdx.x; idx < UNIT_ROWS * p.M; idx += CONS_THREADS) {
+            const bool whole = u_begin >= s_begin && u_end <= s_end;
+            const int ntile = UNIT_ROWS * p.M;
+            if (ok && whole) {
+                // the unit is entirely this CTA's: requantize and store
+                for (int idx = threadIdx.x; idx < ntile; idx += CONS_THREADS) {
                     const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
                     const int n = rb * UNIT_ROWS + row;
                     const int32_t sum = s.red[row][tok];
                     s.red[row][tok] = 0;
-                    if (n >= p.N) continue;
-                    const int32_t cs = __ldg(p.colsum + n);
-                    const int32_t m0 = __ldg(p.M0 + n);
-                    const int32_t sh = __ldg(p.shift + n);
-                    // sum(w x) = sum(u x) - bias * sum(x); acc = sum(w x) - zx colsum
-                    // (two's-complement wrap is exact: the result fits in int32)
-                    const int32_t a = (int32_t)((uint32_t)sum -
-                                                (uint32_t)(C::BIAS * s.xsum[tok]) -
-                                                (uint32_t)(p.zx * cs));
-                    const int64_t v = (int64_t)a * (int64_t)m0;
-                    const int64_t q = (v + ((int64_t)1 << (sh - 1))) >> sh;
-                    int64_t yv = (int64_t)p.zy + q;
-                    yv = yv < -128 ? -128 : (yv > 127 ? 127 : yv);
-                    if (p.residual) {
-                        yv += (int64_t)p.residual[(size_t)tok * (size_t)p.ldy + n];
-                        yv = yv < -128 ? -128 : (yv > 127 ? 127 : yv);
+                    // sum(w x) = sum(u x) - bias * sum(x)
+                    if (n < p.N)
+                        store_out(p, s, row, n, tok,
+                                  (int32_t)((uint32_t)sum -
+                                            (uint32_t)(C::BIAS * s.xsum[par][tok])));
+                }
+            } else if (ok) {
+                // a split unit: add this piece to the slot of its first contributor
+                const int first = cta_of(u_begin, S, G), last_c = cta_of(u_end - 1, S, G);
+                int32_t *slot_sum = P.ws_sum + (size_t)first * UNIT_ROWS * 16;
+                for (int idx = threadIdx.x; idx < ntile; idx += CONS_THREADS) {
+                    const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
+                    const int32_t part = (int32_t)((uint32_t)s.red[row][tok] -
+                                                   (uint32_t)(C::BIAS * s.xsum[par][tok]));
+                    s.red[row][tok] = 0;
+                    atomicAdd(slot_sum + row * 16 + tok, part);
+                }
+                __threadfence();
+                cons_sync();
+                if (threadIdx.x == 0) {
+                    const int done = atomicAdd(P.ws_count + first, 1);
+                    s.last[par] = done == last_c - first;
+                    __threadfence();
+                }
+                cons_sync();
+                if (s.last[par]) {
+                    // ntile <= 1024 = 4 * CONS_THREADS: all loads first, then use
+                    int32_t sums[4];
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const int idx = threadIdx.x + r * CONS_THREADS;
+                        const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
+                        sums[r] = idx < ntile ? __ldcg(slot_sum + row * 16 + tok) : 0;
                     }
-                    p.y[(size_t)tok * (size_t)p.ldy + n] = (int8_t)yv;
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const int idx = threadIdx.x + r * CONS_THREADS;
+                        if (idx >= ntile) continue;
+                        const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
+                        const int n = rb * UNIT_ROWS + row;
+                        slot_sum[row * 16 + tok] = 0;
+                        if (n < p.N) store_out(p, s, row, n, tok, sums[r]);
+                    }
+                    if (threadIdx.x == 0) P.ws_count[first] = 0;
                 }
             }
-            cons_sync();  // every read of red / xsum of this unit is done
-            if (threadIdx.x < 16) s.xsum[threadIdx.x] = 0;
-            cons_sync();
+            cons_sync();  // every read of red / xsum / last / row params is done
+            // reset this parity's buffers; they are used again two pieces on,
+            // after the next piece's barriers
+            if (threadIdx.x < 16) s.xsum[par][threadIdx.x] = 0;
+            if (threadIdx.x == 0) s.last[par] = 0;
+            par ^= 1;
+            gs = piece_end;
         }
     }
     __syncthreads();
@@ -411,7 +523,8 @@ bool encode_sw128(CUtensorMap *map, const void *base, uint64_t cols, uint64_t ro
 }
 
 template <int BITS, int NT>
-int launch_t(const Problem *probs, int count, cudaStream_t stream) {
+int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t stream) {
+    using C = Cfg<BITS>;
     auto kern = decode_kernel<BITS, NT>;
     static int attr_done = -1;
     int dev = 0;
@@ -428,12 +541,14 @@ int launch_t(const Problem *probs, int count, cudaStream_t stream) {
     for (int begin = 0; begin < count; begin += DECODE_MAX_PROBLEMS) {
         const int n = count - begin < DECODE_MAX_PROBLEMS ? count - begin : DECODE_MAX_PROBLEMS;
         Params P{};
-        int units = 0;
+        long long stages = 0;
         for (int i = 0; i < n; ++i) {
             Problem &q = P.p[i];
             q = probs[begin + i];
-            q.tile_begin = units;
-            units += (q.N + UNIT_ROWS - 1) / UNIT_ROWS;
+            const int nst = q.K > 0 ? (q.K + C::KSTAGE - 1) / C::KSTAGE : 1;
+            q.tile_begin = (int)stages;
+            q.tiles_m = nst;
+            stages += (long long)((q.N + UNIT_ROWS - 1) / UNIT_ROWS) * nst;
             const uint64_t wcols = (uint64_t)q.K * BITS / 8;
             if (q.K > 0 &&
                 (!encode_sw128(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, wcols, UNIT_ROWS) ||
@@ -441,12 +556,17 @@ int launch_t(const Problem *probs, int count, cudaStream_t stream) {
                                16)))
                 return MQ_ERR_CUDA;
         }
+        if (stages == 0) continue;
+        if (stages > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
         P.count = n;
-        P.total_units = units;
+        P.total_stages = (int)stages;
+        P.ws_count = workspace;
+        P.ws_sum = workspace + DECODE_WS_COUNTERS;
         P.status = device_status_ptr();
-        if (units == 0) continue;
-        const int grid = units < 2 * sms ? units : 2 * sms;
-        kern<<<grid, THREADS, SMEM_BYTES, stream>>>(P);
+        long long grid = 2LL * sms;
+        if (grid > DECODE_MAX_GRID) grid = DECODE_MAX_GRID;
+        if (grid > stages) grid = stages;
+        kern<<<(int)grid, THREADS, SMEM_BYTES, stream>>>(P);
         if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;
@@ -454,17 +574,19 @@ int launch_t(const Problem *probs, int count, cudaStream_t stream) {
 
 }  // namespace decode
 
-// All problems passed here have the same bits and M <= DECODE_MAX_M.
-int launch_decode(const Problem *probs, int count, void *stream) {
+// All problems passed here have the same bits and M <= DECODE_MAX_M;
+// `workspace` holds DECODE_WS_BYTES, zero-filled.
+int launch_decode(const Problem *probs, int count, void *workspace, void *stream) {
     using namespace decode;
     if (count <= 0) return MQ_OK;
     int max_m = 0;
     for (int i = 0; i < count; ++i) max_m = probs[i].M > max_m ? probs[i].M : max_m;
     const bool nt2 = max_m > 8;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int32_t *ws = static_cast<int32_t *>(workspace);
     if (probs[0].bits == 4)
-        return nt2 ? launch_t<4, 2>(probs, count, s) : launch_t<4, 1>(probs, count, s);
-    return nt2 ? launch_t<8, 2>(probs, count, s) : launch_t<8, 1>(probs, count, s);
+        return nt2 ? launch_t<4, 2>(probs, count, ws, s) : launch_t<4, 1>(probs, count, ws, s);
+    return nt2 ? launch_t<8, 2>(probs, count, ws, s) : launch_t<8, 1>(probs, count, ws, s);
 }
 
 }  // namespace mq

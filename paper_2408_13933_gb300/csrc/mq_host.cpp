@@ -51,8 +51,6 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
 
 int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws_bytes,
               void *stream) {
-    (void)workspace;
-    (void)ws_bytes;  // no kernel of this version uses a workspace
     if (!descs || count < 1 || count > MQ_MAX_BATCH) return MQ_ERR_INVALID_ARG;
     std::vector<mq::Problem> pre, dec8, dec4;
     pre.reserve(count);
@@ -66,10 +64,17 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         else
             pre.push_back(p);
     }
+    // the decode kernel combines split 64-row units in the caller's workspace
+    if (!dec8.empty() || !dec4.empty()) {
+        if (!workspace || ws_bytes < mq::DECODE_WS_BYTES || !aligned16(workspace))
+            return MQ_ERR_WORKSPACE;
+    }
     int rc = MQ_OK;
     if (!pre.empty()) rc = mq::launch_prefill(pre.data(), (int)pre.size(), stream);
-    if (rc == MQ_OK && !dec8.empty()) rc = mq::launch_decode(dec8.data(), (int)dec8.size(), stream);
-    if (rc == MQ_OK && !dec4.empty()) rc = mq::launch_decode(dec4.data(), (int)dec4.size(), stream);
+    if (rc == MQ_OK && !dec8.empty())
+        rc = mq::launch_decode(dec8.data(), (int)dec8.size(), workspace, stream);
+    if (rc == MQ_OK && !dec4.empty())
+        rc = mq::launch_decode(dec4.data(), (int)dec4.size(), workspace, stream);
     return rc;
 }
 
@@ -209,7 +214,7 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed, int32
 
 int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes) {
     if (!bytes || M < 0 || N < 0 || K < 0 || (bits != 8 && bits != 4)) return MQ_ERR_INVALID_ARG;
-    *bytes = 0;
+    *bytes = (M > 0 && M <= mq::DECODE_MAX_M && N > 0) ? mq::DECODE_WS_BYTES : 0;
     return MQ_OK;
 }
 

@@ -31,6 +31,13 @@ struct Problem {
 // Largest M served by the weight-streaming decode kernel.
 constexpr int DECODE_MAX_M = 16;
 
+// Decode workspace: per CTA of the decode grid (at most DECODE_MAX_GRID) one
+// contributor counter and one 64 x 16 int32 slot of partial sums.
+constexpr int DECODE_MAX_GRID = 320;
+constexpr int DECODE_WS_COUNTERS = 384;  // counters, padded to 1536 bytes
+constexpr size_t DECODE_WS_BYTES =
+    sizeof(int32_t) * ((size_t)DECODE_WS_COUNTERS + (size_t)DECODE_MAX_GRID * 64 * 16);
+
 // Problems per kernel launch (kernel parameter space).
 constexpr int PREFILL_MAX_PROBLEMS = 32;
 constexpr int DECODE_MAX_PROBLEMS = 64;
@@ -43,7 +50,7 @@ int *pack_status_ptr();
 
 // Launchers (asynchronous on `stream`); return MQ_OK or MQ_ERR_CUDA.
 int launch_prefill(const Problem *probs, int count, void *stream);
-int launch_decode(const Problem *probs, int count, void *stream);
+int launch_decode(const Problem *probs, int count, void *workspace, void *stream);
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
                 int *status, void *stream);
 

@@ -154,48 +154,38 @@ __device__ __forceinline__ void cvt_i4x32(uint8_t *tile, const uint32_t (&off)[4
     }
 }
 
-// Requantize one accumulator (acc = sum(x w) - zx colsum, int32):
-// clamp(zy + floor((acc * M0 + 2^(s-1)) / 2^s), -128, 127).  With
-// v = acc * M0 = hi * 2^32 + lo (lo unsigned): for s >= 33 the result is
-// (hi + 2^(s-33)) >> (s-32) exactly (the low word cannot carry across a
-// multiple of 2^(s-32)); for s == 32 it is hi + (lo >> 31); smaller shifts
-// take the 64-bit path.  `s` is uniform across the warp (one column).
-__device__ __forceinline__ int32_t requant(int32_t acc, int32_t m0, int32_t sh, int32_t zy) {
-    int32_t q;
-    if (sh >= 33) {
-        q = (__mulhi(acc, m0) + (1 << (sh - 33))) >> (sh - 32);
-    } else if (sh == 32) {
-        q = __mulhi(acc, m0) + (int32_t)((uint32_t)(acc * m0) >> 31);
-    } else {
-        const int64_t v = ((int64_t)acc * (int64_t)m0 + ((int64_t)1 << (sh - 1))) >> sh;
-        q = (int32_t)(v < -1024 ? -1024 : (v > 1024 ? 1024 : v));
-    }
-    return min(127, max(-128, q + zy));
-}
+// What the epilogue needs of the current tile's problem, in registers (the
+// problem table itself lives in the kernel parameters, where dynamically
+// indexed reads are slow).
+struct EpiArgs {
+    int8_t *y;
+    const int8_t *residual;
+    int M, N, ldy, zy;
+};
 
 // Requantize and store 16 consecutive outputs (tile columns c0 .. c0+15 of
 // `row`; global column = n0 + tile column).
-__device__ __forceinline__ void requant_store16(const Problem &p, const Smem &s, int row, int n0,
+__device__ __forceinline__ void requant_store16(const EpiArgs &e, const Smem &s, int row, int n0,
                                                 int c0, const uint32_t (&acc)[16]) {
-    if (row >= p.M) return;
-    const int8_t *res = p.residual ? p.residual + (size_t)row * (size_t)p.ldy + n0 + c0 : nullptr;
+    if (row >= e.M) return;
+    const int8_t *res = e.residual ? e.residual + (size_t)row * (size_t)e.ldy + n0 + c0 : nullptr;
     uint32_t packed[4];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
         const int c = c0 + i;
-        int32_t out = requant((int32_t)(acc[i] - (uint32_t)s.col_corr[c]), s.col_m0[c],
-                              s.col_shift[c], p.zy);
-        if (res && n0 + c < p.N) out = min(127, max(-128, out + (int32_t)res[i]));
+        int32_t out = mq_requant((int32_t)(acc[i] - (uint32_t)s.col_corr[c]), s.col_m0[c],
+                                 s.col_shift[c], e.zy);
+        if (res && n0 + c < e.N) out = min(127, max(-128, out + (int32_t)res[i]));
         if ((i & 3) == 0) packed[i >> 2] = 0;
         packed[i >> 2] |= ((uint32_t)(out & 0xFF)) << ((i & 3) * 8);
     }
-    int8_t *dst = p.y + (size_t)row * (size_t)p.ldy + n0 + c0;
-    if (n0 + c0 + 16 <= p.N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0)) {
+    int8_t *dst = e.y + (size_t)row * (size_t)e.ldy + n0 + c0;
+    if (n0 + c0 + 16 <= e.N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0)) {
         *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
     } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-            if (n0 + c0 + i < p.N) dst[i] = (int8_t)((packed[i >> 2] >> ((i & 3) * 8)) & 0xFF);
+            if (n0 + c0 + i < e.N) dst[i] = (int8_t)((packed[i >> 2] >> ((i & 3) * 8)) & 0xFF);
     }
 }
 
@@ -388,11 +378,12 @@ __global__ void __launch_bounds__(THREADS, 1) prefill_kernel(const __grid_consta
         for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x) {
             const Tile t = tile_at(P, tile);
             const Problem &p = P.p[t.pi];
+            const EpiArgs e{p.y, p.residual, p.M, p.N, p.ldy, p.zy};
             const int n0 = t.nt * BN;
             epi_sync();  // the previous tile's requant pass is done with the parameters
             {
                 const int n = n0 + et;
-                const bool in = n < p.N;
+                const bool in = n < e.N;
                 s.col_corr[et] = in ? p.zx * __ldg(p.colsum + n) : 0;
                 s.col_m0[et] = in ? __ldg(p.M0 + n) : 0;
                 s.col_shift[et] = in ? __ldg(p.shift + n) : 33;
@@ -446,7 +437,7 @@ __global__ void __launch_bounds__(THREADS, 1) prefill_kernel(const __grid_consta
 #pragma unroll
                     for (int i = 0; i < 16; ++i) acc[i] = 0u;
                 }
-                requant_store16(p, s, row, n0, c0, acc);
+                requant_store16(e, s, row, n0, c0, acc);
             }
         }
     }

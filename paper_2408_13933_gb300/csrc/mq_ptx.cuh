@@ -290,4 +290,23 @@ __device__ __forceinline__ void i4x8_to_f16x8(uint32_t w, uint32_t (&o)[4]) {
     }
 }
 
+// Requantize one accumulator (acc = sum(x w) - zx colsum, int32):
+// clamp(zy + floor((acc * M0 + 2^(s-1)) / 2^s), -128, 127).  With
+// v = acc * M0 = hi * 2^32 + lo (lo unsigned): for s >= 33 the result is
+// (hi + 2^(s-33)) >> (s-32) exactly (the low word cannot carry across a
+// multiple of 2^(s-32)); for s == 32 it is hi + (lo >> 31); smaller shifts
+// take the 64-bit path.  `s` is uniform across the warp (one column).
+__device__ __forceinline__ int32_t mq_requant(int32_t acc, int32_t m0, int32_t sh, int32_t zy) {
+    int32_t q;
+    if (sh >= 33) {
+        q = (__mulhi(acc, m0) + (1 << (sh - 33))) >> (sh - 32);
+    } else if (sh == 32) {
+        q = __mulhi(acc, m0) + (int32_t)((uint32_t)(acc * m0) >> 31);
+    } else {
+        const int64_t v = ((int64_t)acc * (int64_t)m0 + ((int64_t)1 << (sh - 1))) >> sh;
+        q = (int32_t)(v < -1024 ? -1024 : (v > 1024 ? 1024 : v));
+    }
+    return min(127, max(-128, q + zy));
+}
+
 }  // namespace mq

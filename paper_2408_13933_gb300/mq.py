@@ -121,6 +121,14 @@ def workspace_size(m: int, n: int, k: int, bits: int) -> int:
     return out.value
 
 
+def workspace(device=None):
+    """A zero-filled device workspace large enough for any mq_linear_* or
+    mq_linear_batch call (see mq_workspace_size); torch allocates it."""
+    import torch
+    n = workspace_size(1, 1, 0, 4)
+    return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
+
+
 def pack_weights(w, bits: int, stream=None):
     """mq_pack_weights.  `w` int8 [N, K]: a numpy array (host path) or a CUDA
     torch tensor (device path).  Returns (packed, colsum) on the same side."""
@@ -144,8 +152,10 @@ def pack_weights(w, bits: int, stream=None):
 
 def linear(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y, bits: int,
            ldx: int | None = None, ldy: int | None = None, m: int | None = None,
-           k: int | None = None, stream=None, workspace=None, ws_bytes: int = 0) -> int:
+           k: int | None = None, stream=None, workspace=None, ws_bytes: int | None = None) -> int:
     """mq_linear_w8a8 / mq_linear_w4a8 on CUDA tensors; returns the status code."""
+    if ws_bytes is None:
+        ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     m = x.shape[0] if m is None else m
     k = x.shape[1] if k is None else k
     ldx = x.stride(0) if ldx is None else ldx
@@ -169,8 +179,10 @@ def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
     return d
 
 
-def linear_batch(descs, stream=None, workspace=None, ws_bytes: int = 0) -> int:
+def linear_batch(descs, stream=None, workspace=None, ws_bytes: int | None = None) -> int:
     """mq_linear_batch over a list of LinearDesc; returns the status code."""
+    if ws_bytes is None:
+        ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     arr = (LinearDesc * len(descs))(*descs)
     return lib.mq_linear_batch(arr, len(descs), _ptr(workspace), ws_bytes, _stream(stream))
 

@@ -14,6 +14,19 @@ def torch_cuda():
     return torch
 
 
+_WS = None
+
+
+def workspace():
+    """One zero-filled decode workspace shared by the tests (every call leaves
+    it zero-filled again)."""
+    global _WS
+    if _WS is None:
+        from paper_2408_13933_gb300 import mq
+        _WS = mq.workspace()
+    return _WS
+
+
 def upload(a: np.ndarray):
     torch = torch_cuda()
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
@@ -47,7 +60,7 @@ class GpuLinear:
     def run(self) -> np.ndarray:
         c = self.case
         rc = self.mq.linear(self.x, c.zx, self.packed, self.colsum, c.N, self.m0, self.shift, c.zy,
-                            self.y, c.bits, ldy=self.ldy)
+                            self.y, c.bits, ldy=self.ldy, workspace=workspace())
         assert rc == 0, self.mq.status_string(rc)
         return self.result()
 

@@ -18,7 +18,7 @@ import pytest
 
 import oracle
 from gpu_helpers import (GpuLinear, assert_equal_int8, oracle_points, oracle_y, sample_points,
-                         torch_cuda, upload)
+                         torch_cuda, upload, workspace)
 from paper_2408_13933_gb300 import synth
 
 pytestmark = pytest.mark.gpu
@@ -30,7 +30,7 @@ def mq():
 
 
 def run_batch(gls):
-    assert mq().linear_batch([g.desc() for g in gls]) == 0
+    assert mq().linear_batch([g.desc() for g in gls], workspace=workspace()) == 0
     return [g.result() for g in gls]
 
 
@@ -97,10 +97,10 @@ def test_config3_chained_stack():
             return lib.make_desc(xin, c.zx, p[0], p[1], c.N, p[2], p[3], c.zy, out[c.name], 8,
                                  residual=residual)
         first = [desc(c, x) for c in L.cases if c.name in ("q", "k", "v", "gate", "up")]
-        assert lib.linear_batch(first) == 0
+        assert lib.linear_batch(first, workspace=workspace()) == 0
         cs = {c.name: c for c in L.cases}
         second = [desc(cs["o"], out["q"]), desc(cs["down"], out["up"], residual=res)]
-        assert lib.linear_batch(second) == 0
+        assert lib.linear_batch(second, workspace=workspace()) == 0
         torch.cuda.synchronize()
         assert lib.check_device_status() == 0
         gpu_rows.append({k: v[rows].cpu().numpy() for k, v in out.items()})

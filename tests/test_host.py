@@ -100,7 +100,9 @@ def test_host_pack_rejects_int4_out_of_range(mq):
 def test_packed_and_workspace_sizes(mq):
     assert mq.packed_size(3, 64, 8) == 192
     assert mq.packed_size(3, 64, 4) == 96
-    assert mq.workspace_size(1024, 2048, 2048, 8) == 0
+    assert mq.workspace_size(1024, 2048, 2048, 8) == 0      # tensor-core path: none
+    assert mq.workspace_size(16, 2048, 2048, 4) > 0         # decode path: fixed size
+    assert mq.workspace_size(1, 7, 64, 8) == mq.workspace_size(16, 256000, 16384, 4)
     with pytest.raises(mq.MQError):
         mq.packed_size(3, 63, 4)
     with pytest.raises(mq.MQError):
@@ -135,6 +137,18 @@ def test_linear_bad_bits_and_batch_args(mq):
     assert mq.lib.mq_linear_batch(None, 1, None, 0, None) == 1
     assert mq.lib.mq_linear_batch((mq.LinearDesc * 1)(), 0, None, 0, None) == 1
     assert mq.lib.mq_linear_batch((mq.LinearDesc * 1)(), mq.MQ_MAX_BATCH + 1, None, 0, None) == 1
+
+
+def test_decode_requires_workspace(mq):
+    # M <= 16 runs the decode kernel, which needs the caller's workspace; the
+    # check happens before anything is launched
+    fn = mq.lib.mq_linear_w4a8
+    assert fn(FAKE, 8, 64, 64, 0, FAKE, FAKE, 32, FAKE, FAKE, 0, FAKE, 32, None, 0, None) == 7
+    need = mq.workspace_size(8, 32, 64, 4)
+    assert fn(FAKE, 8, 64, 64, 0, FAKE, FAKE, 32, FAKE, FAKE, 0, FAKE, 32, FAKE, need - 1,
+              None) == 7
+    assert fn(FAKE, 8, 64, 64, 0, FAKE, FAKE, 32, FAKE, FAKE, 0, FAKE, 32, FAKE + 4, need,
+              None) == 7   # misaligned
 
 
 def test_empty_problems_launch_nothing(mq):

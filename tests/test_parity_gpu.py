@@ -9,7 +9,7 @@ equality of every int8 output.
 import numpy as np
 import pytest
 
-from gpu_helpers import GpuLinear, assert_equal_int8, oracle_y, torch_cuda, upload
+from gpu_helpers import GpuLinear, assert_equal_int8, oracle_y, torch_cuda, upload, workspace
 from paper_2408_13933_gb300 import synth
 
 pytestmark = pytest.mark.gpu
@@ -118,7 +118,7 @@ def test_residual_epilogue(m, bits):
                                     127).astype(np.int8)
     g = GpuLinear(case)
     from paper_2408_13933_gb300 import mq
-    assert mq.linear_batch([g.desc()]) == 0
+    assert mq.linear_batch([g.desc()], workspace=workspace()) == 0
     assert_equal_int8(g.result(), oracle_y(case), f"residual m={m} bits={bits}")
 
 
@@ -128,7 +128,7 @@ def test_batch_mixes_kernels_and_widths():
          (8, 2048, 256, 4), (333, 64, 17, 8)])]
     gs = [GpuLinear(c) for c in cases]
     from paper_2408_13933_gb300 import mq
-    assert mq.linear_batch([g.desc() for g in gs]) == 0
+    assert mq.linear_batch([g.desc() for g in gs], workspace=workspace()) == 0
     for g, c in zip(gs, cases):
         assert_equal_int8(g.result(), oracle_y(c), f"batch {c.M}x{c.K}x{c.N} bits={c.bits}")
 
@@ -158,3 +158,23 @@ def test_repeated_calls_are_deterministic():
     a = g.run().copy()
     for _ in range(3):
         assert np.array_equal(g.run(), a)
+
+
+@pytest.mark.parametrize("bits,extreme", [(4, None), (4, "mixed"), (8, "mixed"), (8, "min")])
+def test_decode_unit_split_across_many_ctas(bits, extreme):
+    # one 64-row unit of K = 65536: its 256 (int4) or 512 (int8) stages are
+    # spread over up to 320 CTAs, which combine their partial sums in the
+    # workspace; "min" drives the int32 accumulator to its largest magnitude
+    case = synth.random_case(500 + bits, 5, 65536, 64, bits, extreme)
+    case.sw = np.full(case.N, 2e-9, np.float32)
+    assert_equal_int8(GpuLinear(case).run(), oracle_y(case), f"split K=65536 bits={bits}")
+
+
+def test_decode_workspace_left_zero():
+    torch = torch_cuda()
+    for seed, (m, k, n, bits) in enumerate([(1, 5632, 2048, 4), (16, 16384, 300, 8),
+                                            (7, 2080, 70, 4)]):
+        c = synth.random_case(600 + seed, m, k, n, bits)
+        assert_equal_int8(GpuLinear(c).run(), oracle_y(c), f"ws m={m} k={k}")
+    torch.cuda.synchronize()
+    assert int(torch.count_nonzero(workspace())) == 0
