@@ -150,6 +150,36 @@ int mq_linear_w4a8(const int8_t *x, int M, int K, int ldx, int32_t zx,
                    void *stream);
 
 /*
+ * mq_linear_w4a8 for decode shapes (1 <= M <= 16) without a workspace
+ * argument and without allocating device memory.  The paper has no
+ * counterpart: this is a deployment variant of the same layer.
+ *
+ * For callers that cannot provide device memory around a decode step: a C
+ * program with no device allocator of its own, or a serving loop whose memory
+ * pool is fixed after warm-up and must not grow mid-generation.  The split-K
+ * combine scratch (about 1.3 MB) is a static device array inside libmq, one
+ * per device; each call clears it on `stream` with a memset before the
+ * kernel, and no call allocates or frees device memory.
+ *
+ * The first call on each device does set-up with that device current: it
+ * looks up the scratch's address and prepares the decode kernel.  Make that
+ * first call before any stream capture.  Every call on a device shares the
+ * one scratch, so calls must not overlap: two calls on different streams or
+ * from different host threads race and give wrong results.  Calls issued in
+ * order on one stream are fine.
+ *
+ * Arguments and requirements as mq_linear_w4a8.  The result is identical to
+ * mq_linear_w4a8 on the same inputs.
+ * Errors: MQ_ERR_UNSUPPORTED_SHAPE for M > 16, which the scratch does not
+ * hold (use mq_linear_w4a8); otherwise as mq_linear_w4a8, but
+ * MQ_ERR_WORKSPACE does not occur.
+ */
+int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                           const void *packed, const int32_t *colsum, int N,
+                           const int32_t *M0, const int32_t *shift, int32_t zy,
+                           int8_t *y, int ldy, void *stream);
+
+/*
  * Several independent linears in as few launches as possible (one per kernel
  * family): a decoder block's projections that read the same activations, or
  * a whole step's worth of small decode GEMVs.  Each descriptor has the

@@ -37,7 +37,7 @@ MQ_MAX_BATCH = 256
 
 EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_weights",
             "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
-            "mq_check_device_status"]
+            "mq_check_device_status", "mq_linear_w4a8_noalloc"]
 
 _vp, _i32, _int, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int, ctypes.c_size_t
 
@@ -59,6 +59,8 @@ _linear_args = [_vp, _int, _int, _int, _i32, _vp, _vp, _int, _vp, _vp, _i32, _vp
                 _sz, _vp]
 lib.mq_linear_w8a8.argtypes = _linear_args
 lib.mq_linear_w4a8.argtypes = _linear_args
+lib.mq_linear_w4a8_noalloc.argtypes = [_vp, _int, _int, _int, _i32, _vp, _vp, _int, _vp, _vp, _i32,
+                                       _vp, _int, _vp]
 lib.mq_linear_batch.argtypes = [ctypes.POINTER(LinearDesc), _int, _vp, _sz, _vp]
 lib.mq_check_device_status.argtypes = [_vp]
 for _f in EXPORTED:
@@ -163,6 +165,20 @@ def linear(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y, bits: int,
     fn = lib.mq_linear_w8a8 if bits == 8 else lib.mq_linear_w4a8
     return fn(_ptr(x), m, k, ldx, int(zx), _ptr(packed), _ptr(colsum), n, _ptr(m0), _ptr(shift),
               int(zy), _ptr(y), ldy, _ptr(workspace), ws_bytes, _stream(stream))
+
+
+def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y,
+                        ldx: int | None = None, ldy: int | None = None, m: int | None = None,
+                        k: int | None = None, stream=None) -> int:
+    """mq_linear_w4a8_noalloc on CUDA tensors (decode shapes, no workspace);
+    returns the status code."""
+    m = x.shape[0] if m is None else m
+    k = x.shape[1] if k is None else k
+    ldx = x.stride(0) if ldx is None else ldx
+    ldy = y.stride(0) if ldy is None else ldy
+    return lib.mq_linear_w4a8_noalloc(_ptr(x), m, k, ldx, int(zx), _ptr(packed), _ptr(colsum), n,
+                                      _ptr(m0), _ptr(shift), int(zy), _ptr(y), ldy,
+                                      _stream(stream))
 
 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
