@@ -49,6 +49,23 @@ CONFIG_ID_DECODE = 2
 WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
 
 
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one prefill_kernel launch on this
+# workload, from one ncu capture (profiles/prefill_kernel_tinyllama_block_w8a8_m1024.md), valid
+# only for the kernel sources it was taken on: reported as null once they change.
+PREFILL_TRAFFIC_BYTES = 56_395_264 + 1_584_384
+PREFILL_TRAFFIC_SOURCES = ("mq_prefill.cu", "mq_ptx.cuh", "mq_internal.h")
+PREFILL_TRAFFIC_SHA = "fadb121a133daa7f"
+
+
+def prefill_traffic():
+    import hashlib
+    h = hashlib.sha256()
+    for f in PREFILL_TRAFFIC_SOURCES:
+        with open(os.path.join(ROOT, "paper_2408_13933_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return PREFILL_TRAFFIC_BYTES if h.hexdigest()[:16] == PREFILL_TRAFFIC_SHA else None
+
+
 def block_ops(m: int) -> int:
     return sum(2 * m * k * n for _, k, n in synth.TINYLLAMA_LINEARS)
 
@@ -467,7 +484,8 @@ def main():
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "tensor", "achieved": round(kern_tflops, 1),
                      "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                     "frac": round(kern_tflops / peaks["bf16_tflops"], 3), "traffic": None,
+                     "frac": round(kern_tflops / peaks["bf16_tflops"], 3),
+                     "traffic": prefill_traffic(), "traffic_unit": "bytes per launch",
                      "kernel": "mq::prefill::prefill_kernel",
                      "peak_note": f"dense f16 tensor peak = bf16 burst ({peaks['source']}), "
                                   "int8 ops run as exact f16 MMAs"},
