@@ -8,29 +8,49 @@
 // products are then exact and an f32 accumulator stays exact while every
 // partial sum is an integer of magnitude <= 2^24.  The K loop is therefore cut
 // into chunks of 1024 (int8 weights: |x w| <= 2^14) or 16384 (int4: |x w| <=
-// 2^10); after each chunk the epilogue warps convert the f32 chunk sum to
-// int32 and add it to an int32 running sum kept in tensor memory.
+// 2^10); after each chunk the epilogue converts the f32 chunk sum to int32
+// and adds it to an int32 running sum.
 //
-// CTA = one SM, persistent over 128 x 256 output tiles of up to
-// PREFILL_MAX_PROBLEMS independent linears (longest K first).  Data path:
-//   HBM/L2 --TMA--> int8/int4 staging ring (3 stages, zero-filled outside the
-//   tensors) --converter warps--> f16 operand ring (3 stages, 128-byte
-//   swizzled, K-major) --tcgen05.mma--> f32 chunk accumulator F in TMEM.
-// Warp roles:
-//   warp 0     : TMA producer (one thread).
-//   warp 1     : owns the TMEM allocation; one thread issues tcgen05.mma
-//                (M=128, N=256, K=16, f16 x f16 -> f32) and the commits.
-//   warps 2-9  : converters, int8/int4 staging -> exact f16 operand tiles;
-//                every thread converts the same chunks of every stage, so
-//                its shared-memory offsets are computed once.
-//   warps 10-17: epilogue.  Per chunk: F -> int32, T += F (TMEM columns
-//                256-511).  Per tile: acc = T - zx*colsum[n], fixed-point
-//                requant (round half up) with per-column parameters staged in
-//                shared memory, saturate, optional residual, store.
-// All mbarrier waits are bounded (mq_wait_parity).
+// The kernel runs on CTA pairs (clusters of two, one CTA per SM) with pair
+// MMAs (tcgen05 cta_group::2, M = 256, N = 128, K = 16).  Operand A is the
+// weights: 256 output channels per pair tile, 128 in each CTA, widened by the
+// converter warps straight into tensor memory (tcgen05.st), so they never pass
+// through shared memory as f16.  Operand B is the activations: 128 tokens per
+// pair tile, 64 rows in each CTA's shared memory, 128-byte swizzled K-major.
+// Shared-memory bandwidth is what the tensor cores' operand reads and the
+// widening pass compete for; this split keeps the f16 traffic through shared
+// memory to the 64 token rows per CTA.
+//
+// Data path, per CTA and stage of 128 k:
+//   HBM/L2 --TMA--> int8 / int4 staging ring (S8 stages, zero fill outside
+//   the tensors) --converters--> A: TMEM ring (SF stages), B: f16 ring in
+//   shared memory (SF stages) --pair MMA, issued by the even CTA--> f32 chunk
+//   accumulator F[b] in TMEM (two buffers, so the MMAs of chunk c+1 overlap
+//   the drain of chunk c).
+// TMEM columns: F[0] 0-127, F[1] 128-255, A stages 256 + 64 s.
+// Warp roles (both CTAs):
+//   warp 0     : TMA producer (one thread) for this CTA's weight and token rows.
+//   warp 1     : TMEM allocation; in the even CTA one thread issues the MMAs
+//                and the commits (multicast to both CTAs' barriers).
+//   warps 2-9  : converters.  Warp w writes TMEM lanes 32 (w % 4) .. +31 (its
+//                weight rows), k half (w - 2) / 4 of each stage, and widens
+//                two 16-byte chunks of the token tile into shared memory.
+//   warps 10-17: epilogue.  Thread = one output channel (TMEM lane), 64 of
+//                the tile's 128 tokens; the int32 sum of each chunk is kept
+//                in registers; per tile: acc - zx*colsum[n], fixed-point
+//                requant, saturate, optional residual, byte stores (one warp
+//                writes 32 consecutive channels of a token row).
+// Work: pair tiles (256 channels x 128 tokens) of up to PREFILL_MAX_PROBLEMS
+// independent linears, assigned to pairs by the host (longest processing time
+// first) or round-robin when there are too many tiles for the table.
+// All mbarrier waits are bounded (mq_wait_parity / mq_wait_parity_cluster).
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <queue>
+#include <vector>
 
 #include "mq_internal.h"
 #include "mq_ptx.cuh"
@@ -38,55 +58,59 @@
 namespace mq {
 namespace prefill {
 
-constexpr int BM = 128;
-constexpr int BN = 256;
-constexpr int BK = 64;   // k per stage: one 128-byte f16 row segment
-constexpr int S8 = 3;    // int8 staging stages
-constexpr int SF = 3;    // f16 operand stages
+constexpr int TM = 256;  // output channels per pair tile (MMA M, operand A)
+constexpr int TN = 128;  // tokens per pair tile (MMA N, operand B)
+constexpr int CM = 128;  // weight rows per CTA
+constexpr int CN = 64;   // token rows per CTA
+constexpr int KS = 128;  // k per stage
+constexpr int S8 = 6;    // staging stages
+constexpr int SF = 4;    // operand stages (A in TMEM, B in shared memory)
 constexpr int TMA_WARP = 0;
 constexpr int MMA_WARP = 1;
 constexpr int CONV_WARP0 = 2;
 constexpr int CONV_WARPS = 8;
-constexpr int CONV_THREADS = CONV_WARPS * 32;
 constexpr int EPI_WARP0 = 10;
 constexpr int EPI_WARPS = 8;
 constexpr int NUM_WARPS = 18;
 constexpr int THREADS = NUM_WARPS * 32;
-constexpr int EPI_BARRIER = 1;  // named barrier among the epilogue warps
-constexpr int OPA = BM * 128;   // f16 A tile bytes
-constexpr int OPB = BN * 128;   // f16 B tile bytes
-constexpr int STA = BM * BK;    // int8 A staging bytes
-constexpr int STB = BN * BK;    // int8 B staging bytes (int4 uses half)
+constexpr int STA = CM * KS;       // weight staging bytes (int4 uses half)
+constexpr int STB = CN * KS;       // token staging bytes
+constexpr int ATOM = CN * 128;     // one 64-k column of the f16 token tile
+constexpr int OPB = 2 * ATOM;      // f16 token tile of one stage
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t F_COL = 0;
-constexpr uint32_t T_COL = 256;
-constexpr int KB_PER_CHUNK_I8 = 1024 / BK;   // |partial| <= 1024 * 2^14 = 2^24
-constexpr int KB_PER_CHUNK_I4 = 16384 / BK;  // |partial| <= 16384 * 2^10 = 2^24
+constexpr uint32_t F_COL0 = 0;     // F[b] at F_COL0 + 128 b
+constexpr uint32_t A_COL0 = 256;   // A stage s at A_COL0 + 64 s
+constexpr int KB_PER_CHUNK_I8 = 1024 / KS;   // |partial| <= 1024 * 2^14 = 2^24
+constexpr int KB_PER_CHUNK_I4 = 16384 / KS;  // |partial| <= 16384 * 2^10 = 2^24
+constexpr int MAX_SCHED = 4096;    // tile table entries (host LPT schedule)
+constexpr int MAX_PAIRS = 128;
 
 struct Params {
-    CUtensorMap tmap_x[PREFILL_MAX_PROBLEMS];  // int8 [M][ldx], box 64 x 128
-    CUtensorMap tmap_w[PREFILL_MAX_PROBLEMS];  // int8 [N][K] box 64 x 256, or int4 bytes 32 x 256
-    Problem p[PREFILL_MAX_PROBLEMS];
+    CUtensorMap tmap_w[PREFILL_MAX_PROBLEMS];  // int8 [N][K] box 128 B x 128, or int4 bytes box 64 B x 128
+    CUtensorMap tmap_x[PREFILL_MAX_PROBLEMS];  // int8 [M][ldx] box 128 x 64
+    Problem p[PREFILL_MAX_PROBLEMS];           // tile_begin: first tile; tiles_m: token tiles
     int count;
     int total_tiles;
+    int npairs;
+    int use_table;                       // 1: sched / pair_begin, 0: round-robin
+    uint16_t pair_begin[MAX_PAIRS + 1];
+    uint16_t sched[MAX_SCHED];
     int *status;
 };
 
 struct Smem {
-    uint8_t opa[SF][OPA];
-    uint8_t opb[SF][OPB];
     uint8_t sta[S8][STA];
     uint8_t stb[S8][STB];
+    uint8_t opb[SF][OPB];
     uint64_t ld_full[S8];
     uint64_t ld_empty[S8];
-    uint64_t op_full[SF];
-    uint64_t op_empty[SF];
-    uint64_t f_full;
-    uint64_t f_empty;
+    uint64_t op_full[SF];   // even CTA: its converter warps + the MMA thread arrive, the odd
+                            // CTA's converter warps signal 4 transaction bytes each
+    uint64_t op_empty[SF];  // both CTAs: multicast commit
+    uint64_t f_full[2];     // both CTAs: multicast commit
+    uint64_t f_empty[2];    // even CTA: both CTAs' epilogue warps arrive
     uint64_t done;
-    int32_t col_corr[BN];  // zx * colsum[n] of the epilogue's current tile
-    int32_t col_m0[BN];
-    int32_t col_shift[BN];
+    uint32_t sink[CONV_WARPS];  // even CTA: targets of the odd CTA's st.async signals
     uint32_t tmem_base;
     int abort;
 };
@@ -95,7 +119,8 @@ constexpr size_t SMEM_BYTES = sizeof(Smem) + 1024;  // + alignment slack
 
 struct Tile {
     int pi;
-    int mt, nt, nkb, kpc;
+    int ct, tt;    // channel tile, token tile
+    int nkb, kpc;  // stages, stages per exact f32 chunk
 };
 
 __device__ __forceinline__ Tile tile_at(const Params &P, int tile) {
@@ -104,101 +129,57 @@ __device__ __forceinline__ Tile tile_at(const Params &P, int tile) {
     while (t.pi + 1 < P.count && tile >= P.p[t.pi + 1].tile_begin) ++t.pi;
     const Problem &p = P.p[t.pi];
     const int local = tile - p.tile_begin;
-    t.mt = local % p.tiles_m;
-    t.nt = local / p.tiles_m;
-    t.nkb = (p.K + BK - 1) / BK;
+    t.tt = local % p.tiles_m;
+    t.ct = local / p.tiles_m;
+    t.nkb = (p.K + KS - 1) / KS;
     t.kpc = p.bits == 8 ? KB_PER_CHUNK_I8 : KB_PER_CHUNK_I4;
     return t;
 }
 
-// Warp-uniform bounded wait: lane 0 polls, the verdict is broadcast.
+// The i-th tile of pair `pair`, or -1 past its last one.
+__device__ __forceinline__ int pair_tile(const Params &P, int pair, int i) {
+    if (P.use_table) {
+        const int j = P.pair_begin[pair] + i;
+        return j < P.pair_begin[pair + 1] ? (int)P.sched[j] : -1;
+    }
+    const int t = pair + i * P.npairs;
+    return t < P.total_tiles ? t : -1;
+}
+
+// Warp-uniform bounded waits: lane 0 polls, the verdict is broadcast.
 __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, Smem &s, int *status) {
     bool ok = true;
     if ((threadIdx.x & 31) == 0) ok = mq_wait_parity(bar, parity, &s.abort, status);
     return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
 }
 
-// Byte offset of 16-byte chunk `c` (0..7) of row `r` in a 128B-swizzled tile.
-__device__ __forceinline__ uint32_t swz(int r, int c) {
-    return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4));
-}
-
-__device__ __forceinline__ void sts16(uint8_t *base, uint32_t off, uint32_t a, uint32_t b,
-                                      uint32_t c, uint32_t d) {
-    *reinterpret_cast<uint4 *>(base + off) = make_uint4(a, b, c, d);
-}
 
 __device__ __forceinline__ uint4 lds16(const uint8_t *p) {
     return *reinterpret_cast<const uint4 *>(p);
 }
 
-// 16 int8 -> two f16 chunks at precomputed swizzled offsets.
-__device__ __forceinline__ void cvt_i8x16(uint8_t *tile, const uint32_t (&off)[2], const uint4 &v) {
-    uint32_t h[8];
-    i8x4_to_f16x4(v.x, h[0], h[1]);
-    i8x4_to_f16x4(v.y, h[2], h[3]);
-    i8x4_to_f16x4(v.z, h[4], h[5]);
-    i8x4_to_f16x4(v.w, h[6], h[7]);
-    sts16(tile, off[0], h[0], h[1], h[2], h[3]);
-    sts16(tile, off[1], h[4], h[5], h[6], h[7]);
+__device__ __forceinline__ void sts16(uint8_t *p, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+    *reinterpret_cast<uint4 *>(p) = make_uint4(a, b, c, d);
 }
 
-// 32 int4 -> four f16 chunks at precomputed swizzled offsets.
-__device__ __forceinline__ void cvt_i4x32(uint8_t *tile, const uint32_t (&off)[4], const uint4 &v) {
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        uint32_t o[4];
-        i4x8_to_f16x8(w[j], o);
-        sts16(tile, off[j], o[0], o[1], o[2], o[3]);
-    }
-}
-
-// What the epilogue needs of the current tile's problem, in registers (the
-// problem table itself lives in the kernel parameters, where dynamically
-// indexed reads are slow).
+// What the epilogue needs of a tile's problem, copied into registers (the
+// problem table lives in the kernel parameters, where dynamically indexed
+// reads are slow).
 struct EpiArgs {
     int8_t *y;
     const int8_t *residual;
-    int M, N, ldy, zy;
+    int M, ldy, zy;
 };
 
-// Requantize and store 16 consecutive outputs (tile columns c0 .. c0+15 of
-// `row`; global column = n0 + tile column).
-__device__ __forceinline__ void requant_store16(const EpiArgs &e, const Smem &s, int row, int n0,
-                                                int c0, const uint32_t (&acc)[16]) {
-    if (row >= e.M) return;
-    const int8_t *res = e.residual ? e.residual + (size_t)row * (size_t)e.ldy + n0 + c0 : nullptr;
-    uint32_t packed[4];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const int c = c0 + i;
-        int32_t out = mq_requant((int32_t)(acc[i] - (uint32_t)s.col_corr[c]), s.col_m0[c],
-                                 s.col_shift[c], e.zy);
-        if (res && n0 + c < e.N) out = min(127, max(-128, out + (int32_t)res[i]));
-        if ((i & 3) == 0) packed[i >> 2] = 0;
-        packed[i >> 2] |= ((uint32_t)(out & 0xFF)) << ((i & 3) * 8);
-    }
-    int8_t *dst = e.y + (size_t)row * (size_t)e.ldy + n0 + c0;
-    if (n0 + c0 + 16 <= e.N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0)) {
-        *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
-    } else {
-#pragma unroll
-        for (int i = 0; i < 16; ++i)
-            if (n0 + c0 + i < e.N) dst[i] = (int8_t)((packed[i >> 2] >> ((i & 3) * 8)) & 0xFF);
-    }
-}
-
-__device__ __forceinline__ void epi_sync() {
-    asm volatile("bar.sync %0, %1;" ::"n"(EPI_BARRIER), "n"(EPI_WARPS * 32) : "memory");
-}
-
-__global__ void __launch_bounds__(THREADS, 1) prefill_kernel(const __grid_constant__ Params P) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+    prefill_kernel(const __grid_constant__ Params P) {
     extern __shared__ uint8_t smem_raw[];
     Smem &s = *reinterpret_cast<Smem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();  // 0: even CTA (issues the MMAs), 1: odd
+    const int pair = (int)(blockIdx.x >> 1);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < S8; ++i) {
@@ -206,21 +187,23 @@ __global__ void __launch_bounds__(THREADS, 1) prefill_kernel(const __grid_consta
             mbar_init(&s.ld_empty[i], CONV_WARPS);
         }
         for (int i = 0; i < SF; ++i) {
-            mbar_init(&s.op_full[i], CONV_WARPS);
+            mbar_init(&s.op_full[i], CONV_WARPS + 1);
             mbar_init(&s.op_empty[i], 1);
         }
-        mbar_init(&s.f_full, 1);
-        mbar_init(&s.f_empty, EPI_WARPS);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&s.f_full[b], 1);
+            mbar_init(&s.f_empty[b], 2 * EPI_WARPS);
+        }
         mbar_init(&s.done, 1);
         s.abort = 0;
         fence_mbar_init();
     }
     if (warp == MMA_WARP) {
-        tmem_alloc(&s.tmem_base, TMEM_COLS);
-        tmem_relinquish();
+        tmem_alloc2(&s.tmem_base, TMEM_COLS);
+        tmem_relinquish2();
     }
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();  // barriers of both CTAs initialised before any remote arrive
     tc_fence_after();
     const uint32_t tmem = s.tmem_base;
 
@@ -234,10 +217,13 @@ __global__ void __launch_bounds__(THREADS, 1) prefill_kernel(const __grid_consta
             }
             uint32_t it = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < P.total_tiles; tile += gridDim.x) {
+            int tile;
+            for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
                 const Tile t = tile_at(P, tile);
                 const bool i4 = P.p[t.pi].bits == 4;
-                const uint32_t bytes = STA + (i4 ? STB / 2 : STB);
+                const uint32_t bytes = (i4 ? STA / 2 : STA) + STB;
+                const int wrow = t.ct * TM + (int)rank * CM;
+                const int xrow = t.tt * TN + (int)rank * CN;
                 for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                     const int slot = it % S8;
                     if (!mq_wait_parity(&s.ld_empty[slot], ((it / S8) & 1) ^ 1, &s.abort,
@@ -246,83 +232,100 @@ __global__ void __launch_bounds__(THREADS, 1) prefill_kernel(const __grid_consta
                         break;
                     }
                     mbar_arrive_expect_tx(&s.ld_full[slot], bytes);
-                    tma_load_2d(s.sta[slot], &P.tmap_x[t.pi], kb * BK, t.mt * BM, &s.ld_full[slot]);
-                    tma_load_2d(s.stb[slot], &P.tmap_w[t.pi], i4 ? kb * (BK / 2) : kb * BK,
-                                t.nt * BN, &s.ld_full[slot]);
+                    tma_load_2d(s.sta[slot], &P.tmap_w[t.pi], i4 ? kb * (KS / 2) : kb * KS, wrow,
+                                &s.ld_full[slot]);
+                    tma_load_2d(s.stb[slot], &P.tmap_x[t.pi], kb * KS, xrow, &s.ld_full[slot]);
                 }
             }
         }
         __syncwarp();
     } else if (warp == MMA_WARP) {
         // ------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            const uint32_t idesc = idesc_f16_f32(BM, BN);
+        if (rank == 0 && lane == 0) {
+            const uint32_t idesc = idesc_f16_f32(TM, TN);
             uint32_t it = 0, chunks = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < P.total_tiles; tile += gridDim.x) {
+            int tile;
+            for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
                 const Tile t = tile_at(P, tile);
+                uint32_t fcol = 0;
                 for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                     const bool chunk_start = (kb % t.kpc) == 0;
                     if (chunk_start) {
-                        if (!mq_wait_parity(&s.f_empty, (chunks & 1) ^ 1, &s.abort, P.status)) {
+                        const uint32_t b = chunks & 1;
+                        if (!mq_wait_parity_cluster(&s.f_empty[b], ((chunks >> 1) & 1) ^ 1,
+                                                    &s.abort, P.status)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
+                        fcol = F_COL0 + 128 * b;
                     }
                     const int slot = it % SF;
-                    if (!mq_wait_parity(&s.op_full[slot], (it / SF) & 1, &s.abort, P.status)) {
+                    mbar_arrive_expect_tx(&s.op_full[slot], 4 * CONV_WARPS);
+                    if (!mq_wait_parity_cluster(&s.op_full[slot], (it / SF) & 1, &s.abort,
+                                                P.status)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint64_t ad = smem_desc_sw128(smem_u32(s.opa[slot]));
-                    const uint64_t bd = smem_desc_sw128(smem_u32(s.opb[slot]));
+                    const uint32_t acol = tmem + A_COL0 + 64 * slot;
+                    const uint64_t bd0 = smem_desc_sw128(smem_u32(s.opb[slot]));
+                    const uint64_t bd1 = smem_desc_sw128(smem_u32(s.opb[slot] + ATOM));
 #pragma unroll
-                    for (int j = 0; j < BK / 16; ++j)  // +32 B along K: +2 in the (addr >> 4) field
-                        tc_mma_f16(tmem + F_COL, ad + 2 * j, bd + 2 * j, idesc,
-                                   (chunk_start && j == 0) ? 0u : 1u);
-                    tc_commit(&s.op_empty[slot]);
+                    for (int j = 0; j < KS / 16; ++j)  // +32 B along K: +2 in the (addr >> 4) field
+                        tc_mma2_f16_ts(tmem + fcol, acol + 8 * j,
+                                       (j < 4 ? bd0 : bd1) + 2 * (j & 3), idesc,
+                                       (chunk_start && j == 0) ? 0u : 1u);
+                    tc_commit2_mc(&s.op_empty[slot], 3);
                     if (((kb + 1) % t.kpc) == 0 || kb + 1 == t.nkb) {
-                        tc_commit(&s.f_full);
+                        tc_commit2_mc(&s.f_full[chunks & 1], 3);
                         ++chunks;
                     }
                 }
             }
             // every MMA issued above has completed once `done` fires
-            tc_commit(&s.done);
-            mq_wait_parity(&s.done, 0, &s.abort, P.status);
+            tc_commit2_mc(&s.done, 1);
+            mq_wait_parity_cluster(&s.done, 0, &s.abort, P.status);
         }
         __syncwarp();
     } else if (warp < EPI_WARP0) {
         // ------------------------------------------------------ converters
-        // Thread ct converts, in every stage: A chunks ct and ct + 256 (128
-        // rows x 4 chunks of 16 int8); B int8 chunks ct + 256 i, i < 4 (256
-        // rows x 4), or B int4 chunks ct and ct + 256 (256 rows x 2 chunks of
-        // 32 nibbles).  Chunk g of A / int8 B is row g >> 2, chunk g & 3;
-        // of int4 B row g >> 1, half g & 1.
         const int ct = threadIdx.x - CONV_WARP0 * 32;  // 0..255
-        uint32_t a_src[2], a_dst[2][2], b_src[4], b_dst[4][2], q_dst[2][4];
+        const int quad = warp & 3;                     // TMEM lane quarter of this warp
+        const int half = (warp - CONV_WARP0) >> 2;     // k half of the stage
+        const int arow = quad * 32 + lane;             // weight row in this CTA
+        const uint32_t a_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(32 * half);
+        // staging offsets of this thread's weight chunks (128B / 64B swizzle)
+        uint32_t a8_src[4], a4_src[2];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            a8_src[i] = (uint32_t)(arow * 128 + (((4 * half + i) ^ (arow & 7)) << 4));
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+            a4_src[i] = (uint32_t)(arow * 64 + (((2 * half + i) ^ ((arow >> 1) & 3)) << 4));
+        // token chunks g = ct + 256 i: row g >> 3, 16-k chunk g & 7; f16
+        // destination: 64-k column g >> 2 & 1, 16-byte chunks 2 (g & 3), +1
+        uint32_t b_src[2], b_dst[2][2];
 #pragma unroll
         for (int i = 0; i < 2; ++i) {
-            const int g = ct + 256 * i, row = g >> 2, kc = g & 3;
-            a_src[i] = g * 16;
-            a_dst[i][0] = swz(row, 2 * kc);
-            a_dst[i][1] = swz(row, 2 * kc + 1);
-            const int qrow = g >> 1, half = g & 1;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) q_dst[i][j] = swz(qrow, 4 * half + j);
+            const int g = ct + 256 * i, row = g >> 3, kc = g & 7;
+            b_src[i] = (uint32_t)(row * 128 + ((kc ^ (row & 7)) << 4));
+            const uint32_t base = (uint32_t)((kc >> 2) * ATOM + row * 128);
+            const int c0 = 2 * (kc & 3), c1 = c0 + 1;
+            // lanes with kc >= 4 store their second chunk first: the eight lanes
+            // of a row then hit eight different bank groups on each store
+            const int first = (kc & 4) ? c1 : c0, second = (kc & 4) ? c0 : c1;
+            b_dst[i][0] = base + (uint32_t)((first ^ (row & 7)) << 4);
+            b_dst[i][1] = base + (uint32_t)((second ^ (row & 7)) << 4);
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int g = ct + 256 * i, row = g >> 2, kc = g & 3;
-            b_src[i] = g * 16;
-            b_dst[i][0] = swz(row, 2 * kc);
-            b_dst[i][1] = swz(row, 2 * kc + 1);
-        }
+        const bool swap_b = (ct & 4) != 0;
+        const uint32_t leader_op_full = cluster_addr(&s.op_full[0], 0);
+        const uint32_t leader_sink = cluster_addr(&s.sink[warp - CONV_WARP0], 0);
         uint32_t it = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < P.total_tiles; tile += gridDim.x) {
+        int tile;
+        for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
             const Tile t = tile_at(P, tile);
             const bool i4 = P.p[t.pi].bits == 4;
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
@@ -332,121 +335,138 @@ __global__ void __launch_bounds__(THREADS, 1) prefill_kernel(const __grid_consta
                     ok = false;
                     break;
                 }
+                tc_fence_after();
                 const uint8_t *sa = s.sta[s8];
                 const uint8_t *sb = s.stb[s8];
-                uint8_t *oa = s.opa[sf];
+                uint32_t a[32];
+                if (!i4) {
+                    uint4 v[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) v[i] = lds16(sa + a8_src[i]);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        i8x4_to_f16x4(v[i].x, a[8 * i + 0], a[8 * i + 1]);
+                        i8x4_to_f16x4(v[i].y, a[8 * i + 2], a[8 * i + 3]);
+                        i8x4_to_f16x4(v[i].z, a[8 * i + 4], a[8 * i + 5]);
+                        i8x4_to_f16x4(v[i].w, a[8 * i + 6], a[8 * i + 7]);
+                    }
+                } else {
+                    uint4 v[2];
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) v[i] = lds16(sa + a4_src[i]);
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) {
+                        const uint32_t w4[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            uint32_t o[4];
+                            i4x8_to_f16x8(w4[j], o);
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) a[16 * i + 4 * j + e] = o[e];
+                        }
+                    }
+                }
+                uint4 vb[2];
+#pragma unroll
+                for (int i = 0; i < 2; ++i) vb[i] = lds16(sb + b_src[i]);
+                uint32_t h[2][8];
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    i8x4_to_f16x4(vb[i].x, h[i][0], h[i][1]);
+                    i8x4_to_f16x4(vb[i].y, h[i][2], h[i][3]);
+                    i8x4_to_f16x4(vb[i].z, h[i][4], h[i][5]);
+                    i8x4_to_f16x4(vb[i].w, h[i][6], h[i][7]);
+                }
+                tc_st_32x32b_x32(a_lane + A_COL0 + 64 * sf, a);
                 uint8_t *ob = s.opb[sf];
-                uint4 va[2], vb[4];
 #pragma unroll
-                for (int i = 0; i < 2; ++i) va[i] = lds16(sa + a_src[i]);
-                if (!i4) {
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) vb[i] = lds16(sb + b_src[i]);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 2; ++i) vb[i] = lds16(sb + a_src[i]);
+                for (int i = 0; i < 2; ++i) {
+                    if (!swap_b) {
+                        sts16(ob + b_dst[i][0], h[i][0], h[i][1], h[i][2], h[i][3]);
+                        sts16(ob + b_dst[i][1], h[i][4], h[i][5], h[i][6], h[i][7]);
+                    } else {
+                        sts16(ob + b_dst[i][0], h[i][4], h[i][5], h[i][6], h[i][7]);
+                        sts16(ob + b_dst[i][1], h[i][0], h[i][1], h[i][2], h[i][3]);
+                    }
                 }
-#pragma unroll
-                for (int i = 0; i < 2; ++i) cvt_i8x16(oa, a_dst[i], va[i]);
-                if (!i4) {
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) cvt_i8x16(ob, b_dst[i], vb[i]);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 2; ++i) cvt_i4x32(ob, q_dst[i], vb[i]);
-                }
+                // every value read from the staging slot now feeds an issued store
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s.ld_empty[s8]);
+                tc_wait_st();
                 fence_proxy_async_smem();
+                tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
-                    mbar_arrive(&s.op_full[sf]);
-                    mbar_arrive(&s.ld_empty[s8]);
+                    if (rank == 0)
+                        mbar_arrive(&s.op_full[sf]);
+                    else
+                        st_async_signal(leader_sink, it, leader_op_full + 8u * (uint32_t)sf);
                 }
             }
         }
     } else {
         // ------------------------------------------------------ epilogue
-        const int et = threadIdx.x - EPI_WARP0 * 32;  // 0..255
-        const int ew = warp - EPI_WARP0;              // 0..7
-        const int quad = warp & 3;          // TMEM lane quadrant this warp may access
-        const int col0 = (ew >> 2) * 128;   // column half of the tile
-        const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16);
+        const int quad = warp & 3;                  // TMEM lane quarter of this warp
+        const int half = (warp - EPI_WARP0) >> 2;   // token half of the tile
+        const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(64 * half);
+        const uint32_t leader_f_empty = cluster_addr(&s.f_empty[0], 0);
         uint32_t chunks = 0;
-        // After a failed wait (ok == false) the warp keeps walking the tile
-        // loop without touching TMEM, so that every epilogue warp reaches the
-        // same named barriers.
         bool ok = true;
-        for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x) {
+        int tile;
+        for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
             const Tile t = tile_at(P, tile);
             const Problem &p = P.p[t.pi];
-            const EpiArgs e{p.y, p.residual, p.M, p.N, p.ldy, p.zy};
-            const int n0 = t.nt * BN;
-            epi_sync();  // the previous tile's requant pass is done with the parameters
-            {
-                const int n = n0 + et;
-                const bool in = n < e.N;
-                s.col_corr[et] = in ? p.zx * __ldg(p.colsum + n) : 0;
-                s.col_m0[et] = in ? __ldg(p.M0 + n) : 0;
-                s.col_shift[et] = in ? __ldg(p.shift + n) : 33;
-            }
+            const int ch = t.ct * TM + (int)rank * CM + quad * 32 + lane;
+            const bool ch_in = ch < p.N;
+            const int32_t corr = ch_in ? p.zx * __ldg(p.colsum + ch) : 0;
+            const int32_t m0 = ch_in ? __ldg(p.M0 + ch) : 0;
+            const int32_t sh = ch_in ? __ldg(p.shift + ch) : 33;
+            uint32_t acc[64];
+#pragma unroll
+            for (int i = 0; i < 64; ++i) acc[i] = 0u;
             const int nchunks = t.nkb ? (t.nkb + t.kpc - 1) / t.kpc : 0;
-            for (int c = 0; ok && c < nchunks; ++c) {
-                if (!warp_wait(&s.f_full, chunks & 1, s, P.status)) {
+            for (int c = 0; c < nchunks; ++c, ++chunks) {
+                const uint32_t b = chunks & 1;
+                if (!warp_wait(&s.f_full[b], (chunks >> 1) & 1, s, P.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                // drain F into T, one 16-column slice at a time; the TMEM
-                // loads of slice sl+1 overlap the arithmetic of slice sl
-                uint32_t f[2][16], acc[2][16];
-                tc_ld_32x32b_x16(t_lane + F_COL + col0, f[0]);
-                if (c > 0) tc_ld_32x32b_x16(t_lane + T_COL + col0, acc[0]);
-                tc_wait_ld();
 #pragma unroll
-                for (int sl = 0; sl < 8; ++sl) {
-                    const int b = sl & 1;
-                    if (sl + 1 < 8) {
-                        const uint32_t nc = (uint32_t)(col0 + (sl + 1) * 16);
-                        tc_ld_32x32b_x16(t_lane + F_COL + nc, f[b ^ 1]);
-                        if (c > 0) tc_ld_32x32b_x16(t_lane + T_COL + nc, acc[b ^ 1]);
-                    }
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t f[16];
+                    tc_ld_32x32b_x16(t_lane + F_COL0 + 128 * b + 16 * q, f);
+                    tc_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int32_t part = __float2int_rn(__uint_as_float(f[b][i]));
-                        acc[b][i] = (c > 0 ? acc[b][i] : 0u) + (uint32_t)part;
-                    }
-                    tc_st_32x32b_x16(t_lane + T_COL + (uint32_t)(col0 + sl * 16), acc[b]);
-                    if (sl + 1 < 8) tc_wait_ld();
+                    for (int i = 0; i < 16; ++i)
+                        acc[16 * q + i] += (uint32_t)__float2int_rn(__uint_as_float(f[i]));
                 }
-                tc_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&s.f_empty);
-                ++chunks;
+                if (lane == 0) mbar_arrive_cluster(leader_f_empty + 8u * b);
             }
-            epi_sync();  // column parameters visible to every epilogue warp
-            if (!ok) continue;
-            const int row = t.mt * BM + quad * 32 + lane;
-#pragma unroll 1
-            for (int sl = 0; sl < 8; ++sl) {
-                const int c0 = col0 + sl * 16;
-                uint32_t acc[16];
-                if (nchunks > 0) {
-                    tc_ld_32x32b_x16(t_lane + T_COL + (uint32_t)c0, acc);
-                    tc_wait_ld();
-                } else {
+            if (!ok) break;
+            if (!ch_in) continue;
+            const EpiArgs e{p.y, p.residual, p.M, p.ldy, p.zy};
+            const int tok0 = t.tt * TN + 64 * half;
+            int8_t *yp = e.y + (size_t)tok0 * (size_t)e.ldy + ch;
+            const int8_t *rp = e.residual ? e.residual + (size_t)tok0 * (size_t)e.ldy + ch : nullptr;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) acc[i] = 0u;
+            for (int i = 0; i < 64; ++i) {
+                if (tok0 + i < e.M) {
+                    int32_t out = mq_requant((int32_t)(acc[i] - (uint32_t)corr), m0, sh, e.zy);
+                    if (rp) out = min(127, max(-128, out + (int32_t)rp[(size_t)i * e.ldy]));
+                    yp[(size_t)i * e.ldy] = (int8_t)out;
                 }
-                requant_store16(e, s, row, n0, c0, acc);
             }
         }
     }
 
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();  // the pair's MMAs are done with both CTAs' TMEM and shared memory
     if (warp == MMA_WARP) {
         tc_fence_after();
-        tmem_dealloc(tmem, TMEM_COLS);
+        tmem_dealloc2(tmem, TMEM_COLS);
     }
 }
 
@@ -465,7 +485,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// 2-D uint8 tensor [rows][cols] with row pitch `pitch` bytes, box box_cols x box_rows.
+// 2-D uint8 tensor [rows][cols] with row pitch `pitch` bytes, box box_cols x
+// box_rows, 128- or 64-byte swizzle (box_cols bytes per row).
 bool encode_2d(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows, uint64_t pitch,
                uint32_t box_cols, uint32_t box_rows) {
     auto fn = encode_fn();
@@ -474,10 +495,65 @@ bool encode_2d(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows,
     const cuuint64_t strides[1] = {pitch};
     const cuuint32_t box[2] = {box_cols, box_rows};
     const cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle swz =
+        box_cols == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
     return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box,
-              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
-           CUDA_SUCCESS;
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Pairs the device can run at once (one CTA per SM, clusters of two).
+int max_pairs(int dev) {
+    static int cached[64] = {0};
+    if (dev >= 0 && dev < 64 && cached[dev]) return cached[dev];
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    int n = sms / 2;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(2 * n, 1, 1);
+    cfg.blockDim = dim3(THREADS, 1, 1);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, prefill_kernel, &cfg) == cudaSuccess &&
+        clusters > 0 && clusters < n)
+        n = clusters;
+    if (n > MAX_PAIRS) n = MAX_PAIRS;
+    if (dev >= 0 && dev < 64) cached[dev] = n;
+    return n;
+}
+
+// Longest-processing-time-first assignment of tiles to pairs.  Tile ids are
+// numbered problem by problem; work = stages + a fixed epilogue share.
+void lpt_schedule(Params &P, int npairs) {
+    std::vector<std::pair<int, int>> work;  // (work, tile)
+    work.reserve(P.total_tiles);
+    for (int pi = 0; pi < P.count; ++pi) {
+        const Problem &q = P.p[pi];
+        const int tiles = q.tiles_m * ((q.N + TM - 1) / TM);
+        const int w = (q.K + KS - 1) / KS + 2;
+        for (int i = 0; i < tiles; ++i) work.emplace_back(w, q.tile_begin + i);
+    }
+    std::stable_sort(work.begin(), work.end(),
+                     [](const std::pair<int, int> &a, const std::pair<int, int> &b) {
+                         return a.first > b.first;
+                     });
+    using Load = std::pair<long long, int>;  // (load, pair)
+    std::priority_queue<Load, std::vector<Load>, std::greater<Load>> heap;
+    for (int i = 0; i < npairs; ++i) heap.emplace(0LL, i);
+    std::vector<std::vector<int>> lists(npairs);
+    for (const auto &wt : work) {
+        Load l = heap.top();
+        heap.pop();
+        lists[l.second].push_back(wt.second);
+        l.first += wt.first;
+        heap.push(l);
+    }
+    int at = 0;
+    for (int i = 0; i < npairs; ++i) {
+        P.pair_begin[i] = (uint16_t)at;
+        for (int tile : lists[i]) P.sched[at++] = (uint16_t)tile;
+    }
+    P.pair_begin[npairs] = (uint16_t)at;
 }
 
 }  // namespace prefill
@@ -493,14 +569,13 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
             return MQ_ERR_CUDA;
         attr_done = dev;
     }
-    int sms = 0;
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        return MQ_ERR_CUDA;
+    const int pairs_max = max_pairs(dev);
+    if (pairs_max < 1) return MQ_ERR_CUDA;
     for (int begin = 0; begin < count; begin += PREFILL_MAX_PROBLEMS) {
         const int n = count - begin < PREFILL_MAX_PROBLEMS ? count - begin : PREFILL_MAX_PROBLEMS;
         Params P{};
-        int tiles = 0;
-        // longest K first: the longest tiles start in the first wave
+        long long tiles = 0;
+        // longest K first (round-robin order; the table orders by work itself)
         int order[PREFILL_MAX_PROBLEMS];
         for (int i = 0; i < n; ++i) order[i] = begin + i;
         for (int i = 1; i < n; ++i)
@@ -512,24 +587,28 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
         for (int i = 0; i < n; ++i) {
             Problem &q = P.p[i];
             q = probs[order[i]];
-            q.tiles_m = (q.M + BM - 1) / BM;
-            q.tile_begin = tiles;
-            tiles += q.tiles_m * ((q.N + BN - 1) / BN);
+            q.tiles_m = (q.M + TN - 1) / TN;
+            q.tile_begin = (int)tiles;
+            tiles += (long long)q.tiles_m * ((q.N + TM - 1) / TM);
             if (q.K > 0) {
-                const uint64_t wcols = q.bits == 8 ? (uint64_t)q.K : (uint64_t)q.K / 2;
+                const bool i4 = q.bits == 4;
+                const uint64_t wcols = i4 ? (uint64_t)q.K / 2 : (uint64_t)q.K;
                 if (!encode_2d(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M, (uint64_t)q.ldx,
-                               BK, BM) ||
-                    !encode_2d(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, wcols,
-                               q.bits == 8 ? BK : BK / 2, BN))
+                               KS, CN) ||
+                    !encode_2d(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, wcols, i4 ? KS / 2 : KS,
+                               CM))
                     return MQ_ERR_CUDA;
             }
         }
-        P.count = n;
-        P.total_tiles = tiles;
-        P.status = device_status_ptr();
         if (tiles == 0) continue;
-        const int grid = tiles < sms ? tiles : sms;
-        prefill_kernel<<<grid, THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(P);
+        if (tiles > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
+        P.count = n;
+        P.total_tiles = (int)tiles;
+        P.status = device_status_ptr();
+        P.npairs = tiles < pairs_max ? (int)tiles : pairs_max;
+        P.use_table = tiles <= MAX_SCHED ? 1 : 0;
+        if (P.use_table) lpt_schedule(P, P.npairs);
+        prefill_kernel<<<2 * P.npairs, THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(P);
         if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;

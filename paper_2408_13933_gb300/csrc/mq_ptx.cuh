@@ -114,18 +114,88 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// ----------------------------------------------------------------- tcgen05
-__device__ __forceinline__ void tmem_alloc(uint32_t *dst_smem, uint32_t ncols) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+// ----------------------------------------------------------------- clusters
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// All threads of every CTA of the cluster (release / acquire at cluster scope).
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Shared-memory address of the same variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t cluster_addr(const void *p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+    return r;
+}
+
+// Arrive (release, cluster scope) on an mbarrier given by its cluster address.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];"
+                 ::"r"(cluster_bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// mq_wait_parity for phases completed by arrivals from other CTAs of the
+// cluster (remote arrives, multicast commits): acquire at cluster scope.
+__device__ __forceinline__ bool mq_wait_parity_cluster(uint64_t *bar, uint32_t parity,
+                                                       volatile int *abort, int *status) {
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t n = 0;; ++n) {
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if ((n & 15) == 15) {
+            if (*abort) return false;
+            if (global_timer_ns() - t0 > MQ_WAIT_LIMIT_NS) {
+                *abort = 1;
+                atomicOr(status, MQ_DEVICE_STATUS_TIMEOUT);
+                return false;
+            }
+        }
+    }
+}
+
+// Non-blocking 4-byte store into another CTA's shared memory that signals the
+// mbarrier next to it (complete_tx of 4 bytes, release at cluster scope): a
+// cheap cross-CTA "data ready" signal.  Both addresses are cluster addresses
+// in the same CTA.
+__device__ __forceinline__ void st_async_signal(uint32_t cluster_dst, uint32_t value,
+                                                uint32_t cluster_bar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];"
+                 ::"r"(cluster_dst), "r"(value), "r"(cluster_bar) : "memory");
+}
+
+// ------------------------------------------------- tcgen05, CTA-pair mode
+// Every tcgen05 instruction of a kernel uses the same CTA group; libmq's
+// tensor-core kernel runs on CTA pairs (cta_group::2).  Allocation and
+// deallocation are collective over one warp of each CTA of the pair; the
+// pair's MMAs are issued by one thread of the even CTA.
+__device__ __forceinline__ void tmem_alloc2(uint32_t *dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;"
                  ::"r"(smem_u32(dst_smem)), "r"(ncols) : "memory");
 }
 
-__device__ __forceinline__ void tmem_relinquish() {
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+__device__ __forceinline__ void tmem_relinquish2() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;"
+__device__ __forceinline__ void tmem_dealloc2(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;"
                  ::"r"(taddr), "r"(ncols) : "memory");
 }
 
@@ -137,23 +207,27 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (f16 operands, f32 accumulate).
-__device__ __forceinline__ void tc_mma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                           uint32_t idesc, uint32_t accumulate) {
+// Pair MMA, kind::f16: D[tmem] (+)= A[tmem] * B[smem]^T.  A (M = 256) is split
+// by rows over the pair (128 TMEM lanes in each CTA at the same address), B
+// by rows (N / 2 in each CTA's shared memory at the same address), D by rows
+// like A.
+__device__ __forceinline__ void tc_mma2_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                               uint32_t idesc, uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
-        ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 
-// Arrive once on `bar` when every tcgen05 operation issued so far by this
-// thread has completed.
-__device__ __forceinline__ void tc_commit(uint64_t *bar) {
+// Arrive once on the mbarrier at `bar`'s offset in every CTA of `cta_mask`
+// when every tcgen05 operation issued so far by this thread has completed.
+__device__ __forceinline__ void tc_commit2_mc(uint64_t *bar, uint16_t cta_mask) {
     asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
-        ::"r"(smem_u32(bar)) : "memory");
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;"
+        ::"r"(smem_u32(bar)), "h"(cta_mask) : "memory");
 }
 
 __device__ __forceinline__ void tc_wait_ld() {
