@@ -451,12 +451,31 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const int tok0 = t.tt * TN + 64 * half;
             int8_t *yp = e.y + (size_t)tok0 * (size_t)e.ldy + ch;
             const int8_t *rp = e.residual ? e.residual + (size_t)tok0 * (size_t)e.ldy + ch : nullptr;
+            const int ntok = min(64, e.M - tok0);
+            // quarters of 16 tokens: the residual bytes of a quarter are all
+            // loaded before its first store (the compiler cannot know that y
+            // and the residual do not alias), so each costs one round trip
 #pragma unroll
-            for (int i = 0; i < 64; ++i) {
-                if (tok0 + i < e.M) {
-                    int32_t out = mq_requant((int32_t)(acc[i] - (uint32_t)corr), m0, sh, e.zy);
-                    if (rp) out = min(127, max(-128, out + (int32_t)rp[(size_t)i * e.ldy]));
-                    yp[(size_t)i * e.ldy] = (int8_t)out;
+            for (int q4 = 0; q4 < 4; ++q4) {
+                uint32_t res[4] = {0u, 0u, 0u, 0u};  // 4 bytes each
+                if (rp) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i)
+                        if (16 * q4 + i < ntok)
+                            res[i >> 2] |= (uint32_t)(uint8_t)rp[(size_t)(16 * q4 + i) * e.ldy]
+                                           << (8 * (i & 3));
+                }
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int j = 16 * q4 + i;
+                    if (j < ntok) {
+                        int32_t out = mq_requant((int32_t)(acc[j] - (uint32_t)corr), m0, sh, e.zy);
+                        if (rp) {
+                            const int32_t r = (int32_t)(int8_t)(res[i >> 2] >> (8 * (i & 3)));
+                            out = min(127, max(-128, out + r));
+                        }
+                        yp[(size_t)j * e.ldy] = (int8_t)out;
+                    }
                 }
             }
         }
