@@ -32,9 +32,10 @@
 //   warp 0     : TMA producer (one thread) for this CTA's weight and token rows.
 //   warp 1     : TMEM allocation; in the even CTA one thread issues the MMAs
 //                and the commits (multicast to both CTAs' barriers).
-//   warps 2-9  : converters.  Warp w writes TMEM lanes 32 (w % 4) .. +31 (its
-//                weight rows), k half (w - 2) / 4 of each stage, and widens
-//                two 16-byte chunks of the token tile into shared memory.
+//   warps 2-9  : converters, two groups of four taking alternate stages.  In
+//                its stage warp w writes TMEM lanes 32 (w % 4) .. +31 (its
+//                weight rows, all 128 k) and widens four 16-byte chunks of
+//                the token tile into shared memory.
 //   warps 10-17: epilogue.  Thread = one output channel (TMEM lane), 64 of
 //                the tile's 128 tokens; the int32 sum of each chunk is kept
 //                in registers; per tile: acc - zx*colsum[n], fixed-point
@@ -184,10 +185,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < S8; ++i) {
             mbar_init(&s.ld_full[i], 1);
-            mbar_init(&s.ld_empty[i], CONV_WARPS);
+            mbar_init(&s.ld_empty[i], CONV_WARPS / 2);
         }
         for (int i = 0; i < SF; ++i) {
-            mbar_init(&s.op_full[i], CONV_WARPS + 1);
+            mbar_init(&s.op_full[i], CONV_WARPS / 2 + 1);
             mbar_init(&s.op_empty[i], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -262,7 +263,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         fcol = F_COL0 + 128 * b;
                     }
                     const int slot = it % SF;
-                    mbar_arrive_expect_tx(&s.op_full[slot], 4 * CONV_WARPS);
+                    mbar_arrive_expect_tx(&s.op_full[slot], 4 * (CONV_WARPS / 2));
                     if (!mq_wait_parity_cluster(&s.op_full[slot], (it / SF) & 1, &s.abort,
                                                 P.status)) {
                         ok = false;
@@ -291,25 +292,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         __syncwarp();
     } else if (warp < EPI_WARP0) {
         // ------------------------------------------------------ converters
-        const int ct = threadIdx.x - CONV_WARP0 * 32;  // 0..255
-        const int quad = warp & 3;                     // TMEM lane quarter of this warp
-        const int half = (warp - CONV_WARP0) >> 2;     // k half of the stage
-        const int arow = quad * 32 + lane;             // weight row in this CTA
-        const uint32_t a_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(32 * half);
+        // Two groups of four warps take alternate stages, so that the waits
+        // and signals of one group overlap the widening work of the other.
+        // In its stage, warp w widens all 128 k of weight rows 32 (w % 4) ..
+        // +31 (TMEM lanes it may write) and four 16-byte token chunks.
+        const int grp = (warp - CONV_WARP0) >> 2;          // 0 or 1
+        const int gt = threadIdx.x - (CONV_WARP0 + 4 * grp) * 32;  // 0..127 in the group
+        const int quad = warp & 3;                          // TMEM lane quarter of this warp
+        const int arow = quad * 32 + lane;                  // weight row in this CTA
+        const uint32_t a_lane = tmem + ((uint32_t)(quad * 32) << 16);
         // staging offsets of this thread's weight chunks (128B / 64B swizzle)
-        uint32_t a8_src[4], a4_src[2];
+        uint32_t a8_src[8], a4_src[4];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a8_src[i] = (uint32_t)(arow * 128 + ((i ^ (arow & 7)) << 4));
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-            a8_src[i] = (uint32_t)(arow * 128 + (((4 * half + i) ^ (arow & 7)) << 4));
-#pragma unroll
-        for (int i = 0; i < 2; ++i)
-            a4_src[i] = (uint32_t)(arow * 64 + (((2 * half + i) ^ ((arow >> 1) & 3)) << 4));
-        // token chunks g = ct + 256 i: row g >> 3, 16-k chunk g & 7; f16
+            a4_src[i] = (uint32_t)(arow * 64 + ((i ^ ((arow >> 1) & 3)) << 4));
+        // token chunks g = gt + 128 i: row g >> 3, 16-k chunk g & 7; f16
         // destination: 64-k column g >> 2 & 1, 16-byte chunks 2 (g & 3), +1
-        uint32_t b_src[2], b_dst[2][2];
+        uint32_t b_src[4], b_dst[4][2];
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
-            const int g = ct + 256 * i, row = g >> 3, kc = g & 7;
+        for (int i = 0; i < 4; ++i) {
+            const int g = gt + 128 * i, row = g >> 3, kc = g & 7;
             b_src[i] = (uint32_t)(row * 128 + ((kc ^ (row & 7)) << 4));
             const uint32_t base = (uint32_t)((kc >> 2) * ATOM + row * 128);
             const int c0 = 2 * (kc & 3), c1 = c0 + 1;
@@ -319,7 +323,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             b_dst[i][0] = base + (uint32_t)((first ^ (row & 7)) << 4);
             b_dst[i][1] = base + (uint32_t)((second ^ (row & 7)) << 4);
         }
-        const bool swap_b = (ct & 4) != 0;
+        const bool swap_b = (gt & 4) != 0;
         const uint32_t leader_op_full = cluster_addr(&s.op_full[0], 0);
         const uint32_t leader_sink = cluster_addr(&s.sink[warp - CONV_WARP0], 0);
         uint32_t it = 0;
@@ -329,6 +333,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const Tile t = tile_at(P, tile);
             const bool i4 = P.p[t.pi].bits == 4;
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+                if ((int)(it & 1) != grp) continue;
                 const int s8 = it % S8, sf = it % SF;
                 if (!warp_wait(&s.ld_full[s8], (it / S8) & 1, s, P.status) ||
                     !warp_wait(&s.op_empty[sf], ((it / SF) & 1) ^ 1, s, P.status)) {
@@ -338,55 +343,54 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 tc_fence_after();
                 const uint8_t *sa = s.sta[s8];
                 const uint8_t *sb = s.stb[s8];
-                uint32_t a[32];
-                if (!i4) {
-                    uint4 v[4];
+                const uint32_t acol = a_lane + A_COL0 + 64 * sf;
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) v[i] = lds16(sa + a8_src[i]);
+                for (int hk = 0; hk < 2; ++hk) {  // 64 k of the row per TMEM store
+                    uint32_t a[32];
+                    if (!i4) {
+                        uint4 v[4];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        i8x4_to_f16x4(v[i].x, a[8 * i + 0], a[8 * i + 1]);
-                        i8x4_to_f16x4(v[i].y, a[8 * i + 2], a[8 * i + 3]);
-                        i8x4_to_f16x4(v[i].z, a[8 * i + 4], a[8 * i + 5]);
-                        i8x4_to_f16x4(v[i].w, a[8 * i + 6], a[8 * i + 7]);
-                    }
-                } else {
-                    uint4 v[2];
+                        for (int i = 0; i < 4; ++i) v[i] = lds16(sa + a8_src[4 * hk + i]);
 #pragma unroll
-                    for (int i = 0; i < 2; ++i) v[i] = lds16(sa + a4_src[i]);
+                        for (int i = 0; i < 4; ++i) {
+                            i8x4_to_f16x4(v[i].x, a[8 * i + 0], a[8 * i + 1]);
+                            i8x4_to_f16x4(v[i].y, a[8 * i + 2], a[8 * i + 3]);
+                            i8x4_to_f16x4(v[i].z, a[8 * i + 4], a[8 * i + 5]);
+                            i8x4_to_f16x4(v[i].w, a[8 * i + 6], a[8 * i + 7]);
+                        }
+                    } else {
+                        uint4 v[2];
 #pragma unroll
-                    for (int i = 0; i < 2; ++i) {
-                        const uint32_t w4[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+                        for (int i = 0; i < 2; ++i) v[i] = lds16(sa + a4_src[2 * hk + i]);
 #pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            uint32_t o[4];
-                            i4x8_to_f16x8(w4[j], o);
+                        for (int i = 0; i < 2; ++i) {
+                            const uint32_t w4[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
 #pragma unroll
-                            for (int e = 0; e < 4; ++e) a[16 * i + 4 * j + e] = o[e];
+                            for (int j = 0; j < 4; ++j) {
+                                uint32_t o[4];
+                                i4x8_to_f16x8(w4[j], o);
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) a[16 * i + 4 * j + e] = o[e];
+                            }
                         }
                     }
+                    tc_st_32x32b_x32(acol + 32 * hk, a);
                 }
-                uint4 vb[2];
-#pragma unroll
-                for (int i = 0; i < 2; ++i) vb[i] = lds16(sb + b_src[i]);
-                uint32_t h[2][8];
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    i8x4_to_f16x4(vb[i].x, h[i][0], h[i][1]);
-                    i8x4_to_f16x4(vb[i].y, h[i][2], h[i][3]);
-                    i8x4_to_f16x4(vb[i].z, h[i][4], h[i][5]);
-                    i8x4_to_f16x4(vb[i].w, h[i][6], h[i][7]);
-                }
-                tc_st_32x32b_x32(a_lane + A_COL0 + 64 * sf, a);
                 uint8_t *ob = s.opb[sf];
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
+                for (int i = 0; i < 4; ++i) {
+                    const uint4 vb = lds16(sb + b_src[i]);
+                    uint32_t h[8];
+                    i8x4_to_f16x4(vb.x, h[0], h[1]);
+                    i8x4_to_f16x4(vb.y, h[2], h[3]);
+                    i8x4_to_f16x4(vb.z, h[4], h[5]);
+                    i8x4_to_f16x4(vb.w, h[6], h[7]);
                     if (!swap_b) {
-                        sts16(ob + b_dst[i][0], h[i][0], h[i][1], h[i][2], h[i][3]);
-                        sts16(ob + b_dst[i][1], h[i][4], h[i][5], h[i][6], h[i][7]);
+                        sts16(ob + b_dst[i][0], h[0], h[1], h[2], h[3]);
+                        sts16(ob + b_dst[i][1], h[4], h[5], h[6], h[7]);
                     } else {
-                        sts16(ob + b_dst[i][0], h[i][4], h[i][5], h[i][6], h[i][7]);
-                        sts16(ob + b_dst[i][1], h[i][0], h[i][1], h[i][2], h[i][3]);
+                        sts16(ob + b_dst[i][0], h[4], h[5], h[6], h[7]);
+                        sts16(ob + b_dst[i][1], h[0], h[1], h[2], h[3]);
                     }
                 }
                 // every value read from the staging slot now feeds an issued store
@@ -449,9 +453,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             if (!ch_in) continue;
             const EpiArgs e{p.y, p.residual, p.M, p.ldy, p.zy};
             const int tok0 = t.tt * TN + 64 * half;
-            int8_t *yp = e.y + (size_t)tok0 * (size_t)e.ldy + ch;
-            const int8_t *rp = e.residual ? e.residual + (size_t)tok0 * (size_t)e.ldy + ch : nullptr;
             const int ntok = min(64, e.M - tok0);
+            const size_t ldy = (size_t)e.ldy;
+            int8_t *yp = e.y + (size_t)tok0 * ldy + ch;
+            const int8_t *rp = e.residual ? e.residual + (size_t)tok0 * ldy + ch : nullptr;
             // quarters of 16 tokens: the residual bytes of a quarter are all
             // loaded before its first store (the compiler cannot know that y
             // and the residual do not alias), so each costs one round trip
@@ -459,22 +464,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             for (int q4 = 0; q4 < 4; ++q4) {
                 uint32_t res[4] = {0u, 0u, 0u, 0u};  // 4 bytes each
                 if (rp) {
+                    const int8_t *r = rp;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i)
-                        if (16 * q4 + i < ntok)
-                            res[i >> 2] |= (uint32_t)(uint8_t)rp[(size_t)(16 * q4 + i) * e.ldy]
-                                           << (8 * (i & 3));
+                    for (int i = 0; i < 16; ++i, r += ldy)
+                        if (16 * q4 + i < ntok) res[i >> 2] |= (uint32_t)(uint8_t)*r << (8 * (i & 3));
+                    rp = r;
                 }
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
+                for (int i = 0; i < 16; ++i, yp += ldy) {
                     const int j = 16 * q4 + i;
                     if (j < ntok) {
                         int32_t out = mq_requant((int32_t)(acc[j] - (uint32_t)corr), m0, sh, e.zy);
-                        if (rp) {
+                        if (e.residual) {
                             const int32_t r = (int32_t)(int8_t)(res[i >> 2] >> (8 * (i & 3)));
                             out = min(127, max(-128, out + r));
                         }
-                        yp[(size_t)j * e.ldy] = (int8_t)out;
+                        *yp = (int8_t)out;
                     }
                 }
             }
