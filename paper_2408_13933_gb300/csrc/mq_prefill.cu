@@ -172,6 +172,50 @@ struct EpiArgs {
     int M, ldy, zy;
 };
 
+// Requantize and store this thread's 64 outputs (one channel, 64 tokens
+// `ldy` bytes apart), with the residual added when RES.  The shift is the
+// thread's own (one channel), so its requant case is decided once; FULL
+// tiles skip the per-token bound.  The residual bytes of 16 tokens are all
+// loaded before their first store (the compiler cannot know that y and the
+// residual do not alias), so each group of 16 costs one round trip.
+template <bool RES, bool FULL, bool FAST>
+__device__ __forceinline__ void store_channel(const uint32_t (&acc)[64], int32_t corr, int32_t m0,
+                                              int32_t sh, int32_t zy, int8_t *yp,
+                                              const int8_t *rp, size_t ldy, int ntok) {
+    // FAST: shift >= 33, (mulhi + 2^(s-33)) >> (s-32); other shifts: mq_requant
+    const int32_t rnd = FAST ? (1 << (sh - 33)) : 0;
+    const int32_t rs = FAST ? sh - 32 : 0;
+#pragma unroll
+    for (int q4 = 0; q4 < 4; ++q4) {
+        uint32_t res[4] = {0u, 0u, 0u, 0u};  // 4 bytes each
+        if (RES) {
+            const int8_t *r = rp;
+#pragma unroll
+            for (int i = 0; i < 16; ++i, r += ldy)
+                if (FULL || 16 * q4 + i < ntok) res[i >> 2] |= (uint32_t)(uint8_t)*r << (8 * (i & 3));
+            rp = r;
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i, yp += ldy) {
+            const int j = 16 * q4 + i;
+            if (FULL || j < ntok) {
+                const int32_t a = (int32_t)(acc[j] - (uint32_t)corr);
+                int32_t out = FAST ? min(127, max(-128, ((__mulhi(a, m0) + rnd) >> rs) + zy))
+                                   : mq_requant(a, m0, sh, zy);
+                if (RES) {
+                    const int32_t r = (int32_t)(int8_t)(res[i >> 2] >> (8 * (i & 3)));
+                    out = min(127, max(-128, out + r));
+                }
+                *yp = (int8_t)out;
+            }
+        }
+    }
+}
+
+// Barrier scopes: arrivals from the other CTA are releases at cluster scope
+// (st.async complete_tx, mbarrier.arrive.release.cluster, multicast commits),
+// so the data they publish is visible cluster-wide before the phase can
+// complete; waiters acquire at CTA scope, which is far cheaper per wait.
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     prefill_kernel(const __grid_constant__ Params P) {
     extern __shared__ uint8_t smem_raw[];
@@ -254,8 +298,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     const bool chunk_start = (kb % t.kpc) == 0;
                     if (chunk_start) {
                         const uint32_t b = chunks & 1;
-                        if (!mq_wait_parity_cluster(&s.f_empty[b], ((chunks >> 1) & 1) ^ 1,
-                                                    &s.abort, P.status)) {
+                        if (!mq_wait_parity(&s.f_empty[b], ((chunks >> 1) & 1) ^ 1, &s.abort,
+                                            P.status)) {
                             ok = false;
                             break;
                         }
@@ -264,8 +308,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     }
                     const int slot = it % SF;
                     mbar_arrive_expect_tx(&s.op_full[slot], 4 * (CONV_WARPS / 2));
-                    if (!mq_wait_parity_cluster(&s.op_full[slot], (it / SF) & 1, &s.abort,
-                                                P.status)) {
+                    if (!mq_wait_parity(&s.op_full[slot], (it / SF) & 1, &s.abort, P.status)) {
                         ok = false;
                         break;
                     }
@@ -287,7 +330,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             }
             // every MMA issued above has completed once `done` fires
             tc_commit2_mc(&s.done, 1);
-            mq_wait_parity_cluster(&s.done, 0, &s.abort, P.status);
+            mq_wait_parity(&s.done, 0, &s.abort, P.status);
         }
         __syncwarp();
     } else if (warp < EPI_WARP0) {
@@ -457,31 +500,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const size_t ldy = (size_t)e.ldy;
             int8_t *yp = e.y + (size_t)tok0 * ldy + ch;
             const int8_t *rp = e.residual ? e.residual + (size_t)tok0 * ldy + ch : nullptr;
-            // quarters of 16 tokens: the residual bytes of a quarter are all
-            // loaded before its first store (the compiler cannot know that y
-            // and the residual do not alias), so each costs one round trip
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-                uint32_t res[4] = {0u, 0u, 0u, 0u};  // 4 bytes each
-                if (rp) {
-                    const int8_t *r = rp;
-#pragma unroll
-                    for (int i = 0; i < 16; ++i, r += ldy)
-                        if (16 * q4 + i < ntok) res[i >> 2] |= (uint32_t)(uint8_t)*r << (8 * (i & 3));
-                    rp = r;
-                }
-#pragma unroll
-                for (int i = 0; i < 16; ++i, yp += ldy) {
-                    const int j = 16 * q4 + i;
-                    if (j < ntok) {
-                        int32_t out = mq_requant((int32_t)(acc[j] - (uint32_t)corr), m0, sh, e.zy);
-                        if (e.residual) {
-                            const int32_t r = (int32_t)(int8_t)(res[i >> 2] >> (8 * (i & 3)));
-                            out = min(127, max(-128, out + r));
-                        }
-                        *yp = (int8_t)out;
-                    }
-                }
+            const bool full = ntok == 64, fast = sh >= 33;
+            if (rp) {
+                if (full && fast) store_channel<true, true, true>(acc, corr, m0, sh, e.zy, yp, rp, ldy, 64);
+                else store_channel<true, false, false>(acc, corr, m0, sh, e.zy, yp, rp, ldy, ntok);
+            } else {
+                if (full && fast) store_channel<false, true, true>(acc, corr, m0, sh, e.zy, yp, rp, ldy, 64);
+                else store_channel<false, false, false>(acc, corr, m0, sh, e.zy, yp, rp, ldy, ntok);
             }
         }
     }
