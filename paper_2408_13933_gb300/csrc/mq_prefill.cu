@@ -105,8 +105,8 @@ struct Smem {
     uint8_t opb[SF][OPB];
     uint64_t ld_full[S8];
     uint64_t ld_empty[S8];
-    uint64_t op_full[SF];   // even CTA: its converter warps + the MMA thread arrive, the odd
-                            // CTA's converter warps signal 4 transaction bytes each
+    uint64_t op_full[SF];   // even CTA: its converter warps arrive (one announcing 16
+                            // bytes), the odd CTA's converter warps signal 4 bytes each
     uint64_t op_empty[SF];  // both CTAs: multicast commit
     uint64_t f_full[2];     // both CTAs: multicast commit
     uint64_t f_empty[2];    // even CTA: both CTAs' epilogue warps arrive
@@ -232,7 +232,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             mbar_init(&s.ld_empty[i], CONV_WARPS / 2);
         }
         for (int i = 0; i < SF; ++i) {
-            mbar_init(&s.op_full[i], CONV_WARPS / 2 + 1);
+            mbar_init(&s.op_full[i], CONV_WARPS / 2);
             mbar_init(&s.op_empty[i], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -294,8 +294,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
                 const Tile t = tile_at(P, tile);
                 uint32_t fcol = 0;
+                int kc = 0;  // stage within the exact-f32 chunk
                 for (int kb = 0; kb < t.nkb; ++kb, ++it) {
-                    const bool chunk_start = (kb % t.kpc) == 0;
+                    const bool chunk_start = kc == 0;
                     if (chunk_start) {
                         const uint32_t b = chunks & 1;
                         if (!mq_wait_parity(&s.f_empty[b], ((chunks >> 1) & 1) ^ 1, &s.abort,
@@ -307,7 +308,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         fcol = F_COL0 + 128 * b;
                     }
                     const int slot = it % SF;
-                    mbar_arrive_expect_tx(&s.op_full[slot], 4 * (CONV_WARPS / 2));
                     if (!mq_wait_parity(&s.op_full[slot], (it / SF) & 1, &s.abort, P.status)) {
                         ok = false;
                         break;
@@ -322,9 +322,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                                        (j < 4 ? bd0 : bd1) + 2 * (j & 3), idesc,
                                        (chunk_start && j == 0) ? 0u : 1u);
                     tc_commit2_mc(&s.op_empty[slot], 3);
-                    if (((kb + 1) % t.kpc) == 0 || kb + 1 == t.nkb) {
+                    if (++kc == t.kpc || kb + 1 == t.nkb) {
                         tc_commit2_mc(&s.f_full[chunks & 1], 3);
                         ++chunks;
+                        kc = 0;
                     }
                 }
             }
@@ -444,7 +445,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
-                    if (rank == 0)
+                    if (rank == 0 && gt == 0)  // also announces the odd CTA's signal bytes
+                        mbar_arrive_expect_tx(&s.op_full[sf], 4 * (CONV_WARPS / 2));
+                    else if (rank == 0)
                         mbar_arrive(&s.op_full[sf]);
                     else
                         st_async_signal(leader_sink, it, leader_op_full + 8u * (uint32_t)sf);
