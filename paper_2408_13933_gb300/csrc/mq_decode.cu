@@ -67,7 +67,10 @@ constexpr int ROW_BYTES = 128;         // weight bytes per row per stage
 constexpr int W_BYTES = UNIT_ROWS * ROW_BYTES;  // 8 KB of weights
 constexpr int X_BOX = 16 * 128;                 // one x box: 16 tokens x 128 k
 constexpr int STAGE_BYTES = W_BYTES + 2 * X_BOX;
-constexpr int STAGES = 8;
+// Ring depth: the cross-warp reduction buffer grows with the token tiles, so
+// the ring shrinks to keep two CTAs per SM.
+template <int NT>
+constexpr int stages_for() { return NT == 1 ? 7 : 6; }
 constexpr int CONS_BARRIER = 1;        // named barrier among the consumer warps
 
 struct Params {
@@ -81,12 +84,16 @@ struct Params {
     int *status;
 };
 
+template <int NT>
 struct Smem {
+    static constexpr int STAGES = stages_for<NT>();
     uint8_t ring[STAGES][STAGE_BYTES];
     uint64_t full[STAGES];
     uint64_t empty[STAGES];
-    int32_t red[UNIT_ROWS][16];   // per (row, token) int32 partial sums
-    int32_t xsum[2][16];          // per token activation sum, by piece parity
+    // each consumer warp's int32 partial sums of a piece, by mma fragment
+    // element e = (rt * NT + nt) * 4 + i and lane (conflict-free both ways)
+    int32_t part[CONS_WARPS][16 * NT][32];
+    int32_t xpart[CONS_WARPS][16];  // each warp's activation sums per token
     int32_t row_corr[UNIT_ROWS];  // zx * colsum[n] of the current unit's rows
     int32_t row_m0[UNIT_ROWS];
     int32_t row_shift[UNIT_ROWS];
@@ -95,7 +102,8 @@ struct Smem {
     int abort;
 };
 
-constexpr size_t SMEM_BYTES = sizeof(Smem) + 1024;
+template <int NT>
+constexpr size_t smem_bytes() { return sizeof(Smem<NT>) + 1024; }
 
 __device__ __forceinline__ void cons_sync() {
     asm volatile("bar.sync %0, %1;" ::"n"(CONS_BARRIER), "n"(CONS_THREADS) : "memory");
@@ -161,7 +169,8 @@ __device__ __forceinline__ int cta_of(int s, int S, int G) {
 
 // Problem holding global stage s, searching forward from `pi` (stages are
 // visited in increasing order, so the walk is amortized O(1)).
-__device__ __forceinline__ int problem_from(const Smem &sm, int count, int pi, int s) {
+template <class SM>
+__device__ __forceinline__ int problem_from(const SM &sm, int count, int pi, int s) {
     while (pi + 1 < count && s >= sm.prob[pi + 1].tile_begin) ++pi;
     return pi;
 }
@@ -169,7 +178,8 @@ __device__ __forceinline__ int problem_from(const Smem &sm, int count, int pi, i
 // Requantize one output of tile row `row` (global row n, token tok) from
 // sum(w x): acc = sum(w x) - zx colsum[n], fixed point, saturate, optional
 // residual.
-__device__ __forceinline__ void store_out(const Problem &p, const Smem &sm, int row, int n,
+template <class SM>
+__device__ __forceinline__ void store_out(const Problem &p, const SM &sm, int row, int n,
                                           int tok, int32_t sum_wx) {
     // two's-complement wrap is exact: the true value fits in int32
     const int32_t a = (int32_t)((uint32_t)sum_wx - (uint32_t)sm.row_corr[row]);
@@ -273,8 +283,10 @@ __device__ __forceinline__ void compute_stage(const uint8_t *ring, int warp, int
 template <int BITS, int NT>
 __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constant__ Params P) {
     using C = Cfg<BITS>;
+    using SM = Smem<NT>;
+    constexpr int STAGES = SM::STAGES;
     extern __shared__ uint8_t smem_raw[];
-    Smem &s = *reinterpret_cast<Smem *>(
+    SM &s = *reinterpret_cast<SM *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int S = P.total_stages, G = gridDim.x, cta = blockIdx.x;
@@ -289,8 +301,6 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
         s.last[0] = s.last[1] = 0;
         fence_mbar_init();
     }
-    for (int i = threadIdx.x; i < UNIT_ROWS * 16; i += THREADS) (&s.red[0][0])[i] = 0;
-    if (threadIdx.x < 32) (&s.xsum[0][0])[threadIdx.x] = 0;
     for (int i = threadIdx.x; i < P.count; i += THREADS) s.prob[i] = P.p[i];
     __syncthreads();
     const int count = P.count;
@@ -398,8 +408,10 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     }
                 }
             }
-            // ---- this CTA's partial of the unit: fragment element i of tile
-            // (rt, nt) is row rt*16 + g (+8 for i >= 2), token nt*8 + 2t + (i & 1)
+            // ---- this CTA's partial of the unit.  Fragment element i of tile
+            // (rt, nt) is row rt*16 + g (+8 for i >= 2), token nt*8 + 2t + (i & 1);
+            // each warp writes its partials to its own slice, then every
+            // thread sums a fixed set of slots over the eight warps.
             if (ok) {
 #pragma unroll
                 for (int rt = 0; rt < 4; ++rt)
@@ -407,18 +419,16 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
                         for (int i = 0; i < 4; ++i) {
-                            const int row = rt * 16 + g + (i >= 2 ? 8 : 0);
-                            const int tok = nt * 8 + 2 * t + (i & 1);
                             int32_t v = __float2int_rn(acc[rt][nt][i] * 16777216.0f);
                             if constexpr (C::FLUSH) v += iacc[rt][nt][i];
-                            if (tok < p.M) atomicAdd(&s.red[row][tok], v);
+                            s.part[warp][(rt * NT + nt) * 4 + i][lane] = v;
                         }
 #pragma unroll
                 for (int nt = 0; nt < NT; ++nt) {
                     int v = xs[nt];
                     v += __shfl_xor_sync(0xffffffffu, v, 1);
                     v += __shfl_xor_sync(0xffffffffu, v, 2);
-                    if (t == 0 && nt * 8 + g < p.M) atomicAdd(&s.xsum[par][nt * 8 + g], v);
+                    if (t == 0) s.xpart[warp][nt * 8 + g] = v;
                 }
             }
             if (threadIdx.x < UNIT_ROWS) {
@@ -428,30 +438,45 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             }
             cons_sync();
             const bool whole = u_begin >= s_begin && u_end <= s_end;
-            const int ntile = UNIT_ROWS * p.M;
+            // this thread's slots j + 256 q share one fragment element i, one
+            // token tile and one lane: the token is fixed
+            const int e0 = threadIdx.x >> 5, ln = threadIdx.x & 31;
+            const int tok = (NT == 2 ? ((e0 >> 2) & 1) * 8 : 0) + 2 * (ln & 3) + (e0 & 1);
+            int32_t xsum = 0;
+            if (ok && tok < p.M) {
+#pragma unroll
+                for (int w = 0; w < CONS_WARPS; ++w) xsum += s.xpart[w][tok];
+            }
             if (ok && whole) {
                 // the unit is entirely this CTA's: requantize and store
-                for (int idx = threadIdx.x; idx < ntile; idx += CONS_THREADS) {
-                    const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
+#pragma unroll
+                for (int q = 0; q < 2 * NT; ++q) {
+                    const int e = e0 + 8 * q;
+                    const int row = ((e >> 2) / NT) * 16 + (ln >> 2) + ((e & 2) ? 8 : 0);
                     const int n = rb * UNIT_ROWS + row;
-                    const int32_t sum = s.red[row][tok];
-                    s.red[row][tok] = 0;
+                    if (tok >= p.M || n >= p.N) continue;
+                    int32_t sum = 0;
+#pragma unroll
+                    for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
                     // sum(w x) = sum(u x) - bias * sum(x)
-                    if (n < p.N)
-                        store_out(p, s, row, n, tok,
-                                  (int32_t)((uint32_t)sum -
-                                            (uint32_t)(C::BIAS * s.xsum[par][tok])));
+                    store_out(p, s, row, n, tok,
+                              (int32_t)((uint32_t)sum - (uint32_t)(C::BIAS * xsum)));
                 }
             } else if (ok) {
                 // a split unit: add this piece to the slot of its first contributor
                 const int first = cta_of(u_begin, S, G), last_c = cta_of(u_end - 1, S, G);
                 int32_t *slot_sum = P.ws_sum + (size_t)first * UNIT_ROWS * 16;
-                for (int idx = threadIdx.x; idx < ntile; idx += CONS_THREADS) {
-                    const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
-                    const int32_t part = (int32_t)((uint32_t)s.red[row][tok] -
-                                                   (uint32_t)(C::BIAS * s.xsum[par][tok]));
-                    s.red[row][tok] = 0;
-                    atomicAdd(slot_sum + row * 16 + tok, part);
+                if (tok < p.M) {
+#pragma unroll
+                    for (int q = 0; q < 2 * NT; ++q) {
+                        const int e = e0 + 8 * q;
+                        const int row = ((e >> 2) / NT) * 16 + (ln >> 2) + ((e & 2) ? 8 : 0);
+                        int32_t sum = 0;
+#pragma unroll
+                        for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
+                        atomicAdd(slot_sum + row * 16 + tok,
+                                  (int32_t)((uint32_t)sum - (uint32_t)(C::BIAS * xsum)));
+                    }
                 }
                 __threadfence();
                 cons_sync();
@@ -462,30 +487,30 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                 }
                 cons_sync();
                 if (s.last[par]) {
+                    const int ntile = UNIT_ROWS * p.M;
                     // ntile <= 1024 = 4 * CONS_THREADS: all loads first, then use
                     int32_t sums[4];
 #pragma unroll
                     for (int r = 0; r < 4; ++r) {
                         const int idx = threadIdx.x + r * CONS_THREADS;
-                        const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
-                        sums[r] = idx < ntile ? __ldcg(slot_sum + row * 16 + tok) : 0;
+                        const int row = idx % UNIT_ROWS, tk = idx / UNIT_ROWS;
+                        sums[r] = idx < ntile ? __ldcg(slot_sum + row * 16 + tk) : 0;
                     }
 #pragma unroll
                     for (int r = 0; r < 4; ++r) {
                         const int idx = threadIdx.x + r * CONS_THREADS;
                         if (idx >= ntile) continue;
-                        const int row = idx % UNIT_ROWS, tok = idx / UNIT_ROWS;
+                        const int row = idx % UNIT_ROWS, tk = idx / UNIT_ROWS;
                         const int n = rb * UNIT_ROWS + row;
-                        slot_sum[row * 16 + tok] = 0;
-                        if (n < p.N) store_out(p, s, row, n, tok, sums[r]);
+                        slot_sum[row * 16 + tk] = 0;
+                        if (n < p.N) store_out(p, s, row, n, tk, sums[r]);
                     }
                     if (threadIdx.x == 0) P.ws_count[first] = 0;
                 }
             }
-            cons_sync();  // every read of red / xsum / last / row params is done
-            // reset this parity's buffers; they are used again two pieces on,
-            // after the next piece's barriers
-            if (threadIdx.x < 16) s.xsum[par][threadIdx.x] = 0;
+            cons_sync();  // every read of part / xpart / last / row params is done
+            // reset this parity's flag; it is used again two pieces on, after
+            // the next piece's barriers
             if (threadIdx.x == 0) s.last[par] = 0;
             par ^= 1;
             gs = piece_end;
@@ -531,7 +556,7 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
     if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
     if (attr_done != dev) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)SMEM_BYTES) != cudaSuccess)
+                                 (int)smem_bytes<NT>()) != cudaSuccess)
             return MQ_ERR_CUDA;
         attr_done = dev;
     }
@@ -566,7 +591,7 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
         long long grid = 2LL * sms;
         if (grid > DECODE_MAX_GRID) grid = DECODE_MAX_GRID;
         if (grid > stages) grid = stages;
-        kern<<<(int)grid, THREADS, SMEM_BYTES, stream>>>(P);
+        kern<<<(int)grid, THREADS, smem_bytes<NT>(), stream>>>(P);
         if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;
