@@ -125,7 +125,12 @@ int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes);
  *   workspace: device, ws_bytes >= mq_workspace_size (may be NULL when 0);
  *              see the workspace contract at mq_workspace_size
  * Requirements: 0 <= M, N; 0 <= K <= MQ_MAX_K; K % 16 == 0; ldx % 16 == 0;
- * x and packed 16-byte aligned.  With K == 0 (every output is requant(0),
+ * x and packed 16-byte aligned.  Kernels are launched with programmatic
+ * stream serialization: a call may start while the previous kernel in the
+ * stream is finishing, and it reads `packed` (a constant input) before
+ * waiting for that kernel; x, colsum, M0, shift, residual, y and the
+ * workspace are touched only after it has completed.  So `packed` must not be
+ * written by kernels still running in the same stream.  With K == 0 (every output is requant(0),
  * i.e. zy) x and packed are not read and may be NULL.  M <= 16 runs the
  * weight-streaming decode kernel, larger M the tcgen05 tensor-core kernel;
  * both are bit-exact.

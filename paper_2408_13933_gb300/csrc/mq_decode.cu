@@ -303,6 +303,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
     }
     for (int i = threadIdx.x; i < P.count; i += THREADS) s.prob[i] = P.p[i];
     __syncthreads();
+    if (threadIdx.x == 0) griddep_launch_dependents();
     const int count = P.count;
 
     if (warp == PROD_WARP) {
@@ -314,8 +315,24 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     prefetch_tensormap(&P.tmap_x[i]);
                 }
             constexpr int XBOXES = C::KSTAGE / 128;  // x boxes per stage (int4: 2, int8: 1)
-            uint32_t it = 0;
+            // Packed weights are constant inputs: the weight boxes of the first
+            // ring stages are requested before waiting for the previous grid
+            // in the stream; activations only after it.
+            const int npre = s_end - s_begin < STAGES ? s_end - s_begin : STAGES;
             int pi = 0;
+            for (int i = 0; i < npre; ++i) {
+                const int gs = s_begin + i;
+                pi = problem_from(s, count, pi, gs);
+                const Problem &p = s.prob[pi];
+                if (p.K == 0) continue;
+                const int local = gs - p.tile_begin;
+                const int rb = local / p.tiles_m, j = local % p.tiles_m;
+                mbar_arrive_expect_tx(&s.full[i], W_BYTES + XBOXES * X_BOX);
+                tma_load_2d(s.ring[i], &P.tmap_w[pi], j * ROW_BYTES, rb * UNIT_ROWS, &s.full[i]);
+            }
+            griddep_wait();
+            uint32_t it = 0;
+            pi = 0;
             for (int gs = s_begin; gs < s_end; ++gs, ++it) {
                 pi = problem_from(s, count, pi, gs);
                 const Problem &p = s.prob[pi];
@@ -328,9 +345,11 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     mbar_arrive(&s.full[slot]);
                     continue;
                 }
-                mbar_arrive_expect_tx(&s.full[slot], W_BYTES + XBOXES * X_BOX);
-                tma_load_2d(s.ring[slot], &P.tmap_w[pi], j * ROW_BYTES, rb * UNIT_ROWS,
-                            &s.full[slot]);
+                if ((int)it >= npre) {
+                    mbar_arrive_expect_tx(&s.full[slot], W_BYTES + XBOXES * X_BOX);
+                    tma_load_2d(s.ring[slot], &P.tmap_w[pi], j * ROW_BYTES, rb * UNIT_ROWS,
+                                &s.full[slot]);
+                }
 #pragma unroll
                 for (int h = 0; h < XBOXES; ++h)
                     tma_load_2d(s.ring[slot] + W_BYTES + h * X_BOX, &P.tmap_x[pi],
@@ -340,6 +359,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
         __syncwarp();
     } else {
         // ------------------------------------------------------ consumers
+        griddep_wait();  // before the first global access (parameters, workspace, y)
         const int g = lane >> 2, t = lane & 3;
         uint32_t it = 0;
         bool ok = true;  // after a failed wait the warps still walk the barriers
@@ -591,8 +611,19 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
         long long grid = 2LL * sms;
         if (grid > DECODE_MAX_GRID) grid = DECODE_MAX_GRID;
         if (grid > stages) grid = stages;
-        kern<<<(int)grid, THREADS, smem_bytes<NT>(), stream>>>(P);
-        if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
+        // programmatic stream serialization: this launch may start while the
+        // previous kernel in the stream finishes (see griddep_wait)
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)grid, 1, 1);
+        cfg.blockDim = dim3(THREADS, 1, 1);
+        cfg.dynamicSmemBytes = smem_bytes<NT>();
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&cfg, kern, P) != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;
 }

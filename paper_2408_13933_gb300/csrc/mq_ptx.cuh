@@ -114,6 +114,20 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// ------------------------------------------ programmatic dependent launch
+// Wait until the grids this one depends on (the previous kernel in the
+// stream, when launched with programmatic stream serialization) have
+// completed and their memory is visible; a no-op otherwise.
+__device__ __forceinline__ void griddep_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Let the next kernel in the stream be scheduled once every CTA of this grid
+// has signalled (it still waits for this grid's completion before reading).
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ----------------------------------------------------------------- clusters
 __device__ __forceinline__ uint32_t cluster_ctarank() {
     uint32_t r;
