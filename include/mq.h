@@ -130,8 +130,8 @@ int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes);
  * stream is finishing, and it reads `packed` (a constant input) before
  * waiting for that kernel; x, colsum, M0, shift, residual, y and the
  * workspace are touched only after it has completed.  So `packed` must not be
- * written by kernels still running in the same stream.  With K == 0 (every output is requant(0),
- * i.e. zy) x and packed are not read and may be NULL.  M <= 16 runs the
+ * written by kernels still running in the same stream.  With K == 0 (every
+ * output is requant(0), i.e. zy) x and packed are not read and may be NULL.  M <= 16 runs the
  * weight-streaming decode kernel, larger M the tcgen05 tensor-core kernel;
  * both are bit-exact.
  * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_K_OVERFLOW, MQ_ERR_ALIGNMENT,

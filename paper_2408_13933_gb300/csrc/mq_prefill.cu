@@ -250,6 +250,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     tc_fence_before();
     cluster_sync();  // barriers of both CTAs initialised before any remote arrive
     tc_fence_after();
+    if (threadIdx.x == 0) griddep_launch_dependents();
     const uint32_t tmem = s.tmem_base;
 
     if (warp == TMA_WARP) {
@@ -260,6 +261,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 prefetch_tensormap(&P.tmap_x[i]);
                 prefetch_tensormap(&P.tmap_w[i]);
             }
+            // Packed weights are constant inputs: the weight boxes of the first
+            // S8 stages are requested before waiting for the previous grid in
+            // the stream; activations only after it.
+            uint32_t npre = 0;
+            {
+                int tile;
+                for (int ti = 0; npre < (uint32_t)S8 && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
+                    const Tile t = tile_at(P, tile);
+                    const bool i4 = P.p[t.pi].bits == 4;
+                    const int wrow = t.ct * TM + (int)rank * CM;
+                    for (int kb = 0; kb < t.nkb && npre < (uint32_t)S8; ++kb, ++npre) {
+                        mbar_arrive_expect_tx(&s.ld_full[npre], (i4 ? STA / 2 : STA) + STB);
+                        tma_load_2d(s.sta[npre], &P.tmap_w[t.pi], i4 ? kb * (KS / 2) : kb * KS,
+                                    wrow, &s.ld_full[npre]);
+                    }
+                }
+            }
+            griddep_wait();
             uint32_t it = 0;
             bool ok = true;
             int tile;
@@ -276,9 +295,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&s.ld_full[slot], bytes);
-                    tma_load_2d(s.sta[slot], &P.tmap_w[t.pi], i4 ? kb * (KS / 2) : kb * KS, wrow,
-                                &s.ld_full[slot]);
+                    if (it >= npre) {
+                        mbar_arrive_expect_tx(&s.ld_full[slot], bytes);
+                        tma_load_2d(s.sta[slot], &P.tmap_w[t.pi], i4 ? kb * (KS / 2) : kb * KS,
+                                    wrow, &s.ld_full[slot]);
+                    }
                     tma_load_2d(s.stb[slot], &P.tmap_x[t.pi], kb * KS, xrow, &s.ld_full[slot]);
                 }
             }
@@ -456,6 +477,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         }
     } else {
         // ------------------------------------------------------ epilogue
+        griddep_wait();  // before the first global access (parameters, residual, y)
         const int quad = warp & 3;                  // TMEM lane quarter of this warp
         const int half = (warp - EPI_WARP0) >> 2;   // token half of the tile
         const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(64 * half);
@@ -660,8 +682,19 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
         P.npairs = tiles < pairs_max ? (int)tiles : pairs_max;
         P.use_table = tiles <= MAX_SCHED ? 1 : 0;
         if (P.use_table) lpt_schedule(P, P.npairs);
-        prefill_kernel<<<2 * P.npairs, THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(P);
-        if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
+        // programmatic stream serialization: this launch may start while the
+        // previous kernel in the stream finishes (see griddep_wait)
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)(2 * P.npairs), 1, 1);
+        cfg.blockDim = dim3(THREADS, 1, 1);
+        cfg.dynamicSmemBytes = SMEM_BYTES;
+        cfg.stream = static_cast<cudaStream_t>(stream);
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&cfg, prefill_kernel, P) != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;
 }
