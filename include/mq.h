@@ -100,8 +100,9 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed,
 /*
  * Device workspace bytes a mq_linear_* call of this shape needs: 0 for the
  * tensor-core path (M > 16); for the decode path (1 <= M <= 16) a fixed size
- * (about 1.3 MB) holding per-CTA int32 partial sums and counters, used to
- * combine 64-row units whose K range is split among CTAs.  For
+ * (2.5 MB) holding, per CTA of the decode grid, int32 partial sums tagged with
+ * a launch number, used to combine 64-row units whose K range is split among
+ * CTAs.  For
  * mq_linear_batch the workspace must hold the largest size of its
  * descriptors.
  * Workspace contract: device memory, 16-byte aligned, zero-filled before its
@@ -162,7 +163,7 @@ int mq_linear_w4a8(const int8_t *x, int M, int K, int ldx, int32_t zx,
  * For callers that cannot provide device memory around a decode step: a C
  * program with no device allocator of its own, or a serving loop whose memory
  * pool is fixed after warm-up and must not grow mid-generation.  The split-K
- * combine scratch (about 1.3 MB) is a static device array inside libmq, one
+ * combine scratch (2.5 MB) is a static device array inside libmq, one
  * per device; each call clears it on `stream` with a memset before the
  * kernel, and no call allocates or frees device memory.
  *

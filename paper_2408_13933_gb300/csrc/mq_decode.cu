@@ -10,9 +10,12 @@
 // global sequence of stages is split evenly among the CTAs of a persistent
 // grid (two per SM), so every SM streams the same number of weight bytes no
 // matter how the linears' sizes differ.  A unit whose stages fall to several
-// CTAs is combined in the caller's workspace: each contributor adds its int32
-// partial sums with atomics and counts itself in; the last one requantizes,
-// stores, and leaves the slot and counter zero again.
+// CTAs is finished by its first CTA, which reaches the unit at the end of its
+// range; the later contributors, which process the unit's tail at the start
+// of theirs, store their int32 partial sums in their own workspace slot, each
+// with the launch's epoch in the same 8-byte store, and go on without
+// waiting.  The first CTA polls the entries for the epoch, adds them,
+// requantizes, and stores zero back, so the workspace is left zero.
 //
 // Data path.  In each CTA one producer thread streams the weight rows of its
 // stages with TMA into an 8-stage shared-memory ring, continuing across unit
@@ -44,13 +47,18 @@
 // k index is whatever the unpacking yields; the activation fragments use the
 // same assignment.
 //
-// Epilogue (per unit): the eight warps' int32 partials and activation sums
-// meet in shared memory; acc = sum(u x) - bias sum(x) - zx colsum[n], then
+// Epilogue (per unit): each warp writes its int32 partials and activation sums
+// to its own shared-memory slice; every thread then sums a fixed set of slots
+// over the eight warps; acc = sum(u x) - bias sum(x) - zx colsum[n], then
 // fixed-point requant (round half up), saturation, optional residual, store.
+// Launches use programmatic dependent launch: the first ring stages' weights
+// are requested before waiting for the previous kernel in the stream.
 // All mbarrier waits are bounded (mq_wait_parity).
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
+
+#include <atomic>
 
 #include "mq_internal.h"
 #include "mq_ptx.cuh"
@@ -79,8 +87,8 @@ struct Params {
     Problem p[DECODE_MAX_PROBLEMS];  // tile_begin = first global stage, tiles_m = stages per unit
     int count;
     int total_stages;
-    int32_t *ws_count;   // [gridDim.x] contributor counters (zero between calls)
-    int32_t *ws_sum;     // [gridDim.x][UNIT_ROWS][16] partial sums (zero between calls)
+    int2 *ws;            // [gridDim.x][UNIT_ROWS][16] {partial sum, epoch} (zero between calls)
+    uint32_t epoch;      // nonzero, different for every launch
     int *status;
 };
 
@@ -98,7 +106,6 @@ struct Smem {
     int32_t row_m0[UNIT_ROWS];
     int32_t row_shift[UNIT_ROWS];
     Problem prob[DECODE_MAX_PROBLEMS];  // the kernel's problem table, read once
-    int last[2];                  // this CTA completes a split unit, by piece parity
     int abort;
 };
 
@@ -173,6 +180,36 @@ template <class SM>
 __device__ __forceinline__ int problem_from(const SM &sm, int count, int pi, int s) {
     while (pi + 1 < count && s >= sm.prob[pi + 1].tile_begin) ++pi;
     return pi;
+}
+
+__device__ __forceinline__ void st_relaxed_v2(int2 *p, uint32_t a, uint32_t b) {
+    asm volatile("st.relaxed.gpu.global.v2.b32 [%0], {%1, %2};" ::"l"(p), "r"(a), "r"(b) : "memory");
+}
+
+// Wait (bounded, like every wait in this library) until the entry carries
+// `epoch`; its value is returned in `val`.
+__device__ __forceinline__ bool poll_entry(const int2 *p, uint32_t epoch, int32_t &val,
+                                           volatile int *abort, int *status) {
+    uint64_t t0 = 0;
+    while (true) {
+        int32_t a;
+        uint32_t b;
+        asm volatile("ld.relaxed.gpu.global.v2.b32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "l"(p) : "memory");
+        if (b == epoch) {
+            val = a;
+            return true;
+        }
+        if (*abort) return false;
+        const uint64_t t = global_timer_ns();
+        if (t0 == 0) {
+            t0 = t;
+        } else if (t - t0 > MQ_WAIT_LIMIT_NS) {
+            *abort = 1;
+            atomicOr(status, MQ_DEVICE_STATUS_TIMEOUT);
+            return false;
+        }
+        __nanosleep(128);
+    }
 }
 
 // Requantize one output of tile row `row` (global row n, token tok) from
@@ -298,7 +335,6 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             mbar_init(&s.empty[i], CONS_WARPS);
         }
         s.abort = 0;
-        s.last[0] = s.last[1] = 0;
         fence_mbar_init();
     }
     for (int i = threadIdx.x; i < P.count; i += THREADS) s.prob[i] = P.p[i];
@@ -483,55 +519,60 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                               (int32_t)((uint32_t)sum - (uint32_t)(C::BIAS * xsum)));
                 }
             } else if (ok) {
-                // a split unit: add this piece to the slot of its first contributor
-                const int first = cta_of(u_begin, S, G), last_c = cta_of(u_end - 1, S, G);
-                int32_t *slot_sum = P.ws_sum + (size_t)first * UNIT_ROWS * 16;
+                // A split unit.  Its first CTA finishes it: that CTA reaches the
+                // unit at the end of its range, while the later contributors
+                // process the unit's tail at the start of theirs.  A
+                // contributor stores each of its sums together with this
+                // launch's epoch as one 8-byte store (single-copy atomic) and
+                // goes on; the first CTA polls each entry until it carries the
+                // epoch, adds it, and stores zero back.  No fences or counters.
+                const int cf = cta_of(u_begin, S, G), cl = cta_of(u_end - 1, S, G);
                 if (tok < p.M) {
+                    uint32_t v[2 * NT];
+                    int rows[2 * NT];
 #pragma unroll
                     for (int q = 0; q < 2 * NT; ++q) {
                         const int e = e0 + 8 * q;
-                        const int row = ((e >> 2) / NT) * 16 + (ln >> 2) + ((e & 2) ? 8 : 0);
+                        rows[q] = ((e >> 2) / NT) * 16 + (ln >> 2) + ((e & 2) ? 8 : 0);
                         int32_t sum = 0;
 #pragma unroll
                         for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
-                        atomicAdd(slot_sum + row * 16 + tok,
-                                  (int32_t)((uint32_t)sum - (uint32_t)(C::BIAS * xsum)));
+                        v[q] = (uint32_t)sum - (uint32_t)(C::BIAS * xsum);
                     }
-                }
-                __threadfence();
-                cons_sync();
-                if (threadIdx.x == 0) {
-                    const int done = atomicAdd(P.ws_count + first, 1);
-                    s.last[par] = done == last_c - first;
-                    __threadfence();
-                }
-                cons_sync();
-                if (s.last[par]) {
-                    const int ntile = UNIT_ROWS * p.M;
-                    // ntile <= 1024 = 4 * CONS_THREADS: all loads first, then use
-                    int32_t sums[4];
+                    if (cta != cf) {
+                        int2 *mine = P.ws + (size_t)cta * UNIT_ROWS * 16;
 #pragma unroll
-                    for (int r = 0; r < 4; ++r) {
-                        const int idx = threadIdx.x + r * CONS_THREADS;
-                        const int row = idx % UNIT_ROWS, tk = idx / UNIT_ROWS;
-                        sums[r] = idx < ntile ? __ldcg(slot_sum + row * 16 + tk) : 0;
-                    }
+                        for (int q = 0; q < 2 * NT; ++q)
+                            st_relaxed_v2(mine + rows[q] * 16 + tok, v[q], P.epoch);
+                    } else {
+                        bool got = true;
+                        for (int c = cf + 1; got && c <= cl; ++c) {
+                            const int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
 #pragma unroll
-                    for (int r = 0; r < 4; ++r) {
-                        const int idx = threadIdx.x + r * CONS_THREADS;
-                        if (idx >= ntile) continue;
-                        const int row = idx % UNIT_ROWS, tk = idx / UNIT_ROWS;
-                        const int n = rb * UNIT_ROWS + row;
-                        slot_sum[row * 16 + tk] = 0;
-                        if (n < p.N) store_out(p, s, row, n, tk, sums[r]);
+                            for (int q = 0; q < 2 * NT; ++q) {
+                                int32_t x = 0;
+                                got = got && poll_entry(src + rows[q] * 16 + tok, P.epoch, x,
+                                                        &s.abort, P.status);
+                                v[q] += (uint32_t)x;
+                            }
+                        }
+                        if (got) {
+                            for (int c = cf + 1; c <= cl; ++c) {
+                                int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
+#pragma unroll
+                                for (int q = 0; q < 2 * NT; ++q)
+                                    st_relaxed_v2(src + rows[q] * 16 + tok, 0u, 0u);
+                            }
+#pragma unroll
+                            for (int q = 0; q < 2 * NT; ++q) {
+                                const int n = rb * UNIT_ROWS + rows[q];
+                                if (n < p.N) store_out(p, s, rows[q], n, tok, (int32_t)v[q]);
+                            }
+                        }
                     }
-                    if (threadIdx.x == 0) P.ws_count[first] = 0;
                 }
             }
-            cons_sync();  // every read of part / xpart / last / row params is done
-            // reset this parity's flag; it is used again two pieces on, after
-            // the next piece's barriers
-            if (threadIdx.x == 0) s.last[par] = 0;
+            cons_sync();  // every read of part / xpart / row params is done
             par ^= 1;
             gs = piece_end;
         }
@@ -565,6 +606,16 @@ bool encode_sw128(CUtensorMap *map, const void *base, uint64_t cols, uint64_t ro
               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
            CUDA_SUCCESS;
+}
+
+// Launch epochs: nonzero and different for consecutive launches (wraps after
+// 2^32 - 1 launches; entries are zeroed after use, so an old epoch never
+// lingers in the workspace).
+uint32_t next_epoch() {
+    static std::atomic<uint32_t> counter{0};
+    uint32_t e = counter.fetch_add(1, std::memory_order_relaxed) + 1;
+    if (e == 0) e = counter.fetch_add(1, std::memory_order_relaxed) + 1;
+    return e;
 }
 
 template <int BITS, int NT>
@@ -605,8 +656,8 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
         if (stages > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
         P.count = n;
         P.total_stages = (int)stages;
-        P.ws_count = workspace;
-        P.ws_sum = workspace + DECODE_WS_COUNTERS;
+        P.ws = reinterpret_cast<int2 *>(workspace);
+        P.epoch = next_epoch();
         P.status = device_status_ptr();
         long long grid = 2LL * sms;
         if (grid > DECODE_MAX_GRID) grid = DECODE_MAX_GRID;

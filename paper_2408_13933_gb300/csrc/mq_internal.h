@@ -32,11 +32,10 @@ struct Problem {
 constexpr int DECODE_MAX_M = 16;
 
 // Decode workspace: per CTA of the decode grid (at most DECODE_MAX_GRID) one
-// contributor counter and one 64 x 16 int32 slot of partial sums.
+// slot of 64 x 16 entries {int32 partial sum, uint32 launch epoch}, written
+// by a CTA that contributes to a 64-row unit finished by another CTA.
 constexpr int DECODE_MAX_GRID = 320;
-constexpr int DECODE_WS_COUNTERS = 384;  // counters, padded to 1536 bytes
-constexpr size_t DECODE_WS_BYTES =
-    sizeof(int32_t) * ((size_t)DECODE_WS_COUNTERS + (size_t)DECODE_MAX_GRID * 64 * 16);
+constexpr size_t DECODE_WS_BYTES = 8 * (size_t)DECODE_MAX_GRID * 64 * 16;
 
 // Problems per kernel launch (kernel parameter space).
 constexpr int PREFILL_MAX_PROBLEMS = 32;

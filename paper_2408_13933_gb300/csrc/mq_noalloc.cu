@@ -9,9 +9,9 @@
 // entry point gives them the same result as mq_linear_w4a8 without asking for
 // a workspace and without allocating one.
 //
-// The scratch is one fixed-size array per device (DECODE_WS_BYTES, about
-// 1.3 MB: the decode kernel's contributor counters plus one 64 x 16 int32 slot
-// of partial sums per CTA of its grid), so every call on a device shares it.
+// The scratch is one fixed-size array per device (DECODE_WS_BYTES, 2.5 MB:
+// per CTA of the decode grid one slot of 64 x 16 {partial sum, launch epoch}
+// entries), so every call on a device shares it.
 // Calls on that device must therefore not overlap: two calls on different
 // streams, or from different host threads, race on the scratch and give
 // wrong results.  Calls issued one after another on one stream are fine.
