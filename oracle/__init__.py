@@ -47,6 +47,9 @@ def _bind(lib):
     lib.oracle_unpack.argtypes = [p, ci, ci, ci, p]
     lib.oracle_linear.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci, p]
     lib.oracle_linear_points.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci, p, p]
+    lib.oracle_linear_asym.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, p, i32, p, ci, p]
+    lib.oracle_linear_points_asym.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, p, i32, p,
+                                              ci, p, p]
     lib.oracle_requant_one.argtypes = [i64, i32, i32, i32]
     lib.oracle_requant_one.restype = i32
     lib.oracle_residual_add.argtypes = [p, p, i64, p]
@@ -101,8 +104,10 @@ class Oracle:
         return w
 
     def linear(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
-               m0: np.ndarray, shift: np.ndarray, zy: int, want_acc: bool = False):
-        """Full integer linear layer: returns y int8 [M, N] (and acc int32 [M, N])."""
+               m0: np.ndarray, shift: np.ndarray, zy: int, want_acc: bool = False,
+               zw: np.ndarray | None = None):
+        """Full integer linear layer: returns y int8 [M, N] (and acc int32 [M, N]).
+        `zw` (int32 [N]) gives asymmetric weights (oracle_linear_asym)."""
         x = np.ascontiguousarray(x, dtype=np.int8)
         m, k = x.shape
         packed = np.ascontiguousarray(packed, dtype=np.uint8)
@@ -110,14 +115,22 @@ class Oracle:
         shift = np.ascontiguousarray(shift, dtype=np.int32)
         y = np.zeros((m, n), np.int8)
         acc = np.zeros((m, n), np.int32) if want_acc else None
-        _check(self.lib.oracle_linear(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
-                                      _ptr(m0), _ptr(shift), int(zy), _ptr(y), n,
-                                      _ptr(acc) if acc is not None else None),
-               "oracle_linear")
+        accp = _ptr(acc) if acc is not None else None
+        if zw is None:
+            _check(self.lib.oracle_linear(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
+                                          _ptr(m0), _ptr(shift), int(zy), _ptr(y), n, accp),
+                   "oracle_linear")
+        else:
+            zw = np.ascontiguousarray(zw, dtype=np.int32)
+            _check(self.lib.oracle_linear_asym(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
+                                               _ptr(zw), _ptr(m0), _ptr(shift), int(zy),
+                                               _ptr(y), n, accp),
+                   "oracle_linear_asym")
         return (y, acc) if want_acc else y
 
     def linear_points(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
-                      m0: np.ndarray, shift: np.ndarray, zy: int, pts: np.ndarray):
+                      m0: np.ndarray, shift: np.ndarray, zy: int, pts: np.ndarray,
+                      zw: np.ndarray | None = None):
         """The layer at listed (m, n) coordinates only: returns (y[i], acc[i])."""
         x = np.ascontiguousarray(x, dtype=np.int8)
         m, k = x.shape
@@ -128,10 +141,18 @@ class Oracle:
         packed = np.ascontiguousarray(packed, dtype=np.uint8)
         m0 = np.ascontiguousarray(m0, dtype=np.int32)
         shift = np.ascontiguousarray(shift, dtype=np.int32)
-        _check(self.lib.oracle_linear_points(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
-                                             _ptr(m0), _ptr(shift), int(zy), _ptr(pts), cnt,
-                                             _ptr(y), _ptr(acc)),
-               "oracle_linear_points")
+        if zw is None:
+            _check(self.lib.oracle_linear_points(_ptr(x), m, k, k, int(zx), _ptr(packed), bits,
+                                                 n, _ptr(m0), _ptr(shift), int(zy), _ptr(pts),
+                                                 cnt, _ptr(y), _ptr(acc)),
+                   "oracle_linear_points")
+        else:
+            zw = np.ascontiguousarray(zw, dtype=np.int32)
+            _check(self.lib.oracle_linear_points_asym(_ptr(x), m, k, k, int(zx), _ptr(packed),
+                                                      bits, n, _ptr(zw), _ptr(m0), _ptr(shift),
+                                                      int(zy), _ptr(pts), cnt, _ptr(y),
+                                                      _ptr(acc)),
+                   "oracle_linear_points_asym")
         return y, acc
 
     def requant_one(self, acc: int, m0: int, shift: int, zy: int) -> int:
@@ -167,12 +188,12 @@ def unpack(packed, n, k, bits):
     return _default().unpack(packed, n, k, bits)
 
 
-def linear(x, zx, packed, bits, n, m0, shift, zy, want_acc=False):
-    return _default().linear(x, zx, packed, bits, n, m0, shift, zy, want_acc)
+def linear(x, zx, packed, bits, n, m0, shift, zy, want_acc=False, zw=None):
+    return _default().linear(x, zx, packed, bits, n, m0, shift, zy, want_acc, zw)
 
 
-def linear_points(x, zx, packed, bits, n, m0, shift, zy, pts):
-    return _default().linear_points(x, zx, packed, bits, n, m0, shift, zy, pts)
+def linear_points(x, zx, packed, bits, n, m0, shift, zy, pts, zw=None):
+    return _default().linear_points(x, zx, packed, bits, n, m0, shift, zy, pts, zw)
 
 
 def requant_one(acc, m0, shift, zy):

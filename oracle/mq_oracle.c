@@ -175,6 +175,74 @@ int oracle_linear_points(const int8_t *x, int M, int K, int ldx, int32_t zx,
     return ORACLE_OK;
 }
 
+/* sum_k (x[m][k] - zx) * (w[n][k] - zw), the asymmetric-weight dot product. */
+static int64_t oracle_dot_asym(const int8_t *x, int K, int ldx, int32_t zx,
+                               const uint8_t *packed, int bits, int m, int n,
+                               int32_t zw) {
+    int64_t acc = 0;
+    for (int k = 0; k < K; ++k) {
+        int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - zx;
+        int64_t wv = oracle_weight_at(packed, bits, K, n, k) - zw;
+        acc += xv * wv;
+    }
+    return acc;
+}
+
+static int oracle_check_zw(const int32_t *zw, int N, int bits) {
+    if (!zw) return ORACLE_OK;
+    const int32_t lo = bits == 8 ? -128 : -8, hi = bits == 8 ? 127 : 7;
+    for (int n = 0; n < N; ++n)
+        if (zw[n] < lo || zw[n] > hi) return ORACLE_EINVAL;
+    return ORACLE_OK;
+}
+
+int oracle_linear_asym(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                       const uint8_t *packed, int bits, int N,
+                       const int32_t *zw, const int32_t *M0,
+                       const int32_t *shift, int32_t zy, int8_t *y, int ldy,
+                       int32_t *acc_out) {
+    int rc = oracle_check_args(M, K, ldx, bits, N, zx, zy);
+    if (rc != ORACLE_OK) return rc;
+    if (ldy < N) return ORACLE_EINVAL;
+    rc = oracle_check_zw(zw, N, bits);
+    if (rc != ORACLE_OK) return rc;
+    for (int m = 0; m < M; ++m) {
+        for (int n = 0; n < N; ++n) {
+            int64_t acc = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, zw ? zw[n] : 0);
+            if (acc >= ((int64_t)1 << 31) || acc < -((int64_t)1 << 31))
+                return ORACLE_EOVERFLOW;
+            if (acc_out) acc_out[(size_t)m * (size_t)N + (size_t)n] = (int32_t)acc;
+            if (y)
+                y[(size_t)m * (size_t)ldy + (size_t)n] =
+                    (int8_t)oracle_requant_one(acc, M0[n], shift[n], zy);
+        }
+    }
+    return ORACLE_OK;
+}
+
+int oracle_linear_points_asym(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                              const uint8_t *packed, int bits, int N,
+                              const int32_t *zw, const int32_t *M0,
+                              const int32_t *shift, int32_t zy,
+                              const int64_t *pts, int count, int8_t *y_out,
+                              int32_t *acc_out) {
+    int rc = oracle_check_args(M, K, ldx, bits, N, zx, zy);
+    if (rc != ORACLE_OK) return rc;
+    rc = oracle_check_zw(zw, N, bits);
+    if (rc != ORACLE_OK) return rc;
+    for (int i = 0; i < count; ++i) {
+        int64_t m = pts[2 * i], n = pts[2 * i + 1];
+        if (m < 0 || m >= M || n < 0 || n >= N) return ORACLE_EINVAL;
+        int64_t acc = oracle_dot_asym(x, K, ldx, zx, packed, bits, (int)m, (int)n,
+                                      zw ? zw[n] : 0);
+        if (acc >= ((int64_t)1 << 31) || acc < -((int64_t)1 << 31))
+            return ORACLE_EOVERFLOW;
+        if (acc_out) acc_out[i] = (int32_t)acc;
+        if (y_out) y_out[i] = (int8_t)oracle_requant_one(acc, M0[n], shift[n], zy);
+    }
+    return ORACLE_OK;
+}
+
 void oracle_residual_add(const int8_t *a, const int8_t *b, int64_t n,
                          int8_t *out) {
     for (int64_t i = 0; i < n; ++i) {

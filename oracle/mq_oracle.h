@@ -95,6 +95,33 @@ int oracle_linear_points(const int8_t *x, int M, int K, int ldx, int32_t zx,
                          int32_t *acc_out);
 
 /*
+ * The same layer with asymmetric weights: a per-output-channel weight zero
+ * point zw[n] (zw == NULL: all zero, i.e. oracle_linear).  The paper's main
+ * W8A8 / W4A8 runs quantize weights asymmetrically with the quantizer of
+ * Sec. 4.2, eqs. 2-4 (per tensor, and per channel for the down projection,
+ * Sec. 5.1); a per-tensor zero point is the case of equal zw[n].
+ *   acc[m][n] = sum_k (x[m][k] - zx) * (w[n][k] - zw[n])           (int64)
+ * then requantized exactly as in oracle_linear.  zw[n] must lie in the
+ * weight code range ([-128, 127] for bits 8, [-8, 7] for bits 4).
+ * Pinned by: exhaustive K=1 brute force over x and w for several zero points,
+ * the expanded identity sum(xw) - zx colsum - zw rowsum(x) + K zx zw,
+ * reduction to oracle_linear at zw = 0, exact dequantization.
+ */
+int oracle_linear_asym(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                       const uint8_t *packed, int bits, int N,
+                       const int32_t *zw, const int32_t *M0,
+                       const int32_t *shift, int32_t zy, int8_t *y, int ldy,
+                       int32_t *acc_out);
+
+/* oracle_linear_asym at listed output coordinates (as oracle_linear_points). */
+int oracle_linear_points_asym(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                              const uint8_t *packed, int bits, int N,
+                              const int32_t *zw, const int32_t *M0,
+                              const int32_t *shift, int32_t zy,
+                              const int64_t *pts, int count, int8_t *y_out,
+                              int32_t *acc_out);
+
+/*
  * Requantize one accumulator: clamp(zy + floor(acc*M0 / 2^s + 1/2), -128, 127).
  * Exposed so that tests can sweep accumulators around rounding ties.
  */

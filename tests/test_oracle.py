@@ -193,9 +193,93 @@ def pin_requant_params_bound(orc: Oracle):
         assert (int(m0[0]), int(sh[0])) == (1 << 30, 30 + t)
 
 
+# ---- asymmetric weights (per-channel weight zero point zw) ----------------
+
+def pin_asym_k1_exhaustive(orc: Oracle):
+    # every int8 x against every int8 w (K = 1) for several zero-point pairs:
+    # acc = (x - zx) (w - zw), checked against the product of Python integers
+    xs = np.arange(-128, 128, dtype=np.int16).astype(np.int8).reshape(256, 1)
+    ws = np.arange(-128, 128, dtype=np.int16).astype(np.int8).reshape(256, 1)
+    packed, _ = orc.pack(ws, 8)
+    m0 = np.full(256, 1 << 30, np.int32)
+    sh = np.full(256, 31, np.int32)
+    for zx, zw in ((-128, 127), (0, -128), (5, -3), (127, 0), (-1, 1)):
+        _, acc = orc.linear(xs, zx, packed, 8, 256, m0, sh, 0, want_acc=True,
+                            zw=np.full(256, zw, np.int32))
+        ref = np.array([[(int(a) - zx) * (int(b) - zw) for b in ws[:, 0]] for a in xs[:, 0]])
+        assert np.array_equal(acc.astype(np.int64), ref), (zx, zw)
+
+
+def pin_asym_int4_pairs(orc: Oracle):
+    # every pair of int4 weights (K = 2), every int4 weight zero point
+    ws = np.array([[a, b] for a in range(-8, 8) for b in range(-8, 8)], np.int8)
+    xs = np.array([[a, b] for a in (-128, -9, 0, 3, 127) for b in (-128, 0, 77, 127)], np.int8)
+    packed, _ = orc.pack(ws, 4)
+    m0 = np.full(ws.shape[0], 1 << 30, np.int32)
+    sh = np.full(ws.shape[0], 31, np.int32)
+    for zw in range(-8, 8):
+        for zx in (-128, 0, 127):
+            _, acc = orc.linear(xs, zx, packed, 4, ws.shape[0], m0, sh, 0, want_acc=True,
+                                zw=np.full(ws.shape[0], zw, np.int32))
+            ref = (xs.astype(np.int64) - zx) @ (ws.astype(np.int64) - zw).T
+            assert np.array_equal(acc.astype(np.int64), ref), (zw, zx)
+
+
+def pin_asym_identity(orc: Oracle, seeds=(4, 5)):
+    # sum((x - zx)(w - zw)) = sum(x w) - zx colsum(w) - zw rowsum(x) + K zx zw,
+    # with per-channel zw spanning the code range
+    for seed in seeds:
+        rng = np.random.default_rng(seed)
+        for bits in (8, 4):
+            lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+            for extreme in (None, "min", "max", "mixed"):
+                c = synth.random_case(seed, 6, 96, 11, bits, extreme)
+                zw = rng.integers(lo, hi + 1, size=c.N).astype(np.int32)
+                zw[0], zw[-1] = lo, hi
+                packed, colsum = orc.pack(c.w, bits)
+                m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+                _, acc = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True,
+                                    zw=zw)
+                x64, w64 = c.x.astype(np.int64), c.w.astype(np.int64)
+                ref = (x64 @ w64.T - c.zx * w64.sum(1)[None, :]
+                       - zw.astype(np.int64)[None, :] * x64.sum(1)[:, None]
+                       + c.K * c.zx * zw.astype(np.int64)[None, :])
+                assert np.array_equal(acc.astype(np.int64), ref), (seed, bits, extreme)
+
+
+def pin_asym_reduces_to_symmetric(orc: Oracle):
+    for bits in (8, 4):
+        c = synth.random_case(6, 5, 64, 9, bits, "mixed")
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+        y0, a0 = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True)
+        y1, a1 = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True,
+                            zw=np.zeros(c.N, np.int32))
+        assert np.array_equal(a0, a1) and np.array_equal(y0, y1)
+
+
+def pin_asym_exact_dequant(orc: Oracle):
+    # power-of-two scales: the float64 matmul of the dequantized operands
+    # s_x (x - zx) and s_w (w - zw) is exact and equals acc s_x s_w
+    rng = np.random.default_rng(8)
+    for bits in (8, 4):
+        lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+        c = synth.random_case(12, 9, 160, 17, bits)
+        zw = rng.integers(lo, hi + 1, size=c.N).astype(np.int32)
+        sx = 2.0 ** -6
+        sw = 2.0 ** -rng.integers(3, 12, size=c.N).astype(np.float64)
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(1.0, np.ones(c.N, np.float32), 1.0)
+        _, acc = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, 0, want_acc=True, zw=zw)
+        xd = (c.x.astype(np.float64) - c.zx) * sx
+        wd = (c.w.astype(np.float64) - zw[:, None]) * sw[:, None]
+        assert np.array_equal(xd @ wd.T, acc.astype(np.float64) * sx * sw[None, :])
+
+
 PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zero_point_identity,
                pin_exact_dequant, pin_requant_closed_form, pin_requant_ties, pin_requant_vs_eq4,
-               pin_requant_params_bound]
+               pin_requant_params_bound, pin_asym_k1_exhaustive, pin_asym_int4_pairs,
+               pin_asym_identity, pin_asym_reduces_to_symmetric, pin_asym_exact_dequant]
 
 
 # ----------------------------------------------------------------------------
@@ -308,6 +392,34 @@ def test_accumulator_overflow_detected(O):
                 O.linear(x, 127, packed, 8, 1, m0, sh, 0)
 
 
+def test_asym_k1_exhaustive(O):
+    pin_asym_k1_exhaustive(O)
+
+
+def test_asym_int4_pairs(O):
+    pin_asym_int4_pairs(O)
+
+
+def test_asym_identity(O):
+    pin_asym_identity(O)
+
+
+def test_asym_reduces_to_symmetric(O):
+    pin_asym_reduces_to_symmetric(O)
+
+
+def test_asym_exact_dequant(O):
+    pin_asym_exact_dequant(O)
+
+
+def test_asym_rejects_zero_point_out_of_range(O):
+    c = synth.random_case(3, 2, 32, 4, 4)
+    packed, _ = O.pack(c.w, 4)
+    m0, sh = O.requant_params(c.sx, c.sw, c.sy)
+    with pytest.raises(oracle.OracleError):
+        O.linear(c.x, c.zx, packed, 4, c.N, m0, sh, c.zy, zw=np.array([0, 8, 0, 0], np.int32))
+
+
 def test_linear_points_agree_with_full(O):
     c = synth.random_case(21, 11, 64, 19, 4)
     packed, _ = O.pack(c.w, 4)
@@ -345,6 +457,10 @@ MUTATIONS = [
     ("colsum of first row only", "if (colsum) colsum[n] = (int32_t)sum;",
      "if (colsum) colsum[n] = (int32_t)(n == 0 ? sum : 0);"),
     ("saturation bound", "if (out > 127) out = 127;", "if (out > 126) out = 126;"),
+    ("weight zero point sign", "int64_t wv = oracle_weight_at(packed, bits, K, n, k) - zw;",
+     "int64_t wv = oracle_weight_at(packed, bits, K, n, k) + zw;"),
+    ("weight zero point ignored", "int64_t acc = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, zw ? zw[n] : 0);",
+     "int64_t acc = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, 0);"),
 ]
 
 
