@@ -193,8 +193,22 @@ int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, int32_t zx,
  * addition `residual` (device int8 [M][ldy], may be NULL) is added to the
  * requantized output with int8 saturation, the int8 residual glue between
  * chained layers.  Descriptors must not write overlapping outputs.
- *   descs : host array of `count` descriptors (1 <= count <= MQ_MAX_BATCH)
- * Errors: as the single calls; the index of the first bad descriptor is not
+ *
+ * Asymmetric weights: `zw` (device int32 [N], may be NULL for symmetric
+ * weights) is a per-output-channel weight zero point, the asymmetric weight
+ * quantizer of the paper's main W8A8 / W4A8 runs (Sec. 4.2 eqs. 2-4 applied
+ * to weights, Sec. 5.1; a per-tensor zero point is the case of equal zw[n]):
+ *   acc[m][n] = sum_k (x[m][k] - zx) * (w[n][k] - zw[n])
+ *             = sum_k x w - zx colsum[n] - zw[n] rowsum(x)[m] + K zx zw[n]
+ * zw[n] must lie in the weight code range ([-128, 127] for bits 8, [-8, 7]
+ * for bits 4), and with int8 weights K <= MQ_MAX_K_ASYM8 (so that
+ * |acc| <= 255 * 255 * K stays below 2^31).  Descriptors with M > 16 and zw
+ * need workspace for rowsum(x): see mq_workspace_size_batch.
+ *
+ *   descs     : host array of `count` descriptors (1 <= count <= MQ_MAX_BATCH)
+ *   workspace : device, ws_bytes >= mq_workspace_size_batch(descs, count)
+ * Errors: as the single calls, and MQ_ERR_K_OVERFLOW for int8 weights with
+ * zw and K > MQ_MAX_K_ASYM8; the index of the first bad descriptor is not
  * reported, nothing is launched when any descriptor is invalid.
  */
 typedef struct mq_linear_desc {
@@ -204,11 +218,26 @@ typedef struct mq_linear_desc {
     const int32_t *M0;
     const int32_t *shift;
     const int8_t *residual; /* may be NULL */
+    const int32_t *zw;      /* may be NULL: symmetric weights */
     int8_t *y;
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;
     int32_t bits; /* 8 or 4 */
 } mq_linear_desc;
+
+/* Largest K for int8 weights with a weight zero point: 255 * 255 * K < 2^31. */
+#define MQ_MAX_K_ASYM8 32768
+
+/*
+ * Device workspace bytes one mq_linear_batch call over `descs` needs: the
+ * decode workspace (see mq_workspace_size) if any descriptor has
+ * 1 <= M <= 16, plus 4*M bytes (rounded up to 16) for every descriptor with
+ * M > 16 and a weight zero point, which holds rowsum(x) of its tokens (filled
+ * by the call).  0 when neither applies.  The contract of mq_workspace_size
+ * holds for the whole buffer.
+ * Errors: MQ_ERR_INVALID_ARG (null pointers, count out of range, bad bits).
+ */
+int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *bytes);
 
 int mq_linear_batch(const mq_linear_desc *descs, int count, void *workspace,
                     size_t ws_bytes, void *stream);

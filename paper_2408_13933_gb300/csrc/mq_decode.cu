@@ -92,6 +92,39 @@ struct Params {
     int *status;
 };
 
+// What the kernel reads of a problem, kept in shared memory (the TMA tensor
+// maps replace x and the weights).
+struct DecProb {
+    const int32_t *colsum;
+    const int32_t *M0;
+    const int32_t *shift;
+    const int8_t *residual;
+    const int32_t *zw;
+    int8_t *y;
+    int32_t M, N, K, ldy, zx, zy;
+    int32_t tile_begin;  // first global stage
+    int32_t tiles_m;     // stages per unit
+};
+
+__device__ __forceinline__ DecProb dec_prob(const Problem &p) {
+    DecProb d;
+    d.colsum = p.colsum;
+    d.M0 = p.M0;
+    d.shift = p.shift;
+    d.residual = p.residual;
+    d.zw = p.zw;
+    d.y = p.y;
+    d.M = p.M;
+    d.N = p.N;
+    d.K = p.K;
+    d.ldy = p.ldy;
+    d.zx = p.zx;
+    d.zy = p.zy;
+    d.tile_begin = p.tile_begin;
+    d.tiles_m = p.tiles_m;
+    return d;
+}
+
 template <int NT>
 struct Smem {
     static constexpr int STAGES = stages_for<NT>();
@@ -102,10 +135,11 @@ struct Smem {
     // element e = (rt * NT + nt) * 4 + i and lane (conflict-free both ways)
     int32_t part[CONS_WARPS][16 * NT][32];
     int32_t xpart[CONS_WARPS][16];  // each warp's activation sums per token
-    int32_t row_corr[UNIT_ROWS];  // zx * colsum[n] of the current unit's rows
+    int32_t row_corr[UNIT_ROWS];  // zx * colsum[n] - K zx zw[n] of the current unit's rows
+    int32_t row_zw[UNIT_ROWS];    // weight zero points of the current unit's rows
     int32_t row_m0[UNIT_ROWS];
     int32_t row_shift[UNIT_ROWS];
-    Problem prob[DECODE_MAX_PROBLEMS];  // the kernel's problem table, read once
+    DecProb prob[DECODE_MAX_PROBLEMS];  // the kernel's problem table, read once
     int abort;
 };
 
@@ -216,7 +250,7 @@ __device__ __forceinline__ bool poll_entry(const int2 *p, uint32_t epoch, int32_
 // sum(w x): acc = sum(w x) - zx colsum[n], fixed point, saturate, optional
 // residual.
 template <class SM>
-__device__ __forceinline__ void store_out(const Problem &p, const SM &sm, int row, int n,
+__device__ __forceinline__ void store_out(const DecProb &p, const SM &sm, int row, int n,
                                           int tok, int32_t sum_wx) {
     // two's-complement wrap is exact: the true value fits in int32
     const int32_t a = (int32_t)((uint32_t)sum_wx - (uint32_t)sm.row_corr[row]);
@@ -337,7 +371,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
         s.abort = 0;
         fence_mbar_init();
     }
-    for (int i = threadIdx.x; i < P.count; i += THREADS) s.prob[i] = P.p[i];
+    for (int i = threadIdx.x; i < P.count; i += THREADS) s.prob[i] = dec_prob(P.p[i]);
     __syncthreads();
     if (threadIdx.x == 0) griddep_launch_dependents();
     const int count = P.count;
@@ -359,7 +393,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             for (int i = 0; i < npre; ++i) {
                 const int gs = s_begin + i;
                 pi = problem_from(s, count, pi, gs);
-                const Problem &p = s.prob[pi];
+                const DecProb &p = s.prob[pi];
                 if (p.K == 0) continue;
                 const int local = gs - p.tile_begin;
                 const int rb = local / p.tiles_m, j = local % p.tiles_m;
@@ -371,7 +405,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             pi = 0;
             for (int gs = s_begin; gs < s_end; ++gs, ++it) {
                 pi = problem_from(s, count, pi, gs);
-                const Problem &p = s.prob[pi];
+                const DecProb &p = s.prob[pi];
                 const int local = gs - p.tile_begin;
                 const int rb = local / p.tiles_m, j = local % p.tiles_m;
                 const int slot = it % STAGES;
@@ -405,7 +439,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
         while (gs < s_end) {
             // the piece [gs, piece_end) of one unit that this CTA owns
             pi = problem_from(s, count, pi, gs);
-            const Problem &p = s.prob[pi];
+            const DecProb &p = s.prob[pi];
             const int nst = p.tiles_m;
             const int local = gs - p.tile_begin;
             const int rb = local / nst;
@@ -414,13 +448,14 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             // requant parameters of the unit's rows: loaded now, published to
             // shared memory when the piece is done, so the loads overlap the
             // stage loop instead of stalling the warp here
-            int32_t prm_cs = 0, prm_m0 = 0, prm_sh = 33;
+            int32_t prm_cs = 0, prm_m0 = 0, prm_sh = 33, prm_zw = 0;
             if (threadIdx.x < UNIT_ROWS) {
                 const int n = rb * UNIT_ROWS + threadIdx.x;
                 if (n < p.N) {
                     prm_cs = __ldg(p.colsum + n);
                     prm_m0 = __ldg(p.M0 + n);
                     prm_sh = __ldg(p.shift + n);
+                    if (p.zw) prm_zw = __ldg(p.zw + n);
                 }
             }
             float acc[4][NT][4];
@@ -488,7 +523,11 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                 }
             }
             if (threadIdx.x < UNIT_ROWS) {
-                s.row_corr[threadIdx.x] = p.zx * prm_cs;
+                // sum((x - zx)(w - zw)) = sum(x w) - zx colsum - zw sum(x) + K zx zw;
+                // the zw sum(x) term is taken per piece with the bias below
+                s.row_corr[threadIdx.x] =
+                    (int32_t)((uint32_t)(p.zx * prm_cs) - (uint32_t)p.K * (uint32_t)(p.zx * prm_zw));
+                s.row_zw[threadIdx.x] = prm_zw;
                 s.row_m0[threadIdx.x] = prm_m0;
                 s.row_shift[threadIdx.x] = prm_sh;
             }
@@ -514,9 +553,10 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     int32_t sum = 0;
 #pragma unroll
                     for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
-                    // sum(w x) = sum(u x) - bias * sum(x)
+                    // sum((x - zx)(w - zw)) = sum(u x) - (bias + zw) sum(x) - corr
                     store_out(p, s, row, n, tok,
-                              (int32_t)((uint32_t)sum - (uint32_t)(C::BIAS * xsum)));
+                              (int32_t)((uint32_t)sum -
+                                        (uint32_t)((C::BIAS + s.row_zw[row]) * xsum)));
                 }
             } else if (ok) {
                 // A split unit.  Its first CTA finishes it: that CTA reaches the
@@ -537,7 +577,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                         int32_t sum = 0;
 #pragma unroll
                         for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
-                        v[q] = (uint32_t)sum - (uint32_t)(C::BIAS * xsum);
+                        v[q] = (uint32_t)sum - (uint32_t)((C::BIAS + s.row_zw[rows[q]]) * xsum);
                     }
                     if (cta != cf) {
                         int2 *mine = P.ws + (size_t)cta * UNIT_ROWS * 16;

@@ -20,6 +20,7 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     if (d.M < 0 || d.N < 0 || d.K < 0) return MQ_ERR_INVALID_ARG;
     if (d.zx < -128 || d.zx > 127 || d.zy < -128 || d.zy > 127) return MQ_ERR_INVALID_ARG;
     if (d.K > MQ_MAX_K) return MQ_ERR_K_OVERFLOW;
+    if (d.zw && d.bits == 8 && d.K > MQ_MAX_K_ASYM8) return MQ_ERR_K_OVERFLOW;
     if (d.M > 0 && d.N > 0) {
         if (!d.colsum || !d.M0 || !d.shift || !d.y || d.ldy < d.N) return MQ_ERR_INVALID_ARG;
         if (d.K > 0) {  // with K == 0 neither x nor the weights are read
@@ -35,6 +36,8 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     out.M0 = d.M0;
     out.shift = d.shift;
     out.residual = d.residual;
+    out.zw = d.zw;
+    out.rowsum = nullptr;
     out.y = d.y;
     out.M = d.M;
     out.N = d.N;
@@ -47,6 +50,26 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     out.tile_begin = 0;
     out.tiles_m = 0;
     return MQ_OK;
+}
+
+size_t align16(size_t v) { return (v + 15) & ~static_cast<size_t>(15); }
+
+// Workspace layout of one batch: the decode region first (if any decode
+// shape), then rowsum(x) of every prefill descriptor with a weight zero
+// point, in descriptor order.
+size_t batch_workspace(const mq_linear_desc *descs, int count, bool *any_decode) {
+    bool dec = false;
+    size_t rows = 0;
+    for (int i = 0; i < count; ++i) {
+        const mq_linear_desc &d = descs[i];
+        if (d.M <= 0 || d.N <= 0) continue;
+        if (d.M <= mq::DECODE_MAX_M)
+            dec = true;
+        else if (d.zw && d.K > 0)
+            rows += align16(4 * (size_t)d.M);
+    }
+    if (any_decode) *any_decode = dec;
+    return (dec ? mq::DECODE_WS_BYTES : 0) + rows;
 }
 
 int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws_bytes,
@@ -64,13 +87,23 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         else
             pre.push_back(p);
     }
-    // the decode kernel combines split 64-row units in the caller's workspace
-    if (!dec8.empty() || !dec4.empty()) {
-        if (!workspace || ws_bytes < mq::DECODE_WS_BYTES || !aligned16(workspace))
-            return MQ_ERR_WORKSPACE;
+    // the decode kernel combines split 64-row units in the workspace; prefill
+    // descriptors with a weight zero point keep rowsum(x) there
+    bool any_decode = false;
+    const size_t need = batch_workspace(descs, count, &any_decode);
+    if (need > 0 && (!workspace || ws_bytes < need || !aligned16(workspace)))
+        return MQ_ERR_WORKSPACE;
+    size_t off = any_decode ? mq::DECODE_WS_BYTES : 0;
+    bool any_rowsum = false;
+    for (auto &p : pre) {
+        if (!p.zw || p.K == 0) continue;
+        p.rowsum = reinterpret_cast<const int32_t *>(static_cast<uint8_t *>(workspace) + off);
+        off += align16(4 * (size_t)p.M);
+        any_rowsum = true;
     }
     int rc = MQ_OK;
-    if (!pre.empty()) rc = mq::launch_prefill(pre.data(), (int)pre.size(), stream);
+    if (any_rowsum) rc = mq::launch_rowsum(pre.data(), (int)pre.size(), stream);
+    if (rc == MQ_OK && !pre.empty()) rc = mq::launch_prefill(pre.data(), (int)pre.size(), stream);
     if (rc == MQ_OK && !dec8.empty())
         rc = mq::launch_decode(dec8.data(), (int)dec8.size(), workspace, stream);
     if (rc == MQ_OK && !dec4.empty())
@@ -88,6 +121,7 @@ int single(int bits, const int8_t *x, int M, int K, int ldx, int32_t zx, const v
     d.M0 = M0;
     d.shift = shift;
     d.residual = nullptr;
+    d.zw = nullptr;
     d.y = y;
     d.M = M;
     d.N = N;
@@ -232,6 +266,14 @@ int mq_linear_w4a8(const int8_t *x, int M, int K, int ldx, int32_t zx, const voi
                    void *stream) {
     return single(4, x, M, K, ldx, zx, packed, colsum, N, M0, shift, zy, y, ldy, workspace,
                   ws_bytes, stream);
+}
+
+int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *bytes) {
+    if (!descs || !bytes || count < 1 || count > MQ_MAX_BATCH) return MQ_ERR_INVALID_ARG;
+    for (int i = 0; i < count; ++i)
+        if (descs[i].bits != 8 && descs[i].bits != 4) return MQ_ERR_INVALID_ARG;
+    *bytes = batch_workspace(descs, count, nullptr);
+    return MQ_OK;
 }
 
 int mq_linear_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws_bytes,

@@ -20,6 +20,8 @@ struct Problem {
     const int32_t *M0;
     const int32_t *shift;
     const int8_t *residual;
+    const int32_t *zw;      // per-channel weight zero point, or null
+    const int32_t *rowsum;  // prefill with zw: rowsum(x) [M] in the workspace
     int8_t *y;
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;
@@ -52,5 +54,7 @@ int launch_prefill(const Problem *probs, int count, void *stream);
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream);
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
                 int *status, void *stream);
+// rowsum(x)[m] = sum_k x[m][k] of every problem with a rowsum pointer.
+int launch_rowsum(const Problem *probs, int count, void *stream);
 
 }  // namespace mq

@@ -89,4 +89,44 @@ int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *
     return cudaGetLastError() == cudaSuccess ? MQ_OK : MQ_ERR_CUDA;
 }
 
+namespace rowsum {
+
+constexpr int ROWS_PER_BLOCK = 8;  // one warp per row
+
+// rowsum[m] = sum_k x[m][k]; K and ldx are multiples of 16 and x is 16-byte
+// aligned (the library's validation), so every load is a whole uint4.
+__global__ void __launch_bounds__(ROWS_PER_BLOCK * 32)
+    rowsum_kernel(const int8_t *__restrict__ x, int M, int K, int ldx, int32_t *__restrict__ out) {
+    const int row = blockIdx.x * ROWS_PER_BLOCK + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= M) return;
+    const int8_t *r = x + (size_t)row * (size_t)ldx;
+    int acc = 0;
+    for (int k = lane * 16; k < K; k += 32 * 16) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(r + k));
+        acc = __dp4a((int)v.x, 0x01010101, acc);
+        acc = __dp4a((int)v.y, 0x01010101, acc);
+        acc = __dp4a((int)v.z, 0x01010101, acc);
+        acc = __dp4a((int)v.w, 0x01010101, acc);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) out[row] = acc;
+}
+
+}  // namespace rowsum
+
+int launch_rowsum(const Problem *probs, int count, void *stream) {
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    for (int i = 0; i < count; ++i) {
+        const Problem &p = probs[i];
+        if (!p.rowsum || p.M <= 0) continue;
+        const int blocks = (p.M + rowsum::ROWS_PER_BLOCK - 1) / rowsum::ROWS_PER_BLOCK;
+        rowsum::rowsum_kernel<<<blocks, rowsum::ROWS_PER_BLOCK * 32, 0, s>>>(
+            p.x, p.M, p.K, p.ldx, const_cast<int32_t *>(p.rowsum));
+        if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
+    }
+    return MQ_OK;
+}
+
 }  // namespace mq

@@ -490,7 +490,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const Problem &p = P.p[t.pi];
             const int ch = t.ct * TM + (int)rank * CM + quad * 32 + lane;
             const bool ch_in = ch < p.N;
-            const int32_t corr = ch_in ? p.zx * __ldg(p.colsum + ch) : 0;
+            const int32_t zw = (ch_in && p.zw) ? __ldg(p.zw + ch) : 0;
+            // sum((x - zx)(w - zw)) = sum(x w) - zx colsum - zw rowsum(x) + K zx zw
+            const int32_t corr =
+                ch_in ? (int32_t)((uint32_t)(p.zx * __ldg(p.colsum + ch)) -
+                                  (uint32_t)p.K * (uint32_t)(p.zx * zw))
+                      : 0;
             const int32_t m0 = ch_in ? __ldg(p.M0 + ch) : 0;
             const int32_t sh = ch_in ? __ldg(p.shift + ch) : 33;
             uint32_t acc[64];
@@ -522,6 +527,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const EpiArgs e{p.y, p.residual, p.M, p.ldy, p.zy};
             const int tok0 = t.tt * TN + 64 * half;
             const int ntok = min(64, e.M - tok0);
+            if (p.zw && ntok > 0) {
+                // the weight zero point's term: - zw rowsum(x)[token]
+                const int32_t *rs = p.rowsum + tok0;
+                if (ntok == 64) {
+#pragma unroll
+                    for (int j = 0; j < 64; j += 4) {
+                        const int4 v = __ldg(reinterpret_cast<const int4 *>(rs + j));
+                        acc[j + 0] -= (uint32_t)(zw * v.x);
+                        acc[j + 1] -= (uint32_t)(zw * v.y);
+                        acc[j + 2] -= (uint32_t)(zw * v.z);
+                        acc[j + 3] -= (uint32_t)(zw * v.w);
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 64; ++j)
+                        if (j < ntok) acc[j] -= (uint32_t)(zw * __ldg(rs + j));
+                }
+            }
             const size_t ldy = (size_t)e.ldy;
             int8_t *yp = e.y + (size_t)tok0 * ldy + ch;
             const int8_t *rp = e.residual ? e.residual + (size_t)tok0 * ldy + ch : nullptr;

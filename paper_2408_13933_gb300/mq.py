@@ -33,11 +33,12 @@ MQ_ERR_CUDA = 5
 MQ_ERR_DEVICE_TIMEOUT = 6
 MQ_ERR_WORKSPACE = 7
 MQ_MAX_K = 65536
+MQ_MAX_K_ASYM8 = 32768
 MQ_MAX_BATCH = 256
 
 EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_weights",
             "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
-            "mq_check_device_status", "mq_linear_w4a8_noalloc"]
+            "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch"]
 
 _vp, _i32, _int, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int, ctypes.c_size_t
 
@@ -45,7 +46,7 @@ _vp, _i32, _int, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int, ctypes.c_s
 class LinearDesc(ctypes.Structure):
     """Mirror of mq_linear_desc."""
     _fields_ = [("x", _vp), ("packed", _vp), ("colsum", _vp), ("M0", _vp), ("shift", _vp),
-                ("residual", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
+                ("residual", _vp), ("zw", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
                 ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32)]
 
 
@@ -62,6 +63,7 @@ lib.mq_linear_w4a8.argtypes = _linear_args
 lib.mq_linear_w4a8_noalloc.argtypes = [_vp, _int, _int, _int, _i32, _vp, _vp, _int, _vp, _vp, _i32,
                                        _vp, _int, _vp]
 lib.mq_linear_batch.argtypes = [ctypes.POINTER(LinearDesc), _int, _vp, _sz, _vp]
+lib.mq_workspace_size_batch.argtypes = [ctypes.POINTER(LinearDesc), _int, ctypes.POINTER(_sz)]
 lib.mq_check_device_status.argtypes = [_vp]
 for _f in EXPORTED:
     if _f != "mq_status_string":
@@ -182,10 +184,12 @@ def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, 
 
 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
-              ldx=None, ldy=None, m=None, k=None) -> LinearDesc:
+              ldx=None, ldy=None, m=None, k=None, zw=None) -> LinearDesc:
+    """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights."""
     d = LinearDesc()
     d.x, d.packed, d.colsum = _ptr(x), _ptr(packed), _ptr(colsum)
     d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
+    d.zw = _ptr(zw)
     d.M = x.shape[0] if m is None else m
     d.K = x.shape[1] if k is None else k
     d.N = n
@@ -193,6 +197,15 @@ def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
     d.ldy = y.stride(0) if ldy is None else ldy
     d.zx, d.zy, d.bits = int(zx), int(zy), int(bits)
     return d
+
+
+def workspace_size_batch(descs) -> int:
+    """mq_workspace_size_batch over a list of LinearDesc."""
+    arr = (LinearDesc * len(descs))(*descs)
+    out = _sz(0)
+    _check(lib.mq_workspace_size_batch(arr, len(descs), ctypes.byref(out)),
+           "mq_workspace_size_batch")
+    return out.value
 
 
 def linear_batch(descs, stream=None, workspace=None, ws_bytes: int | None = None) -> int:

@@ -155,3 +155,32 @@ def test_empty_problems_launch_nothing(mq):
     # M == 0 or N == 0 is valid and returns without touching the device
     assert _call(mq, M=0) == 0
     assert _call(mq, N=0) == 0
+
+
+def _desc(mq, M, K, N, bits, zw):
+    d = mq.LinearDesc()
+    d.x = d.packed = d.colsum = d.M0 = d.shift = d.y = FAKE
+    d.zw = FAKE if zw else None
+    d.M, d.K, d.N, d.ldx, d.ldy, d.bits = M, K, N, K, N, bits
+    return d
+
+
+def test_asym_int8_k_limit_and_workspace(mq):
+    # int8 weights with a weight zero point: K <= MQ_MAX_K_ASYM8, checked
+    # before anything is launched; int4 keeps MQ_MAX_K
+    k = mq.MQ_MAX_K_ASYM8 + 16
+    bad = (mq.LinearDesc * 1)(_desc(mq, 64, k, 32, 8, True))
+    assert mq.lib.mq_linear_batch(bad, 1, None, 0, None) == mq.MQ_ERR_K_OVERFLOW
+    ok4 = _desc(mq, 64, k, 32, 4, True)
+    assert mq.workspace_size_batch([ok4]) == 4 * 64
+    # workspace of a batch: decode region + 16-byte-rounded rowsum regions of
+    # the asymmetric prefill descriptors; symmetric prefill needs none
+    dec = mq.workspace_size(8, 32, 64, 4)
+    assert mq.workspace_size_batch([_desc(mq, 100, 64, 32, 8, False)]) == 0
+    assert mq.workspace_size_batch([_desc(mq, 100, 64, 32, 8, True)]) == 400
+    assert mq.workspace_size_batch([_desc(mq, 101, 64, 32, 8, True),
+                                    _desc(mq, 8, 64, 32, 4, True)]) == dec + 416
+    assert mq.workspace_size_batch([_desc(mq, 8, 64, 32, 4, False)]) == dec
+    # an asymmetric prefill batch without its workspace is rejected up front
+    one = (mq.LinearDesc * 1)(_desc(mq, 100, 64, 32, 8, True))
+    assert mq.lib.mq_linear_batch(one, 1, None, 0, None) == mq.MQ_ERR_WORKSPACE
