@@ -12,7 +12,9 @@ kernel.  Steps rotate over three layers' weights and activations (216 MB,
 more than the 129 MB L2), so no step reads another's data from L2.
 
 Reported beside it, measured in the same run: W4A8 decode of the same block's
-linears at M = 1, 4, 16 (weight GB/s), rotating over 12 layers (264 MB).
+linears at M = 1, 4, 16 (weight GB/s), rotating over 12 layers (264 MB); and
+both with asymmetric weights in the paper's settings (W8A8 per tensor with a
+per-channel down projection; W4A8 per channel).
 
 Multi-GPU (torchrun, one rank per GPU): replicas only -- every rank runs the
 same workload on its own GPU, no collective on the data path; value is the
@@ -176,10 +178,12 @@ class ClockSampler:
 
 # --------------------------------------------------------------------------- workload
 class PrefillBlock:
-    """Device-resident operands of one layer's seven W8A8 linears at M tokens."""
+    """Device-resident operands of one layer's seven W8A8 linears at M tokens
+    (with asym, asymmetric weights in the paper's W8A8 setting)."""
 
-    def __init__(self, mq, torch, layer: int, m: int):
-        self.cases = synth.block_linears(CONFIG_ID_PREFILL, m, 8, layer=layer, shared_input=True)
+    def __init__(self, mq, torch, layer: int, m: int, asym: bool = False):
+        self.cases = synth.block_linears(CONFIG_ID_PREFILL, m, 8, layer=layer, shared_input=True,
+                                         asym=asym)
         down = self.cases[-1]
         down.residual = synth.residual_codes(CONFIG_ID_PREFILL, layer, m, down.N)
         dev = "cuda"
@@ -199,11 +203,16 @@ class PrefillBlock:
             t = [torch.from_numpy(a).to(dev) for a in (packed, colsum, m0, sh)]
             y = torch.empty((m, c.N), dtype=torch.int8, device=dev)
             res = torch.from_numpy(c.residual).to(dev) if c.residual is not None else None
-            self.keep += t + ([res] if res is not None else [])
+            zw = torch.from_numpy(c.zw).to(dev) if c.zw is not None else None
+            self.keep += t + [a for a in (res, zw) if a is not None]
             self.y.append(y)
             self.descs.append(mq.make_desc(self.x_dev[id(c.x)], c.zx, t[0], t[1], c.N, t[2], t[3],
-                                           c.zy, y, 8, residual=res))
+                                           c.zy, y, 8, residual=res, zw=zw))
         self.arr = (mq.LinearDesc * len(self.descs))(*self.descs)
+        # asymmetric weights: rowsum(x) of each distinct input lives in the workspace
+        self.ws_bytes = mq.workspace_size_batch(self.descs)
+        self.ws = torch.zeros(max(16, self.ws_bytes), dtype=torch.uint8, device=dev)
+        self.wsp = self.ws.data_ptr() if self.ws_bytes else None
         self.y_host = [torch.empty(y.shape, dtype=torch.int8).pin_memory() for y in self.y]
         self.h2d_bytes = sum(v.numel() for v in self.x_host.values())
         self.d2h_bytes = sum(y.numel() for y in self.y)
@@ -213,23 +222,24 @@ class DecodeLayer:
     """One layer's seven W4A8 linears, uploaded once; descriptors for each
     decode width M use the first M rows of a 16-row seeded input."""
 
-    def __init__(self, mq, torch, layer: int):
-        cases = synth.block_linears(CONFIG_ID_DECODE, max(DECODE_MS), 4, layer=layer)
+    def __init__(self, mq, torch, layer: int, asym: bool = False, ms=DECODE_MS):
+        cases = synth.block_linears(CONFIG_ID_DECODE, max(ms), 4, layer=layer, asym=asym)
         self.arr, self.keep = {}, []
         dev = []
         for c in cases:
             packed, colsum = mq.pack_weights(c.w, 4)
             m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
             t = [torch.from_numpy(a).cuda() for a in (c.x, packed, colsum, m0, sh)]
-            self.keep += t
+            t.append(torch.from_numpy(c.zw).cuda() if c.zw is not None else None)
+            self.keep += [a for a in t if a is not None]
             dev.append((c, t))
-        for m in DECODE_MS:
+        for m in ms:
             descs = []
             for c, t in dev:
                 y = torch.empty((m, c.N), dtype=torch.int8, device="cuda")
                 self.keep.append(y)
                 descs.append(mq.make_desc(t[0], c.zx, t[1], t[2], c.N, t[3], t[4], c.zy, y, 4,
-                                          m=m))
+                                          m=m, zw=t[5]))
             self.arr[m] = (mq.LinearDesc * len(descs))(*descs)
         self.count = len(cases)
 
@@ -242,7 +252,7 @@ def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
 
     def step(i):
         b = blocks[i % len(blocks)]
-        rc = call(b.arr, len(b.descs), None, 0, sp)
+        rc = call(b.arr, len(b.descs), b.wsp, b.ws_bytes, sp)
         if rc:
             raise RuntimeError(f"mq_linear_batch failed: {mq.status_string(rc)}")
 
@@ -301,21 +311,22 @@ def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
     }
 
 
-def run_decode(mq, torch, steps_per_m: int = 240):
+def run_decode(mq, torch, steps_per_m: int = 240, asym: bool = False, ms=DECODE_MS):
     """Weight GB/s of the W4A8 block linears at M = 1, 4, 16 (one batched
     launch per layer, 12 layers in rotation), timed with CUDA events per launch
-    (kernel) and over a captured CUDA graph of back-to-back launches (stream)."""
+    (kernel) and over a captured CUDA graph of back-to-back launches (stream).
+    With asym, the weights are asymmetric per channel (the paper's W4A8)."""
     out = {}
     wbytes = block_weight_bytes(4)
     stream = torch.cuda.current_stream()
-    layers = [DecodeLayer(mq, torch, layer) for layer in range(DECODE_LAYERS)]
+    layers = [DecodeLayer(mq, torch, layer, asym, ms) for layer in range(DECODE_LAYERS)]
     ws = mq.workspace()
     wsp, wsn = ws.data_ptr(), ws.numel()
 
     def call(arr, count, _ws, _n, strm):
         return mq.lib.mq_linear_batch(arr, count, wsp, wsn, strm)
     sp = stream.cuda_stream
-    for m in DECODE_MS:
+    for m in ms:
         for L in layers * 2:
             assert call(L.arr[m], L.count, None, 0, sp) == 0
         torch.cuda.synchronize()
@@ -352,6 +363,57 @@ def run_decode(mq, torch, steps_per_m: int = 240):
                         "stream_us": round(gms * 1e3, 2), "stream_gbs": round(wbytes / gms / 1e6, 1)}
         del g
     return out
+
+
+def run_asym_prefill(mq, torch, steps: int = 900, check_rows: int = 4):
+    """The same block with asymmetric weights in the paper's W8A8 setting (per
+    tensor, down per channel): int8 TOPS over `steps` back-to-back batched
+    calls (rowsum pre-pass + prefill kernel each), rotating over three layers,
+    and the first `check_rows` token rows of layer 0 checked against the oracle."""
+    blocks = [PrefillBlock(mq, torch, layer, PREFILL_M, asym=True)
+              for layer in range(PREFILL_LAYERS)]
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+
+    def step(i):
+        b = blocks[i % len(blocks)]
+        rc = mq.lib.mq_linear_batch(b.arr, len(b.descs), b.wsp, b.ws_bytes, sp)
+        if rc:
+            raise RuntimeError(f"mq_linear_batch failed: {mq.status_string(rc)}")
+
+    for i in range(6):
+        step(i)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(steps):
+        step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in the asymmetric prefill run")
+    ms = e0.elapsed_time(e1) / steps
+    # parity sample: run layer 0 once more, then compare its first rows
+    step(0)
+    torch.cuda.synchronize()
+    import oracle
+    oracle.build()
+    mism = checked = 0
+    for j, c in enumerate(blocks[0].cases):
+        packed, _ = oracle.pack(c.w, 8)
+        m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
+        y = oracle.linear(np.ascontiguousarray(c.x[:check_rows]), c.zx, packed, 8, c.N, m0, sh,
+                          c.zy, zw=c.zw)
+        if c.residual is not None:
+            y = oracle.residual_add(y, np.ascontiguousarray(c.residual[:check_rows]))
+        got = blocks[0].y[j][:check_rows].cpu().numpy()
+        checked += y.size
+        mism += int(np.count_nonzero(got != y))
+    return {"us_per_block": round(ms * 1e3, 2),
+            "tops": round(block_ops(PREFILL_M) / (ms * 1e-3) / 1e12, 1),
+            "launches_per_step": 2, "steps": steps,
+            "weights": "asymmetric: per tensor (q k v o gate up), per channel (down)",
+            "parity_sample": {"rows": check_rows, "outputs": checked, "mismatches": mism}}
 
 
 # --------------------------------------------------------------------------- CPU oracle
@@ -459,6 +521,8 @@ def main():
 
     pre = run_prefill(mq, torch, dist, args.steps, args.warmup)
     decode = run_decode(mq, torch)
+    asym_pre = run_asym_prefill(mq, torch)
+    asym_dec = run_decode(mq, torch, asym=True, ms=(1, 16))
     peaks = measured_peaks()
 
     ops = block_ops(PREFILL_M)
@@ -467,7 +531,7 @@ def main():
     kern_tflops = ops / (pre["kernel_ms_mean"] * 1e-3) / 1e12
     e2e_value = ops * pre["e2e_steps"] * world / (pre["e2e_ms"] * 1e-3) / 1e12
     hbm = peaks["hbm_gbs"]
-    for v in decode.values():
+    for v in list(decode.values()) + list(asym_dec.values()):
         v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
 
     line = {
@@ -495,6 +559,10 @@ def main():
         "decode_w4a8": {"unit": "GB/s of int4 weights", "weight_bytes_per_block":
                         block_weight_bytes(4), "layers_rotated": DECODE_LAYERS,
                         "hbm_peak_gbs": hbm, **decode},
+        "asym_prefill_w8a8": {**asym_pre, "symmetric_us_per_block":
+                              round(pre["total_ms"] / args.steps * 1e3, 2)},
+        "asym_decode_w4a8": {"unit": "GB/s of int4 weights",
+                             "weights": "asymmetric per channel", **asym_dec},
     }
     if rank == 0 and world == 1:
         line["cpu_baseline"] = cpu_baseline(pre["blocks"], torch)

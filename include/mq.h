@@ -231,9 +231,11 @@ typedef struct mq_linear_desc {
 /*
  * Device workspace bytes one mq_linear_batch call over `descs` needs: the
  * decode workspace (see mq_workspace_size) if any descriptor has
- * 1 <= M <= 16, plus 4*M bytes (rounded up to 16) for every descriptor with
- * M > 16 and a weight zero point, which holds rowsum(x) of its tokens (filled
- * by the call).  0 when neither applies.  The contract of mq_workspace_size
+ * 1 <= M <= 16, plus 4*M bytes (rounded up to 16) for every distinct input
+ * (x, M, K, ldx) of the descriptors with M > 16 and a weight zero point, which
+ * holds rowsum(x) of its tokens (filled by the call; descriptors reading the
+ * same input, e.g. q/k/v/gate/up of one block, share it).  0 when neither
+ * applies.  The contract of mq_workspace_size
  * holds for the whole buffer.
  * Errors: MQ_ERR_INVALID_ARG (null pointers, count out of range, bad bits).
  */

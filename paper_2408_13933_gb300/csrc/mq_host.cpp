@@ -55,20 +55,40 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
 size_t align16(size_t v) { return (v + 15) & ~static_cast<size_t>(15); }
 
 // Workspace layout of one batch: the decode region first (if any decode
-// shape), then rowsum(x) of every prefill descriptor with a weight zero
-// point, in descriptor order.
-size_t batch_workspace(const mq_linear_desc *descs, int count, bool *any_decode) {
+// shape), then one rowsum(x) array per distinct input (x, M, K, ldx) of the
+// prefill descriptors with a weight zero point, in order of first use.
+// `jobs` (may be null) receives those inputs and `offsets` their byte
+// offsets from the start of the rowsum region.
+size_t batch_workspace(const mq_linear_desc *descs, int count, bool *any_decode,
+                       std::vector<mq::RowsumJob> *jobs, std::vector<size_t> *offsets) {
     bool dec = false;
+    std::vector<mq::RowsumJob> uniq;
+    std::vector<size_t> offs;
     size_t rows = 0;
     for (int i = 0; i < count; ++i) {
         const mq_linear_desc &d = descs[i];
         if (d.M <= 0 || d.N <= 0) continue;
-        if (d.M <= mq::DECODE_MAX_M)
+        if (d.M <= mq::DECODE_MAX_M) {
             dec = true;
-        else if (d.zw && d.K > 0)
-            rows += align16(4 * (size_t)d.M);
+            continue;
+        }
+        if (!d.zw || d.K <= 0) continue;
+        bool seen = false;
+        for (const auto &j : uniq)
+            seen |= j.x == d.x && j.M == d.M && j.K == d.K && j.ldx == d.ldx;
+        if (seen) continue;
+        mq::RowsumJob j{};
+        j.x = d.x;
+        j.M = d.M;
+        j.K = d.K;
+        j.ldx = d.ldx;
+        uniq.push_back(j);
+        offs.push_back(rows);
+        rows += align16(4 * (size_t)d.M);
     }
     if (any_decode) *any_decode = dec;
+    if (jobs) *jobs = uniq;
+    if (offsets) *offsets = offs;
     return (dec ? mq::DECODE_WS_BYTES : 0) + rows;
 }
 
@@ -88,21 +108,23 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
             pre.push_back(p);
     }
     // the decode kernel combines split 64-row units in the workspace; prefill
-    // descriptors with a weight zero point keep rowsum(x) there
+    // descriptors with a weight zero point read rowsum(x) from there
     bool any_decode = false;
-    const size_t need = batch_workspace(descs, count, &any_decode);
+    std::vector<mq::RowsumJob> jobs;
+    std::vector<size_t> offsets;
+    const size_t need = batch_workspace(descs, count, &any_decode, &jobs, &offsets);
     if (need > 0 && (!workspace || ws_bytes < need || !aligned16(workspace)))
         return MQ_ERR_WORKSPACE;
-    size_t off = any_decode ? mq::DECODE_WS_BYTES : 0;
-    bool any_rowsum = false;
+    uint8_t *region = static_cast<uint8_t *>(workspace) + (any_decode ? mq::DECODE_WS_BYTES : 0);
+    for (size_t i = 0; i < jobs.size(); ++i)
+        jobs[i].out = reinterpret_cast<int32_t *>(region + offsets[i]);
     for (auto &p : pre) {
         if (!p.zw || p.K == 0) continue;
-        p.rowsum = reinterpret_cast<const int32_t *>(static_cast<uint8_t *>(workspace) + off);
-        off += align16(4 * (size_t)p.M);
-        any_rowsum = true;
+        for (const auto &j : jobs)
+            if (j.x == p.x && j.M == p.M && j.K == p.K && j.ldx == p.ldx) p.rowsum = j.out;
     }
     int rc = MQ_OK;
-    if (any_rowsum) rc = mq::launch_rowsum(pre.data(), (int)pre.size(), stream);
+    if (!jobs.empty()) rc = mq::launch_rowsum(jobs.data(), (int)jobs.size(), stream);
     if (rc == MQ_OK && !pre.empty()) rc = mq::launch_prefill(pre.data(), (int)pre.size(), stream);
     if (rc == MQ_OK && !dec8.empty())
         rc = mq::launch_decode(dec8.data(), (int)dec8.size(), workspace, stream);
@@ -272,7 +294,7 @@ int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *byte
     if (!descs || !bytes || count < 1 || count > MQ_MAX_BATCH) return MQ_ERR_INVALID_ARG;
     for (int i = 0; i < count; ++i)
         if (descs[i].bits != 8 && descs[i].bits != 4) return MQ_ERR_INVALID_ARG;
-    *bytes = batch_workspace(descs, count, nullptr);
+    *bytes = batch_workspace(descs, count, nullptr, nullptr, nullptr);
     return MQ_OK;
 }
 

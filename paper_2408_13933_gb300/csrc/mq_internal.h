@@ -54,7 +54,14 @@ int launch_prefill(const Problem *probs, int count, void *stream);
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream);
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
                 int *status, void *stream);
-// rowsum(x)[m] = sum_k x[m][k] of every problem with a rowsum pointer.
-int launch_rowsum(const Problem *probs, int count, void *stream);
+// One distinct input of a batch whose rowsum(x)[m] = sum_k x[m][k] a prefill
+// problem with a weight zero point needs (problems sharing x share the job).
+struct RowsumJob {
+    const int8_t *x;
+    int32_t *out;  // [M] in the workspace
+    int32_t M, K, ldx;
+};
+constexpr int ROWSUM_MAX_JOBS = 64;  // jobs per launch (kernel parameter space)
+int launch_rowsum(const RowsumJob *jobs, int count, void *stream);
 
 }  // namespace mq

@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include "mq_internal.h"
+#include "mq_ptx.cuh"
 
 namespace mq {
 
@@ -92,39 +93,81 @@ int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *
 namespace rowsum {
 
 constexpr int ROWS_PER_BLOCK = 8;  // one warp per row
+constexpr int LOADS = 8;           // 16-byte loads in flight per lane
 
-// rowsum[m] = sum_k x[m][k]; K and ldx are multiples of 16 and x is 16-byte
-// aligned (the library's validation), so every load is a whole uint4.
-__global__ void __launch_bounds__(ROWS_PER_BLOCK * 32)
-    rowsum_kernel(const int8_t *__restrict__ x, int M, int K, int ldx, int32_t *__restrict__ out) {
-    const int row = blockIdx.x * ROWS_PER_BLOCK + (threadIdx.x >> 5);
+struct Params {
+    RowsumJob job[ROWSUM_MAX_JOBS];
+    int32_t block_begin[ROWSUM_MAX_JOBS + 1];  // first block of each job, then the total
+    int32_t count;
+};
+
+// out[m] = sum_k x[m][k] for every job; K and ldx are multiples of 16 and x
+// is 16-byte aligned (the library's validation), so every load is a whole
+// uint4.  Launched with programmatic stream serialization: x may be the output
+// of the previous kernel in the stream, so nothing is read before
+// griddep_wait; the kernel that follows (the prefill) reads `out` only after
+// its own griddep_wait, i.e. after this grid has completed.
+__global__ void __launch_bounds__(ROWS_PER_BLOCK * 32) rowsum_kernel(const __grid_constant__ Params P) {
+    griddep_wait();
+    griddep_launch_dependents();
+    int j = 0;
+    while (j + 1 < P.count && (int)blockIdx.x >= P.block_begin[j + 1]) ++j;
+    const RowsumJob &q = P.job[j];
+    const int row = ((int)blockIdx.x - P.block_begin[j]) * ROWS_PER_BLOCK + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
-    if (row >= M) return;
-    const int8_t *r = x + (size_t)row * (size_t)ldx;
+    if (row >= q.M) return;
+    const uint4 *r = reinterpret_cast<const uint4 *>(q.x + (size_t)row * (size_t)q.ldx);
+    const int n16 = q.K >> 4;  // 16-byte chunks of the row
     int acc = 0;
-    for (int k = lane * 16; k < K; k += 32 * 16) {
-        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(r + k));
-        acc = __dp4a((int)v.x, 0x01010101, acc);
-        acc = __dp4a((int)v.y, 0x01010101, acc);
-        acc = __dp4a((int)v.z, 0x01010101, acc);
-        acc = __dp4a((int)v.w, 0x01010101, acc);
+    // LOADS chunks per lane in flight per round: a row of K <= 4096 takes one
+    // round of memory latency
+    for (int base = lane; base < n16; base += 32 * LOADS) {
+        uint4 v[LOADS];
+#pragma unroll
+        for (int u = 0; u < LOADS; ++u) {
+            const int i = base + 32 * u;
+            v[u] = i < n16 ? __ldg(r + i) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < LOADS; ++u) {
+            acc = __dp4a((int)v[u].x, 0x01010101, acc);
+            acc = __dp4a((int)v[u].y, 0x01010101, acc);
+            acc = __dp4a((int)v[u].z, 0x01010101, acc);
+            acc = __dp4a((int)v[u].w, 0x01010101, acc);
+        }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) out[row] = acc;
+    if (lane == 0) q.out[row] = acc;
 }
 
 }  // namespace rowsum
 
-int launch_rowsum(const Problem *probs, int count, void *stream) {
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    for (int i = 0; i < count; ++i) {
-        const Problem &p = probs[i];
-        if (!p.rowsum || p.M <= 0) continue;
-        const int blocks = (p.M + rowsum::ROWS_PER_BLOCK - 1) / rowsum::ROWS_PER_BLOCK;
-        rowsum::rowsum_kernel<<<blocks, rowsum::ROWS_PER_BLOCK * 32, 0, s>>>(
-            p.x, p.M, p.K, p.ldx, const_cast<int32_t *>(p.rowsum));
-        if (cudaGetLastError() != cudaSuccess) return MQ_ERR_CUDA;
+int launch_rowsum(const RowsumJob *jobs, int count, void *stream) {
+    for (int base = 0; base < count; base += ROWSUM_MAX_JOBS) {
+        rowsum::Params P{};
+        const int n = count - base < ROWSUM_MAX_JOBS ? count - base : ROWSUM_MAX_JOBS;
+        int64_t blocks = 0;
+        for (int i = 0; i < n; ++i) {
+            P.job[i] = jobs[base + i];
+            P.block_begin[i] = (int32_t)blocks;
+            blocks += (jobs[base + i].M + rowsum::ROWS_PER_BLOCK - 1) / rowsum::ROWS_PER_BLOCK;
+        }
+        if (blocks == 0) continue;
+        if (blocks > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
+        P.block_begin[n] = (int32_t)blocks;
+        P.count = n;
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)blocks, 1, 1);
+        cfg.blockDim = dim3(rowsum::ROWS_PER_BLOCK * 32, 1, 1);
+        cfg.dynamicSmemBytes = 0;
+        cfg.stream = static_cast<cudaStream_t>(stream);
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&cfg, rowsum::rowsum_kernel, P) != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;
 }

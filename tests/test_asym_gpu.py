@@ -30,14 +30,18 @@ def zero_points(seed, n, bits, ends=True):
 class AsymCase:
     """Device operands of one asymmetric problem and its oracle result."""
 
-    def __init__(self, seed, m, k, n, bits, extreme=None, residual=False, zw=None):
+    def __init__(self, seed, m, k, n, bits, extreme=None, residual=False, zw=None, share=None):
         lib = mq()
         torch = torch_cuda()
         self.c = c = synth.random_case(seed, m, k, n, bits, extreme)
+        if share is not None:  # read the input of another case (same device buffer)
+            c.x, c.zx = share.c.x, share.c.zx
         self.zw = zero_points(seed, n, bits) if zw is None else zw
         packed, colsum = lib.pack_weights(c.w, bits)
         m0, sh = lib.requant_params(c.sw, c.sx, c.sy)
         self.dev = [upload(a) for a in (c.x, packed, colsum, m0, sh, self.zw)]
+        if share is not None:
+            self.dev[0] = share.dev[0]
         self.res = synth.residual_codes(seed, 0, m, n) if residual else None
         self.dres = upload(self.res) if residual else None
         self.y = torch.full((m, n), 77, dtype=torch.int8, device="cuda")
@@ -135,3 +139,26 @@ def test_asym_batch_mixes_kernels_and_symmetric():
     assert lib.check_device_status() == 0
     for x in cases:
         assert_equal_int8(x.y.cpu().numpy(), x.want(), f"batch {x.c.name}")
+
+
+def test_asym_shared_input_one_rowsum():
+    # q/k/v/gate/up-like problems reading one input: one rowsum region for
+    # all of them, next to another input's region
+    a = AsymCase(61, 96, 512, 128, 8)
+    b = AsymCase(62, 96, 512, 64, 4, share=a)
+    c = AsymCase(63, 96, 512, 200, 8, share=a)
+    d = AsymCase(64, 96, 512, 48, 8, share=a, zw=np.zeros(48, np.int32))
+    e = AsymCase(65, 80, 256, 72, 4)
+    cases = [a, b, c, d, e]
+    lib = mq()
+    descs = [x.desc() for x in cases]
+    descs[3].zw = None
+    need = lib.workspace_size_batch(descs)
+    assert need == 16 * ((4 * 96 + 15) // 16) + 16 * ((4 * 80 + 15) // 16)
+    torch = torch_cuda()
+    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+    assert lib.linear_batch(descs, workspace=ws, ws_bytes=need) == 0
+    torch.cuda.synchronize()
+    assert lib.check_device_status() == 0
+    for x in cases:
+        assert_equal_int8(x.y.cpu().numpy(), x.want(), f"shared input {x.c.name}")

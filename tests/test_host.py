@@ -181,6 +181,45 @@ def test_asym_int8_k_limit_and_workspace(mq):
     assert mq.workspace_size_batch([_desc(mq, 101, 64, 32, 8, True),
                                     _desc(mq, 8, 64, 32, 4, True)]) == dec + 416
     assert mq.workspace_size_batch([_desc(mq, 8, 64, 32, 4, False)]) == dec
+    # descriptors reading one input share its rowsum region; another x, M, K
+    # or ldx is another input
+    same = [_desc(mq, 100, 64, 32, 8, True), _desc(mq, 100, 64, 48, 4, True)]
+    assert mq.workspace_size_batch(same) == 400
+    other = _desc(mq, 100, 64, 32, 8, True)
+    other.x = FAKE + 4096
+    assert mq.workspace_size_batch(same + [other]) == 800
+    longer = _desc(mq, 100, 128, 32, 8, True)
+    longer.ldx = 128
+    assert mq.workspace_size_batch(same + [longer]) == 800
     # an asymmetric prefill batch without its workspace is rejected up front
     one = (mq.LinearDesc * 1)(_desc(mq, 100, 64, 32, 8, True))
     assert mq.lib.mq_linear_batch(one, 1, None, 0, None) == mq.MQ_ERR_WORKSPACE
+
+
+def test_synth_asymmetric_weights():
+    # the asymmetric weight generator: codes span the range, the zero point
+    # maps 0.0 into the code range, and dequantization s (w - z) is within half
+    # a step of the float weight wherever the code did not clip
+    import numpy as np
+    from paper_2408_13933_gb300 import synth
+    rng = np.random.default_rng(5)
+    wf = (rng.standard_normal((40, 256)) * 0.02).astype(np.float32)
+    wf[3] += 0.01  # a channel biased positive
+    for bits in (8, 4):
+        lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+        for per_channel in (False, True):
+            q, s, z = synth.quantize_asymmetric(wf, bits, per_channel)
+            assert q.dtype == np.int8 and q.min() >= lo and q.max() <= hi
+            assert (z >= lo).all() and (z <= hi).all()
+            if not per_channel:
+                assert len(set(s.tolist())) == 1 and len(set(z.tolist())) == 1
+            deq = s[:, None].astype(np.float64) * (q.astype(np.float64) - z[:, None])
+            inside = (q > lo) & (q < hi)
+            assert np.all(np.abs(deq - wf)[inside] <= 0.5 * s[:, None].repeat(256, 1)[inside] * 1.001)
+            # the range ends are reached (per channel: in every channel)
+            if per_channel:
+                assert ((q == lo) | (q == hi)).any(axis=1).all()
+    # the paper's settings: W8A8 per tensor except down per channel; W4A8 per channel
+    assert synth.paper_weight_scheme("q", 8) == "asym_tensor"
+    assert synth.paper_weight_scheme("down", 8) == "asym_channel"
+    assert synth.paper_weight_scheme("q", 4) == "asym_channel"
