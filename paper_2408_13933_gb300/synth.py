@@ -64,19 +64,21 @@ def float_activations(rng: np.random.Generator, m: int, k: int, n_outliers: int 
     return xf
 
 
-def quantize_per_tensor(xf: np.ndarray):
-    """Asymmetric per-tensor int8 codes (eqs. 2-4, shifted to signed int8)."""
+def quantize_per_tensor(xf: np.ndarray, bits: int = 8):
+    """Asymmetric per-tensor codes (eqs. 2-4, shifted to the signed range):
+    int8, or int16 with bits=16 (the 16-bit activations of Sec. 4.1 / 5.6)."""
+    qmin, qmax = (-128, 127) if bits == 8 else (-32768, 32767)
     lo = float(min(xf.min(), 0.0)) if xf.size else -1.0
     hi = float(max(xf.max(), 0.0)) if xf.size else 1.0
     if hi - lo <= 0:
         hi = lo + 1.0
-    s = np.float32((hi - lo) / 255.0)
-    z = int(rint_clip(np.array(-128.0 - lo / float(s)), -128, 127))
+    s = np.float32((hi - lo) / float(qmax - qmin))
+    z = int(rint_clip(np.array(qmin - lo / float(s)), qmin, qmax))
     t = xf / s
     t += np.float32(z)
     np.rint(t, out=t)
-    np.clip(t, -128, 127, out=t)
-    return t.astype(np.int8), float(s), z
+    np.clip(t, qmin, qmax, out=t)
+    return t.astype(np.int8 if bits == 8 else np.int16), float(s), z
 
 
 _POOL = None
@@ -130,26 +132,55 @@ def quantize_per_channel_symmetric(wf: np.ndarray, bits: int, inplace: bool = Fa
     return t.astype(np.int8), sw
 
 
-def output_range(yf: np.ndarray):
+def quantize_asymmetric(wf: np.ndarray, bits: int, per_channel: bool, inplace: bool = False):
+    """Asymmetric weight codes, the min-max quantizer of Sec. 4.2 applied to
+    weights as in the paper's main W8A8 / W4A8 settings: s = (max - min) /
+    (2^bits - 1), z = clamp(rint(qmin - min / s), qmin, qmax),
+    w = clamp(rint(w / s) + z, qmin, qmax), with min/max over the whole tensor
+    or over each output channel.  Returns (codes int8 [N,K], sw float32 [N],
+    zw int32 [N]); per tensor, sw and zw repeat one value."""
+    qmin, qmax = (-128, 127) if bits == 8 else (-8, 7)
+    n = wf.shape[0]
+    if per_channel:
+        lo = wf.min(axis=1) if wf.size else np.zeros(n, np.float32)
+        hi = wf.max(axis=1) if wf.size else np.zeros(n, np.float32)
+    else:
+        lo = np.full(n, wf.min() if wf.size else 0.0, np.float32)
+        hi = np.full(n, wf.max() if wf.size else 0.0, np.float32)
+    lo, hi = np.minimum(lo, 0).astype(np.float32), np.maximum(hi, 0).astype(np.float32)
+    span = np.where(hi - lo > 0, hi - lo, np.float32(1e-8)).astype(np.float32)
+    sw = (span / np.float32(qmax - qmin)).astype(np.float32)
+    zw = rint_clip(np.float32(qmin) - lo / sw, qmin, qmax).astype(np.int32)
+    t = wf if inplace else wf.copy()
+    np.divide(t, sw[:, None], out=t)
+    np.rint(t, out=t)
+    t += zw[:, None].astype(np.float32)
+    np.clip(t, qmin, qmax, out=t)
+    return t.astype(np.int8), sw, zw
+
+
+def output_range(yf: np.ndarray, bits: int = 8):
     """Static output (sy, zy) from the float layer's min/max (calibration)."""
     return quantize_params_from_range(float(yf.min()) if yf.size else -1.0,
-                                      float(yf.max()) if yf.size else 1.0)
+                                      float(yf.max()) if yf.size else 1.0, bits)
 
 
-def quantize_params_from_range(lo: float, hi: float):
+def quantize_params_from_range(lo: float, hi: float, bits: int = 8):
+    qmin, qmax = (-128, 127) if bits == 8 else (-32768, 32767)
     lo, hi = min(lo, 0.0), max(hi, 0.0)
     if hi - lo <= 0:
         hi = lo + 1.0
-    s = np.float32((hi - lo) / 255.0)
-    z = int(rint_clip(np.array(-128.0 - lo / float(s)), -128, 127))
+    s = np.float32((hi - lo) / float(qmax - qmin))
+    z = int(rint_clip(np.array(qmin - lo / float(s)), qmin, qmax))
     return float(s), z
 
 
 @dataclass
 class LinearCase:
-    """One quantized linear problem: int8 x [M,K], int weights [N,K], scales."""
+    """One quantized linear problem: int8 (or int16) x [M,K], int weights
+    [N,K], scales; the output has the activations' width."""
     name: str
-    x: np.ndarray          # int8 [M, K]
+    x: np.ndarray          # int8 [M, K], or int16 for 16-bit activations
     zx: int
     sx: float
     w: np.ndarray          # int8 values [N, K] (int4 range if bits == 4)
@@ -158,6 +189,7 @@ class LinearCase:
     sy: float
     zy: int
     residual: np.ndarray | None = None   # optional int8 [M, N]
+    zw: np.ndarray | None = None         # int32 [N] weight zero point, None = symmetric
     meta: dict = field(default_factory=dict)
 
     @property
@@ -169,11 +201,15 @@ class LinearCase:
     @property
     def N(self): return self.w.shape[0]
 
+    @property
+    def abits(self): return 16 if self.x.dtype == np.int16 else 8
+
 
 def make_linear(config: int, layer: int, linear: int, name: str, m: int, k: int, n: int,
                 bits: int, t_rows_frac: float = 0.0, calib_rows: int = 64,
-                x: tuple | None = None) -> LinearCase:
-    """A seeded linear problem.  `x` may pass (x_int8, sx, zx) to reuse inputs."""
+                x: tuple | None = None, weights: str = "symmetric") -> LinearCase:
+    """A seeded linear problem.  `x` may pass (x_int8, sx, zx) to reuse inputs.
+    `weights`: "symmetric" (per channel), "asym_tensor" or "asym_channel"."""
     if x is None:
         xf = float_activations(rng_for(config, layer, linear, ROLE_X), m, k,
                                orng=rng_for(config, layer, linear, ROLE_OUTLIER))
@@ -188,14 +224,28 @@ def make_linear(config: int, layer: int, linear: int, name: str, m: int, k: int,
     xdq = (xq[:rows].astype(np.float32) - np.float32(zx)) * np.float32(sx)
     yf = xdq @ wf.T if rows and n else np.zeros((0, n), np.float32)
     sy, zy = output_range(yf)
-    wq, sw = quantize_per_channel_symmetric(wf, bits, inplace=True)
-    return LinearCase(name, xq, zx, sx, wq, sw, bits, sy, zy)
+    if weights == "symmetric":
+        wq, sw = quantize_per_channel_symmetric(wf, bits, inplace=True)
+        return LinearCase(name, xq, zx, sx, wq, sw, bits, sy, zy)
+    if weights not in ("asym_tensor", "asym_channel"):
+        raise ValueError(f"unknown weight scheme {weights!r}")
+    wq, sw, zw = quantize_asymmetric(wf, bits, weights == "asym_channel", inplace=True)
+    return LinearCase(name, xq, zx, sx, wq, sw, bits, sy, zy, zw=zw)
+
+
+def paper_weight_scheme(name: str, bits: int) -> str:
+    """The paper's main asymmetric settings (Sec. 5.1): W8A8 per tensor except
+    the MLP's last projection (down) per channel; W4A8 per channel."""
+    if bits == 4 or name == "down":
+        return "asym_channel"
+    return "asym_tensor"
 
 
 def block_linears(config: int, m: int, bits: int, shapes=TINYLLAMA_LINEARS, layer: int = 0,
-                  t_rows_frac: float = 0.0, shared_input: bool = False):
+                  t_rows_frac: float = 0.0, shared_input: bool = False, asym: bool = False):
     """All linears of one decoder block, each with its own seeded input
-    (or, with shared_input, q/k/v/gate/up reading one x of width 2048)."""
+    (or, with shared_input, q/k/v/gate/up reading one x of width 2048);
+    with asym, weights follow paper_weight_scheme."""
     out = []
     shared = None
     for j, (name, k, n) in enumerate(shapes):
@@ -207,7 +257,8 @@ def block_linears(config: int, m: int, bits: int, shapes=TINYLLAMA_LINEARS, laye
                 shared = quantize_per_tensor(xf)
             xin = shared
         out.append(make_linear(config, layer, j, name, m, k, n, bits,
-                               t_rows_frac=t_rows_frac, x=xin))
+                               t_rows_frac=t_rows_frac, x=xin,
+                               weights=paper_weight_scheme(name, bits) if asym else "symmetric"))
     return out
 
 
@@ -215,6 +266,72 @@ def residual_codes(config: int, layer: int, m: int, n: int, scale: float = 8.0) 
     """Seeded fixed int8 residual for the chained stack (reading R8)."""
     r = rng_for(config, layer, 0, ROLE_RES).standard_normal((m, n), dtype=np.float32) * scale
     return rint_clip(r, -128, 127).astype(np.int8)
+
+
+def make_linear_a16(config: int, layer: int, linear: int, name: str, m: int, k: int, n: int,
+                    bits: int, calib_rows: int = 64, x: tuple | None = None) -> LinearCase:
+    """A seeded linear problem with 16-bit activations and outputs (W8A16 /
+    W4A16): the float data of make_linear, activations quantized per tensor
+    to int16, the output range calibrated on the 16-bit grid, weights
+    symmetric per channel.  `x` may pass (x_int16, sx, zx) to reuse inputs."""
+    if x is None:
+        xf = float_activations(rng_for(config, layer, linear, ROLE_X), m, k,
+                               orng=rng_for(config, layer, linear, ROLE_OUTLIER))
+        xq, sx, zx = quantize_per_tensor(xf, bits=16)
+    else:
+        xq, sx, zx = x
+    wf = float_weights(rng_for(config, layer, linear, ROLE_W), n, k)
+    rows = min(m, calib_rows)
+    xdq = (xq[:rows].astype(np.float32) - np.float32(zx)) * np.float32(sx)
+    yf = xdq @ wf.T if rows and n else np.zeros((0, n), np.float32)
+    sy, zy = output_range(yf, bits=16)
+    wq, sw = quantize_per_channel_symmetric(wf, bits, inplace=True)
+    return LinearCase(name, xq, zx, sx, wq, sw, bits, sy, zy)
+
+
+def block_linears_a16(config: int, m: int, bits: int, shapes=TINYLLAMA_LINEARS,
+                      layer: int = 0, shared_input: bool = False):
+    """All linears of one decoder block with 16-bit activations (see
+    block_linears)."""
+    out = []
+    shared = None
+    for j, (name, k, n) in enumerate(shapes):
+        xin = None
+        if shared_input and name in ("q", "k", "v", "gate", "up"):
+            if shared is None:
+                xf = float_activations(rng_for(config, layer, 99, ROLE_X), m, k,
+                                       orng=rng_for(config, layer, 99, ROLE_OUTLIER))
+                shared = quantize_per_tensor(xf, bits=16)
+            xin = shared
+        out.append(make_linear_a16(config, layer, j, name, m, k, n, bits, x=xin))
+    return out
+
+
+def random_case_a16(seed: int, m: int, k: int, n: int, bits: int,
+                    extreme: str | None = None) -> LinearCase:
+    """Small seeded problem with int16 activations for parity tests, optionally
+    with extreme codes: 'min', 'max' or 'mixed' (as random_case)."""
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([BASE_SEED, 16, seed])))
+    wlo, whi = (-128, 127) if bits == 8 else (-8, 7)
+    x = rng.integers(-32768, 32768, size=(m, k), dtype=np.int32).astype(np.int16)
+    w = rng.integers(wlo, whi + 1, size=(n, k), dtype=np.int16).astype(np.int8)
+    zx = int(rng.integers(-32768, 32768))
+    if extreme == "min":
+        x[:] = -32768
+        w[:] = wlo
+        zx = 32767
+    elif extreme == "max":
+        x[:] = 32767
+        w[:] = whi
+        zx = -32768
+    elif extreme == "mixed":
+        x[:] = np.where(rng.random((m, k)) < 0.5, -32768, 32767).astype(np.int16)
+        w[:] = np.where(rng.random((n, k)) < 0.5, wlo, whi).astype(np.int8)
+    sx = float(np.float32(rng.uniform(2e-5, 2e-4)))
+    sw = rng.uniform(1e-4, 3e-3, size=n).astype(np.float32)
+    sy = float(np.float32(rng.uniform(5e-6, 5e-5) * (16 if bits == 8 else 1)))
+    zy = int(rng.integers(-16384, 16384))
+    return LinearCase(f"a16rand{seed}", x, zx, sx, w, sw, bits, sy, zy)
 
 
 def random_case(seed: int, m: int, k: int, n: int, bits: int, extreme: str | None = None) -> LinearCase:
