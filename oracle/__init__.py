@@ -52,6 +52,11 @@ def _bind(lib):
                                               ci, p, p]
     lib.oracle_requant_one.argtypes = [i64, i32, i32, i32]
     lib.oracle_requant_one.restype = i32
+    lib.oracle_linear_a16.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci, p]
+    lib.oracle_linear_points_a16.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci,
+                                             p, p]
+    lib.oracle_requant_one_a16.argtypes = [i64, i32, i32, i32]
+    lib.oracle_requant_one_a16.restype = i32
     lib.oracle_residual_add.argtypes = [p, p, i64, p]
     lib.oracle_residual_add.restype = None
     return lib
@@ -158,6 +163,44 @@ class Oracle:
     def requant_one(self, acc: int, m0: int, shift: int, zy: int) -> int:
         return int(self.lib.oracle_requant_one(int(acc), int(m0), int(shift), int(zy)))
 
+    def linear_a16(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
+                   m0: np.ndarray, shift: np.ndarray, zy: int, want_acc: bool = False):
+        """The layer with int16 activations (oracle_linear_a16): returns y int16
+        [M, N] (and acc int64 [M, N])."""
+        x = np.ascontiguousarray(x, dtype=np.int16)
+        m, k = x.shape
+        packed = np.ascontiguousarray(packed, dtype=np.uint8)
+        m0 = np.ascontiguousarray(m0, dtype=np.int32)
+        shift = np.ascontiguousarray(shift, dtype=np.int32)
+        y = np.zeros((m, n), np.int16)
+        acc = np.zeros((m, n), np.int64) if want_acc else None
+        _check(self.lib.oracle_linear_a16(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
+                                          _ptr(m0), _ptr(shift), int(zy), _ptr(y), n,
+                                          _ptr(acc) if acc is not None else None),
+               "oracle_linear_a16")
+        return (y, acc) if want_acc else y
+
+    def linear_points_a16(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
+                          m0: np.ndarray, shift: np.ndarray, zy: int, pts: np.ndarray):
+        """oracle_linear_a16 at listed (m, n) coordinates: returns (y[i], acc[i])."""
+        x = np.ascontiguousarray(x, dtype=np.int16)
+        m, k = x.shape
+        pts = np.ascontiguousarray(pts, dtype=np.int64).reshape(-1, 2)
+        cnt = pts.shape[0]
+        y = np.zeros(cnt, np.int16)
+        acc = np.zeros(cnt, np.int64)
+        packed = np.ascontiguousarray(packed, dtype=np.uint8)
+        m0 = np.ascontiguousarray(m0, dtype=np.int32)
+        shift = np.ascontiguousarray(shift, dtype=np.int32)
+        _check(self.lib.oracle_linear_points_a16(_ptr(x), m, k, k, int(zx), _ptr(packed), bits,
+                                                 n, _ptr(m0), _ptr(shift), int(zy), _ptr(pts),
+                                                 cnt, _ptr(y), _ptr(acc)),
+               "oracle_linear_points_a16")
+        return y, acc
+
+    def requant_one_a16(self, acc: int, m0: int, shift: int, zy: int) -> int:
+        return int(self.lib.oracle_requant_one_a16(int(acc), int(m0), int(shift), int(zy)))
+
     def residual_add(self, a: np.ndarray, b: np.ndarray) -> np.ndarray:
         a = np.ascontiguousarray(a, dtype=np.int8)
         b = np.ascontiguousarray(b, dtype=np.int8)
@@ -198,6 +241,18 @@ def linear_points(x, zx, packed, bits, n, m0, shift, zy, pts, zw=None):
 
 def requant_one(acc, m0, shift, zy):
     return _default().requant_one(acc, m0, shift, zy)
+
+
+def linear_a16(x, zx, packed, bits, n, m0, shift, zy, want_acc=False):
+    return _default().linear_a16(x, zx, packed, bits, n, m0, shift, zy, want_acc)
+
+
+def linear_points_a16(x, zx, packed, bits, n, m0, shift, zy, pts):
+    return _default().linear_points_a16(x, zx, packed, bits, n, m0, shift, zy, pts)
+
+
+def requant_one_a16(acc, m0, shift, zy):
+    return _default().requant_one_a16(acc, m0, shift, zy)
 
 
 def residual_add(a, b):

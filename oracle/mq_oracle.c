@@ -243,6 +243,79 @@ int oracle_linear_points_asym(const int8_t *x, int M, int K, int ldx, int32_t zx
     return ORACLE_OK;
 }
 
+/* floor(acc * M0 / 2^s + 1/2) on exact integers (|acc| < 2^40, M0 < 2^31,
+ * so |2 acc M0 + 2^s| < 2^73). */
+static __int128 oracle_round_shift(int64_t acc, int32_t M0, int32_t shift) {
+    __int128 v = (__int128)acc * (__int128)M0;
+    __int128 two_s = (__int128)1 << shift;
+    return oracle_floor_div(2 * v + two_s, 2 * two_s);
+}
+
+int32_t oracle_requant_one_a16(int64_t acc, int32_t M0, int32_t shift, int32_t zy) {
+    __int128 out = (__int128)zy + oracle_round_shift(acc, M0, shift);
+    if (out < -32768) out = -32768;
+    if (out > 32767) out = 32767;
+    return (int32_t)out;
+}
+
+/* acc = sum_k (x[m][k] - zx) * w[n][k] in int64, 16-bit activations. */
+static int64_t oracle_dot_a16(const int16_t *x, int K, int ldx, int32_t zx,
+                              const uint8_t *packed, int bits, int m, int n) {
+    int64_t acc16 = 0;
+    for (int k = 0; k < K; ++k) {
+        int64_t x16 = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - (int64_t)zx;
+        int64_t w16 = oracle_weight_at(packed, bits, K, n, k);
+        acc16 += x16 * w16;
+    }
+    return acc16;
+}
+
+static int oracle_check_args_a16(int M, int K, int ldx, int bits, int N,
+                                 int32_t zx, int32_t zy) {
+    if (M < 0 || K < 0 || N < 0 || K > 65536) return ORACLE_EINVAL;
+    if (bits != 8 && bits != 4) return ORACLE_EINVAL;
+    if (bits == 4 && K % 2 != 0) return ORACLE_EINVAL;
+    if (ldx < K) return ORACLE_EINVAL;
+    if (zx < -32768 || zx > 32767 || zy < -32768 || zy > 32767) return ORACLE_EINVAL;
+    return ORACLE_OK;
+}
+
+int oracle_linear_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                      const uint8_t *packed, int bits, int N, const int32_t *M0,
+                      const int32_t *shift, int32_t zy, int16_t *y, int ldy,
+                      int64_t *acc_out) {
+    int rc = oracle_check_args_a16(M, K, ldx, bits, N, zx, zy);
+    if (rc != ORACLE_OK) return rc;
+    if (ldy < N) return ORACLE_EINVAL;
+    for (int m = 0; m < M; ++m) {
+        for (int n = 0; n < N; ++n) {
+            int64_t acc = oracle_dot_a16(x, K, ldx, zx, packed, bits, m, n);
+            if (acc_out) acc_out[(size_t)m * (size_t)N + (size_t)n] = acc;
+            if (y)
+                y[(size_t)m * (size_t)ldy + (size_t)n] =
+                    (int16_t)oracle_requant_one_a16(acc, M0[n], shift[n], zy);
+        }
+    }
+    return ORACLE_OK;
+}
+
+int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                             const uint8_t *packed, int bits, int N,
+                             const int32_t *M0, const int32_t *shift, int32_t zy,
+                             const int64_t *pts, int count, int16_t *y_out,
+                             int64_t *acc_out) {
+    int rc = oracle_check_args_a16(M, K, ldx, bits, N, zx, zy);
+    if (rc != ORACLE_OK) return rc;
+    for (int i = 0; i < count; ++i) {
+        int64_t m = pts[2 * i], n = pts[2 * i + 1];
+        if (m < 0 || m >= M || n < 0 || n >= N) return ORACLE_EINVAL;
+        int64_t acc = oracle_dot_a16(x, K, ldx, zx, packed, bits, (int)m, (int)n);
+        if (acc_out) acc_out[i] = acc;
+        if (y_out) y_out[i] = (int16_t)oracle_requant_one_a16(acc, M0[n], shift[n], zy);
+    }
+    return ORACLE_OK;
+}
+
 void oracle_residual_add(const int8_t *a, const int8_t *b, int64_t n,
                          int8_t *out) {
     for (int64_t i = 0; i < n; ++i) {

@@ -122,6 +122,39 @@ int oracle_linear_points_asym(const int8_t *x, int M, int K, int ldx, int32_t zx
                               int32_t *acc_out);
 
 /*
+ * The layer with 16-bit activations (W8A16 / W4A16): the paper keeps the
+ * activations of its 16-bit baselines, and those around non-linear operators,
+ * in 16-bit integers (Sec. 4.1 challenge i; Sec. 5.6 on-device settings
+ * W8A16 and W4A16, Table 5).  The 16-bit unsigned code range is shifted by
+ * -32768 to signed int16, as for 8 bits (reading R1): x is int16 [M][ldx]
+ * with zx in [-32768, 32767], the output y is int16 [M][ldy] with zy in
+ * [-32768, 32767]; weights as in oracle_linear (symmetric per channel).
+ *   acc[m][n] = sum_k (x[m][k] - zx) * w[n][k]      (int64; |acc| < 2^40)
+ *   v         = acc * M0[n]                          (exact, __int128)
+ *   q         = floor(v / 2^s + 1/2)                 (round half up)
+ *   y[m][n]   = clamp(zy + q, -32768, 32767)
+ * acc_out (may be NULL) receives acc as int64 [M][N] (row stride N).
+ * K must not exceed 65536 (ORACLE_EINVAL).
+ * Pinned by: brute force on Python integers and exact rationals, exhaustive
+ * K=1 over all int16 activation codes, reduction to oracle_linear on int8
+ * codes, the split into two int8 planes, exact dequantization, saturation.
+ */
+int oracle_linear_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                      const uint8_t *packed, int bits, int N, const int32_t *M0,
+                      const int32_t *shift, int32_t zy, int16_t *y, int ldy,
+                      int64_t *acc_out);
+
+/* oracle_linear_a16 at listed output coordinates (as oracle_linear_points). */
+int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                             const uint8_t *packed, int bits, int N,
+                             const int32_t *M0, const int32_t *shift, int32_t zy,
+                             const int64_t *pts, int count, int16_t *y_out,
+                             int64_t *acc_out);
+
+/* One 16-bit output: clamp(zy + floor(acc*M0 / 2^s + 1/2), -32768, 32767). */
+int32_t oracle_requant_one_a16(int64_t acc, int32_t M0, int32_t shift, int32_t zy);
+
+/*
  * Requantize one accumulator: clamp(zy + floor(acc*M0 / 2^s + 1/2), -128, 127).
  * Exposed so that tests can sweep accumulators around rounding ties.
  */

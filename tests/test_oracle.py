@@ -276,10 +276,175 @@ def pin_asym_exact_dequant(orc: Oracle):
         assert np.array_equal(xd @ wd.T, acc.astype(np.float64) * sx * sw[None, :])
 
 
+# ---- 16-bit activations (W8A16 / W4A16) -------------------------------------
+
+def _py_requant16(acc: int, m0: int, s: int, zy: int) -> int:
+    # round half up of the exact rational acc m0 / 2^s, saturated to int16
+    return max(-32768, min(32767, zy + _round_half_up_frac(Fraction(acc * m0, 1 << s))))
+
+
+def pin_a16_k1_exhaustive(orc: Oracle):
+    # every int16 code against int8 weights at the ends and middle of the
+    # range (K = 1), several activation zero points: acc = (x - zx) w exactly
+    xs = np.arange(-32768, 32768, dtype=np.int64).astype(np.int16).reshape(-1, 1)
+    w = np.array([[-128], [-1], [0], [1], [127], [-77]], np.int8)
+    packed, _ = orc.pack(w, 8)
+    m0 = np.full(w.shape[0], 1 << 30, np.int32)
+    sh = np.full(w.shape[0], 40, np.int32)
+    for zx in (-32768, -1, 0, 12345, 32767):
+        y, acc = orc.linear_a16(xs, zx, packed, 8, w.shape[0], m0, sh, 7, want_acc=True)
+        ref = (xs.astype(np.int64) - zx) * w[:, 0].astype(np.int64)[None, :]
+        assert np.array_equal(acc, ref), zx
+        # requant of a sample of them against exact rationals (shift 40: acc / 2^10)
+        for i in range(0, xs.shape[0], 4099):
+            for j in range(w.shape[0]):
+                assert int(y[i, j]) == _py_requant16(int(ref[i, j]), 1 << 30, 40, 7), (zx, i, j)
+
+
+def pin_a16_int4_pairs(orc: Oracle):
+    # K = 2, every pair of int4 weights, activation pairs at the range ends
+    w = np.array([[a, b] for a in range(-8, 8) for b in range(-8, 8)], np.int8)
+    packed, _ = orc.pack(w, 4)
+    xs = np.array([[-32768, 32767], [32767, -32768], [-1, 1], [12345, -23456], [0, 0]],
+                  np.int16)
+    m0 = np.full(w.shape[0], 1 << 30, np.int32)
+    sh = np.full(w.shape[0], 31, np.int32)
+    for zx in (-32768, 0, 32767):
+        _, acc = orc.linear_a16(xs, zx, packed, 4, w.shape[0], m0, sh, 0, want_acc=True)
+        ref = (xs.astype(np.int64) - zx) @ w.astype(np.int64).T
+        assert np.array_equal(acc, ref), zx
+
+
+def pin_a16_matmul_and_brute_force(orc: Oracle):
+    # acc against numpy's int64 matmul (exact) on random codes, and every
+    # output of a small case against round half up of exact rationals
+    for seed, bits in ((1, 8), (2, 4), (3, 8)):
+        c = synth.random_case_a16(seed, 7, 96, 13, bits)
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+        y, acc = orc.linear_a16(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True)
+        ref = (c.x.astype(np.int64) - c.zx) @ c.w.astype(np.int64).T
+        assert np.array_equal(acc, ref), seed
+        for m in range(c.M):
+            for n in range(c.N):
+                assert int(y[m, n]) == _py_requant16(int(ref[m, n]), int(m0[n]), int(sh[n]),
+                                                     c.zy), (seed, m, n)
+
+
+def pin_a16_large_accumulators(orc: Oracle):
+    # extreme codes with |acc| up to 65535 * 128 * 1024 ~ 2^33 (int8 weights)
+    # or 65535 * 8 * 8192 ~ 2^32 (int4), outside int32, against numpy's int64
+    # matmul and exact rationals
+    for extreme in ("min", "max", "mixed"):
+        for bits, k in ((8, 1024), (4, 8192)):
+            c = synth.random_case_a16(61, 3, k, 6, bits, extreme)
+            packed, _ = orc.pack(c.w, bits)
+            m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+            y, acc = orc.linear_a16(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True)
+            ref = (c.x.astype(np.int64) - c.zx) @ c.w.astype(np.int64).T
+            assert np.array_equal(acc, ref), (extreme, bits)
+            if extreme != "mixed":
+                assert np.abs(ref).max() >= (1 << 31)
+            for m in range(c.M):
+                for n in range(c.N):
+                    assert int(y[m, n]) == _py_requant16(int(ref[m, n]), int(m0[n]),
+                                                         int(sh[n]), c.zy)
+
+
+def pin_a16_reduces_to_int8(orc: Oracle):
+    # activation codes and zero points inside the int8 range: the same
+    # accumulator as the (separately pinned) int8 layer
+    for bits in (8, 4):
+        c = synth.random_case(21, 9, 128, 11, bits)
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+        _, a8 = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True)
+        _, a16 = orc.linear_a16(c.x.astype(np.int16), c.zx, packed, bits, c.N, m0, sh, c.zy,
+                                want_acc=True)
+        assert np.array_equal(a16, a8.astype(np.int64))
+
+
+def pin_a16_byte_planes(orc: Oracle):
+    # x = 256 hi + (lo - 128) + 128 with hi the signed high byte and lo the
+    # unsigned low byte: the int16 accumulator is 256 times the int8 layer on
+    # the hi plane plus the int8 layer on the (lo - 128) plane plus
+    # (128 - zx) colsum, each int8 layer with zero point 0
+    for bits in (8, 4):
+        c = synth.random_case_a16(31 + bits, 6, 160, 9, bits, "mixed" if bits == 4 else None)
+        packed, colsum = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+        _, acc = orc.linear_a16(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True)
+        u = c.x.view(np.uint16).astype(np.int64)
+        hi = ((u >> 8).astype(np.uint8)).view(np.int8)
+        lo = ((u & 255) - 128).astype(np.int8)
+        _, a_hi = orc.linear(hi, 0, packed, bits, c.N, m0, sh, 0, want_acc=True)
+        _, a_lo = orc.linear(lo, 0, packed, bits, c.N, m0, sh, 0, want_acc=True)
+        want = (256 * a_hi.astype(np.int64) + a_lo.astype(np.int64)
+                + (128 - c.zx) * colsum.astype(np.int64)[None, :])
+        assert np.array_equal(acc, want), bits
+
+
+def pin_a16_exact_dequant(orc: Oracle):
+    # power-of-two scales: the float64 matmul of sx (x - zx) and sw w is
+    # exact (|partial sums| < 2^53) and equals acc sx sw
+    rng = np.random.default_rng(15)
+    for bits in (8, 4):
+        c = synth.random_case_a16(41, 9, 160, 17, bits)
+        sx = 2.0 ** -20
+        sw = 2.0 ** -rng.integers(3, 12, size=c.N).astype(np.float64)
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(1.0, np.ones(c.N, np.float32), 1.0)
+        _, acc = orc.linear_a16(c.x, c.zx, packed, bits, c.N, m0, sh, 0, want_acc=True)
+        xd = (c.x.astype(np.float64) - c.zx) * sx
+        wd = c.w.astype(np.float64) * sw[:, None]
+        assert np.array_equal(xd @ wd.T, acc.astype(np.float64) * sx * sw[None, :])
+
+
+def pin_a16_requant_closed_form_and_saturation(orc: Oracle):
+    # multiplier 2^-t (M0 = 2^30, shift 30 + t) is a rounding right shift,
+    # for accumulators up to the 2^40 bound; the output saturates at the
+    # int16 ends, not the int8 ones
+    rng = random.Random(16)
+    for t in (1, 3, 9, 17, 25, 32):
+        for _ in range(300):
+            acc = rng.randint(-(1 << 40), 1 << 40) if rng.random() < 0.5 \
+                else rng.randint(-(3 << t) * 40000, (3 << t) * 40000)
+            zy = rng.randint(-32768, 32767)
+            want = max(-32768, min(32767, zy + ((acc + (1 << (t - 1))) >> t)))
+            assert orc.requant_one_a16(acc, 1 << 30, 30 + t, zy) == want, (t, acc, zy)
+    # exact ties, both signs
+    for s in range(1, 9):
+        for acc in range(-300, 301):
+            assert orc.requant_one_a16(acc, 1 << 30, s, 0) == _py_requant16(acc, 1 << 30, s, 0)
+    assert orc.requant_one_a16(1 << 39, (1 << 31) - 1, 31, 0) == 32767
+    assert orc.requant_one_a16(-(1 << 39), (1 << 31) - 1, 31, 0) == -32768
+    assert orc.requant_one_a16(200, 1 << 30, 30, 32700) == 32767
+    assert orc.requant_one_a16(-200, 1 << 30, 30, -32700) == -32768
+    assert orc.requant_one_a16(200, 1 << 30, 30, -100) == 100
+
+
+def pin_a16_requant_vs_eq4(orc: Oracle):
+    """The 16-bit layer against eq. 4 on the 16-bit output grid applied to
+    the real-valued layer output (float64): equal except at near-ties."""
+    c = synth.make_linear_a16(0, 0, 0, "q", 64, 256, 96, 8)
+    packed, _ = orc.pack(c.w, 8)
+    m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+    y, acc = orc.linear_a16(c.x, c.zx, packed, 8, c.N, m0, sh, c.zy, want_acc=True)
+    yf = acc.astype(np.float64) * (c.sx * c.sw.astype(np.float64))[None, :]
+    ref = np.clip(np.floor(yf / c.sy + 0.5) + c.zy, -32768, 32767)
+    diff = np.abs(y.astype(np.int64) - ref)
+    assert diff.max() <= 1
+    assert (diff != 0).mean() < 1e-3
+    assert np.mean(np.abs(y.astype(np.int64)) < 32767) > 0.9
+
+
 PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zero_point_identity,
                pin_exact_dequant, pin_requant_closed_form, pin_requant_ties, pin_requant_vs_eq4,
                pin_requant_params_bound, pin_asym_k1_exhaustive, pin_asym_int4_pairs,
-               pin_asym_identity, pin_asym_reduces_to_symmetric, pin_asym_exact_dequant]
+               pin_asym_identity, pin_asym_reduces_to_symmetric, pin_asym_exact_dequant,
+               pin_a16_k1_exhaustive, pin_a16_int4_pairs, pin_a16_matmul_and_brute_force,
+               pin_a16_large_accumulators, pin_a16_reduces_to_int8, pin_a16_byte_planes, pin_a16_exact_dequant,
+               pin_a16_requant_closed_form_and_saturation, pin_a16_requant_vs_eq4]
 
 
 # ----------------------------------------------------------------------------
@@ -436,6 +601,64 @@ def test_residual_add_saturates(O):
     assert O.residual_add(a, b).tolist() == [-128, -128, 5, 127, 127, -1, 0]
 
 
+def test_a16_k1_exhaustive(O):
+    pin_a16_k1_exhaustive(O)
+
+
+def test_a16_int4_pairs(O):
+    pin_a16_int4_pairs(O)
+
+
+def test_a16_matmul_and_brute_force(O):
+    pin_a16_matmul_and_brute_force(O)
+
+
+def test_a16_large_accumulators(O):
+    pin_a16_large_accumulators(O)
+
+
+def test_a16_reduces_to_int8(O):
+    pin_a16_reduces_to_int8(O)
+
+
+def test_a16_byte_planes(O):
+    pin_a16_byte_planes(O)
+
+
+def test_a16_exact_dequant(O):
+    pin_a16_exact_dequant(O)
+
+
+def test_a16_requant_closed_form_and_saturation(O):
+    pin_a16_requant_closed_form_and_saturation(O)
+
+
+def test_a16_requant_vs_eq4(O):
+    pin_a16_requant_vs_eq4(O)
+
+
+def test_a16_rejects_bad_arguments(O):
+    w = np.zeros((2, 32), np.int8)
+    packed, _ = O.pack(w, 8)
+    m0 = np.full(2, 1 << 30, np.int32)
+    sh = np.full(2, 31, np.int32)
+    x = np.zeros((1, 32), np.int16)
+    for zx, zy in ((32768, 0), (-32769, 0), (0, 32768), (0, -32769)):
+        with pytest.raises(oracle.OracleError):
+            O.linear_a16(x, zx, packed, 8, 2, m0, sh, zy)
+
+
+def test_a16_points_agree_with_full(O):
+    c = synth.random_case_a16(51, 11, 64, 23, 4)
+    packed, _ = O.pack(c.w, 4)
+    m0, sh = O.requant_params(c.sx, c.sw, c.sy)
+    y, acc = O.linear_a16(c.x, c.zx, packed, 4, c.N, m0, sh, c.zy, want_acc=True)
+    pts = np.array([[m, n] for m in range(0, 11, 3) for n in range(0, 23, 5)], np.int64)
+    yp, ap = O.linear_points_a16(c.x, c.zx, packed, 4, c.N, m0, sh, c.zy, pts)
+    assert np.array_equal(yp, y[pts[:, 0], pts[:, 1]])
+    assert np.array_equal(ap, acc[pts[:, 0], pts[:, 1]])
+
+
 MUTATIONS = [
     ("zero point sign", "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - zx;",
      "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] + zx;"),
@@ -461,6 +684,18 @@ MUTATIONS = [
      "int64_t wv = oracle_weight_at(packed, bits, K, n, k) + zw;"),
     ("weight zero point ignored", "int64_t acc = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, zw ? zw[n] : 0);",
      "int64_t acc = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, 0);"),
+    ("a16 zero point sign", "- (int64_t)zx;", "+ (int64_t)zx;"),
+    ("a16 activation narrowed to int8",
+     "int64_t x16 = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k]",
+     "int64_t x16 = (int64_t)(int8_t)x[(size_t)m * (size_t)ldx + (size_t)k]"),
+    ("a16 accumulator narrowed to int32", "acc16 += x16 * w16;",
+     "acc16 = (int32_t)(acc16 + x16 * w16);"),
+    ("a16 saturation at int8", "if (out > 32767) out = 32767;", "if (out > 127) out = 127;"),
+    ("a16 round half down", "return oracle_floor_div(2 * v + two_s, 2 * two_s);",
+     "return oracle_floor_div(2 * v + two_s - 1, 2 * two_s);"),
+    ("a16 output zero point dropped",
+     "__int128 out = (__int128)zy + oracle_round_shift(acc, M0, shift);",
+     "__int128 out = oracle_round_shift(acc, M0, shift);"),
 ]
 
 
