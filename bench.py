@@ -14,7 +14,8 @@ more than the 129 MB L2), so no step reads another's data from L2.
 Reported beside it, measured in the same run: W4A8 decode of the same block's
 linears at M = 1, 4, 16 (weight GB/s), rotating over 12 layers (264 MB); and
 both with asymmetric weights in the paper's settings (W8A8 per tensor with a
-per-channel down projection; W4A8 per channel).
+per-channel down projection; W4A8 per channel); and the 16-bit-activation
+baselines W8A16 (prefill) and W4A16 (decode at M = 1 and 8).
 
 Multi-GPU (torchrun, one rank per GPU): replicas only -- every rank runs the
 same workload on its own GPU, no collective on the data path; value is the
@@ -416,6 +417,95 @@ def run_asym_prefill(mq, torch, steps: int = 900, check_rows: int = 4):
             "parity_sample": {"rows": check_rows, "outputs": checked, "mismatches": mism}}
 
 
+class A16Block:
+    """Device-resident operands of one layer's seven linears with 16-bit
+    activations and outputs (int8 or int4 weights) at M tokens."""
+
+    def __init__(self, mq, torch, layer: int, m: int, bits: int, config: int, shared: bool):
+        self.cases = synth.block_linears_a16(config, m, bits, layer=layer, shared_input=shared)
+        xdev = {}
+        self.descs, self.y, self.keep = [], [], []
+        for c in self.cases:
+            if id(c.x) not in xdev:
+                xdev[id(c.x)] = torch.from_numpy(c.x).cuda()
+            packed, colsum = mq.pack_weights(c.w, bits)
+            m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
+            t = [torch.from_numpy(a).cuda() for a in (packed, colsum, m0, sh)]
+            y = torch.empty((m, c.N), dtype=torch.int16, device="cuda")
+            self.keep += t
+            self.y.append(y)
+            self.descs.append(mq.make_desc(xdev[id(c.x)], c.zx, t[0], t[1], c.N, t[2], t[3], c.zy,
+                                           y, bits, abits=16))
+        self.keep += list(xdev.values())
+        self.arr = (mq.LinearDesc * len(self.descs))(*self.descs)
+        self.ws_bytes = mq.workspace_size_batch(self.descs)
+        self.ws = torch.zeros(max(16, self.ws_bytes), dtype=torch.uint8, device="cuda")
+
+
+def _time_blocks(mq, torch, blocks, steps: int):
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+
+    def step(i):
+        b = blocks[i % len(blocks)]
+        rc = mq.lib.mq_linear_batch(b.arr, len(b.descs), b.ws.data_ptr(), b.ws_bytes, sp)
+        if rc:
+            raise RuntimeError(f"mq_linear_batch failed: {mq.status_string(rc)}")
+
+    for i in range(2 * len(blocks)):
+        step(i)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(steps):
+        step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in a 16-bit activation run")
+    step(0)  # layer 0 last, for the parity sample
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def run_a16(mq, torch, prefill_steps: int = 600, decode_steps: int = 480, check_rows: int = 4):
+    """W8A16 prefill of the block at M = 1024 (the paper's 16-bit-activation
+    baseline, Sec. 5.6) and W4A16 decode at M = 1 and 8, back-to-back batched
+    calls (split pre-pass + kernel each) rotating over layers larger than L2
+    together; the first rows of layer 0's prefill checked against the oracle."""
+    import oracle
+    oracle.build()
+    out = {}
+    blocks = [A16Block(mq, torch, layer, PREFILL_M, 8, CONFIG_ID_PREFILL, True)
+              for layer in range(PREFILL_LAYERS)]
+    ms = _time_blocks(mq, torch, blocks, prefill_steps)
+    mism = checked = 0
+    for j, c in enumerate(blocks[0].cases):
+        packed, _ = oracle.pack(c.w, 8)
+        m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
+        y = oracle.linear_a16(np.ascontiguousarray(c.x[:check_rows]), c.zx, packed, 8, c.N, m0,
+                              sh, c.zy)
+        got = blocks[0].y[j][:check_rows].cpu().numpy()
+        checked += y.size
+        mism += int(np.count_nonzero(got != y))
+    out["prefill_w8a16"] = {"us_per_block": round(ms * 1e3, 2),
+                            "tops": round(block_ops(PREFILL_M) / (ms * 1e-3) / 1e12, 1),
+                            "launches_per_step": 2, "steps": prefill_steps,
+                            "parity_sample": {"rows": check_rows, "outputs": checked,
+                                              "mismatches": mism}}
+    del blocks
+    wbytes = block_weight_bytes(4)
+    for m in (1, 8):
+        layers = [A16Block(mq, torch, layer, m, 4, CONFIG_ID_DECODE, False)
+                  for layer in range(DECODE_LAYERS)]
+        ms = _time_blocks(mq, torch, layers, decode_steps)
+        out[f"decode_w4a16_m{m}"] = {"us_per_block": round(ms * 1e3, 2),
+                                     "gbs": round(wbytes / ms / 1e6, 1),
+                                     "launches_per_step": 2, "steps": decode_steps}
+        del layers
+    return out
+
+
 # --------------------------------------------------------------------------- CPU oracle
 def oracle_sample(blocks_cases, rows: range, col_frac: float = 1.0):
     """Run the oracle on `rows` of every linear of one block; returns
@@ -523,6 +613,7 @@ def main():
     decode = run_decode(mq, torch)
     asym_pre = run_asym_prefill(mq, torch)
     asym_dec = run_decode(mq, torch, asym=True, ms=(1, 16))
+    a16 = run_a16(mq, torch)
     peaks = measured_peaks()
 
     ops = block_ops(PREFILL_M)
@@ -563,6 +654,9 @@ def main():
                               round(pre["total_ms"] / args.steps * 1e3, 2)},
         "asym_decode_w4a8": {"unit": "GB/s of int4 weights",
                              "weights": "asymmetric per channel", **asym_dec},
+        "a16": {"activations": "int16 in and out", "ops": "2 M K N per block", **a16,
+                "w8a8_us_per_block": round(pre["total_ms"] / args.steps * 1e3, 2),
+                "w4a8_m1_stream_us": decode["m1"]["stream_us"]},
     }
     if rank == 0 and world == 1:
         line["cpu_baseline"] = cpu_baseline(pre["blocks"], torch)

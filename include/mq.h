@@ -186,10 +186,60 @@ int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, int32_t zx,
                            int8_t *y, int ldy, void *stream);
 
 /*
+ * One quantized linear layer with 16-bit activations and outputs (W8A16): the
+ * paper's 16-bit-activation baseline and the width it keeps around
+ * non-linear operators (Sec. 4.1, Sec. 5.6, Table 5).  The 16-bit code range
+ * is the signed int16 range (the unsigned codes shifted by -32768).
+ *   x        : device int16 [M][ldx] (ldx in elements), ldx >= K
+ *   zx       : input zero point in [-32768, 32767]
+ *   packed, colsum, M0, shift: as mq_linear_w8a8 (int8 weights)
+ *   zy       : output zero point in [-32768, 32767]
+ *   y        : device int16 [M][ldy], ldy >= N, written
+ *   workspace: device, ws_bytes >= mq_workspace_size_a16(M, N, K, 8)
+ *   acc[m][n] = sum_k (x[m][k] - zx) * w[n][k]        (exact, |acc| < 2^40)
+ *   y[m][n]   = clamp(zy + floor(acc M0[n] / 2^shift[n] + 1/2), -32768, 32767)
+ * Method: with hi the signed high byte and lo the unsigned low byte of a
+ * code, x = 256 hi + (lo - 128) + 128.  A pre-pass writes the two int8
+ * planes hi and lo - 128 as rows 2m and 2m+1 of a [2M][K] int8 matrix in the
+ * workspace; the int8 kernels contract it exactly, and their epilogues form
+ * 256 S_hi + S_lo + (128 - zx) colsum[n] in int64 and requantize it.  2M <= 16
+ * runs the decode kernel, larger M the tensor-core kernel.
+ * Requirements: 0 <= M, N; 0 <= K <= MQ_MAX_K; K % 16 == 0; ldx % 8 == 0;
+ * x and packed 16-byte aligned.  No residual and no weight zero point.  The
+ * stream rules of mq_linear_w8a8 apply.
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_K_OVERFLOW, MQ_ERR_ALIGNMENT,
+ * MQ_ERR_WORKSPACE, MQ_ERR_CUDA.
+ */
+int mq_linear_w8a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                    const void *packed, const int32_t *colsum, int N,
+                    const int32_t *M0, const int32_t *shift, int32_t zy,
+                    int16_t *y, int ldy, void *workspace, size_t ws_bytes,
+                    void *stream);
+
+/* The same layer with int4 weights (W4A16).  Requires K % 32 == 0; otherwise
+ * as mq_linear_w8a16. */
+int mq_linear_w4a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                    const void *packed, const int32_t *colsum, int N,
+                    const int32_t *M0, const int32_t *shift, int32_t zy,
+                    int16_t *y, int ldy, void *workspace, size_t ws_bytes,
+                    void *stream);
+
+/*
+ * Device workspace bytes of one mq_linear_w8a16 / mq_linear_w4a16 call: the
+ * decode workspace (see mq_workspace_size) when 1 <= 2M <= 16, followed by
+ * the two int8 planes of x (2 M K bytes, rounded up to 128).  The decode part
+ * follows the contract of mq_workspace_size; the planes are scratch,
+ * overwritten by each call.
+ * Errors: MQ_ERR_INVALID_ARG.
+ */
+int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
+
+/*
  * Several independent linears in as few launches as possible (one per kernel
  * family): a decoder block's projections that read the same activations, or
  * a whole step's worth of small decode GEMVs.  Each descriptor has the
- * meaning and requirements of one mq_linear_w8a8 / mq_linear_w4a8 call; in
+ * meaning and requirements of one mq_linear_w8a8 / mq_linear_w4a8 call (with
+ * abits 16: mq_linear_w8a16 / mq_linear_w4a16); in
  * addition `residual` (device int8 [M][ldy], may be NULL) is added to the
  * requantized output with int8 saturation, the int8 residual glue between
  * chained layers.  Descriptors must not write overlapping outputs.
@@ -212,17 +262,18 @@ int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, int32_t zx,
  * reported, nothing is launched when any descriptor is invalid.
  */
 typedef struct mq_linear_desc {
-    const int8_t *x;
+    const void *x;          /* int8 [M][ldx], or int16 with abits == 16 */
     const void *packed;
     const int32_t *colsum;
     const int32_t *M0;
     const int32_t *shift;
-    const int8_t *residual; /* may be NULL */
-    const int32_t *zw;      /* may be NULL: symmetric weights */
-    int8_t *y;
+    const int8_t *residual; /* may be NULL; int8 activations only */
+    const int32_t *zw;      /* may be NULL: symmetric weights; int8 activations only */
+    void *y;                /* int8 [M][ldy], or int16 with abits == 16 */
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;
-    int32_t bits; /* 8 or 4 */
+    int32_t bits;  /* weight bits: 8 or 4 */
+    int32_t abits; /* activation and output bits: 8 (0 reads as 8) or 16, see mq_linear_w8a16 */
 } mq_linear_desc;
 
 /* Largest K for int8 weights with a weight zero point: 255 * 255 * K < 2^31. */
@@ -231,13 +282,19 @@ typedef struct mq_linear_desc {
 /*
  * Device workspace bytes one mq_linear_batch call over `descs` needs: the
  * decode workspace (see mq_workspace_size) if any descriptor has
- * 1 <= M <= 16, plus 4*M bytes (rounded up to 16) for every distinct input
- * (x, M, K, ldx) of the descriptors with M > 16 and a weight zero point, which
- * holds rowsum(x) of its tokens (filled by the call; descriptors reading the
- * same input, e.g. q/k/v/gate/up of one block, share it).  0 when neither
- * applies.  The contract of mq_workspace_size
- * holds for the whole buffer.
- * Errors: MQ_ERR_INVALID_ARG (null pointers, count out of range, bad bits).
+ * 1 <= M <= 16 (abits 8) or 1 <= 2M <= 16 (abits 16); plus 4*M bytes
+ * (rounded up to 16) for every distinct input (x, M, K, ldx) of the
+ * descriptors with M > 16 and a weight zero point, which holds rowsum(x) of
+ * its tokens; plus 2*M*K bytes (rounded up to 128) for every distinct input
+ * of the descriptors with abits 16, which holds its two int8 planes (both
+ * filled by the call; descriptors reading the same input, e.g. q/k/v/gate/up
+ * of one block, share them).  0 when none applies.  The decode region (the
+ * first mq_workspace_size bytes, when present) follows the contract of
+ * mq_workspace_size: zero-filled before first use and left zero by every
+ * call that completes; the rowsum and plane regions are scratch, overwritten
+ * by each call.
+ * Errors: MQ_ERR_INVALID_ARG (null pointers, count out of range, bad bits or
+ * abits).
  */
 int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *bytes);
 

@@ -351,7 +351,97 @@ __device__ __forceinline__ void compute_stage(const uint8_t *ring, int warp, int
     }
 }
 
-template <int BITS, int NT>
+// Exchange buffer of the 16-bit epilogue, laid over the reduction buffer
+// (free once every thread has read its slots): the final sums per plane row
+// and unit row, row stride 68 words (conflict-free for both the fragment-
+// ordered writes and the row-ordered reads).
+constexpr int YV_STRIDE = UNIT_ROWS + 4;
+
+// The 16-bit epilogue of one piece.  Every consumer thread calls it (its
+// barriers are unconditional); `ok` / `tok` say whether the thread holds
+// valid slots.  Sums are formed as in the int8 epilogue (including the split
+// unit protocol), then the CTA that finishes the unit writes them to the
+// exchange buffer and combines plane rows 2j, 2j + 1 of every unit row:
+// sum((x - zx) w) = 256 S(2j) + S(2j + 1) + (128 - zx) colsum, requantized
+// to int16.
+template <int BITS, int NT, class SM>
+__device__ __forceinline__ void a16_epilogue(const Params &P, SM &s, const DecProb &p, int rb,
+                                             bool whole, bool ok, int tok, int32_t xsum, int e0,
+                                             int ln, int S, int G, int cta) {
+    using C = Cfg<BITS>;
+    const int u_begin = p.tile_begin + rb * p.tiles_m, u_end = u_begin + p.tiles_m;
+    const int cf = whole ? cta : cta_of(u_begin, S, G);
+    const int cl = whole ? cta : cta_of(u_end - 1, S, G);
+    const bool finisher = cta == cf;
+    bool have = ok && tok < p.M;
+    uint32_t v[2 * NT];
+    int rows[2 * NT];
+#pragma unroll
+    for (int q = 0; q < 2 * NT; ++q) {
+        const int e = e0 + 8 * q;
+        rows[q] = ((e >> 2) / NT) * 16 + (ln >> 2) + ((e & 2) ? 8 : 0);
+        int32_t sum = 0;
+        if (have) {
+#pragma unroll
+            for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
+        }
+        v[q] = (uint32_t)sum - (uint32_t)(C::BIAS * xsum);
+    }
+    if (have && !whole) {
+        if (!finisher) {
+            int2 *mine = P.ws + (size_t)cta * UNIT_ROWS * 16;
+#pragma unroll
+            for (int q = 0; q < 2 * NT; ++q) st_relaxed_v2(mine + rows[q] * 16 + tok, v[q], P.epoch);
+            have = false;
+        } else {
+            bool got = true;
+            for (int c = cf + 1; got && c <= cl; ++c) {
+                const int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
+#pragma unroll
+                for (int q = 0; q < 2 * NT; ++q) {
+                    int32_t x = 0;
+                    got = got && poll_entry(src + rows[q] * 16 + tok, P.epoch, x, &s.abort,
+                                            P.status);
+                    v[q] += (uint32_t)x;
+                }
+            }
+            if (got) {
+                for (int c = cf + 1; c <= cl; ++c) {
+                    int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
+#pragma unroll
+                    for (int q = 0; q < 2 * NT; ++q) st_relaxed_v2(src + rows[q] * 16 + tok, 0u, 0u);
+                }
+            }
+            have = got;
+        }
+    }
+    int32_t *yv = &s.part[0][0][0];
+    cons_sync();  // every read of the reduction buffer is done
+    if (finisher && have) {
+#pragma unroll
+        for (int q = 0; q < 2 * NT; ++q) yv[tok * YV_STRIDE + rows[q]] = (int32_t)v[q];
+    }
+    cons_sync();
+    if (finisher && !s.abort) {
+        const int ntok = p.M >> 1;
+        int16_t *y = reinterpret_cast<int16_t *>(p.y);
+        for (int i = threadIdx.x; i < UNIT_ROWS * ntok; i += CONS_THREADS) {
+            const int row = i & (UNIT_ROWS - 1), j = i / UNIT_ROWS;
+            const int n = rb * UNIT_ROWS + row;
+            if (n >= p.N) continue;
+            const int64_t a = 256 * (int64_t)yv[(2 * j) * YV_STRIDE + row] +
+                              (int64_t)yv[(2 * j + 1) * YV_STRIDE + row] +
+                              (int64_t)(128 - p.zx) * (int64_t)s.row_corr[row];
+            y[(size_t)j * (size_t)p.ldy + n] =
+                (int16_t)mq_requant16(a, s.row_m0[row], s.row_shift[row], p.zy);
+        }
+    }
+}
+
+// A16: every problem has 16-bit activations (Problem::a16): x is the plane
+// matrix (rows 2m, 2m + 1 = high and low planes of token m) and the outputs
+// are int16, formed from row pairs after an exchange through shared memory.
+template <int BITS, int NT, bool A16>
 __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constant__ Params P) {
     using C = Cfg<BITS>;
     using SM = Smem<NT>;
@@ -525,8 +615,11 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             if (threadIdx.x < UNIT_ROWS) {
                 // sum((x - zx)(w - zw)) = sum(x w) - zx colsum - zw sum(x) + K zx zw;
                 // the zw sum(x) term is taken per piece with the bias below
+                // (16-bit activations: colsum itself, the combine applies (128 - zx))
                 s.row_corr[threadIdx.x] =
-                    (int32_t)((uint32_t)(p.zx * prm_cs) - (uint32_t)p.K * (uint32_t)(p.zx * prm_zw));
+                    A16 ? prm_cs
+                        : (int32_t)((uint32_t)(p.zx * prm_cs) -
+                                    (uint32_t)p.K * (uint32_t)(p.zx * prm_zw));
                 s.row_zw[threadIdx.x] = prm_zw;
                 s.row_m0[threadIdx.x] = prm_m0;
                 s.row_shift[threadIdx.x] = prm_sh;
@@ -542,7 +635,9 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
 #pragma unroll
                 for (int w = 0; w < CONS_WARPS; ++w) xsum += s.xpart[w][tok];
             }
-            if (ok && whole) {
+            if constexpr (A16) {
+                a16_epilogue<BITS, NT>(P, s, p, rb, whole, ok, tok, xsum, e0, ln, S, G, cta);
+            } else if (ok && whole) {
                 // the unit is entirely this CTA's: requantize and store
 #pragma unroll
                 for (int q = 0; q < 2 * NT; ++q) {
@@ -658,10 +753,10 @@ uint32_t next_epoch() {
     return e;
 }
 
-template <int BITS, int NT>
+template <int BITS, int NT, bool A16>
 int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t stream) {
     using C = Cfg<BITS>;
-    auto kern = decode_kernel<BITS, NT>;
+    auto kern = decode_kernel<BITS, NT, A16>;
     static int attr_done = -1;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
@@ -721,7 +816,7 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
 
 }  // namespace decode
 
-// All problems passed here have the same bits and M <= DECODE_MAX_M;
+// All problems passed here have the same bits and a16 and M <= DECODE_MAX_M;
 // `workspace` holds DECODE_WS_BYTES, zero-filled.
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream) {
     using namespace decode;
@@ -731,9 +826,18 @@ int launch_decode(const Problem *probs, int count, void *workspace, void *stream
     const bool nt2 = max_m > 8;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     int32_t *ws = static_cast<int32_t *>(workspace);
+    if (probs[0].a16) {
+        if (probs[0].bits == 4)
+            return nt2 ? launch_t<4, 2, true>(probs, count, ws, s)
+                       : launch_t<4, 1, true>(probs, count, ws, s);
+        return nt2 ? launch_t<8, 2, true>(probs, count, ws, s)
+                   : launch_t<8, 1, true>(probs, count, ws, s);
+    }
     if (probs[0].bits == 4)
-        return nt2 ? launch_t<4, 2>(probs, count, ws, s) : launch_t<4, 1>(probs, count, ws, s);
-    return nt2 ? launch_t<8, 2>(probs, count, ws, s) : launch_t<8, 1>(probs, count, ws, s);
+        return nt2 ? launch_t<4, 2, false>(probs, count, ws, s)
+                   : launch_t<4, 1, false>(probs, count, ws, s);
+    return nt2 ? launch_t<8, 2, false>(probs, count, ws, s)
+               : launch_t<8, 1, false>(probs, count, ws, s);
 }
 
 }  // namespace mq

@@ -14,11 +14,18 @@ namespace {
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Validate one linear problem; on success fill the kernel-side Problem.
+int abits_of(const mq_linear_desc &d) { return d.abits == 0 ? 8 : d.abits; }
+
+// Validate one linear problem; on success fill the kernel-side Problem (for
+// 16-bit activations, x is filled in later with the planes' address).
 int check_desc(const mq_linear_desc &d, mq::Problem &out) {
+    const int ab = abits_of(d);
     if (d.bits != 8 && d.bits != 4) return MQ_ERR_INVALID_ARG;
+    if (ab != 8 && ab != 16) return MQ_ERR_INVALID_ARG;
     if (d.M < 0 || d.N < 0 || d.K < 0) return MQ_ERR_INVALID_ARG;
-    if (d.zx < -128 || d.zx > 127 || d.zy < -128 || d.zy > 127) return MQ_ERR_INVALID_ARG;
+    const int32_t zlo = ab == 8 ? -128 : -32768, zhi = ab == 8 ? 127 : 32767;
+    if (d.zx < zlo || d.zx > zhi || d.zy < zlo || d.zy > zhi) return MQ_ERR_INVALID_ARG;
+    if (ab == 16 && (d.residual || d.zw)) return MQ_ERR_INVALID_ARG;
     if (d.K > MQ_MAX_K) return MQ_ERR_K_OVERFLOW;
     if (d.zw && d.bits == 8 && d.K > MQ_MAX_K_ASYM8) return MQ_ERR_K_OVERFLOW;
     if (d.M > 0 && d.N > 0) {
@@ -26,11 +33,12 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
         if (d.K > 0) {  // with K == 0 neither x nor the weights are read
             if (!d.x || !d.packed || d.ldx < d.K) return MQ_ERR_INVALID_ARG;
             const int kq = d.bits == 8 ? 16 : 32;  // k per 16-byte weight segment
-            if (d.K % kq != 0 || d.ldx % 16 != 0) return MQ_ERR_ALIGNMENT;
+            const int lq = ab == 8 ? 16 : 8;       // x elements per 16 bytes
+            if (d.K % kq != 0 || d.ldx % lq != 0) return MQ_ERR_ALIGNMENT;
             if (!aligned16(d.x) || !aligned16(d.packed)) return MQ_ERR_ALIGNMENT;
         }
     }
-    out.x = d.x;
+    out.x = ab == 8 ? static_cast<const int8_t *>(d.x) : nullptr;
     out.w = static_cast<const uint8_t *>(d.packed);
     out.colsum = d.colsum;
     out.M0 = d.M0;
@@ -38,15 +46,16 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     out.residual = d.residual;
     out.zw = d.zw;
     out.rowsum = nullptr;
-    out.y = d.y;
-    out.M = d.M;
+    out.y = static_cast<int8_t *>(d.y);
+    out.M = ab == 8 ? d.M : 2 * d.M;  // 16 bits: rows of the plane matrix
     out.N = d.N;
     out.K = d.K;
-    out.ldx = d.ldx;
+    out.ldx = ab == 8 ? d.ldx : d.K;
     out.ldy = d.ldy;
     out.zx = d.zx;
     out.zy = d.zy;
     out.bits = d.bits;
+    out.a16 = ab == 16;
     out.tile_begin = 0;
     out.tiles_m = 0;
     return MQ_OK;
@@ -54,82 +63,120 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
 
 size_t align16(size_t v) { return (v + 15) & ~static_cast<size_t>(15); }
 
+size_t align128(size_t v) { return (v + 127) & ~static_cast<size_t>(127); }
+
+// A decode shape: at most DECODE_MAX_M rows of the (plane) matrix.
+bool is_decode(const mq_linear_desc &d) {
+    const int64_t rows = abits_of(d) == 16 ? 2LL * d.M : d.M;
+    return rows > 0 && rows <= mq::DECODE_MAX_M;
+}
+
 // Workspace layout of one batch: the decode region first (if any decode
 // shape), then one rowsum(x) array per distinct input (x, M, K, ldx) of the
-// prefill descriptors with a weight zero point, in order of first use.
-// `jobs` (may be null) receives those inputs and `offsets` their byte
-// offsets from the start of the rowsum region.
-size_t batch_workspace(const mq_linear_desc *descs, int count, bool *any_decode,
-                       std::vector<mq::RowsumJob> *jobs, std::vector<size_t> *offsets) {
-    bool dec = false;
-    std::vector<mq::RowsumJob> uniq;
-    std::vector<size_t> offs;
-    size_t rows = 0;
+// prefill descriptors with a weight zero point, then one [2M][K] int8 plane
+// matrix per distinct input of the 16-bit descriptors, each in order of
+// first use, with offsets relative to the end of the decode region.
+struct Plan {
+    bool any_decode = false;
+    std::vector<mq::RowsumJob> rowsum;
+    std::vector<size_t> rowsum_off;
+    std::vector<mq::SplitJob> split;
+    std::vector<size_t> split_off;
+    size_t bytes = 0;
+};
+
+template <class J>
+int find_job(const std::vector<J> &jobs, const void *x, int M, int K, int ldx) {
+    for (size_t i = 0; i < jobs.size(); ++i)
+        if (jobs[i].x == x && jobs[i].M == M && jobs[i].K == K && jobs[i].ldx == ldx) return (int)i;
+    return -1;
+}
+
+Plan batch_plan(const mq_linear_desc *descs, int count) {
+    Plan pl;
+    size_t off = 0;
     for (int i = 0; i < count; ++i) {
         const mq_linear_desc &d = descs[i];
         if (d.M <= 0 || d.N <= 0) continue;
-        if (d.M <= mq::DECODE_MAX_M) {
-            dec = true;
-            continue;
+        if (is_decode(d)) pl.any_decode = true;
+        if (d.K <= 0) continue;
+        if (abits_of(d) == 8 && d.zw && !is_decode(d) &&
+            find_job(pl.rowsum, d.x, d.M, d.K, d.ldx) < 0) {
+            mq::RowsumJob j{};
+            j.x = static_cast<const int8_t *>(d.x);
+            j.M = d.M;
+            j.K = d.K;
+            j.ldx = d.ldx;
+            pl.rowsum.push_back(j);
+            pl.rowsum_off.push_back(off);
+            off += align16(4 * (size_t)d.M);
         }
-        if (!d.zw || d.K <= 0) continue;
-        bool seen = false;
-        for (const auto &j : uniq)
-            seen |= j.x == d.x && j.M == d.M && j.K == d.K && j.ldx == d.ldx;
-        if (seen) continue;
-        mq::RowsumJob j{};
-        j.x = d.x;
+    }
+    for (int i = 0; i < count; ++i) {
+        const mq_linear_desc &d = descs[i];
+        if (d.M <= 0 || d.N <= 0 || d.K <= 0 || abits_of(d) != 16) continue;
+        if (find_job(pl.split, d.x, d.M, d.K, d.ldx) >= 0) continue;
+        off = align128(off);
+        mq::SplitJob j{};
+        j.x = static_cast<const int16_t *>(d.x);
         j.M = d.M;
         j.K = d.K;
         j.ldx = d.ldx;
-        uniq.push_back(j);
-        offs.push_back(rows);
-        rows += align16(4 * (size_t)d.M);
+        pl.split.push_back(j);
+        pl.split_off.push_back(off);
+        off += align128(2 * (size_t)d.M * (size_t)d.K);
     }
-    if (any_decode) *any_decode = dec;
-    if (jobs) *jobs = uniq;
-    if (offsets) *offsets = offs;
-    return (dec ? mq::DECODE_WS_BYTES : 0) + rows;
+    pl.bytes = (pl.any_decode ? mq::DECODE_WS_BYTES : 0) + off;
+    return pl;
 }
 
 int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws_bytes,
               void *stream) {
     if (!descs || count < 1 || count > MQ_MAX_BATCH) return MQ_ERR_INVALID_ARG;
-    std::vector<mq::Problem> pre, dec8, dec4;
-    pre.reserve(count);
+    std::vector<mq::Problem> probs(count);
     for (int i = 0; i < count; ++i) {
-        mq::Problem p{};
-        const int rc = check_desc(descs[i], p);
+        const int rc = check_desc(descs[i], probs[i]);
         if (rc != MQ_OK) return rc;
-        if (p.M == 0 || p.N == 0) continue;  // nothing to compute or write
-        if (p.M <= mq::DECODE_MAX_M)
-            (p.bits == 8 ? dec8 : dec4).push_back(p);
-        else
-            pre.push_back(p);
     }
     // the decode kernel combines split 64-row units in the workspace; prefill
-    // descriptors with a weight zero point read rowsum(x) from there
-    bool any_decode = false;
-    std::vector<mq::RowsumJob> jobs;
-    std::vector<size_t> offsets;
-    const size_t need = batch_workspace(descs, count, &any_decode, &jobs, &offsets);
-    if (need > 0 && (!workspace || ws_bytes < need || !aligned16(workspace)))
+    // descriptors with a weight zero point read rowsum(x) from there, 16-bit
+    // descriptors their int8 planes
+    Plan pl = batch_plan(descs, count);
+    if (pl.bytes > 0 && (!workspace || ws_bytes < pl.bytes || !aligned16(workspace)))
         return MQ_ERR_WORKSPACE;
-    uint8_t *region = static_cast<uint8_t *>(workspace) + (any_decode ? mq::DECODE_WS_BYTES : 0);
-    for (size_t i = 0; i < jobs.size(); ++i)
-        jobs[i].out = reinterpret_cast<int32_t *>(region + offsets[i]);
-    for (auto &p : pre) {
-        if (!p.zw || p.K == 0) continue;
-        for (const auto &j : jobs)
-            if (j.x == p.x && j.M == p.M && j.K == p.K && j.ldx == p.ldx) p.rowsum = j.out;
+    uint8_t *region = static_cast<uint8_t *>(workspace) + (pl.any_decode ? mq::DECODE_WS_BYTES : 0);
+    for (size_t i = 0; i < pl.rowsum.size(); ++i)
+        pl.rowsum[i].out = reinterpret_cast<int32_t *>(region + pl.rowsum_off[i]);
+    for (size_t i = 0; i < pl.split.size(); ++i)
+        pl.split[i].out = reinterpret_cast<int8_t *>(region + pl.split_off[i]);
+    // kernel families: prefill (int8 / 16-bit activations), decode by weight
+    // bits and activation width
+    std::vector<mq::Problem> pre8, pre16, dec[2][2];  // dec[bits == 8][a16]
+    for (int i = 0; i < count; ++i) {
+        mq::Problem &p = probs[i];
+        const mq_linear_desc &d = descs[i];
+        if (p.M == 0 || p.N == 0) continue;  // nothing to compute or write
+        if (p.K > 0 && p.zw && !p.a16 && !is_decode(d)) {
+            const int j = find_job(pl.rowsum, d.x, d.M, d.K, d.ldx);
+            p.rowsum = pl.rowsum[j].out;
+        }
+        if (p.K > 0 && p.a16) p.x = pl.split[find_job(pl.split, d.x, d.M, d.K, d.ldx)].out;
+        if (is_decode(d))
+            dec[p.bits == 8][p.a16].push_back(p);
+        else
+            (p.a16 ? pre16 : pre8).push_back(p);
     }
     int rc = MQ_OK;
-    if (!jobs.empty()) rc = mq::launch_rowsum(jobs.data(), (int)jobs.size(), stream);
-    if (rc == MQ_OK && !pre.empty()) rc = mq::launch_prefill(pre.data(), (int)pre.size(), stream);
-    if (rc == MQ_OK && !dec8.empty())
-        rc = mq::launch_decode(dec8.data(), (int)dec8.size(), workspace, stream);
-    if (rc == MQ_OK && !dec4.empty())
-        rc = mq::launch_decode(dec4.data(), (int)dec4.size(), workspace, stream);
+    if (!pl.rowsum.empty()) rc = mq::launch_rowsum(pl.rowsum.data(), (int)pl.rowsum.size(), stream);
+    if (rc == MQ_OK && !pl.split.empty())
+        rc = mq::launch_split16(pl.split.data(), (int)pl.split.size(), stream);
+    if (rc == MQ_OK && !pre8.empty()) rc = mq::launch_prefill(pre8.data(), (int)pre8.size(), stream);
+    if (rc == MQ_OK && !pre16.empty())
+        rc = mq::launch_prefill(pre16.data(), (int)pre16.size(), stream);
+    for (int b = 1; b >= 0; --b)
+        for (int a = 0; a < 2; ++a)
+            if (rc == MQ_OK && !dec[b][a].empty())
+                rc = mq::launch_decode(dec[b][a].data(), (int)dec[b][a].size(), workspace, stream);
     return rc;
 }
 
@@ -153,6 +200,29 @@ int single(int bits, const int8_t *x, int M, int K, int ldx, int32_t zx, const v
     d.zx = zx;
     d.zy = zy;
     d.bits = bits;
+    d.abits = 8;
+    return run_batch(&d, 1, workspace, ws_bytes, stream);
+}
+
+int single_a16(int bits, const int16_t *x, int M, int K, int ldx, int32_t zx, const void *packed,
+               const int32_t *colsum, int N, const int32_t *M0, const int32_t *shift, int32_t zy,
+               int16_t *y, int ldy, void *workspace, size_t ws_bytes, void *stream) {
+    mq_linear_desc d{};
+    d.x = x;
+    d.packed = packed;
+    d.colsum = colsum;
+    d.M0 = M0;
+    d.shift = shift;
+    d.y = y;
+    d.M = M;
+    d.N = N;
+    d.K = K;
+    d.ldx = ldx;
+    d.ldy = ldy;
+    d.zx = zx;
+    d.zy = zy;
+    d.bits = bits;
+    d.abits = 16;
     return run_batch(&d, 1, workspace, ws_bytes, stream);
 }
 
@@ -292,10 +362,42 @@ int mq_linear_w4a8(const int8_t *x, int M, int K, int ldx, int32_t zx, const voi
 
 int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *bytes) {
     if (!descs || !bytes || count < 1 || count > MQ_MAX_BATCH) return MQ_ERR_INVALID_ARG;
-    for (int i = 0; i < count; ++i)
+    for (int i = 0; i < count; ++i) {
         if (descs[i].bits != 8 && descs[i].bits != 4) return MQ_ERR_INVALID_ARG;
-    *bytes = batch_workspace(descs, count, nullptr, nullptr, nullptr);
+        if (abits_of(descs[i]) != 8 && abits_of(descs[i]) != 16) return MQ_ERR_INVALID_ARG;
+    }
+    *bytes = batch_plan(descs, count).bytes;
     return MQ_OK;
+}
+
+int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes) {
+    if (!bytes || M < 0 || N < 0 || K < 0 || (bits != 8 && bits != 4)) return MQ_ERR_INVALID_ARG;
+    mq_linear_desc d{};
+    d.x = reinterpret_cast<const void *>(16);  // a placeholder address: only sizes are planned
+    d.M = M;
+    d.N = N;
+    d.K = K;
+    d.ldx = K;
+    d.bits = bits;
+    d.abits = 16;
+    *bytes = batch_plan(&d, 1).bytes;
+    return MQ_OK;
+}
+
+int mq_linear_w8a16(const int16_t *x, int M, int K, int ldx, int32_t zx, const void *packed,
+                    const int32_t *colsum, int N, const int32_t *M0, const int32_t *shift,
+                    int32_t zy, int16_t *y, int ldy, void *workspace, size_t ws_bytes,
+                    void *stream) {
+    return single_a16(8, x, M, K, ldx, zx, packed, colsum, N, M0, shift, zy, y, ldy, workspace,
+                      ws_bytes, stream);
+}
+
+int mq_linear_w4a16(const int16_t *x, int M, int K, int ldx, int32_t zx, const void *packed,
+                    const int32_t *colsum, int N, const int32_t *M0, const int32_t *shift,
+                    int32_t zy, int16_t *y, int ldy, void *workspace, size_t ws_bytes,
+                    void *stream) {
+    return single_a16(4, x, M, K, ldx, zx, packed, colsum, N, M0, shift, zy, y, ldy, workspace,
+                      ws_bytes, stream);
 }
 
 int mq_linear_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws_bytes,

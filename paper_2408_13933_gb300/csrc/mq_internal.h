@@ -26,6 +26,11 @@ struct Problem {
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;
     int32_t bits;
+    // 16-bit activations: x is the [2M'][K] int8 plane matrix of the M' int16
+    // tokens (rows 2m = high bytes, 2m + 1 = low bytes - 128, ldx = K), M is
+    // its row count 2M', y points to int16 [M'][ldy], and the epilogues form
+    // 256 S(2m) + S(2m + 1) + (128 - zx) colsum.
+    int32_t a16;
     int32_t tile_begin;  // first global tile / block index of this problem
     int32_t tiles_m;     // prefill: number of 128-row tiles
 };
@@ -49,7 +54,9 @@ constexpr int DECODE_MAX_PROBLEMS = 64;
 int *device_status_ptr();
 int *pack_status_ptr();
 
-// Launchers (asynchronous on `stream`); return MQ_OK or MQ_ERR_CUDA.
+// Launchers (asynchronous on `stream`); return MQ_OK or MQ_ERR_CUDA.  The
+// problems of one launch_prefill call have the same a16; those of one
+// launch_decode call the same bits and a16.
 int launch_prefill(const Problem *probs, int count, void *stream);
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream);
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
@@ -63,5 +70,15 @@ struct RowsumJob {
 };
 constexpr int ROWSUM_MAX_JOBS = 64;  // jobs per launch (kernel parameter space)
 int launch_rowsum(const RowsumJob *jobs, int count, void *stream);
+
+// One distinct int16 input of a batch and where its two int8 planes go:
+// out row 2m = high bytes of x row m, row 2m + 1 = low bytes - 128 (pitch K).
+struct SplitJob {
+    const int16_t *x;
+    int8_t *out;  // [2M][K] in the workspace
+    int32_t M, K, ldx;
+};
+constexpr int SPLIT_MAX_JOBS = 64;
+int launch_split16(const SplitJob *jobs, int count, void *stream);
 
 }  // namespace mq

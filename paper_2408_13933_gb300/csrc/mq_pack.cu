@@ -172,4 +172,83 @@ int launch_rowsum(const RowsumJob *jobs, int count, void *stream) {
     return MQ_OK;
 }
 
+namespace split16 {
+
+constexpr int THREADS = 256;
+
+struct Params {
+    SplitJob job[SPLIT_MAX_JOBS];
+    int64_t block_begin[SPLIT_MAX_JOBS + 1];  // first block of each job, then the total
+    int32_t count;
+};
+
+// The two int8 planes of 16-bit activation codes: with hi the signed high
+// byte and lo the unsigned low byte, x = 256 hi + (lo - 128) + 128, so row 2m
+// of `out` gets the hi bytes of x row m and row 2m + 1 the bytes lo ^ 0x80
+// (= lo - 128 as a signed byte).  One thread per 16 codes of a row (two
+// 16-byte loads, two 16-byte stores); K is a multiple of 16, ldx of 8, and x
+// and out are 16-byte aligned (the library's validation).  Launched with
+// programmatic stream serialization: x is read only after griddep_wait.
+__global__ void __launch_bounds__(THREADS) split16_kernel(const __grid_constant__ Params P) {
+    griddep_wait();
+    griddep_launch_dependents();
+    int j = 0;
+    while (j + 1 < P.count && (int64_t)blockIdx.x >= P.block_begin[j + 1]) ++j;
+    const SplitJob &q = P.job[j];
+    const int64_t g = ((int64_t)blockIdx.x - P.block_begin[j]) * THREADS + threadIdx.x;
+    const int per_row = q.K >> 4;
+    const int64_t row = g / per_row;
+    if (row >= q.M) return;
+    const int c = (int)(g - row * per_row);
+    const uint4 *src = reinterpret_cast<const uint4 *>(q.x + (size_t)row * (size_t)q.ldx + 16 * c);
+    const uint4 a = __ldg(src), b = __ldg(src + 1);
+    // bytes 1, 3 of each 32-bit word are the high bytes of its two codes,
+    // bytes 0, 2 the low bytes
+    uint4 hi, lo;
+    hi.x = __byte_perm(a.x, a.y, 0x7531);
+    hi.y = __byte_perm(a.z, a.w, 0x7531);
+    hi.z = __byte_perm(b.x, b.y, 0x7531);
+    hi.w = __byte_perm(b.z, b.w, 0x7531);
+    lo.x = __byte_perm(a.x, a.y, 0x6420) ^ 0x80808080u;
+    lo.y = __byte_perm(a.z, a.w, 0x6420) ^ 0x80808080u;
+    lo.z = __byte_perm(b.x, b.y, 0x6420) ^ 0x80808080u;
+    lo.w = __byte_perm(b.z, b.w, 0x6420) ^ 0x80808080u;
+    int8_t *dst = q.out + (size_t)(2 * row) * (size_t)q.K + 16 * c;
+    *reinterpret_cast<uint4 *>(dst) = hi;
+    *reinterpret_cast<uint4 *>(dst + q.K) = lo;
+}
+
+}  // namespace split16
+
+int launch_split16(const SplitJob *jobs, int count, void *stream) {
+    for (int base = 0; base < count; base += SPLIT_MAX_JOBS) {
+        split16::Params P{};
+        const int n = count - base < SPLIT_MAX_JOBS ? count - base : SPLIT_MAX_JOBS;
+        int64_t blocks = 0;
+        for (int i = 0; i < n; ++i) {
+            P.job[i] = jobs[base + i];
+            P.block_begin[i] = blocks;
+            const int64_t groups = (int64_t)jobs[base + i].M * (jobs[base + i].K / 16);
+            blocks += (groups + split16::THREADS - 1) / split16::THREADS;
+        }
+        if (blocks == 0) continue;
+        if (blocks > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
+        P.block_begin[n] = blocks;
+        P.count = n;
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)blocks, 1, 1);
+        cfg.blockDim = dim3(split16::THREADS, 1, 1);
+        cfg.dynamicSmemBytes = 0;
+        cfg.stream = static_cast<cudaStream_t>(stream);
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&cfg, split16::split16_kernel, P) != cudaSuccess)
+            return MQ_ERR_CUDA;
+    }
+    return MQ_OK;
+}
+
 }  // namespace mq

@@ -212,10 +212,31 @@ __device__ __forceinline__ void store_channel(const uint32_t (&acc)[64], int32_t
     }
 }
 
+// 16-bit activations: columns 2j and 2j + 1 of the thread's 64 are the high
+// and low planes of token j, so sum((x - zx) w) = 256 S(2j) + S(2j + 1) +
+// (128 - zx) colsum (c16); requantize and store its n16 int16 outputs.  Kept
+// out of line: its 64-bit arithmetic would otherwise crowd the registers of
+// the accumulation loop (the call passes the sums through the stack once per
+// tile).
+__device__ __noinline__ void store_channel16(const uint32_t (&acc)[64], int64_t c16, int32_t m0,
+                                             int32_t sh, int32_t zy, int16_t *yp, size_t ldy,
+                                             int n16) {
+#pragma unroll 4
+    for (int j = 0; j < 32; ++j)
+        if (j < n16) {
+            const int64_t a = 256 * (int64_t)(int32_t)acc[2 * j] +
+                              (int64_t)(int32_t)acc[2 * j + 1] + c16;
+            yp[(size_t)j * ldy] = (int16_t)mq_requant16(a, m0, sh, zy);
+        }
+}
+
 // Barrier scopes: arrivals from the other CTA are releases at cluster scope
 // (st.async complete_tx, mbarrier.arrive.release.cluster, multicast commits),
 // so the data they publish is visible cluster-wide before the phase can
 // complete; waiters acquire at CTA scope, which is far cheaper per wait.
+// A16: every problem has 16-bit activations (Problem::a16): its x is the
+// plane matrix, and the epilogue combines row pairs and stores int16.
+template <bool A16>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     prefill_kernel(const __grid_constant__ Params P) {
     extern __shared__ uint8_t smem_raw[];
@@ -527,6 +548,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const EpiArgs e{p.y, p.residual, p.M, p.ldy, p.zy};
             const int tok0 = t.tt * TN + 64 * half;
             const int ntok = min(64, e.M - tok0);
+            if constexpr (A16) {
+                const int64_t c16 = (int64_t)(128 - p.zx) * (int64_t)__ldg(p.colsum + ch);
+                int16_t *yp = reinterpret_cast<int16_t *>(e.y) + (size_t)(tok0 >> 1) * (size_t)e.ldy + ch;
+                store_channel16(acc, c16, m0, sh, e.zy, yp, (size_t)e.ldy, ntok >> 1);
+                continue;
+            }
             if (p.zw && ntok > 0) {
                 // the weight zero point's term: - zw rowsum(x)[token]
                 const int32_t *rs = p.rowsum + tok0;
@@ -611,7 +638,7 @@ int max_pairs(int dev) {
     cfg.blockDim = dim3(THREADS, 1, 1);
     cfg.dynamicSmemBytes = SMEM_BYTES;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, prefill_kernel, &cfg) == cudaSuccess &&
+    if (cudaOccupancyMaxActiveClusters(&clusters, prefill_kernel<false>, &cfg) == cudaSuccess &&
         clusters > 0 && clusters < n)
         n = clusters;
     if (n > MAX_PAIRS) n = MAX_PAIRS;
@@ -661,11 +688,15 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
     if (attr_done != dev) {
-        if (cudaFuncSetAttribute(prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)SMEM_BYTES) != cudaSuccess ||
+            cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)SMEM_BYTES) != cudaSuccess)
             return MQ_ERR_CUDA;
         attr_done = dev;
     }
+    if (count <= 0) return MQ_OK;
+    auto kern = probs[0].a16 ? prefill_kernel<true> : prefill_kernel<false>;
     const int pairs_max = max_pairs(dev);
     if (pairs_max < 1) return MQ_ERR_CUDA;
     for (int begin = 0; begin < count; begin += PREFILL_MAX_PROBLEMS) {
@@ -717,7 +748,7 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        if (cudaLaunchKernelEx(&cfg, prefill_kernel, P) != cudaSuccess) return MQ_ERR_CUDA;
+        if (cudaLaunchKernelEx(&cfg, kern, P) != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;
 }

@@ -397,4 +397,26 @@ __device__ __forceinline__ int32_t mq_requant(int32_t acc, int32_t m0, int32_t s
     return min(127, max(-128, q + zy));
 }
 
+// The 16-bit output: clamp(zy + floor((acc m0 + 2^(sh-1)) / 2^sh), -32768,
+// 32767) for |acc| < 2^41, 0 <= m0 < 2^31, 1 <= sh <= 62, in int64.  For
+// sh >= 16, with m0 = mh 2^16 + ml (0 <= ml < 2^16) and
+// Y = acc ml + 2^(sh-1):  acc m0 + 2^(sh-1) = 2^16 (acc mh + floor(Y / 2^16))
+// + (Y mod 2^16), so the quotient is (acc mh + (Y >> 16)) >> (sh - 16) (the
+// dropped remainder is below 2^16 <= 2^sh; arithmetic shifts floor); every
+// term stays below 2^62.  For sh < 16 the multiplier is at least 2^15, so
+// |acc| >= 2^32 saturates and smaller accumulators fit a plain int64 product.
+__device__ __forceinline__ int32_t mq_requant16(int64_t acc, int32_t m0, int32_t sh, int32_t zy) {
+    int64_t q;
+    if (sh >= 16) {
+        const int64_t y = acc * (int64_t)(m0 & 0xFFFF) + ((int64_t)1 << (sh - 1));
+        q = (acc * (int64_t)(m0 >> 16) + (y >> 16)) >> (sh - 16);
+    } else if (acc >= ((int64_t)1 << 32) || acc <= -((int64_t)1 << 32)) {
+        q = acc > 0 ? (m0 ? 131072 : 0) : (m0 ? -131072 : 0);
+    } else {
+        q = (acc * (int64_t)m0 + ((int64_t)1 << (sh - 1))) >> sh;
+    }
+    const int32_t qc = (int32_t)(q < -131072 ? -131072 : (q > 131072 ? 131072 : q));
+    return min(32767, max(-32768, qc + zy));
+}
+
 }  // namespace mq

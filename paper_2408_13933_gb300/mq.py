@@ -38,7 +38,8 @@ MQ_MAX_BATCH = 256
 
 EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_weights",
             "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
-            "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch"]
+            "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch",
+            "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16"]
 
 _vp, _i32, _int, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int, ctypes.c_size_t
 
@@ -47,7 +48,8 @@ class LinearDesc(ctypes.Structure):
     """Mirror of mq_linear_desc."""
     _fields_ = [("x", _vp), ("packed", _vp), ("colsum", _vp), ("M0", _vp), ("shift", _vp),
                 ("residual", _vp), ("zw", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
-                ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32)]
+                ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32),
+                ("abits", _i32)]
 
 
 lib.mq_status_string.argtypes = [_int]
@@ -60,6 +62,9 @@ _linear_args = [_vp, _int, _int, _int, _i32, _vp, _vp, _int, _vp, _vp, _i32, _vp
                 _sz, _vp]
 lib.mq_linear_w8a8.argtypes = _linear_args
 lib.mq_linear_w4a8.argtypes = _linear_args
+lib.mq_linear_w8a16.argtypes = _linear_args
+lib.mq_linear_w4a16.argtypes = _linear_args
+lib.mq_workspace_size_a16.argtypes = [_int, _int, _int, _int, ctypes.POINTER(_sz)]
 lib.mq_linear_w4a8_noalloc.argtypes = [_vp, _int, _int, _int, _i32, _vp, _vp, _int, _vp, _vp, _i32,
                                        _vp, _int, _vp]
 lib.mq_linear_batch.argtypes = [ctypes.POINTER(LinearDesc), _int, _vp, _sz, _vp]
@@ -125,6 +130,12 @@ def workspace_size(m: int, n: int, k: int, bits: int) -> int:
     return out.value
 
 
+def workspace_size_a16(m: int, n: int, k: int, bits: int) -> int:
+    out = _sz(0)
+    _check(lib.mq_workspace_size_a16(m, n, k, bits, ctypes.byref(out)), "mq_workspace_size_a16")
+    return out.value
+
+
 def workspace(device=None):
     """A zero-filled device workspace large enough for any mq_linear_* or
     mq_linear_batch call (see mq_workspace_size); torch allocates it."""
@@ -169,6 +180,23 @@ def linear(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y, bits: int,
               int(zy), _ptr(y), ldy, _ptr(workspace), ws_bytes, _stream(stream))
 
 
+def linear_a16(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y, bits: int,
+               ldx: int | None = None, ldy: int | None = None, m: int | None = None,
+               k: int | None = None, stream=None, workspace=None,
+               ws_bytes: int | None = None) -> int:
+    """mq_linear_w8a16 / mq_linear_w4a16 on CUDA tensors (int16 x and y);
+    returns the status code."""
+    if ws_bytes is None:
+        ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    m = x.shape[0] if m is None else m
+    k = x.shape[1] if k is None else k
+    ldx = x.stride(0) if ldx is None else ldx
+    ldy = y.stride(0) if ldy is None else ldy
+    fn = lib.mq_linear_w8a16 if bits == 8 else lib.mq_linear_w4a16
+    return fn(_ptr(x), m, k, ldx, int(zx), _ptr(packed), _ptr(colsum), n, _ptr(m0), _ptr(shift),
+              int(zy), _ptr(y), ldy, _ptr(workspace), ws_bytes, _stream(stream))
+
+
 def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y,
                         ldx: int | None = None, ldy: int | None = None, m: int | None = None,
                         k: int | None = None, stream=None) -> int:
@@ -184,9 +212,13 @@ def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, 
 
 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
-              ldx=None, ldy=None, m=None, k=None, zw=None) -> LinearDesc:
-    """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights."""
+              ldx=None, ldy=None, m=None, k=None, zw=None, abits=None) -> LinearDesc:
+    """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights;
+    abits 16 (default: 16 for an int16 x) gives int16 activations and outputs."""
     d = LinearDesc()
+    if abits is None:
+        abits = 16 if getattr(x, "element_size", lambda: 1)() == 2 else 8
+    d.abits = int(abits)
     d.x, d.packed, d.colsum = _ptr(x), _ptr(packed), _ptr(colsum)
     d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
     d.zw = _ptr(zw)

@@ -223,3 +223,60 @@ def test_synth_asymmetric_weights():
     assert synth.paper_weight_scheme("q", 8) == "asym_tensor"
     assert synth.paper_weight_scheme("down", 8) == "asym_channel"
     assert synth.paper_weight_scheme("q", 4) == "asym_channel"
+
+
+def _desc16(mq, M, K, N, bits, **kw):
+    d = _desc(mq, M, K, N, bits, False)
+    d.abits = 16
+    for k, v in kw.items():
+        setattr(d, k, v)
+    return d
+
+
+def test_a16_validation_and_workspace(mq):
+    # 16-bit activations: zero points over the int16 range, no residual or
+    # weight zero point, 16-byte rows (ldx % 8), abits 8 or 16 only; every
+    # rejection happens before anything is launched
+    def rc(d):
+        return mq.lib.mq_linear_batch((mq.LinearDesc * 1)(d), 1, FAKE, 1 << 30, None)
+    assert rc(_desc16(mq, 4, 64, 32, 8, abits=12)) == mq.MQ_ERR_INVALID_ARG
+    assert rc(_desc16(mq, 4, 64, 32, 8, zx=32768)) == mq.MQ_ERR_INVALID_ARG
+    assert rc(_desc16(mq, 4, 64, 32, 8, zy=-32769)) == mq.MQ_ERR_INVALID_ARG
+    assert rc(_desc16(mq, 4, 64, 32, 8, residual=FAKE)) == mq.MQ_ERR_INVALID_ARG
+    assert rc(_desc16(mq, 4, 64, 32, 8, zw=FAKE)) == mq.MQ_ERR_INVALID_ARG
+    assert rc(_desc16(mq, 4, 64, 32, 8, ldx=68)) == mq.MQ_ERR_ALIGNMENT
+    assert rc(_desc16(mq, 4, 48, 32, 4, ldx=48)) == mq.MQ_ERR_ALIGNMENT   # int4: K % 32
+    assert rc(_desc16(mq, 4, 65552, 32, 8, ldx=65552)) == mq.MQ_ERR_K_OVERFLOW
+    # int8 zero points outside [-128, 127] stay invalid for 8-bit activations
+    d8 = _desc(mq, 4, 64, 32, 8, False)
+    d8.zx = 200
+    assert rc(d8) == mq.MQ_ERR_INVALID_ARG
+    # an A16 call without its workspace is rejected
+    one = (mq.LinearDesc * 1)(_desc16(mq, 100, 64, 32, 8))
+    assert mq.lib.mq_linear_batch(one, 1, None, 0, None) == mq.MQ_ERR_WORKSPACE
+    # workspace: decode region when 2M <= 16, then the planes (2 M K, to 128)
+    dec = mq.workspace_size(1, 1, 0, 4)
+    assert mq.workspace_size_a16(100, 32, 64, 8) == 12800
+    assert mq.workspace_size_a16(9, 32, 64, 8) == 1152            # 2M = 18: tensor cores
+    assert mq.workspace_size_a16(8, 32, 64, 4) == dec + 1024      # 2M = 16: decode
+    assert mq.workspace_size_a16(1, 32, 48, 8) == dec + 128
+    assert mq.workspace_size_a16(0, 32, 64, 8) == 0
+    assert mq.workspace_size_a16(5, 32, 0, 8) == dec              # K = 0: no planes
+    # batch: shared int16 input planned once; after a rowsum region the
+    # planes start on a 128-byte boundary
+    a = _desc16(mq, 100, 64, 32, 8)
+    b = _desc16(mq, 100, 64, 48, 4)
+    assert mq.workspace_size_batch([a, b]) == 12800
+    r = _desc(mq, 20, 64, 32, 8, True)
+    r.x = FAKE + 8192
+    assert mq.workspace_size_batch([r, a]) == 128 + 12800
+    assert mq.workspace_size_batch([r]) == 80
+
+
+def test_a16_single_call_symbols(mq):
+    for name in ("mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16"):
+        assert hasattr(mq.lib, name)
+    # the single calls validate like the batch (int16 zero point out of range)
+    f = mq.lib.mq_linear_w8a16
+    assert f(FAKE, 4, 64, 64, 40000, FAKE, FAKE, 32, FAKE, FAKE, 0, FAKE, 32, FAKE, 1 << 30,
+             None) == mq.MQ_ERR_INVALID_ARG
