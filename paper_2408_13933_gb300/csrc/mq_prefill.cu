@@ -44,6 +44,11 @@
 // Work: pair tiles (256 channels x 128 tokens) of up to PREFILL_MAX_PROBLEMS
 // independent linears, assigned to pairs by the host (longest processing time
 // first) or round-robin when there are too many tiles for the table.
+// 16-bit activations (the A16 instantiation): x is the plane matrix, whose
+// rows 2m and 2m + 1 hold the high bytes and the low bytes - 128 of token m,
+// so a tile covers 64 tokens; the epilogue adds 256 times the first column of
+// each pair and the second into an int64 sum per token and chunk, adds
+// (128 - zx) colsum and stores the int16 result.
 // All mbarrier waits are bounded (mq_wait_parity / mq_wait_parity_cluster).
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -210,24 +215,6 @@ __device__ __forceinline__ void store_channel(const uint32_t (&acc)[64], int32_t
             }
         }
     }
-}
-
-// 16-bit activations: columns 2j and 2j + 1 of the thread's 64 are the high
-// and low planes of token j, so sum((x - zx) w) = 256 S(2j) + S(2j + 1) +
-// (128 - zx) colsum (c16); requantize and store its n16 int16 outputs.  Kept
-// out of line: its 64-bit arithmetic would otherwise crowd the registers of
-// the accumulation loop (the call passes the sums through the stack once per
-// tile).
-__device__ __noinline__ void store_channel16(const uint32_t (&acc)[64], int64_t c16, int32_t m0,
-                                             int32_t sh, int32_t zy, int16_t *yp, size_t ldy,
-                                             int n16) {
-#pragma unroll 4
-    for (int j = 0; j < 32; ++j)
-        if (j < n16) {
-            const int64_t a = 256 * (int64_t)(int32_t)acc[2 * j] +
-                              (int64_t)(int32_t)acc[2 * j + 1] + c16;
-            yp[(size_t)j * ldy] = (int16_t)mq_requant16(a, m0, sh, zy);
-        }
 }
 
 // Barrier scopes: arrivals from the other CTA are releases at cluster scope
@@ -535,9 +522,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     uint32_t f[16];
                     tc_ld_32x32b_x16(t_lane + F_COL0 + 128 * b + 16 * q, f);
                     tc_wait_ld();
+                    if constexpr (A16) {
+                        // token 8q + i: 256 S(hi) + S(lo) of the chunk, added to the
+                        // token's int64 sum (halves in acc[16q + 2i], acc[16q + 2i + 1])
 #pragma unroll
-                    for (int i = 0; i < 16; ++i)
-                        acc[16 * q + i] += (uint32_t)__float2int_rn(__uint_as_float(f[i]));
+                        for (int i = 0; i < 8; ++i) {
+                            const int64_t d =
+                                256 * (int64_t)__float2int_rn(__uint_as_float(f[2 * i])) +
+                                (int64_t)__float2int_rn(__uint_as_float(f[2 * i + 1]));
+                            uint64_t v = ((uint64_t)acc[16 * q + 2 * i + 1] << 32) | acc[16 * q + 2 * i];
+                            v += (uint64_t)d;
+                            acc[16 * q + 2 * i] = (uint32_t)v;
+                            acc[16 * q + 2 * i + 1] = (uint32_t)(v >> 32);
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            acc[16 * q + i] += (uint32_t)__float2int_rn(__uint_as_float(f[i]));
+                    }
                 }
                 tc_fence_before();
                 __syncwarp();
@@ -549,9 +551,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const int tok0 = t.tt * TN + 64 * half;
             const int ntok = min(64, e.M - tok0);
             if constexpr (A16) {
+                // acc pairs hold each token's int64 sum 256 S(hi) + S(lo):
+                // sum((x - zx) w) = that + (128 - zx) colsum
                 const int64_t c16 = (int64_t)(128 - p.zx) * (int64_t)__ldg(p.colsum + ch);
                 int16_t *yp = reinterpret_cast<int16_t *>(e.y) + (size_t)(tok0 >> 1) * (size_t)e.ldy + ch;
-                store_channel16(acc, c16, m0, sh, e.zy, yp, (size_t)e.ldy, ntok >> 1);
+                const int n16 = ntok >> 1;
+                const size_t ldy16 = (size_t)e.ldy;
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (j < n16) {
+                        const int64_t a =
+                            (int64_t)(((uint64_t)acc[2 * j + 1] << 32) | acc[2 * j]) + c16;
+                        yp[(size_t)j * ldy16] = (int16_t)mq_requant16(a, m0, sh, e.zy);
+                    }
                 continue;
             }
             if (p.zw && ntok > 0) {
