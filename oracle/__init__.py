@@ -57,6 +57,9 @@ def _bind(lib):
                                              p, p]
     lib.oracle_requant_one_a16.argtypes = [i64, i32, i32, i32]
     lib.oracle_requant_one_a16.restype = i32
+    lib.oracle_quantize_f32.argtypes = [p, i64, f32, i32, ci, p]
+    lib.oracle_dequantize.argtypes = [p, ci, i64, f32, i32, p]
+    lib.oracle_requantize.argtypes = [p, ci, i64, i32, i32, i32, i32, p, ci]
     lib.oracle_residual_add.argtypes = [p, p, i64, p]
     lib.oracle_residual_add.restype = None
     return lib
@@ -201,6 +204,31 @@ class Oracle:
     def requant_one_a16(self, acc: int, m0: int, shift: int, zy: int) -> int:
         return int(self.lib.oracle_requant_one_a16(int(acc), int(m0), int(shift), int(zy)))
 
+    def quantize(self, x: np.ndarray, alpha: float, z: int, bits: int) -> np.ndarray:
+        """oracle_quantize_f32: f32 values -> int8 / int16 codes."""
+        x = np.ascontiguousarray(x, dtype=np.float32)
+        q = np.zeros(x.shape, np.int8 if bits == 8 else np.int16)
+        _check(self.lib.oracle_quantize_f32(_ptr(x), x.size, float(alpha), int(z), bits, _ptr(q)),
+               "oracle_quantize_f32")
+        return q
+
+    def dequantize(self, q: np.ndarray, alpha: float, z: int) -> np.ndarray:
+        bits = 8 if q.dtype == np.int8 else 16
+        q = np.ascontiguousarray(q)
+        f = np.zeros(q.shape, np.float32)
+        _check(self.lib.oracle_dequantize(_ptr(q), bits, q.size, float(alpha), int(z), _ptr(f)),
+               "oracle_dequantize")
+        return f
+
+    def requantize(self, q: np.ndarray, zx: int, m0: int, shift: int, zy: int,
+                   out_bits: int) -> np.ndarray:
+        in_bits = 8 if q.dtype == np.int8 else 16
+        q = np.ascontiguousarray(q)
+        y = np.zeros(q.shape, np.int8 if out_bits == 8 else np.int16)
+        _check(self.lib.oracle_requantize(_ptr(q), in_bits, q.size, int(zx), int(m0), int(shift),
+                                          int(zy), _ptr(y), out_bits), "oracle_requantize")
+        return y
+
     def residual_add(self, a: np.ndarray, b: np.ndarray) -> np.ndarray:
         a = np.ascontiguousarray(a, dtype=np.int8)
         b = np.ascontiguousarray(b, dtype=np.int8)
@@ -253,6 +281,18 @@ def linear_points_a16(x, zx, packed, bits, n, m0, shift, zy, pts):
 
 def requant_one_a16(acc, m0, shift, zy):
     return _default().requant_one_a16(acc, m0, shift, zy)
+
+
+def quantize(x, alpha, z, bits):
+    return _default().quantize(x, alpha, z, bits)
+
+
+def dequantize(q, alpha, z):
+    return _default().dequantize(q, alpha, z)
+
+
+def requantize(q, zx, m0, shift, zy, out_bits):
+    return _default().requantize(q, zx, m0, shift, zy, out_bits)
 
 
 def residual_add(a, b):

@@ -316,6 +316,82 @@ int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx
     return ORACLE_OK;
 }
 
+static int oracle_code_range(int bits, int32_t *lo, int32_t *hi) {
+    if (bits == 8) {
+        *lo = -128;
+        *hi = 127;
+        return ORACLE_OK;
+    }
+    if (bits == 16) {
+        *lo = -32768;
+        *hi = 32767;
+        return ORACLE_OK;
+    }
+    return ORACLE_EINVAL;
+}
+
+static int32_t oracle_code_at(const void *q, int bits, int64_t i) {
+    return bits == 8 ? (int32_t)((const int8_t *)q)[i] : (int32_t)((const int16_t *)q)[i];
+}
+
+static void oracle_code_store(void *q, int bits, int64_t i, int32_t v) {
+    if (bits == 8)
+        ((int8_t *)q)[i] = (int8_t)v;
+    else
+        ((int16_t *)q)[i] = (int16_t)v;
+}
+
+int oracle_quantize_f32(const float *x, int64_t n, float alpha, int32_t z, int bits,
+                        void *q) {
+    int32_t lo, hi;
+    if (oracle_code_range(bits, &lo, &hi) != ORACLE_OK || n < 0) return ORACLE_EINVAL;
+    if (!(isfinite(alpha) && alpha > 0.0f) || z < lo || z > hi) return ORACLE_EINVAL;
+    for (int64_t i = 0; i < n; ++i) {
+        float quotient = x[i] / alpha; /* f32 division, rounded to nearest */
+        int32_t code;
+        if (isnan(quotient)) {
+            code = z;
+        } else {
+            double t = (double)rintf(quotient) + (double)z; /* ties to even */
+            if (t < lo) t = lo;
+            if (t > hi) t = hi;
+            code = (int32_t)t;
+        }
+        oracle_code_store(q, bits, i, code);
+    }
+    return ORACLE_OK;
+}
+
+int oracle_dequantize(const void *q, int bits, int64_t n, float alpha, int32_t z, float *f) {
+    int32_t lo, hi;
+    if (oracle_code_range(bits, &lo, &hi) != ORACLE_OK || n < 0) return ORACLE_EINVAL;
+    if (!isfinite(alpha) || z < lo || z > hi) return ORACLE_EINVAL;
+    for (int64_t i = 0; i < n; ++i) {
+        double exact = (double)(oracle_code_at(q, bits, i) - z) * (double)alpha;
+        f[i] = (float)exact;
+    }
+    return ORACLE_OK;
+}
+
+int oracle_requantize(const void *q, int in_bits, int64_t n, int32_t zx, int32_t M0,
+                      int32_t shift, int32_t zy, void *y, int out_bits) {
+    int32_t ilo, ihi, olo, ohi;
+    if (oracle_code_range(in_bits, &ilo, &ihi) != ORACLE_OK ||
+        oracle_code_range(out_bits, &olo, &ohi) != ORACLE_OK || n < 0)
+        return ORACLE_EINVAL;
+    if (zx < ilo || zx > ihi || zy < olo || zy > ohi) return ORACLE_EINVAL;
+    if (M0 < 0 || shift < 1 || shift > 62) return ORACLE_EINVAL;
+    for (int64_t i = 0; i < n; ++i) {
+        int64_t centered = (int64_t)oracle_code_at(q, in_bits, i) - zx;
+        __int128 rounded = oracle_round_shift(centered, M0, shift);
+        __int128 out = (__int128)zy + rounded;
+        if (out < olo) out = olo;
+        if (out > ohi) out = ohi;
+        oracle_code_store(y, out_bits, i, (int32_t)out);
+    }
+    return ORACLE_OK;
+}
+
 void oracle_residual_add(const int8_t *a, const int8_t *b, int64_t n,
                          int8_t *out) {
     for (int64_t i = 0; i < n; ++i) {

@@ -155,6 +155,43 @@ int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx
 int32_t oracle_requant_one_a16(int64_t acc, int32_t M0, int32_t shift, int32_t zy);
 
 /*
+ * Boundary quantizers between the float, int16 and int8 domains of an
+ * integer block: the activations of linears are 8-bit, those around
+ * non-linear operators 16-bit (Sec. 4.1, Sec. 1); every step is a static
+ * per-tensor quantizer (Sec. 3.1).  `bits` selects int8 (8) or int16 (16)
+ * codes, stored as int8_t / int16_t arrays.
+ *
+ * oracle_quantize_f32: the forward quantizer of eqs. 2-4, shifted to the
+ * signed range (readings R1, R2): q = clamp(rint(x / alpha) + z, qmin, qmax).
+ * The integer decision is taken in f32 (reading R12): x / alpha is the
+ * correctly rounded f32 quotient and rint rounds ties to even; a NaN input
+ * gives z.  alpha must be finite and > 0, z inside the code range.
+ * Pinned by: exact rationals (f32 rounding of the true quotient, then ties to
+ * even), dequantization within half a step, monotonicity, saturation.
+ */
+int oracle_quantize_f32(const float *x, int64_t n, float alpha, int32_t z, int bits,
+                        void *q);
+
+/*
+ * Dequantization f = (q - z) * alpha, rounded once to f32 (the product of
+ * an integer below 2^17 and an f32 is exact in double).
+ * Pinned by: exact rationals, round trip with oracle_quantize_f32.
+ */
+int oracle_dequantize(const void *q, int bits, int64_t n, float alpha, int32_t z, float *f);
+
+/*
+ * Fixed-point requantization between integer domains (int8 / int16 in,
+ * int8 / int16 out), the output quantizer of eq. 4 with the multiplier
+ * alpha_in / alpha_out in the fixed-point form of oracle_requant_params:
+ *   y = clamp(zy + floor(((q - zx) M0 + 2^(s-1)) / 2^s), ymin, ymax).
+ * zx and zy lie in their domains' code ranges.
+ * Pinned by: exhaustive sweeps over every int16 / int8 code against exact
+ * rationals, the power-of-two closed form, eq. 4 with the real multiplier.
+ */
+int oracle_requantize(const void *q, int in_bits, int64_t n, int32_t zx, int32_t M0,
+                      int32_t shift, int32_t zy, void *y, int out_bits);
+
+/*
  * Requantize one accumulator: clamp(zy + floor(acc*M0 / 2^s + 1/2), -128, 127).
  * Exposed so that tests can sweep accumulators around rounding ties.
  */

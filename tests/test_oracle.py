@@ -438,13 +438,137 @@ def pin_a16_requant_vs_eq4(orc: Oracle):
     assert np.mean(np.abs(y.astype(np.int64)) < 32767) > 0.9
 
 
+# ---- boundary quantizers (float / int16 / int8 domains) ----------------------
+
+def _f32_nearest(fr: Fraction) -> float:
+    """The f32 value nearest to the rational fr, ties to even mantissa (IEEE
+    round to nearest), found among the f32 neighbours of a first guess."""
+    g = np.float32(float(fr))
+    cands = {np.float32(g), np.nextafter(g, np.float32(np.inf)),
+             np.nextafter(g, np.float32(-np.inf))}
+    best = None
+    for c in cands:
+        if not np.isfinite(c):
+            continue
+        d = abs(Fraction(float(c)) - fr)
+        key = (d, int(np.array(c, np.float32).view(np.int32)) & 1)  # ties: even mantissa first
+        if best is None or key < best[0]:
+            best = (key, c)
+    return float(best[1])
+
+
+def _quantize_ref(x: float, alpha: float, z: int, bits: int) -> int:
+    lo, hi = (-128, 127) if bits == 8 else (-32768, 32767)
+    if np.isnan(x):
+        return z
+    if np.isinf(x):
+        return hi if x > 0 else lo
+    qf = _f32_nearest(Fraction(float(np.float32(x))) / Fraction(float(np.float32(alpha))))
+    return max(lo, min(hi, round(qf) + z))  # Python round: ties to even
+
+
+def pin_quantize_exact(orc: Oracle):
+    rng = np.random.default_rng(101)
+    for bits in (8, 16):
+        for alpha, z in ((np.float32(0.0371), -3), (np.float32(1.0 / 3.0), 17),
+                         (np.float32(2.5e-4), -1000 if bits == 16 else -100)):
+            scale = 140 if bits == 8 else 40000
+            x = (rng.standard_normal(1500) * float(alpha) * scale / 3).astype(np.float32)
+            # values whose quotient lies within an ulp of a .5 tie
+            k = rng.integers(-scale, scale, size=300)
+            near = ((k + 0.5) * float(alpha)).astype(np.float32)
+            x = np.concatenate([x, near, np.nextafter(near, np.float32(np.inf)),
+                                np.nextafter(near, np.float32(-np.inf)),
+                                np.array([np.inf, -np.inf, np.nan, 0.0, -0.0], np.float32)])
+            zz = z if bits == 16 else max(-128, min(127, z))
+            got = orc.quantize(x, float(alpha), zz, bits)
+            for i in range(x.size):
+                assert int(got[i]) == _quantize_ref(float(x[i]), float(alpha), zz, bits), \
+                    (bits, float(alpha), i, float(x[i]))
+
+
+def pin_quantize_ties_and_invariants(orc: Oracle):
+    # power-of-two scale: the quotient (k + 1/2) is exact, ties go to even
+    k = np.arange(-100, 100)
+    x = ((k + 0.5) / 8).astype(np.float32)
+    got = orc.quantize(x, 0.125, 0, 8).astype(np.int64)
+    want = np.where(k % 2 == 0, k, k + 1)
+    assert np.array_equal(got, np.clip(want, -128, 127))
+    # monotone, and within half a step of the value wherever not saturated
+    rng = np.random.default_rng(102)
+    xs = np.sort(rng.uniform(-6, 6, 5000).astype(np.float32))
+    for bits, alpha, z in ((8, 0.03, 5), (16, 1e-4, -77)):
+        q = orc.quantize(xs, alpha, z, bits).astype(np.int64)
+        assert np.all(np.diff(q) >= 0)
+        lo, hi = (-128, 127) if bits == 8 else (-32768, 32767)
+        inside = (q > lo) & (q < hi)
+        a64 = np.float64(np.float32(alpha))
+        err = np.abs((q - z) * a64 - xs.astype(np.float64))
+        # half a step, plus the f32 rounding of the quotient (half an ulp of |x / alpha|)
+        bound = a64 * (0.5 + np.abs(xs.astype(np.float64) / a64) * 2.0 ** -24) * (1 + 1e-9)
+        assert np.all(err[inside] <= bound[inside])
+        assert inside.mean() > 0.5
+
+
+def pin_dequantize_exact(orc: Oracle):
+    for bits, alpha, z in ((8, np.float32(0.0371), -3), (16, np.float32(2.5e-4), 1234)):
+        lo, hi = (-128, 127) if bits == 8 else (-32768, 32767)
+        q = np.arange(lo, hi + 1, dtype=np.int64).astype(np.int8 if bits == 8 else np.int16)
+        f = orc.dequantize(q, float(alpha), z)
+        for i in range(0, q.size, 1 if bits == 8 else 97):
+            want = _f32_nearest(Fraction(int(q[i]) - z) * Fraction(float(alpha)))
+            assert float(f[i]) == want, (bits, int(q[i]))
+
+
+def pin_requantize_exhaustive(orc: Oracle):
+    # every int16 code to int8 and every int8 code to int16, for several
+    # multipliers, against floor((q - zx) M0 / 2^s + 1/2) on Python integers
+    rng = random.Random(103)
+    all16 = np.arange(-32768, 32768, dtype=np.int64).astype(np.int16)
+    all8 = np.arange(-128, 128, dtype=np.int64).astype(np.int8)
+    for q, out_bits in ((all16, 8), (all8, 16), (all16, 16), (all8, 8)):
+        in_lo, in_hi = (-128, 127) if q.dtype == np.int8 else (-32768, 32767)
+        lo, hi = (-128, 127) if out_bits == 8 else (-32768, 32767)
+        for _ in range(4):
+            m0 = rng.randint(1 << 30, (1 << 31) - 1)
+            s = rng.randint(20, 45)
+            zx, zy = rng.randint(in_lo, in_hi), rng.randint(lo, hi)
+            got = orc.requantize(q, zx, m0, s, zy, out_bits)
+            for i in range(0, q.size, 1 if q.size <= 256 else 61):
+                v = Fraction((int(q[i]) - zx) * m0, 1 << s)
+                want = max(lo, min(hi, zy + _round_half_up_frac(v)))
+                assert int(got[i]) == want, (out_bits, i, m0, s)
+            # all codes at once with exact integer floor division
+            v = (q.astype(np.int64) - zx) * m0 + (1 << (s - 1))
+            want = np.clip(zy + np.floor_divide(v, 1 << s), lo, hi)
+            assert np.array_equal(got.astype(np.int64), want)
+
+
+def pin_requantize_vs_eq4(orc: Oracle):
+    # int16 codes of one range requantized to int8 codes of another: within
+    # one step of eq. 4 applied to the real value (float64)
+    rng = np.random.default_rng(104)
+    xf = rng.standard_normal(20000).astype(np.float32) * 3
+    import paper_2408_13933_gb300.synth as sy
+    q16, s16, z16 = sy.quantize_per_tensor(xf, bits=16)
+    s8, z8 = sy.quantize_params_from_range(float(xf.min()), float(xf.max()))
+    m0, sh = orc.requant_params(s16, np.ones(1, np.float32), s8)
+    y = orc.requantize(q16, z16, int(m0[0]), int(sh[0]), z8, 8).astype(np.int64)
+    real = (q16.astype(np.float64) - z16) * s16
+    ref = np.clip(np.floor(real / s8 + 0.5) + z8, -128, 127)
+    diff = np.abs(y - ref)
+    assert diff.max() <= 1 and (diff != 0).mean() < 1e-3
+
+
 PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zero_point_identity,
                pin_exact_dequant, pin_requant_closed_form, pin_requant_ties, pin_requant_vs_eq4,
                pin_requant_params_bound, pin_asym_k1_exhaustive, pin_asym_int4_pairs,
                pin_asym_identity, pin_asym_reduces_to_symmetric, pin_asym_exact_dequant,
                pin_a16_k1_exhaustive, pin_a16_int4_pairs, pin_a16_matmul_and_brute_force,
                pin_a16_large_accumulators, pin_a16_reduces_to_int8, pin_a16_byte_planes, pin_a16_exact_dequant,
-               pin_a16_requant_closed_form_and_saturation, pin_a16_requant_vs_eq4]
+               pin_a16_requant_closed_form_and_saturation, pin_a16_requant_vs_eq4,
+               pin_quantize_exact, pin_quantize_ties_and_invariants, pin_dequantize_exact,
+               pin_requantize_exhaustive, pin_requantize_vs_eq4]
 
 
 # ----------------------------------------------------------------------------
@@ -659,6 +783,39 @@ def test_a16_points_agree_with_full(O):
     assert np.array_equal(ap, acc[pts[:, 0], pts[:, 1]])
 
 
+def test_quantize_exact(O):
+    pin_quantize_exact(O)
+
+
+def test_quantize_ties_and_invariants(O):
+    pin_quantize_ties_and_invariants(O)
+
+
+def test_dequantize_exact(O):
+    pin_dequantize_exact(O)
+
+
+def test_requantize_exhaustive(O):
+    pin_requantize_exhaustive(O)
+
+
+def test_requantize_vs_eq4(O):
+    pin_requantize_vs_eq4(O)
+
+
+def test_boundary_quantizers_reject_bad_arguments(O):
+    x = np.zeros(4, np.float32)
+    for alpha, z, bits in ((0.0, 0, 8), (float("nan"), 0, 8), (1.0, 128, 8), (1.0, 0, 12),
+                           (1.0, 40000, 16)):
+        with pytest.raises(oracle.OracleError):
+            O.quantize(x, alpha, z, bits)
+    q = np.zeros(4, np.int8)
+    with pytest.raises(oracle.OracleError):
+        O.requantize(q, 0, 1 << 30, 0, 0, 8)      # shift 0
+    with pytest.raises(oracle.OracleError):
+        O.requantize(q, 200, 1 << 30, 31, 0, 8)   # zx outside int8
+
+
 MUTATIONS = [
     ("zero point sign", "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - zx;",
      "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] + zx;"),
@@ -693,6 +850,18 @@ MUTATIONS = [
     ("a16 saturation at int8", "if (out > 32767) out = 32767;", "if (out > 127) out = 127;"),
     ("a16 round half down", "return oracle_floor_div(2 * v + two_s, 2 * two_s);",
      "return oracle_floor_div(2 * v + two_s - 1, 2 * two_s);"),
+    ("quantize rounds half away from zero", "double t = (double)rintf(quotient) + (double)z;",
+     "double t = (double)roundf(quotient) + (double)z;"),
+    ("quantize by reciprocal multiply", "float quotient = x[i] / alpha;",
+     "float quotient = x[i] * (1.0f / alpha);"),
+    ("quantize zero point dropped", "double t = (double)rintf(quotient) + (double)z;",
+     "double t = (double)rintf(quotient);"),
+    ("dequantize zero point sign", "(double)(oracle_code_at(q, bits, i) - z)",
+     "(double)(oracle_code_at(q, bits, i) + z)"),
+    ("requantize input zero point dropped",
+     "int64_t centered = (int64_t)oracle_code_at(q, in_bits, i) - zx;",
+     "int64_t centered = (int64_t)oracle_code_at(q, in_bits, i);"),
+    ("requantize wrong output range", "if (out > ohi) out = ohi;", "if (out > ihi) out = ihi;"),
     ("a16 output zero point dropped",
      "__int128 out = (__int128)zy + oracle_round_shift(acc, M0, shift);",
      "__int128 out = oracle_round_shift(acc, M0, shift);"),
