@@ -506,6 +506,39 @@ def run_a16(mq, torch, prefill_steps: int = 600, decode_steps: int = 480, check_
     return out
 
 
+def run_glue(mq, torch, n: int = 1 << 26, reps: int = 20):
+    """The boundary quantizers on 64M elements (inputs larger than L2): GB/s
+    of algorithmic bytes (input + output) per launch, back to back."""
+    out = {}
+    stream = torch.cuda.current_stream()
+    g = torch.Generator(device="cuda")
+    g.manual_seed(5)
+    xf = torch.randn(n, device="cuda", generator=g) * 3
+    q16 = torch.randint(-32768, 32768, (n,), device="cuda", generator=g, dtype=torch.int32).to(
+        torch.int16)
+    q8 = torch.empty(n, dtype=torch.int8, device="cuda")
+    m0, sh = mq.requant_params(np.array([3.1e-4], np.float32), 1.0, 0.011)
+    cases = {
+        "quantize_f32_i8": (lambda: mq.quantize(xf, 0.05, 3, q8), 4 + 1),
+        "requantize_i16_i8": (lambda: mq.requantize(q16, -40, int(m0[0]), int(sh[0]), 9, q8), 2 + 1),
+    }
+    for name, (fn, bpe) in cases.items():
+        for _ in range(3):
+            assert fn() == 0
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        out[name] = {"elements": n, "us": round(ms * 1e3, 1),
+                     "gbs": round(n * bpe / (ms * 1e-3) / 1e9, 1)}
+    del xf, q16, q8
+    return out
+
+
 # --------------------------------------------------------------------------- CPU oracle
 def oracle_sample(blocks_cases, rows: range, col_frac: float = 1.0):
     """Run the oracle on `rows` of every linear of one block; returns
@@ -614,6 +647,7 @@ def main():
     asym_pre = run_asym_prefill(mq, torch)
     asym_dec = run_decode(mq, torch, asym=True, ms=(1, 16))
     a16 = run_a16(mq, torch)
+    glue = run_glue(mq, torch)
     peaks = measured_peaks()
 
     ops = block_ops(PREFILL_M)
@@ -624,6 +658,8 @@ def main():
     hbm = peaks["hbm_gbs"]
     for v in list(decode.values()) + list(asym_dec.values()):
         v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
+    for v in glue.values():
+        v["frac_hbm"] = round(v["gbs"] / hbm, 3)
 
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world,
@@ -657,6 +693,7 @@ def main():
         "a16": {"activations": "int16 in and out", "ops": "2 M K N per block", **a16,
                 "w8a8_us_per_block": round(pre["total_ms"] / args.steps * 1e3, 2),
                 "w4a8_m1_stream_us": decode["m1"]["stream_us"]},
+        "boundary_quantizers": {"unit": "GB/s of input + output bytes", **glue},
     }
     if rank == 0 and world == 1:
         line["cpu_baseline"] = cpu_baseline(pre["blocks"], torch)

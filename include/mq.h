@@ -301,6 +301,56 @@ int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *byte
 int mq_linear_batch(const mq_linear_desc *descs, int count, void *workspace,
                     size_t ws_bytes, void *stream);
 
+/* ---- Boundary quantizers --------------------------------------------------
+ * The steps on either side of the linear in an integer block: activations of
+ * linears are 8-bit, those around non-linear operators 16-bit integers
+ * (Sec. 4.1), and every change of domain is a static per-tensor quantizer
+ * (Sec. 3.1).  Element types: */
+#define MQ_TYPE_F32 0
+#define MQ_TYPE_F16 1
+#define MQ_TYPE_BF16 2
+#define MQ_TYPE_I8 3
+#define MQ_TYPE_I16 4
+
+/*
+ * Static per-tensor activation quantizer, the forward quantizer of eqs. 2-4
+ * (Sec. 4.2) in the signed code range:
+ *   q[i] = clamp(rint(x[i] / alpha) + z, qmin, qmax)
+ * x[i] / alpha is the correctly rounded f32 quotient (f16 and bf16 values are
+ * widened to f32 exactly first); rint rounds ties to even; NaN gives z and
+ * +-inf saturates.
+ *   x     : device, n values of in_type (MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16)
+ *   q     : device, n codes of out_type (MQ_TYPE_I8 or MQ_TYPE_I16), written
+ *   alpha : finite, > 0;  z inside the output code range
+ * Requirements: n >= 0; x and q aligned to their element size (16-byte
+ * alignment of both takes the vector path).  Launched with programmatic
+ * stream serialization; x is read only after the previous kernel completes.
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_CUDA.
+ */
+int mq_quantize(const void *x, int in_type, int64_t n, float alpha, int32_t z, void *q,
+                int out_type, void *stream);
+
+/*
+ * Dequantization f[i] = (q[i] - z) * alpha, rounded once to f32.
+ *   q: device, n codes of in_type (MQ_TYPE_I8 or MQ_TYPE_I16); f: device f32 [n]
+ *   alpha finite; z inside the input code range.  Otherwise as mq_quantize.
+ */
+int mq_dequantize(const void *q, int in_type, int64_t n, float alpha, int32_t z, float *f,
+                  void *stream);
+
+/*
+ * Fixed-point requantization between integer domains (int8 / int16 codes in,
+ * int8 / int16 codes out):
+ *   y[i] = clamp(zy + floor(((q[i] - zx) M0 + 2^(shift-1)) / 2^shift), ymin, ymax)
+ * with M0 * 2^-shift ~= alpha_in / alpha_out, e.g. from
+ * mq_requant_params(&alpha_in, 1, 1.0f, alpha_out, &M0, &shift).
+ *   q, y : device, n codes of in_type / out_type (MQ_TYPE_I8 or MQ_TYPE_I16)
+ *   zx, zy inside their code ranges; 0 <= M0 < 2^31; 1 <= shift <= 62
+ * Otherwise as mq_quantize.
+ */
+int mq_requantize(const void *q, int in_type, int64_t n, int32_t zx, int32_t M0, int32_t shift,
+                  int32_t zy, void *y, int out_type, void *stream);
+
 /*
  * Wait for `stream` and report device-side failures recorded by this
  * library's kernels since the previous call: MQ_ERR_DEVICE_TIMEOUT if a

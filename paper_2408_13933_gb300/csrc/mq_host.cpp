@@ -405,6 +405,69 @@ int mq_linear_batch(const mq_linear_desc *descs, int count, void *workspace, siz
     return run_batch(descs, count, workspace, ws_bytes, stream);
 }
 
+namespace {
+
+bool code_range(int type, int32_t *lo, int32_t *hi) {
+    if (type == MQ_TYPE_I8) {
+        *lo = -128;
+        *hi = 127;
+        return true;
+    }
+    if (type == MQ_TYPE_I16) {
+        *lo = -32768;
+        *hi = 32767;
+        return true;
+    }
+    return false;
+}
+
+bool float_type(int type) {
+    return type == MQ_TYPE_F32 || type == MQ_TYPE_F16 || type == MQ_TYPE_BF16;
+}
+
+size_t type_size(int type) { return type == MQ_TYPE_F32 ? 4 : (type == MQ_TYPE_I8 ? 1 : 2); }
+
+bool aligned_to(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace
+
+int mq_quantize(const void *x, int in_type, int64_t n, float alpha, int32_t z, void *q,
+                int out_type, void *stream) {
+    int32_t lo, hi;
+    if (!float_type(in_type) || !code_range(out_type, &lo, &hi) || n < 0) return MQ_ERR_INVALID_ARG;
+    if (!(std::isfinite(alpha) && alpha > 0.0f) || z < lo || z > hi) return MQ_ERR_INVALID_ARG;
+    if (n == 0) return MQ_OK;
+    if (!x || !q) return MQ_ERR_INVALID_ARG;
+    if (!aligned_to(x, type_size(in_type)) || !aligned_to(q, type_size(out_type)))
+        return MQ_ERR_ALIGNMENT;
+    return mq::launch_glue(0, in_type, out_type, x, q, n, alpha, 0, z, 0, 1, lo, hi, stream);
+}
+
+int mq_dequantize(const void *q, int in_type, int64_t n, float alpha, int32_t z, float *f,
+                  void *stream) {
+    int32_t lo, hi;
+    if (!code_range(in_type, &lo, &hi) || n < 0) return MQ_ERR_INVALID_ARG;
+    if (!std::isfinite(alpha) || z < lo || z > hi) return MQ_ERR_INVALID_ARG;
+    if (n == 0) return MQ_OK;
+    if (!q || !f) return MQ_ERR_INVALID_ARG;
+    if (!aligned_to(q, type_size(in_type)) || !aligned_to(f, 4)) return MQ_ERR_ALIGNMENT;
+    return mq::launch_glue(1, in_type, MQ_TYPE_F32, q, f, n, alpha, z, 0, 0, 1, 0, 0, stream);
+}
+
+int mq_requantize(const void *q, int in_type, int64_t n, int32_t zx, int32_t M0, int32_t shift,
+                  int32_t zy, void *y, int out_type, void *stream) {
+    int32_t ilo, ihi, lo, hi;
+    if (!code_range(in_type, &ilo, &ihi) || !code_range(out_type, &lo, &hi) || n < 0)
+        return MQ_ERR_INVALID_ARG;
+    if (zx < ilo || zx > ihi || zy < lo || zy > hi || M0 < 0 || shift < 1 || shift > 62)
+        return MQ_ERR_INVALID_ARG;
+    if (n == 0) return MQ_OK;
+    if (!q || !y) return MQ_ERR_INVALID_ARG;
+    if (!aligned_to(q, type_size(in_type)) || !aligned_to(y, type_size(out_type)))
+        return MQ_ERR_ALIGNMENT;
+    return mq::launch_glue(2, in_type, out_type, q, y, n, 0.0f, zx, zy, M0, shift, lo, hi, stream);
+}
+
 int mq_check_device_status(void *stream) {
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (cudaStreamSynchronize(s) != cudaSuccess) return MQ_ERR_CUDA;

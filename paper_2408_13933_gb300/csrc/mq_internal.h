@@ -81,4 +81,11 @@ struct SplitJob {
 constexpr int SPLIT_MAX_JOBS = 64;
 int launch_split16(const SplitJob *jobs, int count, void *stream);
 
+// Boundary quantizers (mq_glue.cu): kind 0 quantize (float -> codes),
+// 1 dequantize (codes -> f32), 2 requantize (codes -> codes); types are the
+// MQ_TYPE_* of mq.h; [lo, hi] is the output code range.
+int launch_glue(int kind, int in_type, int out_type, const void *in, void *out, int64_t n,
+                float alpha, int32_t zin, int32_t zout, int32_t m0, int32_t shift, int32_t lo,
+                int32_t hi, void *stream);
+
 }  // namespace mq

@@ -389,7 +389,7 @@ __device__ __forceinline__ int32_t mq_requant(int32_t acc, int32_t m0, int32_t s
     if (sh >= 33) {
         q = (__mulhi(acc, m0) + (1 << (sh - 33))) >> (sh - 32);
     } else if (sh == 32) {
-        q = __mulhi(acc, m0) + (int32_t)((uint32_t)(acc * m0) >> 31);
+        q = __mulhi(acc, m0) + (int32_t)(((uint32_t)acc * (uint32_t)m0) >> 31);
     } else {
         const int64_t v = ((int64_t)acc * (int64_t)m0 + ((int64_t)1 << (sh - 1))) >> sh;
         q = (int32_t)(v < -1024 ? -1024 : (v > 1024 ? 1024 : v));

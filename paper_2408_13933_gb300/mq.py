@@ -39,7 +39,9 @@ MQ_MAX_BATCH = 256
 EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_weights",
             "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
             "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch",
-            "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16"]
+            "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16", "mq_quantize",
+            "mq_dequantize", "mq_requantize"]
+MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
 _vp, _i32, _int, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int, ctypes.c_size_t
 
@@ -70,6 +72,10 @@ lib.mq_linear_w4a8_noalloc.argtypes = [_vp, _int, _int, _int, _i32, _vp, _vp, _i
 lib.mq_linear_batch.argtypes = [ctypes.POINTER(LinearDesc), _int, _vp, _sz, _vp]
 lib.mq_workspace_size_batch.argtypes = [ctypes.POINTER(LinearDesc), _int, ctypes.POINTER(_sz)]
 lib.mq_check_device_status.argtypes = [_vp]
+_i64, _f32 = ctypes.c_int64, ctypes.c_float
+lib.mq_quantize.argtypes = [_vp, _int, _i64, _f32, _i32, _vp, _int, _vp]
+lib.mq_dequantize.argtypes = [_vp, _int, _i64, _f32, _i32, _vp, _vp]
+lib.mq_requantize.argtypes = [_vp, _int, _i64, _i32, _i32, _i32, _i32, _vp, _int, _vp]
 for _f in EXPORTED:
     if _f != "mq_status_string":
         getattr(lib, _f).restype = _int
@@ -195,6 +201,30 @@ def linear_a16(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y, bits: 
     fn = lib.mq_linear_w8a16 if bits == 8 else lib.mq_linear_w4a16
     return fn(_ptr(x), m, k, ldx, int(zx), _ptr(packed), _ptr(colsum), n, _ptr(m0), _ptr(shift),
               int(zy), _ptr(y), ldy, _ptr(workspace), ws_bytes, _stream(stream))
+
+
+def _type_of(t) -> int:
+    import torch
+    return {torch.float32: MQ_TYPE_F32, torch.float16: MQ_TYPE_F16, torch.bfloat16: MQ_TYPE_BF16,
+            torch.int8: MQ_TYPE_I8, torch.int16: MQ_TYPE_I16}[t.dtype]
+
+
+def quantize(x, alpha: float, z: int, q, stream=None) -> int:
+    """mq_quantize on CUDA tensors (float x -> int8 / int16 q); returns the status."""
+    return lib.mq_quantize(_ptr(x), _type_of(x), x.numel(), float(alpha), int(z), _ptr(q),
+                           _type_of(q), _stream(stream))
+
+
+def dequantize(q, alpha: float, z: int, f, stream=None) -> int:
+    """mq_dequantize on CUDA tensors (int8 / int16 q -> f32 f); returns the status."""
+    return lib.mq_dequantize(_ptr(q), _type_of(q), q.numel(), float(alpha), int(z), _ptr(f),
+                             _stream(stream))
+
+
+def requantize(q, zx: int, m0: int, shift: int, zy: int, y, stream=None) -> int:
+    """mq_requantize on CUDA tensors (int8 / int16 codes -> int8 / int16 codes)."""
+    return lib.mq_requantize(_ptr(q), _type_of(q), q.numel(), int(zx), int(m0), int(shift),
+                             int(zy), _ptr(y), _type_of(y), _stream(stream))
 
 
 def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y,

@@ -280,3 +280,30 @@ def test_a16_single_call_symbols(mq):
     f = mq.lib.mq_linear_w8a16
     assert f(FAKE, 4, 64, 64, 40000, FAKE, FAKE, 32, FAKE, FAKE, 0, FAKE, 32, FAKE, 1 << 30,
              None) == mq.MQ_ERR_INVALID_ARG
+
+
+def test_boundary_quantizer_validation(mq):
+    # every rejection happens on the host, before a launch
+    T = mq
+    q = mq.lib.mq_quantize
+    assert q(FAKE, T.MQ_TYPE_F32, 16, 0.0, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert q(FAKE, T.MQ_TYPE_F32, 16, float("inf"), 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert q(FAKE, T.MQ_TYPE_F32, 16, 1.0, 128, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert q(FAKE, T.MQ_TYPE_I8, 16, 1.0, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert q(FAKE, T.MQ_TYPE_F32, 16, 1.0, 0, FAKE, T.MQ_TYPE_F32, None) == mq.MQ_ERR_INVALID_ARG
+    assert q(FAKE, T.MQ_TYPE_F32, -1, 1.0, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert q(None, T.MQ_TYPE_F32, 0, 1.0, 0, None, T.MQ_TYPE_I8, None) == 0   # nothing to do
+    assert q(None, T.MQ_TYPE_F32, 4, 1.0, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert q(FAKE + 2, T.MQ_TYPE_F32, 4, 1.0, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_ALIGNMENT
+    assert q(FAKE, T.MQ_TYPE_F16, 4, 1.0, 0, FAKE + 1, T.MQ_TYPE_I16, None) == mq.MQ_ERR_ALIGNMENT
+    d = mq.lib.mq_dequantize
+    assert d(FAKE, T.MQ_TYPE_I16, 4, 1.0, 40000, FAKE, None) == mq.MQ_ERR_INVALID_ARG
+    assert d(FAKE, T.MQ_TYPE_F32, 4, 1.0, 0, FAKE, None) == mq.MQ_ERR_INVALID_ARG
+    assert d(FAKE, T.MQ_TYPE_I8, 4, 1.0, 0, FAKE + 2, None) == mq.MQ_ERR_ALIGNMENT
+    r = mq.lib.mq_requantize
+    assert r(FAKE, T.MQ_TYPE_I16, 4, 0, 1 << 30, 0, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert r(FAKE, T.MQ_TYPE_I16, 4, 0, 1 << 30, 63, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert r(FAKE, T.MQ_TYPE_I16, 4, 0, -1, 31, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert r(FAKE, T.MQ_TYPE_I8, 4, 200, 1 << 30, 31, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert r(FAKE, T.MQ_TYPE_I8, 4, 0, 1 << 30, 31, 200, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
+    assert r(FAKE + 1, T.MQ_TYPE_I16, 4, 0, 1 << 30, 31, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_ALIGNMENT
