@@ -33,8 +33,8 @@ def build(force: bool = False) -> str:
     if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < newest:
         tmp = _LIB + ".tmp.%d" % os.getpid()
         subprocess.check_call(
-            ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-Wall", "-Wextra",
-             "-o", tmp, _SRC, "-lm"])
+            ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared", "-Wall",
+             "-Wextra", "-o", tmp, _SRC, "-lm"])
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -60,6 +60,9 @@ def _bind(lib):
     lib.oracle_quantize_f32.argtypes = [p, i64, f32, i32, ci, p]
     lib.oracle_dequantize.argtypes = [p, ci, i64, f32, i32, p]
     lib.oracle_requantize.argtypes = [p, ci, i64, i32, i32, i32, i32, p, ci]
+    lib.oracle_fold_weights.argtypes = [p, ci, ci, p, p, p]
+    lib.oracle_quantize_weights.argtypes = [p, ci, ci, ci, ci, p, p, p]
+    lib.oracle_fold_norm.argtypes = [p, p, p, ci, p, p]
     lib.oracle_residual_add.argtypes = [p, p, i64, p]
     lib.oracle_residual_add.restype = None
     return lib
@@ -204,6 +207,41 @@ class Oracle:
     def requant_one_a16(self, acc: int, m0: int, shift: int, zy: int) -> int:
         return int(self.lib.oracle_requant_one_a16(int(acc), int(m0), int(shift), int(zy)))
 
+    def fold_weights(self, w: np.ndarray, s_in, s_out) -> np.ndarray:
+        """oracle_fold_weights: f32 [N, K] -> folded f32 [N, K]."""
+        w = np.ascontiguousarray(w, dtype=np.float32)
+        n, k = w.shape
+        si = np.ascontiguousarray(s_in, dtype=np.float32) if s_in is not None else None
+        so = np.ascontiguousarray(s_out, dtype=np.float32) if s_out is not None else None
+        out = np.zeros((n, k), np.float32)
+        _check(self.lib.oracle_fold_weights(_ptr(w), n, k, _ptr(si) if si is not None else None,
+                                            _ptr(so) if so is not None else None, _ptr(out)),
+               "oracle_fold_weights")
+        return out
+
+    def quantize_weights(self, w: np.ndarray, bits: int, scheme: int):
+        """oracle_quantize_weights: f32 [N, K] -> (codes int8 [N, K], sw f32 [N], zw int32 [N])."""
+        w = np.ascontiguousarray(w, dtype=np.float32)
+        n, k = w.shape
+        codes = np.zeros((n, k), np.int8)
+        sw = np.zeros(n, np.float32)
+        zw = np.zeros(n, np.int32)
+        _check(self.lib.oracle_quantize_weights(_ptr(w), n, k, bits, scheme, _ptr(codes), _ptr(sw),
+                                                _ptr(zw)), "oracle_quantize_weights")
+        return codes, sw, zw
+
+    def fold_norm(self, gamma: np.ndarray, beta, s: np.ndarray):
+        gamma = np.ascontiguousarray(gamma, dtype=np.float32)
+        s = np.ascontiguousarray(s, dtype=np.float32)
+        k = gamma.size
+        g = np.zeros(k, np.float32)
+        b = np.zeros(k, np.float32) if beta is not None else None
+        beta = np.ascontiguousarray(beta, dtype=np.float32) if beta is not None else None
+        _check(self.lib.oracle_fold_norm(_ptr(gamma), _ptr(beta) if beta is not None else None,
+                                         _ptr(s), k, _ptr(g), _ptr(b) if b is not None else None),
+               "oracle_fold_norm")
+        return g, b
+
     def quantize(self, x: np.ndarray, alpha: float, z: int, bits: int) -> np.ndarray:
         """oracle_quantize_f32: f32 values -> int8 / int16 codes."""
         x = np.ascontiguousarray(x, dtype=np.float32)
@@ -283,6 +321,18 @@ def requant_one_a16(acc, m0, shift, zy):
     return _default().requant_one_a16(acc, m0, shift, zy)
 
 
+def fold_weights(w, s_in, s_out):
+    return _default().fold_weights(w, s_in, s_out)
+
+
+def quantize_weights(w, bits, scheme):
+    return _default().quantize_weights(w, bits, scheme)
+
+
+def fold_norm(gamma, beta, s):
+    return _default().fold_norm(gamma, beta, s)
+
+
 def quantize(x, alpha, z, bits):
     return _default().quantize(x, alpha, z, bits)
 
@@ -307,8 +357,8 @@ def compile_variant(src_text: str, out_path: str) -> str:
         f.write(src_text)
     import shutil
     shutil.copy(_HDR, os.path.join(d, "mq_oracle.h"))
-    subprocess.check_call(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-o", out_path,
-                           c_path, "-lm"])
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared",
+                           "-o", out_path, c_path, "-lm"])
     return out_path
 
 

@@ -392,6 +392,81 @@ int oracle_requantize(const void *q, int in_bits, int64_t n, int32_t zx, int32_t
     return ORACLE_OK;
 }
 
+int oracle_fold_weights(const float *w, int N, int K, const float *s_in, const float *s_out,
+                        float *w_out) {
+    if (N < 0 || K < 0) return ORACLE_EINVAL;
+    for (int n = 0; n < N; ++n)
+        for (int k = 0; k < K; ++k) {
+            float v = w[(size_t)n * (size_t)K + (size_t)k];
+            if (s_in) v = v * s_in[k];   /* S W: input channel k */
+            if (s_out) v = v / s_out[n]; /* S^-1 of the next transform: output channel n */
+            w_out[(size_t)n * (size_t)K + (size_t)k] = v;
+        }
+    return ORACLE_OK;
+}
+
+int oracle_quantize_weights(const float *w, int N, int K, int bits, int scheme, int8_t *codes,
+                            float *sw, int32_t *zw) {
+    if (N < 0 || K < 0 || (bits != 8 && bits != 4) || scheme < 0 || scheme > 2)
+        return ORACLE_EINVAL;
+    if (scheme != 0 && !zw) return ORACLE_EINVAL;
+    const int32_t qmin = bits == 8 ? -128 : -8, qmax = bits == 8 ? 127 : 7;
+    /* per-tensor statistics (scheme 2) */
+    float tlo = 0.0f, thi = 0.0f;
+    for (int n = 0; scheme == 2 && n < N; ++n)
+        for (int k = 0; k < K; ++k) {
+            float v = w[(size_t)n * (size_t)K + (size_t)k];
+            if (v < tlo) tlo = v;
+            if (v > thi) thi = v;
+        }
+    for (int n = 0; n < N; ++n) {
+        const float *row = w + (size_t)n * (size_t)K;
+        float lo = 0.0f, hi = 0.0f;
+        if (scheme == 2) {
+            lo = tlo;
+            hi = thi;
+        } else {
+            for (int k = 0; k < K; ++k) {
+                if (row[k] < lo) lo = row[k];
+                if (row[k] > hi) hi = row[k];
+            }
+        }
+        float scale;
+        int32_t zero = 0;
+        if (scheme == 0) {
+            float amax = -lo > hi ? -lo : hi;
+            if (!(amax > 0.0f)) amax = 1e-8f;
+            scale = amax / (float)qmax;
+        } else {
+            float span = hi - lo;
+            if (!(span > 0.0f)) span = 1e-8f;
+            scale = span / (float)(qmax - qmin);
+            float zf = rintf((float)qmin - lo / scale);
+            zero = (int32_t)(zf < qmin ? qmin : (zf > qmax ? qmax : zf));
+        }
+        const int32_t cmin = (scheme == 0 && bits == 8) ? -qmax : qmin;
+        for (int k = 0; k < K; ++k) {
+            double c = (double)rintf(row[k] / scale) + (double)zero;
+            if (c < cmin) c = cmin;
+            if (c > qmax) c = qmax;
+            codes[(size_t)n * (size_t)K + (size_t)k] = (int8_t)c;
+        }
+        sw[n] = scale;
+        if (zw) zw[n] = zero;
+    }
+    return ORACLE_OK;
+}
+
+int oracle_fold_norm(const float *gamma, const float *beta, const float *s, int K,
+                     float *gamma_out, float *beta_out) {
+    if (K < 0 || (K > 0 && (!gamma || !s || !gamma_out))) return ORACLE_EINVAL;
+    for (int k = 0; k < K; ++k) {
+        gamma_out[k] = gamma[k] / s[k];
+        if (beta && beta_out) beta_out[k] = beta[k] / s[k];
+    }
+    return ORACLE_OK;
+}
+
 void oracle_residual_add(const int8_t *a, const int8_t *b, int64_t n,
                          int8_t *out) {
     for (int64_t i = 0; i < n; ++i) {

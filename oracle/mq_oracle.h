@@ -192,6 +192,47 @@ int oracle_requantize(const void *q, int in_bits, int64_t n, int32_t zx, int32_t
                       int32_t shift, int32_t zy, void *y, int out_bits);
 
 /*
+ * Offline weight preparation, step 1: the equivalent transform of eq. 1
+ * folded into the weights.  With weights stored [N out][K in] (the transpose
+ * of the paper's W), eq. 1's S W scales input channel k by s_in[k], and the
+ * S^-1 of the next transform (Figure 3: S0 W1 S1^-1, S1 W2) scales output
+ * channel n by 1 / s_out[n]:
+ *   w_out[n][k] = (w[n][k] * s_in[k]) / s_out[n]
+ * in f32, multiply first, each operation rounded to nearest; s_in or s_out
+ * may be NULL (that factor is skipped).
+ * Pinned by: exact rationals, float equivalence of eq. 1 through one layer
+ * and through norm + two layers (Figure 3).
+ */
+int oracle_fold_weights(const float *w, int N, int K, const float *s_in, const float *s_out,
+                        float *w_out);
+
+/*
+ * Step 2: weight quantization of f32 weights [N][K], the integer decisions
+ * taken in f32 (reading R12), per output channel or per tensor:
+ *   scheme 0, symmetric per channel: amax = max|w[n]| (1e-8 if 0),
+ *     sw = amax / qmax, q = clamp(rint(w / sw), -qmax, qmax) for int8
+ *     (qmax 127) and clamp(., -8, 7) with qmax 7 for int4; zw = 0.
+ *   scheme 1 / 2, asymmetric per channel / per tensor (eqs. 2-4 on weights,
+ *     Sec. 5.1): lo = min(min w, 0), hi = max(max w, 0), span = hi - lo
+ *     (1e-8 if 0), sw = span / (qmax - qmin), zw = clamp(rint(qmin - lo / sw)),
+ *     q = clamp(rint(w / sw) + zw, qmin, qmax) with [qmin, qmax] the code range.
+ * codes: int8 [N][K] (values in the bits' range), sw: f32 [N], zw: int32 [N]
+ * (may be NULL for scheme 0).
+ * Pinned by: exact rationals (every f32 operation rounded by hand), the code
+ * range reached, the half-step bound, zero mapping to zw, per-tensor sharing.
+ */
+int oracle_quantize_weights(const float *w, int N, int K, int bits, int scheme, int8_t *codes,
+                            float *sw, int32_t *zw);
+
+/*
+ * The norm's affine A before the first transformed linear absorbs S0^-1
+ * (Figure 3): gamma'[k] = gamma[k] / s[k], beta'[k] = beta[k] / s[k] in f32.
+ * beta / beta_out may be NULL (RMSNorm has no shift).
+ */
+int oracle_fold_norm(const float *gamma, const float *beta, const float *s, int K,
+                     float *gamma_out, float *beta_out);
+
+/*
  * Requantize one accumulator: clamp(zy + floor(acc*M0 / 2^s + 1/2), -128, 127).
  * Exposed so that tests can sweep accumulators around rounding ties.
  */

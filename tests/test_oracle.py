@@ -560,6 +560,138 @@ def pin_requantize_vs_eq4(orc: Oracle):
     assert diff.max() <= 1 and (diff != 0).mean() < 1e-3
 
 
+# ---- offline fold of eq. 1 and weight quantization ------------------------------
+
+def _fold_ref(w, s_in, s_out):
+    n_, k_ = w.shape
+    out = np.zeros((n_, k_), np.float64)
+    for n in range(n_):
+        for k in range(k_):
+            v = float(w[n, k])
+            if s_in is not None:
+                v = _f32_nearest(Fraction(v) * Fraction(float(s_in[k])))
+            if s_out is not None:
+                v = _f32_nearest(Fraction(v) / Fraction(float(s_out[n])))
+            out[n, k] = v
+    return out
+
+
+def _quantize_weights_ref(w, bits, scheme):
+    """Every f32 operation of the definition rounded by hand from exact rationals."""
+    qmin, qmax = (-128, 127) if bits == 8 else (-8, 7)
+    n_, k_ = w.shape
+    codes = np.zeros((n_, k_), np.int64)
+    sw = np.zeros(n_)
+    zw = np.zeros(n_, np.int64)
+    tlo, thi = min(float(w.min()), 0.0), max(float(w.max()), 0.0)
+    for n in range(n_):
+        lo, hi = (tlo, thi) if scheme == 2 else (min(float(w[n].min()), 0.0),
+                                                  max(float(w[n].max()), 0.0))
+        if scheme == 0:
+            amax = max(-lo, hi) or float(np.float32(1e-8))
+            scale = _f32_nearest(Fraction(amax) / qmax)
+            zero, cmin = 0, (-qmax if bits == 8 else qmin)
+        else:
+            span = _f32_nearest(Fraction(hi) - Fraction(lo))
+            if not span > 0:
+                span = float(np.float32(1e-8))
+            scale = _f32_nearest(Fraction(span) / (qmax - qmin))
+            zf = round(_f32_nearest(Fraction(qmin) - Fraction(_f32_nearest(Fraction(lo) /
+                                                                             Fraction(scale)))))
+            zero, cmin = max(qmin, min(qmax, zf)), qmin
+        for k in range(k_):
+            t = round(_f32_nearest(Fraction(float(w[n, k])) / Fraction(scale)))
+            codes[n, k] = max(cmin, min(qmax, t + zero))
+        sw[n], zw[n] = scale, zero
+    return codes, sw, zw
+
+
+def pin_fold_exact(orc: Oracle):
+    rng = np.random.default_rng(201)
+    w = (rng.standard_normal((5, 24)) * 0.02).astype(np.float32)
+    s_in = rng.uniform(0.3, 3.0, 24).astype(np.float32)
+    s_out = rng.uniform(0.3, 3.0, 5).astype(np.float32)
+    for si, so in ((s_in, None), (None, s_out), (s_in, s_out)):
+        got = orc.fold_weights(w, si, so).astype(np.float64)
+        assert np.array_equal(got, _fold_ref(w, si, so))
+
+
+def pin_quantize_weights_exact(orc: Oracle):
+    rng = np.random.default_rng(202)
+    w = (rng.standard_normal((6, 40)) * 0.02).astype(np.float32)
+    w[2] += 0.01           # a channel biased positive
+    w[3] = 0.0             # an all-zero channel
+    w[4, :5] = [0.0625, -0.03125, 0.015625, 0.0, -0.0625]   # exact power-of-two values
+    for bits in (8, 4):
+        for scheme in (0, 1, 2):
+            c, sw, zw = orc.quantize_weights(w, bits, scheme)
+            rc, rsw, rzw = _quantize_weights_ref(w, bits, scheme)
+            assert np.array_equal(c.astype(np.int64), rc), (bits, scheme)
+            assert np.array_equal(sw.astype(np.float64), rsw), (bits, scheme)
+            assert np.array_equal(zw.astype(np.int64), rzw), (bits, scheme)
+
+
+def pin_fold_equivalence(orc: Oracle):
+    """Eq. 1: X W = (X S^-1)(S W), before quantization, through one layer and
+    through the norm + two linears of Figure 3 (S0 on the norm and W1's
+    inputs, S1 between W1 and W2)."""
+    rng = np.random.default_rng(203)
+    x = rng.standard_normal((16, 64))
+    w1 = (rng.standard_normal((48, 64)) * 0.05).astype(np.float32)
+    w2 = (rng.standard_normal((32, 48)) * 0.05).astype(np.float32)
+    s0 = rng.uniform(0.2, 5.0, 64).astype(np.float32)
+    s1 = rng.uniform(0.2, 5.0, 48).astype(np.float32)
+    gamma = rng.uniform(0.5, 1.5, 64).astype(np.float32)
+    beta = rng.uniform(-0.2, 0.2, 64).astype(np.float32)
+    ref1 = x @ w1.astype(np.float64).T
+    f1 = orc.fold_weights(w1, s0, None).astype(np.float64)
+    got1 = (x / s0.astype(np.float64)) @ f1.T
+    assert np.allclose(got1, ref1, rtol=0, atol=1e-6 * np.abs(ref1).max())
+    g1, b1 = orc.fold_norm(gamma, beta, s0)
+    f1 = orc.fold_weights(w1, s0, s1).astype(np.float64)
+    f2 = orc.fold_weights(w2, s1, None).astype(np.float64)
+    h = x * gamma.astype(np.float64) + beta.astype(np.float64)
+    ref2 = (h @ w1.astype(np.float64).T) @ w2.astype(np.float64).T
+    hf = x * g1.astype(np.float64) + b1.astype(np.float64)
+    got2 = (hf @ f1.T) @ f2.T
+    assert np.allclose(got2, ref2, rtol=0, atol=2e-6 * np.abs(ref2).max())
+    # with a wrong direction of either factor the equivalence breaks
+    bad = orc.fold_weights(w1, 1 / s0, None).astype(np.float64)
+    assert not np.allclose((x / s0) @ bad.T, ref1, atol=1e-3 * np.abs(ref1).max())
+
+
+def pin_quantize_weights_properties(orc: Oracle):
+    rng = np.random.default_rng(204)
+    w = (rng.standard_normal((20, 300)) * 0.02).astype(np.float32)
+    w[::3] -= 0.015
+    for bits in (8, 4):
+        qmin, qmax = (-128, 127) if bits == 8 else (-8, 7)
+        c, sw, _ = orc.quantize_weights(w, bits, 0)
+        c = c.astype(np.int64)
+        # the largest magnitude of each row lands on +-qmax; half-step error
+        assert np.all(np.abs(c).max(axis=1) == qmax)
+        err = np.abs(c * sw[:, None].astype(np.float64) - w.astype(np.float64))
+        assert np.all(err[np.abs(c) < qmax] <= 0.5 * sw[:, None].repeat(300, 1)[np.abs(c) < qmax]
+                      * (1 + 1e-6))
+        for scheme in (1, 2):
+            c, sw, zw = orc.quantize_weights(w, bits, scheme)
+            c = c.astype(np.int64)
+            assert c.min() >= qmin and c.max() <= qmax
+            # the real zero maps to the zero point exactly
+            cz, _, zz = orc.quantize_weights(np.concatenate([w, np.zeros((20, 1), np.float32)], 1),
+                                             bits, scheme)
+            assert np.array_equal(cz[:, -1].astype(np.int64), zz.astype(np.int64))
+            deq = (c - zw[:, None]) * sw[:, None].astype(np.float64)
+            inside = (c > qmin) & (c < qmax)
+            assert np.all(np.abs(deq - w)[inside] <= 0.5 * np.repeat(sw[:, None], 300, 1)[inside]
+                          * (1 + 1e-5))
+            if scheme == 2:
+                assert len(set(sw.tolist())) == 1 and len(set(zw.tolist())) == 1
+                assert c.min() == qmin or c.max() == qmax
+            else:
+                assert np.all((c.min(axis=1) == qmin) | (c.max(axis=1) == qmax))
+
+
 PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zero_point_identity,
                pin_exact_dequant, pin_requant_closed_form, pin_requant_ties, pin_requant_vs_eq4,
                pin_requant_params_bound, pin_asym_k1_exhaustive, pin_asym_int4_pairs,
@@ -568,7 +700,8 @@ PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zer
                pin_a16_large_accumulators, pin_a16_reduces_to_int8, pin_a16_byte_planes, pin_a16_exact_dequant,
                pin_a16_requant_closed_form_and_saturation, pin_a16_requant_vs_eq4,
                pin_quantize_exact, pin_quantize_ties_and_invariants, pin_dequantize_exact,
-               pin_requantize_exhaustive, pin_requantize_vs_eq4]
+               pin_requantize_exhaustive, pin_requantize_vs_eq4, pin_fold_exact,
+               pin_quantize_weights_exact, pin_fold_equivalence, pin_quantize_weights_properties]
 
 
 # ----------------------------------------------------------------------------
@@ -816,6 +949,22 @@ def test_boundary_quantizers_reject_bad_arguments(O):
         O.requantize(q, 200, 1 << 30, 31, 0, 8)   # zx outside int8
 
 
+def test_fold_exact(O):
+    pin_fold_exact(O)
+
+
+def test_quantize_weights_exact(O):
+    pin_quantize_weights_exact(O)
+
+
+def test_fold_equivalence(O):
+    pin_fold_equivalence(O)
+
+
+def test_quantize_weights_properties(O):
+    pin_quantize_weights_properties(O)
+
+
 MUTATIONS = [
     ("zero point sign", "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - zx;",
      "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] + zx;"),
@@ -862,6 +1011,16 @@ MUTATIONS = [
      "int64_t centered = (int64_t)oracle_code_at(q, in_bits, i) - zx;",
      "int64_t centered = (int64_t)oracle_code_at(q, in_bits, i);"),
     ("requantize wrong output range", "if (out > ohi) out = ohi;", "if (out > ihi) out = ihi;"),
+    ("fold by reciprocal multiply", "if (s_out) v = v / s_out[n];",
+     "if (s_out) v = v * (1.0f / s_out[n]);"),
+    ("fold divides the input channel", "if (s_in) v = v * s_in[k];", "if (s_in) v = v / s_in[k];"),
+    ("norm fold multiplies", "gamma_out[k] = gamma[k] / s[k];", "gamma_out[k] = gamma[k] * s[k];"),
+    ("symmetric amax ignores negatives", "float amax = -lo > hi ? -lo : hi;", "float amax = hi;"),
+    ("quantizer weight zero point sign", "float zf = rintf((float)qmin - lo / scale);",
+     "float zf = rintf((float)qmin + lo / scale);"),
+    ("per-tensor statistics per row", "        if (scheme == 2) {\n            lo = tlo;",
+     "        if (scheme == 3) {\n            lo = tlo;"),
+    ("asymmetric span from the row maximum only", "float span = hi - lo;", "float span = hi;"),
     ("a16 output zero point dropped",
      "__int128 out = (__int128)zy + oracle_round_shift(acc, M0, shift);",
      "__int128 out = oracle_round_shift(acc, M0, shift);"),
