@@ -539,6 +539,42 @@ def run_glue(mq, torch, n: int = 1 << 26, reps: int = 20):
     return out
 
 
+def run_weight_pipeline(mq, torch, reps: int = 5):
+    """The offline weight pipeline (fold of eq. 1, quantization, packing,
+    colsum) over the TinyLlama block's seven f32 weight matrices (176 MB), in
+    the paper's W8A8 setting (asymmetric per tensor, down per channel) and
+    W4A8 (asymmetric per channel): microseconds per block and GB/s of f32
+    weights (each read twice: statistics, then codes)."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(9)
+    mats = [(torch.randn((n, k), device="cuda", generator=g) * 0.02,
+             torch.rand(k, device="cuda", generator=g) + 0.5) for _, k, n in synth.TINYLLAMA_LINEARS]
+    stream = torch.cuda.current_stream()
+    out = {}
+    fbytes = sum(w.numel() * 4 for w, _ in mats)
+    for bits in (8, 4):
+        schemes = [synth.paper_weight_scheme(name, bits) for name, _, _ in synth.TINYLLAMA_LINEARS]
+        codes = [mq.MQ_WEIGHTS_ASYM_TENSOR if s_ == "asym_tensor" else mq.MQ_WEIGHTS_ASYM_CHANNEL
+                 for s_ in schemes]
+
+        def block():
+            for (w, s_in), sc in zip(mats, codes):
+                mq.fold_quantize_pack(w, bits, sc, s_in)
+        block()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            block()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        out[f"w{bits}a8_block"] = {"us": round(ms * 1e3, 1),
+                                   "gbs_f32_weights": round(fbytes / (ms * 1e-3) / 1e9, 1)}
+    del mats
+    return out
+
+
 # --------------------------------------------------------------------------- CPU oracle
 def oracle_sample(blocks_cases, rows: range, col_frac: float = 1.0):
     """Run the oracle on `rows` of every linear of one block; returns
@@ -648,6 +684,7 @@ def main():
     asym_dec = run_decode(mq, torch, asym=True, ms=(1, 16))
     a16 = run_a16(mq, torch)
     glue = run_glue(mq, torch)
+    wpipe = run_weight_pipeline(mq, torch)
     peaks = measured_peaks()
 
     ops = block_ops(PREFILL_M)
@@ -694,6 +731,8 @@ def main():
                 "w8a8_us_per_block": round(pre["total_ms"] / args.steps * 1e3, 2),
                 "w4a8_m1_stream_us": decode["m1"]["stream_us"]},
         "boundary_quantizers": {"unit": "GB/s of input + output bytes", **glue},
+        "weight_pipeline": {"what": "fold of eq. 1 + quantize + pack + colsum, 7 linears, "
+                                    "176 MB of f32 weights", **wpipe},
     }
     if rank == 0 and world == 1:
         line["cpu_baseline"] = cpu_baseline(pre["blocks"], torch)

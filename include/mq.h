@@ -351,6 +351,50 @@ int mq_dequantize(const void *q, int in_type, int64_t n, float alpha, int32_t z,
 int mq_requantize(const void *q, int in_type, int64_t n, int32_t zx, int32_t M0, int32_t shift,
                   int32_t zy, void *y, int out_type, void *stream);
 
+/* ---- Offline weight pipeline ---------------------------------------------- */
+#define MQ_WEIGHTS_SYM_CHANNEL 0  /* symmetric per output channel (Appendix A) */
+#define MQ_WEIGHTS_ASYM_CHANNEL 1 /* asymmetric per output channel (Sec. 5.1: W4A8, down_proj) */
+#define MQ_WEIGHTS_ASYM_TENSOR 2  /* asymmetric per tensor (Sec. 5.1: W8A8) */
+
+/*
+ * The producer of the weights the layer consumes, on the device, for one
+ * linear: fold the equivalent transform of eq. 1 into f32 weights, quantize,
+ * pack and compute colsum.  Weights are stored [N out][K in]; eq. 1's S W
+ * scales input channel k by s_in[k], and the S^-1 of the next transform
+ * (Figure 3: S0 W1 S1^-1, S1 W2) scales output channel n by 1 / s_out[n]:
+ *   w'[n][k] = (w[n][k] * s_in[k]) / s_out[n]          (f32, multiply first)
+ * then, with every step one f32 operation rounded to nearest:
+ *   MQ_WEIGHTS_SYM_CHANNEL: amax = max|w'[n]| (1e-8 if 0), sw = amax / qmax,
+ *     q = clamp(rint(w' / sw), -qmax, qmax), qmax 127 (int8); for int4
+ *     clamp(., -8, 7) with qmax 7; zw = 0.
+ *   MQ_WEIGHTS_ASYM_CHANNEL / _TENSOR: lo = min(min w', 0), hi = max(max w', 0)
+ *     over the channel / the tensor, sw = (hi - lo) / (qmax - qmin) (1e-8
+ *     span if 0), zw = clamp(rint(qmin - lo / sw)), q = clamp(rint(w' / sw) + zw).
+ * rint rounds ties to even.
+ *   w       : device f32 [N][K], finite values
+ *   s_in    : device f32 [K] or NULL;  s_out: device f32 [N] or NULL (positive)
+ *   packed, colsum : as mq_pack_weights(bits) (colsum of the codes)
+ *   sw      : device f32 [N], the weight scales (for mq_requant_params)
+ *   zw      : device int32 [N], the weight zero points (the `zw` of
+ *             mq_linear_desc); may be NULL for MQ_WEIGHTS_SYM_CHANNEL
+ *   stats   : device f32 [2N] scratch
+ * Requirements: N, K >= 0; bits 8, or 4 with K even; pointers aligned to
+ * their element size.  Asynchronous on `stream`.
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_ALIGNMENT, MQ_ERR_CUDA.
+ */
+int mq_fold_quantize_pack(const float *w, int N, int K, const float *s_in, const float *s_out,
+                          int bits, int scheme, void *packed, int32_t *colsum, float *sw,
+                          int32_t *zw, float *stats, void *stream);
+
+/*
+ * The norm's affine before the first transformed linear absorbs S0^-1
+ * (Figure 3): gamma_out[k] = gamma[k] / s[k], beta_out[k] = beta[k] / s[k],
+ * f32.  Host arrays; beta and beta_out may be NULL (RMSNorm has no shift).
+ * Errors: MQ_ERR_INVALID_ARG.
+ */
+int mq_fold_norm(const float *gamma, const float *beta, const float *s, int K, float *gamma_out,
+                 float *beta_out);
+
 /*
  * Wait for `stream` and report device-side failures recorded by this
  * library's kernels since the previous call: MQ_ERR_DEVICE_TIMEOUT if a

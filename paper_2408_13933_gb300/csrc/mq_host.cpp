@@ -468,6 +468,36 @@ int mq_requantize(const void *q, int in_type, int64_t n, int32_t zx, int32_t M0,
     return mq::launch_glue(2, in_type, out_type, q, y, n, 0.0f, zx, zy, M0, shift, lo, hi, stream);
 }
 
+int mq_fold_quantize_pack(const float *w, int N, int K, const float *s_in, const float *s_out,
+                          int bits, int scheme, void *packed, int32_t *colsum, float *sw,
+                          int32_t *zw, float *stats, void *stream) {
+    if (N < 0 || K < 0 || (bits != 8 && bits != 4) || scheme < MQ_WEIGHTS_SYM_CHANNEL ||
+        scheme > MQ_WEIGHTS_ASYM_TENSOR)
+        return MQ_ERR_INVALID_ARG;
+    if (bits == 4 && (K & 1)) return MQ_ERR_INVALID_ARG;
+    if (N == 0) return MQ_OK;
+    if (!colsum || !sw || !stats || (scheme != MQ_WEIGHTS_SYM_CHANNEL && !zw))
+        return MQ_ERR_INVALID_ARG;
+    if (K > 0 && (!w || !packed)) return MQ_ERR_INVALID_ARG;
+    if (!aligned_to(w, 4) || !aligned_to(s_in, 4) || !aligned_to(s_out, 4) ||
+        !aligned_to(colsum, 4) || !aligned_to(sw, 4) || !aligned_to(zw, 4) || !aligned_to(stats, 4))
+        return MQ_ERR_ALIGNMENT;
+    return mq::launch_fold(w, N, K, s_in, s_out, bits, scheme, packed, colsum, sw, zw, stats,
+                           stream);
+}
+
+int mq_fold_norm(const float *gamma, const float *beta, const float *s, int K, float *gamma_out,
+                 float *beta_out) {
+    if (K < 0) return MQ_ERR_INVALID_ARG;
+    if (K > 0 && (!gamma || !s || !gamma_out || (beta && !beta_out))) return MQ_ERR_INVALID_ARG;
+    for (int k = 0; k < K; ++k) {
+        if (!(std::isfinite(s[k]) && s[k] > 0.0f)) return MQ_ERR_INVALID_ARG;
+        gamma_out[k] = gamma[k] / s[k];
+        if (beta) beta_out[k] = beta[k] / s[k];
+    }
+    return MQ_OK;
+}
+
 int mq_check_device_status(void *stream) {
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (cudaStreamSynchronize(s) != cudaSuccess) return MQ_ERR_CUDA;

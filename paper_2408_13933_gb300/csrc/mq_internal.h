@@ -88,4 +88,10 @@ int launch_glue(int kind, int in_type, int out_type, const void *in, void *out, 
                 float alpha, int32_t zin, int32_t zout, int32_t m0, int32_t shift, int32_t lo,
                 int32_t hi, void *stream);
 
+// Offline weight pipeline (mq_fold.cu): fold eq. 1 into f32 weights,
+// quantize by `scheme` (MQ_WEIGHTS_*), pack, colsum.
+int launch_fold(const float *w, int N, int K, const float *s_in, const float *s_out, int bits,
+                int scheme, void *packed, int32_t *colsum, float *sw, int32_t *zw, float *stats,
+                void *stream);
+
 }  // namespace mq

@@ -40,7 +40,8 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
             "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch",
             "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16", "mq_quantize",
-            "mq_dequantize", "mq_requantize"]
+            "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm"]
+MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
 _vp, _i32, _int, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int, ctypes.c_size_t
@@ -76,6 +77,9 @@ _i64, _f32 = ctypes.c_int64, ctypes.c_float
 lib.mq_quantize.argtypes = [_vp, _int, _i64, _f32, _i32, _vp, _int, _vp]
 lib.mq_dequantize.argtypes = [_vp, _int, _i64, _f32, _i32, _vp, _vp]
 lib.mq_requantize.argtypes = [_vp, _int, _i64, _i32, _i32, _i32, _i32, _vp, _int, _vp]
+lib.mq_fold_quantize_pack.argtypes = [_vp, _int, _int, _vp, _vp, _int, _int, _vp, _vp, _vp, _vp,
+                                      _vp, _vp]
+lib.mq_fold_norm.argtypes = [_vp, _vp, _vp, _int, _vp, _vp]
 for _f in EXPORTED:
     if _f != "mq_status_string":
         getattr(lib, _f).restype = _int
@@ -225,6 +229,36 @@ def requantize(q, zx: int, m0: int, shift: int, zy: int, y, stream=None) -> int:
     """mq_requantize on CUDA tensors (int8 / int16 codes -> int8 / int16 codes)."""
     return lib.mq_requantize(_ptr(q), _type_of(q), q.numel(), int(zx), int(m0), int(shift),
                              int(zy), _ptr(y), _type_of(y), _stream(stream))
+
+
+def fold_quantize_pack(w, bits: int, scheme: int, s_in=None, s_out=None, stream=None):
+    """mq_fold_quantize_pack on a CUDA f32 tensor [N, K]: returns (packed, colsum,
+    sw, zw) on the device (zw None for the symmetric scheme)."""
+    import torch
+    n, k = w.shape
+    dev = w.device
+    packed = torch.empty(packed_size(n, k, bits), dtype=torch.uint8, device=dev)
+    colsum = torch.empty(n, dtype=torch.int32, device=dev)
+    sw = torch.empty(n, dtype=torch.float32, device=dev)
+    zw = torch.empty(n, dtype=torch.int32, device=dev) if scheme != MQ_WEIGHTS_SYM_CHANNEL else None
+    stats = torch.empty(2 * max(n, 1), dtype=torch.float32, device=dev)
+    _check(lib.mq_fold_quantize_pack(_ptr(w), n, k, _ptr(s_in), _ptr(s_out), bits, scheme,
+                                     _ptr(packed), _ptr(colsum), _ptr(sw), _ptr(zw), _ptr(stats),
+                                     _stream(stream)), "mq_fold_quantize_pack")
+    return (packed.view(n, packed.numel() // n) if n else packed), colsum, sw, zw
+
+
+def fold_norm(gamma: np.ndarray, beta, s: np.ndarray):
+    """mq_fold_norm on host f32 arrays: returns (gamma', beta')."""
+    gamma = np.ascontiguousarray(gamma, dtype=np.float32)
+    s = np.ascontiguousarray(s, dtype=np.float32)
+    g = np.zeros_like(gamma)
+    b = np.zeros_like(gamma) if beta is not None else None
+    if beta is not None:
+        beta = np.ascontiguousarray(beta, dtype=np.float32)
+    _check(lib.mq_fold_norm(_ptr(gamma), _ptr(beta), _ptr(s), gamma.size, _ptr(g), _ptr(b)),
+           "mq_fold_norm")
+    return g, b
 
 
 def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y,

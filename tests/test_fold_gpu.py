@@ -1,0 +1,104 @@
+"""The offline weight pipeline on the GPU (fold of eq. 1, weight quantization,
+packing, colsum) against the oracle's fold_weights -> quantize_weights ->
+pack, bit for bit, for every scheme and weight width; and the folded,
+quantized weights driving the integer layer end to end."""
+import numpy as np
+import pytest
+
+import oracle
+from gpu_helpers import assert_equal_int8, torch_cuda, upload
+from paper_2408_13933_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def mq():
+    from paper_2408_13933_gb300 import mq as m
+    return m
+
+
+def _weights(seed, n, k):
+    rng = np.random.default_rng(seed)
+    w = (rng.standard_normal((n, k)) * 0.02).astype(np.float32)
+    if n > 3:
+        w[1] += 0.012          # biased channel
+        w[2] = 0.0             # all-zero channel
+        w[3, ::7] *= 15.0      # outliers
+    s_in = rng.uniform(0.25, 4.0, k).astype(np.float32)
+    s_out = rng.uniform(0.25, 4.0, n).astype(np.float32)
+    return w, s_in, s_out
+
+
+def _run(w, s_in, s_out, bits, scheme):
+    lib = mq()
+    wd = upload(w)
+    si = upload(s_in) if s_in is not None else None
+    so = upload(s_out) if s_out is not None else None
+    packed, colsum, sw, zw = lib.fold_quantize_pack(wd, bits, scheme, si, so)
+    torch_cuda().cuda.synchronize()
+    return (packed.cpu().numpy(), colsum.cpu().numpy(), sw.cpu().numpy(),
+            zw.cpu().numpy() if zw is not None else None)
+
+
+def _want(w, s_in, s_out, bits, scheme):
+    f = oracle.fold_weights(w, s_in, s_out)
+    codes, sw, zw = oracle.quantize_weights(f, bits, scheme)
+    packed, colsum = oracle.pack(codes, bits)
+    return packed, colsum, sw, zw, codes
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("scheme", [0, 1, 2])
+@pytest.mark.parametrize("factors", ["none", "in", "out", "both"])
+@pytest.mark.parametrize("shape", [(37, 200), (256, 2048), (5, 5632)],
+                         ids=lambda s: "x".join(map(str, s)))
+def test_fold_quantize_pack(shape, factors, scheme, bits):
+    n, k = shape
+    w, s_in, s_out = _weights(n + k + scheme, n, k)
+    si = s_in if factors in ("in", "both") else None
+    so = s_out if factors in ("out", "both") else None
+    got = _run(w, si, so, bits, scheme)
+    want = _want(w, si, so, bits, scheme)
+    assert np.array_equal(got[2].view(np.uint32), want[2].view(np.uint32)), "scales"
+    assert np.array_equal(got[0].reshape(want[0].shape), want[0]), "packed codes"
+    assert np.array_equal(got[1], want[1]), "colsum"
+    if scheme != 0:
+        assert np.array_equal(got[3], want[3]), "zero points"
+
+
+def test_fold_edge_shapes():
+    for n, k in ((1, 2), (3, 0), (1, 64)):
+        w, _, _ = _weights(9, n, k)
+        for scheme in (0, 2):
+            got = _run(w, None, None, 4 if k % 2 == 0 else 8, scheme)
+            want = _want(w, None, None, 4 if k % 2 == 0 else 8, scheme)
+            assert np.array_equal(got[1], want[1]) and np.array_equal(got[2], want[2])
+
+
+@pytest.mark.parametrize("bits,scheme", [(8, 2), (8, 1), (4, 1), (4, 0)])
+def test_folded_weights_drive_the_layer(bits, scheme):
+    # fold -> quantize -> pack on the device, then the integer layer with the
+    # resulting (asymmetric) weights, against the oracle's chain
+    torch = torch_cuda()
+    lib = mq()
+    m, n, k = 40, 96, 512
+    w, s_in, _ = _weights(77 + bits + scheme, n, k)
+    packed, colsum, sw, zw = lib.fold_quantize_pack(upload(w), bits, scheme, upload(s_in))
+    x = synth.random_case(78, m, k, n, bits).x
+    zx, sx, sy, zy = 5, 0.02, 0.05, -7
+    m0, sh = lib.requant_params(sw.cpu().numpy(), sx, sy)
+    y = torch.full((m, n), 99, dtype=torch.int8, device="cuda")
+    # the descriptor holds raw addresses: keep every operand alive until the call is done
+    keep = [upload(a) for a in (x, m0, sh)]
+    d = lib.make_desc(keep[0], zx, packed, colsum, n, keep[1], keep[2], zy, y, bits, zw=zw)
+    need = lib.workspace_size_batch([d])
+    ws = torch.zeros(max(need, 16), dtype=torch.uint8, device="cuda")
+    assert lib.linear_batch([d], workspace=ws, ws_bytes=need) == 0
+    torch.cuda.synchronize()
+    assert lib.check_device_status() == 0
+    _, _, osw, ozw, codes = _want(w, s_in, None, bits, scheme)
+    opk, _ = oracle.pack(codes, bits)
+    om0, osh = oracle.requant_params(sx, osw, sy)
+    want = oracle.linear(x, zx, opk, bits, n, om0, osh, zy,
+                         zw=ozw if scheme != 0 else None)
+    assert_equal_int8(y.cpu().numpy(), want, f"folded layer bits={bits} scheme={scheme}")

@@ -307,3 +307,26 @@ def test_boundary_quantizer_validation(mq):
     assert r(FAKE, T.MQ_TYPE_I8, 4, 200, 1 << 30, 31, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
     assert r(FAKE, T.MQ_TYPE_I8, 4, 0, 1 << 30, 31, 200, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_INVALID_ARG
     assert r(FAKE + 1, T.MQ_TYPE_I16, 4, 0, 1 << 30, 31, 0, FAKE, T.MQ_TYPE_I8, None) == mq.MQ_ERR_ALIGNMENT
+
+
+def test_fold_validation_and_norm(mq):
+    import numpy as np
+    f = mq.lib.mq_fold_quantize_pack
+    # rejections before any launch
+    assert f(FAKE, 4, 64, None, None, 6, 0, FAKE, FAKE, FAKE, None, FAKE, None) == mq.MQ_ERR_INVALID_ARG
+    assert f(FAKE, 4, 63, None, None, 4, 0, FAKE, FAKE, FAKE, None, FAKE, None) == mq.MQ_ERR_INVALID_ARG
+    assert f(FAKE, 4, 64, None, None, 8, 3, FAKE, FAKE, FAKE, FAKE, FAKE, None) == mq.MQ_ERR_INVALID_ARG
+    assert f(FAKE, 4, 64, None, None, 8, 1, FAKE, FAKE, FAKE, None, FAKE, None) == mq.MQ_ERR_INVALID_ARG
+    assert f(FAKE, 4, 64, None, None, 8, 0, FAKE, FAKE, FAKE, None, None, None) == mq.MQ_ERR_INVALID_ARG
+    assert f(FAKE + 2, 4, 64, None, None, 8, 0, FAKE, FAKE, FAKE, None, FAKE, None) == mq.MQ_ERR_ALIGNMENT
+    assert f(None, 0, 64, None, None, 8, 0, None, None, None, None, None, None) == 0
+    # the norm fold on the host: gamma / s, beta / s in f32
+    g = np.array([1.0, 2.0, -3.0, 0.5], np.float32)
+    b = np.array([0.1, -0.2, 0.3, 0.0], np.float32)
+    s = np.array([2.0, 0.5, 3.0, 1.0], np.float32)
+    g2, b2 = mq.fold_norm(g, b, s)
+    assert np.array_equal(g2, g / s) and np.array_equal(b2, b / s)
+    g3, b3 = mq.fold_norm(g, None, s)
+    assert b3 is None and np.array_equal(g3, g / s)
+    with pytest.raises(mq.MQError):
+        mq.fold_norm(g, b, np.array([1.0, 0.0, 1.0, 1.0], np.float32))
