@@ -188,21 +188,29 @@ class PrefillBlock:
         down = self.cases[-1]
         down.residual = synth.residual_codes(CONFIG_ID_PREFILL, layer, m, down.N)
         dev = "cuda"
-        # distinct inputs: the shared x (q/k/v/gate/up), o's input, down's input
-        self.x_host = {}
-        self.x_dev = {}
+        # distinct inputs (the shared x of q/k/v/gate/up, o's input, down's
+        # input) as views of one device buffer, mirrored by one pinned host
+        # buffer, so that a step uploads them with one copy; the outputs alike
+        xs = []
         for c in self.cases:
-            key = id(c.x)
-            if key not in self.x_dev:
-                self.x_host[key] = torch.from_numpy(c.x).pin_memory()
-                self.x_dev[key] = torch.empty(c.x.shape, dtype=torch.int8, device=dev)
-                self.x_dev[key].copy_(self.x_host[key])
+            if all(c.x is not a for a in xs):
+                xs.append(c.x)
+        self.x_all_host = torch.from_numpy(np.concatenate([a.reshape(-1) for a in xs])).pin_memory()
+        self.x_all = self.x_all_host.to(dev)
+        self.x_dev, off = {}, 0
+        for a in xs:
+            self.x_dev[id(a)] = self.x_all[off:off + a.size].view(a.shape)
+            off += a.size
+        self.y_all = torch.empty(sum(m * c.N for c in self.cases), dtype=torch.int8, device=dev)
+        self.y_all_host = torch.empty(self.y_all.numel(), dtype=torch.int8).pin_memory()
         self.descs, self.y, self.keep = [], [], []
+        yoff = 0
         for c in self.cases:
             packed, colsum = mq.pack_weights(c.w, 8)
             m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
             t = [torch.from_numpy(a).to(dev) for a in (packed, colsum, m0, sh)]
-            y = torch.empty((m, c.N), dtype=torch.int8, device=dev)
+            y = self.y_all[yoff:yoff + m * c.N].view(m, c.N)
+            yoff += m * c.N
             res = torch.from_numpy(c.residual).to(dev) if c.residual is not None else None
             zw = torch.from_numpy(c.zw).to(dev) if c.zw is not None else None
             self.keep += t + [a for a in (res, zw) if a is not None]
@@ -214,9 +222,8 @@ class PrefillBlock:
         self.ws_bytes = mq.workspace_size_batch(self.descs)
         self.ws = torch.zeros(max(16, self.ws_bytes), dtype=torch.uint8, device=dev)
         self.wsp = self.ws.data_ptr() if self.ws_bytes else None
-        self.y_host = [torch.empty(y.shape, dtype=torch.int8).pin_memory() for y in self.y]
-        self.h2d_bytes = sum(v.numel() for v in self.x_host.values())
-        self.d2h_bytes = sum(y.numel() for y in self.y)
+        self.h2d_bytes = self.x_all.numel()
+        self.d2h_bytes = self.y_all.numel()
 
 
 class DecodeLayer:
@@ -287,20 +294,41 @@ def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
         raise RuntimeError(f"device status {mq.status_string(status)} after timed region")
     max_total_ms = dist.max(total_ms)
 
-    # end to end through the public API: pinned host inputs in, outputs back out
-    e2e_steps = min(steps, 50)
+    # end to end through the public API: every step copies its inputs in from
+    # pinned host memory and its outputs back out.  The copies run on their own
+    # streams, so step i + 1's inputs upload and step i - 1's outputs download
+    # while step i computes; events order each layer's buffers between steps
+    # i and i + 3 (the layers rotate over three).
+    e2e_steps = min(steps, 300)
     torch.cuda.synchronize()
     dist.barrier()
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    nb = len(blocks)
+    in_done = [torch.cuda.Event() for _ in range(e2e_steps)]
+    comp_done = [torch.cuda.Event() for _ in range(e2e_steps)]
+    out_done = [torch.cuda.Event() for _ in range(e2e_steps)]
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    s_in.wait_event(e0)
+    s_out.wait_event(e0)
     for i in range(e2e_steps):
-        b = blocks[i % len(blocks)]
-        for key, xh in b.x_host.items():
-            b.x_dev[key].copy_(xh, non_blocking=True)
+        b = blocks[i % nb]
+        with torch.cuda.stream(s_in):
+            if i >= nb:
+                s_in.wait_event(comp_done[i - nb])  # step i - 3 no longer reads x
+            b.x_all.copy_(b.x_all_host, non_blocking=True)
+            in_done[i].record(s_in)
+        stream.wait_event(in_done[i])
+        if i >= nb:
+            stream.wait_event(out_done[i - nb])  # step i - 3's outputs are copied out
         step(i)
-        for y, yh in zip(b.y, b.y_host):
-            yh.copy_(y, non_blocking=True)
+        comp_done[i].record(stream)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(comp_done[i])
+            b.y_all_host.copy_(b.y_all, non_blocking=True)
+            out_done[i].record(s_out)
+    stream.wait_stream(s_out)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = dist.max(e0.elapsed_time(e1))
