@@ -230,8 +230,11 @@ class DecodeLayer:
     """One layer's seven W4A8 linears, uploaded once; descriptors for each
     decode width M use the first M rows of a 16-row seeded input."""
 
-    def __init__(self, mq, torch, layer: int, asym: bool = False, ms=DECODE_MS):
-        cases = synth.block_linears(CONFIG_ID_DECODE, max(ms), 4, layer=layer, asym=asym)
+    def __init__(self, mq, torch, layer: int, asym: bool = False, ms=DECODE_MS, a16: bool = False):
+        if a16:  # 16-bit activations and outputs (W4A16)
+            cases = synth.block_linears_a16(CONFIG_ID_DECODE, max(ms), 4, layer=layer)
+        else:
+            cases = synth.block_linears(CONFIG_ID_DECODE, max(ms), 4, layer=layer, asym=asym)
         self.arr, self.keep = {}, []
         dev = []
         for c in cases:
@@ -244,7 +247,7 @@ class DecodeLayer:
         for m in ms:
             descs = []
             for c, t in dev:
-                y = torch.empty((m, c.N), dtype=torch.int8, device="cuda")
+                y = torch.empty((m, c.N), dtype=torch.int16 if a16 else torch.int8, device="cuda")
                 self.keep.append(y)
                 descs.append(mq.make_desc(t[0], c.zx, t[1], t[2], c.N, t[3], t[4], c.zy, y, 4,
                                           m=m, zw=t[5]))
@@ -340,7 +343,8 @@ def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
     }
 
 
-def run_decode(mq, torch, steps_per_m: int = 240, asym: bool = False, ms=DECODE_MS):
+def run_decode(mq, torch, steps_per_m: int = 240, asym: bool = False, ms=DECODE_MS,
+               a16: bool = False):
     """Weight GB/s of the W4A8 block linears at M = 1, 4, 16 (one batched
     launch per layer, 12 layers in rotation), timed with CUDA events per launch
     (kernel) and over a captured CUDA graph of back-to-back launches (stream).
@@ -348,7 +352,7 @@ def run_decode(mq, torch, steps_per_m: int = 240, asym: bool = False, ms=DECODE_
     out = {}
     wbytes = block_weight_bytes(4)
     stream = torch.cuda.current_stream()
-    layers = [DecodeLayer(mq, torch, layer, asym, ms) for layer in range(DECODE_LAYERS)]
+    layers = [DecodeLayer(mq, torch, layer, asym, ms, a16) for layer in range(DECODE_LAYERS)]
     ws = mq.workspace()
     wsp, wsn = ws.data_ptr(), ws.numel()
 
@@ -496,11 +500,12 @@ def _time_blocks(mq, torch, blocks, steps: int):
     return e0.elapsed_time(e1) / steps
 
 
-def run_a16(mq, torch, prefill_steps: int = 600, decode_steps: int = 480, check_rows: int = 4):
+def run_a16(mq, torch, prefill_steps: int = 600, check_rows: int = 4):
     """W8A16 prefill of the block at M = 1024 (the paper's 16-bit-activation
-    baseline, Sec. 5.6) and W4A16 decode at M = 1 and 8, back-to-back batched
-    calls (split pre-pass + kernel each) rotating over layers larger than L2
-    together; the first rows of layer 0's prefill checked against the oracle."""
+    baseline, Sec. 5.6), back-to-back batched calls (split pre-pass + kernel)
+    rotating over three layers, the first rows of layer 0 checked against the
+    oracle; and W4A16 decode at M = 1 and 8, timed like the W4A8 decode
+    (one launch per layer, per launch and over a CUDA graph)."""
     import oracle
     oracle.build()
     out = {}
@@ -522,15 +527,8 @@ def run_a16(mq, torch, prefill_steps: int = 600, decode_steps: int = 480, check_
                             "parity_sample": {"rows": check_rows, "outputs": checked,
                                               "mismatches": mism}}
     del blocks
-    wbytes = block_weight_bytes(4)
-    for m in (1, 8):
-        layers = [A16Block(mq, torch, layer, m, 4, CONFIG_ID_DECODE, False)
-                  for layer in range(DECODE_LAYERS)]
-        ms = _time_blocks(mq, torch, layers, decode_steps)
-        out[f"decode_w4a16_m{m}"] = {"us_per_block": round(ms * 1e3, 2),
-                                     "gbs": round(wbytes / ms / 1e6, 1),
-                                     "launches_per_step": 2, "steps": decode_steps}
-        del layers
+    for m, v in run_decode(mq, torch, a16=True, ms=(1, 8)).items():
+        out[f"decode_w4a16_{m}"] = v
     return out
 
 
@@ -725,6 +723,9 @@ def main():
         v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
     for v in glue.values():
         v["frac_hbm"] = round(v["gbs"] / hbm, 3)
+    for k, v in a16.items():
+        if k.startswith("decode_"):
+            v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
 
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world,

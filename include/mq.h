@@ -199,11 +199,13 @@ int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, int32_t zx,
  *   acc[m][n] = sum_k (x[m][k] - zx) * w[n][k]        (exact, |acc| < 2^40)
  *   y[m][n]   = clamp(zy + floor(acc M0[n] / 2^shift[n] + 1/2), -32768, 32767)
  * Method: with hi the signed high byte and lo the unsigned low byte of a
- * code, x = 256 hi + (lo - 128) + 128.  A pre-pass writes the two int8
- * planes hi and lo - 128 as rows 2m and 2m+1 of a [2M][K] int8 matrix in the
- * workspace; the int8 kernels contract it exactly, and their epilogues form
- * 256 S_hi + S_lo + (128 - zx) colsum[n] in int64 and requantize it.  2M <= 16
- * runs the decode kernel, larger M the tensor-core kernel.
+ * code, x = 256 hi + (lo - 128) + 128; both planes hi and lo - 128 are int8
+ * values, which the int8 kernels contract exactly, and their epilogues form
+ * 256 S_hi + S_lo + (128 - zx) colsum[n] in int64 and requantize it.
+ * 2M <= 16 runs the decode kernel, which splits the codes into the planes
+ * as it builds its operands; larger M runs the tensor-core kernel after a
+ * pre-pass that writes the planes as rows 2m and 2m+1 of a [2M][K] int8
+ * matrix in the workspace.
  * Requirements: 0 <= M, N; 0 <= K <= MQ_MAX_K; K % 16 == 0; ldx % 8 == 0;
  * x and packed 16-byte aligned.  No residual and no weight zero point.  The
  * stream rules of mq_linear_w8a8 apply.
@@ -226,10 +228,10 @@ int mq_linear_w4a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
 
 /*
  * Device workspace bytes of one mq_linear_w8a16 / mq_linear_w4a16 call: the
- * decode workspace (see mq_workspace_size) when 1 <= 2M <= 16, followed by
- * the two int8 planes of x (2 M K bytes, rounded up to 128).  The decode part
- * follows the contract of mq_workspace_size; the planes are scratch,
- * overwritten by each call.
+ * decode workspace (see mq_workspace_size) when 1 <= 2M <= 16; otherwise the
+ * two int8 planes of x (2 M K bytes, rounded up to 128), which are scratch,
+ * overwritten by each call.  The decode part follows the contract of
+ * mq_workspace_size.
  * Errors: MQ_ERR_INVALID_ARG.
  */
 int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
@@ -286,7 +288,7 @@ typedef struct mq_linear_desc {
  * (rounded up to 16) for every distinct input (x, M, K, ldx) of the
  * descriptors with M > 16 and a weight zero point, which holds rowsum(x) of
  * its tokens; plus 2*M*K bytes (rounded up to 128) for every distinct input
- * of the descriptors with abits 16, which holds its two int8 planes (both
+ * of the descriptors with abits 16 and 2M > 16, which holds its two int8 planes (both
  * filled by the call; descriptors reading the same input, e.g. q/k/v/gate/up
  * of one block, share them).  0 when none applies.  The decode region (the
  * first mq_workspace_size bytes, when present) follows the contract of

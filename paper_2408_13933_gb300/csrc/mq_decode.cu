@@ -74,6 +74,7 @@ constexpr int UNIT_ROWS = 64;          // four 16-row mma tiles
 constexpr int ROW_BYTES = 128;         // weight bytes per row per stage
 constexpr int W_BYTES = UNIT_ROWS * ROW_BYTES;  // 8 KB of weights
 constexpr int X_BOX = 16 * 128;                 // one x box: 16 tokens x 128 k
+constexpr int X16_BOX = 8 * 128;                // one 16-bit x box: 8 tokens x 64 codes
 constexpr int STAGE_BYTES = W_BYTES + 2 * X_BOX;
 // Ring depth: the cross-warp reduction buffer grows with the token tiles, so
 // the ring shrinks to keep two CTAs per SM.
@@ -262,7 +263,13 @@ __device__ __forceinline__ void store_out(const DecProb &p, const SM &sm, int ro
 
 // One stage of one warp: activation fragment and weight words from the ring
 // slot, widening, mma.  Returns nothing; accumulates into acc and xs.
-template <int BITS, int NT>
+// One plane of four 16-bit codes held in two words (codes 2i, 2i+1 in word
+// i): the high bytes (plane 0) or the low bytes - 128 (plane 1).
+__device__ __forceinline__ uint32_t code_plane(uint32_t w0, uint32_t w1, bool low) {
+    return low ? (__byte_perm(w0, w1, 0x6420) ^ 0x80808080u) : __byte_perm(w0, w1, 0x7531);
+}
+
+template <int BITS, int NT, bool A16>
 __device__ __forceinline__ void compute_stage(const uint8_t *ring, int warp, int g, int t,
                                               float (&acc)[4][NT][4], int (&xs)[NT]) {
     using C = Cfg<BITS>;
@@ -270,7 +277,29 @@ __device__ __forceinline__ void compute_stage(const uint8_t *ring, int warp, int
     // stage offset warp * KWARP + t * KWARP/4 of token row m (zero outside M
     // and K: TMA fill)
     uint32_t xa[NT], xb[NT];
-    {
+    if constexpr (A16) {
+        // 16-bit codes: plane row m is token m >> 1, plane m & 1 (high bytes,
+        // low bytes - 128).  Box h of the stage holds 64 codes of the 8
+        // tokens (128-byte rows, 128-byte swizzle); this lane's KWARP/4 codes
+        // start at stage offset `off`.
+        const int off = warp * C::KWARP + t * (C::KWARP / 4);
+        const uint8_t *xbox = ring + W_BYTES + (off >> 6) * X16_BOX;
+        const int c = (off & 63) >> 3, inner = (off & 7) * 2;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            const int m = nt * 8 + g, tok = m >> 1;
+            const uint8_t *src = xbox + tok * 128 + ((c ^ (tok & 7)) << 4) + inner;
+            if (BITS == 4) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(src);
+                xa[nt] = code_plane(v.x, v.y, m & 1);
+                xb[nt] = code_plane(v.z, v.w, m & 1);
+            } else {
+                const uint2 v = *reinterpret_cast<const uint2 *>(src);
+                xa[nt] = code_plane(v.x, v.y, m & 1);
+                xb[nt] = 0u;
+            }
+        }
+    } else {
         const int off = warp * C::KWARP + t * (C::KWARP / 4);
         const uint8_t *xbox = ring + W_BYTES + (off >> 7) * X_BOX;
         const int c = (off & 127) >> 4, inner = off & 15;
@@ -510,10 +539,19 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     tma_load_2d(s.ring[slot], &P.tmap_w[pi], j * ROW_BYTES, rb * UNIT_ROWS,
                                 &s.full[slot]);
                 }
+                if constexpr (A16) {
+                    // 16-bit codes: KSTAGE / 64 boxes of 8 tokens x 64 codes
+                    // (the same bytes as the 8-bit boxes)
 #pragma unroll
-                for (int h = 0; h < XBOXES; ++h)
-                    tma_load_2d(s.ring[slot] + W_BYTES + h * X_BOX, &P.tmap_x[pi],
-                                j * C::KSTAGE + h * 128, 0, &s.full[slot]);
+                    for (int h = 0; h < C::KSTAGE / 64; ++h)
+                        tma_load_2d(s.ring[slot] + W_BYTES + h * X16_BOX, &P.tmap_x[pi],
+                                    j * C::KSTAGE + h * 64, 0, &s.full[slot]);
+                } else {
+#pragma unroll
+                    for (int h = 0; h < XBOXES; ++h)
+                        tma_load_2d(s.ring[slot] + W_BYTES + h * X_BOX, &P.tmap_x[pi],
+                                    j * C::KSTAGE + h * 128, 0, &s.full[slot]);
+                }
             }
         }
         __syncwarp();
@@ -571,7 +609,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     ok = false;
                     break;
                 }
-                if (p.K > 0) compute_stage<BITS, NT>(s.ring[slot], warp, g, t, acc, xs);
+                if (p.K > 0) compute_stage<BITS, NT, A16>(s.ring[slot], warp, g, t, acc, xs);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&s.empty[slot]);
                 if constexpr (C::FLUSH) {
@@ -743,6 +781,20 @@ bool encode_sw128(CUtensorMap *map, const void *base, uint64_t cols, uint64_t ro
            CUDA_SUCCESS;
 }
 
+// int16 tensor [rows][cols] with row pitch `pitch` bytes, box 64 x 8, 128-byte swizzle.
+bool encode_x16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows, uint64_t pitch) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {pitch};
+    const cuuint32_t box[2] = {64, 8};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<void *>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
 // Launch epochs: nonzero and different for consecutive launches (wraps after
 // 2^32 - 1 launches; entries are zeroed after use, so an old epoch never
 // lingers in the workspace).
@@ -781,10 +833,13 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
             q.tiles_m = nst;
             stages += (long long)((q.N + UNIT_ROWS - 1) / UNIT_ROWS) * nst;
             const uint64_t wcols = (uint64_t)q.K * BITS / 8;
+            // 16-bit codes: q.M counts plane rows, the tensor has q.M / 2 tokens
             if (q.K > 0 &&
                 (!encode_sw128(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, wcols, UNIT_ROWS) ||
-                 !encode_sw128(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M, (uint64_t)q.ldx,
-                               16)))
+                 !(A16 ? encode_x16(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)(q.M / 2),
+                                    2 * (uint64_t)q.ldx)
+                       : encode_sw128(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M,
+                                      (uint64_t)q.ldx, 16))))
                 return MQ_ERR_CUDA;
         }
         if (stages == 0) continue;

@@ -114,7 +114,9 @@ Plan batch_plan(const mq_linear_desc *descs, int count) {
     }
     for (int i = 0; i < count; ++i) {
         const mq_linear_desc &d = descs[i];
-        if (d.M <= 0 || d.N <= 0 || d.K <= 0 || abits_of(d) != 16) continue;
+        // the decode kernel reads 16-bit codes itself; only tensor-core shapes
+        // take the plane matrix
+        if (d.M <= 0 || d.N <= 0 || d.K <= 0 || abits_of(d) != 16 || is_decode(d)) continue;
         if (find_job(pl.split, d.x, d.M, d.K, d.ldx) >= 0) continue;
         off = align128(off);
         mq::SplitJob j{};
@@ -160,7 +162,14 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
             const int j = find_job(pl.rowsum, d.x, d.M, d.K, d.ldx);
             p.rowsum = pl.rowsum[j].out;
         }
-        if (p.K > 0 && p.a16) p.x = pl.split[find_job(pl.split, d.x, d.M, d.K, d.ldx)].out;
+        if (p.K > 0 && p.a16) {
+            if (is_decode(d)) {  // int16 codes, read by the decode kernel's TMA as they are
+                p.x = static_cast<const int8_t *>(d.x);
+                p.ldx = d.ldx;
+            } else {
+                p.x = pl.split[find_job(pl.split, d.x, d.M, d.K, d.ldx)].out;
+            }
+        }
         if (is_decode(d))
             dec[p.bits == 8][p.a16].push_back(p);
         else

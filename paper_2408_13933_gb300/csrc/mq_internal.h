@@ -26,10 +26,12 @@ struct Problem {
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;
     int32_t bits;
-    // 16-bit activations: x is the [2M'][K] int8 plane matrix of the M' int16
-    // tokens (rows 2m = high bytes, 2m + 1 = low bytes - 128, ldx = K), M is
-    // its row count 2M', y points to int16 [M'][ldy], and the epilogues form
-    // 256 S(2m) + S(2m + 1) + (128 - zx) colsum.
+    // 16-bit activations: M is the row count 2M' of the plane matrix of the M'
+    // int16 tokens (rows 2m = high bytes, 2m + 1 = low bytes - 128), y points
+    // to int16 [M'][ldy], and the epilogues form 256 S(2m) + S(2m + 1) +
+    // (128 - zx) colsum.  For the prefill kernel x is that plane matrix
+    // (ldx = K); the decode kernel reads the int16 codes [M'][ldx] and forms
+    // the planes itself.
     int32_t a16;
     int32_t tile_begin;  // first global tile / block index of this problem
     int32_t tiles_m;     // prefill: number of 128-row tiles

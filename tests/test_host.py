@@ -258,8 +258,8 @@ def test_a16_validation_and_workspace(mq):
     dec = mq.workspace_size(1, 1, 0, 4)
     assert mq.workspace_size_a16(100, 32, 64, 8) == 12800
     assert mq.workspace_size_a16(9, 32, 64, 8) == 1152            # 2M = 18: tensor cores
-    assert mq.workspace_size_a16(8, 32, 64, 4) == dec + 1024      # 2M = 16: decode
-    assert mq.workspace_size_a16(1, 32, 48, 8) == dec + 128
+    assert mq.workspace_size_a16(8, 32, 64, 4) == dec             # 2M = 16: decode, no planes
+    assert mq.workspace_size_a16(1, 32, 48, 8) == dec
     assert mq.workspace_size_a16(0, 32, 64, 8) == 0
     assert mq.workspace_size_a16(5, 32, 0, 8) == dec              # K = 0: no planes
     # batch: shared int16 input planned once; after a rowsum region the
