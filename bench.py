@@ -98,14 +98,24 @@ def dist_env():
 
 
 class Dist:
-    def __init__(self, world: int, rank: int, local: int):
+    """One process per GPU, replicas only: a barrier and the maximum over
+    ranks (for the slowest rank's time); no collective touches the data path.
+    The backend is NCCL on GPUs, gloo otherwise (host-side tests)."""
+
+    def __init__(self, world: int, rank: int, local: int, backend: str | None = None):
         self.world, self.rank, self.local = world, rank, local
         self.pg = None
+        self.device = "cpu"
         if world > 1:
             import torch
             import torch.distributed as dist
-            torch.cuda.set_device(local)
-            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+            backend = backend or ("nccl" if torch.cuda.is_available() else "gloo")
+            if backend == "nccl":
+                torch.cuda.set_device(local)
+                dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+                self.device = "cuda"
+            else:
+                dist.init_process_group("gloo", rank=rank, world_size=world)
             self.pg = dist
 
     def barrier(self):
@@ -116,13 +126,19 @@ class Dist:
         if self.pg is None:
             return v
         import torch
-        t = torch.tensor([v], dtype=torch.float64, device="cuda")
+        t = torch.tensor([v], dtype=torch.float64, device=self.device)
         self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
         return float(t.item())
 
     def close(self):
         if self.pg is not None:
             self.pg.destroy_process_group()
+
+
+def whole_job_rate(units_per_rank: float, world: int, max_ms: float) -> float:
+    """Units per second of the whole job: every rank's units over the
+    slowest rank's time (weak scaling: each rank runs the full workload)."""
+    return units_per_rank * world / (max_ms * 1e-3)
 
 
 # --------------------------------------------------------------------------- clocks
@@ -715,9 +731,9 @@ def main():
 
     ops = block_ops(PREFILL_M)
     ms_per_step = pre["total_ms"] / args.steps
-    value = ops * args.steps * world / (pre["total_ms"] * 1e-3) / 1e12
+    value = whole_job_rate(ops * args.steps, world, pre["total_ms"]) / 1e12
     kern_tflops = ops / (pre["kernel_ms_mean"] * 1e-3) / 1e12
-    e2e_value = ops * pre["e2e_steps"] * world / (pre["e2e_ms"] * 1e-3) / 1e12
+    e2e_value = whole_job_rate(ops * pre["e2e_steps"], world, pre["e2e_ms"]) / 1e12
     hbm = peaks["hbm_gbs"]
     for v in list(decode.values()) + list(asym_dec.values()):
         v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
