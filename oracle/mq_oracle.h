@@ -14,7 +14,8 @@
  *       X_int = min(max(round(X/alpha) - beta, 0), q_max).
  *     Applied to the layer output with a static (alpha, beta) it is the
  *     requantization below; shifted by -128 to signed int8 its offset is the
- *     output zero point zy (reading R1 of the design notes).
+ *     output zero point zy (the integer zero point round(-f_min / alpha)
+ *     of the unsigned range, minus 128).
  *   - Sec. 5.1 and Appendix A: symmetric per-output-channel weights (int8, or
  *     int4 in [-8, 7]), so the weight zero point is 0.
  *
@@ -49,7 +50,8 @@ extern "C" {
  * accumulator is under 1/2 in magnitude) are returned as M0 = 0, shift = 1.
  * Multipliers >= 2^30 are rejected (shift would be < 1).
  * Follows the fixed-point statement of Sec. 3.1 / Sec. 1 (all operations in
- * fixed point) with the rounding reading R4 of the design notes.
+ * fixed point); the paper names no rounding mode, and one rounding, half
+ * up, is taken.
  * Pinned by: power-of-two closed forms, relative-error bound 2^-31.
  */
 int oracle_requant_params(float sx, const float *sw, int N, float sy,
@@ -126,7 +128,7 @@ int oracle_linear_points_asym(const int8_t *x, int M, int K, int ldx, int32_t zx
  * activations of its 16-bit baselines, and those around non-linear operators,
  * in 16-bit integers (Sec. 4.1 challenge i; Sec. 5.6 on-device settings
  * W8A16 and W4A16, Table 5).  The 16-bit unsigned code range is shifted by
- * -32768 to signed int16, as for 8 bits (reading R1): x is int16 [M][ldx]
+ * -32768 to signed int16, as the 8-bit codes are by -128: x is int16 [M][ldx]
  * with zx in [-32768, 32767], the output y is int16 [M][ldy] with zy in
  * [-32768, 32767]; weights as in oracle_linear (symmetric per channel).
  *   acc[m][n] = sum_k (x[m][k] - zx) * w[n][k]      (int64; |acc| < 2^40)
@@ -162,8 +164,8 @@ int32_t oracle_requant_one_a16(int64_t acc, int32_t M0, int32_t shift, int32_t z
  * codes, stored as int8_t / int16_t arrays.
  *
  * oracle_quantize_f32: the forward quantizer of eqs. 2-4, shifted to the
- * signed range (readings R1, R2): q = clamp(rint(x / alpha) + z, qmin, qmax).
- * The integer decision is taken in f32 (reading R12): x / alpha is the
+ * signed range: q = clamp(rint(x / alpha) + z, qmin, qmax).  The paper fixes
+ * no precision or tie rule; the integer decision is taken in f32: x / alpha is the
  * correctly rounded f32 quotient and rint rounds ties to even; a NaN input
  * gives z.  alpha must be finite and > 0, z inside the code range.
  * Pinned by: exact rationals (f32 rounding of the true quotient, then ties to
@@ -208,7 +210,7 @@ int oracle_fold_weights(const float *w, int N, int K, const float *s_in, const f
 
 /*
  * Step 2: weight quantization of f32 weights [N][K], the integer decisions
- * taken in f32 (reading R12), per output channel or per tensor:
+ * taken in f32 (the paper fixes no precision), per output channel or per tensor:
  *   scheme 0, symmetric per channel: amax = max|w[n]| (1e-8 if 0),
  *     sw = amax / qmax, q = clamp(rint(w / sw), -qmax, qmax) for int8
  *     (qmax 127) and clamp(., -8, 7) with qmax 7 for int4; zw = 0.
@@ -240,7 +242,7 @@ int32_t oracle_requant_one(int64_t acc, int32_t M0, int32_t shift, int32_t zy);
 
 /*
  * Saturating int8 residual add, out[i] = clamp(a[i] + b[i], -128, 127): the
- * glue between chained layers of the 22-layer stack (reading R8).
+ * glue between chained layers of the 22-layer stack.
  */
 void oracle_residual_add(const int8_t *a, const int8_t *b, int64_t n,
                          int8_t *out);

@@ -8,7 +8,8 @@ calibration set would (Sec. 3.1, "static quantization statistics ... computed
 on a holdout calibration set").  It never computes an integer accumulator,
 a zero-point correction or a fixed-point requantization.
 
-Value recipe (reading R5/R6/R9 of the design notes):
+Value recipe (the paper trains on data this code does not have; these are
+synthetic stand-ins with the same structure):
   * activations: N(0, 1) floats, 4 seeded input channels scaled x20 (outliers),
     quantized per tensor, asymmetric: sx = (max - min) / 255,
     zx = clamp(rint(-128 - min / sx), -128, 127), x = clamp(rint(x / sx) + zx).
@@ -263,7 +264,8 @@ def block_linears(config: int, m: int, bits: int, shapes=TINYLLAMA_LINEARS, laye
 
 
 def residual_codes(config: int, layer: int, m: int, n: int, scale: float = 8.0) -> np.ndarray:
-    """Seeded fixed int8 residual for the chained stack (reading R8)."""
+    """Seeded fixed int8 residual r of the chained stack, whose layers end with
+    x_{l+1} = sat8(y_down + r)."""
     r = rng_for(config, layer, 0, ROLE_RES).standard_normal((m, n), dtype=np.float32) * scale
     return rint_clip(r, -128, 127).astype(np.int8)
 
@@ -378,7 +380,7 @@ class ChainLayer:
 
 def chain_stack(config: int, m: int, layers: int, shapes=TINYLLAMA_LINEARS, head=TINYLLAMA_HEAD,
                 calib_rows: int = 32, t_rows_frac: float = 0.0):
-    """Seeded 22-layer-style W8A8 stack (reading R8 of the design notes).
+    """Seeded 22-layer-style W8A8 stack.
 
     Layer l: q/k/v/gate/up read x_l; o reads q's int8 output (stand-in for the
     attention output); down reads up's int8 output (stand-in for SiLU(gate) *
