@@ -61,6 +61,7 @@ def _bind(lib):
     lib.oracle_dequantize.argtypes = [p, ci, i64, f32, i32, p]
     lib.oracle_requantize.argtypes = [p, ci, i64, i32, i32, i32, i32, p, ci]
     lib.oracle_fold_weights.argtypes = [p, ci, ci, p, p, p]
+    lib.oracle_linear_o16.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, p, i32, p, ci]
     lib.oracle_quantize_weights.argtypes = [p, ci, ci, ci, ci, p, p, p]
     lib.oracle_fold_norm.argtypes = [p, p, p, ci, p, p]
     lib.oracle_residual_add.argtypes = [p, p, i64, p]
@@ -207,6 +208,21 @@ class Oracle:
     def requant_one_a16(self, acc: int, m0: int, shift: int, zy: int) -> int:
         return int(self.lib.oracle_requant_one_a16(int(acc), int(m0), int(shift), int(zy)))
 
+    def linear_o16(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
+                   m0: np.ndarray, shift: np.ndarray, zy: int, zw: np.ndarray | None = None):
+        """oracle_linear_o16: int8 x, 16-bit output y int16 [M, N]."""
+        x = np.ascontiguousarray(x, dtype=np.int8)
+        m, k = x.shape
+        packed = np.ascontiguousarray(packed, dtype=np.uint8)
+        m0 = np.ascontiguousarray(m0, dtype=np.int32)
+        shift = np.ascontiguousarray(shift, dtype=np.int32)
+        zwa = np.ascontiguousarray(zw, dtype=np.int32) if zw is not None else None
+        y = np.zeros((m, n), np.int16)
+        _check(self.lib.oracle_linear_o16(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
+                                          _ptr(zwa) if zwa is not None else None, _ptr(m0),
+                                          _ptr(shift), int(zy), _ptr(y), n), "oracle_linear_o16")
+        return y
+
     def fold_weights(self, w: np.ndarray, s_in, s_out) -> np.ndarray:
         """oracle_fold_weights: f32 [N, K] -> folded f32 [N, K]."""
         w = np.ascontiguousarray(w, dtype=np.float32)
@@ -323,6 +339,10 @@ def requant_one_a16(acc, m0, shift, zy):
 
 def fold_weights(w, s_in, s_out):
     return _default().fold_weights(w, s_in, s_out)
+
+
+def linear_o16(x, zx, packed, bits, n, m0, shift, zy, zw=None):
+    return _default().linear_o16(x, zx, packed, bits, n, m0, shift, zy, zw)
 
 
 def quantize_weights(w, bits, scheme):

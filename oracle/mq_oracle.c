@@ -316,6 +316,26 @@ int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx
     return ORACLE_OK;
 }
 
+int oracle_linear_o16(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                      const uint8_t *packed, int bits, int N, const int32_t *zw,
+                      const int32_t *M0, const int32_t *shift, int32_t zy, int16_t *y,
+                      int ldy) {
+    if (M < 0 || K < 0 || N < 0 || (bits != 8 && bits != 4) || ldx < K || ldy < N)
+        return ORACLE_EINVAL;
+    if (bits == 4 && K % 2 != 0) return ORACLE_EINVAL;
+    if (zx < -128 || zx > 127 || zy < -32768 || zy > 32767) return ORACLE_EINVAL;
+    int rc = oracle_check_zw(zw, N, bits);
+    if (rc != ORACLE_OK) return rc;
+    for (int m = 0; m < M; ++m) {
+        for (int n = 0; n < N; ++n) {
+            int64_t wide = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, zw ? zw[n] : 0);
+            y[(size_t)m * (size_t)ldy + (size_t)n] =
+                (int16_t)oracle_requant_one_a16(wide, M0[n], shift[n], zy);
+        }
+    }
+    return ORACLE_OK;
+}
+
 static int oracle_code_range(int bits, int32_t *lo, int32_t *hi) {
     if (bits == 8) {
         *lo = -128;

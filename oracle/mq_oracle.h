@@ -146,6 +146,25 @@ int oracle_linear_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
                       const int32_t *shift, int32_t zy, int16_t *y, int ldy,
                       int64_t *acc_out);
 
+/*
+ * 8-bit inputs, 16-bit output: the product of two 8-bit activations (or
+ * activations and weights) whose result feeds a non-linear operator, which
+ * MobileQuant keeps in 16-bit integers (Sec. 4.1), e.g. the attention scores
+ * Q K^T ahead of the softmax.  With int8 x [M][ldx], int8 / int4 w [N][K]
+ * (packed as in oracle_linear) and an optional per-channel zero point zw
+ * (NULL: 0):
+ *   acc[m][n] = sum_k (x[m][k] - zx) * (w[n][k] - zw[n])      (int64)
+ *   y[m][n]   = clamp(zy + floor(acc M0[n] / 2^s + 1/2), -32768, 32767)
+ * zx in [-128, 127], zy in [-32768, 32767]; y is int16 [M][ldy].
+ * Pinned by: its accumulator equals oracle_linear_asym's, its outputs are
+ * oracle_requant_one_a16 of it, exhaustive K=1 with outputs checked against
+ * exact rationals, saturation at the int16 ends.
+ */
+int oracle_linear_o16(const int8_t *x, int M, int K, int ldx, int32_t zx,
+                      const uint8_t *packed, int bits, int N, const int32_t *zw,
+                      const int32_t *M0, const int32_t *shift, int32_t zy, int16_t *y,
+                      int ldy);
+
 /* oracle_linear_a16 at listed output coordinates (as oracle_linear_points). */
 int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
                              const uint8_t *packed, int bits, int N,

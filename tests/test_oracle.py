@@ -692,6 +692,45 @@ def pin_quantize_weights_properties(orc: Oracle):
                 assert np.all((c.min(axis=1) == qmin) | (c.max(axis=1) == qmax))
 
 
+# ---- 8-bit inputs, 16-bit outputs (scores ahead of a 16-bit non-linearity) ----
+
+def pin_o16_k1_exhaustive(orc: Oracle):
+    # every int8 x against every int8 w (K = 1), several zero points, outputs
+    # against round half up of exact rationals saturated to int16
+    xs = np.arange(-128, 128, dtype=np.int16).astype(np.int8).reshape(-1, 1)
+    ws = np.arange(-128, 128, dtype=np.int16).astype(np.int8).reshape(-1, 1)
+    packed, _ = orc.pack(ws, 8)
+    n = ws.shape[0]
+    for zx, zwv, m0, s in ((-128, 127, 1 << 30, 31), (5, -3, (1 << 31) - 1, 24), (0, 0, 1 << 30, 30)):
+        y = orc.linear_o16(xs, zx, packed, 8, n, np.full(n, m0, np.int32),
+                           np.full(n, s, np.int32), 7, zw=np.full(n, zwv, np.int32))
+        for i in range(0, 256, 5):
+            for j in range(0, 256, 3):
+                acc = (int(xs[i, 0]) - zx) * (int(ws[j, 0]) - zwv)
+                assert int(y[i, j]) == _py_requant16(acc, m0, s, 7), (zx, zwv, i, j)
+
+
+def pin_o16_matches_asym_and_requant16(orc: Oracle):
+    # the accumulator is oracle_linear_asym's and each output is
+    # oracle_requant_one_a16 of it (both separately pinned)
+    rng = np.random.default_rng(301)
+    for bits in (8, 4):
+        lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+        c = synth.random_case(71 + bits, 7, 96, 13, bits)
+        zw = rng.integers(lo, hi + 1, size=c.N).astype(np.int32)
+        packed, _ = orc.pack(c.w, bits)
+        m0 = rng.integers(1 << 30, 1 << 31, size=c.N).astype(np.int32)
+        sh = rng.integers(14, 40, size=c.N).astype(np.int32)
+        _, acc = orc.linear(c.x, c.zx, packed, bits, c.N, m0, sh, 0, want_acc=True, zw=zw)
+        zy = -1234
+        y = orc.linear_o16(c.x, c.zx, packed, bits, c.N, m0, sh, zy, zw=zw)
+        for m in range(c.M):
+            for n in range(c.N):
+                assert int(y[m, n]) == orc.requant_one_a16(int(acc[m, n]), int(m0[n]), int(sh[n]),
+                                                           zy)
+        assert (np.abs(y.astype(np.int64)) > 127).any()   # the 16-bit range is used
+
+
 PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zero_point_identity,
                pin_exact_dequant, pin_requant_closed_form, pin_requant_ties, pin_requant_vs_eq4,
                pin_requant_params_bound, pin_asym_k1_exhaustive, pin_asym_int4_pairs,
@@ -701,7 +740,8 @@ PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zer
                pin_a16_requant_closed_form_and_saturation, pin_a16_requant_vs_eq4,
                pin_quantize_exact, pin_quantize_ties_and_invariants, pin_dequantize_exact,
                pin_requantize_exhaustive, pin_requantize_vs_eq4, pin_fold_exact,
-               pin_quantize_weights_exact, pin_fold_equivalence, pin_quantize_weights_properties]
+               pin_quantize_weights_exact, pin_fold_equivalence, pin_quantize_weights_properties,
+               pin_o16_k1_exhaustive, pin_o16_matches_asym_and_requant16]
 
 
 # ----------------------------------------------------------------------------
@@ -965,6 +1005,14 @@ def test_quantize_weights_properties(O):
     pin_quantize_weights_properties(O)
 
 
+def test_o16_k1_exhaustive(O):
+    pin_o16_k1_exhaustive(O)
+
+
+def test_o16_matches_asym_and_requant16(O):
+    pin_o16_matches_asym_and_requant16(O)
+
+
 MUTATIONS = [
     ("zero point sign", "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - zx;",
      "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] + zx;"),
@@ -1021,6 +1069,12 @@ MUTATIONS = [
     ("per-tensor statistics per row", "        if (scheme == 2) {\n            lo = tlo;",
      "        if (scheme == 3) {\n            lo = tlo;"),
     ("asymmetric span from the row maximum only", "float span = hi - lo;", "float span = hi;"),
+    ("o16 output narrowed to int8",
+     "(int16_t)oracle_requant_one_a16(wide, M0[n], shift[n], zy);",
+     "(int16_t)oracle_requant_one(wide, M0[n], shift[n], zy);"),
+    ("o16 weight zero point ignored",
+     "int64_t wide = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, zw ? zw[n] : 0);",
+     "int64_t wide = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, 0);"),
     ("a16 output zero point dropped",
      "__int128 out = (__int128)zy + oracle_round_shift(acc, M0, shift);",
      "__int128 out = oracle_round_shift(acc, M0, shift);"),
