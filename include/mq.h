@@ -262,6 +262,17 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
  * Errors: as the single calls, and MQ_ERR_K_OVERFLOW for int8 weights with
  * zw and K > MQ_MAX_K_ASYM8; the index of the first bad descriptor is not
  * reported, nothing is launched when any descriptor is invalid.
+ *
+ * 16-bit output from 8-bit inputs (abits 8, obits 16): y is int16 [M][ldy]
+ * and zy lies in [-32768, 32767]; everything else is as for 8-bit outputs,
+ * without a residual.  For products whose result feeds a non-linear operator,
+ * which MobileQuant keeps in 16-bit integers (Sec. 4.1): the attention scores
+ * Q K^T ahead of the softmax, with the keys as the "weights" (their zero point
+ * as zw, their row sums from mq_row_sums as colsum).
+ * Weight row pitch: `ldw` bytes between weight rows (0: K * bits / 8; else at
+ * least that and a multiple of 16), so that a head's slice of a projection
+ * output ([T][heads * d], one head's d columns) can serve as the weights
+ * without a copy.
  */
 typedef struct mq_linear_desc {
     const void *x;          /* int8 [M][ldx], or int16 with abits == 16 */
@@ -276,6 +287,8 @@ typedef struct mq_linear_desc {
     int32_t zx, zy;
     int32_t bits;  /* weight bits: 8 or 4 */
     int32_t abits; /* activation and output bits: 8 (0 reads as 8) or 16, see mq_linear_w8a16 */
+    int32_t obits; /* output bits: 0 (= abits), or 16 with abits 8: int16 y, see below */
+    int32_t ldw;   /* bytes between weight rows; 0: packed rows (K * bits / 8) */
 } mq_linear_desc;
 
 /* Largest K for int8 weights with a weight zero point: 255 * 255 * K < 2^31. */
@@ -396,6 +409,28 @@ int mq_fold_quantize_pack(const float *w, int N, int K, const float *s_in, const
  */
 int mq_fold_norm(const float *gamma, const float *beta, const float *s, int K, float *gamma_out,
                  float *beta_out);
+
+/* ---- Attention matmul glue ------------------------------------------------ */
+
+/*
+ * out[m] = sum_k x[m][k] (int32) for int8 x [M][ldx]: the colsum of an
+ * activation matrix used as the "weights" operand (the keys of Q K^T, V^T of
+ * P V), or any row sum.  Requirements: M, K >= 0; K % 16 == 0; ldx >= K,
+ * ldx % 16 == 0; x 16-byte aligned; K <= MQ_MAX_K.  Asynchronous on
+ * `stream` (programmatic dependent launch: x is read after the previous
+ * kernel completes).
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_ALIGNMENT, MQ_ERR_CUDA.
+ */
+int mq_row_sums(const int8_t *x, int M, int K, int ldx, int32_t *out, void *stream);
+
+/*
+ * dst[c][r] = src[r][c] for int8 src [rows][lds] -> dst [cols][ldd] (lds >=
+ * cols, ldd >= rows): V [T][d] -> V^T [d][T], the K-major "weights" operand of
+ * P V.  Asynchronous on `stream`.
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_CUDA.
+ */
+int mq_transpose_i8(const int8_t *src, int rows, int cols, int lds, int8_t *dst, int ldd,
+                    void *stream);
 
 /*
  * Wait for `stream` and report device-side failures recorded by this

@@ -249,26 +249,31 @@ __device__ __forceinline__ bool poll_entry(const int2 *p, uint32_t epoch, int32_
 
 // Requantize one output of tile row `row` (global row n, token tok) from
 // sum(w x): acc = sum(w x) - zx colsum[n], fixed point, saturate, optional
-// residual.
-template <class SM>
+// residual; with O16 to a 16-bit output (no residual).
+template <bool O16, class SM>
 __device__ __forceinline__ void store_out(const DecProb &p, const SM &sm, int row, int n,
                                           int tok, int32_t sum_wx) {
     // two's-complement wrap is exact: the true value fits in int32
     const int32_t a = (int32_t)((uint32_t)sum_wx - (uint32_t)sm.row_corr[row]);
+    if constexpr (O16) {
+        reinterpret_cast<int16_t *>(p.y)[(size_t)tok * (size_t)p.ldy + n] =
+            (int16_t)mq_requant16((int64_t)a, sm.row_m0[row], sm.row_shift[row], p.zy);
+        return;
+    }
     int32_t y = mq_requant(a, sm.row_m0[row], sm.row_shift[row], p.zy);
     if (p.residual)
         y = min(127, max(-128, y + (int32_t)p.residual[(size_t)tok * (size_t)p.ldy + n]));
     p.y[(size_t)tok * (size_t)p.ldy + n] = (int8_t)y;
 }
 
-// One stage of one warp: activation fragment and weight words from the ring
-// slot, widening, mma.  Returns nothing; accumulates into acc and xs.
 // One plane of four 16-bit codes held in two words (codes 2i, 2i+1 in word
 // i): the high bytes (plane 0) or the low bytes - 128 (plane 1).
 __device__ __forceinline__ uint32_t code_plane(uint32_t w0, uint32_t w1, bool low) {
     return low ? (__byte_perm(w0, w1, 0x6420) ^ 0x80808080u) : __byte_perm(w0, w1, 0x7531);
 }
 
+// One stage of one warp: activation fragment and weight words from the ring
+// slot, widening, mma.  Returns nothing; accumulates into acc and xs.
 template <int BITS, int NT, bool A16>
 __device__ __forceinline__ void compute_stage(const uint8_t *ring, int warp, int g, int t,
                                               float (&acc)[4][NT][4], int (&xs)[NT]) {
@@ -470,7 +475,8 @@ __device__ __forceinline__ void a16_epilogue(const Params &P, SM &s, const DecPr
 // A16: every problem has 16-bit activations (Problem::a16): x is the plane
 // matrix (rows 2m, 2m + 1 = high and low planes of token m) and the outputs
 // are int16, formed from row pairs after an exchange through shared memory.
-template <int BITS, int NT, bool A16>
+// O16: every problem has 8-bit inputs and a 16-bit output (Problem::o16).
+template <int BITS, int NT, bool A16, bool O16>
 __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constant__ Params P) {
     using C = Cfg<BITS>;
     using SM = Smem<NT>;
@@ -687,7 +693,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
 #pragma unroll
                     for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
                     // sum((x - zx)(w - zw)) = sum(u x) - (bias + zw) sum(x) - corr
-                    store_out(p, s, row, n, tok,
+                    store_out<O16>(p, s, row, n, tok,
                               (int32_t)((uint32_t)sum -
                                         (uint32_t)((C::BIAS + s.row_zw[row]) * xsum)));
                 }
@@ -739,7 +745,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
 #pragma unroll
                             for (int q = 0; q < 2 * NT; ++q) {
                                 const int n = rb * UNIT_ROWS + rows[q];
-                                if (n < p.N) store_out(p, s, rows[q], n, tok, (int32_t)v[q]);
+                                if (n < p.N) store_out<O16>(p, s, rows[q], n, tok, (int32_t)v[q]);
                             }
                         }
                     }
@@ -805,10 +811,10 @@ uint32_t next_epoch() {
     return e;
 }
 
-template <int BITS, int NT, bool A16>
+template <int BITS, int NT, bool A16, bool O16>
 int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t stream) {
     using C = Cfg<BITS>;
-    auto kern = decode_kernel<BITS, NT, A16>;
+    auto kern = decode_kernel<BITS, NT, A16, O16>;
     static int attr_done = -1;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
@@ -835,7 +841,7 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
             const uint64_t wcols = (uint64_t)q.K * BITS / 8;
             // 16-bit codes: q.M counts plane rows, the tensor has q.M / 2 tokens
             if (q.K > 0 &&
-                (!encode_sw128(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, wcols, UNIT_ROWS) ||
+                (!encode_sw128(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, (uint64_t)q.ldw, UNIT_ROWS) ||
                  !(A16 ? encode_x16(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)(q.M / 2),
                                     2 * (uint64_t)q.ldx)
                        : encode_sw128(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M,
@@ -871,7 +877,7 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
 
 }  // namespace decode
 
-// All problems passed here have the same bits and a16 and M <= DECODE_MAX_M;
+// All problems passed here have the same bits, a16 and o16 and M <= DECODE_MAX_M;
 // `workspace` holds DECODE_WS_BYTES, zero-filled.
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream) {
     using namespace decode;
@@ -881,18 +887,19 @@ int launch_decode(const Problem *probs, int count, void *workspace, void *stream
     const bool nt2 = max_m > 8;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     int32_t *ws = static_cast<int32_t *>(workspace);
-    if (probs[0].a16) {
-        if (probs[0].bits == 4)
-            return nt2 ? launch_t<4, 2, true>(probs, count, ws, s)
-                       : launch_t<4, 1, true>(probs, count, ws, s);
-        return nt2 ? launch_t<8, 2, true>(probs, count, ws, s)
-                   : launch_t<8, 1, true>(probs, count, ws, s);
+    const bool a16 = probs[0].a16, o16 = probs[0].o16, i4 = probs[0].bits == 4;
+#define MQ_DECODE_CASE(A, O)                                                              \
+    if (a16 == A && o16 == O) {                                                           \
+        if (i4) return nt2 ? launch_t<4, 2, A, O>(probs, count, ws, s)                    \
+                           : launch_t<4, 1, A, O>(probs, count, ws, s);                   \
+        return nt2 ? launch_t<8, 2, A, O>(probs, count, ws, s)                            \
+                   : launch_t<8, 1, A, O>(probs, count, ws, s);                           \
     }
-    if (probs[0].bits == 4)
-        return nt2 ? launch_t<4, 2, false>(probs, count, ws, s)
-                   : launch_t<4, 1, false>(probs, count, ws, s);
-    return nt2 ? launch_t<8, 2, false>(probs, count, ws, s)
-               : launch_t<8, 1, false>(probs, count, ws, s);
+    MQ_DECODE_CASE(true, false)
+    MQ_DECODE_CASE(false, true)
+    MQ_DECODE_CASE(false, false)
+#undef MQ_DECODE_CASE
+    return MQ_ERR_INVALID_ARG;
 }
 
 }  // namespace mq

@@ -202,7 +202,52 @@ int launch_t(const Args &a, bool vector, cudaStream_t stream) {
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+
+// dst[c][r] = src[r][c] through a 32 x 32 byte tile in shared memory (rows
+// padded to 33 bytes): coalesced reads along src rows, coalesced writes along
+// dst rows.  Launched with programmatic dependent launch (src is read after
+// griddep_wait).
+__global__ void __launch_bounds__(256) transpose_i8_kernel(const int8_t *__restrict__ src, int rows,
+                                                           int cols, int lds,
+                                                           int8_t *__restrict__ dst, int ldd) {
+    __shared__ int8_t tile[32][33];
+    griddep_wait();
+    griddep_launch_dependents();
+    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8 threads
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) {
+        const int r = r0 + ty + i, c = c0 + tx;
+        if (r < rows && c < cols) tile[ty + i][tx] = src[(size_t)r * (size_t)lds + c];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) {
+        const int c = c0 + ty + i, r = r0 + tx;
+        if (r < rows && c < cols) dst[(size_t)c * (size_t)ldd + r] = tile[tx][ty + i];
+    }
+}
+
 }  // namespace glue
+
+int launch_transpose_i8(const int8_t *src, int rows, int cols, int lds, int8_t *dst, int ldd,
+                        void *stream) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)((cols + 31) / 32), (unsigned)((rows + 31) / 32), 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = static_cast<cudaStream_t>(stream);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cfg.gridDim.y > 65535) return MQ_ERR_UNSUPPORTED_SHAPE;
+    return cudaLaunchKernelEx(&cfg, glue::transpose_i8_kernel, src, rows, cols, lds, dst, ldd) ==
+                   cudaSuccess
+               ? MQ_OK
+               : MQ_ERR_CUDA;
+}
 
 // Arguments are validated by the host entry points (mq_host.cpp).
 int launch_glue(int kind, int in_type, int out_type, const void *in, void *out, int64_t n,

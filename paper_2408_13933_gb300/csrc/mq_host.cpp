@@ -15,17 +15,25 @@ namespace {
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 int abits_of(const mq_linear_desc &d) { return d.abits == 0 ? 8 : d.abits; }
+int obits_of(const mq_linear_desc &d) { return d.obits == 0 ? abits_of(d) : d.obits; }
 
 // Validate one linear problem; on success fill the kernel-side Problem (for
 // 16-bit activations, x is filled in later with the planes' address).
 int check_desc(const mq_linear_desc &d, mq::Problem &out) {
-    const int ab = abits_of(d);
+    const int ab = abits_of(d), ob = obits_of(d);
     if (d.bits != 8 && d.bits != 4) return MQ_ERR_INVALID_ARG;
-    if (ab != 8 && ab != 16) return MQ_ERR_INVALID_ARG;
+    // activation / output widths: 8 / 8, 16 / 16, or 8 / 16
+    if (!((ab == 8 && ob == 8) || (ab == 16 && ob == 16) || (ab == 8 && ob == 16)))
+        return MQ_ERR_INVALID_ARG;
     if (d.M < 0 || d.N < 0 || d.K < 0) return MQ_ERR_INVALID_ARG;
     const int32_t zlo = ab == 8 ? -128 : -32768, zhi = ab == 8 ? 127 : 32767;
-    if (d.zx < zlo || d.zx > zhi || d.zy < zlo || d.zy > zhi) return MQ_ERR_INVALID_ARG;
+    const int32_t ylo = ob == 8 ? -128 : -32768, yhi = ob == 8 ? 127 : 32767;
+    if (d.zx < zlo || d.zx > zhi || d.zy < ylo || d.zy > yhi) return MQ_ERR_INVALID_ARG;
     if (ab == 16 && (d.residual || d.zw)) return MQ_ERR_INVALID_ARG;
+    if (ob == 16 && d.residual) return MQ_ERR_INVALID_ARG;
+    const int64_t wrow = (int64_t)d.K * d.bits / 8;  // packed bytes of one weight row
+    if (d.ldw < 0 || (d.ldw > 0 && d.ldw < wrow)) return MQ_ERR_INVALID_ARG;
+    if (d.ldw % 16 != 0) return MQ_ERR_ALIGNMENT;
     if (d.K > MQ_MAX_K) return MQ_ERR_K_OVERFLOW;
     if (d.zw && d.bits == 8 && d.K > MQ_MAX_K_ASYM8) return MQ_ERR_K_OVERFLOW;
     if (d.M > 0 && d.N > 0) {
@@ -56,6 +64,8 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     out.zy = d.zy;
     out.bits = d.bits;
     out.a16 = ab == 16;
+    out.o16 = ab == 8 && ob == 16;
+    out.ldw = d.ldw > 0 ? d.ldw : (int32_t)wrow;
     out.tile_begin = 0;
     out.tiles_m = 0;
     return MQ_OK;
@@ -151,9 +161,9 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         pl.rowsum[i].out = reinterpret_cast<int32_t *>(region + pl.rowsum_off[i]);
     for (size_t i = 0; i < pl.split.size(); ++i)
         pl.split[i].out = reinterpret_cast<int8_t *>(region + pl.split_off[i]);
-    // kernel families: prefill (int8 / 16-bit activations), decode by weight
-    // bits and activation width
-    std::vector<mq::Problem> pre8, pre16, dec[2][2];  // dec[bits == 8][a16]
+    // kernel families: prefill by activation / output width, decode by weight
+    // bits and activation / output width (0: 8 / 8, 1: 16 / 16, 2: 8 / 16)
+    std::vector<mq::Problem> pre[3], dec[2][3];
     for (int i = 0; i < count; ++i) {
         mq::Problem &p = probs[i];
         const mq_linear_desc &d = descs[i];
@@ -170,20 +180,21 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
                 p.x = pl.split[find_job(pl.split, d.x, d.M, d.K, d.ldx)].out;
             }
         }
+        const int mode = p.a16 ? 1 : (p.o16 ? 2 : 0);
         if (is_decode(d))
-            dec[p.bits == 8][p.a16].push_back(p);
+            dec[p.bits == 8][mode].push_back(p);
         else
-            (p.a16 ? pre16 : pre8).push_back(p);
+            pre[mode].push_back(p);
     }
     int rc = MQ_OK;
     if (!pl.rowsum.empty()) rc = mq::launch_rowsum(pl.rowsum.data(), (int)pl.rowsum.size(), stream);
     if (rc == MQ_OK && !pl.split.empty())
         rc = mq::launch_split16(pl.split.data(), (int)pl.split.size(), stream);
-    if (rc == MQ_OK && !pre8.empty()) rc = mq::launch_prefill(pre8.data(), (int)pre8.size(), stream);
-    if (rc == MQ_OK && !pre16.empty())
-        rc = mq::launch_prefill(pre16.data(), (int)pre16.size(), stream);
+    for (int mode = 0; mode < 3; ++mode)
+        if (rc == MQ_OK && !pre[mode].empty())
+            rc = mq::launch_prefill(pre[mode].data(), (int)pre[mode].size(), stream);
     for (int b = 1; b >= 0; --b)
-        for (int a = 0; a < 2; ++a)
+        for (int a = 0; a < 3; ++a)
             if (rc == MQ_OK && !dec[b][a].empty())
                 rc = mq::launch_decode(dec[b][a].data(), (int)dec[b][a].size(), workspace, stream);
     return rc;
@@ -374,6 +385,7 @@ int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *byte
     for (int i = 0; i < count; ++i) {
         if (descs[i].bits != 8 && descs[i].bits != 4) return MQ_ERR_INVALID_ARG;
         if (abits_of(descs[i]) != 8 && abits_of(descs[i]) != 16) return MQ_ERR_INVALID_ARG;
+        if (obits_of(descs[i]) != 8 && obits_of(descs[i]) != 16) return MQ_ERR_INVALID_ARG;
     }
     *bytes = batch_plan(descs, count).bytes;
     return MQ_OK;
@@ -505,6 +517,28 @@ int mq_fold_norm(const float *gamma, const float *beta, const float *s, int K, f
         if (beta) beta_out[k] = beta[k] / s[k];
     }
     return MQ_OK;
+}
+
+int mq_row_sums(const int8_t *x, int M, int K, int ldx, int32_t *out, void *stream) {
+    if (M < 0 || K < 0 || K > MQ_MAX_K || ldx < K) return MQ_ERR_INVALID_ARG;
+    if (M == 0) return MQ_OK;
+    if (!out || (K > 0 && !x)) return MQ_ERR_INVALID_ARG;
+    if (K % 16 != 0 || ldx % 16 != 0 || (K > 0 && !aligned16(x))) return MQ_ERR_ALIGNMENT;
+    mq::RowsumJob j{};
+    j.x = x;
+    j.out = out;
+    j.M = M;
+    j.K = K;
+    j.ldx = ldx;
+    return mq::launch_rowsum(&j, 1, stream);
+}
+
+int mq_transpose_i8(const int8_t *src, int rows, int cols, int lds, int8_t *dst, int ldd,
+                    void *stream) {
+    if (rows < 0 || cols < 0 || lds < cols || ldd < rows) return MQ_ERR_INVALID_ARG;
+    if (rows == 0 || cols == 0) return MQ_OK;
+    if (!src || !dst) return MQ_ERR_INVALID_ARG;
+    return mq::launch_transpose_i8(src, rows, cols, lds, dst, ldd, stream);
 }
 
 int mq_check_device_status(void *stream) {

@@ -33,6 +33,8 @@ struct Problem {
     // (ldx = K); the decode kernel reads the int16 codes [M'][ldx] and forms
     // the planes itself.
     int32_t a16;
+    int32_t o16;         // 8-bit inputs, int16 output y [M][ldy] (requantized to 16 bits)
+    int32_t ldw;         // bytes between weight rows
     int32_t tile_begin;  // first global tile / block index of this problem
     int32_t tiles_m;     // prefill: number of 128-row tiles
 };
@@ -57,8 +59,8 @@ int *device_status_ptr();
 int *pack_status_ptr();
 
 // Launchers (asynchronous on `stream`); return MQ_OK or MQ_ERR_CUDA.  The
-// problems of one launch_prefill call have the same a16; those of one
-// launch_decode call the same bits and a16.
+// problems of one launch_prefill call have the same a16 and o16; those of one
+// launch_decode call the same bits, a16 and o16.
 int launch_prefill(const Problem *probs, int count, void *stream);
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream);
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
@@ -72,6 +74,8 @@ struct RowsumJob {
 };
 constexpr int ROWSUM_MAX_JOBS = 64;  // jobs per launch (kernel parameter space)
 int launch_rowsum(const RowsumJob *jobs, int count, void *stream);
+int launch_transpose_i8(const int8_t *src, int rows, int cols, int lds, int8_t *dst, int ldd,
+                        void *stream);
 
 // One distinct int16 input of a batch and where its two int8 planes go:
 // out row 2m = high bytes of x row m, row 2m + 1 = low bytes - 128 (pitch K).

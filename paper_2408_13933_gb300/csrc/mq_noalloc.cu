@@ -89,5 +89,6 @@ extern "C" int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, in
     p.zx = zx;
     p.zy = zy;
     p.bits = 4;
+    p.ldw = K / 2;
     return mq::launch_decode(&p, 1, scratch, stream);
 }

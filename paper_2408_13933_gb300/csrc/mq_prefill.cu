@@ -223,7 +223,8 @@ __device__ __forceinline__ void store_channel(const uint32_t (&acc)[64], int32_t
 // complete; waiters acquire at CTA scope, which is far cheaper per wait.
 // A16: every problem has 16-bit activations (Problem::a16): its x is the
 // plane matrix, and the epilogue combines row pairs and stores int16.
-template <bool A16>
+// O16: every problem has 8-bit inputs and a 16-bit output (Problem::o16).
+template <bool A16, bool O16>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     prefill_kernel(const __grid_constant__ Params P) {
     extern __shared__ uint8_t smem_raw[];
@@ -585,6 +586,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 }
             }
             const size_t ldy = (size_t)e.ldy;
+            if constexpr (O16) {
+                // the same sum, requantized to 16 bits (no residual)
+                int16_t *yp16 = reinterpret_cast<int16_t *>(e.y) + (size_t)tok0 * ldy + ch;
+#pragma unroll
+                for (int j = 0; j < 64; ++j)
+                    if (j < ntok)
+                        yp16[(size_t)j * ldy] = (int16_t)mq_requant16(
+                            (int64_t)(int32_t)(acc[j] - (uint32_t)corr), m0, sh, e.zy);
+                continue;
+            }
             int8_t *yp = e.y + (size_t)tok0 * ldy + ch;
             const int8_t *rp = e.residual ? e.residual + (size_t)tok0 * ldy + ch : nullptr;
             const bool full = ntok == 64, fast = sh >= 33;
@@ -650,7 +661,7 @@ int max_pairs(int dev) {
     cfg.blockDim = dim3(THREADS, 1, 1);
     cfg.dynamicSmemBytes = SMEM_BYTES;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, prefill_kernel<false>, &cfg) == cudaSuccess &&
+    if (cudaOccupancyMaxActiveClusters(&clusters, prefill_kernel<false, false>, &cfg) == cudaSuccess &&
         clusters > 0 && clusters < n)
         n = clusters;
     if (n > MAX_PAIRS) n = MAX_PAIRS;
@@ -700,15 +711,22 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
     if (attr_done != dev) {
-        if (cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(prefill_kernel<false, false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)SMEM_BYTES) != cudaSuccess ||
-            cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            cudaFuncSetAttribute(prefill_kernel<true, false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)SMEM_BYTES) != cudaSuccess ||
+            cudaFuncSetAttribute(prefill_kernel<false, true>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)SMEM_BYTES) != cudaSuccess)
             return MQ_ERR_CUDA;
         attr_done = dev;
     }
     if (count <= 0) return MQ_OK;
-    auto kern = probs[0].a16 ? prefill_kernel<true> : prefill_kernel<false>;
+    auto kern = probs[0].a16   ? prefill_kernel<true, false>
+                : probs[0].o16 ? prefill_kernel<false, true>
+                               : prefill_kernel<false, false>;
     const int pairs_max = max_pairs(dev);
     if (pairs_max < 1) return MQ_ERR_CUDA;
     for (int begin = 0; begin < count; begin += PREFILL_MAX_PROBLEMS) {
@@ -735,8 +753,8 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
                 const uint64_t wcols = i4 ? (uint64_t)q.K / 2 : (uint64_t)q.K;
                 if (!encode_2d(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M, (uint64_t)q.ldx,
                                KS, CN) ||
-                    !encode_2d(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, wcols, i4 ? KS / 2 : KS,
-                               CM))
+                    !encode_2d(&P.tmap_w[i], q.w, wcols, (uint64_t)q.N, (uint64_t)q.ldw,
+                               i4 ? KS / 2 : KS, CM))
                     return MQ_ERR_CUDA;
             }
         }

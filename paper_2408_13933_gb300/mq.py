@@ -40,7 +40,8 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
             "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch",
             "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16", "mq_quantize",
-            "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm"]
+            "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm",
+            "mq_row_sums", "mq_transpose_i8"]
 MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
@@ -52,7 +53,7 @@ class LinearDesc(ctypes.Structure):
     _fields_ = [("x", _vp), ("packed", _vp), ("colsum", _vp), ("M0", _vp), ("shift", _vp),
                 ("residual", _vp), ("zw", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
                 ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32),
-                ("abits", _i32)]
+                ("abits", _i32), ("obits", _i32), ("ldw", _i32)]
 
 
 lib.mq_status_string.argtypes = [_int]
@@ -80,6 +81,8 @@ lib.mq_requantize.argtypes = [_vp, _int, _i64, _i32, _i32, _i32, _i32, _vp, _int
 lib.mq_fold_quantize_pack.argtypes = [_vp, _int, _int, _vp, _vp, _int, _int, _vp, _vp, _vp, _vp,
                                       _vp, _vp]
 lib.mq_fold_norm.argtypes = [_vp, _vp, _vp, _int, _vp, _vp]
+lib.mq_row_sums.argtypes = [_vp, _int, _int, _int, _vp, _vp]
+lib.mq_transpose_i8.argtypes = [_vp, _int, _int, _int, _vp, _int, _vp]
 for _f in EXPORTED:
     if _f != "mq_status_string":
         getattr(lib, _f).restype = _int
@@ -261,6 +264,29 @@ def fold_norm(gamma: np.ndarray, beta, s: np.ndarray):
     return g, b
 
 
+def row_sums(x, out=None, m=None, k=None, ldx=None, stream=None):
+    """mq_row_sums on an int8 CUDA tensor [M, K] (or a strided view): int32 [M]."""
+    import torch
+    m = x.shape[0] if m is None else m
+    k = x.shape[1] if k is None else k
+    ldx = x.stride(0) if ldx is None else ldx
+    if out is None:
+        out = torch.empty(m, dtype=torch.int32, device=x.device)
+    _check(lib.mq_row_sums(_ptr(x), m, k, ldx, _ptr(out), _stream(stream)), "mq_row_sums")
+    return out
+
+
+def transpose_i8(src, dst=None, stream=None):
+    """mq_transpose_i8 on an int8 CUDA tensor [R, C] (or a row-strided view)."""
+    import torch
+    rows, cols = src.shape
+    if dst is None:
+        dst = torch.empty((cols, rows), dtype=torch.int8, device=src.device)
+    _check(lib.mq_transpose_i8(_ptr(src), rows, cols, src.stride(0), _ptr(dst), dst.stride(0),
+                               _stream(stream)), "mq_transpose_i8")
+    return dst
+
+
 def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, y,
                         ldx: int | None = None, ldy: int | None = None, m: int | None = None,
                         k: int | None = None, stream=None) -> int:
@@ -276,13 +302,20 @@ def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, 
 
 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
-              ldx=None, ldy=None, m=None, k=None, zw=None, abits=None) -> LinearDesc:
+              ldx=None, ldy=None, m=None, k=None, zw=None, abits=None, obits=None,
+              ldw: int = 0) -> LinearDesc:
     """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights;
-    abits 16 (default: 16 for an int16 x) gives int16 activations and outputs."""
+    abits 16 (default: 16 for an int16 x) gives int16 activations and outputs;
+    obits 16 with int8 x (default: 16 for an int16 y) an int16 output; `ldw`
+    the bytes between weight rows (0: packed)."""
     d = LinearDesc()
     if abits is None:
         abits = 16 if getattr(x, "element_size", lambda: 1)() == 2 else 8
+    if obits is None:
+        obits = 16 if getattr(y, "element_size", lambda: 1)() == 2 else 8
     d.abits = int(abits)
+    d.obits = int(obits)
+    d.ldw = int(ldw)
     d.x, d.packed, d.colsum = _ptr(x), _ptr(packed), _ptr(colsum)
     d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
     d.zw = _ptr(zw)

@@ -1,0 +1,190 @@
+"""The attention matmul glue on the GPU against the oracle: 8-bit inputs with a
+16-bit output (scores ahead of the 16-bit softmax), weights read through a
+row pitch (a head's slice of a projection output), row sums of activation
+matrices used as colsum, the int8 transpose, and grouped-query attention's
+Q K^T (int16 scores) and P V (int8) through the batch call."""
+import numpy as np
+import pytest
+
+import oracle
+from gpu_helpers import assert_equal_int8, torch_cuda, upload
+from paper_2408_13933_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def mq():
+    from paper_2408_13933_gb300 import mq as m
+    return m
+
+
+def assert_equal(got, want, what):
+    if not np.array_equal(got, want):
+        bad = np.argwhere(got != want)
+        i = tuple(bad[0])
+        raise AssertionError(f"{what}: {len(bad)} of {want.size} differ; first at {i}: "
+                             f"got {int(got[i])}, want {int(want[i])}")
+
+
+def _run(descs, keep):
+    torch = torch_cuda()
+    lib = mq()
+    need = lib.workspace_size_batch(descs)
+    ws = torch.zeros(max(need, 16), dtype=torch.uint8, device="cuda")
+    keep.append(ws)
+    assert lib.linear_batch(descs, workspace=ws, ws_bytes=need) == 0
+    torch.cuda.synchronize()
+    assert lib.check_device_status() == 0
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("asym", [False, True])
+@pytest.mark.parametrize("shape", [(128, 256, 512), (300, 100, 320), (1, 256, 2048), (9, 70, 1024)],
+                         ids=lambda s: "x".join(map(str, s)))
+def test_o16_parity(shape, asym, bits):
+    torch = torch_cuda()
+    lib = mq()
+    m, n, k = shape
+    c = synth.random_case(400 + m + n, m, k, n, bits)
+    rng = np.random.default_rng(m * n)
+    lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+    zw = rng.integers(lo, hi + 1, size=n).astype(np.int32) if asym else None
+    m0 = rng.integers(1 << 30, 1 << 31, size=n).astype(np.int32)
+    sh = rng.integers(28, 47, size=n).astype(np.int32)
+    zy = int(rng.integers(-20000, 20000))
+    packed, colsum = lib.pack_weights(c.w, bits)
+    keep = [upload(a) for a in (c.x, packed, colsum, m0, sh)]
+    zwd = upload(zw) if zw is not None else None
+    y = torch.full((m, n), 7, dtype=torch.int16, device="cuda")
+    keep += [zwd, y]
+    d = lib.make_desc(keep[0], c.zx, keep[1], keep[2], n, keep[3], keep[4], zy, y, bits, zw=zwd)
+    assert d.obits == 16 and d.abits == 8
+    _run([d], keep)
+    opk, _ = oracle.pack(c.w, bits)
+    want = oracle.linear_o16(c.x, c.zx, opk, bits, n, m0, sh, zy, zw=zw)
+    assert_equal(y.cpu().numpy(), want, f"o16 {shape} asym={asym} bits={bits}")
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("m", [2, 80])
+def test_weights_through_a_row_pitch(m, bits):
+    # the weights are columns [64, 64 + K) of a wider matrix: ldw = its row bytes
+    torch = torch_cuda()
+    lib = mq()
+    n, k, kfull, off = 96, 128, 320, 64
+    big = synth.random_case(500 + m + bits, m, kfull, n, bits)
+    w = np.ascontiguousarray(big.w[:, off:off + k])
+    x = np.ascontiguousarray(big.x[:, :k])
+    packed_full, _ = lib.pack_weights(big.w, bits)
+    _, colsum = lib.pack_weights(w, bits)
+    m0, sh = lib.requant_params(big.sw, big.sx, big.sy)
+    row = kfull if bits == 8 else kfull // 2
+    first = off if bits == 8 else off // 2
+    pk = upload(packed_full)
+    keep = [upload(a) for a in (x, colsum, m0, sh)] + [pk]
+    y = torch.full((m, n), 5, dtype=torch.int8, device="cuda")
+    keep.append(y)
+    d = lib.make_desc(keep[0], big.zx, pk[:, first:], keep[1], n, keep[2], keep[3], big.zy, y, bits,
+                      ldw=row)
+    _run([d], keep)
+    opk, _ = oracle.pack(w, bits)
+    om0, osh = oracle.requant_params(big.sx, big.sw, big.sy)
+    want = oracle.linear(x, big.zx, opk, bits, n, om0, osh, big.zy)
+    assert_equal_int8(y.cpu().numpy(), want, f"ldw m={m} bits={bits}")
+
+
+def test_row_sums_and_transpose():
+    torch = torch_cuda()
+    lib = mq()
+    rng = np.random.default_rng(3)
+    for rows, cols in ((1, 16), (100, 64), (1024, 4096), (33, 2048)):
+        a = rng.integers(-128, 128, size=(rows, cols), dtype=np.int16).astype(np.int8)
+        ad = upload(a)
+        got = lib.row_sums(ad).cpu().numpy()
+        assert np.array_equal(got, a.astype(np.int64).sum(1))
+    # a strided view: columns 64..127 of a [200, 256] matrix
+    a = rng.integers(-128, 128, size=(200, 256), dtype=np.int16).astype(np.int8)
+    ad = upload(a)
+    assert np.array_equal(lib.row_sums(ad[:, 64:128]).cpu().numpy(),
+                          a[:, 64:128].astype(np.int64).sum(1))
+    for rows, cols in ((1, 1), (33, 70), (1024, 64), (64, 1000), (257, 129)):
+        a = rng.integers(-128, 128, size=(rows, cols), dtype=np.int16).astype(np.int8)
+        ad = upload(a)
+        t = lib.transpose_i8(ad)
+        torch.cuda.synchronize()
+        assert np.array_equal(t.cpu().numpy(), a.T)
+    a = rng.integers(-128, 128, size=(96, 256), dtype=np.int16).astype(np.int8)
+    ad = upload(a)
+    t = lib.transpose_i8(ad[:, 128:192])   # a head's slice
+    torch.cuda.synchronize()
+    assert np.array_equal(t.cpu().numpy(), a[:, 128:192].T)
+
+
+@pytest.mark.parametrize("t_q", [96, 1])
+def test_grouped_query_attention_matmuls(t_q):
+    # 4 query heads over 2 KV heads, head dim 64, T = 96 keys; t_q query tokens
+    # (96: prefill kernel, 1: decode kernel for the scores)
+    torch = torch_cuda()
+    lib = mq()
+    rng = np.random.default_rng(11 + t_q)
+    T, H, G, D = 96, 4, 2, 64
+    i8 = lambda *s: rng.integers(-128, 128, size=s, dtype=np.int16).astype(np.int8)
+    q, kk, v = i8(t_q, H * D), i8(T, G * D), i8(T, G * D)
+    zq, zk, zv = -5, 12, -20
+    qd, kd, vd = upload(q), upload(kk), upload(v)
+    keep = [qd, kd, vd]
+    # ---- scores S_h = Q_h K_g^T, int16 (obits 16), keys as weights through ldw
+    m0s = np.full(T, 1 << 30, np.int32)
+    shs = np.full(T, 33, np.int32)          # scale 1/8
+    zys = 100
+    m0d, shd = upload(m0s), upload(shs)
+    zwk = upload(np.full(T, zk, np.int32))
+    keep += [m0d, shd, zwk]
+    descs, outs, colsums = [], [], []
+    for g in range(G):
+        colsums.append(lib.row_sums(kd[:, g * D:(g + 1) * D]))
+    keep += colsums
+    for h in range(H):
+        g = h // (H // G)
+        s = torch.full((t_q, T), 3, dtype=torch.int16, device="cuda")
+        outs.append(s)
+        descs.append(lib.make_desc(qd[:, h * D:(h + 1) * D], zq, kd[:, g * D:(g + 1) * D],
+                                   colsums[g], T, m0d, shd, zys, s, 8, zw=zwk, k=D,
+                                   ldx=H * D, ldw=G * D))
+    keep += outs
+    _run(descs, keep)
+    for h in range(H):
+        g = h // (H // G)
+        kg = np.ascontiguousarray(kk[:, g * D:(g + 1) * D])
+        opk, _ = oracle.pack(kg, 8)
+        want = oracle.linear_o16(np.ascontiguousarray(q[:, h * D:(h + 1) * D]), zq, opk, 8, T,
+                                 m0s, shs, zys, zw=np.full(T, zk, np.int32))
+        assert_equal(outs[h].cpu().numpy(), want, f"scores head {h}")
+    # ---- O_h = P_h V_g: P (the requantized softmax output) int8, V^T as weights
+    p = i8(H, t_q, T)
+    zp = 7
+    pd = upload(p)
+    keep.append(pd)
+    vts = [lib.transpose_i8(vd[:, g * D:(g + 1) * D]) for g in range(G)]
+    vcs = [lib.row_sums(vt) for vt in vts]
+    keep += vts + vcs
+    m0o = np.full(D, 1 << 30, np.int32)
+    sho = np.full(D, 40, np.int32)          # scale 2^-10
+    m0od, shod = upload(m0o), upload(sho)
+    zwv = upload(np.full(D, zv, np.int32))
+    keep += [m0od, shod, zwv]
+    descs, outs = [], []
+    for h in range(H):
+        g = h // (H // G)
+        o = torch.full((t_q, D), 9, dtype=torch.int8, device="cuda")
+        outs.append(o)
+        descs.append(lib.make_desc(pd[h], zp, vts[g], vcs[g], D, m0od, shod, -3, o, 8, zw=zwv))
+    keep += outs
+    _run(descs, keep)
+    for h in range(H):
+        g = h // (H // G)
+        vt = np.ascontiguousarray(v[:, g * D:(g + 1) * D].T)
+        opk, _ = oracle.pack(vt, 8)
+        want = oracle.linear(np.ascontiguousarray(p[h]), zp, opk, 8, D, m0o, sho, -3,
+                             zw=np.full(D, zv, np.int32))
+        assert_equal_int8(outs[h].cpu().numpy(), want, f"P V head {h}")

@@ -330,3 +330,38 @@ def test_fold_validation_and_norm(mq):
     assert b3 is None and np.array_equal(g3, g / s)
     with pytest.raises(mq.MQError):
         mq.fold_norm(g, b, np.array([1.0, 0.0, 1.0, 1.0], np.float32))
+
+
+def test_o16_ldw_rowsums_transpose_validation(mq):
+    # every rejection happens before a launch
+    def rc(d):
+        return mq.lib.mq_linear_batch((mq.LinearDesc * 1)(d), 1, FAKE, 1 << 30, None)
+    d = _desc(mq, 40, 64, 32, 8, False)
+    d.obits = 16
+    d.zy = 40000
+    assert rc(d) == mq.MQ_ERR_INVALID_ARG           # zy outside int16
+    d.zy = 0
+    d.residual = FAKE
+    assert rc(d) == mq.MQ_ERR_INVALID_ARG           # no residual with a 16-bit output
+    d = _desc(mq, 40, 64, 32, 8, False)
+    d.abits, d.obits = 16, 8
+    assert rc(d) == mq.MQ_ERR_INVALID_ARG           # 16-bit inputs need 16-bit outputs
+    d = _desc(mq, 40, 64, 32, 8, False)
+    d.obits = 12
+    assert rc(d) == mq.MQ_ERR_INVALID_ARG
+    d = _desc(mq, 40, 64, 32, 8, False)
+    d.ldw = 48
+    assert rc(d) == mq.MQ_ERR_INVALID_ARG           # pitch below the packed row (64 bytes)
+    d.ldw = 72
+    assert rc(d) == mq.MQ_ERR_ALIGNMENT             # not a multiple of 16
+    d4 = _desc(mq, 40, 64, 32, 4, False)
+    d4.ldw = 16
+    assert rc(d4) == mq.MQ_ERR_INVALID_ARG          # int4 rows of K = 64 take 32 bytes
+    r = mq.lib.mq_row_sums
+    assert r(FAKE, 4, 40, 48, FAKE, None) == mq.MQ_ERR_ALIGNMENT
+    assert r(FAKE, 4, 64, 32, FAKE, None) == mq.MQ_ERR_INVALID_ARG
+    assert r(None, 0, 64, 64, None, None) == 0
+    t = mq.lib.mq_transpose_i8
+    assert t(FAKE, 4, 8, 4, FAKE, 4, None) == mq.MQ_ERR_INVALID_ARG   # lds < cols
+    assert t(FAKE, 4, 8, 8, FAKE, 2, None) == mq.MQ_ERR_INVALID_ARG   # ldd < rows
+    assert t(None, 0, 8, 8, None, 8, None) == 0
