@@ -234,7 +234,7 @@ class PrefillBlock:
             self.descs.append(mq.make_desc(self.x_dev[id(c.x)], c.zx, t[0], t[1], c.N, t[2], t[3],
                                            c.zy, y, 8, residual=res, zw=zw))
         self.arr = (mq.LinearDesc * len(self.descs))(*self.descs)
-        # asymmetric weights: rowsum(x) of each distinct input lives in the workspace
+        # decode shapes need the decode region; prefill (asymmetric or not) nothing
         self.ws_bytes = mq.workspace_size_batch(self.descs)
         self.ws = torch.zeros(max(16, self.ws_bytes), dtype=torch.uint8, device=dev)
         self.wsp = self.ws.data_ptr() if self.ws_bytes else None
@@ -417,8 +417,8 @@ def run_decode(mq, torch, steps_per_m: int = 240, asym: bool = False, ms=DECODE_
 def run_asym_prefill(mq, torch, steps: int = 900, check_rows: int = 4):
     """The same block with asymmetric weights in the paper's W8A8 setting (per
     tensor, down per channel): int8 TOPS over `steps` back-to-back batched
-    calls (rowsum pre-pass + prefill kernel each), rotating over three layers,
-    and the first `check_rows` token rows of layer 0 checked against the oracle."""
+    calls (one prefill launch each), rotating over three layers,
+    and the first `check_rows` token rows of layer 0 handed to the oracle check."""
     blocks = [PrefillBlock(mq, torch, layer, PREFILL_M, asym=True)
               for layer in range(PREFILL_LAYERS)]
     stream = torch.cuda.current_stream()
@@ -442,28 +442,17 @@ def run_asym_prefill(mq, torch, steps: int = 900, check_rows: int = 4):
     if mq.check_device_status() != 0:
         raise RuntimeError("device status error in the asymmetric prefill run")
     ms = e0.elapsed_time(e1) / steps
-    # parity sample: run layer 0 once more, then compare its first rows
+    # parity sample: run layer 0 once more; its first rows are checked against
+    # the oracle in the cpu_baseline leg
     step(0)
     torch.cuda.synchronize()
-    import oracle
-    oracle.build()
-    mism = checked = 0
-    for j, c in enumerate(blocks[0].cases):
-        packed, _ = oracle.pack(c.w, 8)
-        m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
-        y = oracle.linear(np.ascontiguousarray(c.x[:check_rows]), c.zx, packed, 8, c.N, m0, sh,
-                          c.zy, zw=c.zw)
-        if c.residual is not None:
-            y = oracle.residual_add(y, np.ascontiguousarray(c.residual[:check_rows]))
-        got = blocks[0].y[j][:check_rows].cpu().numpy()
-        checked += y.size
-        mism += int(np.count_nonzero(got != y))
+    checks = [ParityCheck("asym_prefill_w8a8", "linear", c, check_rows,
+                          blocks[0].y[j][:check_rows].cpu().numpy())
+              for j, c in enumerate(blocks[0].cases)]
     return {"us_per_block": round(ms * 1e3, 2),
             "tops": round(block_ops(PREFILL_M) / (ms * 1e-3) / 1e12, 1),
-            "launches_per_step": 2, "steps": steps,
-            "weights": "asymmetric: per tensor (q k v o gate up), per channel (down)",
-            "parity_sample": {"rows": check_rows, "outputs": checked, "mismatches": mism}}
-
+            "launches_per_step": 1, "steps": steps,
+            "weights": "asymmetric: per tensor (q k v o gate up), per channel (down)"}, checks
 
 class A16Block:
     """Device-resident operands of one layer's seven linears with 16-bit
@@ -519,33 +508,23 @@ def _time_blocks(mq, torch, blocks, steps: int):
 def run_a16(mq, torch, prefill_steps: int = 600, check_rows: int = 4):
     """W8A16 prefill of the block at M = 1024 (the paper's 16-bit-activation
     baseline, Sec. 5.6), back-to-back batched calls (split pre-pass + kernel)
-    rotating over three layers, the first rows of layer 0 checked against the
-    oracle; and W4A16 decode at M = 1 and 8, timed like the W4A8 decode
+    rotating over three layers, the first rows of layer 0 handed to the oracle
+    check; and W4A16 decode at M = 1 and 8, timed like the W4A8 decode
     (one launch per layer, per launch and over a CUDA graph)."""
-    import oracle
-    oracle.build()
     out = {}
     blocks = [A16Block(mq, torch, layer, PREFILL_M, 8, CONFIG_ID_PREFILL, True)
               for layer in range(PREFILL_LAYERS)]
     ms = _time_blocks(mq, torch, blocks, prefill_steps)
-    mism = checked = 0
-    for j, c in enumerate(blocks[0].cases):
-        packed, _ = oracle.pack(c.w, 8)
-        m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
-        y = oracle.linear_a16(np.ascontiguousarray(c.x[:check_rows]), c.zx, packed, 8, c.N, m0,
-                              sh, c.zy)
-        got = blocks[0].y[j][:check_rows].cpu().numpy()
-        checked += y.size
-        mism += int(np.count_nonzero(got != y))
+    checks = [ParityCheck("a16.prefill_w8a16", "a16", c, check_rows,
+                          blocks[0].y[j][:check_rows].cpu().numpy())
+              for j, c in enumerate(blocks[0].cases)]
     out["prefill_w8a16"] = {"us_per_block": round(ms * 1e3, 2),
                             "tops": round(block_ops(PREFILL_M) / (ms * 1e-3) / 1e12, 1),
-                            "launches_per_step": 2, "steps": prefill_steps,
-                            "parity_sample": {"rows": check_rows, "outputs": checked,
-                                              "mismatches": mism}}
+                            "launches_per_step": 2, "steps": prefill_steps}
     del blocks
     for m, v in run_decode(mq, torch, a16=True, ms=(1, 8)).items():
         out[f"decode_w4a16_{m}"] = v
-    return out
+    return out, checks
 
 
 def run_glue(mq, torch, n: int = 1 << 26, reps: int = 20):
@@ -617,6 +596,165 @@ def run_weight_pipeline(mq, torch, reps: int = 5):
     return out
 
 
+ATT_T, ATT_SETS = 1024, 3
+
+
+class ParityCheck:
+    """Host copies of the first `rows` token rows of one device output and of
+    the operands that made it; the cpu_baseline leg recomputes them with the
+    oracle.  kind: "linear" (int8 out, optional asymmetric weights and
+    residual), "a16" (16-bit activations), "o16" (int8 in, int16 out).  With
+    m0/sh given they are the device's fixed-point parameters; otherwise the
+    oracle derives them from the case's float scales."""
+
+    def __init__(self, leg: str, kind: str, case, rows: int, got: np.ndarray, m0=None, sh=None):
+        self.leg, self.kind, self.case, self.rows, self.got = leg, kind, case, rows, got
+        self.m0, self.sh = m0, sh
+
+
+class AttentionSet:
+    """Device operands and batched descriptors of one layer's attention matmuls
+    (TinyLlama: 32 query heads over 4 KV heads, head dim 64, T tokens):
+    S_h = Q_h K_g^T (int8 in, int16 scores, keys as the weights read through a
+    row pitch, asymmetric per tensor: zw = zk) and O_h = P_h V_g (int8, V_g^T as
+    the weights, zw = zv), O written into head h's columns of [T][32 * 64].
+    Both read weights written on the device in the same stream (wdynamic)."""
+
+    M0_S, SH_S = 1 << 30, 34     # scores: scale 2^-5 (int16 output)
+    M0_O, SH_O = 1 << 30, 40     # outputs: scale 2^-11
+    ZY_S, ZY_O = 0, -3
+
+    def __init__(self, mq, torch, layer: int, t: int):
+        a = synth.attention_operands(CONFIG_ID_PREFILL, layer, t)
+        self.ops_host = a
+        H, G, D = a.heads, a.kv_heads, a.d
+        dev = "cuda"
+        up = lambda arr: torch.from_numpy(np.ascontiguousarray(arr)).to(dev)
+        self.q, self.k, self.v, self.p = up(a.q), up(a.k), up(a.v), up(a.p)
+        self.s = torch.empty((H, t, t), dtype=torch.int16, device=dev)
+        self.o = torch.empty((t, H * D), dtype=torch.int8, device=dev)
+        self.colk = torch.empty((G, t), dtype=torch.int32, device=dev)
+        self.vt = torch.empty((G, D, t), dtype=torch.int8, device=dev)
+        self.colv = torch.empty((G, D), dtype=torch.int32, device=dev)
+        i32 = lambda n, v: up(np.full(n, v, np.int32))
+        self.keep = [i32(t, self.M0_S), i32(t, self.SH_S), i32(t, a.zk),
+                     i32(D, self.M0_O), i32(D, self.SH_O), i32(D, a.zv)]
+        m0s, shs, zwk, m0o, sho, zwv = self.keep
+        rep = H // G
+        ds = [mq.make_desc(self.q[:, h * D:(h + 1) * D], a.zq, self.k[:, (h // rep) * D:],
+                           self.colk[h // rep], t, m0s, shs, self.ZY_S, self.s[h], 8, zw=zwk,
+                           ldw=G * D, wdynamic=True) for h in range(H)]
+        do = [mq.make_desc(self.p[h], a.zp, self.vt[h // rep], self.colv[h // rep], D, m0o, sho,
+                           self.ZY_O, self.o[:, h * D:(h + 1) * D], 8, zw=zwv, wdynamic=True)
+              for h in range(H)]
+        self.arr_s = (mq.LinearDesc * H)(*ds)
+        self.arr_o = (mq.LinearDesc * H)(*do)
+        self.ws_s_bytes = mq.workspace_size_batch(ds)
+        self.ws_o_bytes = mq.workspace_size_batch(do)
+        self.ws_s = torch.zeros(max(16, self.ws_s_bytes), dtype=torch.uint8, device=dev)
+        self.ws_o = torch.zeros(max(16, self.ws_o_bytes), dtype=torch.uint8, device=dev)
+        self.H, self.G, self.D, self.t = H, G, D, t
+        self.bytes = (self.q.numel() + self.k.numel() + self.v.numel() + 2 * self.s.numel()
+                      + self.p.numel() + self.o.numel())
+
+    def enqueue(self, mq, sp, phase: str = "all"):
+        lib, H, G, D, t = mq.lib, self.H, self.G, self.D, self.t
+        rcs = []
+        if phase in ("all", "scores"):
+            for g in range(G):
+                rcs.append(lib.mq_row_sums(self.k[:, g * D:].data_ptr(), t, D, G * D,
+                                           self.colk[g].data_ptr(), sp))
+            rcs.append(lib.mq_linear_batch(self.arr_s, H, self.ws_s.data_ptr(), self.ws_s_bytes,
+                                           sp))
+        if phase in ("all", "pv"):
+            for g in range(G):
+                rcs.append(lib.mq_transpose_i8(self.v[:, g * D:].data_ptr(), t, D, G * D,
+                                               self.vt[g].data_ptr(), t, sp))
+                rcs.append(lib.mq_row_sums(self.vt[g].data_ptr(), D, t, t,
+                                           self.colv[g].data_ptr(), sp))
+            rcs.append(lib.mq_linear_batch(self.arr_o, H, self.ws_o.data_ptr(), self.ws_o_bytes,
+                                           sp))
+        if any(rcs):
+            raise RuntimeError(f"attention launch failed: {[mq.status_string(r) for r in rcs]}")
+        return len(rcs)
+
+    def checks(self, rows: int, heads=(0, 31)):
+        """ParityChecks of the scores and outputs of `heads`, first `rows` rows."""
+        a, D, rep = self.ops_host, self.D, self.H // self.G
+        out = []
+        for h in heads:
+            g = h // rep
+            kg = np.ascontiguousarray(a.k[:, g * D:(g + 1) * D])
+            sc = synth.LinearCase(f"scores{h}", np.ascontiguousarray(a.q[:rows, h * D:(h + 1) * D]),
+                                  a.zq, 0.0, kg, None, 8, 0.0, self.ZY_S)
+            sc.zw = np.full(self.t, a.zk, np.int32)
+            out.append(ParityCheck("attention_w8a8_t1024", "o16", sc, rows,
+                                   self.s[h, :rows].cpu().numpy(),
+                                   np.full(self.t, self.M0_S, np.int32),
+                                   np.full(self.t, self.SH_S, np.int32)))
+            vt = np.ascontiguousarray(a.v[:, g * D:(g + 1) * D].T)
+            pc = synth.LinearCase(f"pv{h}", np.ascontiguousarray(a.p[h, :rows]), a.zp, 0.0, vt,
+                                  None, 8, 0.0, self.ZY_O)
+            pc.zw = np.full(D, a.zv, np.int32)
+            out.append(ParityCheck("attention_w8a8_t1024", "linear", pc, rows,
+                                   self.o[:rows, h * D:(h + 1) * D].cpu().numpy(),
+                                   np.full(D, self.M0_O, np.int32),
+                                   np.full(D, self.SH_O, np.int32)))
+        return out
+
+
+def run_attention(mq, torch, reps: int = 60, check_rows: int = 4):
+    """Grouped-query attention's two integer matmuls of one TinyLlama layer at
+    T = 1024 (the softmax between them is outside the integer layer): per step
+    the key row sums, S = Q K^T for 32 heads (one batched call, one prefill
+    launch, int16 scores), the V^T transposes and their row
+    sums, and O = P V for 32 heads (one batched call).  Steps rotate over three
+    layers' operands (about 300 MB, more than L2).  The host enqueues the timed
+    steps behind a device sleep, so the region measures the device, not the
+    ctypes call rate; a second pass times the two phases alone."""
+    sets = [AttentionSet(mq, torch, layer, ATT_T) for layer in range(ATT_SETS)]
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    launches = 0
+    for i in range(2 * ATT_SETS):
+        launches = sets[i % ATT_SETS].enqueue(mq, sp)
+    torch.cuda.synchronize()
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in the attention warm-up")
+
+    def timed(phase: str, n: int) -> float:
+        torch.cuda.synchronize()
+        torch.cuda._sleep(100_000_000)  # about 50 ms: the host enqueues every step meanwhile
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(n):
+            sets[i % ATT_SETS].enqueue(mq, sp, phase)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / n
+
+    ms = timed("all", reps)
+    ms_s = timed("scores", reps)
+    ms_o = timed("pv", reps)
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in the attention run")
+    sets[0].enqueue(mq, sp)   # layer 0 last, for the parity sample
+    torch.cuda.synchronize()
+    b = sets[0]
+    ops = 2 * 2 * b.t * b.t * b.D * b.H
+    checks = b.checks(check_rows)
+    res = {"what": "S = Q K^T (int16 scores) and O = P V, 32 query heads over 4 KV heads, "
+                   "head dim 64, T = 1024; full T x T scores (the causal mask is applied by "
+                   "the softmax, not here)",
+           "us_per_layer": round(ms * 1e3, 2), "tops": round(ops / (ms * 1e-3) / 1e12, 1),
+           "algorithmic_bytes": b.bytes,
+           "gbs": round(b.bytes / (ms * 1e-3) / 1e9, 1),
+           "scores_us": round(ms_s * 1e3, 2), "pv_us": round(ms_o * 1e3, 2),
+           "launches_per_step": launches, "steps": reps}
+    del sets
+    return res, checks
+
+
 # --------------------------------------------------------------------------- CPU oracle
 def oracle_sample(blocks_cases, rows: range, col_frac: float = 1.0):
     """Run the oracle on `rows` of every linear of one block; returns
@@ -638,11 +776,39 @@ def oracle_sample(blocks_cases, rows: range, col_frac: float = 1.0):
     return ops, time.perf_counter() - t0, outs
 
 
-def cpu_baseline(blocks, torch, rows: int = 192):
+def run_checks(checks) -> dict:
+    """Recompute every ParityCheck with the oracle: {leg: {rows, outputs,
+    mismatches}}."""
+    import oracle
+    out = {}
+    for ck in checks:
+        c = ck.case
+        x = np.ascontiguousarray(c.x[:ck.rows])
+        packed, _ = oracle.pack(c.w, c.bits)
+        if ck.m0 is not None:
+            m0, sh = ck.m0, ck.sh
+        else:
+            m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
+        if ck.kind == "a16":
+            y = oracle.linear_a16(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy)
+        elif ck.kind == "o16":
+            y = oracle.linear_o16(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy, zw=c.zw)
+        else:
+            y = oracle.linear(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy, zw=c.zw)
+            if c.residual is not None:
+                y = oracle.residual_add(y, np.ascontiguousarray(c.residual[:ck.rows]))
+        r = out.setdefault(ck.leg, {"rows": ck.rows, "outputs": 0, "mismatches": 0})
+        r["outputs"] += int(y.size)
+        r["mismatches"] += int(np.count_nonzero(ck.got != y))
+    return out
+
+
+def cpu_baseline(blocks, torch, rows: int = 192, checks=()):
+    """The oracle timed on `rows` token rows of the headline block, its
+    outputs compared with the GPU's; then the other legs' parity samples."""
     cases = blocks[0].cases
     import oracle
     oracle.build()
-    t_pack = time.perf_counter()
     ops, secs, outs = oracle_sample(cases, range(0, rows))
     # the GPU's outputs for the same rows of layer 0 (last written by the
     # e2e loop, which ran layer 0's block at least once)
@@ -652,12 +818,12 @@ def cpu_baseline(blocks, torch, rows: int = 192):
         got = blocks[0].y[j][:rows].cpu().numpy()
         checked += y.size
         mism += int(np.count_nonzero(got != y))
-    _ = t_pack
-    return {"value": round(ops / secs / 1e12, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
+    base = {"value": round(ops / secs / 1e12, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
             "sample": f"rows 0..{rows - 1} of all 7 linears of layer 0 (+ residual): "
                       f"{ops / 1e9:.1f} GOP of the {block_ops(PREFILL_M) / 1e9:.1f} GOP block",
             "seconds": round(secs, 2),
             "parity_sample": {"outputs": checked, "mismatches": mism}}
+    return base, run_checks(checks)
 
 
 def run_reference(args, dist: Dist):
@@ -722,9 +888,12 @@ def main():
 
     pre = run_prefill(mq, torch, dist, args.steps, args.warmup)
     decode = run_decode(mq, torch)
-    asym_pre = run_asym_prefill(mq, torch)
+    asym_pre, checks = run_asym_prefill(mq, torch)
     asym_dec = run_decode(mq, torch, asym=True, ms=(1, 16))
-    a16 = run_a16(mq, torch)
+    a16, more = run_a16(mq, torch)
+    checks += more
+    attention, more = run_attention(mq, torch)
+    checks += more
     glue = run_glue(mq, torch)
     wpipe = run_weight_pipeline(mq, torch)
     peaks = measured_peaks()
@@ -775,12 +944,19 @@ def main():
         "a16": {"activations": "int16 in and out", "ops": "2 M K N per block", **a16,
                 "w8a8_us_per_block": round(pre["total_ms"] / args.steps * 1e3, 2),
                 "w4a8_m1_stream_us": decode["m1"]["stream_us"]},
+        "attention_w8a8_t1024": {**attention,
+                                 "frac_hbm": round(attention["gbs"] / hbm, 3)},
         "boundary_quantizers": {"unit": "GB/s of input + output bytes", **glue},
         "weight_pipeline": {"what": "fold of eq. 1 + quantize + pack + colsum, 7 linears, "
                                     "176 MB of f32 weights", **wpipe},
     }
     if rank == 0 and world == 1:
-        line["cpu_baseline"] = cpu_baseline(pre["blocks"], torch)
+        line["cpu_baseline"], parity = cpu_baseline(pre["blocks"], torch, checks=checks)
+        for leg, r in parity.items():
+            node = line
+            for key in leg.split("."):
+                node = node[key]
+            node["parity_sample"] = r
     if rank == 0:
         print(json.dumps(line), flush=True)
     dist.close()

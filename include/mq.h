@@ -251,11 +251,11 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
  * quantizer of the paper's main W8A8 / W4A8 runs (Sec. 4.2 eqs. 2-4 applied
  * to weights, Sec. 5.1; a per-tensor zero point is the case of equal zw[n]):
  *   acc[m][n] = sum_k (x[m][k] - zx) * (w[n][k] - zw[n])
- *             = sum_k x w - zx colsum[n] - zw[n] rowsum(x)[m] + K zx zw[n]
+ *             = sum_k x (w - zw[n]) - zx (colsum[n] - K zw[n])
  * zw[n] must lie in the weight code range ([-128, 127] for bits 8, [-8, 7]
  * for bits 4), and with int8 weights K <= MQ_MAX_K_ASYM8 (so that
- * |acc| <= 255 * 255 * K stays below 2^31).  Descriptors with M > 16 and zw
- * need workspace for rowsum(x): see mq_workspace_size_batch.
+ * |acc| <= 255 * 255 * K stays below 2^31).  No workspace beyond that of the
+ * symmetric case: the weights are widened to w - zw[n] on the fly.
  *
  *   descs     : host array of `count` descriptors (1 <= count <= MQ_MAX_BATCH)
  *   workspace : device, ws_bytes >= mq_workspace_size_batch(descs, count)
@@ -273,6 +273,12 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
  * least that and a multiple of 16), so that a head's slice of a projection
  * output ([T][heads * d], one head's d columns) can serve as the weights
  * without a copy.
+ * Weights written on the device: the kernels read `packed` before waiting for
+ * the previous kernel in the stream (see mq_linear_w8a8).  A descriptor whose
+ * weights are produced by earlier work on the same stream (keys, or V^T from
+ * mq_transpose_i8, in attention) sets `wdynamic` nonzero; every launch that
+ * holds such a descriptor then reads all its weights after the previous
+ * kernel has completed.
  */
 typedef struct mq_linear_desc {
     const void *x;          /* int8 [M][ldx], or int16 with abits == 16 */
@@ -289,6 +295,7 @@ typedef struct mq_linear_desc {
     int32_t abits; /* activation and output bits: 8 (0 reads as 8) or 16, see mq_linear_w8a16 */
     int32_t obits; /* output bits: 0 (= abits), or 16 with abits 8: int16 y, see below */
     int32_t ldw;   /* bytes between weight rows; 0: packed rows (K * bits / 8) */
+    int32_t wdynamic; /* nonzero: packed is written by earlier work on the stream, see above */
 } mq_linear_desc;
 
 /* Largest K for int8 weights with a weight zero point: 255 * 255 * K < 2^31. */
@@ -297,17 +304,15 @@ typedef struct mq_linear_desc {
 /*
  * Device workspace bytes one mq_linear_batch call over `descs` needs: the
  * decode workspace (see mq_workspace_size) if any descriptor has
- * 1 <= M <= 16 (abits 8) or 1 <= 2M <= 16 (abits 16); plus 4*M bytes
- * (rounded up to 16) for every distinct input (x, M, K, ldx) of the
- * descriptors with M > 16 and a weight zero point, which holds rowsum(x) of
- * its tokens; plus 2*M*K bytes (rounded up to 128) for every distinct input
- * of the descriptors with abits 16 and 2M > 16, which holds its two int8 planes (both
- * filled by the call; descriptors reading the same input, e.g. q/k/v/gate/up
+ * 1 <= M <= 16 (abits 8) or 1 <= 2M <= 16 (abits 16); plus 2*M*K bytes
+ * (rounded up to 128) for every distinct input (x, M, K, ldx) of the
+ * descriptors with abits 16 and 2M > 16, which holds its two int8 planes
+ * (filled by the call; descriptors reading the same input, e.g. q/k/v/gate/up
  * of one block, share them).  0 when none applies.  The decode region (the
  * first mq_workspace_size bytes, when present) follows the contract of
  * mq_workspace_size: zero-filled before first use and left zero by every
- * call that completes; the rowsum and plane regions are scratch, overwritten
- * by each call.
+ * call that completes; the plane regions are scratch, overwritten by each
+ * call.
  * Errors: MQ_ERR_INVALID_ARG (null pointers, count out of range, bad bits or
  * abits).
  */

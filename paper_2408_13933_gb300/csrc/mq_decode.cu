@@ -90,6 +90,7 @@ struct Params {
     int total_stages;
     int2 *ws;            // [gridDim.x][UNIT_ROWS][16] {partial sum, epoch} (zero between calls)
     uint32_t epoch;      // nonzero, different for every launch
+    int pre_w;           // 1: load weights before griddep_wait (all constant)
     int *status;
 };
 
@@ -510,10 +511,11 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                     prefetch_tensormap(&P.tmap_x[i]);
                 }
             constexpr int XBOXES = C::KSTAGE / 128;  // x boxes per stage (int4: 2, int8: 1)
-            // Packed weights are constant inputs: the weight boxes of the first
-            // ring stages are requested before waiting for the previous grid
-            // in the stream; activations only after it.
-            const int npre = s_end - s_begin < STAGES ? s_end - s_begin : STAGES;
+            // Packed weights are constant inputs (unless a problem says they are
+            // written by earlier work, pre_w == 0): the weight boxes of the
+            // first ring stages are requested before waiting for the previous
+            // grid in the stream; activations only after it.
+            const int npre = !P.pre_w ? 0 : s_end - s_begin < STAGES ? s_end - s_begin : STAGES;
             int pi = 0;
             for (int i = 0; i < npre; ++i) {
                 const int gs = s_begin + i;
@@ -830,10 +832,12 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
     for (int begin = 0; begin < count; begin += DECODE_MAX_PROBLEMS) {
         const int n = count - begin < DECODE_MAX_PROBLEMS ? count - begin : DECODE_MAX_PROBLEMS;
         Params P{};
+        P.pre_w = 1;
         long long stages = 0;
         for (int i = 0; i < n; ++i) {
             Problem &q = P.p[i];
             q = probs[begin + i];
+            if (q.wdynamic) P.pre_w = 0;
             const int nst = q.K > 0 ? (q.K + C::KSTAGE - 1) / C::KSTAGE : 1;
             q.tile_begin = (int)stages;
             q.tiles_m = nst;

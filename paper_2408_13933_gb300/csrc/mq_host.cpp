@@ -53,7 +53,6 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     out.shift = d.shift;
     out.residual = d.residual;
     out.zw = d.zw;
-    out.rowsum = nullptr;
     out.y = static_cast<int8_t *>(d.y);
     out.M = ab == 8 ? d.M : 2 * d.M;  // 16 bits: rows of the plane matrix
     out.N = d.N;
@@ -66,6 +65,7 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     out.a16 = ab == 16;
     out.o16 = ab == 8 && ob == 16;
     out.ldw = d.ldw > 0 ? d.ldw : (int32_t)wrow;
+    out.wdynamic = d.wdynamic != 0;
     out.tile_begin = 0;
     out.tiles_m = 0;
     return MQ_OK;
@@ -82,14 +82,11 @@ bool is_decode(const mq_linear_desc &d) {
 }
 
 // Workspace layout of one batch: the decode region first (if any decode
-// shape), then one rowsum(x) array per distinct input (x, M, K, ldx) of the
-// prefill descriptors with a weight zero point, then one [2M][K] int8 plane
-// matrix per distinct input of the 16-bit descriptors, each in order of
-// first use, with offsets relative to the end of the decode region.
+// shape), then one [2M][K] int8 plane matrix per distinct input (x, M, K,
+// ldx) of the 16-bit tensor-core descriptors, in order of first use, with
+// offsets relative to the end of the decode region.
 struct Plan {
     bool any_decode = false;
-    std::vector<mq::RowsumJob> rowsum;
-    std::vector<size_t> rowsum_off;
     std::vector<mq::SplitJob> split;
     std::vector<size_t> split_off;
     size_t bytes = 0;
@@ -109,18 +106,6 @@ Plan batch_plan(const mq_linear_desc *descs, int count) {
         const mq_linear_desc &d = descs[i];
         if (d.M <= 0 || d.N <= 0) continue;
         if (is_decode(d)) pl.any_decode = true;
-        if (d.K <= 0) continue;
-        if (abits_of(d) == 8 && d.zw && !is_decode(d) &&
-            find_job(pl.rowsum, d.x, d.M, d.K, d.ldx) < 0) {
-            mq::RowsumJob j{};
-            j.x = static_cast<const int8_t *>(d.x);
-            j.M = d.M;
-            j.K = d.K;
-            j.ldx = d.ldx;
-            pl.rowsum.push_back(j);
-            pl.rowsum_off.push_back(off);
-            off += align16(4 * (size_t)d.M);
-        }
     }
     for (int i = 0; i < count; ++i) {
         const mq_linear_desc &d = descs[i];
@@ -150,15 +135,12 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         const int rc = check_desc(descs[i], probs[i]);
         if (rc != MQ_OK) return rc;
     }
-    // the decode kernel combines split 64-row units in the workspace; prefill
-    // descriptors with a weight zero point read rowsum(x) from there, 16-bit
-    // descriptors their int8 planes
+    // the decode kernel combines split 64-row units in the workspace, 16-bit
+    // tensor-core descriptors read their int8 planes from there
     Plan pl = batch_plan(descs, count);
     if (pl.bytes > 0 && (!workspace || ws_bytes < pl.bytes || !aligned16(workspace)))
         return MQ_ERR_WORKSPACE;
     uint8_t *region = static_cast<uint8_t *>(workspace) + (pl.any_decode ? mq::DECODE_WS_BYTES : 0);
-    for (size_t i = 0; i < pl.rowsum.size(); ++i)
-        pl.rowsum[i].out = reinterpret_cast<int32_t *>(region + pl.rowsum_off[i]);
     for (size_t i = 0; i < pl.split.size(); ++i)
         pl.split[i].out = reinterpret_cast<int8_t *>(region + pl.split_off[i]);
     // kernel families: prefill by activation / output width, decode by weight
@@ -168,10 +150,6 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         mq::Problem &p = probs[i];
         const mq_linear_desc &d = descs[i];
         if (p.M == 0 || p.N == 0) continue;  // nothing to compute or write
-        if (p.K > 0 && p.zw && !p.a16 && !is_decode(d)) {
-            const int j = find_job(pl.rowsum, d.x, d.M, d.K, d.ldx);
-            p.rowsum = pl.rowsum[j].out;
-        }
         if (p.K > 0 && p.a16) {
             if (is_decode(d)) {  // int16 codes, read by the decode kernel's TMA as they are
                 p.x = static_cast<const int8_t *>(d.x);
@@ -187,8 +165,7 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
             pre[mode].push_back(p);
     }
     int rc = MQ_OK;
-    if (!pl.rowsum.empty()) rc = mq::launch_rowsum(pl.rowsum.data(), (int)pl.rowsum.size(), stream);
-    if (rc == MQ_OK && !pl.split.empty())
+    if (!pl.split.empty())
         rc = mq::launch_split16(pl.split.data(), (int)pl.split.size(), stream);
     for (int mode = 0; mode < 3; ++mode)
         if (rc == MQ_OK && !pre[mode].empty())

@@ -21,7 +21,6 @@ struct Problem {
     const int32_t *shift;
     const int8_t *residual;
     const int32_t *zw;      // per-channel weight zero point, or null
-    const int32_t *rowsum;  // prefill with zw: rowsum(x) [M] in the workspace
     int8_t *y;
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;
@@ -35,6 +34,7 @@ struct Problem {
     int32_t a16;
     int32_t o16;         // 8-bit inputs, int16 output y [M][ldy] (requantized to 16 bits)
     int32_t ldw;         // bytes between weight rows
+    int32_t wdynamic;    // weights written by earlier work in the stream: read after the wait
     int32_t tile_begin;  // first global tile / block index of this problem
     int32_t tiles_m;     // prefill: number of 128-row tiles
 };
@@ -65,8 +65,7 @@ int launch_prefill(const Problem *probs, int count, void *stream);
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream);
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
                 int *status, void *stream);
-// One distinct input of a batch whose rowsum(x)[m] = sum_k x[m][k] a prefill
-// problem with a weight zero point needs (problems sharing x share the job).
+// One row-sum job: out[m] = sum_k x[m][k] (mq_row_sums).
 struct RowsumJob {
     const int8_t *x;
     int32_t *out;  // [M] in the workspace

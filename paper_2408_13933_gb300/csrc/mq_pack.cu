@@ -105,8 +105,8 @@ struct Params {
 // is 16-byte aligned (the library's validation), so every load is a whole
 // uint4.  Launched with programmatic stream serialization: x may be the output
 // of the previous kernel in the stream, so nothing is read before
-// griddep_wait; the kernel that follows (the prefill) reads `out` only after
-// its own griddep_wait, i.e. after this grid has completed.
+// griddep_wait; a library kernel that follows reads `out` (a colsum) only
+// after its own griddep_wait, i.e. after this grid has completed.
 __global__ void __launch_bounds__(ROWS_PER_BLOCK * 32) rowsum_kernel(const __grid_constant__ Params P) {
     griddep_wait();
     griddep_launch_dependents();

@@ -88,6 +88,10 @@ constexpr uint32_t F_COL0 = 0;     // F[b] at F_COL0 + 128 b
 constexpr uint32_t A_COL0 = 256;   // A stage s at A_COL0 + 64 s
 constexpr int KB_PER_CHUNK_I8 = 1024 / KS;   // |partial| <= 1024 * 2^14 = 2^24
 constexpr int KB_PER_CHUNK_I4 = 16384 / KS;  // |partial| <= 16384 * 2^10 = 2^24
+// with a weight zero point the widened weights are w - zw: |x (w - zw)| <=
+// 128 * 255 (int8) or 128 * 15 (int4)
+constexpr int KB_PER_CHUNK_I8Z = 512 / KS;   // |partial| <= 512 * 32640 < 2^24
+constexpr int KB_PER_CHUNK_I4Z = 8192 / KS;  // |partial| <= 8192 * 1920 < 2^24
 constexpr int MAX_SCHED = 4096;    // tile table entries (host LPT schedule)
 constexpr int MAX_PAIRS = 128;
 
@@ -99,6 +103,7 @@ struct Params {
     int total_tiles;
     int npairs;
     int use_table;                       // 1: sched / pair_begin, 0: round-robin
+    int pre_w;                           // 1: load weights before griddep_wait (all constant)
     uint16_t pair_begin[MAX_PAIRS + 1];
     uint16_t sched[MAX_SCHED];
     int *status;
@@ -138,7 +143,8 @@ __device__ __forceinline__ Tile tile_at(const Params &P, int tile) {
     t.tt = local % p.tiles_m;
     t.ct = local / p.tiles_m;
     t.nkb = (p.K + KS - 1) / KS;
-    t.kpc = p.bits == 8 ? KB_PER_CHUNK_I8 : KB_PER_CHUNK_I4;
+    t.kpc = p.bits == 8 ? (p.zw ? KB_PER_CHUNK_I8Z : KB_PER_CHUNK_I8)
+                        : (p.zw ? KB_PER_CHUNK_I4Z : KB_PER_CHUNK_I4);
     return t;
 }
 
@@ -217,6 +223,25 @@ __device__ __forceinline__ void store_channel(const uint32_t (&acc)[64], int32_t
     }
 }
 
+// The 16-bit output of 8-bit inputs: the same 64 outputs requantized to int16
+// (no residual).  The accumulator fits int32, so for shifts >= 33 the int8
+// path's multiply-high form gives floor((acc M0 + 2^(sh-1)) / 2^sh) exactly
+// (|q| <= 2^30, so q + zy cannot overflow); other shifts take mq_requant16.
+template <bool FULL, bool FAST>
+__device__ __forceinline__ void store_channel16(const uint32_t (&acc)[64], int32_t corr,
+                                                int32_t m0, int32_t sh, int32_t zy, int16_t *yp,
+                                                size_t ldy, int ntok) {
+    const int32_t rnd = FAST ? (1 << (sh - 33)) : 0;
+    const int32_t rs = FAST ? sh - 32 : 0;
+#pragma unroll
+    for (int j = 0; j < 64; ++j, yp += ldy)
+        if (FULL || j < ntok) {
+            const int32_t a = (int32_t)(acc[j] - (uint32_t)corr);
+            *yp = (int16_t)(FAST ? min(32767, max(-32768, ((__mulhi(a, m0) + rnd) >> rs) + zy))
+                                 : mq_requant16((int64_t)a, m0, sh, zy));
+        }
+}
+
 // Barrier scopes: arrivals from the other CTA are releases at cluster scope
 // (st.async complete_tx, mbarrier.arrive.release.cluster, multicast commits),
 // so the data they publish is visible cluster-wide before the phase can
@@ -224,7 +249,11 @@ __device__ __forceinline__ void store_channel(const uint32_t (&acc)[64], int32_t
 // A16: every problem has 16-bit activations (Problem::a16): its x is the
 // plane matrix, and the epilogue combines row pairs and stores int16.
 // O16: every problem has 8-bit inputs and a 16-bit output (Problem::o16).
-template <bool A16, bool O16>
+// ZW: problems may have a weight zero point, folded into the widening of the
+// weights (w - zw); without it the widening offsets are immediate constants
+// (a register offset in the converters' loop costs about 4% on symmetric
+// blocks).
+template <bool A16, bool O16, bool ZW>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     prefill_kernel(const __grid_constant__ Params P) {
     extern __shared__ uint8_t smem_raw[];
@@ -270,11 +299,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 prefetch_tensormap(&P.tmap_x[i]);
                 prefetch_tensormap(&P.tmap_w[i]);
             }
-            // Packed weights are constant inputs: the weight boxes of the first
+            // Packed weights are constant inputs (unless a problem says they are
+            // written by earlier work, pre_w == 0): the weight boxes of the first
             // S8 stages are requested before waiting for the previous grid in
             // the stream; activations only after it.
             uint32_t npre = 0;
-            {
+            if (P.pre_w) {
                 int tile;
                 for (int ti = 0; npre < (uint32_t)S8 && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
                     const Tile t = tile_at(P, tile);
@@ -398,6 +428,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             b_dst[i][1] = base + (uint32_t)((second ^ (row & 7)) << 4);
         }
         const bool swap_b = (gt & 4) != 0;
+        if constexpr (ZW) griddep_wait();  // the weight zero points are read below
         const uint32_t leader_op_full = cluster_addr(&s.op_full[0], 0);
         const uint32_t leader_sink = cluster_addr(&s.sink[warp - CONV_WARP0], 0);
         uint32_t it = 0;
@@ -406,6 +437,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
             const Tile t = tile_at(P, tile);
             const bool i4 = P.p[t.pi].bits == 4;
+            // weight row arow widens to w - zw (zw = 0 for symmetric weights):
+            // the MMA then sums x (w - zw) and the epilogue needs no rowsum(x)
+            uint32_t aoff = i4 ? 0xD480E408u : F16X2_1152;
+            if constexpr (ZW) {
+                const int32_t *zwp = P.p[t.pi].zw;
+                const int wch = t.ct * TM + (int)rank * CM + arow;
+                const int32_t zwr = (zwp && wch < P.p[t.pi].N) ? __ldg(zwp + wch) : 0;
+                aoff = i4 ? f16x2_i4_offset(zwr) : f16x2_i8_offset(zwr);
+            }
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                 if ((int)(it & 1) != grp) continue;
                 const int s8 = it % S8, sf = it % SF;
@@ -427,10 +467,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         for (int i = 0; i < 4; ++i) v[i] = lds16(sa + a8_src[4 * hk + i]);
 #pragma unroll
                         for (int i = 0; i < 4; ++i) {
-                            i8x4_to_f16x4(v[i].x, a[8 * i + 0], a[8 * i + 1]);
-                            i8x4_to_f16x4(v[i].y, a[8 * i + 2], a[8 * i + 3]);
-                            i8x4_to_f16x4(v[i].z, a[8 * i + 4], a[8 * i + 5]);
-                            i8x4_to_f16x4(v[i].w, a[8 * i + 6], a[8 * i + 7]);
+                            i8x4_to_f16x4(v[i].x, a[8 * i + 0], a[8 * i + 1], aoff);
+                            i8x4_to_f16x4(v[i].y, a[8 * i + 2], a[8 * i + 3], aoff);
+                            i8x4_to_f16x4(v[i].z, a[8 * i + 4], a[8 * i + 5], aoff);
+                            i8x4_to_f16x4(v[i].w, a[8 * i + 6], a[8 * i + 7], aoff);
                         }
                     } else {
                         uint4 v[2];
@@ -442,7 +482,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 #pragma unroll
                             for (int j = 0; j < 4; ++j) {
                                 uint32_t o[4];
-                                i4x8_to_f16x8(w4[j], o);
+                                i4x8_to_f16x8(w4[j], o, aoff);
 #pragma unroll
                                 for (int e = 0; e < 4; ++e) a[16 * i + 4 * j + e] = o[e];
                             }
@@ -500,7 +540,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const int ch = t.ct * TM + (int)rank * CM + quad * 32 + lane;
             const bool ch_in = ch < p.N;
             const int32_t zw = (ch_in && p.zw) ? __ldg(p.zw + ch) : 0;
-            // sum((x - zx)(w - zw)) = sum(x w) - zx colsum - zw rowsum(x) + K zx zw
+            // the chunks sum x (w - zw) (the converters widen w - zw), so
+            // sum((x - zx)(w - zw)) = that - zx (colsum - K zw)
             const int32_t corr =
                 ch_in ? (int32_t)((uint32_t)(p.zx * __ldg(p.colsum + ch)) -
                                   (uint32_t)p.K * (uint32_t)(p.zx * zw))
@@ -567,33 +608,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     }
                 continue;
             }
-            if (p.zw && ntok > 0) {
-                // the weight zero point's term: - zw rowsum(x)[token]
-                const int32_t *rs = p.rowsum + tok0;
-                if (ntok == 64) {
-#pragma unroll
-                    for (int j = 0; j < 64; j += 4) {
-                        const int4 v = __ldg(reinterpret_cast<const int4 *>(rs + j));
-                        acc[j + 0] -= (uint32_t)(zw * v.x);
-                        acc[j + 1] -= (uint32_t)(zw * v.y);
-                        acc[j + 2] -= (uint32_t)(zw * v.z);
-                        acc[j + 3] -= (uint32_t)(zw * v.w);
-                    }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 64; ++j)
-                        if (j < ntok) acc[j] -= (uint32_t)(zw * __ldg(rs + j));
-                }
-            }
             const size_t ldy = (size_t)e.ldy;
             if constexpr (O16) {
-                // the same sum, requantized to 16 bits (no residual)
                 int16_t *yp16 = reinterpret_cast<int16_t *>(e.y) + (size_t)tok0 * ldy + ch;
-#pragma unroll
-                for (int j = 0; j < 64; ++j)
-                    if (j < ntok)
-                        yp16[(size_t)j * ldy] = (int16_t)mq_requant16(
-                            (int64_t)(int32_t)(acc[j] - (uint32_t)corr), m0, sh, e.zy);
+                if (ntok == 64 && sh >= 33)
+                    store_channel16<true, true>(acc, corr, m0, sh, e.zy, yp16, ldy, 64);
+                else
+                    store_channel16<false, false>(acc, corr, m0, sh, e.zy, yp16, ldy, ntok);
                 continue;
             }
             int8_t *yp = e.y + (size_t)tok0 * ldy + ch;
@@ -661,7 +682,8 @@ int max_pairs(int dev) {
     cfg.blockDim = dim3(THREADS, 1, 1);
     cfg.dynamicSmemBytes = SMEM_BYTES;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, prefill_kernel<false, false>, &cfg) == cudaSuccess &&
+    if (cudaOccupancyMaxActiveClusters(&clusters, prefill_kernel<false, false, false>, &cfg) ==
+            cudaSuccess &&
         clusters > 0 && clusters < n)
         n = clusters;
     if (n > MAX_PAIRS) n = MAX_PAIRS;
@@ -711,27 +733,30 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
     if (attr_done != dev) {
-        if (cudaFuncSetAttribute(prefill_kernel<false, false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)SMEM_BYTES) != cudaSuccess ||
-            cudaFuncSetAttribute(prefill_kernel<true, false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)SMEM_BYTES) != cudaSuccess ||
-            cudaFuncSetAttribute(prefill_kernel<false, true>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)SMEM_BYTES) != cudaSuccess)
+        const int smem = (int)SMEM_BYTES;
+        const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
+        if (cudaFuncSetAttribute(prefill_kernel<false, false, false>, attr, smem) != cudaSuccess ||
+            cudaFuncSetAttribute(prefill_kernel<false, false, true>, attr, smem) != cudaSuccess ||
+            cudaFuncSetAttribute(prefill_kernel<true, false, false>, attr, smem) != cudaSuccess ||
+            cudaFuncSetAttribute(prefill_kernel<false, true, true>, attr, smem) != cudaSuccess)
             return MQ_ERR_CUDA;
         attr_done = dev;
     }
     if (count <= 0) return MQ_OK;
-    auto kern = probs[0].a16   ? prefill_kernel<true, false>
-                : probs[0].o16 ? prefill_kernel<false, true>
-                               : prefill_kernel<false, false>;
     const int pairs_max = max_pairs(dev);
     if (pairs_max < 1) return MQ_ERR_CUDA;
     for (int begin = 0; begin < count; begin += PREFILL_MAX_PROBLEMS) {
         const int n = count - begin < PREFILL_MAX_PROBLEMS ? count - begin : PREFILL_MAX_PROBLEMS;
+        bool any_zw = false;
+        for (int i = begin; i < begin + n; ++i) any_zw = any_zw || probs[i].zw != nullptr;
+        // 16-bit outputs always take the zero-point variant (their time is the
+        // epilogue's, not the widening's)
+        auto kern = probs[0].a16   ? prefill_kernel<true, false, false>
+                    : probs[0].o16 ? prefill_kernel<false, true, true>
+                    : any_zw       ? prefill_kernel<false, false, true>
+                                   : prefill_kernel<false, false, false>;
         Params P{};
+        P.pre_w = 1;
         long long tiles = 0;
         // longest K first (round-robin order; the table orders by work itself)
         int order[PREFILL_MAX_PROBLEMS];
@@ -745,6 +770,7 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
         for (int i = 0; i < n; ++i) {
             Problem &q = P.p[i];
             q = probs[order[i]];
+            if (q.wdynamic) P.pre_w = 0;
             q.tiles_m = (q.M + TN - 1) / TN;
             q.tile_begin = (int)tiles;
             tiles += (long long)q.tiles_m * ((q.N + TM - 1) / TM);

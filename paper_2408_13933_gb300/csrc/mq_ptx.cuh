@@ -357,10 +357,20 @@ constexpr uint32_t F16X2_1152 = 0x64806480u;  // (1152, 1152)
 
 // Four int8 (one 32-bit word, byte i = element i) -> two f16x2 words
 // (elements 0,1) and (2,3).
-__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi,
+                                              uint32_t off = F16X2_1152) {
     const uint32_t u = w ^ 0x80808080u;
-    lo = hsub2(prmt(u, 0x64646464u, 0x4140u), F16X2_1152);
-    hi = hsub2(prmt(u, 0x64646464u, 0x4342u), F16X2_1152);
+    lo = hsub2(prmt(u, 0x64646464u, 0x4140u), off);
+    hi = hsub2(prmt(u, 0x64646464u, 0x4342u), off);
+}
+
+// The offset of i8x4_to_f16x4 that also subtracts a weight zero point z in
+// [-128, 127]: (1152 + z) in both halves, f16 bits 0x6480 + z (1024 <= 1152 +
+// z < 2048, where f16 steps by 1).  (1024 + u) - (1152 + z) = w - z is exact:
+// both operands and the result (|w - z| <= 255) are f16 integers.
+__device__ __forceinline__ uint32_t f16x2_i8_offset(int32_t z) {
+    const uint32_t c = (uint32_t)(0x6480 + z);
+    return (c << 16) | c;
 }
 
 // Eight int4 (one word, nibble p = element p, two's complement) -> four f16x2
@@ -368,14 +378,22 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
 // 0 and 2; the low nibble of byte 0 becomes 1024 + (e + 8) in the low half,
 // the high nibble of byte 2 becomes 1024 + 16 (e + 8) in the high half; one
 // f16x2 FMA with per-half scale (1, 1/16) and offset (-1032, -72) gives e.
-__device__ __forceinline__ void i4x8_to_f16x8(uint32_t w, uint32_t (&o)[4]) {
+__device__ __forceinline__ void i4x8_to_f16x8(uint32_t w, uint32_t (&o)[4],
+                                              uint32_t offset = 0xD480E408u /* (-1032, -72) */) {
     const uint32_t scale = 0x2C003C00u;   // (1.0, 1/16)
-    const uint32_t offset = 0xD480E408u;  // (-1032, -72)
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const uint32_t t = prmt(w, 0u, 0x1111u * (uint32_t)i);
         o[i] = hfma2(lop3_sel_xor(t, 0x00F0000Fu, 0x64806408u), scale, offset);
     }
+}
+
+// The offset of i4x8_to_f16x8 that also subtracts a weight zero point z in
+// [-8, 7]: (-1032 - z, -72 - z); f16 bits 0xE408 + z (1024 < 1032 + z < 2048,
+// step 1) and 0xD480 + 16 z (64 <= 72 + z < 128, step 1/16).  Each half is one
+// FMA whose exact value e - z (|e - z| <= 15) is an f16 integer.
+__device__ __forceinline__ uint32_t f16x2_i4_offset(int32_t z) {
+    return (((uint32_t)(0xD480 + 16 * z) & 0xFFFFu) << 16) | ((uint32_t)(0xE408 + z) & 0xFFFFu);
 }
 
 // Requantize one accumulator (acc = sum(x w) - zx colsum, int32):

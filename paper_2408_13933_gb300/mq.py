@@ -53,7 +53,8 @@ class LinearDesc(ctypes.Structure):
     _fields_ = [("x", _vp), ("packed", _vp), ("colsum", _vp), ("M0", _vp), ("shift", _vp),
                 ("residual", _vp), ("zw", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
                 ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32),
-                ("abits", _i32), ("obits", _i32), ("ldw", _i32)]
+                ("abits", _i32), ("obits", _i32), ("ldw", _i32),
+                ("wdynamic", _i32)]
 
 
 lib.mq_status_string.argtypes = [_int]
@@ -303,11 +304,12 @@ def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, 
 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
               ldx=None, ldy=None, m=None, k=None, zw=None, abits=None, obits=None,
-              ldw: int = 0) -> LinearDesc:
+              ldw: int = 0, wdynamic: bool = False) -> LinearDesc:
     """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights;
     abits 16 (default: 16 for an int16 x) gives int16 activations and outputs;
     obits 16 with int8 x (default: 16 for an int16 y) an int16 output; `ldw`
-    the bytes between weight rows (0: packed)."""
+    the bytes between weight rows (0: packed); `wdynamic` marks weights written
+    by earlier work on the stream (read only after it completes)."""
     d = LinearDesc()
     if abits is None:
         abits = 16 if getattr(x, "element_size", lambda: 1)() == 2 else 8
@@ -316,6 +318,7 @@ def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
     d.abits = int(abits)
     d.obits = int(obits)
     d.ldw = int(ldw)
+    d.wdynamic = int(bool(wdynamic))
     d.x, d.packed, d.colsum = _ptr(x), _ptr(packed), _ptr(colsum)
     d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
     d.zw = _ptr(zw)

@@ -425,3 +425,54 @@ def chain_stack(config: int, m: int, layers: int, shapes=TINYLLAMA_LINEARS, head
     wq, sw = quantize_per_channel_symmetric(wf, 8, inplace=True)
     head_case = LinearCase(name, np.zeros((0, k), np.int8), cur_z, cur_s, wq, sw, 8, sy, zy)
     return x0, sx0, zx0, out_layers, head_case
+
+
+@dataclass
+class AttentionOperands:
+    """The int8 operands of one layer's grouped-query attention matmuls: Q
+    [T][heads * d], K and V [T][kv_heads * d] (per-tensor asymmetric codes
+    with zero points zq, zk, zv) and P [heads][T][T], the codes of a causal
+    softmax output (scale 1/255, zero point -128)."""
+    q: np.ndarray
+    k: np.ndarray
+    v: np.ndarray
+    p: np.ndarray
+    zq: int
+    zk: int
+    zv: int
+    zp: int
+    heads: int
+    kv_heads: int
+    d: int
+
+
+ROLE_ATT_Q, ROLE_ATT_K, ROLE_ATT_V, ROLE_ATT_P = 10, 11, 12, 13
+
+
+def attention_operands(config: int, layer: int, t: int, heads: int = 32, kv_heads: int = 4,
+                       d: int = 64, logit_std: float = 2.0) -> AttentionOperands:
+    """Seeded stand-ins for the inputs of Q K^T and P V at T = t tokens.
+
+    Q, K, V: N(0, 1) activations (4 outlier channels x20) quantized per tensor
+    like every other activation here.  P: rows of softmax(N(0, logit_std)
+    logits) over keys s <= query t (the causal mask; masked keys get
+    probability 0), coded as clip(rint(255 p) - 128, -128, 127)."""
+    codes = []
+    for role, width in ((ROLE_ATT_Q, heads * d), (ROLE_ATT_K, kv_heads * d),
+                        (ROLE_ATT_V, kv_heads * d)):
+        xf = float_activations(rng_for(config, layer, role, ROLE_X), t, width,
+                               orng=rng_for(config, layer, role, ROLE_OUTLIER))
+        q, _, z = quantize_per_tensor(xf)
+        codes.append((q, z))
+    rng = rng_for(config, layer, ROLE_ATT_P, ROLE_X)
+    p = np.empty((heads, t, t), np.int8)
+    future = np.triu(np.ones((t, t), bool), 1)
+    for h in range(heads):
+        logits = rng.standard_normal((t, t), dtype=np.float32) * np.float32(logit_std)
+        logits[future] = -np.inf
+        logits -= logits.max(axis=1, keepdims=True)
+        e = np.exp(logits)
+        e /= e.sum(axis=1, keepdims=True)
+        p[h] = rint_clip(e * np.float32(255.0) - np.float32(128.0), -128, 127).astype(np.int8)
+    (q, zq), (k, zk), (v, zv) = codes
+    return AttentionOperands(q, k, v, p, zq, zk, zv, -128, heads, kv_heads, d)

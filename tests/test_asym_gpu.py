@@ -104,6 +104,17 @@ def test_asym_extreme_codes(m, extreme, bits):
     assert_equal_int8(run([c])[0], c.want(), f"asym extreme m={m} {extreme} bits={bits}")
 
 
+@pytest.mark.parametrize("extreme", ["min", "max", "mixed"])
+def test_asym_int4_extreme_codes_across_chunks(extreme):
+    # int4 weights with zero points at the range ends, codes at the ends, K =
+    # 20480: the tensor-core kernel's exact-f32 chunks of x (w - zw) (8192 k,
+    # |x (w - zw)| <= 128 * 15) are full twice and ragged once
+    n = 72
+    zw = np.where(np.arange(n) % 2 == 0, -8, 7).astype(np.int32)
+    c = AsymCase(19, 130, 20480, n, 4, extreme, zw=zw)
+    assert_equal_int8(run([c])[0], c.want(), f"asym int4 long K {extreme}")
+
+
 def test_asym_int8_at_k_limit():
     # K = MQ_MAX_K_ASYM8 with int8 weights: |acc| up to 255 * 255 * K < 2^31
     k = mq().MQ_MAX_K_ASYM8
@@ -120,7 +131,8 @@ def test_asym_residual(m):
 
 def test_asym_batch_mixes_kernels_and_symmetric():
     # decode and prefill, asymmetric and symmetric problems in one call: the
-    # workspace holds the decode region and two rowsum regions
+    # workspace holds the decode region only (the tensor-core kernel folds
+    # the weight zero point into the widened weights)
     a = AsymCase(51, 130, 512, 200, 8)
     b = AsymCase(52, 4, 1024, 96, 4)
     c = AsymCase(53, 70, 256, 64, 4)
@@ -131,7 +143,7 @@ def test_asym_batch_mixes_kernels_and_symmetric():
     descs[3].zw = None  # symmetric problem in the same batch
     need = lib.workspace_size_batch(descs)
     dec = lib.workspace_size(4, 96, 1024, 4)
-    assert need == dec + 16 * ((4 * 130 + 15) // 16) + 16 * ((4 * 70 + 15) // 16)
+    assert need == dec
     torch = torch_cuda()
     ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
     assert lib.linear_batch(descs, workspace=ws, ws_bytes=need) == 0
@@ -141,9 +153,9 @@ def test_asym_batch_mixes_kernels_and_symmetric():
         assert_equal_int8(x.y.cpu().numpy(), x.want(), f"batch {x.c.name}")
 
 
-def test_asym_shared_input_one_rowsum():
-    # q/k/v/gate/up-like problems reading one input: one rowsum region for
-    # all of them, next to another input's region
+def test_asym_shared_input():
+    # q/k/v/gate/up-like problems reading one input (one asymmetric with zero
+    # points, one symmetric), next to another input: no workspace
     a = AsymCase(61, 96, 512, 128, 8)
     b = AsymCase(62, 96, 512, 64, 4, share=a)
     c = AsymCase(63, 96, 512, 200, 8, share=a)
@@ -154,9 +166,9 @@ def test_asym_shared_input_one_rowsum():
     descs = [x.desc() for x in cases]
     descs[3].zw = None
     need = lib.workspace_size_batch(descs)
-    assert need == 16 * ((4 * 96 + 15) // 16) + 16 * ((4 * 80 + 15) // 16)
+    assert need == 0
     torch = torch_cuda()
-    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(16, dtype=torch.uint8, device="cuda")
     assert lib.linear_batch(descs, workspace=ws, ws_bytes=need) == 0
     torch.cuda.synchronize()
     assert lib.check_device_status() == 0

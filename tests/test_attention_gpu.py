@@ -123,68 +123,73 @@ def test_row_sums_and_transpose():
 @pytest.mark.parametrize("t_q", [96, 1])
 def test_grouped_query_attention_matmuls(t_q):
     # 4 query heads over 2 KV heads, head dim 64, T = 96 keys; t_q query tokens
-    # (96: prefill kernel, 1: decode kernel for the scores)
+    # (96: prefill kernel, 1: decode kernel).  Three rounds of new K and V
+    # rewrite the same V^T and row-sum buffers, all enqueued back to back on
+    # one stream (programmatic dependent launches from the producers into the
+    # batched calls, weights marked as written on the device), checked after.
     torch = torch_cuda()
     lib = mq()
     rng = np.random.default_rng(11 + t_q)
-    T, H, G, D = 96, 4, 2, 64
+    T, H, G, D, R = 96, 4, 2, 64, 3
+    rep = H // G
     i8 = lambda *s: rng.integers(-128, 128, size=s, dtype=np.int16).astype(np.int8)
-    q, kk, v = i8(t_q, H * D), i8(T, G * D), i8(T, G * D)
-    zq, zk, zv = -5, 12, -20
-    qd, kd, vd = upload(q), upload(kk), upload(v)
-    keep = [qd, kd, vd]
-    # ---- scores S_h = Q_h K_g^T, int16 (obits 16), keys as weights through ldw
-    m0s = np.full(T, 1 << 30, np.int32)
-    shs = np.full(T, 33, np.int32)          # scale 1/8
-    zys = 100
-    m0d, shd = upload(m0s), upload(shs)
-    zwk = upload(np.full(T, zk, np.int32))
-    keep += [m0d, shd, zwk]
-    descs, outs, colsums = [], [], []
-    for g in range(G):
-        colsums.append(lib.row_sums(kd[:, g * D:(g + 1) * D]))
-    keep += colsums
-    for h in range(H):
-        g = h // (H // G)
-        s = torch.full((t_q, T), 3, dtype=torch.int16, device="cuda")
-        outs.append(s)
-        descs.append(lib.make_desc(qd[:, h * D:(h + 1) * D], zq, kd[:, g * D:(g + 1) * D],
-                                   colsums[g], T, m0d, shd, zys, s, 8, zw=zwk, k=D,
-                                   ldx=H * D, ldw=G * D))
-    keep += outs
-    _run(descs, keep)
-    for h in range(H):
-        g = h // (H // G)
-        kg = np.ascontiguousarray(kk[:, g * D:(g + 1) * D])
-        opk, _ = oracle.pack(kg, 8)
-        want = oracle.linear_o16(np.ascontiguousarray(q[:, h * D:(h + 1) * D]), zq, opk, 8, T,
-                                 m0s, shs, zys, zw=np.full(T, zk, np.int32))
-        assert_equal(outs[h].cpu().numpy(), want, f"scores head {h}")
-    # ---- O_h = P_h V_g: P (the requantized softmax output) int8, V^T as weights
-    p = i8(H, t_q, T)
-    zp = 7
-    pd = upload(p)
-    keep.append(pd)
-    vts = [lib.transpose_i8(vd[:, g * D:(g + 1) * D]) for g in range(G)]
-    vcs = [lib.row_sums(vt) for vt in vts]
-    keep += vts + vcs
-    m0o = np.full(D, 1 << 30, np.int32)
-    sho = np.full(D, 40, np.int32)          # scale 2^-10
-    m0od, shod = upload(m0o), upload(sho)
-    zwv = upload(np.full(D, zv, np.int32))
-    keep += [m0od, shod, zwv]
-    descs, outs = [], []
-    for h in range(H):
-        g = h // (H // G)
-        o = torch.full((t_q, D), 9, dtype=torch.int8, device="cuda")
-        outs.append(o)
-        descs.append(lib.make_desc(pd[h], zp, vts[g], vcs[g], D, m0od, shod, -3, o, 8, zw=zwv))
-    keep += outs
-    _run(descs, keep)
-    for h in range(H):
-        g = h // (H // G)
-        vt = np.ascontiguousarray(v[:, g * D:(g + 1) * D].T)
-        opk, _ = oracle.pack(vt, 8)
-        want = oracle.linear(np.ascontiguousarray(p[h]), zp, opk, 8, D, m0o, sho, -3,
-                             zw=np.full(D, zv, np.int32))
-        assert_equal_int8(outs[h].cpu().numpy(), want, f"P V head {h}")
+    q = i8(t_q, H * D)
+    ks, vs, ps = [i8(T, G * D) for _ in range(R)], [i8(T, G * D) for _ in range(R)], \
+        [i8(H, t_q, T) for _ in range(R)]
+    zq, zk, zv, zp = -5, 12, -20, 7
+    qd = upload(q)
+    kds, vds, pds = [upload(a) for a in ks], [upload(a) for a in vs], [upload(a) for a in ps]
+    keep = [qd] + kds + vds + pds
+    m0s, shs, zys = np.full(T, 1 << 30, np.int32), np.full(T, 33, np.int32), 100  # scale 1/8
+    m0o, sho, zyo = np.full(D, 1 << 30, np.int32), np.full(D, 40, np.int32), -3   # 2^-10
+    dev = [upload(a) for a in (m0s, shs, np.full(T, zk, np.int32), m0o, sho,
+                               np.full(D, zv, np.int32))]
+    keep += dev
+    m0sd, shsd, zwk, m0od, shod, zwv = dev
+    colk = torch.empty((G, T), dtype=torch.int32, device="cuda")       # rewritten each round
+    vt = torch.empty((G, D, T), dtype=torch.int8, device="cuda")
+    colv = torch.empty((G, D), dtype=torch.int32, device="cuda")
+    scores = [torch.full((H, t_q, T), 3, dtype=torch.int16, device="cuda") for _ in range(R)]
+    outs = [torch.full((t_q, H * D), 9, dtype=torch.int8, device="cuda") for _ in range(R)]
+    keep += [colk, vt, colv] + scores + outs
+    arr_s, arr_o = [], []
+    for r in range(R):
+        ds = [lib.make_desc(qd[:, h * D:(h + 1) * D], zq, kds[r][:, (h // rep) * D:],
+                            colk[h // rep], T, m0sd, shsd, zys, scores[r][h], 8, zw=zwk, k=D,
+                            ldw=G * D, wdynamic=True) for h in range(H)]
+        do = [lib.make_desc(pds[r][h], zp, vt[h // rep], colv[h // rep], D, m0od, shod, zyo,
+                            outs[r][:, h * D:(h + 1) * D], 8, zw=zwv, wdynamic=True)
+              for h in range(H)]
+        arr_s.append((lib.LinearDesc * H)(*ds))
+        arr_o.append((lib.LinearDesc * H)(*do))
+    need = max(lib.workspace_size_batch(list(a)) for a in arr_s + arr_o)
+    ws = torch.zeros(max(need, 16), dtype=torch.uint8, device="cuda")
+    keep.append(ws)
+    torch.cuda.synchronize()
+    sp = torch.cuda.current_stream().cuda_stream
+    for r in range(R):
+        for g in range(G):
+            assert lib.lib.mq_row_sums(kds[r][:, g * D:].data_ptr(), T, D, G * D,
+                                       colk[g].data_ptr(), sp) == 0
+        assert lib.lib.mq_linear_batch(arr_s[r], H, ws.data_ptr(), need, sp) == 0
+        for g in range(G):
+            assert lib.lib.mq_transpose_i8(vds[r][:, g * D:].data_ptr(), T, D, G * D,
+                                           vt[g].data_ptr(), T, sp) == 0
+            assert lib.lib.mq_row_sums(vt[g].data_ptr(), D, T, T, colv[g].data_ptr(), sp) == 0
+        assert lib.lib.mq_linear_batch(arr_o[r], H, ws.data_ptr(), need, sp) == 0
+    torch.cuda.synchronize()
+    assert lib.check_device_status() == 0
+    for r in range(R):
+        for h in range(H):
+            g = h // rep
+            kg = np.ascontiguousarray(ks[r][:, g * D:(g + 1) * D])
+            opk, _ = oracle.pack(kg, 8)
+            want = oracle.linear_o16(np.ascontiguousarray(q[:, h * D:(h + 1) * D]), zq, opk, 8, T,
+                                     m0s, shs, zys, zw=np.full(T, zk, np.int32))
+            assert_equal(scores[r][h].cpu().numpy(), want, f"round {r} scores head {h}")
+            vtg = np.ascontiguousarray(vs[r][:, g * D:(g + 1) * D].T)
+            opk, _ = oracle.pack(vtg, 8)
+            want = oracle.linear(np.ascontiguousarray(ps[r][h]), zp, opk, 8, D, m0o, sho, zyo,
+                                 zw=np.full(D, zv, np.int32))
+            assert_equal_int8(outs[r][:, h * D:(h + 1) * D].cpu().numpy(), want,
+                              f"round {r} P V head {h}")

@@ -172,27 +172,18 @@ def test_asym_int8_k_limit_and_workspace(mq):
     bad = (mq.LinearDesc * 1)(_desc(mq, 64, k, 32, 8, True))
     assert mq.lib.mq_linear_batch(bad, 1, None, 0, None) == mq.MQ_ERR_K_OVERFLOW
     ok4 = _desc(mq, 64, k, 32, 4, True)
-    assert mq.workspace_size_batch([ok4]) == 4 * 64
-    # workspace of a batch: decode region + 16-byte-rounded rowsum regions of
-    # the asymmetric prefill descriptors; symmetric prefill needs none
+    # the tensor-core kernel folds the weight zero point into the widened
+    # weights: asymmetric prefill needs no workspace; decode shapes need the
+    # decode region whatever their weights
+    assert mq.workspace_size_batch([ok4]) == 0
     dec = mq.workspace_size(8, 32, 64, 4)
     assert mq.workspace_size_batch([_desc(mq, 100, 64, 32, 8, False)]) == 0
-    assert mq.workspace_size_batch([_desc(mq, 100, 64, 32, 8, True)]) == 400
+    assert mq.workspace_size_batch([_desc(mq, 100, 64, 32, 8, True)]) == 0
     assert mq.workspace_size_batch([_desc(mq, 101, 64, 32, 8, True),
-                                    _desc(mq, 8, 64, 32, 4, True)]) == dec + 416
+                                    _desc(mq, 8, 64, 32, 4, True)]) == dec
     assert mq.workspace_size_batch([_desc(mq, 8, 64, 32, 4, False)]) == dec
-    # descriptors reading one input share its rowsum region; another x, M, K
-    # or ldx is another input
-    same = [_desc(mq, 100, 64, 32, 8, True), _desc(mq, 100, 64, 48, 4, True)]
-    assert mq.workspace_size_batch(same) == 400
-    other = _desc(mq, 100, 64, 32, 8, True)
-    other.x = FAKE + 4096
-    assert mq.workspace_size_batch(same + [other]) == 800
-    longer = _desc(mq, 100, 128, 32, 8, True)
-    longer.ldx = 128
-    assert mq.workspace_size_batch(same + [longer]) == 800
-    # an asymmetric prefill batch without its workspace is rejected up front
-    one = (mq.LinearDesc * 1)(_desc(mq, 100, 64, 32, 8, True))
+    # a decode-shaped asymmetric batch without its workspace is rejected up front
+    one = (mq.LinearDesc * 1)(_desc(mq, 8, 64, 32, 8, True))
     assert mq.lib.mq_linear_batch(one, 1, None, 0, None) == mq.MQ_ERR_WORKSPACE
 
 
@@ -262,15 +253,17 @@ def test_a16_validation_and_workspace(mq):
     assert mq.workspace_size_a16(1, 32, 48, 8) == dec
     assert mq.workspace_size_a16(0, 32, 64, 8) == 0
     assert mq.workspace_size_a16(5, 32, 0, 8) == dec              # K = 0: no planes
-    # batch: shared int16 input planned once; after a rowsum region the
-    # planes start on a 128-byte boundary
+    # batch: shared int16 input planned once; asymmetric int8 prefill next to
+    # it adds nothing; after the decode region the planes start on a
+    # 128-byte boundary
     a = _desc16(mq, 100, 64, 32, 8)
     b = _desc16(mq, 100, 64, 48, 4)
     assert mq.workspace_size_batch([a, b]) == 12800
     r = _desc(mq, 20, 64, 32, 8, True)
     r.x = FAKE + 8192
-    assert mq.workspace_size_batch([r, a]) == 128 + 12800
-    assert mq.workspace_size_batch([r]) == 80
+    assert mq.workspace_size_batch([r, a]) == 12800
+    assert mq.workspace_size_batch([r]) == 0
+    assert mq.workspace_size_batch([_desc(mq, 3, 64, 32, 4, True), a]) == dec + 12800
 
 
 def test_a16_single_call_symbols(mq):
@@ -365,3 +358,21 @@ def test_o16_ldw_rowsums_transpose_validation(mq):
     assert t(FAKE, 4, 8, 4, FAKE, 4, None) == mq.MQ_ERR_INVALID_ARG   # lds < cols
     assert t(FAKE, 4, 8, 8, FAKE, 2, None) == mq.MQ_ERR_INVALID_ARG   # ldd < rows
     assert t(None, 0, 8, 8, None, 8, None) == 0
+
+
+def test_descriptor_layout_matches_the_header(mq, tmp_path):
+    # the binding's ctypes struct against the C compiler's layout of mq_linear_desc
+    fields = [f[0] for f in mq.LinearDesc._fields_]
+    src = tmp_path / "layout.c"
+    body = "".join(f'    printf("{f} %zu\\n", offsetof(mq_linear_desc, {f}));\n' for f in fields)
+    src.write_text('#include <stddef.h>\n#include <stdio.h>\n#include "mq.h"\nint main(void) {\n'
+                   + body + '    printf("sizeof %zu\\n", sizeof(mq_linear_desc));\n    return 0;\n}\n')
+    exe = tmp_path / "layout"
+    import subprocess
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o",
+                    str(exe)], check=True)
+    out = dict(line.split() for line in subprocess.run([str(exe)], check=True, capture_output=True,
+                                                       text=True).stdout.splitlines())
+    for f in fields:
+        assert int(out[f]) == getattr(mq.LinearDesc, f).offset, f
+    assert int(out["sizeof"]) == ctypes.sizeof(mq.LinearDesc)
