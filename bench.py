@@ -55,9 +55,9 @@ WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one prefill_kernel launch on this
 # workload, from one ncu capture (profiles/prefill_kernel_tinyllama_block_w8a8_m1024.md), valid
 # only for the kernel sources it was taken on: reported as null once they change.
-PREFILL_TRAFFIC_BYTES = 56_422_400 + 3_017_472
+PREFILL_TRAFFIC_BYTES = 56_420_352 + 2_874_368
 PREFILL_TRAFFIC_SOURCES = ("mq_prefill.cu", "mq_ptx.cuh", "mq_internal.h")
-PREFILL_TRAFFIC_SHA = "2455fe7bd83defd7"
+PREFILL_TRAFFIC_SHA = "df24c867c0f1bbb9"
 
 
 def prefill_traffic():

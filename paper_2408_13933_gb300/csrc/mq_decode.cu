@@ -88,7 +88,7 @@ struct Params {
     Problem p[DECODE_MAX_PROBLEMS];  // tile_begin = first global stage, tiles_m = stages per unit
     int count;
     int total_stages;
-    int2 *ws;            // [gridDim.x][UNIT_ROWS][16] {partial sum, epoch} (zero between calls)
+    int2 *ws;            // [gridDim.x][UNIT_ROWS * 16] 8-byte {sum, epoch} words (zero between calls)
     uint32_t epoch;      // nonzero, different for every launch
     int pre_w;           // 1: load weights before griddep_wait (all constant)
     int *status;
@@ -218,23 +218,42 @@ __device__ __forceinline__ int problem_from(const SM &sm, int count, int pi, int
     return pi;
 }
 
-__device__ __forceinline__ void st_relaxed_v2(int2 *p, uint32_t a, uint32_t b) {
-    asm volatile("st.relaxed.gpu.global.v2.b32 [%0], {%1, %2};" ::"l"(p), "r"(a), "r"(b) : "memory");
+// Split-unit entries in the workspace: per CTA slot, consumer thread t's
+// 2 NT sums at words [2 NT t, 2 NT t + 2 NT), each one 8-byte word {sum in the
+// low half, launch epoch in the high half}.  An aligned 8-byte access is
+// single-copy atomic, so a reader sees either zero or the whole entry; a
+// thread's words are adjacent, so a pair of them is one 16-byte access.  The
+// mapping from a thread to its outputs depends only on the thread index, so
+// thread t of the finishing CTA reads exactly what thread t of a contributor
+// wrote.
+template <int NT>
+__device__ __forceinline__ uint64_t *unit_entries(const Params &P, int c) {
+    return reinterpret_cast<uint64_t *>(P.ws) + (size_t)c * UNIT_ROWS * 16 +
+           (size_t)threadIdx.x * (2 * NT);
 }
 
-// Wait (bounded, like every wait in this library) until the entry carries
-// `epoch`; its value is returned in `val`.
-__device__ __forceinline__ bool poll_entry(const int2 *p, uint32_t epoch, int32_t &val,
-                                           volatile int *abort, int *status) {
+__device__ __forceinline__ uint64_t pack_entry(uint32_t v, uint32_t epoch) {
+    return (uint64_t)v | ((uint64_t)epoch << 32);
+}
+
+__device__ __forceinline__ void st_pair(uint64_t *p, uint64_t a, uint64_t b) {
+    asm volatile("st.relaxed.gpu.global.v2.b64 [%0], {%1, %2};" ::"l"(p), "l"(a), "l"(b)
+                 : "memory");
+}
+
+__device__ __forceinline__ void ld_pair(const uint64_t *p, uint64_t &a, uint64_t &b) {
+    asm volatile("ld.relaxed.gpu.global.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(p)
+                 : "memory");
+}
+
+// Wait (bounded, like every wait in this library) until the word carries
+// `epoch`; the word is returned in `w`.
+__device__ __forceinline__ bool poll_word(const uint64_t *p, uint32_t epoch, uint64_t &w,
+                                          volatile int *abort, int *status) {
     uint64_t t0 = 0;
     while (true) {
-        int32_t a;
-        uint32_t b;
-        asm volatile("ld.relaxed.gpu.global.v2.b32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "l"(p) : "memory");
-        if (b == epoch) {
-            val = a;
-            return true;
-        }
+        asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
+        if ((uint32_t)(w >> 32) == epoch) return true;
         if (*abort) return false;
         const uint64_t t = global_timer_ns();
         if (t0 == 0) {
@@ -246,6 +265,56 @@ __device__ __forceinline__ bool poll_entry(const int2 *p, uint32_t epoch, int32_
         }
         __nanosleep(128);
     }
+}
+
+// A contributor's sums, stored with this launch's epoch; it does not wait.
+template <int NT>
+__device__ __forceinline__ void put_partials(const Params &P, int cta, const uint32_t (&v)[2 * NT]) {
+    uint64_t *m = unit_entries<NT>(P, cta);
+#pragma unroll
+    for (int q = 0; q < 2 * NT; q += 2)
+        st_pair(m + q, pack_entry(v[q], P.epoch), pack_entry(v[q + 1], P.epoch));
+}
+
+// A read of CTA c's entries for this thread (possibly before they are written).
+template <int NT>
+__device__ __forceinline__ void read_partials(const Params &P, int c, uint64_t (&e)[2 * NT]) {
+    const uint64_t *src = unit_entries<NT>(P, c);
+#pragma unroll
+    for (int q = 0; q < 2 * NT; q += 2) ld_pair(src + q, e[q], e[q + 1]);
+}
+
+// The finishing CTA adds the sums of contributors cf + 1 .. cl into v.  `first`
+// is an earlier read of CTA cf + 1's entries; words that do not carry this
+// launch's epoch yet are polled.  Every entry read is stored back as zero.
+template <int NT>
+__device__ __forceinline__ bool gather_partials(const Params &P, volatile int *abort, int cf,
+                                                int cl, const uint64_t (&first)[2 * NT],
+                                                uint32_t (&v)[2 * NT]) {
+    bool got = true;
+    for (int c = cf + 1; got && c <= cl; ++c) {
+        uint64_t e[2 * NT];
+        if (c == cf + 1) {
+#pragma unroll
+            for (int q = 0; q < 2 * NT; ++q) e[q] = first[q];
+        } else {
+            read_partials<NT>(P, c, e);
+        }
+        const uint64_t *src = unit_entries<NT>(P, c);
+#pragma unroll
+        for (int q = 0; q < 2 * NT; ++q) {
+            if ((uint32_t)(e[q] >> 32) != P.epoch)
+                got = got && poll_word(src + q, P.epoch, e[q], abort, P.status);
+            v[q] += (uint32_t)e[q];
+        }
+    }
+    if (got)
+        for (int c = cf + 1; c <= cl; ++c) {
+            uint64_t *src = unit_entries<NT>(P, c);
+#pragma unroll
+            for (int q = 0; q < 2 * NT; q += 2) st_pair(src + q, 0ull, 0ull);
+        }
+    return got;
 }
 
 // Requantize one output of tile row `row` (global row n, token tok) from
@@ -424,30 +493,12 @@ __device__ __forceinline__ void a16_epilogue(const Params &P, SM &s, const DecPr
     }
     if (have && !whole) {
         if (!finisher) {
-            int2 *mine = P.ws + (size_t)cta * UNIT_ROWS * 16;
-#pragma unroll
-            for (int q = 0; q < 2 * NT; ++q) st_relaxed_v2(mine + rows[q] * 16 + tok, v[q], P.epoch);
+            put_partials<NT>(P, cta, v);
             have = false;
         } else {
-            bool got = true;
-            for (int c = cf + 1; got && c <= cl; ++c) {
-                const int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
-#pragma unroll
-                for (int q = 0; q < 2 * NT; ++q) {
-                    int32_t x = 0;
-                    got = got && poll_entry(src + rows[q] * 16 + tok, P.epoch, x, &s.abort,
-                                            P.status);
-                    v[q] += (uint32_t)x;
-                }
-            }
-            if (got) {
-                for (int c = cf + 1; c <= cl; ++c) {
-                    int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
-#pragma unroll
-                    for (int q = 0; q < 2 * NT; ++q) st_relaxed_v2(src + rows[q] * 16 + tok, 0u, 0u);
-                }
-            }
-            have = got;
+            uint64_t first[2 * NT];
+            read_partials<NT>(P, cf + 1, first);
+            have = gather_partials<NT>(P, &s.abort, cf, cl, first, v);
         }
     }
     int32_t *yv = &s.part[0][0][0];
@@ -581,6 +632,22 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             const int rb = local / nst;
             const int u_begin = p.tile_begin + rb * nst, u_end = u_begin + nst;
             const int piece_end = u_end < s_end ? u_end : s_end;
+            const bool whole = u_begin >= s_begin && u_end <= s_end;
+            // this thread's slots j + 256 q share one fragment element i, one
+            // token tile and one lane: the token is fixed
+            const int e0 = threadIdx.x >> 5, ln = threadIdx.x & 31;
+            const int tok = (NT == 2 ? ((e0 >> 2) & 1) * 8 : 0) + 2 * (ln & 3) + (e0 & 1);
+            // a split unit is finished by its first CTA (cf), at the end of
+            // its range; the contributors cf + 1 .. cl store their sums at
+            // the start of theirs.  The finishing CTA reads the first
+            // contributor's entries before its last stage, so that the round
+            // trip overlaps that stage.
+            const int cf = whole ? cta : cta_of(u_begin, S, G);
+            const int cl = whole ? cta : cta_of(u_end - 1, S, G);
+            const bool early = !A16 && !whole && cta == cf && cl > cf && tok < p.M;
+            uint64_t first[2 * NT];
+#pragma unroll
+            for (int q = 0; q < 2 * NT; ++q) first[q] = 0;
             // requant parameters of the unit's rows: loaded now, published to
             // shared memory when the piece is done, so the loads overlap the
             // stage loop instead of stalling the warp here
@@ -610,6 +677,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             for (int nt = 0; nt < NT; ++nt) xs[nt] = 0;
             for (int q = gs; ok && q < piece_end; ++q, ++it) {
                 const int slot = it % STAGES;
+                if (early && q == piece_end - 1) read_partials<NT>(P, cf + 1, first);
                 bool got = true;
                 if (lane == 0)
                     got = mq_wait_parity(&s.full[slot], (it / STAGES) & 1, &s.abort, P.status);
@@ -671,11 +739,6 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                 s.row_shift[threadIdx.x] = prm_sh;
             }
             cons_sync();
-            const bool whole = u_begin >= s_begin && u_end <= s_end;
-            // this thread's slots j + 256 q share one fragment element i, one
-            // token tile and one lane: the token is fixed
-            const int e0 = threadIdx.x >> 5, ln = threadIdx.x & 31;
-            const int tok = (NT == 2 ? ((e0 >> 2) & 1) * 8 : 0) + 2 * (ln & 3) + (e0 & 1);
             int32_t xsum = 0;
             if (ok && tok < p.M) {
 #pragma unroll
@@ -700,14 +763,8 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                                         (uint32_t)((C::BIAS + s.row_zw[row]) * xsum)));
                 }
             } else if (ok) {
-                // A split unit.  Its first CTA finishes it: that CTA reaches the
-                // unit at the end of its range, while the later contributors
-                // process the unit's tail at the start of theirs.  A
-                // contributor stores each of its sums together with this
-                // launch's epoch as one 8-byte store (single-copy atomic) and
-                // goes on; the first CTA polls each entry until it carries the
-                // epoch, adds it, and stores zero back.  No fences or counters.
-                const int cf = cta_of(u_begin, S, G), cl = cta_of(u_end - 1, S, G);
+                // a split unit (see above): contributors store, the first CTA
+                // gathers, requantizes and stores
                 if (tok < p.M) {
                     uint32_t v[2 * NT];
                     int rows[2 * NT];
@@ -721,29 +778,10 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                         v[q] = (uint32_t)sum - (uint32_t)((C::BIAS + s.row_zw[rows[q]]) * xsum);
                     }
                     if (cta != cf) {
-                        int2 *mine = P.ws + (size_t)cta * UNIT_ROWS * 16;
-#pragma unroll
-                        for (int q = 0; q < 2 * NT; ++q)
-                            st_relaxed_v2(mine + rows[q] * 16 + tok, v[q], P.epoch);
+                        put_partials<NT>(P, cta, v);
                     } else {
-                        bool got = true;
-                        for (int c = cf + 1; got && c <= cl; ++c) {
-                            const int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
-#pragma unroll
-                            for (int q = 0; q < 2 * NT; ++q) {
-                                int32_t x = 0;
-                                got = got && poll_entry(src + rows[q] * 16 + tok, P.epoch, x,
-                                                        &s.abort, P.status);
-                                v[q] += (uint32_t)x;
-                            }
-                        }
-                        if (got) {
-                            for (int c = cf + 1; c <= cl; ++c) {
-                                int2 *src = P.ws + (size_t)c * UNIT_ROWS * 16;
-#pragma unroll
-                                for (int q = 0; q < 2 * NT; ++q)
-                                    st_relaxed_v2(src + rows[q] * 16 + tok, 0u, 0u);
-                            }
+                        if (!early) read_partials<NT>(P, cf + 1, first);
+                        if (gather_partials<NT>(P, &s.abort, cf, cl, first, v)) {
 #pragma unroll
                             for (int q = 0; q < 2 * NT; ++q) {
                                 const int n = rb * UNIT_ROWS + rows[q];
