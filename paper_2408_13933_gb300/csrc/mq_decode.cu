@@ -90,6 +90,7 @@ struct Params {
     int total_stages;
     int2 *ws;            // [gridDim.x][UNIT_ROWS * 16] 8-byte {sum, epoch} words (zero between calls)
     uint32_t epoch;      // nonzero, different for every launch
+    int wide;            // total_stages * gridDim.x >= 2^32: 64-bit range arithmetic
     int pre_w;           // 1: load weights before griddep_wait (all constant)
     int *status;
 };
@@ -197,16 +198,20 @@ struct Cfg<8> {
     static constexpr int BIAS = 128;
 };
 
-// First global stage of CTA c when S stages are split among G CTAs.
-__device__ __forceinline__ int range_begin(int c, int S, int G) {
-    return (int)(((long long)c * S) / G);
+// First global stage of CTA c when S stages are split among G CTAs.  With
+// S * G < 2^32 (the launcher sets `wide` otherwise) the products fit 32 bits:
+// a 64-bit division is a long software sequence, and these run in every
+// CTA's prologue and for every split unit.
+__device__ __forceinline__ int range_begin(int c, int S, int G, bool wide) {
+    return wide ? (int)(((long long)c * S) / G)
+                : (int)(((uint32_t)c * (uint32_t)S) / (uint32_t)G);
 }
 
 // The CTA whose range holds global stage s.
-__device__ __forceinline__ int cta_of(int s, int S, int G) {
-    int c = (int)(((long long)s * G) / S);
-    while (c + 1 < G && range_begin(c + 1, S, G) <= s) ++c;
-    while (c > 0 && range_begin(c, S, G) > s) --c;
+__device__ __forceinline__ int cta_of(int s, int S, int G, bool wide) {
+    int c = wide ? (int)(((long long)s * G) / S) : (int)(((uint32_t)s * (uint32_t)G) / (uint32_t)S);
+    while (c + 1 < G && range_begin(c + 1, S, G, wide) <= s) ++c;
+    while (c > 0 && range_begin(c, S, G, wide) > s) --c;
     return c;
 }
 
@@ -471,12 +476,9 @@ constexpr int YV_STRIDE = UNIT_ROWS + 4;
 template <int BITS, int NT, class SM>
 __device__ __forceinline__ void a16_epilogue(const Params &P, SM &s, const DecProb &p, int rb,
                                              bool whole, bool ok, int tok, int32_t xsum, int e0,
-                                             int ln, int S, int G, int cta) {
+                                             int ln, bool finisher, int cl, int cta) {
     using C = Cfg<BITS>;
-    const int u_begin = p.tile_begin + rb * p.tiles_m, u_end = u_begin + p.tiles_m;
-    const int cf = whole ? cta : cta_of(u_begin, S, G);
-    const int cl = whole ? cta : cta_of(u_end - 1, S, G);
-    const bool finisher = cta == cf;
+    const int cf = cta;  // read only by the finisher
     bool have = ok && tok < p.M;
     uint32_t v[2 * NT];
     int rows[2 * NT];
@@ -538,7 +540,8 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int S = P.total_stages, G = gridDim.x, cta = blockIdx.x;
-    const int s_begin = range_begin(cta, S, G), s_end = range_begin(cta + 1, S, G);
+    const bool wide = P.wide != 0;
+    const int s_begin = range_begin(cta, S, G, wide), s_end = range_begin(cta + 1, S, G, wide);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
@@ -637,14 +640,15 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             // token tile and one lane: the token is fixed
             const int e0 = threadIdx.x >> 5, ln = threadIdx.x & 31;
             const int tok = (NT == 2 ? ((e0 >> 2) & 1) * 8 : 0) + 2 * (ln & 3) + (e0 & 1);
-            // a split unit is finished by its first CTA (cf), at the end of
-            // its range; the contributors cf + 1 .. cl store their sums at
-            // the start of theirs.  The finishing CTA reads the first
-            // contributor's entries before its last stage, so that the round
-            // trip overlaps that stage.
-            const int cf = whole ? cta : cta_of(u_begin, S, G);
-            const int cl = whole ? cta : cta_of(u_end - 1, S, G);
-            const bool early = !A16 && !whole && cta == cf && cl > cf && tok < p.M;
+            // a split unit is finished by its first CTA (the one holding its
+            // first stage), at the end of that CTA's range; the contributors
+            // cf + 1 .. cl store their sums at the start of theirs.  The
+            // finishing CTA reads the first contributor's entries before its
+            // last stage, so that the round trip overlaps that stage.
+            const bool finisher = u_begin >= s_begin;
+            const int cf = cta;  // read only when finisher
+            const int cl = (whole || !finisher) ? cta : cta_of(u_end - 1, S, G, wide);
+            const bool early = !A16 && !whole && finisher && tok < p.M;
             uint64_t first[2 * NT];
 #pragma unroll
             for (int q = 0; q < 2 * NT; ++q) first[q] = 0;
@@ -745,7 +749,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                 for (int w = 0; w < CONS_WARPS; ++w) xsum += s.xpart[w][tok];
             }
             if constexpr (A16) {
-                a16_epilogue<BITS, NT>(P, s, p, rb, whole, ok, tok, xsum, e0, ln, S, G, cta);
+                a16_epilogue<BITS, NT>(P, s, p, rb, whole, ok, tok, xsum, e0, ln, finisher, cl, cta);
             } else if (ok && whole) {
                 // the unit is entirely this CTA's: requantize and store
 #pragma unroll
@@ -777,7 +781,7 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                         for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
                         v[q] = (uint32_t)sum - (uint32_t)((C::BIAS + s.row_zw[rows[q]]) * xsum);
                     }
-                    if (cta != cf) {
+                    if (!finisher) {
                         put_partials<NT>(P, cta, v);
                     } else {
                         if (!early) read_partials<NT>(P, cf + 1, first);
@@ -900,6 +904,7 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
         long long grid = 2LL * sms;
         if (grid > DECODE_MAX_GRID) grid = DECODE_MAX_GRID;
         if (grid > stages) grid = stages;
+        P.wide = (unsigned long long)stages * (unsigned long long)grid >= (1ull << 32);
         // programmatic stream serialization: this launch may start while the
         // previous kernel in the stream finishes (see griddep_wait)
         cudaLaunchConfig_t cfg{};
