@@ -633,9 +633,11 @@ class AttentionSet:
         self.q, self.k, self.v, self.p = up(a.q), up(a.k), up(a.v), up(a.p)
         self.s = torch.empty((H, t, t), dtype=torch.int16, device=dev)
         self.o = torch.empty((t, H * D), dtype=torch.int8, device=dev)
+        # keys' row sums per KV head [G][T]; V^T of all heads at once [G d][T]
+        # (head g is rows g d .. g d + d - 1) and its row sums [G d]
         self.colk = torch.empty((G, t), dtype=torch.int32, device=dev)
-        self.vt = torch.empty((G, D, t), dtype=torch.int8, device=dev)
-        self.colv = torch.empty((G, D), dtype=torch.int32, device=dev)
+        self.vt = torch.empty((G * D, t), dtype=torch.int8, device=dev)
+        self.colv = torch.empty((G * D,), dtype=torch.int32, device=dev)
         i32 = lambda n, v: up(np.full(n, v, np.int32))
         self.keep = [i32(t, self.M0_S), i32(t, self.SH_S), i32(t, a.zk),
                      i32(D, self.M0_O), i32(D, self.SH_O), i32(D, a.zv)]
@@ -644,7 +646,9 @@ class AttentionSet:
         ds = [mq.make_desc(self.q[:, h * D:(h + 1) * D], a.zq, self.k[:, (h // rep) * D:],
                            self.colk[h // rep], t, m0s, shs, self.ZY_S, self.s[h], 8, zw=zwk,
                            ldw=G * D, wdynamic=True) for h in range(H)]
-        do = [mq.make_desc(self.p[h], a.zp, self.vt[h // rep], self.colv[h // rep], D, m0o, sho,
+        vt_g = lambda g: self.vt[g * D:(g + 1) * D]
+        cv_g = lambda g: self.colv[g * D:(g + 1) * D]
+        do = [mq.make_desc(self.p[h], a.zp, vt_g(h // rep), cv_g(h // rep), D, m0o, sho,
                            self.ZY_O, self.o[:, h * D:(h + 1) * D], 8, zw=zwv, wdynamic=True)
               for h in range(H)]
         self.arr_s = (mq.LinearDesc * H)(*ds)
@@ -661,17 +665,14 @@ class AttentionSet:
         lib, H, G, D, t = mq.lib, self.H, self.G, self.D, self.t
         rcs = []
         if phase in ("all", "scores"):
-            for g in range(G):
-                rcs.append(lib.mq_row_sums(self.k[:, g * D:].data_ptr(), t, D, G * D,
-                                           self.colk[g].data_ptr(), sp))
+            rcs.append(lib.mq_head_row_sums(self.k.data_ptr(), t, G, D, G * D,
+                                            self.colk.data_ptr(), sp))
             rcs.append(lib.mq_linear_batch(self.arr_s, H, self.ws_s.data_ptr(), self.ws_s_bytes,
                                            sp))
         if phase in ("all", "pv"):
-            for g in range(G):
-                rcs.append(lib.mq_transpose_i8(self.v[:, g * D:].data_ptr(), t, D, G * D,
-                                               self.vt[g].data_ptr(), t, sp))
-                rcs.append(lib.mq_row_sums(self.vt[g].data_ptr(), D, t, t,
-                                           self.colv[g].data_ptr(), sp))
+            rcs.append(lib.mq_transpose_i8(self.v.data_ptr(), t, G * D, G * D, self.vt.data_ptr(),
+                                           t, sp))
+            rcs.append(lib.mq_row_sums(self.vt.data_ptr(), G * D, t, t, self.colv.data_ptr(), sp))
             rcs.append(lib.mq_linear_batch(self.arr_o, H, self.ws_o.data_ptr(), self.ws_o_bytes,
                                            sp))
         if any(rcs):
@@ -706,9 +707,10 @@ class AttentionSet:
 def run_attention(mq, torch, reps: int = 60, check_rows: int = 4):
     """Grouped-query attention's two integer matmuls of one TinyLlama layer at
     T = 1024 (the softmax between them is outside the integer layer): per step
-    the key row sums, S = Q K^T for 32 heads (one batched call, one prefill
-    launch, int16 scores), the V^T transposes and their row
-    sums, and O = P V for 32 heads (one batched call).  Steps rotate over three
+    the key row sums of the 4 KV heads (one launch), S = Q K^T for 32 heads
+    (one batched call, one prefill launch, int16 scores), V^T of all heads
+    (one transpose) and its row sums (one launch), and O = P V for 32 heads
+    (one batched call).  Steps rotate over three
     layers' operands (about 300 MB, more than L2).  The host enqueues the timed
     steps behind a device sleep, so the region measures the device, not the
     ctypes call rate; a second pass times the two phases alone."""

@@ -429,6 +429,19 @@ int mq_fold_norm(const float *gamma, const float *beta, const float *s, int K, f
 int mq_row_sums(const int8_t *x, int M, int K, int ldx, int32_t *out, void *stream);
 
 /*
+ * out[h][m] = sum_{k < d} x[m][h d + k] (int32) for int8 x [M][ldx] and h < heads:
+ * the row sums of every head slice of a projection output [T][heads d] in one
+ * launch (the keys' colsum of every KV head for Q K^T).  out is [heads][M]
+ * (device int32, written).  Requirements: M, d >= 0; 0 <= heads; d % 16 == 0;
+ * ldx >= heads d, ldx % 16 == 0; x 16-byte aligned; d <= MQ_MAX_K.  Asynchronous
+ * on `stream` (programmatic dependent launch: x is read after the previous
+ * kernel completes).
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_ALIGNMENT, MQ_ERR_CUDA.
+ */
+int mq_head_row_sums(const int8_t *x, int M, int heads, int d, int ldx, int32_t *out,
+                     void *stream);
+
+/*
  * dst[c][r] = src[r][c] for int8 src [rows][lds] -> dst [cols][ldd] (lds >=
  * cols, ldd >= rows): V [T][d] -> V^T [d][T], the K-major "weights" operand of
  * P V.  Asynchronous on `stream`.

@@ -510,6 +510,30 @@ int mq_row_sums(const int8_t *x, int M, int K, int ldx, int32_t *out, void *stre
     return mq::launch_rowsum(&j, 1, stream);
 }
 
+int mq_head_row_sums(const int8_t *x, int M, int heads, int d, int ldx, int32_t *out,
+                     void *stream) {
+    if (M < 0 || heads < 0 || d < 0 || d > MQ_MAX_K || (int64_t)heads * d > ldx)
+        return MQ_ERR_INVALID_ARG;
+    if (M == 0 || heads == 0) return MQ_OK;
+    if (!out || (d > 0 && !x)) return MQ_ERR_INVALID_ARG;
+    if (d % 16 != 0 || ldx % 16 != 0 || (d > 0 && !aligned16(x))) return MQ_ERR_ALIGNMENT;
+    for (int h0 = 0; h0 < heads; h0 += mq::ROWSUM_MAX_JOBS) {
+        const int n = heads - h0 < mq::ROWSUM_MAX_JOBS ? heads - h0 : mq::ROWSUM_MAX_JOBS;
+        mq::RowsumJob jobs[mq::ROWSUM_MAX_JOBS];
+        for (int i = 0; i < n; ++i) {
+            jobs[i] = mq::RowsumJob{};
+            jobs[i].x = x + (size_t)(h0 + i) * (size_t)d;
+            jobs[i].out = out + (size_t)(h0 + i) * (size_t)M;
+            jobs[i].M = M;
+            jobs[i].K = d;
+            jobs[i].ldx = ldx;
+        }
+        const int rc = mq::launch_rowsum(jobs, n, stream);
+        if (rc != MQ_OK) return rc;
+    }
+    return MQ_OK;
+}
+
 int mq_transpose_i8(const int8_t *src, int rows, int cols, int lds, int8_t *dst, int ldd,
                     void *stream) {
     if (rows < 0 || cols < 0 || lds < cols || ldd < rows) return MQ_ERR_INVALID_ARG;

@@ -41,7 +41,7 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch",
             "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16", "mq_quantize",
             "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm",
-            "mq_row_sums", "mq_transpose_i8"]
+            "mq_row_sums", "mq_head_row_sums", "mq_transpose_i8"]
 MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
@@ -83,6 +83,7 @@ lib.mq_fold_quantize_pack.argtypes = [_vp, _int, _int, _vp, _vp, _int, _int, _vp
                                       _vp, _vp]
 lib.mq_fold_norm.argtypes = [_vp, _vp, _vp, _int, _vp, _vp]
 lib.mq_row_sums.argtypes = [_vp, _int, _int, _int, _vp, _vp]
+lib.mq_head_row_sums.argtypes = [_vp, _int, _int, _int, _int, _vp, _vp]
 lib.mq_transpose_i8.argtypes = [_vp, _int, _int, _int, _vp, _int, _vp]
 for _f in EXPORTED:
     if _f != "mq_status_string":
@@ -274,6 +275,20 @@ def row_sums(x, out=None, m=None, k=None, ldx=None, stream=None):
     if out is None:
         out = torch.empty(m, dtype=torch.int32, device=x.device)
     _check(lib.mq_row_sums(_ptr(x), m, k, ldx, _ptr(out), _stream(stream)), "mq_row_sums")
+    return out
+
+
+def head_row_sums(x, heads: int, out=None, stream=None):
+    """mq_head_row_sums on an int8 CUDA tensor [M, heads * d] (or a row-strided
+    view): int32 [heads, M], the row sums of every d-wide head slice."""
+    import torch
+    m, width = x.shape
+    assert width % heads == 0
+    d = width // heads
+    if out is None:
+        out = torch.empty((heads, m), dtype=torch.int32, device=x.device)
+    _check(lib.mq_head_row_sums(_ptr(x), m, heads, d, x.stride(0), _ptr(out), _stream(stream)),
+           "mq_head_row_sums")
     return out
 
 

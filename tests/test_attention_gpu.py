@@ -118,6 +118,13 @@ def test_row_sums_and_transpose():
     t = lib.transpose_i8(ad[:, 128:192])   # a head's slice
     torch.cuda.synchronize()
     assert np.array_equal(t.cpu().numpy(), a[:, 128:192].T)
+    # every head slice at once: [M, heads * d] -> [heads, M], incl. more heads than one launch takes
+    for m, heads, d, pad in ((1024, 4, 64, 0), (33, 3, 16, 32), (7, 70, 16, 0)):
+        a = rng.integers(-128, 128, size=(m, heads * d + pad), dtype=np.int16).astype(np.int8)
+        ad = upload(a)
+        got = lib.head_row_sums(ad[:, :heads * d], heads).cpu().numpy()
+        want = a[:, :heads * d].astype(np.int64).reshape(m, heads, d).sum(2).T
+        assert np.array_equal(got, want), (m, heads, d)
 
 
 @pytest.mark.parametrize("t_q", [96, 1])
@@ -168,14 +175,24 @@ def test_grouped_query_attention_matmuls(t_q):
     torch.cuda.synchronize()
     sp = torch.cuda.current_stream().cuda_stream
     for r in range(R):
-        for g in range(G):
-            assert lib.lib.mq_row_sums(kds[r][:, g * D:].data_ptr(), T, D, G * D,
-                                       colk[g].data_ptr(), sp) == 0
+        if r == 0:  # per head
+            for g in range(G):
+                assert lib.lib.mq_row_sums(kds[r][:, g * D:].data_ptr(), T, D, G * D,
+                                           colk[g].data_ptr(), sp) == 0
+        else:       # all heads in one launch
+            assert lib.lib.mq_head_row_sums(kds[r].data_ptr(), T, G, D, G * D,
+                                            colk.data_ptr(), sp) == 0
         assert lib.lib.mq_linear_batch(arr_s[r], H, ws.data_ptr(), need, sp) == 0
-        for g in range(G):
-            assert lib.lib.mq_transpose_i8(vds[r][:, g * D:].data_ptr(), T, D, G * D,
-                                           vt[g].data_ptr(), T, sp) == 0
-            assert lib.lib.mq_row_sums(vt[g].data_ptr(), D, T, T, colv[g].data_ptr(), sp) == 0
+        if r == 0:  # per head
+            for g in range(G):
+                assert lib.lib.mq_transpose_i8(vds[r][:, g * D:].data_ptr(), T, D, G * D,
+                                               vt[g].data_ptr(), T, sp) == 0
+                assert lib.lib.mq_row_sums(vt[g].data_ptr(), D, T, T, colv[g].data_ptr(),
+                                           sp) == 0
+        else:       # V^T of all heads [G d][T] at once (vt is [G][d][T] contiguous)
+            assert lib.lib.mq_transpose_i8(vds[r].data_ptr(), T, G * D, G * D, vt.data_ptr(),
+                                           T, sp) == 0
+            assert lib.lib.mq_row_sums(vt.data_ptr(), G * D, T, T, colv.data_ptr(), sp) == 0
         assert lib.lib.mq_linear_batch(arr_o[r], H, ws.data_ptr(), need, sp) == 0
     torch.cuda.synchronize()
     assert lib.check_device_status() == 0

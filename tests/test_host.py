@@ -354,6 +354,14 @@ def test_o16_ldw_rowsums_transpose_validation(mq):
     assert r(FAKE, 4, 40, 48, FAKE, None) == mq.MQ_ERR_ALIGNMENT
     assert r(FAKE, 4, 64, 32, FAKE, None) == mq.MQ_ERR_INVALID_ARG
     assert r(None, 0, 64, 64, None, None) == 0
+    hr = mq.lib.mq_head_row_sums
+    assert hr(FAKE, 4, 4, 64, 192, FAKE, None) == mq.MQ_ERR_INVALID_ARG   # ldx < heads d
+    assert hr(FAKE, 4, 4, 40, 160, FAKE, None) == mq.MQ_ERR_ALIGNMENT     # d % 16
+    assert hr(FAKE, 4, 4, 64, 264, FAKE, None) == mq.MQ_ERR_ALIGNMENT     # ldx % 16
+    assert hr(FAKE + 8, 4, 4, 64, 256, FAKE, None) == mq.MQ_ERR_ALIGNMENT
+    assert hr(FAKE, 4, 4, 64, 256, None, None) == mq.MQ_ERR_INVALID_ARG
+    assert hr(None, 0, 4, 64, 256, None, None) == 0
+    assert hr(None, 4, 0, 64, 256, None, None) == 0
     t = mq.lib.mq_transpose_i8
     assert t(FAKE, 4, 8, 4, FAKE, 4, None) == mq.MQ_ERR_INVALID_ARG   # lds < cols
     assert t(FAKE, 4, 8, 8, FAKE, 2, None) == mq.MQ_ERR_INVALID_ARG   # ldd < rows
