@@ -12,17 +12,19 @@
 // matter how the linears' sizes differ.  A unit whose stages fall to several
 // CTAs is finished by its first CTA, which reaches the unit at the end of its
 // range; the later contributors, which process the unit's tail at the start
-// of theirs, store their int32 partial sums in their own workspace slot, each
-// with the launch's epoch in the same 8-byte store, and go on without
-// waiting.  The first CTA polls the entries for the epoch, adds them,
-// requantizes, and stores zero back, so the workspace is left zero.
+// of theirs, store their int32 partial sums in their own workspace slot as
+// 8-byte words {sum, launch epoch} (a thread's words adjacent) and go on
+// without waiting.  The first CTA reads a contributor's words before its own
+// last stage of the unit, polls only words that do not carry the epoch yet,
+// adds them, requantizes, and stores zero back, so the workspace is left zero.
 //
 // Data path.  In each CTA one producer thread streams the weight rows of its
-// stages with TMA into an 8-stage shared-memory ring, continuing across unit
-// boundaries.  A stage holds 64 weight rows x 128
-// bytes and the matching k slice of the 16 (zero-padded) token rows of x,
-// both 128-byte swizzled, so up to 64 KB of weights per CTA are in flight and
-// the activation fragments come from shared memory without bank conflicts.
+// stages with TMA into a 7-stage (one token tile) or 6-stage (two) shared-
+// memory ring, continuing across unit boundaries.  A stage holds 64 weight
+// rows x 128 bytes and the matching k slice of the 16 (zero-padded) token rows
+// of x, both 128-byte swizzled, so up to 56 KB of weights per CTA are in
+// flight and the activation fragments come from shared memory without bank
+// conflicts.
 // Eight consumer warps read the ring, widen weights in registers to f16 and multiply with warp-level
 // mma.sync m16n8k16 (f16 x f16 -> f32): weights are the 16-row A operand, the
 // (zero-padded) tokens the 8-column B operand.  Warp w of the consumers owns
