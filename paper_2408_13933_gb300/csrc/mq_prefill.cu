@@ -9,7 +9,10 @@
 // partial sum is an integer of magnitude <= 2^24.  The K loop is therefore cut
 // into chunks of 1024 (int8 weights: |x w| <= 2^14) or 16384 (int4: |x w| <=
 // 2^10); after each chunk the epilogue converts the f32 chunk sum to int32
-// and adds it to an int32 running sum.
+// and adds it to an int32 running sum.  With a weight zero point zw the
+// converters widen w - zw instead (the widening's f16 offset absorbs zw), the
+// chunks shrink to 512 and 8192 (|x (w - zw)| <= 128 * 255, 128 * 15) and the
+// epilogue subtracts zx (colsum - K zw).
 //
 // The kernel runs on CTA pairs (clusters of two, one CTA per SM) with pair
 // MMAs (tcgen05 cta_group::2, M = 256, N = 128, K = 16).  Operand A is the
