@@ -210,3 +210,92 @@ def test_grouped_query_attention_matmuls(t_q):
                                  zw=np.full(D, zv, np.int32))
             assert_equal_int8(outs[r][:, h * D:(h + 1) * D].cpu().numpy(), want,
                               f"round {r} P V head {h}")
+
+
+@pytest.mark.parametrize("m", [3, 140])
+def test_o16_int4_zero_points_across_chunks(m):
+    # int16 outputs, int4 weights with zero points at the range ends, K = 20480:
+    # the tensor-core kernel's 8192-k chunks of x (w - zw) full twice and
+    # ragged once (m = 140), the decode kernel's stages (m = 3)
+    torch = torch_cuda()
+    lib = mq()
+    n, k = 72, 20480
+    c = synth.random_case(900 + m, m, k, n, 4, "mixed")
+    zw = np.where(np.arange(n) % 2 == 0, -8, 7).astype(np.int32)
+    rng = np.random.default_rng(m)
+    m0 = rng.integers(1 << 30, 1 << 31, size=n).astype(np.int32)
+    sh = rng.integers(36, 48, size=n).astype(np.int32)
+    packed, colsum = lib.pack_weights(c.w, 4)
+    keep = [upload(a) for a in (c.x, packed, colsum, m0, sh, zw)]
+    y = torch.full((m, n), 1, dtype=torch.int16, device="cuda")
+    keep.append(y)
+    d = lib.make_desc(keep[0], c.zx, keep[1], keep[2], n, keep[3], keep[4], -1000, y, 4,
+                      zw=keep[5])
+    _run([d], keep)
+    opk, _ = oracle.pack(c.w, 4)
+    want = oracle.linear_o16(c.x, c.zx, opk, 4, n, m0, sh, -1000, zw=zw)
+    assert_equal(y.cpu().numpy(), want, f"o16 int4 zw K=20480 m={m}")
+
+
+def test_batch_mixes_output_widths_and_kernels():
+    # one call: int16-output problems (prefill and decode), 8-bit problems (one
+    # asymmetric, one decode) and 16-bit-activation problems: every (kernel,
+    # width) family is launched, results as if each ran alone
+    torch = torch_cuda()
+    lib = mq()
+    keep, descs, wants, outs = [], [], [], []
+
+    def add(seed, m, k, n, bits, obits=8, abits=8, asym=False):
+        case = (synth.random_case_a16(seed, m, k, n, bits) if abits == 16
+                else synth.random_case(seed, m, k, n, bits))
+        rng = np.random.default_rng(seed)
+        if obits == 16 and abits == 8:
+            m0 = rng.integers(1 << 30, 1 << 31, size=n).astype(np.int32)
+            sh = rng.integers(36, 46, size=n).astype(np.int32)
+        else:
+            m0, sh = lib.requant_params(case.sw, case.sx, case.sy)
+        lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+        zw = rng.integers(lo, hi + 1, size=n).astype(np.int32) if asym else None
+        packed, colsum = lib.pack_weights(case.w, bits)
+        dev = [upload(a) for a in (case.x, packed, colsum, m0, sh)]
+        zwd = upload(zw) if asym else None
+        y = torch.full((m, n), 3, dtype=torch.int16 if 16 in (obits, abits) else torch.int8,
+                       device="cuda")
+        keep.extend(dev + [zwd, y])
+        descs.append(lib.make_desc(dev[0], case.zx, dev[1], dev[2], n, dev[3], dev[4], case.zy
+                                   if obits == 8 or abits == 16 else 77, y, bits, zw=zwd,
+                                   abits=abits))
+        opk, _ = oracle.pack(case.w, bits)
+        if abits == 16:
+            om0, osh = oracle.requant_params(case.sx, case.sw, case.sy)
+            wants.append(oracle.linear_a16(case.x, case.zx, opk, bits, n, om0, osh, case.zy))
+        elif obits == 16:
+            wants.append(oracle.linear_o16(case.x, case.zx, opk, bits, n, m0, sh, 77, zw=zw))
+        else:
+            om0, osh = oracle.requant_params(case.sx, case.sw, case.sy)
+            wants.append(oracle.linear(case.x, case.zx, opk, bits, n, om0, osh, case.zy, zw=zw))
+        outs.append(y)
+
+    add(1001, 96, 512, 100, 8, obits=16, asym=True)    # prefill, int16 out
+    add(1002, 4, 1024, 80, 4, obits=16)                # decode, int16 out
+    add(1003, 130, 768, 64, 8, asym=True)              # prefill, int8, asymmetric
+    add(1004, 2, 512, 96, 4)                           # decode, int8
+    add(1005, 40, 256, 72, 8, abits=16)                # prefill, 16-bit activations
+    add(1006, 3, 256, 48, 4, abits=16)                 # decode, 16-bit activations
+    _run(descs, keep)
+    for i, (y, want) in enumerate(zip(outs, wants)):
+        assert_equal(y.cpu().numpy(), want, f"mixed batch problem {i}")
+
+
+def test_transpose_into_a_padded_destination():
+    torch = torch_cuda()
+    lib = mq()
+    rng = np.random.default_rng(21)
+    a = rng.integers(-128, 128, size=(70, 200), dtype=np.int16).astype(np.int8)
+    ad = upload(a)
+    dst = torch.full((200, 96), 5, dtype=torch.int8, device="cuda")   # ldd 96 > rows 70
+    lib.transpose_i8(ad[:, 8:200], dst=dst[:192])
+    torch.cuda.synchronize()
+    got = dst.cpu().numpy()
+    assert np.array_equal(got[:192, :70], a[:, 8:200].T)
+    assert np.all(got[:192, 70:] == 5) and np.all(got[192:] == 5)   # padding untouched
