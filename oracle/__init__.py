@@ -53,6 +53,7 @@ def _bind(lib):
     lib.oracle_requant_one.argtypes = [i64, i32, i32, i32]
     lib.oracle_requant_one.restype = i32
     lib.oracle_linear_a16.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci, p]
+    lib.oracle_linear_a16_asym.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, p, i32, p, ci, p]
     lib.oracle_linear_points_a16.argtypes = [p, ci, ci, ci, i32, p, ci, ci, p, p, i32, p, ci,
                                              p, p]
     lib.oracle_requant_one_a16.argtypes = [i64, i32, i32, i32]
@@ -171,9 +172,11 @@ class Oracle:
         return int(self.lib.oracle_requant_one(int(acc), int(m0), int(shift), int(zy)))
 
     def linear_a16(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
-                   m0: np.ndarray, shift: np.ndarray, zy: int, want_acc: bool = False):
-        """The layer with int16 activations (oracle_linear_a16): returns y int16
-        [M, N] (and acc int64 [M, N])."""
+                   m0: np.ndarray, shift: np.ndarray, zy: int, want_acc: bool = False,
+                   zw=None):
+        """The layer with int16 activations (oracle_linear_a16; with a weight
+        zero point zw [N], oracle_linear_a16_asym): returns y int16 [M, N] (and
+        acc int64 [M, N])."""
         x = np.ascontiguousarray(x, dtype=np.int16)
         m, k = x.shape
         packed = np.ascontiguousarray(packed, dtype=np.uint8)
@@ -181,10 +184,17 @@ class Oracle:
         shift = np.ascontiguousarray(shift, dtype=np.int32)
         y = np.zeros((m, n), np.int16)
         acc = np.zeros((m, n), np.int64) if want_acc else None
-        _check(self.lib.oracle_linear_a16(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
-                                          _ptr(m0), _ptr(shift), int(zy), _ptr(y), n,
-                                          _ptr(acc) if acc is not None else None),
-               "oracle_linear_a16")
+        if zw is not None:
+            zw = np.ascontiguousarray(zw, dtype=np.int32)
+            _check(self.lib.oracle_linear_a16_asym(_ptr(x), m, k, k, int(zx), _ptr(packed), bits,
+                                                   n, _ptr(zw), _ptr(m0), _ptr(shift), int(zy),
+                                                   _ptr(y), n, _ptr(acc) if acc is not None
+                                                   else None), "oracle_linear_a16_asym")
+        else:
+            _check(self.lib.oracle_linear_a16(_ptr(x), m, k, k, int(zx), _ptr(packed), bits, n,
+                                              _ptr(m0), _ptr(shift), int(zy), _ptr(y), n,
+                                              _ptr(acc) if acc is not None else None),
+                   "oracle_linear_a16")
         return (y, acc) if want_acc else y
 
     def linear_points_a16(self, x: np.ndarray, zx: int, packed: np.ndarray, bits: int, n: int,
@@ -325,8 +335,8 @@ def requant_one(acc, m0, shift, zy):
     return _default().requant_one(acc, m0, shift, zy)
 
 
-def linear_a16(x, zx, packed, bits, n, m0, shift, zy, want_acc=False):
-    return _default().linear_a16(x, zx, packed, bits, n, m0, shift, zy, want_acc)
+def linear_a16(x, zx, packed, bits, n, m0, shift, zy, want_acc=False, zw=None):
+    return _default().linear_a16(x, zx, packed, bits, n, m0, shift, zy, want_acc, zw)
 
 
 def linear_points_a16(x, zx, packed, bits, n, m0, shift, zy, pts):

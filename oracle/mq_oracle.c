@@ -299,6 +299,33 @@ int oracle_linear_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
     return ORACLE_OK;
 }
 
+int oracle_linear_a16_asym(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                           const uint8_t *packed, int bits, int N, const int32_t *zw,
+                           const int32_t *M0, const int32_t *shift, int32_t zy, int16_t *y,
+                           int ldy, int64_t *acc_out) {
+    int rc = oracle_check_args_a16(M, K, ldx, bits, N, zx, zy);
+    if (rc != ORACLE_OK) return rc;
+    if (ldy < N) return ORACLE_EINVAL;
+    rc = oracle_check_zw(zw, N, bits);
+    if (rc != ORACLE_OK) return rc;
+    for (int m = 0; m < M; ++m) {
+        for (int n = 0; n < N; ++n) {
+            const int64_t zwn = zw ? (int64_t)zw[n] : 0;
+            int64_t acc = 0;
+            for (int k = 0; k < K; ++k) {
+                int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - (int64_t)zx;
+                int64_t wv = oracle_weight_at(packed, bits, K, n, k) - zwn;
+                acc += xv * wv;
+            }
+            if (acc_out) acc_out[(size_t)m * (size_t)N + (size_t)n] = acc;
+            if (y)
+                y[(size_t)m * (size_t)ldy + (size_t)n] =
+                    (int16_t)oracle_requant_one_a16(acc, M0[n], shift[n], zy);
+        }
+    }
+    return ORACLE_OK;
+}
+
 int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
                              const uint8_t *packed, int bits, int N,
                              const int32_t *M0, const int32_t *shift, int32_t zy,

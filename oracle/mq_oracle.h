@@ -165,6 +165,24 @@ int oracle_linear_o16(const int8_t *x, int M, int K, int ldx, int32_t zx,
                       const int32_t *M0, const int32_t *shift, int32_t zy, int16_t *y,
                       int ldy);
 
+/*
+ * 16-bit activations against weights (or 8-bit activations used as the
+ * "weights" operand) with a per-channel zero point: the matmul of self-
+ * attention in the paper's W8A16 setting, between 8-bit and 16-bit activations
+ * (Sec. 5.6, on-device setup), and asymmetric weights (Sec. 5.1) under 16-bit
+ * activations.  With x int16 [M][ldx], int8 / int4 w [N][K] and zw [N] in the
+ * weight code range (NULL: 0):
+ *   acc[m][n] = sum_k (x[m][k] - zx) * (w[n][k] - zw[n])      (int64)
+ *   y[m][n]   = oracle_requant_one_a16(acc[m][n], M0[n], shift[n], zy)
+ * Pinned by: exhaustive K=1 over every int16 code and every int8 weight code
+ * with zero points at the range ends, against exact integers and rationals;
+ * numpy's int64 matmul of the shifted operands; oracle_linear_a16 at zw = 0.
+ */
+int oracle_linear_a16_asym(const int16_t *x, int M, int K, int ldx, int32_t zx,
+                           const uint8_t *packed, int bits, int N, const int32_t *zw,
+                           const int32_t *M0, const int32_t *shift, int32_t zy, int16_t *y,
+                           int ldy, int64_t *acc_out);
+
 /* oracle_linear_a16 at listed output coordinates (as oracle_linear_points). */
 int oracle_linear_points_a16(const int16_t *x, int M, int K, int ldx, int32_t zx,
                              const uint8_t *packed, int bits, int N,

@@ -731,6 +731,46 @@ def pin_o16_matches_asym_and_requant16(orc: Oracle):
         assert (np.abs(y.astype(np.int64)) > 127).any()   # the 16-bit range is used
 
 
+def pin_a16_asym_k1_exhaustive(orc: Oracle):
+    # every int16 code x against int8 weight codes at the ends of the range and
+    # spread over it (K = 1), weight zero points at the ends and middle of the
+    # range: acc = (x - zx)(w - zw) exactly, and sampled outputs against round
+    # half up of exact rationals
+    xs = np.arange(-32768, 32768, dtype=np.int64).astype(np.int16).reshape(-1, 1)
+    ws = np.array([-128, -127, -100, -64, -17, -2, -1, 0, 1, 2, 19, 63, 64, 101, 126, 127],
+                  np.int8).reshape(-1, 1)
+    packed, _ = orc.pack(ws, 8)
+    n = ws.shape[0]
+    for zx, zwv in ((-32768, 127), (0, -128), (12345, -3)):
+        zw = np.full(n, zwv, np.int32)
+        m0, s, zy = (1 << 30) + 12345, 44, -77
+        y, acc = orc.linear_a16(xs, zx, packed, 8, n, np.full(n, m0, np.int32),
+                                np.full(n, s, np.int32), zy, want_acc=True, zw=zw)
+        ref = (xs.astype(np.int64) - zx) * (ws[:, 0].astype(np.int64) - zwv)[None, :]
+        assert np.array_equal(acc, ref), (zx, zwv)
+        for i in range(0, xs.shape[0], 3001):
+            for j in range(n):
+                assert int(y[i, j]) == _py_requant16(int(ref[i, j]), m0, s, zy), (zx, zwv, i, j)
+
+
+def pin_a16_asym_identity_and_reduction(orc: Oracle):
+    # numpy's int64 matmul of the shifted operands (int8 and int4 weights,
+    # per-channel zero points), and oracle_linear_a16 when every zw is 0
+    rng = np.random.default_rng(403)
+    for seed, bits in ((11, 8), (12, 4)):
+        c = synth.random_case_a16(seed, 6, 128, 17, bits, "mixed" if bits == 4 else None)
+        lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+        zw = rng.integers(lo, hi + 1, size=c.N).astype(np.int32)
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+        _, acc = orc.linear_a16(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy, want_acc=True, zw=zw)
+        ref = (c.x.astype(np.int64) - c.zx) @ (c.w.astype(np.int64) - zw[:, None]).T
+        assert np.array_equal(acc, ref), seed
+        y0 = orc.linear_a16(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy,
+                            zw=np.zeros(c.N, np.int32))
+        assert np.array_equal(y0, orc.linear_a16(c.x, c.zx, packed, bits, c.N, m0, sh, c.zy))
+
+
 PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zero_point_identity,
                pin_exact_dequant, pin_requant_closed_form, pin_requant_ties, pin_requant_vs_eq4,
                pin_requant_params_bound, pin_asym_k1_exhaustive, pin_asym_int4_pairs,
@@ -741,7 +781,8 @@ PIN_BATTERY = [pin_golden, pin_k1_exhaustive, pin_int4_exhaustive_pairs, pin_zer
                pin_quantize_exact, pin_quantize_ties_and_invariants, pin_dequantize_exact,
                pin_requantize_exhaustive, pin_requantize_vs_eq4, pin_fold_exact,
                pin_quantize_weights_exact, pin_fold_equivalence, pin_quantize_weights_properties,
-               pin_o16_k1_exhaustive, pin_o16_matches_asym_and_requant16]
+               pin_o16_k1_exhaustive, pin_o16_matches_asym_and_requant16,
+               pin_a16_asym_k1_exhaustive, pin_a16_asym_identity_and_reduction]
 
 
 # ----------------------------------------------------------------------------
@@ -1013,6 +1054,14 @@ def test_o16_matches_asym_and_requant16(O):
     pin_o16_matches_asym_and_requant16(O)
 
 
+def test_a16_asym_k1_exhaustive(O):
+    pin_a16_asym_k1_exhaustive(O)
+
+
+def test_a16_asym_identity_and_reduction(O):
+    pin_a16_asym_identity_and_reduction(O)
+
+
 MUTATIONS = [
     ("zero point sign", "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] - zx;",
      "int64_t xv = (int64_t)x[(size_t)m * (size_t)ldx + (size_t)k] + zx;"),
@@ -1072,6 +1121,12 @@ MUTATIONS = [
     ("o16 output narrowed to int8",
      "(int16_t)oracle_requant_one_a16(wide, M0[n], shift[n], zy);",
      "(int16_t)oracle_requant_one(wide, M0[n], shift[n], zy);"),
+    ("a16 weight zero point ignored",
+     "int64_t wv = oracle_weight_at(packed, bits, K, n, k) - zwn;",
+     "int64_t wv = oracle_weight_at(packed, bits, K, n, k);"),
+    ("a16 weight zero point sign",
+     "int64_t wv = oracle_weight_at(packed, bits, K, n, k) - zwn;",
+     "int64_t wv = oracle_weight_at(packed, bits, K, n, k) + zwn;"),
     ("o16 weight zero point ignored",
      "int64_t wide = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, zw ? zw[n] : 0);",
      "int64_t wide = oracle_dot_asym(x, K, ldx, zx, packed, bits, m, n, 0);"),
