@@ -57,7 +57,7 @@ WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
 # only for the kernel sources it was taken on: reported as null once they change.
 PREFILL_TRAFFIC_BYTES = 56_420_352 + 2_874_368
 PREFILL_TRAFFIC_SOURCES = ("mq_prefill.cu", "mq_ptx.cuh", "mq_internal.h")
-PREFILL_TRAFFIC_SHA = "b82109662bf341ea"
+PREFILL_TRAFFIC_SHA = "b9edf84356213752"
 
 
 def prefill_traffic():

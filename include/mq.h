@@ -207,7 +207,10 @@ int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, int32_t zx,
  * pre-pass that writes the planes as rows 2m and 2m+1 of a [2M][K] int8
  * matrix in the workspace.
  * Requirements: 0 <= M, N; 0 <= K <= MQ_MAX_K; K % 16 == 0; ldx % 8 == 0;
- * x and packed 16-byte aligned.  No residual and no weight zero point.  The
+ * x and packed 16-byte aligned.  No residual.  Weights with a zero point
+ * (the matmul of self-attention in the paper's W8A16 setting, between 16-bit
+ * and 8-bit activations, Sec. 5.6) go through mq_linear_batch with `zw` and
+ * abits 16: acc = sum_k (x - zx)(w - zw[n]), exact in int64 for every K.  The
  * stream rules of mq_linear_w8a8 apply.
  * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_K_OVERFLOW, MQ_ERR_ALIGNMENT,
  * MQ_ERR_WORKSPACE, MQ_ERR_CUDA.
@@ -253,8 +256,9 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
  *   acc[m][n] = sum_k (x[m][k] - zx) * (w[n][k] - zw[n])
  *             = sum_k x (w - zw[n]) - zx (colsum[n] - K zw[n])
  * zw[n] must lie in the weight code range ([-128, 127] for bits 8, [-8, 7]
- * for bits 4), and with int8 weights K <= MQ_MAX_K_ASYM8 (so that
- * |acc| <= 255 * 255 * K stays below 2^31).  No workspace beyond that of the
+ * for bits 4), and with int8 weights and 8-bit activations K <= MQ_MAX_K_ASYM8
+ * (so that |acc| <= 255 * 255 * K stays below 2^31; 16-bit activations
+ * accumulate in int64).  No workspace beyond that of the
  * symmetric case: the weights are widened to w - zw[n] on the fly.
  *
  *   descs     : host array of `count` descriptors (1 <= count <= MQ_MAX_BATCH)
@@ -287,7 +291,7 @@ typedef struct mq_linear_desc {
     const int32_t *M0;
     const int32_t *shift;
     const int8_t *residual; /* may be NULL; int8 activations only */
-    const int32_t *zw;      /* may be NULL: symmetric weights; int8 activations only */
+    const int32_t *zw;      /* may be NULL: symmetric weights */
     void *y;                /* int8 [M][ldy], or int16 with abits == 16 */
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;

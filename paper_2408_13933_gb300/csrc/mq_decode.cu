@@ -493,7 +493,8 @@ __device__ __forceinline__ void a16_epilogue(const Params &P, SM &s, const DecPr
 #pragma unroll
             for (int w = 0; w < CONS_WARPS; ++w) sum += s.part[w][e][ln];
         }
-        v[q] = (uint32_t)sum - (uint32_t)(C::BIAS * xsum);
+        // sum(plane (w - zw)) = sum(u plane) - (bias + zw) sum(plane)
+        v[q] = (uint32_t)sum - (uint32_t)((C::BIAS + s.row_zw[rows[q]]) * xsum);
     }
     if (have && !whole) {
         if (!finisher) {
@@ -735,9 +736,9 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
             if (threadIdx.x < UNIT_ROWS) {
                 // sum((x - zx)(w - zw)) = sum(x w) - zx colsum - zw sum(x) + K zx zw;
                 // the zw sum(x) term is taken per piece with the bias below
-                // (16-bit activations: colsum itself, the combine applies (128 - zx))
+                // (16-bit activations: colsum - K zw, the combine applies (128 - zx))
                 s.row_corr[threadIdx.x] =
-                    A16 ? prm_cs
+                    A16 ? (int32_t)((uint32_t)prm_cs - (uint32_t)p.K * (uint32_t)prm_zw)
                         : (int32_t)((uint32_t)(p.zx * prm_cs) -
                                     (uint32_t)p.K * (uint32_t)(p.zx * prm_zw));
                 s.row_zw[threadIdx.x] = prm_zw;

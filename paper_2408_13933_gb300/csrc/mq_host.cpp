@@ -29,13 +29,16 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     const int32_t zlo = ab == 8 ? -128 : -32768, zhi = ab == 8 ? 127 : 32767;
     const int32_t ylo = ob == 8 ? -128 : -32768, yhi = ob == 8 ? 127 : 32767;
     if (d.zx < zlo || d.zx > zhi || d.zy < ylo || d.zy > yhi) return MQ_ERR_INVALID_ARG;
-    if (ab == 16 && (d.residual || d.zw)) return MQ_ERR_INVALID_ARG;
+    if (ab == 16 && d.residual) return MQ_ERR_INVALID_ARG;
     if (ob == 16 && d.residual) return MQ_ERR_INVALID_ARG;
     const int64_t wrow = (int64_t)d.K * d.bits / 8;  // packed bytes of one weight row
     if (d.ldw < 0 || (d.ldw > 0 && d.ldw < wrow)) return MQ_ERR_INVALID_ARG;
     if (d.ldw % 16 != 0) return MQ_ERR_ALIGNMENT;
     if (d.K > MQ_MAX_K) return MQ_ERR_K_OVERFLOW;
-    if (d.zw && d.bits == 8 && d.K > MQ_MAX_K_ASYM8) return MQ_ERR_K_OVERFLOW;
+    // int32 accumulators of 8-bit activations with int8 weights and a zero point
+    // (16-bit activations accumulate in int64; their int8 planes stay below
+    // 128 * 255 * 65536 < 2^31)
+    if (d.zw && ab == 8 && d.bits == 8 && d.K > MQ_MAX_K_ASYM8) return MQ_ERR_K_OVERFLOW;
     if (d.M > 0 && d.N > 0) {
         if (!d.colsum || !d.M0 || !d.shift || !d.y || d.ldy < d.N) return MQ_ERR_INVALID_ARG;
         if (d.K > 0) {  // with K == 0 neither x nor the weights are read

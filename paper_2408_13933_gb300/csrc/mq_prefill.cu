@@ -596,9 +596,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const int tok0 = t.tt * TN + 64 * half;
             const int ntok = min(64, e.M - tok0);
             if constexpr (A16) {
-                // acc pairs hold each token's int64 sum 256 S(hi) + S(lo):
-                // sum((x - zx) w) = that + (128 - zx) colsum
-                const int64_t c16 = (int64_t)(128 - p.zx) * (int64_t)__ldg(p.colsum + ch);
+                // acc pairs hold each token's int64 sum 256 S(hi) + S(lo) of
+                // x (w - zw) (the converters widen w - zw):
+                // sum((x - zx)(w - zw)) = that + (128 - zx) (colsum - K zw)
+                const int64_t cs = (int64_t)__ldg(p.colsum + ch);
+                const int64_t c16 =
+                    (int64_t)(128 - p.zx) * (ZW ? cs - (int64_t)p.K * zw : cs);
                 int16_t *yp = reinterpret_cast<int16_t *>(e.y) + (size_t)(tok0 >> 1) * (size_t)e.ldy + ch;
                 const int n16 = ntok >> 1;
                 const size_t ldy16 = (size_t)e.ldy;
@@ -741,6 +744,7 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
         if (cudaFuncSetAttribute(prefill_kernel<false, false, false>, attr, smem) != cudaSuccess ||
             cudaFuncSetAttribute(prefill_kernel<false, false, true>, attr, smem) != cudaSuccess ||
             cudaFuncSetAttribute(prefill_kernel<true, false, false>, attr, smem) != cudaSuccess ||
+            cudaFuncSetAttribute(prefill_kernel<true, false, true>, attr, smem) != cudaSuccess ||
             cudaFuncSetAttribute(prefill_kernel<false, true, true>, attr, smem) != cudaSuccess)
             return MQ_ERR_CUDA;
         attr_done = dev;
@@ -754,7 +758,8 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
         for (int i = begin; i < begin + n; ++i) any_zw = any_zw || probs[i].zw != nullptr;
         // 16-bit outputs always take the zero-point variant (their time is the
         // epilogue's, not the widening's)
-        auto kern = probs[0].a16   ? prefill_kernel<true, false, false>
+        auto kern = probs[0].a16   ? (any_zw ? prefill_kernel<true, false, true>
+                                             : prefill_kernel<true, false, false>)
                     : probs[0].o16 ? prefill_kernel<false, true, true>
                     : any_zw       ? prefill_kernel<false, false, true>
                                    : prefill_kernel<false, false, false>;

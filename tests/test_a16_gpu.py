@@ -29,10 +29,11 @@ def assert_equal_int16(got: np.ndarray, want: np.ndarray, what: str):
 class A16Case:
     """Device operands of one 16-bit-activation problem and its oracle result."""
 
-    def __init__(self, case, m0=None, shift=None, share=None):
+    def __init__(self, case, m0=None, shift=None, share=None, zw=None):
         lib = mq()
         torch = torch_cuda()
         self.c = c = case
+        self.zw = None if zw is None else np.asarray(zw, np.int32)
         if share is not None:  # read the input of another case (same device buffer)
             c.x, c.zx = share.c.x, share.c.zx
         packed, colsum = lib.pack_weights(c.w, c.bits)
@@ -40,6 +41,7 @@ class A16Case:
             m0, shift = lib.requant_params(c.sw, c.sx, c.sy)
         self.m0, self.shift = np.asarray(m0, np.int32), np.asarray(shift, np.int32)
         self.dev = [upload(a) for a in (c.x, packed, colsum, self.m0, self.shift)]
+        self.zw_dev = upload(self.zw) if self.zw is not None else None
         if share is not None:
             self.dev[0] = share.dev[0]
         self.y = torch.full((c.M, max(c.N, 1)), 12345, dtype=torch.int16, device="cuda")
@@ -48,7 +50,7 @@ class A16Case:
         c = self.c
         x, packed, colsum, m0, sh = self.dev
         return mq().make_desc(x, c.zx, packed, colsum, c.N, m0, sh, c.zy, self.y, c.bits,
-                              abits=16)
+                              abits=16, zw=self.zw_dev)
 
     def run_single(self):
         c = self.c
@@ -67,7 +69,8 @@ class A16Case:
     def want(self):
         c = self.c
         packed, _ = oracle.pack(c.w, c.bits)
-        return oracle.linear_a16(c.x, c.zx, packed, c.bits, c.N, self.m0, self.shift, c.zy)
+        return oracle.linear_a16(c.x, c.zx, packed, c.bits, c.N, self.m0, self.shift, c.zy,
+                                 zw=self.zw)
 
 
 def run_batch(cases):
@@ -181,3 +184,61 @@ def test_a16_batch_mixed_widths_kernels_and_shared_inputs():
     for g in (g8, g4):
         assert_equal_int8(g.y.cpu().numpy(), oracle_y(g.case), f"batch {g.case.name}")
     assert int(torch.count_nonzero(ws[:dec])) == 0
+
+
+def run_desc(c):
+    # one 16-bit problem through the batch call (weight zero points are a
+    # descriptor field)
+    torch = torch_cuda()
+    lib = mq()
+    d = c.desc()
+    need = lib.workspace_size_batch([d])
+    ws = torch.zeros(max(need, 16), dtype=torch.uint8, device="cuda")
+    assert lib.linear_batch([d], workspace=ws, ws_bytes=need) == 0
+    torch.cuda.synchronize()
+    assert lib.check_device_status() == 0
+    return c.y.cpu().numpy()[:, :c.c.N], ws
+
+
+def ends(n, bits):
+    lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+    return np.where(np.arange(n) % 3 == 0, lo, np.where(np.arange(n) % 3 == 1, hi, 0)).astype(np.int32)
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("shape", SHAPES_PRE[:3] + SHAPES_DEC[:3], ids=lambda s: "x".join(map(str, s)))
+def test_a16_weight_zero_points(shape, bits):
+    # 16-bit activations against weights with per-channel zero points (the
+    # attention matmul of the W8A16 setting, keys or V as the 8-bit operand)
+    m, n, k = shape
+    rng = np.random.default_rng(m * 7 + n)
+    lo, hi = (-128, 127) if bits == 8 else (-8, 7)
+    c = A16Case(synth.random_case_a16(5 * m + n + k, m, k, n, bits),
+                zw=rng.integers(lo, hi + 1, size=n))
+    got, _ = run_desc(c)
+    assert_equal_int16(got, c.want(), f"a16 zw {shape} bits={bits}")
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("extreme", ["min", "max", "mixed"])
+@pytest.mark.parametrize("m", [1, 8, 150])
+def test_a16_weight_zero_points_extreme(m, extreme, bits):
+    # codes and zero points at the range ends: |plane (w - zw)| up to 128 * 255
+    c = A16Case(synth.random_case_a16(190 + m, m, 1024, 96, bits, extreme), zw=ends(96, bits))
+    got, _ = run_desc(c)
+    assert_equal_int16(got, c.want(), f"a16 zw extreme m={m} {extreme} bits={bits}")
+
+
+@pytest.mark.parametrize("m", [2, 24])
+def test_a16_weight_zero_points_k_limit(m):
+    # K = 65536 with codes and zero points at the range ends: the decode
+    # kernel's int32 plane sums reach 128 * 255 * 65536 < 2^31, the tensor-core
+    # kernel's 512-k chunks run 128 times
+    for bits in (8, 4):
+        c = A16Case(synth.random_case_a16(280 + m + bits, m, 65536, 40, bits, "max"),
+                    zw=ends(40, bits))
+        got, ws = run_desc(c)
+        assert_equal_int16(got, c.want(), f"a16 zw K=65536 m={m} bits={bits}")
+        if 2 * m <= 16:
+            dec = mq().workspace_size(1, 1, 0, 4)
+            assert int(torch_cuda().count_nonzero(ws[:dec])) == 0

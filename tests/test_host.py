@@ -225,8 +225,8 @@ def _desc16(mq, M, K, N, bits, **kw):
 
 
 def test_a16_validation_and_workspace(mq):
-    # 16-bit activations: zero points over the int16 range, no residual or
-    # weight zero point, 16-byte rows (ldx % 8), abits 8 or 16 only; every
+    # 16-bit activations: zero points over the int16 range, no residual,
+    # 16-byte rows (ldx % 8), abits 8 or 16 only; every
     # rejection happens before anything is launched
     def rc(d):
         return mq.lib.mq_linear_batch((mq.LinearDesc * 1)(d), 1, FAKE, 1 << 30, None)
@@ -234,7 +234,9 @@ def test_a16_validation_and_workspace(mq):
     assert rc(_desc16(mq, 4, 64, 32, 8, zx=32768)) == mq.MQ_ERR_INVALID_ARG
     assert rc(_desc16(mq, 4, 64, 32, 8, zy=-32769)) == mq.MQ_ERR_INVALID_ARG
     assert rc(_desc16(mq, 4, 64, 32, 8, residual=FAKE)) == mq.MQ_ERR_INVALID_ARG
-    assert rc(_desc16(mq, 4, 64, 32, 8, zw=FAKE)) == mq.MQ_ERR_INVALID_ARG
+    # weight zero points are allowed with 16-bit activations (int64 accumulators);
+    # with a residual the descriptor is still rejected before any launch
+    assert rc(_desc16(mq, 4, 64, 32, 8, zw=FAKE, residual=FAKE)) == mq.MQ_ERR_INVALID_ARG
     assert rc(_desc16(mq, 4, 64, 32, 8, ldx=68)) == mq.MQ_ERR_ALIGNMENT
     assert rc(_desc16(mq, 4, 48, 32, 4, ldx=48)) == mq.MQ_ERR_ALIGNMENT   # int4: K % 32
     assert rc(_desc16(mq, 4, 65552, 32, 8, ldx=65552)) == mq.MQ_ERR_K_OVERFLOW
