@@ -623,16 +623,21 @@ class AttentionSet:
     M0_S, SH_S = 1 << 30, 34     # scores: scale 2^-5 (int16 output)
     M0_O, SH_O = 1 << 30, 40     # outputs: scale 2^-11
     ZY_S, ZY_O = 0, -3
+    # the W8A16 setting: 16-bit Q and P against 8-bit keys and V, int16 outputs
+    SH_S16, SH_O16 = 41, 39
 
-    def __init__(self, mq, torch, layer: int, t: int):
-        a = synth.attention_operands(CONFIG_ID_PREFILL, layer, t)
+    def __init__(self, mq, torch, layer: int, t: int, bits16: bool = False):
+        a = synth.attention_operands(CONFIG_ID_PREFILL, layer, t, bits16=bits16)
+        self.bits16 = bits16
+        if bits16:
+            self.SH_S, self.SH_O = self.SH_S16, self.SH_O16
         self.ops_host = a
         H, G, D = a.heads, a.kv_heads, a.d
         dev = "cuda"
         up = lambda arr: torch.from_numpy(np.ascontiguousarray(arr)).to(dev)
         self.q, self.k, self.v, self.p = up(a.q), up(a.k), up(a.v), up(a.p)
         self.s = torch.empty((H, t, t), dtype=torch.int16, device=dev)
-        self.o = torch.empty((t, H * D), dtype=torch.int8, device=dev)
+        self.o = torch.empty((t, H * D), dtype=torch.int16 if bits16 else torch.int8, device=dev)
         # keys' row sums per KV head [G][T]; V^T of all heads at once [G d][T]
         # (head g is rows g d .. g d + d - 1) and its row sums [G d]
         self.colk = torch.empty((G, t), dtype=torch.int32, device=dev)
@@ -658,8 +663,9 @@ class AttentionSet:
         self.ws_s = torch.zeros(max(16, self.ws_s_bytes), dtype=torch.uint8, device=dev)
         self.ws_o = torch.zeros(max(16, self.ws_o_bytes), dtype=torch.uint8, device=dev)
         self.H, self.G, self.D, self.t = H, G, D, t
-        self.bytes = (self.q.numel() + self.k.numel() + self.v.numel() + 2 * self.s.numel()
-                      + self.p.numel() + self.o.numel())
+        self.bytes = (self.q.numel() * self.q.element_size() + self.k.numel() + self.v.numel()
+                      + 2 * self.s.numel() + self.p.numel() * self.p.element_size()
+                      + self.o.numel() * self.o.element_size())
 
     def enqueue(self, mq, sp, phase: str = "all"):
         lib, H, G, D, t = mq.lib, self.H, self.G, self.D, self.t
@@ -689,7 +695,8 @@ class AttentionSet:
             sc = synth.LinearCase(f"scores{h}", np.ascontiguousarray(a.q[:rows, h * D:(h + 1) * D]),
                                   a.zq, 0.0, kg, None, 8, 0.0, self.ZY_S)
             sc.zw = np.full(self.t, a.zk, np.int32)
-            out.append(ParityCheck("attention_w8a8_t1024", "o16", sc, rows,
+            leg = "attention_w8a16_t1024" if self.bits16 else "attention_w8a8_t1024"
+            out.append(ParityCheck(leg, "a16" if self.bits16 else "o16", sc, rows,
                                    self.s[h, :rows].cpu().numpy(),
                                    np.full(self.t, self.M0_S, np.int32),
                                    np.full(self.t, self.SH_S, np.int32)))
@@ -697,14 +704,14 @@ class AttentionSet:
             pc = synth.LinearCase(f"pv{h}", np.ascontiguousarray(a.p[h, :rows]), a.zp, 0.0, vt,
                                   None, 8, 0.0, self.ZY_O)
             pc.zw = np.full(D, a.zv, np.int32)
-            out.append(ParityCheck("attention_w8a8_t1024", "linear", pc, rows,
+            out.append(ParityCheck(leg, "a16" if self.bits16 else "linear", pc, rows,
                                    self.o[:rows, h * D:(h + 1) * D].cpu().numpy(),
                                    np.full(D, self.M0_O, np.int32),
                                    np.full(D, self.SH_O, np.int32)))
         return out
 
 
-def run_attention(mq, torch, reps: int = 60, check_rows: int = 4):
+def run_attention(mq, torch, reps: int = 60, check_rows: int = 4, bits16: bool = False):
     """Grouped-query attention's two integer matmuls of one TinyLlama layer at
     T = 1024 (the softmax between them is outside the integer layer): per step
     the key row sums of the 4 KV heads (one launch), S = Q K^T for 32 heads
@@ -714,7 +721,7 @@ def run_attention(mq, torch, reps: int = 60, check_rows: int = 4):
     layers' operands (about 300 MB, more than L2).  The host enqueues the timed
     steps behind a device sleep, so the region measures the device, not the
     ctypes call rate; a second pass times the two phases alone."""
-    sets = [AttentionSet(mq, torch, layer, ATT_T) for layer in range(ATT_SETS)]
+    sets = [AttentionSet(mq, torch, layer, ATT_T, bits16) for layer in range(ATT_SETS)]
     stream = torch.cuda.current_stream()
     sp = stream.cuda_stream
     launches = 0
@@ -745,9 +752,11 @@ def run_attention(mq, torch, reps: int = 60, check_rows: int = 4):
     b = sets[0]
     ops = 2 * 2 * b.t * b.t * b.D * b.H
     checks = b.checks(check_rows)
-    res = {"what": "S = Q K^T (int16 scores) and O = P V, 32 query heads over 4 KV heads, "
-                   "head dim 64, T = 1024; full T x T scores (the causal mask is applied by "
-                   "the softmax, not here)",
+    res = {"what": ("S = Q K^T (int16 scores) and O = P V, 32 query heads over 4 KV heads, "
+                    "head dim 64, T = 1024; full T x T scores (the causal mask is applied by "
+                    "the softmax, not here)"
+                    + ("; W8A16 setting: 16-bit Q and P against 8-bit keys and V (with their "
+                       "zero points), int16 outputs" if bits16 else "")),
            "us_per_layer": round(ms * 1e3, 2), "tops": round(ops / (ms * 1e-3) / 1e12, 1),
            "algorithmic_bytes": b.bytes,
            "gbs": round(b.bytes / (ms * 1e-3) / 1e9, 1),
@@ -792,7 +801,7 @@ def run_checks(checks) -> dict:
         else:
             m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
         if ck.kind == "a16":
-            y = oracle.linear_a16(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy)
+            y = oracle.linear_a16(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy, zw=c.zw)
         elif ck.kind == "o16":
             y = oracle.linear_o16(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy, zw=c.zw)
         else:
@@ -896,6 +905,8 @@ def main():
     checks += more
     attention, more = run_attention(mq, torch)
     checks += more
+    attention16, more = run_attention(mq, torch, bits16=True)
+    checks += more
     glue = run_glue(mq, torch)
     wpipe = run_weight_pipeline(mq, torch)
     peaks = measured_peaks()
@@ -948,6 +959,8 @@ def main():
                 "w4a8_m1_stream_us": decode["m1"]["stream_us"]},
         "attention_w8a8_t1024": {**attention,
                                  "frac_hbm": round(attention["gbs"] / hbm, 3)},
+        "attention_w8a16_t1024": {**attention16,
+                                  "frac_hbm": round(attention16["gbs"] / hbm, 3)},
         "boundary_quantizers": {"unit": "GB/s of input + output bytes", **glue},
         "weight_pipeline": {"what": "fold of eq. 1 + quantize + pack + colsum, 7 linears, "
                                     "176 MB of f32 weights", **wpipe},

@@ -516,13 +516,19 @@ __device__ __forceinline__ void a16_epilogue(const Params &P, SM &s, const DecPr
     if (finisher && !s.abort) {
         const int ntok = p.M >> 1;
         int16_t *y = reinterpret_cast<int16_t *>(p.y);
+        // The codes past K are zero-filled, so each of the unit's n_oob
+        // missing k has low plane -128 against a zero weight code: with a
+        // weight zero point it adds (0 - zw)(-128) to the low plane's sum,
+        // which the combine takes back (per row, like the colsum term).
+        const int64_t oob128 = p.K > 0 ? 128 * (int64_t)(p.tiles_m * C::KSTAGE - p.K) : 0;
         for (int i = threadIdx.x; i < UNIT_ROWS * ntok; i += CONS_THREADS) {
             const int row = i & (UNIT_ROWS - 1), j = i / UNIT_ROWS;
             const int n = rb * UNIT_ROWS + row;
             if (n >= p.N) continue;
             const int64_t a = 256 * (int64_t)yv[(2 * j) * YV_STRIDE + row] +
                               (int64_t)yv[(2 * j + 1) * YV_STRIDE + row] +
-                              (int64_t)(128 - p.zx) * (int64_t)s.row_corr[row];
+                              (int64_t)(128 - p.zx) * (int64_t)s.row_corr[row] -
+                              oob128 * (int64_t)s.row_zw[row];
             y[(size_t)j * (size_t)p.ldy + n] =
                 (int16_t)mq_requant16(a, s.row_m0[row], s.row_shift[row], p.zy);
         }

@@ -450,22 +450,25 @@ ROLE_ATT_Q, ROLE_ATT_K, ROLE_ATT_V, ROLE_ATT_P = 10, 11, 12, 13
 
 
 def attention_operands(config: int, layer: int, t: int, heads: int = 32, kv_heads: int = 4,
-                       d: int = 64, logit_std: float = 2.0) -> AttentionOperands:
+                       d: int = 64, logit_std: float = 2.0, bits16: bool = False) -> AttentionOperands:
     """Seeded stand-ins for the inputs of Q K^T and P V at T = t tokens.
 
     Q, K, V: N(0, 1) activations (4 outlier channels x20) quantized per tensor
     like every other activation here.  P: rows of softmax(N(0, logit_std)
     logits) over keys s <= query t (the causal mask; masked keys get
-    probability 0), coded as clip(rint(255 p) - 128, -128, 127)."""
+    probability 0), coded as clip(rint(255 p) - 128, -128, 127).  With bits16
+    (the W8A16 setting), Q and P are 16-bit codes: Q quantized per tensor to
+    int16, P coded as clip(rint(65535 p) - 32768, -32768, 32767), zero point
+    -32768; K and V stay 8-bit."""
     codes = []
     for role, width in ((ROLE_ATT_Q, heads * d), (ROLE_ATT_K, kv_heads * d),
                         (ROLE_ATT_V, kv_heads * d)):
         xf = float_activations(rng_for(config, layer, role, ROLE_X), t, width,
                                orng=rng_for(config, layer, role, ROLE_OUTLIER))
-        q, _, z = quantize_per_tensor(xf)
+        q, _, z = quantize_per_tensor(xf, 16 if (bits16 and role == ROLE_ATT_Q) else 8)
         codes.append((q, z))
     rng = rng_for(config, layer, ROLE_ATT_P, ROLE_X)
-    p = np.empty((heads, t, t), np.int8)
+    p = np.empty((heads, t, t), np.int16 if bits16 else np.int8)
     future = np.triu(np.ones((t, t), bool), 1)
     for h in range(heads):
         logits = rng.standard_normal((t, t), dtype=np.float32) * np.float32(logit_std)
@@ -473,6 +476,10 @@ def attention_operands(config: int, layer: int, t: int, heads: int = 32, kv_head
         logits -= logits.max(axis=1, keepdims=True)
         e = np.exp(logits)
         e /= e.sum(axis=1, keepdims=True)
-        p[h] = rint_clip(e * np.float32(255.0) - np.float32(128.0), -128, 127).astype(np.int8)
+        if bits16:
+            p[h] = rint_clip(e * np.float32(65535.0) - np.float32(32768.0), -32768,
+                             32767).astype(np.int16)
+        else:
+            p[h] = rint_clip(e * np.float32(255.0) - np.float32(128.0), -128, 127).astype(np.int8)
     (q, zq), (k, zk), (v, zv) = codes
-    return AttentionOperands(q, k, v, p, zq, zk, zv, -128, heads, kv_heads, d)
+    return AttentionOperands(q, k, v, p, zq, zk, zv, -32768 if bits16 else -128, heads, kv_heads, d)

@@ -242,3 +242,18 @@ def test_a16_weight_zero_points_k_limit(m):
         if 2 * m <= 16:
             dec = mq().workspace_size(1, 1, 0, 4)
             assert int(torch_cuda().count_nonzero(ws[:dec])) == 0
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("k", [0, 16, 64, 144, 1040, 2080])
+@pytest.mark.parametrize("m", [1, 3, 8, 20])
+def test_a16_weight_zero_points_ragged_k(m, k, bits):
+    # K not a multiple of the decode stage (128 k int8, 256 k int4): the
+    # zero-filled codes past K meet the zero point; K = 0: every output is
+    # requant(0) = zy.  m = 20 runs the tensor-core kernel.
+    if bits == 4 and k % 32:
+        pytest.skip("int4 K is a multiple of 32")
+    c = A16Case(synth.random_case_a16(700 + m + k + bits, m, k, 56, bits, "mixed"),
+                zw=ends(56, bits))
+    got, _ = run_desc(c)
+    assert_equal_int16(got, c.want(), f"a16 zw ragged K={k} m={m} bits={bits}")

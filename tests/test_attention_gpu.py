@@ -299,3 +299,55 @@ def test_transpose_into_a_padded_destination():
     got = dst.cpu().numpy()
     assert np.array_equal(got[:192, :70], a[:, 8:200].T)
     assert np.all(got[:192, 70:] == 5) and np.all(got[192:] == 5)   # padding untouched
+
+
+@pytest.mark.parametrize("t_q", [96, 2])
+def test_w8a16_setting_attention_matmuls(t_q):
+    # the W8A16 setting's attention: 16-bit Q against 8-bit keys (a head's
+    # slice through the row pitch, key zero point as zw), 16-bit P against 8-bit
+    # V^T (value zero point), int16 outputs; t_q = 96: tensor-core kernel (plane
+    # pre-pass), t_q = 2: decode kernel
+    torch = torch_cuda()
+    lib = mq()
+    rng = np.random.default_rng(77 + t_q)
+    T, H, G, D = 96, 4, 2, 64
+    rep = H // G
+    q = rng.integers(-32768, 32768, size=(t_q, H * D)).astype(np.int16)
+    kk = rng.integers(-128, 128, size=(T, G * D)).astype(np.int8)
+    v = rng.integers(-128, 128, size=(T, G * D)).astype(np.int8)
+    p = rng.integers(-32768, 32768, size=(H, t_q, T)).astype(np.int16)
+    zq, zk, zv, zp = 1234, -7, 100, -32768
+    qd, kd, vd, pd = upload(q), upload(kk), upload(v), upload(p)
+    keep = [qd, kd, vd, pd]
+    colk = lib.head_row_sums(kd, G)
+    vt = lib.transpose_i8(vd)                 # [G d][T]
+    colv = lib.row_sums(vt)
+    m0s, shs = np.full(T, 1 << 30, np.int32), np.full(T, 40, np.int32)
+    m0o, sho = np.full(D, 1 << 30, np.int32), np.full(D, 44, np.int32)
+    dev = [upload(a) for a in (m0s, shs, np.full(T, zk, np.int32), m0o, sho,
+                               np.full(D, zv, np.int32))]
+    keep += [colk, vt, colv] + dev
+    m0sd, shsd, zwk, m0od, shod, zwv = dev
+    s = torch.full((H, t_q, T), 3, dtype=torch.int16, device="cuda")
+    o = torch.full((t_q, H * D), 3, dtype=torch.int16, device="cuda")
+    keep += [s, o]
+    descs = [lib.make_desc(qd[:, h * D:(h + 1) * D], zq, kd[:, (h // rep) * D:], colk[h // rep],
+                           T, m0sd, shsd, 11, s[h], 8, zw=zwk, ldw=G * D, wdynamic=True)
+             for h in range(H)]
+    descs += [lib.make_desc(pd[h], zp, vt[(h // rep) * D:(h // rep + 1) * D],
+                            colv[(h // rep) * D:(h // rep + 1) * D], D, m0od, shod, -9,
+                            o[:, h * D:(h + 1) * D], 8, zw=zwv, wdynamic=True)
+              for h in range(H)]
+    assert all(d.abits == 16 and d.obits == 16 for d in descs)
+    _run(descs[:H], keep)
+    _run(descs[H:], keep)
+    for h in range(H):
+        g = h // rep
+        opk, _ = oracle.pack(np.ascontiguousarray(kk[:, g * D:(g + 1) * D]), 8)
+        want = oracle.linear_a16(np.ascontiguousarray(q[:, h * D:(h + 1) * D]), zq, opk, 8, T,
+                                 m0s, shs, 11, zw=np.full(T, zk, np.int32))
+        assert_equal(s[h].cpu().numpy(), want, f"w8a16 scores head {h}")
+        opk, _ = oracle.pack(np.ascontiguousarray(v[:, g * D:(g + 1) * D].T), 8)
+        want = oracle.linear_a16(np.ascontiguousarray(p[h]), zp, opk, 8, D, m0o, sho, -9,
+                                 zw=np.full(D, zv, np.int32))
+        assert_equal(o[:, h * D:(h + 1) * D].cpu().numpy(), want, f"w8a16 P V head {h}")
