@@ -14,8 +14,12 @@ more than the 129 MB L2), so no step reads another's data from L2.
 Reported beside it, measured in the same run: W4A8 decode of the same block's
 linears at M = 1, 4, 16 (weight GB/s), rotating over 12 layers (264 MB); and
 both with asymmetric weights in the paper's settings (W8A8 per tensor with a
-per-channel down projection; W4A8 per channel); and the 16-bit-activation
-baselines W8A16 (prefill) and W4A16 (decode at M = 1 and 8).
+per-channel down projection; W4A8 per channel); the 16-bit-activation
+baselines W8A16 (prefill) and W4A16 (decode at M = 1 and 8); one layer's
+attention matmuls at T = 1024 (Q K^T with int16 scores and P V; also in the
+W8A16 setting, 16-bit Q and P against 8-bit keys and V); the boundary
+quantizers; and the offline weight pipeline.  Every leg's parity sample is
+recomputed by the oracle in the cpu_baseline leg (rank 0, one GPU).
 
 Multi-GPU (torchrun, one rank per GPU): replicas only -- every rank runs the
 same workload on its own GPU, no collective on the data path; value is the
