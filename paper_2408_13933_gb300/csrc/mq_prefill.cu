@@ -139,8 +139,17 @@ struct Tile {
 
 __device__ __forceinline__ Tile tile_at(const Params &P, int tile) {
     Tile t;
-    t.pi = 0;
-    while (t.pi + 1 < P.count && tile >= P.p[t.pi + 1].tile_begin) ++t.pi;
+    // the last problem whose first tile is <= tile (binary search: the
+    // problem table lives in the kernel parameters, whose reads are slow)
+    int lo = 0, hi = P.count - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (P.p[mid].tile_begin <= tile)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    t.pi = lo;
     const Problem &p = P.p[t.pi];
     const int local = tile - p.tile_begin;
     t.tt = local % p.tiles_m;
