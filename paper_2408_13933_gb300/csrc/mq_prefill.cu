@@ -109,6 +109,7 @@ struct Params {
     int pre_w;                           // 1: load weights before griddep_wait (all constant)
     uint16_t pair_begin[MAX_PAIRS + 1];
     uint16_t sched[MAX_SCHED];
+    uint8_t sched_pi[MAX_SCHED];  // the problem of each table entry
     int *status;
 };
 
@@ -137,10 +138,9 @@ struct Tile {
     int nkb, kpc;  // stages, stages per exact f32 chunk
 };
 
-__device__ __forceinline__ Tile tile_at(const Params &P, int tile) {
-    Tile t;
-    // the last problem whose first tile is <= tile (binary search: the
-    // problem table lives in the kernel parameters, whose reads are slow)
+// The last problem whose first tile is <= tile (binary search: the problem
+// table lives in the kernel parameters, whose reads are slow).
+__device__ __forceinline__ int problem_of(const Params &P, int tile) {
     int lo = 0, hi = P.count - 1;
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
@@ -149,7 +149,12 @@ __device__ __forceinline__ Tile tile_at(const Params &P, int tile) {
         else
             hi = mid - 1;
     }
-    t.pi = lo;
+    return lo;
+}
+
+__device__ __forceinline__ Tile tile_of(const Params &P, int tile, int pi) {
+    Tile t;
+    t.pi = pi;
     const Problem &p = P.p[t.pi];
     const int local = tile - p.tile_begin;
     t.tt = local % p.tiles_m;
@@ -161,13 +166,19 @@ __device__ __forceinline__ Tile tile_at(const Params &P, int tile) {
 }
 
 // The i-th tile of pair `pair`, or -1 past its last one.
-__device__ __forceinline__ int pair_tile(const Params &P, int pair, int i) {
+// The i-th tile of pair `pair` (false past its last one).  The table gives
+// each entry's problem; round-robin tiles search for it.
+__device__ __forceinline__ bool pair_tile_at(const Params &P, int pair, int i, Tile &t) {
     if (P.use_table) {
         const int j = P.pair_begin[pair] + i;
-        return j < P.pair_begin[pair + 1] ? (int)P.sched[j] : -1;
+        if (j >= P.pair_begin[pair + 1]) return false;
+        t = tile_of(P, P.sched[j], P.sched_pi[j]);
+        return true;
     }
-    const int t = pair + i * P.npairs;
-    return t < P.total_tiles ? t : -1;
+    const int tile = pair + i * P.npairs;
+    if (tile >= P.total_tiles) return false;
+    t = tile_of(P, tile, problem_of(P, tile));
+    return true;
 }
 
 // Warp-uniform bounded waits: lane 0 polls, the verdict is broadcast.
@@ -317,9 +328,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             // the stream; activations only after it.
             uint32_t npre = 0;
             if (P.pre_w) {
-                int tile;
-                for (int ti = 0; npre < (uint32_t)S8 && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
-                    const Tile t = tile_at(P, tile);
+                Tile t;
+                for (int ti = 0; npre < (uint32_t)S8 && pair_tile_at(P, pair, ti, t); ++ti) {
                     const bool i4 = P.p[t.pi].bits == 4;
                     const int wrow = t.ct * TM + (int)rank * CM;
                     for (int kb = 0; kb < t.nkb && npre < (uint32_t)S8; ++kb, ++npre) {
@@ -332,9 +342,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             griddep_wait();
             uint32_t it = 0;
             bool ok = true;
-            int tile;
-            for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
-                const Tile t = tile_at(P, tile);
+            Tile t;
+            for (int ti = 0; ok && pair_tile_at(P, pair, ti, t); ++ti) {
                 const bool i4 = P.p[t.pi].bits == 4;
                 const uint32_t bytes = (i4 ? STA / 2 : STA) + STB;
                 const int wrow = t.ct * TM + (int)rank * CM;
@@ -362,9 +371,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const uint32_t idesc = idesc_f16_f32(TM, TN);
             uint32_t it = 0, chunks = 0;
             bool ok = true;
-            int tile;
-            for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
-                const Tile t = tile_at(P, tile);
+            Tile t;
+            for (int ti = 0; ok && pair_tile_at(P, pair, ti, t); ++ti) {
                 uint32_t fcol = 0;
                 int kc = 0;  // stage within the exact-f32 chunk
                 for (int kb = 0; kb < t.nkb; ++kb, ++it) {
@@ -445,9 +453,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         const uint32_t leader_sink = cluster_addr(&s.sink[warp - CONV_WARP0], 0);
         uint32_t it = 0;
         bool ok = true;
-        int tile;
-        for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
-            const Tile t = tile_at(P, tile);
+        Tile t;
+        for (int ti = 0; ok && pair_tile_at(P, pair, ti, t); ++ti) {
             const bool i4 = P.p[t.pi].bits == 4;
             // weight row arow widens to w - zw (zw = 0 for symmetric weights):
             // the MMA then sums x (w - zw) and the epilogue needs no rowsum(x)
@@ -545,9 +552,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         const uint32_t leader_f_empty = cluster_addr(&s.f_empty[0], 0);
         uint32_t chunks = 0;
         bool ok = true;
-        int tile;
-        for (int ti = 0; ok && (tile = pair_tile(P, pair, ti)) >= 0; ++ti) {
-            const Tile t = tile_at(P, tile);
+        Tile t;
+        for (int ti = 0; ok && pair_tile_at(P, pair, ti, t); ++ti) {
             const Problem &p = P.p[t.pi];
             const int ch = t.ct * TM + (int)rank * CM + quad * 32 + lane;
             const bool ch_in = ch < p.N;
@@ -710,12 +716,16 @@ int max_pairs(int dev) {
 // numbered problem by problem; work = stages + a fixed epilogue share.
 void lpt_schedule(Params &P, int npairs) {
     std::vector<std::pair<int, int>> work;  // (work, tile)
+    std::vector<uint8_t> tile_pi(P.total_tiles);
     work.reserve(P.total_tiles);
     for (int pi = 0; pi < P.count; ++pi) {
         const Problem &q = P.p[pi];
         const int tiles = q.tiles_m * ((q.N + TM - 1) / TM);
         const int w = (q.K + KS - 1) / KS + 2;
-        for (int i = 0; i < tiles; ++i) work.emplace_back(w, q.tile_begin + i);
+        for (int i = 0; i < tiles; ++i) {
+            work.emplace_back(w, q.tile_begin + i);
+            tile_pi[q.tile_begin + i] = (uint8_t)pi;
+        }
     }
     std::stable_sort(work.begin(), work.end(),
                      [](const std::pair<int, int> &a, const std::pair<int, int> &b) {
@@ -735,7 +745,10 @@ void lpt_schedule(Params &P, int npairs) {
     int at = 0;
     for (int i = 0; i < npairs; ++i) {
         P.pair_begin[i] = (uint16_t)at;
-        for (int tile : lists[i]) P.sched[at++] = (uint16_t)tile;
+        for (int tile : lists[i]) {
+            P.sched_pi[at] = tile_pi[tile];
+            P.sched[at++] = (uint16_t)tile;
+        }
     }
     P.pair_begin[npairs] = (uint16_t)at;
 }
