@@ -569,7 +569,9 @@ def run_weight_pipeline(mq, torch, reps: int = 5):
     colsum) over the TinyLlama block's seven f32 weight matrices (176 MB), in
     the paper's W8A8 setting (asymmetric per tensor, down per channel) and
     W4A8 (asymmetric per channel): microseconds per block and GB/s of f32
-    weights (each read twice: statistics, then codes)."""
+    weights (each read twice: statistics, then codes).  Each call allocates
+    its outputs on the host side, so the timed steps are enqueued behind a
+    device sleep and the region measures the device, not the call rate."""
     g = torch.Generator(device="cuda")
     g.manual_seed(9)
     mats = [(torch.randn((n, k), device="cuda", generator=g) * 0.02,
@@ -587,6 +589,7 @@ def run_weight_pipeline(mq, torch, reps: int = 5):
                 mq.fold_quantize_pack(w, bits, sc, s_in)
         block()
         torch.cuda.synchronize()
+        torch.cuda._sleep(100_000_000)  # about 50 ms: the host enqueues every step meanwhile
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(reps):

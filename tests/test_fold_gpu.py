@@ -50,7 +50,7 @@ def _want(w, s_in, s_out, bits, scheme):
 @pytest.mark.parametrize("bits", [8, 4])
 @pytest.mark.parametrize("scheme", [0, 1, 2])
 @pytest.mark.parametrize("factors", ["none", "in", "out", "both"])
-@pytest.mark.parametrize("shape", [(37, 200), (256, 2048), (5, 5632)],
+@pytest.mark.parametrize("shape", [(37, 200), (256, 2048), (5, 5632), (19, 202)],
                          ids=lambda s: "x".join(map(str, s)))
 def test_fold_quantize_pack(shape, factors, scheme, bits):
     n, k = shape
@@ -64,6 +64,59 @@ def test_fold_quantize_pack(shape, factors, scheme, bits):
     assert np.array_equal(got[1], want[1]), "colsum"
     if scheme != 0:
         assert np.array_equal(got[3], want[3]), "zero points"
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_fold_unaligned_rows(bits):
+    # weights and input scales one float past a 16-byte boundary: the kernels
+    # take their one-weight-per-load path even though K is a multiple of 4
+    torch = torch_cuda()
+    n, k = 24, 1024
+    w, s_in, s_out = _weights(31 + bits, n, k)
+    wbuf = torch.zeros(n * k + 1, dtype=torch.float32, device="cuda")
+    wbuf[1:] = torch.from_numpy(w.reshape(-1)).cuda()
+    sbuf = torch.zeros(k + 1, dtype=torch.float32, device="cuda")
+    sbuf[1:] = torch.from_numpy(s_in).cuda()
+    wd, sd = wbuf[1:].view(n, k), sbuf[1:]
+    assert wd.data_ptr() % 16 == 4 and sd.data_ptr() % 16 == 4
+    for scheme in (0, 1, 2):
+        packed, colsum, sw, zw = mq().fold_quantize_pack(wd, bits, scheme, sd, upload(s_out))
+        torch.cuda.synchronize()
+        want = _want(w, s_in, s_out, bits, scheme)
+        assert np.array_equal(packed.cpu().numpy().reshape(want[0].shape), want[0])
+        assert np.array_equal(colsum.cpu().numpy(), want[1])
+        assert np.array_equal(sw.cpu().numpy().view(np.uint32), want[2].view(np.uint32))
+        if scheme != 0:
+            assert np.array_equal(zw.cpu().numpy(), want[3])
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("scheme", [0, 1, 2])
+def test_fold_ties(bits, scheme):
+    # every row spans [-qmax, qmax] (symmetric) or [-qmax - 1, qmax] (the
+    # asymmetric schemes) times a power of two, so the scale is that power of
+    # two and the zero point 0; the other weights put v / scale exactly on a
+    # half-integer or one f32 step to either side, where the code turns on
+    # the tie rule of rint and on the quotient's last bit
+    qmax = 127 if bits == 8 else 7
+    step = np.float32(2.0 ** -7 if bits == 8 else 2.0 ** -3)
+    lo_k = -qmax if scheme == 0 else -qmax - 1
+    ties = (np.arange(lo_k, qmax, dtype=np.float32) + np.float32(0.5)) * step
+    vals = np.concatenate([ties, np.nextafter(ties, np.float32(np.inf)),
+                           np.nextafter(ties, np.float32(-np.inf))]).astype(np.float32)
+    rng = np.random.default_rng(50 + bits + scheme)
+    n, k = 16, 1024
+    w = rng.choice(vals, (n, k)).astype(np.float32)
+    w[:, 0] = np.float32(lo_k) * step
+    w[:, 1] = np.float32(qmax) * step
+    got = _run(w, None, None, bits, scheme)
+    want = _want(w, None, None, bits, scheme)
+    assert np.all(want[2] == step)
+    assert np.array_equal(got[2].view(np.uint32), want[2].view(np.uint32)), "scales"
+    assert np.array_equal(got[0].reshape(want[0].shape), want[0]), "packed codes"
+    assert np.array_equal(got[1], want[1]), "colsum"
+    if scheme != 0:
+        assert np.array_equal(got[3], want[3]) and not np.any(want[3]), "zero points"
 
 
 def test_fold_edge_shapes():
