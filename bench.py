@@ -57,8 +57,8 @@ WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
 
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one prefill_kernel launch on this
-# workload, from one ncu capture (profiles/prefill_kernel_tinyllama_block_w8a8_m1024.md), valid
-# only for the kernel sources it was taken on: reported as null once they change.
+# workload, read from one ncu capture of the kernel (its summary is committed under profiles/),
+# valid only for the kernel sources it was taken on: reported as null once they change.
 PREFILL_TRAFFIC_BYTES = 56_418_816 + 2_899_456
 PREFILL_TRAFFIC_SOURCES = ("mq_prefill.cu", "mq_ptx.cuh", "mq_internal.h")
 PREFILL_TRAFFIC_SHA = "05c0b6e06d34e88f"

@@ -115,7 +115,11 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed,
 int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes);
 
 /*
- * One quantized linear layer, int8 activations x int8 weights (W8A8).
+ * One quantized linear layer, int8 activations x int8 weights (W8A8): the
+ * integer-only linear of Sec. 3.1 (int8 x int8 products, int32 accumulation,
+ * fixed-point requantization) with the static per-tensor activation
+ * quantizer of eqs. 2-4 (Sec. 4.2) on its input (sx, zx) and output (sy, zy)
+ * and symmetric per-channel weights (Appendix A).
  *   x        : device int8 [M][ldx], ldx >= K
  *   zx       : input zero point in [-128, 127]
  *   packed   : device, from mq_pack_weights(bits = 8)
@@ -164,15 +168,17 @@ int mq_linear_w4a8(const int8_t *x, int M, int K, int ldx, int32_t zx,
  * program with no device allocator of its own, or a serving loop whose memory
  * pool is fixed after warm-up and must not grow mid-generation.  The split-K
  * combine scratch (2.5 MB) is a static device array inside libmq, one
- * per device; each call clears it on `stream` with a memset before the
- * kernel, and no call allocates or frees device memory.
+ * per device, and no call allocates or frees device memory.  The scratch
+ * needs no clearing: it starts zeroed, and each launch tags the sums it
+ * leaves there with its own launch number, so a later launch ignores them
+ * (also after MQ_ERR_DEVICE_TIMEOUT).
  *
  * The first call on each device does set-up with that device current: it
- * looks up the scratch's address and prepares the decode kernel.  Make that
- * first call before any stream capture.  Every call on a device shares the
- * one scratch, so calls must not overlap: two calls on different streams or
- * from different host threads race and give wrong results.  Calls issued in
- * order on one stream are fine.
+ * looks up the scratch's address and prepares both decode-kernel variants
+ * (M <= 8 and M > 8).  Make that first call before any stream capture.  Every
+ * call on a device shares the one scratch, so calls must not overlap: two
+ * calls on different streams or from different host threads race and give
+ * wrong results.  Calls issued in order on one stream are fine.
  *
  * Arguments and requirements as mq_linear_w4a8.  The result is identical to
  * mq_linear_w4a8 on the same inputs.
@@ -461,6 +467,41 @@ int mq_transpose_i8(const int8_t *src, int rows, int cols, int lds, int8_t *dst,
  * MQ_OK otherwise.  Clears the recorded status.
  */
 int mq_check_device_status(void *stream);
+
+/* ---- Failure detection ----------------------------------------------------
+ * The paper has no counterpart: these calls serve the library's own failure
+ * detection.  Every device-side wait of the kernels (a pipeline barrier, a
+ * split-K partner's partial sums) gives up after a time limit; the kernel
+ * then records MQ_ERR_DEVICE_TIMEOUT (see mq_check_device_status), abandons
+ * its work -- outputs are unspecified -- after letting its in-flight copies
+ * and tensor-core operations finish, and exits, so the CUDA context stays
+ * usable.
+ */
+
+/*
+ * Set the limit of every device-side wait, in nanoseconds, for the launches
+ * made after this call (process-wide, all devices).  0 restores the default
+ * of 1 second; values below 1000 are raised to 1000.  A short limit makes a
+ * wait that cannot complete end quickly in a test; in production a limit far
+ * above any real wait (the default) only bounds a hang.
+ * Errors: MQ_ERR_INVALID_ARG above 60 seconds.
+ */
+int mq_set_wait_limit_ns(uint64_t ns);
+
+/*
+ * Test hook, not for production: from this call on, CTA `cta` of every
+ * decode-kernel launch (mq_linear_* with M <= 16, the batch call's decode
+ * launches, mq_linear_w4a8_noalloc) skips storing the partial sums of a
+ * 64-row unit it shares with an earlier CTA.  The earlier CTA's bounded wait
+ * for them then runs out and the launch reports MQ_ERR_DEVICE_TIMEOUT: a
+ * split-K partner that never delivers, made on purpose without any fault.
+ * -1 (the initial state) turns it off.  After such a timeout a workspace
+ * keeps stale entries of that launch; the kernels ignore them (every launch
+ * tags its entries with its own number), and zero-filling it again restores
+ * the zero-filled state of the workspace contract.
+ * Errors: MQ_ERR_INVALID_ARG for cta < -1 or beyond the decode grid.
+ */
+int mq_test_skip_partials(int cta);
 
 #ifdef __cplusplus
 }

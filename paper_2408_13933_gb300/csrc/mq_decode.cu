@@ -94,7 +94,9 @@ struct Params {
     uint32_t epoch;      // nonzero, different for every launch
     int wide;            // total_stages * gridDim.x >= 2^32: 64-bit range arithmetic
     int pre_w;           // 1: load weights before griddep_wait (all constant)
+    int skip_cta;        // failure-detection test: this CTA stores no split-unit sums (-1: none)
     int *status;
+    uint64_t wait_ns;    // limit of every bounded wait
 };
 
 // What the kernel reads of a problem, kept in shared memory (the TMA tensor
@@ -256,7 +258,7 @@ __device__ __forceinline__ void ld_pair(const uint64_t *p, uint64_t &a, uint64_t
 // Wait (bounded, like every wait in this library) until the word carries
 // `epoch`; the word is returned in `w`.
 __device__ __forceinline__ bool poll_word(const uint64_t *p, uint32_t epoch, uint64_t &w,
-                                          volatile int *abort, int *status) {
+                                          volatile int *abort, int *status, uint64_t limit_ns) {
     uint64_t t0 = 0;
     while (true) {
         asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
@@ -265,7 +267,7 @@ __device__ __forceinline__ bool poll_word(const uint64_t *p, uint32_t epoch, uin
         const uint64_t t = global_timer_ns();
         if (t0 == 0) {
             t0 = t;
-        } else if (t - t0 > MQ_WAIT_LIMIT_NS) {
+        } else if (t - t0 > limit_ns) {
             *abort = 1;
             atomicOr(status, MQ_DEVICE_STATUS_TIMEOUT);
             return false;
@@ -275,8 +277,11 @@ __device__ __forceinline__ bool poll_word(const uint64_t *p, uint32_t epoch, uin
 }
 
 // A contributor's sums, stored with this launch's epoch; it does not wait.
+// (The failure-detection test names one CTA that skips its stores, so that
+// the finishing CTA's bounded wait for them runs out.)
 template <int NT>
 __device__ __forceinline__ void put_partials(const Params &P, int cta, const uint32_t (&v)[2 * NT]) {
+    if (cta == P.skip_cta) return;
     uint64_t *m = unit_entries<NT>(P, cta);
 #pragma unroll
     for (int q = 0; q < 2 * NT; q += 2)
@@ -311,7 +316,7 @@ __device__ __forceinline__ bool gather_partials(const Params &P, volatile int *a
 #pragma unroll
         for (int q = 0; q < 2 * NT; ++q) {
             if ((uint32_t)(e[q] >> 32) != P.epoch)
-                got = got && poll_word(src + q, P.epoch, e[q], abort, P.status);
+                got = got && poll_word(src + q, P.epoch, e[q], abort, P.status, P.wait_ns);
             v[q] += (uint32_t)e[q];
         }
     }
@@ -599,8 +604,17 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                 const int local = gs - p.tile_begin;
                 const int rb = local / p.tiles_m, j = local % p.tiles_m;
                 const int slot = it % STAGES;
-                if (!mq_wait_parity(&s.empty[slot], ((it / STAGES) & 1) ^ 1, &s.abort, P.status))
+                if (!mq_wait_parity(&s.empty[slot], ((it / STAGES) & 1) ^ 1, &s.abort, P.status,
+                                    P.wait_ns)) {
+                    // Given up: let the loads already issued land before the
+                    // CTA can leave (stages below `it` were issued whole -- the
+                    // waits of the first STAGES stages cannot fail -- and only
+                    // the last STAGES of them can still be in flight).
+                    for (uint32_t i = it > (uint32_t)STAGES ? it - STAGES : 0u; i < it; ++i)
+                        mq_wait_parity_drain(&s.full[i % STAGES], (i / STAGES) & 1, P.status,
+                                             P.wait_ns);
                     break;
+                }
                 if (p.K == 0) {  // an empty stage: nothing to load
                     mbar_arrive(&s.full[slot]);
                     continue;
@@ -693,7 +707,8 @@ __global__ void __launch_bounds__(THREADS, 2) decode_kernel(const __grid_constan
                 if (early && q == piece_end - 1) read_partials<NT>(P, cf + 1, first);
                 bool got = true;
                 if (lane == 0)
-                    got = mq_wait_parity(&s.full[slot], (it / STAGES) & 1, &s.abort, P.status);
+                    got = mq_wait_parity(&s.full[slot], (it / STAGES) & 1, &s.abort, P.status,
+                                         P.wait_ns);
                 if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) {
                     ok = false;
                     break;
@@ -864,19 +879,30 @@ uint32_t next_epoch() {
     return e;
 }
 
+// The kernel's dynamic shared-memory limit, raised once per device (the
+// attribute belongs to the device's context) and instantiation; safe to call
+// from several host threads.
+template <int BITS, int NT, bool A16, bool O16>
+int prepare_t(int dev) {
+    static std::atomic<uint64_t> done{0};  // bit d: device d prepared
+    if (dev < 0 || dev >= 64) return MQ_ERR_CUDA;
+    const uint64_t bit = 1ull << dev;
+    if (done.load(std::memory_order_acquire) & bit) return MQ_OK;
+    if (cudaFuncSetAttribute(decode_kernel<BITS, NT, A16, O16>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem_bytes<NT>()) != cudaSuccess)
+        return MQ_ERR_CUDA;
+    done.fetch_or(bit, std::memory_order_release);
+    return MQ_OK;
+}
+
 template <int BITS, int NT, bool A16, bool O16>
 int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t stream) {
     using C = Cfg<BITS>;
     auto kern = decode_kernel<BITS, NT, A16, O16>;
-    static int attr_done = -1;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
-    if (attr_done != dev) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem_bytes<NT>()) != cudaSuccess)
-            return MQ_ERR_CUDA;
-        attr_done = dev;
-    }
+    if (prepare_t<BITS, NT, A16, O16>(dev) != MQ_OK) return MQ_ERR_CUDA;
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return MQ_ERR_CUDA;
@@ -910,6 +936,8 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
         P.ws = reinterpret_cast<int2 *>(workspace);
         P.epoch = next_epoch();
         P.status = device_status_ptr();
+        P.wait_ns = wait_limit_ns();
+        P.skip_cta = test_skip_cta();
         long long grid = 2LL * sms;
         if (grid > DECODE_MAX_GRID) grid = DECODE_MAX_GRID;
         if (grid > stages) grid = stages;
@@ -932,6 +960,17 @@ int launch_t(const Problem *probs, int count, int32_t *workspace, cudaStream_t s
 }
 
 }  // namespace decode
+
+// Both token-tile variants of the W4A8 decode kernel (8-bit activations and
+// output) prepared on the current device.
+int prepare_decode_w4a8() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
+    if (decode::prepare_t<4, 1, false, false>(dev) != MQ_OK ||
+        decode::prepare_t<4, 2, false, false>(dev) != MQ_OK)
+        return MQ_ERR_CUDA;
+    return MQ_OK;
+}
 
 // All problems passed here have the same bits, a16 and o16 and M <= DECODE_MAX_M;
 // `workspace` holds DECODE_WS_BYTES, zero-filled.

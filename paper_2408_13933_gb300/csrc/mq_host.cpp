@@ -4,11 +4,25 @@
 // kernels, and device status reporting.
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstring>
 #include <vector>
 
 #include "mq_internal.h"
+
+namespace mq {
+
+namespace {
+constexpr uint64_t DEFAULT_WAIT_NS = 1000000000ull;  // 1 second
+std::atomic<uint64_t> g_wait_ns{DEFAULT_WAIT_NS};
+std::atomic<int> g_skip_cta{-1};
+}  // namespace
+
+uint64_t wait_limit_ns() { return g_wait_ns.load(std::memory_order_relaxed); }
+int test_skip_cta() { return g_skip_cta.load(std::memory_order_relaxed); }
+
+}  // namespace mq
 
 namespace {
 
@@ -543,6 +557,20 @@ int mq_transpose_i8(const int8_t *src, int rows, int cols, int lds, int8_t *dst,
     if (rows == 0 || cols == 0) return MQ_OK;
     if (!src || !dst) return MQ_ERR_INVALID_ARG;
     return mq::launch_transpose_i8(src, rows, cols, lds, dst, ldd, stream);
+}
+
+int mq_set_wait_limit_ns(uint64_t ns) {
+    if (ns == 0) ns = mq::DEFAULT_WAIT_NS;
+    if (ns < 1000) ns = 1000;
+    if (ns > 60000000000ull) return MQ_ERR_INVALID_ARG;
+    mq::g_wait_ns.store(ns, std::memory_order_relaxed);
+    return MQ_OK;
+}
+
+int mq_test_skip_partials(int cta) {
+    if (cta < -1 || cta >= mq::DECODE_MAX_GRID) return MQ_ERR_INVALID_ARG;
+    mq::g_skip_cta.store(cta, std::memory_order_relaxed);
+    return MQ_OK;
 }
 
 int mq_check_device_status(void *stream) {

@@ -58,11 +58,21 @@ constexpr int DECODE_MAX_PROBLEMS = 64;
 int *device_status_ptr();
 int *pack_status_ptr();
 
+// Limit of every bounded device-side wait, in nanoseconds, for the launches
+// made from now on (mq_set_wait_limit_ns; 1 second by default).
+uint64_t wait_limit_ns();
+// Failure-detection test hook (mq_test_skip_partials): the decode CTA whose
+// split-unit sums are not stored, or -1.
+int test_skip_cta();
+
 // Launchers (asynchronous on `stream`); return MQ_OK or MQ_ERR_CUDA.  The
 // problems of one launch_prefill call have the same a16 and o16; those of one
 // launch_decode call the same bits, a16 and o16.
 int launch_prefill(const Problem *probs, int count, void *stream);
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream);
+// Set-up of both token-tile variants of the W4A8 decode kernel on the current
+// device (done by the first launch of each variant otherwise).
+int prepare_decode_w4a8();
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
                 int *status, void *stream);
 // One row-sum job: out[m] = sum_k x[m][k] (mq_row_sums).

@@ -15,6 +15,14 @@
 // Calls on that device must therefore not overlap: two calls on different
 // streams, or from different host threads, race on the scratch and give
 // wrong results.  Calls issued one after another on one stream are fine.
+//
+// The scratch is never cleared by a call.  It starts zeroed (a static device
+// array), and the decode kernel only needs that no entry carries the current
+// launch's epoch before a contributor writes it: every launch has its own
+// epoch, the finishing CTA polls each entry until it carries that epoch, and
+// entries left behind by an earlier launch (also one that timed out) carry an
+// older one.  So nothing but the kernel itself sits between two consecutive
+// decode launches, and programmatic dependent launch can overlap them.
 #include <cuda_runtime.h>
 
 #include <atomic>
@@ -23,7 +31,8 @@
 
 namespace mq {
 
-// The decode kernel's combine scratch (counters, then per-CTA slots).
+// The decode kernel's combine scratch: per CTA of the decode grid one slot of
+// 64 x 16 {partial sum, launch epoch} entries, left zero by the kernel.
 static __device__ __align__(256) int32_t g_noalloc_scratch[DECODE_WS_BYTES / sizeof(int32_t)];
 
 namespace {
@@ -32,13 +41,16 @@ constexpr int MAX_DEVICES = 64;
 std::atomic<void *> g_scratch_addr[MAX_DEVICES];
 
 // The scratch's device address, looked up once per device with that device
-// current (on the first call made on it) and cached afterwards.
+// current (on the first call made on it) and cached afterwards; the same
+// first call prepares both variants of the decode kernel this entry point
+// launches, so that later calls do no set-up at all (e.g. inside a capture).
 void *scratch_ptr() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= MAX_DEVICES) return nullptr;
     void *p = g_scratch_addr[dev].load(std::memory_order_acquire);
     if (!p) {
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+        if (prepare_decode_w4a8() != MQ_OK) return nullptr;
         g_scratch_addr[dev].store(p, std::memory_order_release);
     }
     return p;
@@ -68,10 +80,6 @@ extern "C" int mq_linear_w4a8_noalloc(const int8_t *x, int M, int K, int ldx, in
 
     void *scratch = mq::scratch_ptr();
     if (!scratch) return MQ_ERR_CUDA;
-    // the kernel's counters and partial sums start at zero: clear them on the
-    // caller's stream, ahead of the kernel (a memset, no allocation)
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (cudaMemsetAsync(scratch, 0, mq::DECODE_WS_BYTES, s) != cudaSuccess) return MQ_ERR_CUDA;
 
     mq::Problem p{};
     p.x = x;

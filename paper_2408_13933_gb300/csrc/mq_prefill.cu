@@ -58,6 +58,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <queue>
 #include <vector>
 
@@ -111,6 +112,7 @@ struct Params {
     uint16_t sched[MAX_SCHED];
     uint8_t sched_pi[MAX_SCHED];  // the problem of each table entry
     int *status;
+    uint64_t wait_ns;                    // limit of every bounded wait
 };
 
 struct Smem {
@@ -182,10 +184,21 @@ __device__ __forceinline__ bool pair_tile_at(const Params &P, int pair, int i, T
 }
 
 // Warp-uniform bounded waits: lane 0 polls, the verdict is broadcast.
-__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, Smem &s, int *status) {
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, Smem &s,
+                                          const Params &P) {
     bool ok = true;
-    if ((threadIdx.x & 31) == 0) ok = mq_wait_parity(bar, parity, &s.abort, status);
+    if ((threadIdx.x & 31) == 0) ok = mq_wait_parity(bar, parity, &s.abort, P.status, P.wait_ns);
     return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+}
+
+// After a failed wait: raise the other CTA's abort word too, so that the pair
+// gives up together instead of the peer waiting out its own limit.  The peer
+// is still running: neither CTA leaves before the final cluster barrier, and
+// this store is ordered before this thread's arrival there.
+__device__ __forceinline__ void abort_pair(Smem &s, uint32_t rank) {
+    s.abort = 1;
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr(&s.abort, rank ^ 1u)),
+                 "r"(1u) : "memory");
 }
 
 
@@ -351,7 +364,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                     const int slot = it % S8;
                     if (!mq_wait_parity(&s.ld_empty[slot], ((it / S8) & 1) ^ 1, &s.abort,
-                                        P.status)) {
+                                        P.status, P.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -362,6 +375,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     }
                     tma_load_2d(s.stb[slot], &P.tmap_x[t.pi], kb * KS, xrow, &s.ld_full[slot]);
                 }
+            }
+            if (!ok) {
+                // Given up: let the loads already issued land before this CTA
+                // can leave (stages below `it` were issued whole -- the waits
+                // of the first S8 stages cannot fail -- and only the last S8
+                // of them can still be in flight).
+                abort_pair(s, rank);
+                for (uint32_t i = it > (uint32_t)S8 ? it - S8 : 0u; i < it; ++i)
+                    mq_wait_parity_drain(&s.ld_full[i % S8], (i / S8) & 1, P.status, P.wait_ns);
             }
         }
         __syncwarp();
@@ -380,7 +402,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     if (chunk_start) {
                         const uint32_t b = chunks & 1;
                         if (!mq_wait_parity(&s.f_empty[b], ((chunks >> 1) & 1) ^ 1, &s.abort,
-                                            P.status)) {
+                                            P.status, P.wait_ns)) {
                             ok = false;
                             break;
                         }
@@ -388,7 +410,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         fcol = F_COL0 + 128 * b;
                     }
                     const int slot = it % SF;
-                    if (!mq_wait_parity(&s.op_full[slot], (it / SF) & 1, &s.abort, P.status)) {
+                    if (!mq_wait_parity(&s.op_full[slot], (it / SF) & 1, &s.abort, P.status,
+                                        P.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -409,9 +432,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     }
                 }
             }
-            // every MMA issued above has completed once `done` fires
+            if (!ok) abort_pair(s, rank);
+            // every MMA issued above has completed once `done` fires; wait for
+            // it even after giving up (bounded, ignoring the abort word): the
+            // MMAs read both CTAs' operands and write their tensor memory,
+            // which is released after the final cluster barrier
             tc_commit2_mc(&s.done, 1);
-            mq_wait_parity(&s.done, 0, &s.abort, P.status);
+            mq_wait_parity_drain(&s.done, 0, P.status, P.wait_ns);
         }
         __syncwarp();
     } else if (warp < EPI_WARP0) {
@@ -468,8 +495,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                 if ((int)(it & 1) != grp) continue;
                 const int s8 = it % S8, sf = it % SF;
-                if (!warp_wait(&s.ld_full[s8], (it / S8) & 1, s, P.status) ||
-                    !warp_wait(&s.op_empty[sf], ((it / SF) & 1) ^ 1, s, P.status)) {
+                if (!warp_wait(&s.ld_full[s8], (it / S8) & 1, s, P) ||
+                    !warp_wait(&s.op_empty[sf], ((it / SF) & 1) ^ 1, s, P)) {
+                    if (lane == 0) abort_pair(s, rank);
                     ok = false;
                     break;
                 }
@@ -572,7 +600,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             const int nchunks = t.nkb ? (t.nkb + t.kpc - 1) / t.kpc : 0;
             for (int c = 0; c < nchunks; ++c, ++chunks) {
                 const uint32_t b = chunks & 1;
-                if (!warp_wait(&s.f_full[b], (chunks >> 1) & 1, s, P.status)) {
+                if (!warp_wait(&s.f_full[b], (chunks >> 1) & 1, s, P)) {
+                    if (lane == 0) abort_pair(s, rank);
                     ok = false;
                     break;
                 }
@@ -757,10 +786,12 @@ void lpt_schedule(Params &P, int npairs) {
 
 int launch_prefill(const Problem *probs, int count, void *stream) {
     using namespace prefill;
-    static int attr_done = -1;
+    // the kernels' dynamic shared-memory limit, raised once per device (the
+    // attribute belongs to the device's context)
+    static std::atomic<uint64_t> attr_done{0};  // bit d: device d prepared
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
-    if (attr_done != dev) {
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MQ_ERR_CUDA;
+    if (!(attr_done.load(std::memory_order_acquire) & (1ull << dev))) {
         const int smem = (int)SMEM_BYTES;
         const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
         if (cudaFuncSetAttribute(prefill_kernel<false, false, false>, attr, smem) != cudaSuccess ||
@@ -769,7 +800,7 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
             cudaFuncSetAttribute(prefill_kernel<true, false, true>, attr, smem) != cudaSuccess ||
             cudaFuncSetAttribute(prefill_kernel<false, true, true>, attr, smem) != cudaSuccess)
             return MQ_ERR_CUDA;
-        attr_done = dev;
+        attr_done.fetch_or(1ull << dev, std::memory_order_release);
     }
     if (count <= 0) return MQ_OK;
     const int pairs_max = max_pairs(dev);
@@ -819,6 +850,7 @@ int launch_prefill(const Problem *probs, int count, void *stream) {
         P.count = n;
         P.total_tiles = (int)tiles;
         P.status = device_status_ptr();
+        P.wait_ns = wait_limit_ns();
         P.npairs = tiles < pairs_max ? (int)tiles : pairs_max;
         P.use_table = tiles <= MAX_SCHED ? 1 : 0;
         if (P.use_table) lpt_schedule(P, P.npairs);

@@ -1,7 +1,8 @@
 // mq_ptx.cuh -- inline-PTX building blocks for the sm_103a kernels of libmq:
 // shared-memory mbarriers, tcgen05 (TMEM allocation, MMA, commit, loads and
-// stores), proxy fences and bounded waits.  Every wait in this library goes
-// through mq_wait_parity(), which gives up after MQ_WAIT_LIMIT_NS.
+// stores), proxy fences and bounded waits.  Every wait in this library gives
+// up after a time limit that the launcher passes in the kernel parameters
+// (mq_set_wait_limit_ns, 1 second by default).
 #pragma once
 
 #include <cstdint>
@@ -9,10 +10,6 @@
 #include "mq_internal.h"
 
 namespace mq {
-
-// Longest time any single device-side wait may take before the kernel
-// records MQ_ERR_DEVICE_TIMEOUT and abandons its work (1 second).
-constexpr uint64_t MQ_WAIT_LIMIT_NS = 1000000000ull;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -67,19 +64,37 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, uint32_t pari
 }
 
 // Wait until the phase with the given parity of `bar` has completed.  Gives up
-// (returns false) when `abort` becomes non-zero or after MQ_WAIT_LIMIT_NS; in
-// the latter case it raises `abort` and records the timeout in `status`.  The
+// (returns false) when `abort` becomes non-zero or after `limit_ns`; in the
+// latter case it raises `abort` and records the timeout in `status`.  The
 // waiting thread sleeps in hardware between checks instead of spinning, so it
 // takes no issue slots from the warps doing work.
 __device__ __forceinline__ bool mq_wait_parity(uint64_t *bar, uint32_t parity,
-                                               volatile int *abort, int *status) {
+                                               volatile int *abort, int *status,
+                                               uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     while (true) {
         if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
         if (*abort) return false;
-        if (global_timer_ns() - t0 > MQ_WAIT_LIMIT_NS) {
+        if (global_timer_ns() - t0 > limit_ns) {
             *abort = 1;
+            atomicOr(status, MQ_DEVICE_STATUS_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+// A bounded wait that ignores `abort`: for phases that are bound to complete
+// even after the kernel gave up on its work (tensor-core operations already
+// issued), which must be waited for before their operands' memory is
+// released.  Gives up after `limit_ns` and records a timeout then.
+__device__ __forceinline__ bool mq_wait_parity_drain(uint64_t *bar, uint32_t parity, int *status,
+                                                     uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (true) {
+        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+        if (global_timer_ns() - t0 > limit_ns) {
             atomicOr(status, MQ_DEVICE_STATUS_TIMEOUT);
             return false;
         }
@@ -169,13 +184,14 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t *bar, uint32_t pa
 // mq_wait_parity for phases completed by arrivals from other CTAs of the
 // cluster (remote arrives, multicast commits): acquire at cluster scope.
 __device__ __forceinline__ bool mq_wait_parity_cluster(uint64_t *bar, uint32_t parity,
-                                                       volatile int *abort, int *status) {
+                                                       volatile int *abort, int *status,
+                                                       uint64_t limit_ns) {
     const uint64_t t0 = global_timer_ns();
     for (uint32_t n = 0;; ++n) {
         if (mbar_try_wait_cluster(bar, parity)) return true;
         if ((n & 15) == 15) {
             if (*abort) return false;
-            if (global_timer_ns() - t0 > MQ_WAIT_LIMIT_NS) {
+            if (global_timer_ns() - t0 > limit_ns) {
                 *abort = 1;
                 atomicOr(status, MQ_DEVICE_STATUS_TIMEOUT);
                 return false;

@@ -41,7 +41,8 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_check_device_status", "mq_linear_w4a8_noalloc", "mq_workspace_size_batch",
             "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16", "mq_quantize",
             "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm",
-            "mq_row_sums", "mq_head_row_sums", "mq_transpose_i8"]
+            "mq_row_sums", "mq_head_row_sums", "mq_transpose_i8", "mq_set_wait_limit_ns",
+            "mq_test_skip_partials"]
 MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
@@ -85,6 +86,8 @@ lib.mq_fold_norm.argtypes = [_vp, _vp, _vp, _int, _vp, _vp]
 lib.mq_row_sums.argtypes = [_vp, _int, _int, _int, _vp, _vp]
 lib.mq_head_row_sums.argtypes = [_vp, _int, _int, _int, _int, _vp, _vp]
 lib.mq_transpose_i8.argtypes = [_vp, _int, _int, _int, _vp, _int, _vp]
+lib.mq_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
+lib.mq_test_skip_partials.argtypes = [_int]
 for _f in EXPORTED:
     if _f != "mq_status_string":
         getattr(lib, _f).restype = _int
@@ -365,3 +368,14 @@ def linear_batch(descs, stream=None, workspace=None, ws_bytes: int | None = None
 
 def check_device_status(stream=None) -> int:
     return lib.mq_check_device_status(_stream(stream))
+
+
+def set_wait_limit_ns(ns: int) -> int:
+    """mq_set_wait_limit_ns: the limit of every device-side wait of later
+    launches (0 restores the 1-second default)."""
+    return lib.mq_set_wait_limit_ns(int(ns))
+
+
+def test_skip_partials(cta: int) -> int:
+    """mq_test_skip_partials (failure-detection test hook; -1 turns it off)."""
+    return lib.mq_test_skip_partials(int(cta))

@@ -119,6 +119,43 @@ def test_fold_ties(bits, scheme):
         assert np.array_equal(got[3], want[3]) and not np.any(want[3]), "zero points"
 
 
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("scheme", [0, 1, 2])
+def test_fold_ties_general_scales(bits, scheme):
+    # scales that are not powers of two, so 1 / scale is inexact and the
+    # kernel's reciprocal product can land on the other side of a tie than the
+    # correctly rounded quotient: each row fixes its range with two end
+    # weights (scale and zero point follow from them), and every other weight
+    # is the f32 nearest to a half-integer multiple of the row's scale (the
+    # tensor's, per tensor), or up to three f32 steps to either side
+    qmax = 127 if bits == 8 else 7
+    qmin = -qmax if scheme == 0 else -qmax - 1
+    n, k = 24, 1024
+    rng = np.random.default_rng(70 + bits + scheme)
+    unit = (0.003 * (1.0 + rng.random(n) * 3.0)).astype(np.float32)   # about the scale
+    w = np.zeros((n, k), np.float32)
+    w[:, 0] = unit * np.float32(qmin)
+    w[:, 1] = unit * np.float32(qmax)
+    if scheme == 2:   # one range for the whole tensor
+        w[:, 0], w[:, 1] = w[:, 0].min(), w[:, 1].max()
+    sw = _want(w, None, None, bits, scheme)[2]   # the scales these ranges give
+    j = rng.integers(qmin, qmax, size=(n, k - 2)).astype(np.float64) + 0.5
+    mid = (j * sw[:, None].astype(np.float64)).astype(np.float32)     # nearest f32 to the tie
+    for _ in range(3):
+        step = rng.integers(-1, 2, size=mid.shape)
+        mid = np.where(step > 0, np.nextafter(mid, np.float32(np.inf)),
+                       np.where(step < 0, np.nextafter(mid, np.float32(-np.inf)), mid))
+    w[:, 2:] = np.clip(mid, w[:, :1], w[:, 1:2])
+    got = _run(w, None, None, bits, scheme)
+    want = _want(w, None, None, bits, scheme)
+    assert np.array_equal(want[2], sw), "the end weights fix the scales"
+    assert np.array_equal(got[2].view(np.uint32), want[2].view(np.uint32)), "scales"
+    assert np.array_equal(got[0].reshape(want[0].shape), want[0]), "packed codes"
+    assert np.array_equal(got[1], want[1]), "colsum"
+    if scheme != 0:
+        assert np.array_equal(got[3], want[3]), "zero points"
+
+
 def test_fold_edge_shapes():
     for n, k in ((1, 2), (3, 0), (1, 64)):
         w, _, _ = _weights(9, n, k)

@@ -1,12 +1,16 @@
 """mq_linear_w4a8_noalloc on the GPU against mq_linear_w4a8 (the workspace
-entry point, itself checked against the oracle by the parity tests): two calls
-in a row through the library's static scratch give the workspace path's
-output byte for byte.  The file name sorts last, so in a full run these tests
-also run after every other GPU test."""
+entry point) and against the oracle: two calls in a row through the
+library's static scratch give the workspace path's output and the oracle's
+byte for byte, and allocate no device memory (neither through PyTorch's
+caching allocator nor behind it: the device's free memory is unchanged).
+The file name sorts last, so in a full run these tests also run after every
+other GPU test."""
+import copy
+
 import numpy as np
 import pytest
 
-from gpu_helpers import torch_cuda, upload, workspace
+from gpu_helpers import oracle_y, torch_cuda, upload, workspace
 from paper_2408_13933_gb300 import synth
 
 pytestmark = pytest.mark.gpu
@@ -31,6 +35,14 @@ def prepare(m, n, k, seed):
     return c, x, upload(packed), upload(colsum), upload(m0), upload(sh)
 
 
+def oracle_of(c, k):
+    """The oracle's output of the case cut to its first k input features."""
+    o = copy.copy(c)
+    o.x = np.ascontiguousarray(c.x[:, :k])
+    o.w = np.ascontiguousarray(c.w[:, :k])
+    return oracle_y(o)
+
+
 @pytest.mark.parametrize("m,n,k", CASES)
 def test_noalloc_matches_workspace_entry_on_two_calls(m, n, k):
     torch = torch_cuda()
@@ -41,12 +53,15 @@ def test_noalloc_matches_workspace_entry_on_two_calls(m, n, k):
                       workspace=workspace()) == 0
     torch.cuda.synchronize()
     before = torch.cuda.memory_allocated()
+    free_before = torch.cuda.mem_get_info()[0]
     for y in ys[1:]:   # back to back on one stream, no synchronisation between
         assert lib.linear_w4a8_noalloc(x, c.zx, packed, colsum, n, m0, sh, c.zy, y, k=k) == 0
     torch.cuda.synchronize()
     assert lib.check_device_status() == 0
     assert torch.cuda.memory_allocated() == before
+    assert torch.cuda.mem_get_info()[0] == free_before
     want = ys[0].cpu().numpy()
+    assert np.array_equal(want, oracle_of(c, k)), "workspace entry point differs from the oracle"
     for i, y in enumerate(ys[1:]):
         got = y.cpu().numpy()
         assert np.array_equal(got, want), f"call {i + 1}: {int(np.sum(got != want))} differ"
