@@ -3,30 +3,35 @@
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mq|reference]
 
-Headline workload: the seven W8A8 linears of one TinyLlama-1.1B-shaped decoder
-block at prefill M = 1024 tokens (q 2048->2048, k/v 2048->256, o 2048->2048,
-gate/up 2048->5632, down 5632->2048; q/k/v/gate/up share one input), with the
-seeded int8 residual added to down's output.  One step = one pass over the
-block = one batched libmq launch (mq_linear_batch) of the tcgen05 prefill
-kernel.  Steps rotate over three layers' weights and activations (216 MB,
-more than the 129 MB L2), so no step reads another's data from L2.
+Headline workload (the largest single-GPU configuration): a 22-layer
+TinyLlama-1.1B-shaped stack of W8A8 linears at prefill M = 2048 tokens plus
+the 2048 -> 32000 head.  Per layer: q 2048->2048, k/v 2048->256, gate/up
+2048->5632 read x_l; o 2048->2048 reads q's int8 output and down 5632->2048
+reads up's; x_{l+1} = sat8(down + r_l) with a seeded int8 residual, fused
+into down's epilogue.  One step = the whole stack = 45 batched libmq calls
+(two per layer + the head), each one launch of the tcgen05 prefill kernel;
+4.24 T int8 ops and 1.03 GB of int8 weights per step.  `e2e` repeats it with
+x_0 uploaded from pinned host memory and the head's output downloaded every
+step.
 
-Reported beside it, measured in the same run: W4A8 decode of the same block's
-linears at M = 1, 4, 16 (weight GB/s), rotating over 12 layers (264 MB); and
-both with asymmetric weights in the paper's settings (W8A8 per tensor with a
-per-channel down projection; W4A8 per channel); the 16-bit-activation
-baselines W8A16 (prefill) and W4A16 (decode at M = 1 and 8); one layer's
-attention matmuls at T = 1024 (Q K^T with int16 scores and P V; also in the
-W8A16 setting, 16-bit Q and P against 8-bit keys and V); the boundary
-quantizers; and the offline weight pipeline.  Every leg's parity sample is
-recomputed by the oracle in the cpu_baseline leg (rank 0, one GPU).
+Reported beside it, measured in the same run: config 0 (one M = 128 linear),
+config 1 (the TinyLlama block at M = 1024, one launch), config 2 (W4A8 decode
+of that block at M = 1, 4, 16, weight GB/s over 12 rotated layers), config 4
+(the Gemma-2B-shaped block and its 256000-wide head: W8A8 prefill at M = 4096
+and W4A8 decode at M = 1); asymmetric weights in the paper's settings; the
+16-bit-activation baselines W8A16 / W4A16; one layer's attention matmuls at
+T = 1024 (also in the W8A16 setting); the boundary quantizers; and the
+offline weight pipeline.  The oracle re-computes every leg's parity sample
+in the cpu_baseline leg (rank 0, one GPU), where it is also timed on all
+host cores on a sample of the headline stack.
 
 Multi-GPU (torchrun, one rank per GPU): replicas only -- every rank runs the
 same workload on its own GPU, no collective on the data path; value is the
 total over ranks divided by the slowest rank's time.
 
---impl reference runs the CPU oracle (oracle/, plain C, one thread) on a
-bounded sample of the same workload: each step is one token row of the block.
+--impl reference runs the CPU oracle (oracle/, plain C, row blocks on every
+host core) on a bounded sample of the same workload: each step runs a few
+token rows of the stack through all 22 layers and the head.
 """
 from __future__ import annotations
 
@@ -51,9 +56,13 @@ PREFILL_M = 1024
 PREFILL_LAYERS = 3
 DECODE_LAYERS = 12
 DECODE_MS = (1, 4, 16)
+STACK_M, STACK_LAYERS = 2048, 22
 CONFIG_ID_PREFILL = 1
 CONFIG_ID_DECODE = 2
-WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
+CONFIG_ID_STACK = 3
+CONFIG_ID_GEMMA = 4
+WORKLOAD = "tinyllama-1.1b-shaped-22-layer-w8a8-stack-m2048-plus-head"
+BLOCK_WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
 
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one prefill_kernel launch on this
@@ -65,12 +74,26 @@ PREFILL_TRAFFIC_SHA = "05c0b6e06d34e88f"
 
 
 def prefill_traffic():
+    return PREFILL_TRAFFIC_BYTES if sources_sha() == PREFILL_TRAFFIC_SHA else None
+
+
+# DRAM traffic of one step of the headline stack (the sum over its 45 prefill_kernel launches), from
+# a one-pass ncu capture; None until one has been taken on the current kernel sources.
+STACK_TRAFFIC_BYTES = None
+STACK_TRAFFIC_SHA = None
+
+
+def sources_sha() -> str:
     import hashlib
     h = hashlib.sha256()
     for f in PREFILL_TRAFFIC_SOURCES:
         with open(os.path.join(ROOT, "paper_2408_13933_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
-    return PREFILL_TRAFFIC_BYTES if h.hexdigest()[:16] == PREFILL_TRAFFIC_SHA else None
+    return h.hexdigest()[:16]
+
+
+def stack_traffic():
+    return STACK_TRAFFIC_BYTES if STACK_TRAFFIC_SHA and sources_sha() == STACK_TRAFFIC_SHA else None
 
 
 def block_ops(m: int) -> int:
@@ -276,6 +299,8 @@ class DecodeLayer:
 
 
 def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
+    """Config 1: the TinyLlama-shaped block's seven W8A8 linears at M = 1024,
+    one batched launch per step, rotating over three layers."""
     blocks = [PrefillBlock(mq, torch, layer, PREFILL_M) for layer in range(PREFILL_LAYERS)]
     stream = torch.cuda.current_stream()
     sp = stream.cuda_stream
@@ -292,75 +317,21 @@ def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
     torch.cuda.synchronize()
     if mq.check_device_status() != 0:
         raise RuntimeError("device status error after warm-up")
-
     # No events between the launches of the timed region: consecutive launches
     # overlap (programmatic dependent launch) and an event between them would
     # serialize them.  The per-launch time is the region's time / launches.
-    clocks = ClockSampler(dist.local)
-    time.sleep(0.3)
-    dist.barrier()
-    torch.cuda.synchronize()
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
-    clocks.start()
-    t_start.record(stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
     for i in range(steps):
         step(i)
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    clocks.stop()
-    dist.barrier()
-    total_ms = t_start.elapsed_time(t_end)
-    kernel_ms = [total_ms / steps]
-    status = mq.check_device_status()
-    if status != 0:
-        raise RuntimeError(f"device status {mq.status_string(status)} after timed region")
-    max_total_ms = dist.max(total_ms)
-
-    # end to end through the public API: every step copies its inputs in from
-    # pinned host memory and its outputs back out.  The copies run on their own
-    # streams, so step i + 1's inputs upload and step i - 1's outputs download
-    # while step i computes; events order each layer's buffers between steps
-    # i and i + 3 (the layers rotate over three).
-    e2e_steps = min(steps, 300)
-    torch.cuda.synchronize()
-    dist.barrier()
-    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
-    nb = len(blocks)
-    in_done = [torch.cuda.Event() for _ in range(e2e_steps)]
-    comp_done = [torch.cuda.Event() for _ in range(e2e_steps)]
-    out_done = [torch.cuda.Event() for _ in range(e2e_steps)]
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    s_in.wait_event(e0)
-    s_out.wait_event(e0)
-    for i in range(e2e_steps):
-        b = blocks[i % nb]
-        with torch.cuda.stream(s_in):
-            if i >= nb:
-                s_in.wait_event(comp_done[i - nb])  # step i - 3 no longer reads x
-            b.x_all.copy_(b.x_all_host, non_blocking=True)
-            in_done[i].record(s_in)
-        stream.wait_event(in_done[i])
-        if i >= nb:
-            stream.wait_event(out_done[i - nb])  # step i - 3's outputs are copied out
-        step(i)
-        comp_done[i].record(stream)
-        with torch.cuda.stream(s_out):
-            s_out.wait_event(comp_done[i])
-            b.y_all_host.copy_(b.y_all, non_blocking=True)
-            out_done[i].record(s_out)
-    stream.wait_stream(s_out)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = dist.max(e0.elapsed_time(e1))
-    return {
-        "blocks": blocks, "total_ms": max_total_ms, "kernel_ms_mean": statistics.mean(kernel_ms),
-        "kernel_ms_median": statistics.median(kernel_ms), "clocks": clocks.result(),
-        "e2e_ms": e2e_ms, "e2e_steps": e2e_steps,
-        "h2d": blocks[0].h2d_bytes, "d2h": blocks[0].d2h_bytes,
-    }
+    status = mq.check_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {mq.status_string(status)} after the block run")
+    step(0)   # layer 0 last, for the parity sample
+    torch.cuda.synchronize()
+    return {"blocks": blocks, "total_ms": e0.elapsed_time(e1)}
 
 
 def run_decode(mq, torch, steps_per_m: int = 240, asym: bool = False, ms=DECODE_MS,
@@ -614,9 +585,10 @@ class ParityCheck:
     m0/sh given they are the device's fixed-point parameters; otherwise the
     oracle derives them from the case's float scales."""
 
-    def __init__(self, leg: str, kind: str, case, rows: int, got: np.ndarray, m0=None, sh=None):
+    def __init__(self, leg: str, kind: str, case, rows: int, got: np.ndarray, m0=None, sh=None,
+                 threaded: bool = False):
         self.leg, self.kind, self.case, self.rows, self.got = leg, kind, case, rows, got
-        self.m0, self.sh = m0, sh
+        self.m0, self.sh, self.threaded = m0, sh, threaded
 
 
 class AttentionSet:
@@ -773,6 +745,402 @@ def run_attention(mq, torch, reps: int = 60, check_rows: int = 4, bits16: bool =
     return res, checks
 
 
+# --------------------------------------------------------------------------- config 3: the stack
+def stack_ops(m: int = STACK_M, layers: int = STACK_LAYERS) -> int:
+    _, hk, hn = synth.TINYLLAMA_HEAD
+    return layers * block_ops(m) + 2 * m * hk * hn
+
+
+def stack_row_ops(layers: int = STACK_LAYERS) -> int:
+    return stack_ops(1, layers)
+
+
+class Stack:
+    """Device-resident config-3 model: 22 TinyLlama-shaped layers of seven
+    W8A8 linears at M tokens, chained as the workload defines (q/k/v/gate/up
+    read x_l; o reads q's output, down reads up's; x_{l+1} = sat8(down +
+    r_l)), and the 2048 -> 32000 head on x_22.  One step = 2 batched calls per
+    layer + the head = 45 prefill launches.  The step's input x_0 and its
+    result (the head's int8 output) are double-buffered so that the
+    end-to-end loop can upload step i + 1 and download step i - 1 while step i
+    computes; the seeded residuals r_l are model constants, resident like the
+    weights."""
+
+    def __init__(self, mq, torch, m: int = STACK_M, layers: int = STACK_LAYERS):
+        x0, _, _, self.layers, self.head = synth.chain_stack(CONFIG_ID_STACK, m, layers)
+        self.m, self.x0_np = m, x0
+        dev = "cuda"
+        up = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        self.keep = []
+        self.x0 = [up(x0) for _ in range(2)]
+        self.x0_host = torch.from_numpy(np.ascontiguousarray(x0)).pin_memory()
+        _, hk, hn = synth.TINYLLAMA_HEAD
+        self.hy = [torch.empty((m, hn), dtype=torch.int8, device=dev) for _ in range(2)]
+        self.hy_host = torch.empty((m, hn), dtype=torch.int8).pin_memory()
+        self.outs = []
+        calls_a, calls_b = [], []   # per x_0 / head buffer set
+
+        def dev_linear(c):
+            packed, colsum = mq.pack_weights(c.w, 8)
+            m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
+            t = [up(a) for a in (packed, colsum, m0, sh)]
+            self.keep += t
+            return t
+
+        def arr(descs):
+            return ((mq.LinearDesc * len(descs))(*descs), len(descs))
+
+        for li, L in enumerate(self.layers):
+            out = {c.name: torch.empty((m, c.N), dtype=torch.int8, device=dev) for c in L.cases}
+            self.outs.append(out)
+            res = up(L.residual)
+            self.keep.append(res)
+            cs = {c.name: c for c in L.cases}
+            w = {c.name: dev_linear(c) for c in L.cases}
+
+            def desc(name, xin, residual=None):
+                c, t = cs[name], w[name]
+                return mq.make_desc(xin, c.zx, t[0], t[1], c.N, t[2], t[3], c.zy, out[name], 8,
+                                    residual=residual)
+            xin = (self.x0[0], self.x0[1]) if li == 0 else (self.outs[li - 1]["down"],) * 2
+            for j, calls in enumerate((calls_a, calls_b)):
+                calls.append(arr([desc(nm, xin[j]) for nm in ("q", "k", "v", "gate", "up")]))
+            second = arr([desc("o", out["q"]), desc("down", out["up"], residual=res)])
+            calls_a.append(second)
+            calls_b.append(second)
+        ht = dev_linear(self.head)
+        h = self.head
+        for j, calls in enumerate((calls_a, calls_b)):
+            calls.append(arr([mq.make_desc(self.outs[-1]["down"], h.zx, ht[0], ht[1], h.N, ht[2],
+                                           ht[3], h.zy, self.hy[j], 8)]))
+        self.calls = (calls_a, calls_b)
+        self.launches = len(calls_a)
+        self.h2d_bytes = x0.size
+        self.d2h_bytes = m * hn
+
+    def enqueue(self, mq, sp: int, j: int = 0):
+        for a, n in self.calls[j]:
+            rc = mq.lib.mq_linear_batch(a, n, None, 0, sp)
+            if rc:
+                raise RuntimeError(f"mq_linear_batch failed: {mq.status_string(rc)}")
+
+
+def run_stack(mq, torch, dist: Dist, steps: int, warmup: int):
+    """The headline: config 3's 22-layer chained W8A8 stack + head at M = 2048,
+    device-resident (value, roofline), then end to end with host buffers."""
+    st = Stack(mq, torch)
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    for i in range(warmup):
+        st.enqueue(mq, sp, i & 1)
+    torch.cuda.synchronize()
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error after warm-up")
+    # No events between launches: consecutive launches overlap through
+    # programmatic dependent launch, and an event would serialize them.
+    clocks = ClockSampler(dist.local)
+    time.sleep(0.3)
+    dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks.start()
+    e0.record(stream)
+    for i in range(steps):
+        st.enqueue(mq, sp, i & 1)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks.stop()
+    dist.barrier()
+    total_ms = e0.elapsed_time(e1)
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error after the timed region")
+    max_total_ms = dist.max(total_ms)
+
+    # end to end: every step uploads x_0 from pinned host memory and downloads
+    # the head's output into pinned host memory, on their own streams, so that
+    # the copies of neighbouring steps overlap this step's kernels; buffer set
+    # j = i % 2 is reused two steps later, after its copies are done
+    e2e_steps = max(3, min(steps, 100))
+    torch.cuda.synchronize()
+    dist.barrier()
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    in_done = [torch.cuda.Event() for _ in range(e2e_steps)]
+    comp_done = [torch.cuda.Event() for _ in range(e2e_steps)]
+    out_done = [torch.cuda.Event() for _ in range(e2e_steps)]
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a0.record(stream)
+    s_in.wait_event(a0)
+    s_out.wait_event(a0)
+    for i in range(e2e_steps):
+        j = i & 1
+        with torch.cuda.stream(s_in):
+            if i >= 2:
+                s_in.wait_event(comp_done[i - 2])  # step i - 2 no longer reads x_0[j]
+            st.x0[j].copy_(st.x0_host, non_blocking=True)
+            in_done[i].record(s_in)
+        stream.wait_event(in_done[i])
+        if i >= 2:
+            stream.wait_event(out_done[i - 2])  # step i - 2's result is copied out
+        st.enqueue(mq, sp, j)
+        comp_done[i].record(stream)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(comp_done[i])
+            st.hy_host.copy_(st.hy[j], non_blocking=True)
+            out_done[i].record(s_out)
+    stream.wait_stream(s_out)
+    a1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = dist.max(a0.elapsed_time(a1))
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in the end-to-end run")
+    return {"stack": st, "total_ms": max_total_ms, "clocks": clocks.result(), "e2e_ms": e2e_ms,
+            "e2e_steps": e2e_steps, "h2d": st.h2d_bytes, "d2h": st.d2h_bytes,
+            "launches_per_step": st.launches}
+
+
+def stack_parity(st, rows):
+    """The oracle runs the stack's chain on `rows` from the seeded x_0 on every
+    host core (row blocks), and every layer's seven outputs and the head are
+    compared with the device's at those rows (the device buffers hold the
+    last step, which read the same x_0).  Returns the check and the oracle's
+    rate."""
+    import oracle
+    rows = np.asarray(rows)
+
+    def prep(c):
+        packed, _ = oracle.pack(c.w, 8)
+        m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
+        return packed, m0, sh
+    prepared = [{c.name: prep(c) for c in L.cases} for L in st.layers]
+    hp = prep(st.head)
+
+    def lin(c, p, xin):
+        return oracle.linear_mt(xin, c.zx, p[0], 8, c.N, p[1], p[2], c.zy)
+    outputs = mism = 0
+    xr = np.ascontiguousarray(st.x0_np[rows])
+    t0 = time.perf_counter()
+    want = []
+    for L, P in zip(st.layers, prepared):
+        cs = {c.name: c for c in L.cases}
+        ys = {nm: lin(cs[nm], P[nm], xr) for nm in ("q", "k", "v", "gate", "up")}
+        ys["o"] = lin(cs["o"], P["o"], ys["q"])
+        ys["down"] = oracle.residual_add(lin(cs["down"], P["down"], ys["up"]),
+                                         np.ascontiguousarray(L.residual[rows]))
+        want.append(ys)
+        xr = ys["down"]
+    hwant = lin(st.head, hp, xr)
+    secs = time.perf_counter() - t0
+    import torch
+    idx = torch.from_numpy(rows).cuda()
+    for out, ys in zip(st.outs, want):
+        for nm, y in ys.items():
+            got = out[nm].index_select(0, idx).cpu().numpy()
+            outputs += y.size
+            mism += int(np.count_nonzero(got != y))
+    got = st.hy[0].index_select(0, idx).cpu().numpy()
+    outputs += hwant.size
+    mism += int(np.count_nonzero(got != hwant))
+    ops = len(rows) * stack_row_ops()
+    return {"rows": len(rows), "outputs": outputs, "mismatches": mism}, ops, secs
+
+
+# --------------------------------------------------------------------------- config 0
+def run_single_linear(mq, torch, copies: int = 40, reps: int = 2000):
+    """Config 0: one W8A8 linear, M = 128, K = N = 2048 (1.07 G int8 ops, one
+    prefill launch), rotating over `copies` independent operand sets (180 MB
+    > L2): back to back, and with CUDA events around every launch."""
+    c = synth.make_linear(0, 0, 0, "cfg0", 128, 2048, 2048, 8)
+    packed, colsum = mq.pack_weights(c.w, 8)
+    m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
+    up = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    sets, keep, ys = [], [], []
+    for _ in range(copies):
+        t = [up(a) for a in (c.x, packed, colsum, m0, sh)]
+        y = torch.empty((128, 2048), dtype=torch.int8, device="cuda")
+        keep += t
+        ys.append(y)
+        sets.append((mq.LinearDesc * 1)(mq.make_desc(t[0], c.zx, t[1], t[2], 2048, t[3], t[4],
+                                                     c.zy, y, 8)))
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    call = mq.lib.mq_linear_batch
+    for i in range(2 * copies):
+        assert call(sets[i % copies], 1, None, 0, sp) == 0
+    torch.cuda.synchronize()
+    torch.cuda._sleep(50_000_000)  # the host enqueues the region meanwhile
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(reps):
+        call(sets[i % copies], 1, None, 0, sp)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(200)]
+    for i, (a, b) in enumerate(ev):
+        a.record(stream)
+        call(sets[i % copies], 1, None, 0, sp)
+        b.record(stream)
+    torch.cuda.synchronize()
+    kms = statistics.median(a.elapsed_time(b) for a, b in ev)
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in the config-0 run")
+    ops = 2 * 128 * 2048 * 2048
+    check = ParityCheck("config0_single_linear_m128", "linear", c, 128, ys[0].cpu().numpy(),
+                        threaded=True)
+    return {"what": "one W8A8 linear, M = 128, K = N = 2048", "int8_ops": ops,
+            "us_back_to_back": round(ms * 1e3, 2),
+            "tops_back_to_back": round(ops / (ms * 1e-3) / 1e12, 1),
+            "us_per_launch_events": round(kms * 1e3, 2),
+            "tops_per_launch_events": round(ops / (kms * 1e-3) / 1e12, 1),
+            "l2": f"{copies} operand sets rotated"}, [check]
+
+
+# --------------------------------------------------------------------------- config 4
+def gemma_block(m: int, bits: int, layer: int = 0):
+    return synth.block_linears(CONFIG_ID_GEMMA, m, bits, shapes=synth.GEMMA_LINEARS, layer=layer,
+                               t_rows_frac=0.01, shared_input=m > 16)
+
+
+def gemma_head(m: int, bits: int):
+    _, hk, hn = synth.GEMMA_HEAD
+    return synth.make_linear(CONFIG_ID_GEMMA, 0, 7, "head", m, hk, hn, bits, t_rows_frac=0.01)
+
+
+class DeviceCalls:
+    """Device operands and one batched call per group of cases (outputs
+    allocated on the device; the cases' inputs uploaded once per distinct x)."""
+
+    def __init__(self, mq, torch, groups, bits: int):
+        up = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+        xdev, self.keep, self.calls, self.y = {}, [], [], {}
+        for cases in groups:
+            descs = []
+            for c in cases:
+                if id(c.x) not in xdev:
+                    xdev[id(c.x)] = up(c.x)
+                packed, colsum = mq.pack_weights(c.w, bits)
+                m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
+                t = [up(a) for a in (packed, colsum, m0, sh)]
+                y = torch.empty((c.M, c.N), dtype=torch.int8, device="cuda")
+                self.keep += t + [y]
+                self.y[c.name] = y
+                descs.append(mq.make_desc(xdev[id(c.x)], c.zx, t[0], t[1], c.N, t[2], t[3],
+                                          c.zy, y, bits))
+            self.calls.append(((mq.LinearDesc * len(descs))(*descs), len(descs)))
+        self.keep += list(xdev.values())
+
+    def enqueue(self, mq, sp, ws=None, ws_bytes=0, which=None):
+        for i, (a, n) in enumerate(self.calls):
+            if which is None or i in which:
+                rc = mq.lib.mq_linear_batch(a, n, ws, ws_bytes, sp)
+                if rc:
+                    raise RuntimeError(f"mq_linear_batch failed: {mq.status_string(rc)}")
+
+
+def run_gemma_prefill(mq, torch, steps: int = 30, check_rows: int = 64):
+    """Config 4, prefill: the Gemma-2B-shaped block's seven W8A8 linears at
+    M = 4096 (one batched launch) and the 2048 -> 256000 head (one launch);
+    one step is both (0.90 + 4.29 T int8 ops; 630 MB of weights and a 1 GB
+    head output per step, far beyond L2)."""
+    cases, head = gemma_block(4096, 8), gemma_head(4096, 8)
+    dc = DeviceCalls(mq, torch, [cases, [head]], 8)
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    for _ in range(2):
+        dc.enqueue(mq, sp)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    times = {}
+    for name, which in (("step", None), ("block", (0,)), ("head", (1,))):
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(steps):
+            dc.enqueue(mq, sp, which=which)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        times[name] = e0.elapsed_time(e1) / steps
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in the config-4 prefill run")
+    bops = sum(2 * c.M * c.K * c.N for c in cases)
+    hops = 2 * head.M * head.K * head.N
+    checks = [ParityCheck("config4_gemma.prefill_m4096", "linear", c, check_rows,
+                          dc.y[c.name][:check_rows].cpu().numpy(), threaded=True)
+              for c in cases + [head]]
+    out = {"what": "Gemma-2B-shaped block (7 W8A8 linears, one launch) + 2048->256000 head "
+                   "(one launch) at M = 4096", "int8_ops_per_step": bops + hops,
+           "us_per_step": round(times["step"] * 1e3, 1),
+           "tops": round((bops + hops) / (times["step"] * 1e-3) / 1e12, 1),
+           "block_us": round(times["block"] * 1e3, 1),
+           "block_tops": round(bops / (times["block"] * 1e-3) / 1e12, 1),
+           "head_us": round(times["head"] * 1e3, 1),
+           "head_tops": round(hops / (times["head"] * 1e-3) / 1e12, 1), "steps": steps}
+    del dc
+    return out, checks
+
+
+def run_gemma_decode(mq, torch, reps: int = 20, block_layers: int = 4):
+    """Config 4, decode: the Gemma-2B-shaped block's seven W4A8 linears at
+    M = 1 (55.1 MB of int4 weights, one launch) and the 2048 -> 256000 head
+    (262 MB, one launch), timed back to back from CUDA graphs: the step
+    (block + head), the head alone, and the block alone rotating over
+    `block_layers` layers' weights (more than L2)."""
+    ws = mq.workspace()
+    wsp, wsn = ws.data_ptr(), ws.numel()
+    head = gemma_head(1, 4)
+    layers = []
+    for layer in range(block_layers):
+        cases = gemma_block(1, 4, layer=layer)
+        layers.append((cases, DeviceCalls(mq, torch, [cases] + ([[head]] if layer == 0 else []),
+                                          4)))
+    cases0, dc0 = layers[0]
+    bw = sum(c.K * c.N // 2 for c in cases0)
+    hw = head.K * head.N // 2
+    stream = torch.cuda.current_stream()
+
+    def graph_time(fn, n_inner):
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        fn(side.cuda_stream)   # warm-up outside the capture
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(g, stream=side):
+                fn(side.cuda_stream)
+        stream.wait_stream(side)
+        g.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        del g
+        return a.elapsed_time(b) / (reps * n_inner)
+
+    inner = 8
+    step_ms = graph_time(lambda s: [dc0.enqueue(mq, s, wsp, wsn) for _ in range(inner)], inner)
+    head_ms = graph_time(lambda s: [dc0.enqueue(mq, s, wsp, wsn, which=(1,))
+                                    for _ in range(inner)], inner)
+    block_ms = graph_time(lambda s: [dc.enqueue(mq, s, wsp, wsn, which=(0,))
+                                     for _ in range(2) for _, dc in layers], 2 * block_layers)
+    if mq.check_device_status() != 0:
+        raise RuntimeError("device status error in the config-4 decode run")
+    checks = [ParityCheck("config4_gemma.decode_w4a8_m1", "linear", c, 1,
+                          dc0.y[c.name].cpu().numpy()) for c in cases0 + [head]]
+    gbs = lambda b, ms: round(b / (ms * 1e-3) / 1e9, 1)
+    out = {"what": "Gemma-2B-shaped block (7 W4A8 linears, one launch) + 2048->256000 head "
+                   "(one launch) at M = 1, back to back from CUDA graphs",
+           "weight_bytes_per_step": bw + hw, "step_us": round(step_ms * 1e3, 2),
+           "step_gbs": gbs(bw + hw, step_ms), "head_weight_bytes": hw,
+           "head_us": round(head_ms * 1e3, 2), "head_gbs": gbs(hw, head_ms),
+           "block_weight_bytes": bw, "block_us": round(block_ms * 1e3, 2),
+           "block_gbs": gbs(bw, block_ms), "block_layers_rotated": block_layers}
+    del layers, dc0
+    return out, checks
+
+
 # --------------------------------------------------------------------------- CPU oracle
 def oracle_sample(blocks_cases, rows: range, col_frac: float = 1.0):
     """Run the oracle on `rows` of every linear of one block; returns
@@ -812,7 +1180,8 @@ def run_checks(checks) -> dict:
         elif ck.kind == "o16":
             y = oracle.linear_o16(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy, zw=c.zw)
         else:
-            y = oracle.linear(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy, zw=c.zw)
+            fn = oracle.linear_mt if ck.threaded else oracle.linear
+            y = fn(x, c.zx, packed, c.bits, c.N, m0, sh, c.zy, zw=c.zw)
             if c.residual is not None:
                 y = oracle.residual_add(y, np.ascontiguousarray(c.residual[:ck.rows]))
         r = out.setdefault(ck.leg, {"rows": ck.rows, "outputs": 0, "mismatches": 0})
@@ -821,50 +1190,75 @@ def run_checks(checks) -> dict:
     return out
 
 
-def cpu_baseline(blocks, torch, rows: int = 192, checks=()):
-    """The oracle timed on `rows` token rows of the headline block, its
-    outputs compared with the GPU's; then the other legs' parity samples."""
-    cases = blocks[0].cases
+def cpu_baseline(st, rows: int = 128, checks=()):
+    """The oracle timed on every host core (row blocks) on `rows` token rows of
+    the headline stack, spread over its 2048, through all 22 layers and the
+    head; its outputs are compared with the device's at every layer.  Then
+    the other legs' parity samples."""
     import oracle
     oracle.build()
-    ops, secs, outs = oracle_sample(cases, range(0, rows))
-    # the GPU's outputs for the same rows of layer 0 (last written by the
-    # e2e loop, which ran layer 0's block at least once)
-    torch.cuda.synchronize()
-    checked = mism = 0
-    for j, y in outs.items():
-        got = blocks[0].y[j][:rows].cpu().numpy()
-        checked += y.size
-        mism += int(np.count_nonzero(got != y))
-    base = {"value": round(ops / secs / 1e12, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
-            "sample": f"rows 0..{rows - 1} of all 7 linears of layer 0 (+ residual): "
-                      f"{ops / 1e9:.1f} GOP of the {block_ops(PREFILL_M) / 1e9:.1f} GOP block",
-            "seconds": round(secs, 2),
-            "parity_sample": {"outputs": checked, "mismatches": mism}}
+    sel = np.linspace(0, st.m - 1, rows).round().astype(np.int64)
+    par, ops, secs = stack_parity(st, sel)
+    base = {"value": round(ops / secs / 1e12, 6), "unit": "TOPS", "cores": oracle.threads(),
+            "kind": "oracle",
+            "sample": f"{rows} token rows spread over the {st.m} through all {len(st.layers)} "
+                      f"layers' 7 linears (+ residual) and the head: {ops / 1e9:.0f} G of the "
+                      f"{stack_ops() / 1e12:.2f} T int8 ops of a step, row blocks on every core",
+            "seconds": round(secs, 2), "parity_sample": par}
     return base, run_checks(checks)
 
 
+def reference_stack_sample(st_cases, rows: np.ndarray, prepared, nthreads: int):
+    """One reference step: the oracle's chain on `rows` of the stack."""
+    import oracle
+    x0, layers, head = st_cases
+    xr = np.ascontiguousarray(x0[rows])
+
+    def lin(c, p, xin):
+        return oracle.linear_mt(xin, c.zx, p[0], 8, c.N, p[1], p[2], c.zy, nthreads=nthreads)
+    for L, P in zip(layers, prepared[0]):
+        cs = {c.name: c for c in L.cases}
+        ys = {nm: lin(cs[nm], P[nm], xr) for nm in ("q", "up")}
+        for nm in ("k", "v", "gate"):
+            lin(cs[nm], P[nm], xr)
+        lin(cs["o"], P["o"], ys["q"])
+        xr = oracle.residual_add(lin(cs["down"], P["down"], ys["up"]),
+                                 np.ascontiguousarray(L.residual[rows]))
+    lin(head, prepared[1], xr)
+    return len(rows) * stack_row_ops()
+
+
 def run_reference(args, dist: Dist):
-    """Reference arm: the CPU oracle timed on this host, one token row of the
-    block per step (a bounded sample of the same workload)."""
+    """Reference arm: the CPU oracle timed on this host's cores on a bounded
+    sample of the headline workload: each step runs a few token rows of the
+    stack through all 22 layers and the head (row blocks on every core)."""
     if dist.rank != 0:
         return
     import oracle
     oracle.build()
-    cases = synth.block_linears(CONFIG_ID_PREFILL, PREFILL_M, 8, layer=0, shared_input=True)
-    cases[-1].residual = synth.residual_codes(CONFIG_ID_PREFILL, 0, PREFILL_M, cases[-1].N)
+    x0, _, _, layers, head = synth.chain_stack(CONFIG_ID_STACK, STACK_M, STACK_LAYERS)
+
+    def prep(c):
+        packed, _ = oracle.pack(c.w, 8)
+        m0, sh = oracle.requant_params(c.sx, c.sw, c.sy)
+        return packed, m0, sh
+    prepared = ([{c.name: prep(c) for c in L.cases} for L in layers], prep(head))
+    cores = oracle.threads()
+    cases = (x0, layers, head)
     # size the per-step sample so that warm-up + steps take about 90 s at most
-    _, t_row, _ = oracle_sample(cases, range(0, 1))
+    t0 = time.perf_counter()
+    reference_stack_sample(cases, np.arange(cores), prepared, cores)
+    t_step = time.perf_counter() - t0
     budget = 90.0
-    frac = min(1.0, budget / max(1e-9, (args.steps + args.warmup) * t_row))
+    rows = cores if (args.steps + args.warmup) * t_step <= budget else max(
+        1, int(cores * budget / ((args.steps + args.warmup) * t_step)))
+    pick = lambda i: (np.arange(rows) * 131 + 17 * i) % STACK_M
     for i in range(args.warmup):
-        oracle_sample(cases, range(i % PREFILL_M, i % PREFILL_M + 1), frac)
+        reference_stack_sample(cases, pick(i), prepared, cores)
     ops = 0
     t0 = time.perf_counter()
     for i in range(args.steps):
-        r = (args.warmup + i) % PREFILL_M
-        o, _, _ = oracle_sample(cases, range(r, r + 1), frac)
-        ops += o
+        ops += reference_stack_sample(cases, pick(args.warmup + i), prepared, cores)
     secs = time.perf_counter() - t0
     value = ops / secs / 1e12
     line = {
@@ -872,11 +1266,12 @@ def run_reference(args, dist: Dist):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs * 1e3 / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD, "tokens": PREFILL_M, "layers_rotated": 1,
-                   "sample_per_step": f"1 token row x {frac:.3f} of the output columns of "
-                                      "all 7 linears"},
-        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1, "kind": "oracle",
-                         "sample": "one token row of the block per step"},
+        "config": {"workload": WORKLOAD, "tokens": STACK_M, "layers": STACK_LAYERS,
+                   "sample_per_step": f"{rows} token rows through all {STACK_LAYERS} layers' "
+                                      "7 linears and the head"},
+        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": cores, "kind": "oracle",
+                         "sample": f"{rows} token rows of the stack per step, row blocks on "
+                                   f"{cores} threads"},
         "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -886,8 +1281,8 @@ def run_reference(args, dist: Dist):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawTextHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=3000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mq", "reference"], default="mq")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -904,9 +1299,22 @@ def main():
     build.build()
     from paper_2408_13933_gb300 import mq
 
-    pre = run_prefill(mq, torch, dist, args.steps, args.warmup)
+    stack = run_stack(mq, torch, dist, args.steps, args.warmup)
+    checks = []
+    cfg0, more = run_single_linear(mq, torch)
+    checks += more
+    pre = run_prefill(mq, torch, dist, 2000, 5)
+    checks += [ParityCheck("config1_tinyllama_block_m1024", "linear", c, 64,
+                           pre["blocks"][0].y[j][:64].cpu().numpy(), threaded=True)
+               for j, c in enumerate(pre["blocks"][0].cases)]
+    del pre["blocks"]
     decode = run_decode(mq, torch)
-    asym_pre, checks = run_asym_prefill(mq, torch)
+    g_pre, more = run_gemma_prefill(mq, torch)
+    checks += more
+    g_dec, more = run_gemma_decode(mq, torch)
+    checks += more
+    asym_pre, more = run_asym_prefill(mq, torch)
+    checks += more
     asym_dec = run_decode(mq, torch, asym=True, ms=(1, 16))
     a16, more = run_a16(mq, torch)
     checks += more
@@ -918,11 +1326,12 @@ def main():
     wpipe = run_weight_pipeline(mq, torch)
     peaks = measured_peaks()
 
-    ops = block_ops(PREFILL_M)
-    ms_per_step = pre["total_ms"] / args.steps
-    value = whole_job_rate(ops * args.steps, world, pre["total_ms"]) / 1e12
-    kern_tflops = ops / (pre["kernel_ms_mean"] * 1e-3) / 1e12
-    e2e_value = whole_job_rate(ops * pre["e2e_steps"], world, pre["e2e_ms"]) / 1e12
+    st = stack["stack"]
+    ops = stack_ops()
+    ms_per_step = stack["total_ms"] / args.steps
+    value = whole_job_rate(ops * args.steps, world, stack["total_ms"]) / 1e12
+    kern_tflops = ops / (ms_per_step * 1e-3) / 1e12
+    e2e_value = whole_job_rate(ops * stack["e2e_steps"], world, stack["e2e_ms"]) / 1e12
     hbm = peaks["hbm_gbs"]
     for v in list(decode.values()) + list(asym_dec.values()):
         v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
@@ -931,38 +1340,56 @@ def main():
     for k, v in a16.items():
         if k.startswith("decode_"):
             v["frac_hbm"] = round(v["stream_gbs"] / hbm, 3)
+    for k in ("step", "head", "block"):
+        g_dec[f"{k}_frac_hbm"] = round(g_dec[f"{k}_gbs"] / hbm, 3)
+    tc = peaks["bf16_tflops"]
+    g_pre["frac_tensor"] = round(g_pre["tops"] / tc, 3)
+    cfg0["frac_tensor_back_to_back"] = round(cfg0["tops_back_to_back"] / tc, 3)
+    blk_ops = block_ops(PREFILL_M)
+    blk_us = pre["total_ms"] / 2000 * 1e3
+    blk_tops = blk_ops / (blk_us * 1e-6) / 1e12
 
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int8",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD, "tokens": PREFILL_M,
-                   "linears": [f"{n} {k}->{nn}" for n, k, nn in synth.TINYLLAMA_LINEARS],
-                   "int8_ops_per_step": ops, "launches_per_step": 1,
-                   "l2": f"{PREFILL_LAYERS} layers rotated per step "
-                         f"({PREFILL_LAYERS * 72} MB > 129 MB L2)",
+        "config": {"workload": WORKLOAD, "tokens": STACK_M, "layers": STACK_LAYERS,
+                   "linears_per_layer": [f"{n} {k}->{nn}" for n, k, nn in synth.TINYLLAMA_LINEARS],
+                   "head": "{} {}->{}".format(*synth.TINYLLAMA_HEAD),
+                   "chain": "q/k/v/gate/up read x_l; o reads q, down reads up; "
+                            "x_l+1 = sat8(down + r_l)",
+                   "int8_ops_per_step": ops, "launches_per_step": stack["launches_per_step"],
+                   "l2": "each step streams 1.03 GB of int8 weights (more than the 129 MB L2); "
+                         "activations pass between layers through L2 as in a model",
                    "parallelism": f"replicas x{world}"},
-        "roofline": {"bound": "tensor", "achieved": round(kern_tflops, 1),
-                     "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                     "frac": round(kern_tflops / peaks["bf16_tflops"], 3),
-                     "traffic": prefill_traffic(), "traffic_unit": "bytes per launch",
-                     "kernel": "mq::prefill::prefill_kernel",
+        "roofline": {"bound": "tensor", "achieved": round(kern_tflops, 1), "peak": tc,
+                     "unit": "TFLOP/s", "frac": round(kern_tflops / tc, 3),
+                     "traffic": stack_traffic(), "traffic_unit": "bytes per step (45 launches)",
+                     "kernel": "mq::prefill::prefill_kernel (every launch of the step)",
                      "peak_note": f"dense f16 tensor peak = bf16 burst ({peaks['source']}), "
-                                  "int8 ops run as exact f16 MMAs"},
-        "clocks": pre["clocks"],
-        "e2e": {"value": round(e2e_value, 2), "unit": "TOPS", "h2d_bytes_per_step": pre["h2d"],
-                "d2h_bytes_per_step": pre["d2h"]},
-        "gpu_launches": args.steps,
+                                  "int8 ops run as exact f16 MMAs; achieved = the step's int8 "
+                                  "ops / its device time (CUDA events around the timed steps)"},
+        "clocks": stack["clocks"],
+        "e2e": {"value": round(e2e_value, 2), "unit": "TOPS", "h2d_bytes_per_step": stack["h2d"],
+                "d2h_bytes_per_step": stack["d2h"]},
+        "gpu_launches": args.steps * stack["launches_per_step"],
+        "config0_single_linear_m128": cfg0,
+        "config1_tinyllama_block_m1024": {
+            "workload": BLOCK_WORKLOAD, "us_per_block": round(blk_us, 2),
+            "tops": round(blk_tops, 1), "frac_tensor": round(blk_tops / tc, 3),
+            "launches_per_step": 1, "steps": 2000,
+            "l2": f"{PREFILL_LAYERS} layers rotated ({PREFILL_LAYERS * 72} MB > 129 MB L2)",
+            "traffic": prefill_traffic(), "traffic_unit": "bytes per launch"},
         "decode_w4a8": {"unit": "GB/s of int4 weights", "weight_bytes_per_block":
                         block_weight_bytes(4), "layers_rotated": DECODE_LAYERS,
                         "hbm_peak_gbs": hbm, **decode},
-        "asym_prefill_w8a8": {**asym_pre, "symmetric_us_per_block":
-                              round(pre["total_ms"] / args.steps * 1e3, 2)},
+        "config4_gemma": {"prefill_m4096": g_pre, "decode_w4a8_m1": g_dec},
+        "asym_prefill_w8a8": {**asym_pre, "symmetric_us_per_block": round(blk_us, 2)},
         "asym_decode_w4a8": {"unit": "GB/s of int4 weights",
                              "weights": "asymmetric per channel", **asym_dec},
         "a16": {"activations": "int16 in and out", "ops": "2 M K N per block", **a16,
-                "w8a8_us_per_block": round(pre["total_ms"] / args.steps * 1e3, 2),
+                "w8a8_us_per_block": round(blk_us, 2),
                 "w4a8_m1_stream_us": decode["m1"]["stream_us"]},
         "attention_w8a8_t1024": {**attention,
                                  "frac_hbm": round(attention["gbs"] / hbm, 3)},
@@ -973,7 +1400,7 @@ def main():
                                     "176 MB of f32 weights", **wpipe},
     }
     if rank == 0 and world == 1:
-        line["cpu_baseline"], parity = cpu_baseline(pre["blocks"], torch, checks=checks)
+        line["cpu_baseline"], parity = cpu_baseline(st, checks=checks)
         for leg, r in parity.items():
             node = line
             for key in leg.split("."):

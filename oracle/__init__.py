@@ -327,6 +327,31 @@ def linear(x, zx, packed, bits, n, m0, shift, zy, want_acc=False, zw=None):
     return _default().linear(x, zx, packed, bits, n, m0, shift, zy, want_acc, zw)
 
 
+def threads() -> int:
+    """Host threads the row-parallel front end uses (every core)."""
+    return max(1, os.cpu_count() or 1)
+
+
+def linear_mt(x, zx, packed, bits, n, m0, shift, zy, zw=None, nthreads=None):
+    """oracle.linear over row blocks on every host core: the same C function,
+    called on disjoint slices of the token rows from a thread pool (ctypes
+    releases the GIL during the call).  Rows are independent in the layer, so
+    the result is the single-threaded one.  Returns y int8 [M, N]."""
+    from concurrent.futures import ThreadPoolExecutor
+    x = np.ascontiguousarray(x, dtype=np.int8)
+    m = x.shape[0]
+    t = min(nthreads or threads(), max(1, m))
+    if t <= 1:
+        return linear(x, zx, packed, bits, n, m0, shift, zy, zw=zw)
+    bounds = [m * i // t for i in range(t + 1)]
+    o = _default()
+    with ThreadPoolExecutor(max_workers=t) as ex:
+        parts = list(ex.map(
+            lambda i: o.linear(x[bounds[i]:bounds[i + 1]], zx, packed, bits, n, m0, shift, zy,
+                               zw=zw), range(t)))
+    return np.concatenate(parts, axis=0) if parts else np.zeros((0, n), np.int8)
+
+
 def linear_points(x, zx, packed, bits, n, m0, shift, zy, pts, zw=None):
     return _default().linear_points(x, zx, packed, bits, n, m0, shift, zy, pts, zw)
 

@@ -80,6 +80,16 @@ def oracle_y(case) -> np.ndarray:
     return y
 
 
+def oracle_y_mt(case) -> np.ndarray:
+    """oracle_y computed on every host core (the oracle over row blocks)."""
+    packed, _ = oracle.pack(case.w, case.bits)
+    m0, sh = oracle.requant_params(case.sx, case.sw, case.sy)
+    y = oracle.linear_mt(case.x, case.zx, packed, case.bits, case.N, m0, sh, case.zy)
+    if case.residual is not None:
+        y = oracle.residual_add(y, case.residual)
+    return y
+
+
 def oracle_points(case, pts: np.ndarray):
     packed, _ = oracle.pack(case.w, case.bits)
     m0, sh = oracle.requant_params(case.sx, case.sw, case.sy)

@@ -76,4 +76,6 @@ def test_reference_arm_line():
         assert key in line, key
     assert line["impl"] == "reference" and line["value"] > 0 and line["unit"] == "TOPS"
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
-    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    assert line["cpu_baseline"]["kind"] == "oracle"
+    assert line["cpu_baseline"]["cores"] == oracle.threads()
+    assert line["config"]["workload"] == bench.WORKLOAD

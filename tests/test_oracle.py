@@ -1152,3 +1152,17 @@ def test_pins_reject_planted_mistake(tmp_path, name, old, new):
         except (AssertionError, oracle.OracleError):
             failures += 1
     assert failures > 0, f"no pin caught the planted mistake '{name}'"
+
+
+def test_row_parallel_front_end_equals_the_single_threaded_oracle(orc):
+    # linear_mt only cuts the token rows into blocks for a thread pool; rows
+    # are independent, so every output equals the single-threaded call's,
+    # including row counts that do not divide by the thread count
+    from paper_2408_13933_gb300 import synth
+    for m, k, n, bits, t in ((37, 256, 96, 8, 5), (3, 512, 64, 4, 8), (16, 64, 33, 8, 16)):
+        c = synth.random_case(4000 + m, m, k, n, bits)
+        packed, _ = orc.pack(c.w, bits)
+        m0, sh = orc.requant_params(c.sx, c.sw, c.sy)
+        want = orc.linear(c.x, c.zx, packed, bits, n, m0, sh, c.zy)
+        got = orc.linear_mt(c.x, c.zx, packed, bits, n, m0, sh, c.zy, nthreads=t)
+        assert got.shape == want.shape and np.array_equal(got, want)
