@@ -977,6 +977,15 @@ int prepare_decode_w4a8() {
 int launch_decode(const Problem *probs, int count, void *workspace, void *stream) {
     using namespace decode;
     if (count <= 0) return MQ_OK;
+    // one or two tokens: the row-tile kernel (mq_gemv.cu) when the launch suits it
+    const int which = test_decode_kernel();
+    if (which != 2) {
+        int dev = 0, sms = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return MQ_ERR_CUDA;
+        if (gemv_suits(probs, count, sms, which == 1)) return launch_gemv(probs, count, stream);
+    }
     int max_m = 0;
     for (int i = 0; i < count; ++i) max_m = probs[i].M > max_m ? probs[i].M : max_m;
     const bool nt2 = max_m > 8;

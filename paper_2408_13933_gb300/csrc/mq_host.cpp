@@ -17,10 +17,12 @@ namespace {
 constexpr uint64_t DEFAULT_WAIT_NS = 1000000000ull;  // 1 second
 std::atomic<uint64_t> g_wait_ns{DEFAULT_WAIT_NS};
 std::atomic<int> g_skip_cta{-1};
+std::atomic<int> g_decode_kernel{0};
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_ns.load(std::memory_order_relaxed); }
 int test_skip_cta() { return g_skip_cta.load(std::memory_order_relaxed); }
+int test_decode_kernel() { return g_decode_kernel.load(std::memory_order_relaxed); }
 
 }  // namespace mq
 
@@ -570,6 +572,12 @@ int mq_set_wait_limit_ns(uint64_t ns) {
 int mq_test_skip_partials(int cta) {
     if (cta < -1 || cta >= mq::DECODE_MAX_GRID) return MQ_ERR_INVALID_ARG;
     mq::g_skip_cta.store(cta, std::memory_order_relaxed);
+    return MQ_OK;
+}
+
+int mq_test_decode_kernel(int which) {
+    if (which < 0 || which > 2) return MQ_ERR_INVALID_ARG;
+    mq::g_decode_kernel.store(which, std::memory_order_relaxed);
     return MQ_OK;
 }
 

@@ -73,6 +73,14 @@ int launch_decode(const Problem *probs, int count, void *workspace, void *stream
 // Set-up of both token-tile variants of the W4A8 decode kernel on the current
 // device (done by the first launch of each variant otherwise).
 int prepare_decode_w4a8();
+// The weight-streaming kernel for one or two tokens (mq_gemv.cu): whether a
+// decode launch suits it (forced: only the structural conditions), and its
+// launcher.
+bool gemv_suits(const Problem *probs, int count, int sms, bool force);
+int launch_gemv(const Problem *probs, int count, void *stream);
+// Test hook (mq_test_decode_kernel): 0 chooses the decode kernel by shape, 1
+// takes the one-or-two-token kernel whenever it can serve the launch, 2 never.
+int test_decode_kernel();
 int launch_pack(const int8_t *w, int N, int K, int bits, void *packed, int32_t *colsum,
                 int *status, void *stream);
 // One row-sum job: out[m] = sum_k x[m][k] (mq_row_sums).

@@ -37,10 +37,13 @@ def prepare(m, n, k, bits, seed):
 
 @pytest.fixture
 def hooks():
+    # the split-K decode kernel (the one with a partner to wait for)
     lib = mq()
+    assert lib.test_decode_kernel(2) == 0
     yield lib
     assert lib.test_skip_partials(-1) == 0
     assert lib.set_wait_limit_ns(0) == 0
+    assert lib.test_decode_kernel(0) == 0
 
 
 # One 64-row unit with 16 (int4) or 32 (int8) stages: the decode grid has one
