@@ -4,48 +4,42 @@
 // At M <= 2 the layer reads every weight once and does one or two MACs with
 // it: the time is the weight stream (the paper notes that autoregressive
 // generation is memory-bound, Sec. 5.6 and Appendix A.2).  This kernel is
-// built to stream HBM at its rate:
+// built to stream HBM at its rate, with no shared memory and no barriers:
 //
-// Work.  Every problem's weight matrix is cut into row tiles of TR = 8 rows;
-// a row tile is read in stages of at most CHUNK = 1024 bytes of each of its
-// rows.  The row tiles of all problems of a launch form one sequence, and
-// each CTA (one per SM) takes a contiguous run of it, cut by the host so that
-// every CTA streams about the same number of bytes.  A row tile never spans
-// two CTAs, so every output is finished by the CTA that streamed it: no
-// split-K, no exchange between CTAs.
+// Work.  Every problem's weight matrix is cut into row groups of R = 4 rows.
+// The row groups of all problems of a launch form one sequence, weighed by
+// the bytes they stream; each warp of the grid takes a contiguous run of
+// about equal weight (the warps of a CTA take neighbouring runs, so every SM
+// streams about the same number of bytes).  A row group never spans two
+// warps, so every output is finished by the warp that streamed it.
 //
-// Data path.  One producer warp copies each stage into a shared-memory ring
-// with 1-D bulk copies (cp.async.bulk): one contiguous copy per weight row
-// segment (each row lands 16 bytes past a 1024-byte pitch, which spreads the
-// rows over the banks) and one per token of the matching slice of x; the
-// row tile's requantization parameters ride along with its last stage as
-// 4-byte cp.async copies whose completion the same mbarrier tracks.  Weight
-// copies of the first ring stages are issued before waiting for the previous
-// kernel in the stream (programmatic dependent launch): packed weights are
-// constant inputs.
+// Data path.  A warp reads its rows 1 KB at a time: lane l loads the 16 bytes
+// at 16 l and 512 + 16 l of each of the R rows (eight 16-byte loads in flight
+// per lane, streaming past L1), and the matching activation bytes through the
+// L1 cache, where x stays for the whole launch: every SM reads all of it again
+// and again.  The loads of a warp's first step are issued before waiting for
+// the previous kernel in the stream (programmatic dependent launch): packed
+// weights are constant inputs.
 //
-// Compute.  Eight consumer warps share every stage: warp w takes bytes
-// [128 w, 128 w + 128) of the chunk, lane (r, p) = (lane / 4, lane % 4) the
-// 32 bytes at offset 32 p of that slice of row r.  The eight lanes of a warp
-// that read the same slice of x read the same addresses, which the shared
-// memory broadcasts.  int4 weights: one LOP3 (and a shift for the high
-// nibbles) forms u = w + 8 in [0, 15] per byte and two PRMT put the nibbles in
-// k order, so that one dp4a multiplies four weights with four activation
-// bytes as they are stored; int8 weights go to dp4a unchanged.  The int32
-// sums are exact: |partial| <= 15 * 128 * 65536 < 2^31.
+// Compute.  int4 weights: one LOP3 (and a shift for the high nibbles) forms
+// u = w + 8 in [0, 15] per byte and two PRMT put the nibbles in k order, so
+// that one dp4a multiplies four weights with four activation bytes as they
+// are stored; int8 weights go to dp4a unchanged.  The int32 sums are exact:
+// |partial| <= 15 * 128 * 65536 < 2^31.  Bytes past the end of a row load as
+// zero.
 //
-// Epilogue (per row tile).  Each lane's sum is reduced over its four pieces
-// (two shuffles), the warps' sums over shared memory; then one thread per
-// (row, token) removes the bias, sum(w x) = sum(u x) - 8 sum(x) (int4), and
-// forms sum((x - zx)(w - zw)) = sum(w x) - zw sum(x) - zx (colsum - K zw),
-// requantizes (round half up, saturate), adds the optional residual and
-// stores.  sum(x) of each problem's tokens is accumulated while the CTA
-// streams its first row tile of that problem, which covers every k.
-// All mbarrier waits are bounded (mq_wait_parity).
+// Epilogue (per row group).  The R x M lane sums are reduced over the warp by
+// a reduce-scatter (each shuffle halves the values a lane holds), leaving one
+// (row, token) sum per group of lanes; its first lane removes the bias,
+// sum(w x) = sum(u x) - 8 sum(x) (int4), forms sum((x - zx)(w - zw)) =
+// sum(w x) - zw sum(x) - zx (colsum - K zw), requantizes (round half up,
+// saturate), adds the optional residual and stores.  Its parameters were
+// loaded when the group began, so their latency hides behind the weights'.
+// sum(x) of each problem's tokens is accumulated while the warp streams its
+// first row group of that problem, which covers every k.
 #include <cuda_runtime.h>
 
 #include <atomic>
-#include <vector>
 
 #include "mq_internal.h"
 #include "mq_ptx.cuh"
@@ -53,461 +47,280 @@
 namespace mq {
 namespace gemv {
 
-constexpr int CONS_WARPS = 8;
-constexpr int CONS_THREADS = CONS_WARPS * 32;
-constexpr int PROD_WARP = CONS_WARPS;
-constexpr int THREADS = CONS_THREADS + 32;
-constexpr int TR = 8;                     // weight rows per row tile
-constexpr int CHUNK = 1024;               // weight bytes of a row per stage
-constexpr int ROW_PITCH = CHUNK + 16;     // shared-memory row pitch
-constexpr int W_BYTES = TR * ROW_PITCH;
-constexpr int MAX_MT = 2;                 // tokens
-constexpr int PARAM_BYTES = 128;          // colsum, M0, shift, zw of 8 rows
-constexpr int CONS_BARRIER = 1;           // named barrier of the consumer warps
-constexpr int MAX_GRID = 320;
+constexpr int WARPS = 8;                 // per CTA
+constexpr int THREADS = WARPS * 32;
+constexpr int CTAS_PER_SM = 3;
+constexpr int R = 4;                     // rows per group
+constexpr int STEP = 1024;               // weight bytes of a row per step
+constexpr int MAX_MT = 2;                // tokens
 constexpr int MAX_PROBLEMS = DECODE_MAX_PROBLEMS;
-constexpr int MAX_STAGES = 24;
-
-__host__ __device__ constexpr int x_bytes(int bits, int mt) { return mt * CHUNK * (8 / bits); }
-__host__ __device__ constexpr int stage_bytes(int bits, int mt) {
-    return (W_BYTES + x_bytes(bits, mt) + PARAM_BYTES + 127) / 128 * 128;
-}
 
 struct Params {
-    Problem p[MAX_PROBLEMS];      // tile_begin = first global row tile, tiles_m = row tiles
+    Problem p[MAX_PROBLEMS];  // tile_begin = first row group, tiles_m = row groups
+    long long cost_begin[MAX_PROBLEMS + 1];  // weight of the problems before p
+    int cost_group[MAX_PROBLEMS];            // weight of one row group of p
     int count;
-    int stages;                   // ring depth
-    int pre_w;                    // 1: weights are read before griddep_wait
-    int cta_begin[MAX_GRID + 1];  // each CTA's first row tile
-    int *status;
-    uint64_t wait_ns;
+    int pre_w;  // 1: weights are read before griddep_wait
 };
 
-// What the kernel reads of a problem, kept in shared memory.
-struct GProb {
-    const uint8_t *w;
-    const int8_t *x;
-    const int32_t *colsum, *M0, *shift, *zw;
-    const int8_t *residual;
-    int8_t *y;
-    int32_t M, N, K, ldx, ldy, ldw, zx, zy;
-    int32_t tile_begin, tiles;
-    int32_t L;        // weight bytes of a row
-    int32_t nchunks;  // stages per row tile
-};
+__device__ __forceinline__ uint4 ldg_w(const uint8_t *p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+    return v;
+}
 
-template <int MT>
-struct Tail {
-    int32_t red[2][CONS_WARPS][TR][MT];  // the warps' row sums (row-tile parity)
-    int32_t xsred[2][CONS_WARPS][MT];    // the warps' sum(x) pieces
-    int32_t xsum[MT];                    // sum(x) of the current problem's tokens
-    GProb prob[MAX_PROBLEMS];
-    uint64_t full[MAX_STAGES];
-    uint64_t empty[MAX_STAGES];
-    int abort;
+// 16 bytes of x through the L1 cache (read-only for the kernel's lifetime:
+// read only after the previous kernel in the stream has completed).
+__device__ __forceinline__ uint4 ldg_x(const int8_t *p) {
+    uint4 v;
+    asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+    return v;
+}
+
+__device__ __forceinline__ int dp4a4(uint4 w, uint4 x, int acc) {
+    acc = __dp4a((int)w.x, (int)x.x, acc);
+    acc = __dp4a((int)w.y, (int)x.y, acc);
+    acc = __dp4a((int)w.z, (int)x.z, acc);
+    return __dp4a((int)w.w, (int)x.w, acc);
+}
+
+__device__ __forceinline__ int sum4(uint4 x, int acc) {
+    return dp4a4(make_uint4(0x01010101u, 0x01010101u, 0x01010101u, 0x01010101u), x, acc);
+}
+
+// acc += w . x over the 16 weight bytes of `w` (int4: 32 k, x in two vectors;
+// int8: 16 k, x in one).
+template <int BITS>
+__device__ __forceinline__ int dot16(uint4 w, const uint4 *x, int acc) {
+    if constexpr (BITS == 4) {
+        // word i holds k = 8 i .. 8 i + 7; lo / hi are k 8i..8i+3 / 8i+4..8i+7
+        // as bytes u = w + 8
+        const uint32_t wi[4] = {w.x, w.y, w.z, w.w};
+        uint32_t lo[4], hi[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint32_t e = (wi[i] & 0x0F0F0F0Fu) ^ 0x08080808u;
+            const uint32_t o = ((wi[i] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+            lo[i] = prmt(e, o, 0x5140u);
+            hi[i] = prmt(e, o, 0x7362u);
+        }
+        acc = dp4a4(make_uint4(lo[0], hi[0], lo[1], hi[1]), x[0], acc);
+        return dp4a4(make_uint4(lo[2], hi[2], lo[3], hi[3]), x[1], acc);
+    } else {
+        return dp4a4(w, x[0], acc);
+    }
+}
+
+// One step's loads of a row group: 16 weight bytes of each row at two places
+// (c0, c0 + 512) and the activations they meet.
+template <int BITS, int MT>
+struct Step {
+    static constexpr int KPB = 8 / BITS;
+    uint4 w[R][2];
+    uint4 x[MT][2][KPB];
 };
 
 template <int BITS, int MT>
-constexpr size_t smem_bytes(int stages) {
-    return (size_t)stages * stage_bytes(BITS, MT) + sizeof(Tail<MT>) + 128;
+__device__ __forceinline__ void load_weights(Step<BITS, MT> &st, const Problem &p, int n0,
+                                             int rows, int col) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = col + 512 * h;
+        const bool in = c < p.K * BITS / 8;
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            st.w[r][h] = (in && r < rows) ? ldg_w(p.w + (size_t)(n0 + r) * p.ldw + c)
+                                          : make_uint4(0u, 0u, 0u, 0u);
+    }
 }
 
-__device__ __forceinline__ void cons_sync() {
-    asm volatile("bar.sync %0, %1;" ::"n"(CONS_BARRIER), "n"(CONS_THREADS) : "memory");
+template <int BITS, int MT>
+__device__ __forceinline__ void load_x(Step<BITS, MT> &st, const Problem &p, int col) {
+    constexpr int KPB = 8 / BITS;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = col + 512 * h;
+        const bool in = c < p.K * BITS / 8;
+#pragma unroll
+        for (int m = 0; m < MT; ++m)
+#pragma unroll
+            for (int i = 0; i < KPB; ++i)
+                st.x[m][h][i] = (in && m < p.M)
+                                    ? ldg_x(p.x + (size_t)m * p.ldx + (size_t)c * KPB + 16 * i)
+                                    : make_uint4(0u, 0u, 0u, 0u);
+    }
 }
 
-__device__ __forceinline__ uint4 lds128(const uint8_t *p) {
-    return *reinterpret_cast<const uint4 *>(p);
-}
-
-// The problem holding row tile `tile`, searching forward from `pi` (a CTA
-// visits its tiles in increasing order, so the walk is amortized O(1)).
-template <class S>
-__device__ __forceinline__ int problem_from(const S &s, int count, int pi, int tile) {
-    while (pi + 1 < count && tile >= s.prob[pi + 1].tile_begin) ++pi;
-    return pi;
+// Reduce-scatter over the warp: on entry each lane holds R x MT partial sums;
+// on exit lane l holds in v[0] the total of value (l >> 3) (R x MT = 4: row
+// l >> 3) or, for R x MT = 8, of value 2 (l >> 3) + ((l >> 2) & 1).
+template <int NV>
+__device__ __forceinline__ int reduce_scatter(int (&v)[NV], int lane) {
+    static_assert(NV == 4 || NV == 8, "4 or 8 values");
+    // halve the values held at each of the first log2(NV) steps
+#pragma unroll
+    for (int n = NV, bit = 16; n > 1; n >>= 1, bit >>= 1) {
+        const bool upper = (lane & bit) != 0;
+#pragma unroll
+        for (int i = 0; i < n / 2; ++i) {
+            const int keep = upper ? v[i + n / 2] : v[i];
+            const int give = upper ? v[i] : v[i + n / 2];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, give, bit);
+        }
+    }
+    // the remaining lanes of each group: full reduction
+    constexpr int rest = NV == 4 ? 4 : 2;  // bits below the ones used above
+#pragma unroll
+    for (int bit = rest; bit >= 1; bit >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], bit);
+    return v[0];
 }
 
 template <int BITS, int MT, bool O16>
-__global__ void __launch_bounds__(THREADS, 2) gemv_kernel(const __grid_constant__ Params P) {
-    constexpr int KPB = 8 / BITS;  // k per weight byte
-    constexpr int SB = stage_bytes(BITS, MT);
-    constexpr int XOFF = W_BYTES;
-    constexpr int POFF = W_BYTES + x_bytes(BITS, MT);
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *ring = reinterpret_cast<uint8_t *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~static_cast<uintptr_t>(127));
-    const int S = P.stages;
-    Tail<MT> &s = *reinterpret_cast<Tail<MT> *>(ring + (size_t)S * SB);
-    volatile int *abort_flag = &s.abort;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int t_begin = P.cta_begin[blockIdx.x], t_end = P.cta_begin[blockIdx.x + 1];
-    const int count = P.count;
-
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < S; ++i) {
-            mbar_init(&s.full[i], 1);
-            mbar_init(&s.empty[i], CONS_WARPS);
-        }
-        s.abort = 0;
-        fence_mbar_init();
-    }
-    for (int i = threadIdx.x; i < count; i += THREADS) {
-        const Problem &q = P.p[i];
-        GProb g;
-        g.w = q.w;
-        g.x = q.x;
-        g.colsum = q.colsum;
-        g.M0 = q.M0;
-        g.shift = q.shift;
-        g.zw = q.zw;
-        g.residual = q.residual;
-        g.y = q.y;
-        g.M = q.M;
-        g.N = q.N;
-        g.K = q.K;
-        g.ldx = q.ldx;
-        g.ldy = q.ldy;
-        g.ldw = q.ldw;
-        g.zx = q.zx;
-        g.zy = q.zy;
-        g.tile_begin = q.tile_begin;
-        g.tiles = q.tiles_m;
-        g.L = q.K / KPB;
-        g.nchunks = (g.L + CHUNK - 1) / CHUNK;
-        s.prob[i] = g;
-    }
-    __syncthreads();
+__global__ void __launch_bounds__(THREADS, CTAS_PER_SM) gemv_kernel(const __grid_constant__ Params P) {
+    constexpr int NV = R * MT;  // sums per lane
+    const int lane = threadIdx.x & 31;
+    const long long W = (long long)gridDim.x * WARPS;
+    const long long gw = (long long)blockIdx.x * WARPS + (threadIdx.x >> 5);
+    const long long C = P.cost_begin[P.count];
+    const long long c_lo = C * gw / W, c_hi = C * (gw + 1) / W;
     if (threadIdx.x == 0) griddep_launch_dependents();
 
-    if (warp == PROD_WARP) {
-        // ------------------------------------------------------ producer
-        // Weight copies of the first ring stages go out before the wait for
-        // the previous kernel (constant inputs unless pre_w == 0); x and the
-        // parameters only after it.
-        uint32_t npre = 0;
-        if (lane == 0 && P.pre_w) {
-            int pi = 0;
-            for (int t = t_begin; t < t_end && npre < (uint32_t)S; ++t) {
-                pi = problem_from(s, count, pi, t);
-                const GProb &g = s.prob[pi];
-                const int n0 = (t - g.tile_begin) * TR;
-                const int rows = min(TR, g.N - n0);
-                for (int c = 0; c < g.nchunks && npre < (uint32_t)S; ++c, ++npre) {
-                    const int cb = min(CHUNK, g.L - c * CHUNK);
-                    uint8_t *st = ring + (size_t)npre * SB;
-                    mbar_expect_tx(&s.full[npre], (uint32_t)(rows * cb));
-                    for (int r = 0; r < rows; ++r)
-                        bulk_load(st + r * ROW_PITCH, g.w + (size_t)(n0 + r) * g.ldw + c * CHUNK,
-                                  (uint32_t)cb, &s.full[npre]);
-                }
+    // the warp's row groups: those whose starting weight lies in [c_lo, c_hi)
+    int pi = 0;
+    while (pi + 1 < P.count && P.cost_begin[pi + 1] <= c_lo) ++pi;
+    auto first_group = [&](int q, long long c) -> long long {
+        // first group j of problem q with cost_begin[q] + j cost_group[q] >= c
+        const long long d = c - P.cost_begin[q];
+        if (d <= 0) return 0;
+        return (d + P.cost_group[q] - 1) / P.cost_group[q];
+    };
+    long long g = first_group(pi, c_lo);
+    bool waited = !P.pre_w;
+    if (waited) griddep_wait();
+    int xsum[MT];
+    int cur_pi = -1;
+    for (; pi < P.count && P.cost_begin[pi] < c_hi; ++pi, g = 0) {
+        const Problem &p = P.p[pi];
+        const long long g_end = min((long long)p.tiles_m, first_group(pi, c_hi));
+        const int L = p.K * BITS / 8;
+        const int nsteps = (L + STEP - 1) / STEP;
+        for (; g < g_end; ++g) {
+            const int n0 = (int)g * R;
+            const int rows = min(R, p.N - n0);
+            Step<BITS, MT> st;
+            load_weights(st, p, n0, rows, 16 * lane);
+            if (!waited) {  // x, parameters and outputs only after the previous kernel
+                griddep_wait();
+                waited = true;
             }
-        }
-        npre = __shfl_sync(0xffffffffu, npre, 0);
-        griddep_wait();
-        uint32_t it = 0;
-        bool ok = true;
-        int pi = 0;
-        for (int t = t_begin; ok && t < t_end; ++t) {
-            pi = problem_from(s, count, pi, t);
-            const GProb &g = s.prob[pi];
-            const int n0 = (t - g.tile_begin) * TR;
-            const int rows = min(TR, g.N - n0);
-            for (int c = 0; c < g.nchunks; ++c, ++it) {
-                const int slot = it % S;
-                bool got = true;
-                if (lane == 0)
-                    got = mq_wait_parity(&s.empty[slot], ((it / S) & 1) ^ 1, &s.abort, P.status,
-                                         P.wait_ns);
-                if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) {
-                    ok = false;
-                    break;
-                }
-                uint8_t *st = ring + (size_t)slot * SB;
-                const int cb = min(CHUNK, g.L - c * CHUNK);
-                if (c == g.nchunks - 1) {
-                    // the row tile's parameters: lane = 8 array + row
-                    const int arr = lane >> 3, r = lane & 7;
-                    const int32_t *src = arr == 0 ? g.colsum : arr == 1 ? g.M0
-                                       : arr == 2 ? g.shift : g.zw;
-                    if (r < rows && src) cp_async4(st + POFF + lane * 4, src + n0 + r);
-                    cp_async_arrive(&s.full[slot]);
-                }
-                __syncwarp();
-                if (lane == 0) {
-                    if (it >= npre) {
-                        mbar_expect_tx(&s.full[slot], (uint32_t)(rows * cb));
-                        for (int r = 0; r < rows; ++r)
-                            bulk_load(st + r * ROW_PITCH,
-                                      g.w + (size_t)(n0 + r) * g.ldw + c * CHUNK, (uint32_t)cb,
-                                      &s.full[slot]);
-                    }
-                    mbar_arrive_expect_tx(&s.full[slot], (uint32_t)(g.M * cb * KPB));
-                    for (int m = 0; m < g.M; ++m)
-                        bulk_load(st + XOFF + m * CHUNK * KPB,
-                                  g.x + (size_t)m * g.ldx + (size_t)c * CHUNK * KPB,
-                                  (uint32_t)(cb * KPB), &s.full[slot]);
-                }
-            }
-        }
-        if (!ok && lane == 0) {
-            // Given up: let the copies already issued land before the CTA can
-            // leave (only the last S stages can still be in flight; stages
-            // below `it` were issued whole).
-            for (uint32_t i = it > (uint32_t)S ? it - S : 0u; i < it; ++i)
-                mq_wait_parity_drain(&s.full[i % S], (i / S) & 1, P.status, P.wait_ns);
-        }
-        __syncwarp();
-    } else {
-        // ------------------------------------------------------ consumers
-        griddep_wait();  // before the first global access (residual, y)
-        const int r = lane >> 2, pc = lane & 3;
-        const int off = warp * 128 + pc * 32;  // this lane's bytes within a chunk
-        const int et = threadIdx.x;            // epilogue thread: row et % 8, token et / 8
-        uint32_t it = 0;
-        int pi = -1;
-        int parity = 0;
-        for (int t = t_begin; t < t_end; ++t) {
-            const int npi = problem_from(s, count, pi < 0 ? 0 : pi, t);
-            const bool first = npi != pi;  // first row tile of this problem in this CTA
-            pi = npi;
-            const GProb &g = s.prob[pi];
-            const int n0 = (t - g.tile_begin) * TR;
-            const int rows = min(TR, g.N - n0);
-            // the residual of this thread's output, loaded now for the epilogue
-            int32_t res = 0;
-            if (et < TR * MT && g.residual && (et & 7) < rows && (et >> 3) < g.M)
-                res = g.residual[(size_t)(et >> 3) * g.ldy + n0 + (et & 7)];
-            int32_t acc[MT], xs[MT];
-#pragma unroll
-            for (int m = 0; m < MT; ++m) acc[m] = xs[m] = 0;
-            for (int c = 0; c < g.nchunks; ++c, ++it) {
-                const int slot = it % S;
-                bool got = false;
-                if (lane == 0)
-                    got = !*abort_flag && mq_wait_parity(&s.full[slot], (it / S) & 1, &s.abort,
-                                                         P.status, P.wait_ns);
-                got = __shfl_sync(0xffffffffu, got ? 1 : 0, 0) != 0;
-                const uint8_t *st = ring + (size_t)slot * SB;
-                const int cb = min(CHUNK, g.L - c * CHUNK);
-                if (got && off < cb) {
-                    const uint8_t *xp = st + XOFF + off * KPB;
-                    // A chunk ends on a 16-byte boundary, so the last lane's
-                    // piece may hold only 16 valid bytes: the activations of
-                    // the other half then read as zero (the stale weights
-                    // beside them multiply nothing).
-                    const bool h2 = off + 32 <= cb;
-                    auto xld = [&](int m, int q) {
-                        return (q < KPB || h2) ? lds128(xp + m * CHUNK * KPB + 16 * q)
-                                               : make_uint4(0u, 0u, 0u, 0u);
-                    };
-                    if (first) {
-                        // sum(x) of the slice (every k of the problem passes
-                        // through the lanes of row 0 during its first tile)
-#pragma unroll
-                        for (int m = 0; m < MT; ++m)
-#pragma unroll
-                            for (int q = 0; q < 2 * KPB; ++q) {
-                                const uint4 v = xld(m, q);
-                                xs[m] = __dp4a((int)v.x, 0x01010101, xs[m]);
-                                xs[m] = __dp4a((int)v.y, 0x01010101, xs[m]);
-                                xs[m] = __dp4a((int)v.z, 0x01010101, xs[m]);
-                                xs[m] = __dp4a((int)v.w, 0x01010101, xs[m]);
-                            }
-                    }
-                    if (r < rows) {
-                        const uint4 wa = lds128(st + r * ROW_PITCH + off);
-                        const uint4 wb = lds128(st + r * ROW_PITCH + off + 16);
-                        const uint32_t wv[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
-                        if constexpr (BITS == 4) {
-                            // word j holds k = 8 j .. 8 j + 7 of the piece; lo / hi
-                            // are k 8j..8j+3 / 8j+4..8j+7 as bytes u = w + 8
-                            uint32_t lo[8], hi[8];
-#pragma unroll
-                            for (int j = 0; j < 8; ++j) {
-                                const uint32_t e = (wv[j] & 0x0F0F0F0Fu) ^ 0x08080808u;
-                                const uint32_t o = ((wv[j] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
-                                lo[j] = prmt(e, o, 0x5140u);
-                                hi[j] = prmt(e, o, 0x7362u);
-                            }
-#pragma unroll
-                            for (int m = 0; m < MT; ++m)
-#pragma unroll
-                                for (int q = 0; q < 4; ++q) {
-                                    const uint4 v = xld(m, q);
-                                    acc[m] = __dp4a((int)lo[2 * q], (int)v.x, acc[m]);
-                                    acc[m] = __dp4a((int)hi[2 * q], (int)v.y, acc[m]);
-                                    acc[m] = __dp4a((int)lo[2 * q + 1], (int)v.z, acc[m]);
-                                    acc[m] = __dp4a((int)hi[2 * q + 1], (int)v.w, acc[m]);
-                                }
-                        } else {
-#pragma unroll
-                            for (int m = 0; m < MT; ++m)
-#pragma unroll
-                                for (int q = 0; q < 2; ++q) {
-                                    const uint4 v = xld(m, q);
-                                    acc[m] = __dp4a((int)wv[4 * q + 0], (int)v.x, acc[m]);
-                                    acc[m] = __dp4a((int)wv[4 * q + 1], (int)v.y, acc[m]);
-                                    acc[m] = __dp4a((int)wv[4 * q + 2], (int)v.z, acc[m]);
-                                    acc[m] = __dp4a((int)wv[4 * q + 3], (int)v.w, acc[m]);
-                                }
-                        }
-                    }
-                }
-                const bool last = c == g.nchunks - 1;
-                // the last stage of a tile holds its parameters: warp 0 (the
-                // epilogue's) releases it after the epilogue
-                if (!(last && warp == 0)) {
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&s.empty[slot]);
-                }
-            }
-            // ---- epilogue of the row tile
-#pragma unroll
-            for (int m = 0; m < MT; ++m) {
-                acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], 1);
-                acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], 2);
-                if (first) {
-                    xs[m] += __shfl_xor_sync(0xffffffffu, xs[m], 1);
-                    xs[m] += __shfl_xor_sync(0xffffffffu, xs[m], 2);
-                }
-            }
-            if (pc == 0) {
-#pragma unroll
-                for (int m = 0; m < MT; ++m) s.red[parity][warp][r][m] = acc[m];
-            }
-            if (first && lane == 0) {
-#pragma unroll
-                for (int m = 0; m < MT; ++m) s.xsred[parity][warp][m] = xs[m];
-            }
-            cons_sync();
-            const uint32_t lslot = (it - 1) % S;  // the tile's last stage
-            if (et < TR * MT) {
-                const int er = et & 7, m = et >> 3;
-                int32_t sum = 0, xsum;
-#pragma unroll
-                for (int w = 0; w < CONS_WARPS; ++w) sum += s.red[parity][w][er][m];
-                if (first) {
-                    xsum = 0;
-#pragma unroll
-                    for (int w = 0; w < CONS_WARPS; ++w) xsum += s.xsred[parity][w][m];
-                } else {
-                    xsum = s.xsum[m];
-                }
+            const bool first = pi != cur_pi;  // the warp's first group of this problem
+            cur_pi = pi;
+            // this lane's output, if any: value (lane >> 3) of the reduce-scatter
+            const int vi = NV == 4 ? (lane >> 3) : 2 * (lane >> 3) + ((lane >> 2) & 1);
+            const int er = MT == 1 ? vi : vi >> 1, em = MT == 1 ? 0 : vi & 1;
+            const bool owner = (lane & (NV == 4 ? 7 : 3)) == 0 && er < rows && em < p.M;
+            int32_t colsum = 0, m0 = 0, sh = 33, zw = 0, res = 0;
+            if (owner) {
                 const int n = n0 + er;
-                if (!*abort_flag && er < rows && m < g.M) {
-                    const int32_t *prm =
-                        reinterpret_cast<const int32_t *>(ring + (size_t)lslot * SB + POFF);
-                    const int32_t colsum = prm[er], m0 = prm[8 + er], sh = prm[16 + er];
-                    const int32_t zw = g.zw ? prm[24 + er] : 0;
-                    // sum(w x) = sum(u x) - 8 sum(x) (int4); then the zero points:
-                    // sum((x - zx)(w - zw)) = sum(w x) - zw sum(x) - zx (colsum - K zw)
-                    // (two's-complement wrap is exact: the true value fits int32)
-                    const uint32_t wx = (uint32_t)sum - (uint32_t)(BITS == 4 ? 8 * xsum : 0);
-                    const int32_t a =
-                        (int32_t)(wx - (uint32_t)zw * (uint32_t)xsum -
-                                  (uint32_t)g.zx * ((uint32_t)colsum - (uint32_t)g.K * (uint32_t)zw));
-                    if constexpr (O16) {
-                        reinterpret_cast<int16_t *>(g.y)[(size_t)m * g.ldy + n] =
-                            (int16_t)mq_requant16((int64_t)a, m0, sh, g.zy);
-                    } else {
-                        int32_t y = mq_requant(a, m0, sh, g.zy);
-                        if (g.residual) y = min(127, max(-128, y + res));
-                        g.y[(size_t)m * g.ldy + n] = (int8_t)y;
-                    }
+                colsum = __ldg(p.colsum + n);
+                m0 = __ldg(p.M0 + n);
+                sh = __ldg(p.shift + n);
+                if (p.zw) zw = __ldg(p.zw + n);
+                if (p.residual) res = p.residual[(size_t)em * p.ldy + n];
+            }
+            int acc[NV];
+            int xs[MT];
+#pragma unroll
+            for (int i = 0; i < NV; ++i) acc[i] = 0;
+#pragma unroll
+            for (int m = 0; m < MT; ++m) xs[m] = 0;
+            for (int s = 0; s < nsteps; ++s) {
+                if (s > 0) load_weights(st, p, n0, rows, s * STEP + 16 * lane);
+                load_x(st, p, s * STEP + 16 * lane);
+                if (first) {
+#pragma unroll
+                    for (int m = 0; m < MT; ++m)
+#pragma unroll
+                        for (int h = 0; h < 2; ++h)
+#pragma unroll
+                            for (int i = 0; i < 8 / BITS; ++i) xs[m] = sum4(st.x[m][h][i], xs[m]);
                 }
-                if (first && er == 0) s.xsum[m] = xsum;
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+#pragma unroll
+                    for (int m = 0; m < MT; ++m)
+#pragma unroll
+                        for (int h = 0; h < 2; ++h)
+                            acc[r * MT + m] = dot16<BITS>(st.w[r][h], st.x[m][h], acc[r * MT + m]);
             }
-            if (warp == 0) {
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&s.empty[lslot]);
+            if (first) {
+#pragma unroll
+                for (int m = 0; m < MT; ++m) {
+#pragma unroll
+                    for (int bit = 16; bit >= 1; bit >>= 1)
+                        xs[m] += __shfl_xor_sync(0xffffffffu, xs[m], bit);
+                    xsum[m] = xs[m];
+                }
             }
-            parity ^= 1;
+            const int sum = reduce_scatter<NV>(acc, lane);
+            if (owner) {
+                const int n = n0 + er;
+                const int32_t xsm = MT == 1 ? xsum[0] : (em ? xsum[MT - 1] : xsum[0]);
+                // sum(w x) = sum(u x) - 8 sum(x) (int4); then the zero points:
+                // sum((x - zx)(w - zw)) = sum(w x) - zw sum(x) - zx (colsum - K zw)
+                // (two's-complement wrap is exact: the true value fits int32)
+                const uint32_t wx = (uint32_t)sum - (uint32_t)(BITS == 4 ? 8 * xsm : 0);
+                const int32_t a =
+                    (int32_t)(wx - (uint32_t)zw * (uint32_t)xsm -
+                              (uint32_t)p.zx * ((uint32_t)colsum - (uint32_t)p.K * (uint32_t)zw));
+                if constexpr (O16) {
+                    reinterpret_cast<int16_t *>(p.y)[(size_t)em * p.ldy + n] =
+                        (int16_t)mq_requant16((int64_t)a, m0, sh, p.zy);
+                } else {
+                    int32_t y = mq_requant(a, m0, sh, p.zy);
+                    if (p.residual) y = min(127, max(-128, y + res));
+                    p.y[(size_t)em * p.ldy + n] = (int8_t)y;
+                }
+            }
         }
     }
-    __syncthreads();
-}
-
-template <int BITS, int MT, bool O16>
-int prepare_t(int dev, size_t smem) {
-    static std::atomic<uint64_t> done{0};  // bit d: device d prepared
-    if (dev < 0 || dev >= 64) return MQ_ERR_CUDA;
-    const uint64_t bit = 1ull << dev;
-    if (done.load(std::memory_order_acquire) & bit) return MQ_OK;
-    if (cudaFuncSetAttribute(gemv_kernel<BITS, MT, O16>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-        return MQ_ERR_CUDA;
-    done.fetch_or(bit, std::memory_order_release);
-    return MQ_OK;
-}
-
-// Stages of the ring: as deep as fits beside a second CTA of the same size on
-// the SM (the next launch's, which programmatic dependent launch starts while
-// this one drains).
-constexpr int SMEM_BUDGET = 110 * 1024;
-
-template <int BITS, int MT>
-int ring_stages() {
-    int st = (int)((SMEM_BUDGET - sizeof(Tail<MT>) - 128) / stage_bytes(BITS, MT));
-    return st > MAX_STAGES ? MAX_STAGES : st;
+    if (!waited) griddep_wait();  // a warp without work still orders after its predecessor
 }
 
 template <int BITS, int MT, bool O16>
 int launch_t(const Problem *probs, int count, cudaStream_t stream) {
-    constexpr int KPB = 8 / BITS;
-    const int stages = ring_stages<BITS, MT>();
-    const size_t smem = smem_bytes<BITS, MT>(stages);
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ERR_CUDA;
-    if (prepare_t<BITS, MT, O16>(dev, smem_bytes<BITS, MT>(ring_stages<BITS, MT>())) != MQ_OK)
-        return MQ_ERR_CUDA;
-    int sms = 0;
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return MQ_ERR_CUDA;
     for (int begin = 0; begin < count; begin += MAX_PROBLEMS) {
         const int n = count - begin < MAX_PROBLEMS ? count - begin : MAX_PROBLEMS;
         Params P{};
         P.pre_w = 1;
-        // row tiles of every problem, and the bytes each one streams (plus a
-        // fixed share for its epilogue)
-        std::vector<long long> cost;
-        int tiles = 0;
+        long long cost = 0, groups = 0;
         for (int i = 0; i < n; ++i) {
             Problem &q = P.p[i];
             q = probs[begin + i];
             if (q.wdynamic) P.pre_w = 0;
-            q.tile_begin = tiles;
-            q.tiles_m = (q.N + TR - 1) / TR;
-            tiles += q.tiles_m;
-            const long long L = q.K / KPB;
-            for (int t = 0; t < q.tiles_m; ++t) {
-                const int rows = q.N - t * TR < TR ? q.N - t * TR : TR;
-                cost.push_back(rows * L + q.M * L * KPB / 8 + 2048);
-            }
+            q.tiles_m = (q.N + R - 1) / R;
+            // a group's weight: its 1 KB steps and one more for its epilogue
+            P.cost_group[i] = (q.K * q.bits / 8 + STEP - 1) / STEP + 1;
+            P.cost_begin[i] = cost;
+            cost += (long long)q.tiles_m * P.cost_group[i];
+            groups += q.tiles_m;
         }
-        if (tiles == 0) continue;
-        int grid = sms < MAX_GRID ? sms : MAX_GRID;
-        if (grid > tiles) grid = tiles;
-        // contiguous runs of row tiles of about equal cost
-        long long total = 0;
-        for (long long c : cost) total += c;
-        P.cta_begin[0] = 0;
-        long long acc = 0;
-        int t = 0;
-        for (int c = 1; c < grid; ++c) {
-            const long long target = total * c / grid;
-            while (t < tiles && acc + cost[t] / 2 <= target) acc += cost[t++];
-            P.cta_begin[c] = t;
-        }
-        P.cta_begin[grid] = tiles;
+        P.cost_begin[n] = cost;
         P.count = n;
-        P.stages = stages;
-        P.status = device_status_ptr();
-        P.wait_ns = wait_limit_ns();
+        if (groups == 0) continue;
+        long long warps = (long long)CTAS_PER_SM * sms * WARPS;
+        if (warps > groups) warps = groups;
+        const int grid = (int)((warps + WARPS - 1) / WARPS);
         cudaLaunchConfig_t cfg{};
         cfg.gridDim = dim3((unsigned)grid, 1, 1);
         cfg.blockDim = dim3(THREADS, 1, 1);
-        cfg.dynamicSmemBytes = smem;
+        cfg.dynamicSmemBytes = 0;
         cfg.stream = stream;
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -523,24 +336,18 @@ int launch_t(const Problem *probs, int count, cudaStream_t stream) {
 }  // namespace gemv
 
 // Whether a decode launch can take this kernel: 8-bit activations, at most
-// two tokens, K > 0, and (unless forced) enough row tiles of small enough
-// size that contiguous runs of them balance the SMs.
+// two tokens, K > 0, and (unless forced) at least one row group per warp of
+// the grid, so that the launch's bytes spread over every SM.
 bool gemv_suits(const Problem *probs, int count, int sms, bool force) {
     using namespace gemv;
     if (count <= 0) return false;
-    long long total = 0, max_tile = 0, tiles = 0;
+    long long groups = 0;
     for (int i = 0; i < count; ++i) {
         const Problem &q = probs[i];
         if (q.a16 || q.M < 1 || q.M > MAX_MT || q.K <= 0 || q.N <= 0) return false;
-        const long long L = (long long)q.K * q.bits / 8;
-        const long long tile = TR * L;
-        total += (long long)q.N * L;
-        tiles += (q.N + TR - 1) / TR;
-        if (tile > max_tile) max_tile = tile;
+        groups += (q.N + R - 1) / R;
     }
-    if (force) return true;
-    // at least two row tiles per SM, and no tile above a quarter of an SM's share
-    return tiles >= 2LL * sms && max_tile * 4 * sms <= total;
+    return force || groups >= (long long)CTAS_PER_SM * sms * WARPS;
 }
 
 int launch_gemv(const Problem *probs, int count, void *stream) {
