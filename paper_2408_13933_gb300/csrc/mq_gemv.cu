@@ -17,16 +17,23 @@
 // at 16 l and 512 + 16 l of each of the R rows (eight 16-byte loads in flight
 // per lane, streaming past L1), and the matching activation bytes through the
 // L1 cache, where x stays for the whole launch: every SM reads all of it again
-// and again.  The loads of a warp's first step are issued before waiting for
-// the previous kernel in the stream (programmatic dependent launch): packed
-// weights are constant inputs.
+// and again.  Three CTAs of eight warps per SM (two for two tokens) keep about
+// 96 KB of weights in flight per SM.  The weights of a warp's next group are
+// requested before the current group's epilogue, and those of its first group
+// before waiting for the previous kernel in the stream (programmatic
+// dependent launch): packed weights are constant inputs.  Measured against a
+// shared-memory ring fed by bulk or tensor-map copies, this path streams more:
+// one CTA's copy engine stops near 3.9 TB/s over the GPU, and per-stage
+// barriers cost more than the work of an 8 KB stage.
 //
-// Compute.  int4 weights: one LOP3 (and a shift for the high nibbles) forms
-// u = w + 8 in [0, 15] per byte and two PRMT put the nibbles in k order, so
-// that one dp4a multiplies four weights with four activation bytes as they
-// are stored; int8 weights go to dp4a unchanged.  The int32 sums are exact:
-// |partial| <= 15 * 128 * 65536 < 2^31.  Bytes past the end of a row load as
-// zero.
+// Compute.  int4 weights: the low nibbles of a word give u = w + 8 in
+// [0, 15] per byte with one LOP3, the high nibbles 16 u in [0, 240] in place
+// with another; a signed and an unsigned-by-signed dp4a multiply them with the
+// activations of the even and the odd k of the word, which two PRMT per word
+// pair form once per step and token (shared by the R rows).  The sums of the
+// high nibbles are multiples of 16 and are divided back exactly.  int8
+// weights go to dp4a unchanged.  The int32 sums are exact: |partial| <=
+// 240 * 128 * 32768 < 2^31.  Bytes past the end of a row load as zero.
 //
 // Epilogue (per row group).  The R x M lane sums are reduced over the warp by
 // a reduce-scatter (each shuffle halves the values a lane holds), leaving one
@@ -49,11 +56,15 @@ namespace gemv {
 
 constexpr int WARPS = 8;                 // per CTA
 constexpr int THREADS = WARPS * 32;
-constexpr int CTAS_PER_SM = 3;
 constexpr int R = 4;                     // rows per group
 constexpr int STEP = 1024;               // weight bytes of a row per step
 constexpr int MAX_MT = 2;                // tokens
 constexpr int MAX_PROBLEMS = DECODE_MAX_PROBLEMS;
+// CTAs per SM: three for one token (80 registers a thread); two for two
+// tokens, whose activation vectors would not fit 80 registers without spills
+// (measured, two tokens: 9.9 us against 10.5 us per TinyLlama-shaped block).
+template <int MT>
+constexpr int ctas_per_sm() { return MT == 1 ? 3 : 2; }
 
 struct Params {
     Problem p[MAX_PROBLEMS];  // tile_begin = first row group, tiles_m = row groups
@@ -90,26 +101,39 @@ __device__ __forceinline__ int sum4(uint4 x, int acc) {
     return dp4a4(make_uint4(0x01010101u, 0x01010101u, 0x01010101u, 0x01010101u), x, acc);
 }
 
-// acc += w . x over the 16 weight bytes of `w` (int4: 32 k, x in two vectors;
-// int8: 16 k, x in one).
-template <int BITS>
-__device__ __forceinline__ int dot16(uint4 w, const uint4 *x, int acc) {
-    if constexpr (BITS == 4) {
-        // word i holds k = 8 i .. 8 i + 7; lo / hi are k 8i..8i+3 / 8i+4..8i+7
-        // as bytes u = w + 8
-        const uint32_t wi[4] = {w.x, w.y, w.z, w.w};
-        uint32_t lo[4], hi[4];
+// acc + sum of the four unsigned bytes of a times the four signed bytes of b
+__device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int acc) {
+    int d;
+    asm("dp4a.u32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(acc));
+    return d;
+}
+
+// The activations of 32 consecutive k (two 16-byte vectors) regrouped for
+// the int4 words that hold them: word i (k 8i .. 8i + 7, low nibbles the even
+// k) meets e[i] = x of k 8i, 8i+2, 8i+4, 8i+6 and o[i] = x of the odd k.
+struct XEO {
+    uint32_t e[4], o[4];
+};
+
+__device__ __forceinline__ XEO x_even_odd(uint4 a, uint4 b) {
+    const uint32_t v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+    XEO r;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const uint32_t e = (wi[i] & 0x0F0F0F0Fu) ^ 0x08080808u;
-            const uint32_t o = ((wi[i] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
-            lo[i] = prmt(e, o, 0x5140u);
-            hi[i] = prmt(e, o, 0x7362u);
-        }
-        acc = dp4a4(make_uint4(lo[0], hi[0], lo[1], hi[1]), x[0], acc);
-        return dp4a4(make_uint4(lo[2], hi[2], lo[3], hi[3]), x[1], acc);
-    } else {
-        return dp4a4(w, x[0], acc);
+    for (int i = 0; i < 4; ++i) {
+        r.e[i] = prmt(v[2 * i], v[2 * i + 1], 0x6420u);
+        r.o[i] = prmt(v[2 * i], v[2 * i + 1], 0x7531u);
+    }
+    return r;
+}
+
+// int4: lo += sum(u x) over the low nibbles (u = w + 8), hi += 16 sum(u x)
+// over the high nibbles, for the 16 weight bytes of `w`.
+__device__ __forceinline__ void dot16_i4(uint4 w, const XEO &x, int &lo, int &hi) {
+    const uint32_t wi[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        lo = __dp4a((int)((wi[i] & 0x0F0F0F0Fu) ^ 0x08080808u), (int)x.e[i], lo);
+        hi = dp4a_us((wi[i] & 0xF0F0F0F0u) ^ 0x80808080u, x.o[i], hi);
     }
 }
 
@@ -122,43 +146,64 @@ struct Step {
     uint4 x[MT][2][KPB];
 };
 
+// The loads of one step: c0 is the step's first byte in a row (warp-uniform);
+// lane l takes bytes c0 + 16 l and c0 + 512 + 16 l.  Full groups of full
+// steps load without bounds checks; the others read zero past the matrix.
 template <int BITS, int MT>
 __device__ __forceinline__ void load_weights(Step<BITS, MT> &st, const Problem &p, int n0,
-                                             int rows, int col) {
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        const int c = col + 512 * h;
-        const bool in = c < p.K * BITS / 8;
+                                             int rows, int c0, int lane) {
+    const int L = p.K * BITS / 8;
+    const size_t ldw = (size_t)p.ldw;
+    const uint8_t *b = p.w + (size_t)n0 * ldw + c0 + 16 * lane;
+    if (rows == R && c0 + STEP <= L) {
 #pragma unroll
         for (int r = 0; r < R; ++r)
-            st.w[r][h] = (in && r < rows) ? ldg_w(p.w + (size_t)(n0 + r) * p.ldw + c)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) st.w[r][h] = ldg_w(b + r * ldw + 512 * h);
+        return;
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const bool in = c0 + 512 * h + 16 * lane < L;
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            st.w[r][h] = (in && r < rows) ? ldg_w(b + r * ldw + 512 * h)
                                           : make_uint4(0u, 0u, 0u, 0u);
     }
 }
 
 template <int BITS, int MT>
-__device__ __forceinline__ void load_x(Step<BITS, MT> &st, const Problem &p, int col) {
+__device__ __forceinline__ void load_x(Step<BITS, MT> &st, const Problem &p, int c0, int lane) {
     constexpr int KPB = 8 / BITS;
+    const int L = p.K * BITS / 8;
+    const int8_t *b = p.x + ((size_t)c0 + 16 * lane) * KPB;
+    const size_t ldx = (size_t)p.ldx;
+    if (p.M == MT && c0 + STEP <= L) {
+#pragma unroll
+        for (int m = 0; m < MT; ++m)
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int i = 0; i < KPB; ++i) st.x[m][h][i] = ldg_x(b + m * ldx + 512 * KPB * h + 16 * i);
+        return;
+    }
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-        const int c = col + 512 * h;
-        const bool in = c < p.K * BITS / 8;
+        const bool in = c0 + 512 * h + 16 * lane < L;
 #pragma unroll
         for (int m = 0; m < MT; ++m)
 #pragma unroll
             for (int i = 0; i < KPB; ++i)
-                st.x[m][h][i] = (in && m < p.M)
-                                    ? ldg_x(p.x + (size_t)m * p.ldx + (size_t)c * KPB + 16 * i)
-                                    : make_uint4(0u, 0u, 0u, 0u);
+                st.x[m][h][i] = (in && m < p.M) ? ldg_x(b + m * ldx + 512 * KPB * h + 16 * i)
+                                                : make_uint4(0u, 0u, 0u, 0u);
     }
 }
 
-// Reduce-scatter over the warp: on entry each lane holds R x MT partial sums;
-// on exit lane l holds in v[0] the total of value (l >> 3) (R x MT = 4: row
-// l >> 3) or, for R x MT = 8, of value 2 (l >> 3) + ((l >> 2) & 1).
+// Reduce-scatter over the warp: on entry each lane holds NV partial sums; on
+// exit lane l holds in v[0] the total of value l / (32 / NV) over all lanes.
 template <int NV>
 __device__ __forceinline__ int reduce_scatter(int (&v)[NV], int lane) {
-    static_assert(NV == 4 || NV == 8, "4 or 8 values");
+    static_assert(NV == 4 || NV == 8 || NV == 16, "4, 8 or 16 values");
     // halve the values held at each of the first log2(NV) steps
 #pragma unroll
     for (int n = NV, bit = 16; n > 1; n >>= 1, bit >>= 1) {
@@ -171,122 +216,157 @@ __device__ __forceinline__ int reduce_scatter(int (&v)[NV], int lane) {
         }
     }
     // the remaining lanes of each group: full reduction
-    constexpr int rest = NV == 4 ? 4 : 2;  // bits below the ones used above
 #pragma unroll
-    for (int bit = rest; bit >= 1; bit >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], bit);
+    for (int bit = 16 / NV; bit >= 1; bit >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], bit);
     return v[0];
 }
 
 template <int BITS, int MT, bool O16>
-__global__ void __launch_bounds__(THREADS, CTAS_PER_SM) gemv_kernel(const __grid_constant__ Params P) {
+__global__ void __launch_bounds__(THREADS, ctas_per_sm<MT>()) gemv_kernel(const __grid_constant__ Params P) {
     constexpr int NV = R * MT;  // sums per lane
     const int lane = threadIdx.x & 31;
     const long long W = (long long)gridDim.x * WARPS;
     const long long gw = (long long)blockIdx.x * WARPS + (threadIdx.x >> 5);
     const long long C = P.cost_begin[P.count];
+    // the range of weights this warp's groups start in
     const long long c_lo = C * gw / W, c_hi = C * (gw + 1) / W;
     if (threadIdx.x == 0) griddep_launch_dependents();
 
     // the warp's row groups: those whose starting weight lies in [c_lo, c_hi)
-    int pi = 0;
-    while (pi + 1 < P.count && P.cost_begin[pi + 1] <= c_lo) ++pi;
     auto first_group = [&](int q, long long c) -> long long {
         // first group j of problem q with cost_begin[q] + j cost_group[q] >= c
         const long long d = c - P.cost_begin[q];
         if (d <= 0) return 0;
         return (d + P.cost_group[q] - 1) / P.cost_group[q];
     };
+    // (pi, g) advanced by k groups of the warp's sequence; false past its end
+    auto advance = [&](int &q, long long &j, long long k) -> bool {
+        j += k;
+        while (q < P.count && P.cost_begin[q] < c_hi) {
+            const long long last = min((long long)P.p[q].tiles_m, first_group(q, c_hi));
+            if (j < last) return true;
+            j -= last;  // the groups past this problem continue in the next one
+            ++q;
+        }
+        return false;
+    };
+    int pi = 0;
+    while (pi + 1 < P.count && P.cost_begin[pi + 1] <= c_lo) ++pi;
     long long g = first_group(pi, c_lo);
-    bool waited = !P.pre_w;
-    if (waited) griddep_wait();
+    bool have = advance(pi, g, 0);
+    // The weights of a group's first step are loaded before the group begins
+    // (the previous group's epilogue, or the wait for the previous kernel,
+    // overlaps them).
+    Step<BITS, MT> st;
+    if (have && P.pre_w)
+        load_weights(st, P.p[pi], (int)g * R, min(R, P.p[pi].N - (int)g * R), 0, lane);
+    griddep_wait();  // x, parameters and outputs only after the previous kernel
+    if (have && !P.pre_w)
+        load_weights(st, P.p[pi], (int)g * R, min(R, P.p[pi].N - (int)g * R), 0, lane);
     int xsum[MT];
     int cur_pi = -1;
-    for (; pi < P.count && P.cost_begin[pi] < c_hi; ++pi, g = 0) {
+    while (have) {
         const Problem &p = P.p[pi];
-        const long long g_end = min((long long)p.tiles_m, first_group(pi, c_hi));
-        const int L = p.K * BITS / 8;
-        const int nsteps = (L + STEP - 1) / STEP;
-        for (; g < g_end; ++g) {
-            const int n0 = (int)g * R;
-            const int rows = min(R, p.N - n0);
-            Step<BITS, MT> st;
-            load_weights(st, p, n0, rows, 16 * lane);
-            if (!waited) {  // x, parameters and outputs only after the previous kernel
-                griddep_wait();
-                waited = true;
+        const int nsteps = (p.K * BITS / 8 + STEP - 1) / STEP;
+        const int n0 = (int)g * R;
+        const int rows = min(R, p.N - n0);
+        const bool first = pi != cur_pi;  // the warp's first group of this problem
+        cur_pi = pi;
+        // this lane's output, if any: value lane / (32 / NV) of the reduce-scatter
+        const int vi = lane / (32 / NV);
+        const int er = vi / MT, em = vi % MT;
+        const bool owner = lane % (32 / NV) == 0 && er < rows && em < p.M;
+        int32_t colsum = 0, m0 = 0, sh = 33, zw = 0, res = 0;
+        if (owner) {
+            const int n = n0 + er;
+            colsum = __ldg(p.colsum + n);
+            m0 = __ldg(p.M0 + n);
+            sh = __ldg(p.shift + n);
+            if (p.zw) zw = __ldg(p.zw + n);
+            if (p.residual) res = p.residual[(size_t)em * p.ldy + n];
+        }
+        int acc[NV], acc_hi[BITS == 4 ? NV : 1];
+        int xs[MT];
+#pragma unroll
+        for (int i = 0; i < NV; ++i) acc[i] = 0;
+#pragma unroll
+        for (int i = 0; i < (BITS == 4 ? NV : 1); ++i) acc_hi[i] = 0;
+#pragma unroll
+        for (int m = 0; m < MT; ++m) xs[m] = 0;
+        for (int s = 0; s < nsteps; ++s) {
+            if (s > 0) load_weights(st, p, n0, rows, s * STEP, lane);
+            load_x(st, p, s * STEP, lane);
+            if (first) {
+#pragma unroll
+                for (int m = 0; m < MT; ++m)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int i = 0; i < 8 / BITS; ++i) xs[m] = sum4(st.x[m][h][i], xs[m]);
             }
-            const bool first = pi != cur_pi;  // the warp's first group of this problem
-            cur_pi = pi;
-            // this lane's output, if any: value (lane >> 3) of the reduce-scatter
-            const int vi = NV == 4 ? (lane >> 3) : 2 * (lane >> 3) + ((lane >> 2) & 1);
-            const int er = MT == 1 ? vi : vi >> 1, em = MT == 1 ? 0 : vi & 1;
-            const bool owner = (lane & (NV == 4 ? 7 : 3)) == 0 && er < rows && em < p.M;
-            int32_t colsum = 0, m0 = 0, sh = 33, zw = 0, res = 0;
-            if (owner) {
-                const int n = n0 + er;
-                colsum = __ldg(p.colsum + n);
-                m0 = __ldg(p.M0 + n);
-                sh = __ldg(p.shift + n);
-                if (p.zw) zw = __ldg(p.zw + n);
-                if (p.residual) res = p.residual[(size_t)em * p.ldy + n];
-            }
-            int acc[NV];
-            int xs[MT];
+            if constexpr (BITS == 4) {
 #pragma unroll
-            for (int i = 0; i < NV; ++i) acc[i] = 0;
+                for (int m = 0; m < MT; ++m)
 #pragma unroll
-            for (int m = 0; m < MT; ++m) xs[m] = 0;
-            for (int s = 0; s < nsteps; ++s) {
-                if (s > 0) load_weights(st, p, n0, rows, s * STEP + 16 * lane);
-                load_x(st, p, s * STEP + 16 * lane);
-                if (first) {
+                    for (int h = 0; h < 2; ++h) {
+                        const XEO x = x_even_odd(st.x[m][h][0], st.x[m][h][1]);
 #pragma unroll
-                    for (int m = 0; m < MT; ++m)
-#pragma unroll
-                        for (int h = 0; h < 2; ++h)
-#pragma unroll
-                            for (int i = 0; i < 8 / BITS; ++i) xs[m] = sum4(st.x[m][h][i], xs[m]);
-                }
+                        for (int r = 0; r < R; ++r)
+                            dot16_i4(st.w[r][h], x, acc[r * MT + m], acc_hi[r * MT + m]);
+                    }
+            } else {
 #pragma unroll
                 for (int r = 0; r < R; ++r)
 #pragma unroll
                     for (int m = 0; m < MT; ++m)
 #pragma unroll
                         for (int h = 0; h < 2; ++h)
-                            acc[r * MT + m] = dot16<BITS>(st.w[r][h], st.x[m][h], acc[r * MT + m]);
-            }
-            if (first) {
-#pragma unroll
-                for (int m = 0; m < MT; ++m) {
-#pragma unroll
-                    for (int bit = 16; bit >= 1; bit >>= 1)
-                        xs[m] += __shfl_xor_sync(0xffffffffu, xs[m], bit);
-                    xsum[m] = xs[m];
-                }
-            }
-            const int sum = reduce_scatter<NV>(acc, lane);
-            if (owner) {
-                const int n = n0 + er;
-                const int32_t xsm = MT == 1 ? xsum[0] : (em ? xsum[MT - 1] : xsum[0]);
-                // sum(w x) = sum(u x) - 8 sum(x) (int4); then the zero points:
-                // sum((x - zx)(w - zw)) = sum(w x) - zw sum(x) - zx (colsum - K zw)
-                // (two's-complement wrap is exact: the true value fits int32)
-                const uint32_t wx = (uint32_t)sum - (uint32_t)(BITS == 4 ? 8 * xsm : 0);
-                const int32_t a =
-                    (int32_t)(wx - (uint32_t)zw * (uint32_t)xsm -
-                              (uint32_t)p.zx * ((uint32_t)colsum - (uint32_t)p.K * (uint32_t)zw));
-                if constexpr (O16) {
-                    reinterpret_cast<int16_t *>(p.y)[(size_t)em * p.ldy + n] =
-                        (int16_t)mq_requant16((int64_t)a, m0, sh, p.zy);
-                } else {
-                    int32_t y = mq_requant(a, m0, sh, p.zy);
-                    if (p.residual) y = min(127, max(-128, y + res));
-                    p.y[(size_t)em * p.ldy + n] = (int8_t)y;
-                }
+                            acc[r * MT + m] = dp4a4(st.w[r][h], st.x[m][h][0], acc[r * MT + m]);
             }
         }
+        if constexpr (BITS == 4) {
+            // the high nibbles' sums are exact multiples of 16
+#pragma unroll
+            for (int i = 0; i < NV; ++i) acc[i] += acc_hi[i] >> 4;
+        }
+        // the next group's first weights go out before this group's epilogue
+        int npi = pi;
+        long long ng = g;
+        have = advance(npi, ng, 1);
+        if (have) load_weights(st, P.p[npi], (int)ng * R, min(R, P.p[npi].N - (int)ng * R), 0,
+                               lane);
+        if (first) {
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+#pragma unroll
+                for (int bit = 16; bit >= 1; bit >>= 1)
+                    xs[m] += __shfl_xor_sync(0xffffffffu, xs[m], bit);
+                xsum[m] = xs[m];
+            }
+        }
+        const int sum = reduce_scatter<NV>(acc, lane);
+        if (owner) {
+            const int n = n0 + er;
+            const int32_t xsm = MT == 1 ? xsum[0] : (em ? xsum[MT - 1] : xsum[0]);
+            // sum(w x) = sum(u x) - 8 sum(x) (int4); then the zero points:
+            // sum((x - zx)(w - zw)) = sum(w x) - zw sum(x) - zx (colsum - K zw)
+            // (two's-complement wrap is exact: the true value fits int32)
+            const uint32_t wx = (uint32_t)sum - (uint32_t)(BITS == 4 ? 8 * xsm : 0);
+            const int32_t a =
+                (int32_t)(wx - (uint32_t)zw * (uint32_t)xsm -
+                          (uint32_t)p.zx * ((uint32_t)colsum - (uint32_t)p.K * (uint32_t)zw));
+            if constexpr (O16) {
+                reinterpret_cast<int16_t *>(p.y)[(size_t)em * p.ldy + n] =
+                    (int16_t)mq_requant16((int64_t)a, m0, sh, p.zy);
+            } else {
+                int32_t y = mq_requant(a, m0, sh, p.zy);
+                if (p.residual) y = min(127, max(-128, y + res));
+                p.y[(size_t)em * p.ldy + n] = (int8_t)y;
+            }
+        }
+        pi = npi;
+        g = ng;
     }
-    if (!waited) griddep_wait();  // a warp without work still orders after its predecessor
 }
 
 template <int BITS, int MT, bool O16>
@@ -314,7 +394,7 @@ int launch_t(const Problem *probs, int count, cudaStream_t stream) {
         P.cost_begin[n] = cost;
         P.count = n;
         if (groups == 0) continue;
-        long long warps = (long long)CTAS_PER_SM * sms * WARPS;
+        long long warps = (long long)ctas_per_sm<MT>() * sms * WARPS;
         if (warps > groups) warps = groups;
         const int grid = (int)((warps + WARPS - 1) / WARPS);
         cudaLaunchConfig_t cfg{};
@@ -342,12 +422,15 @@ bool gemv_suits(const Problem *probs, int count, int sms, bool force) {
     using namespace gemv;
     if (count <= 0) return false;
     long long groups = 0;
+    int mt = 0;
     for (int i = 0; i < count; ++i) {
         const Problem &q = probs[i];
         if (q.a16 || q.M < 1 || q.M > MAX_MT || q.K <= 0 || q.N <= 0) return false;
         groups += (q.N + R - 1) / R;
+        mt = q.M > mt ? q.M : mt;
     }
-    return force || groups >= (long long)CTAS_PER_SM * sms * WARPS;
+    const int occ = mt == 1 ? ctas_per_sm<1>() : ctas_per_sm<2>();
+    return force || groups >= (long long)occ * sms * WARPS;
 }
 
 int launch_gemv(const Problem *probs, int count, void *stream) {
