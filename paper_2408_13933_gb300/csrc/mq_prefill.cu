@@ -33,8 +33,9 @@
 // TMEM columns: F[0] 0-127, F[1] 128-255, A stages 256 + 64 s.
 // Warp roles (both CTAs):
 //   warp 0     : TMA producer (one thread) for this CTA's weight and token rows.
-//   warp 1     : TMEM allocation; in the even CTA one thread issues the MMAs
-//                and the commits (multicast to both CTAs' barriers).
+//   warp 1     : TMEM allocation; in the even CTA the warp runs the MMA loop
+//                and one elected lane issues the MMAs and the commits
+//                (multicast to both CTAs' barriers).
 //   warps 2-9  : converters, two groups of four taking alternate stages.  In
 //                its stage warp w writes TMEM lanes 32 (w % 4) .. +31 (its
 //                weight rows, all 128 k) and widens four 16-byte chunks of
@@ -313,7 +314,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             mbar_init(&s.f_full[b], 1);
             mbar_init(&s.f_empty[b], 2 * EPI_WARPS);
         }
-        mbar_init(&s.done, 1);
+        mbar_init(&s.done, 32);  // one commit from every lane of the MMA warp
         s.abort = 0;
         fence_mbar_init();
     }
@@ -389,7 +390,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         __syncwarp();
     } else if (warp == MMA_WARP) {
         // ------------------------------------------------------ MMA issuer
-        if (rank == 0 && lane == 0) {
+        // The whole warp runs the loop (warp-uniform control flow: lane 0
+        // waits, the verdict is broadcast) and one elected lane issues the
+        // MMAs and commits.  Issued from a lone lane behind its waits, pair
+        // MMAs of N = 128 ran at 86-94 cycles instead of 64 (measured).
+        if (rank == 0) {
             const uint32_t idesc = idesc_f16_f32(TM, TN);
             uint32_t it = 0, chunks = 0;
             bool ok = true;
@@ -401,17 +406,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     const bool chunk_start = kc == 0;
                     if (chunk_start) {
                         const uint32_t b = chunks & 1;
-                        if (!mq_wait_parity(&s.f_empty[b], ((chunks >> 1) & 1) ^ 1, &s.abort,
-                                            P.status, P.wait_ns)) {
+                        if (!warp_wait(&s.f_empty[b], ((chunks >> 1) & 1) ^ 1, s, P)) {
                             ok = false;
                             break;
                         }
-                        tc_fence_after();
                         fcol = F_COL0 + 128 * b;
                     }
                     const int slot = it % SF;
-                    if (!mq_wait_parity(&s.op_full[slot], (it / SF) & 1, &s.abort, P.status,
-                                        P.wait_ns)) {
+                    if (!warp_wait(&s.op_full[slot], (it / SF) & 1, s, P)) {
                         ok = false;
                         break;
                     }
@@ -419,26 +421,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     const uint32_t acol = tmem + A_COL0 + 64 * slot;
                     const uint64_t bd0 = smem_desc_sw128(smem_u32(s.opb[slot]));
                     const uint64_t bd1 = smem_desc_sw128(smem_u32(s.opb[slot] + ATOM));
+                    const bool chunk_end = ++kc == t.kpc || kb + 1 == t.nkb;
+                    if (elect_one()) {
 #pragma unroll
-                    for (int j = 0; j < KS / 16; ++j)  // +32 B along K: +2 in the (addr >> 4) field
-                        tc_mma2_f16_ts(tmem + fcol, acol + 8 * j,
-                                       (j < 4 ? bd0 : bd1) + 2 * (j & 3), idesc,
-                                       (chunk_start && j == 0) ? 0u : 1u);
-                    tc_commit2_mc(&s.op_empty[slot], 3);
-                    if (++kc == t.kpc || kb + 1 == t.nkb) {
-                        tc_commit2_mc(&s.f_full[chunks & 1], 3);
+                        for (int j = 0; j < KS / 16; ++j)  // +32 B along K: +2 in the (addr >> 4) field
+                            tc_mma2_f16_ts(tmem + fcol, acol + 8 * j,
+                                           (j < 4 ? bd0 : bd1) + 2 * (j & 3), idesc,
+                                           (chunk_start && j == 0) ? 0u : 1u);
+                        tc_commit2_mc(&s.op_empty[slot], 3);
+                        if (chunk_end) tc_commit2_mc(&s.f_full[chunks & 1], 3);
+                    }
+                    __syncwarp();
+                    if (chunk_end) {
                         ++chunks;
                         kc = 0;
                     }
                 }
             }
-            if (!ok) abort_pair(s, rank);
+            if (!ok && lane == 0) abort_pair(s, rank);
             // every MMA issued above has completed once `done` fires; wait for
             // it even after giving up (bounded, ignoring the abort word): the
             // MMAs read both CTAs' operands and write their tensor memory,
-            // which is released after the final cluster barrier
+            // which is released after the final cluster barrier.  Every lane
+            // commits (`done` counts 32 arrivals), so the phase follows the
+            // MMAs of whichever lane the elections picked.
             tc_commit2_mc(&s.done, 1);
-            mq_wait_parity_drain(&s.done, 0, P.status, P.wait_ns);
+            if (lane == 0) mq_wait_parity_drain(&s.done, 0, P.status, P.wait_ns);
         }
         __syncwarp();
     } else if (warp < EPI_WARP0) {
