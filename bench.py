@@ -817,10 +817,15 @@ class Stack:
         self.launches = len(calls_a)
         self.h2d_bytes = x0.size
         self.d2h_bytes = m * hn
+        # one workspace for every call (its widened inputs are scratch; the
+        # calls run one after another on one stream)
+        self.ws_bytes = max(mq.workspace_size_batch(list(a)) for a, _ in calls_a + calls_b)
+        self.ws = torch.zeros(max(16, self.ws_bytes), dtype=torch.uint8, device=dev)
 
     def enqueue(self, mq, sp: int, j: int = 0):
+        wsp = self.ws.data_ptr() if self.ws_bytes else None
         for a, n in self.calls[j]:
-            rc = mq.lib.mq_linear_batch(a, n, None, 0, sp)
+            rc = mq.lib.mq_linear_batch(a, n, wsp, self.ws_bytes, sp)
             if rc:
                 raise RuntimeError(f"mq_linear_batch failed: {mq.status_string(rc)}")
 
@@ -1029,8 +1034,13 @@ class DeviceCalls:
                                           c.zy, y, bits))
             self.calls.append(((mq.LinearDesc * len(descs))(*descs), len(descs)))
         self.keep += list(xdev.values())
+        self.ws_bytes = max(mq.workspace_size_batch(list(a)) for a, _ in self.calls)
+        self.ws = torch.zeros(max(16, self.ws_bytes), dtype=torch.uint8, device="cuda")
 
     def enqueue(self, mq, sp, ws=None, ws_bytes=0, which=None):
+        """One batched call per group; without `ws`, the calls' own workspace."""
+        if ws is None and self.ws_bytes:
+            ws, ws_bytes = self.ws.data_ptr(), self.ws_bytes
         for i, (a, n) in enumerate(self.calls):
             if which is None or i in which:
                 rc = mq.lib.mq_linear_batch(a, n, ws, ws_bytes, sp)

@@ -98,18 +98,24 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed,
                     int32_t *colsum, int on_device, void *stream);
 
 /*
- * Device workspace bytes a mq_linear_* call of this shape needs: 0 for the
- * tensor-core path (M > 16); for the decode path (1 <= M <= 16) a fixed size
- * (2.5 MB) holding, per CTA of the decode grid, int32 partial sums tagged with
- * a launch number, used to combine 64-row units whose K range is split among
- * CTAs.  For
- * mq_linear_batch the workspace must hold the largest size of its
- * descriptors.
+ * Device workspace bytes a mq_linear_* call of this shape needs or can use.
+ * Decode path (1 <= M <= 16): a fixed size (2.5 MB, the decode region)
+ * holding, per CTA of the decode grid, int32 partial sums tagged with a
+ * launch number, used to combine 64-row units whose K range is split among
+ * CTAs.  Tensor-core path (M > 16) from M = 256 tokens on: room for the
+ * 256-token kernel's widened input, i.e. an f16 copy of x (2 M K bytes) and
+ * its row sums of squares (4 M bytes), placed after the size of the decode
+ * region, each rounded up to 1024 bytes, plus 1024 bytes of alignment slack.
+ * That part is optional: a prefill call given less (even no workspace) runs
+ * the 128-token kernel instead, bit-identical and slower.  Smaller M: 0.  For
+ * mq_linear_batch use mq_workspace_size_batch.
  * Workspace contract: device memory, 16-byte aligned, zero-filled before its
- * first use; every call that completes leaves it zero-filled again, so it can
- * be reused by later calls on the same stream.  Calls that may run
+ * first use.  The decode region (the first mq_workspace_size(1, 1, 0, 4)
+ * bytes) is left zero-filled again by every call that completes, so the
+ * workspace can be reused by later calls on the same stream; the widened
+ * inputs after it are scratch, overwritten by each call.  Calls that may run
  * concurrently (different streams) need different workspaces.  After
- * MQ_ERR_DEVICE_TIMEOUT the workspace must be zero-filled again.
+ * MQ_ERR_DEVICE_TIMEOUT the decode region must be zero-filled again.
  * Errors: MQ_ERR_INVALID_ARG.
  */
 int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes);
@@ -318,11 +324,17 @@ typedef struct mq_linear_desc {
  * (rounded up to 128) for every distinct input (x, M, K, ldx) of the
  * descriptors with abits 16 and 2M > 16, which holds its two int8 planes
  * (filled by the call; descriptors reading the same input, e.g. q/k/v/gate/up
- * of one block, share them).  0 when none applies.  The decode region (the
- * first mq_workspace_size bytes, when present) follows the contract of
+ * of one block, share them).  Then, optionally, room for the 256-token
+ * prefill kernel (see mq_workspace_size): for every distinct 8-bit input of
+ * the descriptors with abits 8, obits 8 and M >= 256, its f16 copy (2 M K
+ * bytes) and row sums of squares (4 M bytes), each rounded up to 1024, placed
+ * after the decode region's size, plus 1024 bytes of alignment slack; a call
+ * given only the required part runs those descriptors on the 128-token
+ * kernel.  0 when none applies.  The decode region (the first
+ * mq_workspace_size(1, 1, 0, 4) bytes) follows the contract of
  * mq_workspace_size: zero-filled before first use and left zero by every
- * call that completes; the plane regions are scratch, overwritten by each
- * call.
+ * call that completes; the plane and widened-input regions are scratch,
+ * overwritten by each call.
  * Errors: MQ_ERR_INVALID_ARG (null pointers, count out of range, bad bits or
  * abits).
  */
@@ -514,6 +526,18 @@ int mq_test_skip_partials(int cta);
  * Errors: MQ_ERR_INVALID_ARG for values other than 0, 1, 2.
  */
 int mq_test_decode_kernel(int which);
+
+/*
+ * Test hook, not for production: the choice between the two prefill kernels
+ * for problems with 8-bit activations and outputs (M > 16).  0 (the initial
+ * state) takes the 256-token kernel for M >= 256 when the workspace has room
+ * for the widened inputs (mq_workspace_size, mq_workspace_size_batch count
+ * it), the 128-token kernel otherwise.  1 takes the 256-token kernel for every
+ * such problem the workspace allows, 2 never.  Both are bit-exact; the hook
+ * lets the tests run either one on any shape.
+ * Errors: MQ_ERR_INVALID_ARG for values other than 0, 1, 2.
+ */
+int mq_test_prefill_kernel(int which);
 
 #ifdef __cplusplus
 }

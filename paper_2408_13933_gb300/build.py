@@ -23,7 +23,7 @@ ROOT = os.path.dirname(HERE)
 INCLUDE = os.path.join(ROOT, "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["mq_host.cpp", "mq_pack.cu", "mq_decode.cu", "mq_gemv.cu", "mq_prefill.cu",
+SOURCES = ["mq_host.cpp", "mq_pack.cu", "mq_decode.cu", "mq_gemv.cu", "mq_prefill.cu", "mq_prefill2.cu",
            "mq_noalloc.cu", "mq_glue.cu", "mq_fold.cu"]
 
 

@@ -18,11 +18,13 @@ constexpr uint64_t DEFAULT_WAIT_NS = 1000000000ull;  // 1 second
 std::atomic<uint64_t> g_wait_ns{DEFAULT_WAIT_NS};
 std::atomic<int> g_skip_cta{-1};
 std::atomic<int> g_decode_kernel{0};
+std::atomic<int> g_prefill_kernel{0};
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_ns.load(std::memory_order_relaxed); }
 int test_skip_cta() { return g_skip_cta.load(std::memory_order_relaxed); }
 int test_decode_kernel() { return g_decode_kernel.load(std::memory_order_relaxed); }
+int test_prefill_kernel() { return g_prefill_kernel.load(std::memory_order_relaxed); }
 
 }  // namespace mq
 
@@ -94,21 +96,47 @@ size_t align16(size_t v) { return (v + 15) & ~static_cast<size_t>(15); }
 
 size_t align128(size_t v) { return (v + 127) & ~static_cast<size_t>(127); }
 
+size_t align1024(size_t v) { return (v + 1023) & ~static_cast<size_t>(1023); }
+
 // A decode shape: at most DECODE_MAX_M rows of the (plane) matrix.
 bool is_decode(const mq_linear_desc &d) {
     const int64_t rows = abits_of(d) == 16 ? 2LL * d.M : d.M;
     return rows > 0 && rows <= mq::DECODE_MAX_M;
 }
 
+// Smallest M that takes the 256-token prefill kernel by default (below it
+// the 128-token kernel's tiles fill the GPU better).
+constexpr int WIDE_MIN_M = 256;
+
+// A problem served by the 256-token prefill kernel (mq_prefill2.cu) when the
+// workspace has room for its widened input: a tensor-core shape with 8-bit
+// activations and output.
+bool wide_eligible(const mq_linear_desc &d) {
+    if (d.M <= 0 || d.N <= 0 || d.K <= 0 || is_decode(d)) return false;
+    if (abits_of(d) != 8 || obits_of(d) != 8) return false;
+    const int which = mq::test_prefill_kernel();
+    if (which == 2) return false;
+    return which == 1 || d.M >= WIDE_MIN_M;
+}
+
 // Workspace layout of one batch: the decode region first (if any decode
 // shape), then one [2M][K] int8 plane matrix per distinct input (x, M, K,
 // ldx) of the 16-bit tensor-core descriptors, in order of first use, with
-// offsets relative to the end of the decode region.
+// offsets relative to the end of the decode region.  These make the required
+// size.  Then, optionally, from the first 1024-byte boundary after both the
+// required part and the decode region's size (so that it never overlaps the
+// decode region of another call sharing the workspace), the f16 copy [M][K]
+// and the row sums of squares [M] of every distinct input of the problems the
+// 256-token prefill kernel serves: with room for them the batch takes that
+// kernel, without it the 128-token one.  That region is scratch.
 struct Plan {
     bool any_decode = false;
     std::vector<mq::SplitJob> split;
     std::vector<size_t> split_off;
-    size_t bytes = 0;
+    std::vector<mq::Widen16Job> wide;
+    std::vector<size_t> wide_off;  // f16 copy at wide_off, row sums at + align1024(2 M K)
+    size_t required = 0;           // decode region + planes
+    size_t bytes = 0;              // required + the widened inputs (if any)
 };
 
 template <class J>
@@ -116,6 +144,11 @@ int find_job(const std::vector<J> &jobs, const void *x, int M, int K, int ldx) {
     for (size_t i = 0; i < jobs.size(); ++i)
         if (jobs[i].x == x && jobs[i].M == M && jobs[i].K == K && jobs[i].ldx == ldx) return (int)i;
     return -1;
+}
+
+// Where the widened inputs may start (before rounding up to 1024 bytes).
+size_t wide_at(const Plan &pl) {
+    return pl.required > mq::DECODE_WS_BYTES ? pl.required : mq::DECODE_WS_BYTES;
 }
 
 Plan batch_plan(const mq_linear_desc *descs, int count) {
@@ -142,7 +175,27 @@ Plan batch_plan(const mq_linear_desc *descs, int count) {
         pl.split_off.push_back(off);
         off += align128(2 * (size_t)d.M * (size_t)d.K);
     }
-    pl.bytes = (pl.any_decode ? mq::DECODE_WS_BYTES : 0) + off;
+    pl.required = (pl.any_decode ? mq::DECODE_WS_BYTES : 0) + off;
+    size_t woff = 0;
+    for (int i = 0; i < count; ++i) {
+        const mq_linear_desc &d = descs[i];
+        if (!wide_eligible(d)) continue;
+        const int8_t *x = static_cast<const int8_t *>(d.x);
+        bool seen = false;
+        for (const auto &j : pl.wide)
+            seen = seen || (j.x == x && j.M == d.M && j.K == d.K && j.ldx == d.ldx);
+        if (seen) continue;
+        mq::Widen16Job j{};
+        j.x = x;
+        j.M = d.M;
+        j.K = d.K;
+        j.ldx = d.ldx;
+        pl.wide.push_back(j);
+        pl.wide_off.push_back(woff);
+        woff += align1024(2 * (size_t)d.M * (size_t)d.K) + align1024(4 * (size_t)d.M);
+    }
+    // + 1024: the region starts at the first 1024-byte boundary after wide_at()
+    pl.bytes = pl.wide.empty() ? pl.required : wide_at(pl) + woff + 1024;
     return pl;
 }
 
@@ -157,11 +210,26 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
     // the decode kernel combines split 64-row units in the workspace, 16-bit
     // tensor-core descriptors read their int8 planes from there
     Plan pl = batch_plan(descs, count);
-    if (pl.bytes > 0 && (!workspace || ws_bytes < pl.bytes || !aligned16(workspace)))
+    if (pl.required > 0 && (!workspace || ws_bytes < pl.required || !aligned16(workspace)))
         return MQ_ERR_WORKSPACE;
     uint8_t *region = static_cast<uint8_t *>(workspace) + (pl.any_decode ? mq::DECODE_WS_BYTES : 0);
     for (size_t i = 0; i < pl.split.size(); ++i)
         pl.split[i].out = reinterpret_cast<int8_t *>(region + pl.split_off[i]);
+    // the 256-token kernel when the workspace has room for the widened inputs
+    const bool wide = !pl.wide.empty() && workspace && ws_bytes >= pl.bytes && mq::prefill2_ready();
+    if (wide) {
+        const uintptr_t base =
+            (reinterpret_cast<uintptr_t>(workspace) + wide_at(pl) + 1023) & ~(uintptr_t)1023;
+        for (size_t i = 0; i < pl.wide.size(); ++i) {
+            uint8_t *at = reinterpret_cast<uint8_t *>(base + pl.wide_off[i]);
+            pl.wide[i].out = reinterpret_cast<uint16_t *>(at);
+            pl.wide[i].rowsq = reinterpret_cast<int32_t *>(
+                at + align1024(2 * (size_t)pl.wide[i].M * (size_t)pl.wide[i].K));
+        }
+    }
+    std::vector<mq::Problem> pre2;
+    std::vector<const uint16_t *> pre2_x16;
+    std::vector<const int32_t *> pre2_rowsq;
     // kernel families: prefill by activation / output width, decode by weight
     // bits and activation / output width (0: 8 / 8, 1: 16 / 16, 2: 8 / 16)
     std::vector<mq::Problem> pre[3], dec[2][3];
@@ -178,14 +246,28 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
             }
         }
         const int mode = p.a16 ? 1 : (p.o16 ? 2 : 0);
-        if (is_decode(d))
+        if (is_decode(d)) {
             dec[p.bits == 8][mode].push_back(p);
-        else
+        } else if (wide && wide_eligible(d)) {
+            const mq::Widen16Job *job = nullptr;
+            for (const auto &j : pl.wide)
+                if (j.x == p.x && j.M == d.M && j.K == d.K && j.ldx == d.ldx) job = &j;
+            pre2.push_back(p);
+            pre2_x16.push_back(job->out);
+            pre2_rowsq.push_back(job->rowsq);
+        } else {
             pre[mode].push_back(p);
+        }
     }
     int rc = MQ_OK;
     if (!pl.split.empty())
         rc = mq::launch_split16(pl.split.data(), (int)pl.split.size(), stream);
+    if (rc == MQ_OK && !pre2.empty()) {
+        rc = mq::launch_widen16(pl.wide.data(), (int)pl.wide.size(), stream);
+        if (rc == MQ_OK)
+            rc = mq::launch_prefill2(pre2.data(), pre2_x16.data(), pre2_rowsq.data(),
+                                     (int)pre2.size(), stream);
+    }
     for (int mode = 0; mode < 3; ++mode)
         if (rc == MQ_OK && !pre[mode].empty())
             rc = mq::launch_prefill(pre[mode].data(), (int)pre[mode].size(), stream);
@@ -356,7 +438,14 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed, int32
 
 int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes) {
     if (!bytes || M < 0 || N < 0 || K < 0 || (bits != 8 && bits != 4)) return MQ_ERR_INVALID_ARG;
-    *bytes = (M > 0 && M <= mq::DECODE_MAX_M && N > 0) ? mq::DECODE_WS_BYTES : 0;
+    mq_linear_desc d{};
+    d.x = reinterpret_cast<const void *>(16);  // a placeholder address: only sizes are planned
+    d.M = M;
+    d.N = N;
+    d.K = K;
+    d.ldx = K;
+    d.bits = bits;
+    *bytes = batch_plan(&d, 1).bytes;
     return MQ_OK;
 }
 
@@ -578,6 +667,12 @@ int mq_test_skip_partials(int cta) {
 int mq_test_decode_kernel(int which) {
     if (which < 0 || which > 2) return MQ_ERR_INVALID_ARG;
     mq::g_decode_kernel.store(which, std::memory_order_relaxed);
+    return MQ_OK;
+}
+
+int mq_test_prefill_kernel(int which) {
+    if (which < 0 || which > 2) return MQ_ERR_INVALID_ARG;
+    mq::g_prefill_kernel.store(which, std::memory_order_relaxed);
     return MQ_OK;
 }
 

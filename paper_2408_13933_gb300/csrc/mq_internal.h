@@ -104,6 +104,28 @@ struct SplitJob {
 constexpr int SPLIT_MAX_JOBS = 64;
 int launch_split16(const SplitJob *jobs, int count, void *stream);
 
+// One distinct int8 input of a batch widened for the 256-token prefill kernel
+// (mq_prefill2.cu): out = f16 copy [M][K] (pitch K), rowsq[m] = sum_k x[m][k]^2.
+struct Widen16Job {
+    const int8_t *x;
+    uint16_t *out;
+    int32_t *rowsq;
+    int32_t M, K, ldx;
+};
+constexpr int WIDEN16_MAX_JOBS = 64;
+int launch_widen16(const Widen16Job *jobs, int count, void *stream);
+// The 256-token prefill kernel: problems with 8-bit activations and output;
+// x16[i] / rowsq[i] are problem i's widened input and row sums of squares.
+int launch_prefill2(const Problem *probs, const uint16_t *const *x16, const int32_t *const *rowsq,
+                    int count, void *stream);
+// Whether the 256-token kernel can run on the current device (set-up done
+// once per device; false when its register split does not fit the compiled
+// kernel's launch allocation).
+bool prefill2_ready();
+// Test hook (mq_test_prefill_kernel): 0 chooses the prefill kernel by shape and
+// workspace, 1 takes the 256-token kernel whenever it can serve a problem, 2 never.
+int test_prefill_kernel();
+
 // Boundary quantizers (mq_glue.cu): kind 0 quantize (float -> codes),
 // 1 dequantize (codes -> f32), 2 requantize (codes -> codes); types are the
 // MQ_TYPE_* of mq.h; [lo, hi] is the output code range.

@@ -42,7 +42,7 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16", "mq_quantize",
             "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm",
             "mq_row_sums", "mq_head_row_sums", "mq_transpose_i8", "mq_set_wait_limit_ns",
-            "mq_test_skip_partials", "mq_test_decode_kernel"]
+            "mq_test_skip_partials", "mq_test_decode_kernel", "mq_test_prefill_kernel"]
 MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
@@ -386,3 +386,9 @@ def test_decode_kernel(which: int) -> int:
     """mq_test_decode_kernel (test hook): 0 by shape, 1 the row-tile kernel
     whenever it can serve the launch, 2 never."""
     return lib.mq_test_decode_kernel(int(which))
+
+
+def test_prefill_kernel(which: int) -> int:
+    """mq_test_prefill_kernel (test hook): 0 by shape and workspace, 1 the
+    256-token kernel whenever the workspace allows, 2 never."""
+    return lib.mq_test_prefill_kernel(int(which))

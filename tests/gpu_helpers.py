@@ -15,16 +15,27 @@ def torch_cuda():
 
 
 _WS = None
+# room for the 256-token prefill kernel's widened inputs of every shape the
+# tests run through this workspace (2 M K + 4 M bytes after the decode region)
+WS_BYTES = 256 << 20
 
 
 def workspace():
-    """One zero-filled decode workspace shared by the tests (every call leaves
-    it zero-filled again)."""
+    """One zero-filled workspace shared by the tests: the decode region (left
+    zero-filled by every call) and room for widened prefill inputs (scratch)."""
     global _WS
     if _WS is None:
+        torch = torch_cuda()
         from paper_2408_13933_gb300 import mq
-        _WS = mq.workspace()
+        _WS = torch.zeros(max(WS_BYTES, mq.workspace_size(1, 1, 0, 4)), dtype=torch.uint8,
+                          device="cuda")
     return _WS
+
+
+def decode_region():
+    """The decode region of the shared workspace (zero-filled between calls)."""
+    from paper_2408_13933_gb300 import mq
+    return workspace()[:mq.workspace_size(1, 1, 0, 4)]
 
 
 def upload(a: np.ndarray):

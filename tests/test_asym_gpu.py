@@ -13,6 +13,16 @@ from paper_2408_13933_gb300 import synth
 pytestmark = pytest.mark.gpu
 
 
+@pytest.fixture(autouse=True, params=[1, 2], ids=["tile256", "tile128"])
+def prefill_kernel(request):
+    """Every test runs on both prefill kernels: the 256-token one wherever the
+    workspace allows (1), and the 128-token one (2)."""
+    from paper_2408_13933_gb300 import mq
+    assert mq.test_prefill_kernel(request.param) == 0
+    yield request.param
+    assert mq.test_prefill_kernel(0) == 0
+
+
 def mq():
     from paper_2408_13933_gb300 import mq as m
     return m
@@ -129,10 +139,11 @@ def test_asym_residual(m):
     assert_equal_int8(run([c])[0], c.want(), f"asym residual m={m}")
 
 
-def test_asym_batch_mixes_kernels_and_symmetric():
+def test_asym_batch_mixes_kernels_and_symmetric(prefill_kernel):
     # decode and prefill, asymmetric and symmetric problems in one call: the
-    # workspace holds the decode region only (the tensor-core kernel folds
-    # the weight zero point into the widened weights)
+    # 128-token kernel needs the decode region only (the tensor-core kernel
+    # folds the weight zero point into the widened weights); the 256-token one
+    # adds its widened inputs after it
     a = AsymCase(51, 130, 512, 200, 8)
     b = AsymCase(52, 4, 1024, 96, 4)
     c = AsymCase(53, 70, 256, 64, 4)
@@ -143,7 +154,7 @@ def test_asym_batch_mixes_kernels_and_symmetric():
     descs[3].zw = None  # symmetric problem in the same batch
     need = lib.workspace_size_batch(descs)
     dec = lib.workspace_size(4, 96, 1024, 4)
-    assert need == dec
+    assert need == dec if prefill_kernel == 2 else need > dec
     torch = torch_cuda()
     ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
     assert lib.linear_batch(descs, workspace=ws, ws_bytes=need) == 0
@@ -153,9 +164,10 @@ def test_asym_batch_mixes_kernels_and_symmetric():
         assert_equal_int8(x.y.cpu().numpy(), x.want(), f"batch {x.c.name}")
 
 
-def test_asym_shared_input():
+def test_asym_shared_input(prefill_kernel):
     # q/k/v/gate/up-like problems reading one input (one asymmetric with zero
-    # points, one symmetric), next to another input: no workspace
+    # points, one symmetric), next to another input: no workspace for the
+    # 128-token kernel; the 256-token one widens each distinct input once
     a = AsymCase(61, 96, 512, 128, 8)
     b = AsymCase(62, 96, 512, 64, 4, share=a)
     c = AsymCase(63, 96, 512, 200, 8, share=a)
@@ -166,9 +178,13 @@ def test_asym_shared_input():
     descs = [x.desc() for x in cases]
     descs[3].zw = None
     need = lib.workspace_size_batch(descs)
-    assert need == 0
+    region = lib.workspace_size(1, 1, 0, 4)
+    if prefill_kernel == 2:
+        assert need == 0
+    else:  # two distinct inputs: f16 copies and row sums, each to 1024 bytes
+        assert need == region + (2 * 96 * 512 + 1024) + (2 * 80 * 256 + 1024) + 1024
     torch = torch_cuda()
-    ws = torch.zeros(16, dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(max(need, 16), dtype=torch.uint8, device="cuda")
     assert lib.linear_batch(descs, workspace=ws, ws_bytes=need) == 0
     torch.cuda.synchronize()
     assert lib.check_device_status() == 0

@@ -100,9 +100,15 @@ def test_host_pack_rejects_int4_out_of_range(mq):
 def test_packed_and_workspace_sizes(mq):
     assert mq.packed_size(3, 64, 8) == 192
     assert mq.packed_size(3, 64, 4) == 96
-    assert mq.workspace_size(1024, 2048, 2048, 8) == 0      # tensor-core path: none
-    assert mq.workspace_size(16, 2048, 2048, 4) > 0         # decode path: fixed size
-    assert mq.workspace_size(1, 7, 64, 8) == mq.workspace_size(16, 256000, 16384, 4)
+    dec = mq.workspace_size(16, 2048, 2048, 4)
+    assert dec > 0                                          # decode path: fixed size
+    assert mq.workspace_size(1, 7, 64, 8) == dec
+    assert mq.workspace_size(255, 2048, 2048, 8) == 0       # 128-token tensor-core kernel: none
+    # from 256 tokens on: room for the 256-token kernel's widened input after
+    # the decode region (f16 copy and row sums, each to 1024 bytes, + 1024)
+    assert mq.workspace_size(1024, 2048, 2048, 8) == dec + 2 * 1024 * 2048 + 4096 + 1024
+    assert mq.workspace_size(300, 100, 48, 4) == dec + 29696 + 2048 + 1024
+    assert mq.workspace_size(300, 100, 0, 4) == 0           # K = 0: nothing to widen
     with pytest.raises(mq.MQError):
         mq.packed_size(3, 63, 4)
     with pytest.raises(mq.MQError):

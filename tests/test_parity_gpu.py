@@ -1,5 +1,6 @@
 """GPU parity: libmq's kernels against the CPU oracle, bit for bit.
 
+Every test runs on both prefill kernels (128- and 256-token tiles).
 Shapes span several 128 x 256 tensor-core tiles with ragged M, N and K tails,
 the 1024-deep f32 accumulation chunks of the int8 path, every decode width
 M in [1, 16], both weight widths, and the degenerate cases (K = 0, one row,
@@ -9,10 +10,21 @@ equality of every int8 output.
 import numpy as np
 import pytest
 
-from gpu_helpers import GpuLinear, assert_equal_int8, oracle_y, torch_cuda, upload, workspace
+from gpu_helpers import (GpuLinear, assert_equal_int8, decode_region, oracle_y, torch_cuda, upload,
+                         workspace)
 from paper_2408_13933_gb300 import synth
 
 pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True, params=[1, 2], ids=["tile256", "tile128"])
+def prefill_kernel(request):
+    """Every test runs on both prefill kernels: the 256-token one wherever the
+    workspace allows (1), and the 128-token one (2)."""
+    from paper_2408_13933_gb300 import mq
+    assert mq.test_prefill_kernel(request.param) == 0
+    yield request.param
+    assert mq.test_prefill_kernel(0) == 0
 
 
 PREFILL_SHAPES = [
@@ -177,4 +189,4 @@ def test_decode_workspace_left_zero():
         c = synth.random_case(600 + seed, m, k, n, bits)
         assert_equal_int8(GpuLinear(c).run(), oracle_y(c), f"ws m={m} k={k}")
     torch.cuda.synchronize()
-    assert int(torch.count_nonzero(workspace())) == 0
+    assert int(torch.count_nonzero(decode_region())) == 0
