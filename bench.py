@@ -252,6 +252,7 @@ class PrefillBlock:
             packed, colsum = mq.pack_weights(c.w, 8)
             m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
             t = [torch.from_numpy(a).to(dev) for a in (packed, colsum, m0, sh)]
+            t.append(mq.weight_sq_sums(t[0], c.N, c.K, 8))
             y = self.y_all[yoff:yoff + m * c.N].view(m, c.N)
             yoff += m * c.N
             res = torch.from_numpy(c.residual).to(dev) if c.residual is not None else None
@@ -259,7 +260,7 @@ class PrefillBlock:
             self.keep += t + [a for a in (res, zw) if a is not None]
             self.y.append(y)
             self.descs.append(mq.make_desc(self.x_dev[id(c.x)], c.zx, t[0], t[1], c.N, t[2], t[3],
-                                           c.zy, y, 8, residual=res, zw=zw))
+                                           c.zy, y, 8, residual=res, zw=zw, wsq=t[4]))
         self.arr = (mq.LinearDesc * len(self.descs))(*self.descs)
         # decode shapes need the decode region; prefill (asymmetric or not) nothing
         self.ws_bytes = mq.workspace_size_batch(self.descs)
@@ -784,6 +785,7 @@ class Stack:
             packed, colsum = mq.pack_weights(c.w, 8)
             m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
             t = [up(a) for a in (packed, colsum, m0, sh)]
+            t.append(mq.weight_sq_sums(t[0], c.N, c.K, 8))
             self.keep += t
             return t
 
@@ -801,7 +803,7 @@ class Stack:
             def desc(name, xin, residual=None):
                 c, t = cs[name], w[name]
                 return mq.make_desc(xin, c.zx, t[0], t[1], c.N, t[2], t[3], c.zy, out[name], 8,
-                                    residual=residual)
+                                    residual=residual, wsq=t[4])
             xin = (self.x0[0], self.x0[1]) if li == 0 else (self.outs[li - 1]["down"],) * 2
             for j, calls in enumerate((calls_a, calls_b)):
                 calls.append(arr([desc(nm, xin[j]) for nm in ("q", "k", "v", "gate", "up")]))
@@ -812,7 +814,7 @@ class Stack:
         h = self.head
         for j, calls in enumerate((calls_a, calls_b)):
             calls.append(arr([mq.make_desc(self.outs[-1]["down"], h.zx, ht[0], ht[1], h.N, ht[2],
-                                           ht[3], h.zy, self.hy[j], 8)]))
+                                           ht[3], h.zy, self.hy[j], 8, wsq=ht[4])]))
         self.calls = (calls_a, calls_b)
         self.launches = len(calls_a)
         self.h2d_bytes = x0.size
@@ -1027,11 +1029,12 @@ class DeviceCalls:
                 packed, colsum = mq.pack_weights(c.w, bits)
                 m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
                 t = [up(a) for a in (packed, colsum, m0, sh)]
+                t.append(mq.weight_sq_sums(t[0], c.N, c.K, bits))
                 y = torch.empty((c.M, c.N), dtype=torch.int8, device="cuda")
                 self.keep += t + [y]
                 self.y[c.name] = y
                 descs.append(mq.make_desc(xdev[id(c.x)], c.zx, t[0], t[1], c.N, t[2], t[3],
-                                          c.zy, y, bits))
+                                          c.zy, y, bits, wsq=t[4]))
             self.calls.append(((mq.LinearDesc * len(descs))(*descs), len(descs)))
         self.keep += list(xdev.values())
         self.ws_bytes = max(mq.workspace_size_batch(list(a)) for a, _ in self.calls)

@@ -102,7 +102,8 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed,
  * Decode path (1 <= M <= 16): a fixed size (2.5 MB, the decode region)
  * holding, per CTA of the decode grid, int32 partial sums tagged with a
  * launch number, used to combine 64-row units whose K range is split among
- * CTAs.  Tensor-core path (M > 16) from M = 256 tokens on: room for the
+ * CTAs.  Tensor-core path (M > 16) from M = 256 tokens and N = 256 output
+ * channels on: room for the
  * 256-token kernel's widened input, i.e. an f16 copy of x (2 M K bytes) and
  * its row sums of squares (4 M bytes), placed after the size of the decode
  * region, each rounded up to 1024 bytes, plus 1024 bytes of alignment slack.
@@ -312,7 +313,21 @@ typedef struct mq_linear_desc {
     int32_t obits; /* output bits: 0 (= abits), or 16 with abits 8: int16 y, see below */
     int32_t ldw;   /* bytes between weight rows; 0: packed rows (K * bits / 8) */
     int32_t wdynamic; /* nonzero: packed is written by earlier work on the stream, see above */
+    const int32_t *wsq; /* may be NULL: device int32 [N], wsq[n] = sum_k w[n][k]^2 of the weight
+                           codes (mq_weight_sq_sums), see below */
 } mq_linear_desc;
+
+/*
+ * Weight sums of squares (`wsq`, optional, symmetric weights only): the
+ * tensor-core kernel sums the exact products in f32 runs that must stay
+ * within 2^24.  With wsq it bounds every partial sum of a tile by
+ * sqrt(max_m sum_k x[m][k]^2 * max_n wsq[n]) (Cauchy-Schwarz) and, where that
+ * bound allows, sums the whole K in one run; without it the bound takes
+ * |w| <= 128 and long K splits into several runs.  Either way the result is
+ * exact; wsq is read only by the 256-token prefill kernel, and only when it
+ * has no weight zero point.  Like colsum it is a per-weight constant: compute
+ * it once with mq_weight_sq_sums.
+ */
 
 /* Largest K for int8 weights with a weight zero point: 255 * 255 * K < 2^31. */
 #define MQ_MAX_K_ASYM8 32768
@@ -326,7 +341,7 @@ typedef struct mq_linear_desc {
  * (filled by the call; descriptors reading the same input, e.g. q/k/v/gate/up
  * of one block, share them).  Then, optionally, room for the 256-token
  * prefill kernel (see mq_workspace_size): for every distinct 8-bit input of
- * the descriptors with abits 8, obits 8 and M >= 256, its f16 copy (2 M K
+ * the descriptors with abits 8, obits 8, M >= 256 and N >= 256, its f16 copy (2 M K
  * bytes) and row sums of squares (4 M bytes), each rounded up to 1024, placed
  * after the decode region's size, plus 1024 bytes of alignment slack; a call
  * given only the required part runs those descriptors on the 128-token
@@ -437,6 +452,17 @@ int mq_fold_quantize_pack(const float *w, int N, int K, const float *s_in, const
 int mq_fold_norm(const float *gamma, const float *beta, const float *s, int K, float *gamma_out,
                  float *beta_out);
 
+/*
+ * wsq[n] = sum_k w[n][k]^2 (int32) of packed weights (mq_pack_weights layout,
+ * `bits` 8 or 4; `ldw` bytes between rows, 0 for packed rows): the optional
+ * `wsq` field of mq_linear_desc.  Requirements: N, K >= 0; K % 16 == 0 (int8)
+ * or K % 32 == 0 (int4); K <= MQ_MAX_K; packed 16-byte aligned; ldw 0 or at
+ * least K * bits / 8 and a multiple of 16.  Asynchronous on `stream`.
+ * Errors: MQ_ERR_INVALID_ARG, MQ_ERR_ALIGNMENT, MQ_ERR_CUDA.
+ */
+int mq_weight_sq_sums(const void *packed, int N, int K, int bits, int ldw, int32_t *wsq,
+                      void *stream);
+
 /* ---- Attention matmul glue ------------------------------------------------ */
 
 /*
@@ -530,7 +556,7 @@ int mq_test_decode_kernel(int which);
 /*
  * Test hook, not for production: the choice between the two prefill kernels
  * for problems with 8-bit activations and outputs (M > 16).  0 (the initial
- * state) takes the 256-token kernel for M >= 256 when the workspace has room
+ * state) takes the 256-token kernel for M >= 256 and N >= 256 when the workspace has room
  * for the widened inputs (mq_workspace_size, mq_workspace_size_batch count
  * it), the 128-token kernel otherwise.  1 takes the 256-token kernel for every
  * such problem the workspace allows, 2 never.  Both are bit-exact; the hook

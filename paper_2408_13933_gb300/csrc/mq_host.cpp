@@ -74,6 +74,7 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     out.shift = d.shift;
     out.residual = d.residual;
     out.zw = d.zw;
+    out.wsq = d.wsq;
     out.y = static_cast<int8_t *>(d.y);
     out.M = ab == 8 ? d.M : 2 * d.M;  // 16 bits: rows of the plane matrix
     out.N = d.N;
@@ -104,9 +105,13 @@ bool is_decode(const mq_linear_desc &d) {
     return rows > 0 && rows <= mq::DECODE_MAX_M;
 }
 
-// Smallest M that takes the 256-token prefill kernel by default (below it
-// the 128-token kernel's tiles fill the GPU better).
+// Smallest M and N that take the 256-token prefill kernel by default: below
+// 256 tokens the 128-token kernel's tiles fill the GPU better, and below 256
+// output channels its 256-channel tiles would be mostly empty while the
+// widening of x (2 M K bytes written per call) weighs more against the
+// 2 M N K operations (the attention's P V products, N = 64).
 constexpr int WIDE_MIN_M = 256;
+constexpr int WIDE_MIN_N = 256;
 
 // A problem served by the 256-token prefill kernel (mq_prefill2.cu) when the
 // workspace has room for its widened input: a tensor-core shape with 8-bit
@@ -116,7 +121,7 @@ bool wide_eligible(const mq_linear_desc &d) {
     if (abits_of(d) != 8 || obits_of(d) != 8) return false;
     const int which = mq::test_prefill_kernel();
     if (which == 2) return false;
-    return which == 1 || d.M >= WIDE_MIN_M;
+    return which == 1 || (d.M >= WIDE_MIN_M && d.N >= WIDE_MIN_N);
 }
 
 // Workspace layout of one batch: the decode region first (if any decode
@@ -616,6 +621,19 @@ int mq_row_sums(const int8_t *x, int M, int K, int ldx, int32_t *out, void *stre
     j.K = K;
     j.ldx = ldx;
     return mq::launch_rowsum(&j, 1, stream);
+}
+
+int mq_weight_sq_sums(const void *packed, int N, int K, int bits, int ldw, int32_t *wsq,
+                      void *stream) {
+    if (N < 0 || K < 0 || K > MQ_MAX_K || (bits != 8 && bits != 4)) return MQ_ERR_INVALID_ARG;
+    const int row = K * bits / 8;
+    if (ldw < 0 || (ldw > 0 && ldw < row)) return MQ_ERR_INVALID_ARG;
+    if (N == 0) return MQ_OK;
+    if (!wsq || (K > 0 && !packed)) return MQ_ERR_INVALID_ARG;
+    if (K % (bits == 8 ? 16 : 32) != 0 || ldw % 16 != 0 || (K > 0 && !aligned16(packed)))
+        return MQ_ERR_ALIGNMENT;
+    return mq::launch_weight_sq(static_cast<const uint8_t *>(packed), N, K, bits,
+                                ldw > 0 ? ldw : row, wsq, stream);
 }
 
 int mq_head_row_sums(const int8_t *x, int M, int heads, int d, int ldx, int32_t *out,

@@ -21,6 +21,7 @@ struct Problem {
     const int32_t *shift;
     const int8_t *residual;
     const int32_t *zw;      // per-channel weight zero point, or null
+    const int32_t *wsq;     // per-channel sum of squared weight codes, or null
     int8_t *y;
     int32_t M, N, K, ldx, ldy;
     int32_t zx, zy;
@@ -118,6 +119,9 @@ int launch_widen16(const Widen16Job *jobs, int count, void *stream);
 // x16[i] / rowsq[i] are problem i's widened input and row sums of squares.
 int launch_prefill2(const Problem *probs, const uint16_t *const *x16, const int32_t *const *rowsq,
                     int count, void *stream);
+// wsq[n] = sum_k w[n][k]^2 of packed int8 / int4 weights (ldw bytes a row).
+int launch_weight_sq(const uint8_t *packed, int N, int K, int bits, int ldw, int32_t *wsq,
+                     void *stream);
 // Whether the 256-token kernel can run on the current device (set-up done
 // once per device; false when its register split does not fit the compiled
 // kernel's launch allocation).

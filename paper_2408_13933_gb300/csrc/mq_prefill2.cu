@@ -197,7 +197,9 @@ __device__ __forceinline__ bool pair_tile_at(const Params &P, int pair, int i, T
 // epilogue warps compute the same value).  The data-independent chunk bounds
 // |x (w - zw)| by 128 wmax per product; the data-dependent one uses the
 // tile's largest token-row sum of squares X2: a run of L k's is exact when
-// X2 wmax^2 L <= 2^48 (every partial sum is then at most 2^24 in magnitude).
+// X2 wmax^2 L <= 2^48 (every partial sum is then at most 2^24 in magnitude),
+// or, given the weights' sums of squares (symmetric weights), the whole K
+// when X2 max_n wsq[n] <= 2^48.
 __device__ __forceinline__ int chunk_stages(const Params &P, const Tile &t, int lane) {
     const Problem &p = P.p[t.pi];
     const bool zw = p.zw != nullptr;
@@ -208,6 +210,16 @@ __device__ __forceinline__ int chunk_stages(const Params &P, const Tile &t, int 
     for (int i = lane; i < TN; i += 32)
         if (m0 + i < p.M) mx = max(mx, (uint32_t)__ldg(rq + m0 + i));
     mx = __reduce_max_sync(0xffffffffu, mx);
+    if (p.wsq && !zw) {
+        // both operands' norms: every partial sum over any part of K is at most
+        // sqrt(X2 W2), so X2 W2 <= 2^48 sums the whole K in one run
+        const int n0 = t.ct * TM;
+        uint32_t wm = 0;
+        for (int i = lane; i < TM; i += 32)
+            if (n0 + i < p.N) wm = max(wm, (uint32_t)__ldg(p.wsq + n0 + i));
+        wm = __reduce_max_sync(0xffffffffu, wm);
+        if ((uint64_t)mx * (uint64_t)wm <= (1ull << 48)) return t.nkb < 1 ? 1 : t.nkb;
+    }
     const uint64_t wmax = p.bits == 8 ? (zw ? 255u : 128u) : (zw ? 15u : 8u);
     const uint64_t per_stage = (uint64_t)mx * wmax * wmax * (uint64_t)KS;  // < 2^54
     uint64_t data = per_stage ? (1ull << 48) / per_stage : (uint64_t)t.nkb;
@@ -242,8 +254,18 @@ __device__ __forceinline__ void reg_inc() {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
 }
 
+// Four int32 values saturated to int8 and packed, value i in byte i.
+__device__ __forceinline__ uint32_t pack4_sat_s8(int32_t v0, int32_t v1, int32_t v2, int32_t v3) {
+    uint32_t hi, d;
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(hi) : "r"(v3), "r"(v2), "r"(0u));
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(v1), "r"(v0), "r"(hi));
+    return d;
+}
+
 // Requantize 32 sums of one channel (32 consecutive tokens) and pack them,
-// four tokens a word, into w[0..7].  FAST: the shift is at least 33.
+// four tokens a word, into w[0..7].  FAST: the shift is at least 33, so the
+// round-half-up shift is a multiply-high, an add and a shift; the saturation
+// to int8 happens in the pack.
 template <bool FAST>
 __device__ __forceinline__ void requant_pack32(const uint32_t (&f)[32], int32_t corr, int32_t m0,
                                                int32_t sh, int32_t zy, uint32_t *w) {
@@ -251,15 +273,13 @@ __device__ __forceinline__ void requant_pack32(const uint32_t (&f)[32], int32_t 
     const int32_t rs = FAST ? sh - 32 : 0;
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
-        uint32_t v = 0;
+        int32_t o[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int32_t a = (int32_t)(f[4 * q + i] - (uint32_t)corr);
-            const int32_t out = FAST ? min(127, max(-128, ((__mulhi(a, m0) + rnd) >> rs) + zy))
-                                     : mq_requant(a, m0, sh, zy);
-            v |= ((uint32_t)out & 0xFFu) << (8 * i);
+            o[i] = FAST ? ((__mulhi(a, m0) + rnd) >> rs) + zy : mq_requant(a, m0, sh, zy);
         }
-        w[q] = v;
+        w[q] = pack4_sat_s8(o[0], o[1], o[2], o[3]);
     }
 }
 
@@ -749,6 +769,36 @@ __global__ void __launch_bounds__(256) widen16_kernel(const __grid_constant__ Wi
     }
 }
 
+// One warp per weight row: wsq[n] = sum_k w[n][k]^2 of the codes (int4: both
+// nibbles of a byte, sign-extended per byte).
+__global__ void __launch_bounds__(256) wsq_kernel(const uint8_t *w, int N, int K, int bits, int ldw,
+                                                  int32_t *wsq) {
+    const int n = (int)blockIdx.x * 8 + (int)(threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (n >= N) return;
+    const uint8_t *row = w + (size_t)n * (size_t)ldw;
+    const int bytes = K * bits / 8;
+    int sq = 0;
+    for (int b = 16 * lane; b < bytes; b += 512) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(row + b);
+        const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (bits == 8) {
+                sq = __dp4a((int)u[i], (int)u[i], sq);
+            } else {
+                // nibble -> signed byte: ((x ^ 8) - 8) per byte
+                const int lo = (int)__vsub4((u[i] & 0x0F0F0F0Fu) ^ 0x08080808u, 0x08080808u);
+                const int hi = (int)__vsub4(((u[i] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u, 0x08080808u);
+                sq = __dp4a(lo, lo, sq);
+                sq = __dp4a(hi, hi, sq);
+            }
+        }
+    }
+    sq = __reduce_add_sync(0xffffffffu, sq);
+    if (lane == 0) wsq[n] = sq;
+}
+
 // Pairs the device can run at once (one CTA per SM, clusters of two).
 int max_pairs(int dev) {
     static int cached[64] = {0};
@@ -822,6 +872,14 @@ bool encode_x16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows
 }
 
 }  // namespace prefill2
+
+int launch_weight_sq(const uint8_t *packed, int N, int K, int bits, int ldw, int32_t *wsq,
+                     void *stream) {
+    if (N <= 0) return MQ_OK;
+    prefill2::wsq_kernel<<<(unsigned)((N + 7) / 8), 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        packed, N, K, bits, ldw, wsq);
+    return cudaGetLastError() == cudaSuccess ? MQ_OK : MQ_ERR_CUDA;
+}
 
 int launch_widen16(const Widen16Job *jobs, int count, void *stream) {
     using namespace prefill2;

@@ -42,7 +42,8 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_linear_w8a16", "mq_linear_w4a16", "mq_workspace_size_a16", "mq_quantize",
             "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm",
             "mq_row_sums", "mq_head_row_sums", "mq_transpose_i8", "mq_set_wait_limit_ns",
-            "mq_test_skip_partials", "mq_test_decode_kernel", "mq_test_prefill_kernel"]
+            "mq_test_skip_partials", "mq_test_decode_kernel", "mq_test_prefill_kernel",
+            "mq_weight_sq_sums"]
 MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
@@ -55,7 +56,7 @@ class LinearDesc(ctypes.Structure):
                 ("residual", _vp), ("zw", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
                 ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32),
                 ("abits", _i32), ("obits", _i32), ("ldw", _i32),
-                ("wdynamic", _i32)]
+                ("wdynamic", _i32), ("wsq", _vp)]
 
 
 lib.mq_status_string.argtypes = [_int]
@@ -89,6 +90,8 @@ lib.mq_transpose_i8.argtypes = [_vp, _int, _int, _int, _vp, _int, _vp]
 lib.mq_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
 lib.mq_test_skip_partials.argtypes = [_int]
 lib.mq_test_decode_kernel.argtypes = [_int]
+lib.mq_test_prefill_kernel.argtypes = [_int]
+lib.mq_weight_sq_sums.argtypes = [_vp, _int, _int, _int, _int, _vp, _vp]
 for _f in EXPORTED:
     if _f != "mq_status_string":
         getattr(lib, _f).restype = _int
@@ -270,6 +273,16 @@ def fold_norm(gamma: np.ndarray, beta, s: np.ndarray):
     return g, b
 
 
+def weight_sq_sums(packed, n: int, k: int, bits: int, ldw: int = 0, out=None, stream=None):
+    """mq_weight_sq_sums on packed CUDA weights: int32 [N], sum_k w[n][k]^2."""
+    import torch
+    if out is None:
+        out = torch.empty(n, dtype=torch.int32, device=packed.device)
+    _check(lib.mq_weight_sq_sums(_ptr(packed), n, k, bits, ldw, _ptr(out), _stream(stream)),
+           "mq_weight_sq_sums")
+    return out
+
+
 def row_sums(x, out=None, m=None, k=None, ldx=None, stream=None):
     """mq_row_sums on an int8 CUDA tensor [M, K] (or a strided view): int32 [M]."""
     import torch
@@ -323,12 +336,13 @@ def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, 
 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
               ldx=None, ldy=None, m=None, k=None, zw=None, abits=None, obits=None,
-              ldw: int = 0, wdynamic: bool = False) -> LinearDesc:
+              ldw: int = 0, wdynamic: bool = False, wsq=None) -> LinearDesc:
     """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights;
     abits 16 (default: 16 for an int16 x) gives int16 activations and outputs;
     obits 16 with int8 x (default: 16 for an int16 y) an int16 output; `ldw`
     the bytes between weight rows (0: packed); `wdynamic` marks weights written
-    by earlier work on the stream (read only after it completes)."""
+    by earlier work on the stream (read only after it completes); `wsq`
+    (device int32 [N], weight_sq_sums) the weights' sums of squares."""
     d = LinearDesc()
     if abits is None:
         abits = 16 if getattr(x, "element_size", lambda: 1)() == 2 else 8
@@ -341,6 +355,7 @@ def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
     d.x, d.packed, d.colsum = _ptr(x), _ptr(packed), _ptr(colsum)
     d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
     d.zw = _ptr(zw)
+    d.wsq = _ptr(wsq)
     d.M = x.shape[0] if m is None else m
     d.K = x.shape[1] if k is None else k
     d.N = n

@@ -107,8 +107,9 @@ def test_packed_and_workspace_sizes(mq):
     # from 256 tokens on: room for the 256-token kernel's widened input after
     # the decode region (f16 copy and row sums, each to 1024 bytes, + 1024)
     assert mq.workspace_size(1024, 2048, 2048, 8) == dec + 2 * 1024 * 2048 + 4096 + 1024
-    assert mq.workspace_size(300, 100, 48, 4) == dec + 29696 + 2048 + 1024
-    assert mq.workspace_size(300, 100, 0, 4) == 0           # K = 0: nothing to widen
+    assert mq.workspace_size(300, 256, 48, 4) == dec + 29696 + 2048 + 1024
+    assert mq.workspace_size(300, 255, 48, 4) == 0          # N < 256: the 128-token kernel
+    assert mq.workspace_size(300, 256, 0, 4) == 0           # K = 0: nothing to widen
     with pytest.raises(mq.MQError):
         mq.packed_size(3, 63, 4)
     with pytest.raises(mq.MQError):

@@ -181,3 +181,32 @@ def test_widened_copy_and_row_sums():
     roff = off + ((2 * n16 + 1023) & ~1023)
     rowsq = ws[roff:roff + 4 * 300].view(torch.int32).cpu().numpy()
     assert np.array_equal(rowsq, (case.x.astype(np.int64) ** 2).sum(axis=1))
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_weight_sq_sums(bits):
+    case = synth.random_case(850 + bits, 1, 2080 if bits == 8 else 2112, 301, bits, "mixed")
+    packed, _ = mq().pack_weights(case.w, bits)
+    got = mq().weight_sq_sums(upload(packed), case.N, case.K, bits).cpu().numpy()
+    assert np.array_equal(got, (case.w.astype(np.int64) ** 2).sum(axis=1))
+
+
+def test_weight_norms_allow_one_chunk():
+    # full-range activations at K = 5632 (the down projection's input): the
+    # |w| <= 128 bound splits K into runs of ~12 stages; with the weights'
+    # sums of squares the whole K is one run.  Both plans are exact.
+    lib = mq()
+    case = synth.make_linear(0, 4, 0, "wsq", 512, 5632, 512, 8)
+    rng = np.random.default_rng(9)
+    case.x = rng.integers(-100, 101, size=(512, 5632)).astype(np.int8)
+    want = oracle_y(case)
+    for with_wsq in (False, True):
+        g = GpuLinear(case)
+        wsq = lib.weight_sq_sums(g.packed, case.N, case.K, 8) if with_wsq else None
+        d = lib.make_desc(g.x, case.zx, g.packed, g.colsum, case.N, g.m0, g.shift, case.zy, g.y,
+                          8, wsq=wsq)
+        torch = torch_cuda()
+        need = lib.workspace_size_batch([d])
+        ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+        assert lib.linear_batch([d], workspace=ws, ws_bytes=need) == 0
+        assert_equal_int8(g.result(), want, f"wsq={with_wsq}")
