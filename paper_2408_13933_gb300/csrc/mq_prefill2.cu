@@ -656,30 +656,33 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 }
                 tc_fence_after();
                 const bool last = c + 1 == nchunks;
+                uint32_t f[TPT];
 #pragma unroll
-                for (int q = 0; q < TPT / 32; ++q) {
-                    uint32_t f[32];
-                    tc_ld_32x32b_x32(t_lane + 32 * q, f);
-                    tc_wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        uint32_t v = (uint32_t)__float2int_rn(__uint_as_float(f[i]));
-                        if (nchunks > 1) {
-                            if (c > 0) v += part[32 * q + i];
-                            if (!last) part[32 * q + i] = v;
-                        }
-                        f[i] = v;
-                    }
-                    if (last) {
-                        if (fast)
-                            requant_pack32<true>(f, corr, m0, sh, p.zy, &w[8 * q]);
-                        else
-                            requant_pack32<false>(f, corr, m0, sh, p.zy, &w[8 * q]);
-                    }
-                }
+                for (int q = 0; q < TPT / 32; ++q)
+                    tc_ld_32x32b_x32(t_lane + 32 * q, *reinterpret_cast<uint32_t(*)[32]>(&f[32 * q]));
+                tc_wait_ld();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_cluster(leader_f_empty);  // F may be overwritten
+#pragma unroll
+                for (int i = 0; i < TPT; ++i) {
+                    uint32_t v = (uint32_t)__float2int_rn(__uint_as_float(f[i]));
+                    if (nchunks > 1) {
+                        if (c > 0) v += part[i];
+                        if (!last) part[i] = v;
+                    }
+                    f[i] = v;
+                }
+                if (last) {
+#pragma unroll
+                    for (int q = 0; q < TPT / 32; ++q) {
+                        const uint32_t(&g)[32] = *reinterpret_cast<const uint32_t(*)[32]>(&f[32 * q]);
+                        if (fast)
+                            requant_pack32<true>(g, corr, m0, sh, p.zy, &w[8 * q]);
+                        else
+                            requant_pack32<false>(g, corr, m0, sh, p.zy, &w[8 * q]);
+                    }
+                }
             }
             if (!ok) break;
             if (nchunks == 0) {  // K = 0: every sum is 0
