@@ -65,22 +65,23 @@ WORKLOAD = "tinyllama-1.1b-shaped-22-layer-w8a8-stack-m2048-plus-head"
 BLOCK_WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
 
 
-# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one prefill_kernel launch on this
-# workload, read from one ncu capture of the kernel (its summary is committed under profiles/),
-# valid only for the kernel sources it was taken on: reported as null once they change.
-PREFILL_TRAFFIC_BYTES = 56_418_816 + 2_899_456
-PREFILL_TRAFFIC_SOURCES = ("mq_prefill.cu", "mq_ptx.cuh", "mq_internal.h")
-PREFILL_TRAFFIC_SHA = "05c0b6e06d34e88f"
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the 256-token prefill kernel,
+# from one-pass ncu captures (`--profile block` / `--profile stack`, summaries under profiles/):
+# per launch on the config-1 block, and summed over the 45 launches of one headline-stack step.
+# ncu flushes the caches before every captured launch, so the f16 token copies that the pre-pass
+# has just written are read back from DRAM there (in the pipelined run they come from L2).
+# Valid only for the kernel sources they were taken on: reported as null once those change.
+PREFILL_TRAFFIC_BYTES = 66_789_547 + 1_169_152
+PREFILL_TRAFFIC_SOURCES = ("mq_prefill2.cu", "mq_ptx.cuh", "mq_internal.h")
+PREFILL_TRAFFIC_SHA = "6f7381a3b710138c"
 
 
 def prefill_traffic():
     return PREFILL_TRAFFIC_BYTES if sources_sha() == PREFILL_TRAFFIC_SHA else None
 
 
-# DRAM traffic of one step of the headline stack (the sum over its 45 prefill_kernel launches), from
-# a one-pass ncu capture; None until one has been taken on the current kernel sources.
-STACK_TRAFFIC_BYTES = None
-STACK_TRAFFIC_SHA = None
+STACK_TRAFFIC_BYTES = 2_025_980_672 + 61_377_792
+STACK_TRAFFIC_SHA = PREFILL_TRAFFIC_SHA
 
 
 def sources_sha() -> str:
@@ -1291,12 +1292,35 @@ def run_reference(args, dist: Dist):
 
 
 # --------------------------------------------------------------------------- main
+def run_profile_leg(mq, torch, dist, args):
+    """One leg's timed loop alone, for a profiler (`--profile LEG`): the
+    headline stack, the config-1 block, the config-2 decode block at M = 1,
+    or config 4's prefill step.  Prints the leg's time per step."""
+    t0 = time.time()
+    if args.profile == "stack":
+        r = run_stack(mq, torch, dist, args.steps, args.warmup)
+        per = r["total_ms"] / args.steps
+    elif args.profile == "block":
+        r = run_prefill(mq, torch, dist, args.steps, args.warmup)
+        per = r["total_ms"] / args.steps
+    elif args.profile == "decode":
+        r = run_decode(mq, torch, steps_per_m=args.steps, ms=(1,))
+        per = r["m1"]["stream_us"] * 1e-3
+    else:
+        r, _ = run_gemma_prefill(mq, torch, steps=args.steps, check_rows=1)
+        per = r["us_per_step"] * 1e-3
+    print(f"profile leg {args.profile}: {per:.4f} ms per step ({time.time() - t0:.1f} s)",
+          flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawTextHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mq", "reference"], default="mq")
+    ap.add_argument("--profile", choices=["stack", "block", "decode", "gemma"], default=None,
+                    help="run only this leg's timed loop (for a profiler; no JSON line)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
@@ -1312,6 +1336,9 @@ def main():
     build.build()
     from paper_2408_13933_gb300 import mq
 
+    if args.profile:
+        run_profile_leg(mq, torch, dist, args)
+        return
     stack = run_stack(mq, torch, dist, args.steps, args.warmup)
     checks = []
     cfg0, more = run_single_linear(mq, torch)
@@ -1378,11 +1405,15 @@ def main():
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "tensor", "achieved": round(kern_tflops, 1), "peak": tc,
                      "unit": "TFLOP/s", "frac": round(kern_tflops / tc, 3),
-                     "traffic": stack_traffic(), "traffic_unit": "bytes per step (45 launches)",
-                     "kernel": "mq::prefill::prefill_kernel (every launch of the step)",
+                     "traffic": stack_traffic(),
+                     "traffic_unit": "DRAM bytes per step (45 prefill2_kernel launches; ncu "
+                                     "flushes caches per launch, so the widened tokens count)",
+                     "kernel": "mq::prefill2::prefill2_kernel (45 launches a step), each after "
+                               "its token pre-pass widen16_kernel",
                      "peak_note": f"dense f16 tensor peak = bf16 burst ({peaks['source']}), "
                                   "int8 ops run as exact f16 MMAs; achieved = the step's int8 "
-                                  "ops / its device time (CUDA events around the timed steps)"},
+                                  "ops / its device time (CUDA events around the timed steps, "
+                                  "the pre-pass launches included)"},
         "clocks": stack["clocks"],
         "e2e": {"value": round(e2e_value, 2), "unit": "TOPS", "h2d_bytes_per_step": stack["h2d"],
                 "d2h_bytes_per_step": stack["d2h"]},
