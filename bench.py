@@ -333,7 +333,9 @@ def run_prefill(mq, torch, dist: Dist, steps: int, warmup: int):
         raise RuntimeError(f"device status {mq.status_string(status)} after the block run")
     step(0)   # layer 0 last, for the parity sample
     torch.cuda.synchronize()
-    return {"blocks": blocks, "total_ms": e0.elapsed_time(e1)}
+    # with room for widened inputs the call is the token pre-pass + the 256-token kernel
+    kernels = 2 if blocks[0].ws_bytes > 0 else 1
+    return {"blocks": blocks, "total_ms": e0.elapsed_time(e1), "kernels": kernels}
 
 
 def run_decode(mq, torch, steps_per_m: int = 240, asym: bool = False, ms=DECODE_MS,
@@ -822,8 +824,12 @@ class Stack:
         self.d2h_bytes = m * hn
         # one workspace for every call (its widened inputs are scratch; the
         # calls run one after another on one stream)
-        self.ws_bytes = max(mq.workspace_size_batch(list(a)) for a, _ in calls_a + calls_b)
+        sizes = [mq.workspace_size_batch(list(a)) for a, _ in calls_a]
+        self.ws_bytes = max(sizes + [mq.workspace_size_batch(list(a)) for a, _ in calls_b])
         self.ws = torch.zeros(max(16, self.ws_bytes), dtype=torch.uint8, device=dev)
+        # kernel launches a step: a prefill-only call with workspace beyond the
+        # decode region takes the 256-token kernel after its token pre-pass
+        self.kernels = sum(2 if b > 0 else 1 for b in sizes)
 
     def enqueue(self, mq, sp: int, j: int = 0):
         wsp = self.ws.data_ptr() if self.ws_bytes else None
@@ -903,7 +909,7 @@ def run_stack(mq, torch, dist: Dist, steps: int, warmup: int):
         raise RuntimeError("device status error in the end-to-end run")
     return {"stack": st, "total_ms": max_total_ms, "clocks": clocks.result(), "e2e_ms": e2e_ms,
             "e2e_steps": e2e_steps, "h2d": st.h2d_bytes, "d2h": st.d2h_bytes,
-            "launches_per_step": st.launches}
+            "launches_per_step": st.launches, "kernels_per_step": st.kernels}
 
 
 def stack_parity(st, rows):
@@ -1399,7 +1405,8 @@ def main():
                    "head": "{} {}->{}".format(*synth.TINYLLAMA_HEAD),
                    "chain": "q/k/v/gate/up read x_l; o reads q, down reads up; "
                             "x_l+1 = sat8(down + r_l)",
-                   "int8_ops_per_step": ops, "launches_per_step": stack["launches_per_step"],
+                   "int8_ops_per_step": ops, "calls_per_step": stack["launches_per_step"],
+                   "kernel_launches_per_step": stack["kernels_per_step"],
                    "l2": "each step streams 1.03 GB of int8 weights (more than the 129 MB L2); "
                          "activations pass between layers through L2 as in a model",
                    "parallelism": f"replicas x{world}"},
@@ -1417,12 +1424,12 @@ def main():
         "clocks": stack["clocks"],
         "e2e": {"value": round(e2e_value, 2), "unit": "TOPS", "h2d_bytes_per_step": stack["h2d"],
                 "d2h_bytes_per_step": stack["d2h"]},
-        "gpu_launches": args.steps * stack["launches_per_step"],
+        "gpu_launches": args.steps * stack["kernels_per_step"],
         "config0_single_linear_m128": cfg0,
         "config1_tinyllama_block_m1024": {
             "workload": BLOCK_WORKLOAD, "us_per_block": round(blk_us, 2),
             "tops": round(blk_tops, 1), "frac_tensor": round(blk_tops / tc, 3),
-            "launches_per_step": 1, "steps": 2000,
+            "launches_per_step": pre["kernels"], "steps": 2000,
             "l2": f"{PREFILL_LAYERS} layers rotated ({PREFILL_LAYERS * 72} MB > 129 MB L2)",
             "traffic": prefill_traffic(), "traffic_unit": "bytes per launch"},
         "decode_w4a8": {"unit": "GB/s of int4 weights", "weight_bytes_per_block":
