@@ -543,10 +543,10 @@ int mq_test_skip_partials(int cta);
 
 /*
  * Test hook, not for production: the choice between the two decode kernels
- * (M <= 16).  0 (the initial state) chooses by shape: launches of one or two
- * tokens with 8-bit activations whose row tiles balance over the SMs take the
- * row-tile kernel (one CTA per SM, each streaming whole 8-row tiles), the
- * others the split-K kernel.  1 takes the row-tile kernel for every launch it
+ * (M <= 16).  0 (the initial state) chooses by shape: launches of one to four
+ * tokens with 8-bit activations whose row groups balance over the SMs take the
+ * row-group kernel (each warp streaming a run of 4-row groups), the others the
+ * split-K kernel.  1 takes the row-group kernel for every launch it
  * can serve (any such shape, however small), 2 never.  Both are bit-exact; the
  * hook lets the tests run either one on any shape.
  * Errors: MQ_ERR_INVALID_ARG for values other than 0, 1, 2.

@@ -1,7 +1,7 @@
 // mq_gemv.cu -- weight-streaming kernel for the integer-only quantized linear
-// layer at one or two tokens (autoregressive generation), bit-exact.
+// layer at one to four tokens (autoregressive generation), bit-exact.
 //
-// At M <= 2 the layer reads every weight once and does one or two MACs with
+// At M <= 4 the layer reads every weight once and does one to four MACs with
 // it: the time is the weight stream (the paper notes that autoregressive
 // generation is memory-bound, Sec. 5.6 and Appendix A.2).  This kernel is
 // built to stream HBM at its rate, with no shared memory and no barriers:
@@ -57,12 +57,17 @@ namespace gemv {
 constexpr int WARPS = 8;                 // per CTA
 constexpr int THREADS = WARPS * 32;
 constexpr int R = 4;                     // rows per group
-constexpr int STEP = 1024;               // weight bytes of a row per step
-constexpr int MAX_MT = 2;                // tokens
+constexpr int MAX_MT = 4;                // tokens
+// Weight bytes of a row per step: 1 KB (two 16-byte loads per lane) for one
+// or two tokens; 512 bytes for up to four, whose activations of a step would
+// not fit the registers otherwise.
+template <int MT>
+__host__ __device__ constexpr int step_of() { return MT <= 2 ? 1024 : 512; }
 constexpr int MAX_PROBLEMS = DECODE_MAX_PROBLEMS;
-// CTAs per SM: three for one token (80 registers a thread); two for two
-// tokens, whose activation vectors would not fit 80 registers without spills
-// (measured, two tokens: 9.9 us against 10.5 us per TinyLlama-shaped block).
+// CTAs per SM: three for one token (80 registers a thread); two for two or
+// four tokens, whose activation vectors would not fit 80 registers without
+// spills (measured, two tokens: 9.9 us against 10.5 us per TinyLlama-shaped
+// block).
 template <int MT>
 constexpr int ctas_per_sm() { return MT == 1 ? 3 : 2; }
 
@@ -142,8 +147,9 @@ __device__ __forceinline__ void dot16_i4(uint4 w, const XEO &x, int &lo, int &hi
 template <int BITS, int MT>
 struct Step {
     static constexpr int KPB = 8 / BITS;
-    uint4 w[R][2];
-    uint4 x[MT][2][KPB];
+    static constexpr int H = step_of<MT>() / 512;  // 16-byte loads of a row per lane
+    uint4 w[R][H];
+    uint4 x[MT][H][KPB];
 };
 
 // The loads of one step: c0 is the step's first byte in a row (warp-uniform);
@@ -152,18 +158,19 @@ struct Step {
 template <int BITS, int MT>
 __device__ __forceinline__ void load_weights(Step<BITS, MT> &st, const Problem &p, int n0,
                                              int rows, int c0, int lane) {
+    constexpr int H = Step<BITS, MT>::H;
     const int L = p.K * BITS / 8;
     const size_t ldw = (size_t)p.ldw;
     const uint8_t *b = p.w + (size_t)n0 * ldw + c0 + 16 * lane;
-    if (rows == R && c0 + STEP <= L) {
+    if (rows == R && c0 + step_of<MT>() <= L) {
 #pragma unroll
         for (int r = 0; r < R; ++r)
 #pragma unroll
-            for (int h = 0; h < 2; ++h) st.w[r][h] = ldg_w(b + r * ldw + 512 * h);
+            for (int h = 0; h < H; ++h) st.w[r][h] = ldg_w(b + r * ldw + 512 * h);
         return;
     }
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
+    for (int h = 0; h < H; ++h) {
         const bool in = c0 + 512 * h + 16 * lane < L;
 #pragma unroll
         for (int r = 0; r < R; ++r)
@@ -175,20 +182,21 @@ __device__ __forceinline__ void load_weights(Step<BITS, MT> &st, const Problem &
 template <int BITS, int MT>
 __device__ __forceinline__ void load_x(Step<BITS, MT> &st, const Problem &p, int c0, int lane) {
     constexpr int KPB = 8 / BITS;
+    constexpr int H = Step<BITS, MT>::H;
     const int L = p.K * BITS / 8;
     const int8_t *b = p.x + ((size_t)c0 + 16 * lane) * KPB;
     const size_t ldx = (size_t)p.ldx;
-    if (p.M == MT && c0 + STEP <= L) {
+    if (p.M == MT && c0 + step_of<MT>() <= L) {
 #pragma unroll
         for (int m = 0; m < MT; ++m)
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
+            for (int h = 0; h < H; ++h)
 #pragma unroll
                 for (int i = 0; i < KPB; ++i) st.x[m][h][i] = ldg_x(b + m * ldx + 512 * KPB * h + 16 * i);
         return;
     }
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
+    for (int h = 0; h < H; ++h) {
         const bool in = c0 + 512 * h + 16 * lane < L;
 #pragma unroll
         for (int m = 0; m < MT; ++m)
@@ -224,6 +232,8 @@ __device__ __forceinline__ int reduce_scatter(int (&v)[NV], int lane) {
 template <int BITS, int MT, bool O16>
 __global__ void __launch_bounds__(THREADS, ctas_per_sm<MT>()) gemv_kernel(const __grid_constant__ Params P) {
     constexpr int NV = R * MT;  // sums per lane
+    constexpr int STEP = step_of<MT>();
+    constexpr int H = Step<BITS, MT>::H;
     const int lane = threadIdx.x & 31;
     const long long W = (long long)gridDim.x * WARPS;
     const long long gw = (long long)blockIdx.x * WARPS + (threadIdx.x >> 5);
@@ -300,7 +310,7 @@ __global__ void __launch_bounds__(THREADS, ctas_per_sm<MT>()) gemv_kernel(const 
 #pragma unroll
                 for (int m = 0; m < MT; ++m)
 #pragma unroll
-                    for (int h = 0; h < 2; ++h)
+                    for (int h = 0; h < H; ++h)
 #pragma unroll
                         for (int i = 0; i < 8 / BITS; ++i) xs[m] = sum4(st.x[m][h][i], xs[m]);
             }
@@ -308,7 +318,7 @@ __global__ void __launch_bounds__(THREADS, ctas_per_sm<MT>()) gemv_kernel(const 
 #pragma unroll
                 for (int m = 0; m < MT; ++m)
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {
+                    for (int h = 0; h < H; ++h) {
                         const XEO x = x_even_odd(st.x[m][h][0], st.x[m][h][1]);
 #pragma unroll
                         for (int r = 0; r < R; ++r)
@@ -320,7 +330,7 @@ __global__ void __launch_bounds__(THREADS, ctas_per_sm<MT>()) gemv_kernel(const 
 #pragma unroll
                     for (int m = 0; m < MT; ++m)
 #pragma unroll
-                        for (int h = 0; h < 2; ++h)
+                        for (int h = 0; h < H; ++h)
                             acc[r * MT + m] = dp4a4(st.w[r][h], st.x[m][h][0], acc[r * MT + m]);
             }
         }
@@ -347,7 +357,10 @@ __global__ void __launch_bounds__(THREADS, ctas_per_sm<MT>()) gemv_kernel(const 
         const int sum = reduce_scatter<NV>(acc, lane);
         if (owner) {
             const int n = n0 + er;
-            const int32_t xsm = MT == 1 ? xsum[0] : (em ? xsum[MT - 1] : xsum[0]);
+            int32_t xsm = xsum[0];  // sum(x) of this output's token
+#pragma unroll
+            for (int m = 1; m < MT; ++m)
+                if (em == m) xsm = xsum[m];
             // sum(w x) = sum(u x) - 8 sum(x) (int4); then the zero points:
             // sum((x - zx)(w - zw)) = sum(w x) - zw sum(x) - zx (colsum - K zw)
             // (two's-complement wrap is exact: the true value fits int32)
@@ -386,7 +399,7 @@ int launch_t(const Problem *probs, int count, cudaStream_t stream) {
             if (q.wdynamic) P.pre_w = 0;
             q.tiles_m = (q.N + R - 1) / R;
             // a group's weight: its 1 KB steps and one more for its epilogue
-            P.cost_group[i] = (q.K * q.bits / 8 + STEP - 1) / STEP + 1;
+            P.cost_group[i] = (q.K * q.bits / 8 + step_of<MT>() - 1) / step_of<MT>() + 1;
             P.cost_begin[i] = cost;
             cost += (long long)q.tiles_m * P.cost_group[i];
             groups += q.tiles_m;
@@ -441,14 +454,19 @@ int launch_gemv(const Problem *probs, int count, void *stream) {
     cudaStream_t s = static_cast<cudaStream_t>(stream);
 #define MQ_GEMV_CASE(B, T, O) \
     if ((B == 4) == i4 && mt == T && o16 == O) return launch_t<B, T, O>(probs, count, s);
+    if (mt == 3) mt = 4;  // the four-token variant (tokens past M read as zero)
     MQ_GEMV_CASE(4, 1, false)
     MQ_GEMV_CASE(4, 2, false)
+    MQ_GEMV_CASE(4, 4, false)
     MQ_GEMV_CASE(8, 1, false)
     MQ_GEMV_CASE(8, 2, false)
+    MQ_GEMV_CASE(8, 4, false)
     MQ_GEMV_CASE(4, 1, true)
     MQ_GEMV_CASE(4, 2, true)
+    MQ_GEMV_CASE(4, 4, true)
     MQ_GEMV_CASE(8, 1, true)
     MQ_GEMV_CASE(8, 2, true)
+    MQ_GEMV_CASE(8, 4, true)
 #undef MQ_GEMV_CASE
     return MQ_ERR_INVALID_ARG;
 }

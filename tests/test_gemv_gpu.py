@@ -117,7 +117,7 @@ SHAPES4 = [(1, 32), (5, 64), (9, 2048), (100, 5632), (67, 1024), (24, 16384), (1
 SHAPES8 = [(1, 16), (7, 48), (9, 1024), (100, 5632), (33, 2048), (11, 65536)]
 
 
-@pytest.mark.parametrize("m", [1, 2])
+@pytest.mark.parametrize("m", [1, 2, 3, 4])
 @pytest.mark.parametrize("bits,shape", [(4, s) for s in SHAPES4] + [(8, s) for s in SHAPES8],
                          ids=lambda v: "x".join(map(str, v)) if isinstance(v, tuple) else str(v))
 def test_row_tile_kernel_matches_oracle(row_tile_kernel, bits, shape, m):
@@ -127,13 +127,13 @@ def test_row_tile_kernel_matches_oracle(row_tile_kernel, bits, shape, m):
 
 @pytest.mark.parametrize("bits", [4, 8])
 @pytest.mark.parametrize("extreme", ["min", "max", "mixed"])
-@pytest.mark.parametrize("m", [1, 2])
+@pytest.mark.parametrize("m", [1, 2, 4])
 def test_row_tile_kernel_extremes(row_tile_kernel, bits, extreme, m):
     check([Case(200 + m, m, 4096, 40, bits, extreme=extreme)], f"{extreme} bits={bits} m={m}")
 
 
 @pytest.mark.parametrize("bits,k", [(4, 5632), (8, 2048), (8, 32768), (4, 65536)])
-@pytest.mark.parametrize("m", [1, 2])
+@pytest.mark.parametrize("m", [1, 2, 4])
 def test_row_tile_kernel_weight_zero_points(row_tile_kernel, bits, k, m):
     check([Case(300 + k % 991 + m, m, k, 37, bits, zw=True),
            Case(310 + m, m, k, 16, bits, extreme="mixed", zw=True)], f"zw bits={bits} k={k}")
@@ -145,6 +145,8 @@ def test_row_tile_kernel_int16_output_and_residual(row_tile_kernel, bits):
            Case(401, 2, 64, 300, bits, o16=True)], f"o16 bits={bits}")
     check([Case(402, 2, 5632, 50, bits, residual=True),
            Case(403, 1, 2048, 21, bits, zw=True, residual=True)], f"residual bits={bits}")
+    check([Case(404, 4, 2048, 45, bits, zw=True, o16=True),
+           Case(405, 3, 5632, 50, bits, residual=True)], f"four tokens bits={bits}")
 
 
 def test_row_tile_kernel_pitch_and_device_written_weights(row_tile_kernel):
@@ -162,6 +164,12 @@ def test_row_tile_kernel_mixed_batch(row_tile_kernel):
     b.dev[0] = a.dev[0][:1]
     cases = [a, b, Case(602, 1, 5632, 44, 4, zw=True), Case(603, 2, 64, 8, 4)]
     check(cases, "mixed batch")
+    # up to four tokens: one launch of the four-token variant
+    c = Case(604, 4, 2048, 70, 4)
+    d = Case(605, 3, 2048, 9, 4)
+    d.c.x = c.c.x[:3]
+    d.dev[0] = c.dev[0][:3]
+    check([c, d, Case(606, 1, 5632, 44, 4, zw=True), Case(607, 2, 64, 8, 4)], "mixed batch, 4")
 
 
 def test_both_decode_kernels_agree_on_the_block():
@@ -169,7 +177,7 @@ def test_both_decode_kernels_agree_on_the_block():
     # each decode kernel
     lib = mq()
     try:
-        for m in (1, 2):
+        for m in (1, 2, 4):
             cases = [Case(700 + j, m, k, n, 4) for j, (_, k, n) in
                      enumerate(synth.TINYLLAMA_LINEARS)]
             outs = {}
