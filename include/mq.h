@@ -315,6 +315,12 @@ typedef struct mq_linear_desc {
     int32_t wdynamic; /* nonzero: packed is written by earlier work on the stream, see above */
     const int32_t *wsq; /* may be NULL: device int32 [N], wsq[n] = sum_k w[n][k]^2 of the weight
                            codes (mq_weight_sq_sums), see below */
+    void *y16;          /* may be NULL: device f16 [M][N], also written: y as f16, see below */
+    int32_t *ysq;       /* with y16: device int32 [M], zero-filled by the caller; the call adds
+                           sum_n y[m][n]^2 */
+    const void *x16;    /* may be NULL: device f16 [M][K], an f16 copy of x (a y16 of an earlier
+                           call), see below */
+    const int32_t *xsq; /* with x16: device int32 [M], sum_k x[m][k]^2 (that call's ysq) */
 } mq_linear_desc;
 
 /*
@@ -327,6 +333,22 @@ typedef struct mq_linear_desc {
  * exact; wsq is read only by the 256-token prefill kernel, and only when it
  * has no weight zero point.  Like colsum it is a per-weight constant: compute
  * it once with mq_weight_sq_sums.
+ */
+
+/*
+ * Chained layers (`y16` / `ysq`, `x16` / `xsq`, optional, 8-bit activations and
+ * output): the 256-token prefill kernel contracts an f16 copy of x and needs
+ * each token row's sum of squares; by default every call computes both in a
+ * pre-pass into its workspace.  A call given `y16` and `ysq` also writes its
+ * output y (after the residual) as f16 [M][N] (pitch N) into y16 and adds each
+ * row's sum of squares into ysq (zero-filled by the caller): where the
+ * 256-token kernel computes y, its epilogue does this on the way out, otherwise
+ * the call runs the pre-pass on y after computing it.  A later call whose x is
+ * that y passes them as `x16` / `xsq` and skips its pre-pass for that input.
+ * The copy must be of x exactly (the kernel contracts x16, not x).
+ * Requirements: y16 with ysq, x16 with xsq, both only with abits 8 and obits
+ * 8; y16 and x16 16-byte aligned; with y16, N % 16 == 0, ldy % 16 == 0 and y
+ * 16-byte aligned.
  */
 
 /* Largest K for int8 weights with a weight zero point: 255 * 255 * K < 2^31. */

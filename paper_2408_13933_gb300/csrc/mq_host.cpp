@@ -53,6 +53,13 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     if (d.ldw < 0 || (d.ldw > 0 && d.ldw < wrow)) return MQ_ERR_INVALID_ARG;
     if (d.ldw % 16 != 0) return MQ_ERR_ALIGNMENT;
     if (d.K > MQ_MAX_K) return MQ_ERR_K_OVERFLOW;
+    // f16 copies of chained layers: only 8-bit activations and outputs
+    if ((d.y16 != nullptr) != (d.ysq != nullptr) || (d.x16 != nullptr) != (d.xsq != nullptr))
+        return MQ_ERR_INVALID_ARG;
+    if ((d.y16 || d.x16) && (ab != 8 || ob != 8)) return MQ_ERR_INVALID_ARG;
+    if (d.x16 && !aligned16(d.x16)) return MQ_ERR_ALIGNMENT;
+    if (d.y16 && (d.N % 16 != 0 || d.ldy % 16 != 0 || !aligned16(d.y16) || !aligned16(d.y)))
+        return MQ_ERR_ALIGNMENT;
     // int32 accumulators of 8-bit activations with int8 weights and a zero point
     // (16-bit activations accumulate in int64; their int8 planes stay below
     // 128 * 255 * 65536 < 2^31)
@@ -156,6 +163,19 @@ size_t wide_at(const Plan &pl) {
     return pl.required > mq::DECODE_WS_BYTES ? pl.required : mq::DECODE_WS_BYTES;
 }
 
+// The pre-pass job that writes a problem's output y as f16 into y16 and its
+// row sums of squares into ysq.
+mq::Widen16Job output_copy_job(const mq_linear_desc &d) {
+    mq::Widen16Job j{};
+    j.x = static_cast<const int8_t *>(d.y);
+    j.out = static_cast<uint16_t *>(d.y16);
+    j.rowsq = d.ysq;
+    j.M = d.M;
+    j.K = d.N;
+    j.ldx = d.ldy;
+    return j;
+}
+
 Plan batch_plan(const mq_linear_desc *descs, int count) {
     Plan pl;
     size_t off = 0;
@@ -184,7 +204,7 @@ Plan batch_plan(const mq_linear_desc *descs, int count) {
     size_t woff = 0;
     for (int i = 0; i < count; ++i) {
         const mq_linear_desc &d = descs[i];
-        if (!wide_eligible(d)) continue;
+        if (!wide_eligible(d) || d.x16) continue;  // a given f16 copy needs no pre-pass
         const int8_t *x = static_cast<const int8_t *>(d.x);
         bool seen = false;
         for (const auto &j : pl.wide)
@@ -220,9 +240,19 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
     uint8_t *region = static_cast<uint8_t *>(workspace) + (pl.any_decode ? mq::DECODE_WS_BYTES : 0);
     for (size_t i = 0; i < pl.split.size(); ++i)
         pl.split[i].out = reinterpret_cast<int8_t *>(region + pl.split_off[i]);
-    // the 256-token kernel when the workspace has room for the widened inputs
-    const bool wide = !pl.wide.empty() && workspace && ws_bytes >= pl.bytes && mq::prefill2_ready();
-    if (wide) {
+    // the 256-token kernel for problems whose f16 copy is given, and for the
+    // others when the workspace has room for the widened inputs
+    const bool room = !pl.wide.empty() && workspace && ws_bytes >= pl.bytes;
+    bool ready = false, ready_known = false;
+    auto takes_wide = [&](const mq_linear_desc &d) {
+        if (!wide_eligible(d) || !(d.x16 || room)) return false;
+        if (!ready_known) {
+            ready = mq::prefill2_ready();
+            ready_known = true;
+        }
+        return ready;
+    };
+    if (room) {
         const uintptr_t base =
             (reinterpret_cast<uintptr_t>(workspace) + wide_at(pl) + 1023) & ~(uintptr_t)1023;
         for (size_t i = 0; i < pl.wide.size(); ++i) {
@@ -235,6 +265,9 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
     std::vector<mq::Problem> pre2;
     std::vector<const uint16_t *> pre2_x16;
     std::vector<const int32_t *> pre2_rowsq;
+    std::vector<uint16_t *> pre2_y16;
+    std::vector<int32_t *> pre2_ysq;
+    std::vector<mq::Widen16Job> after;  // f16 copies of outputs the epilogues do not write
     // kernel families: prefill by activation / output width, decode by weight
     // bits and activation / output width (0: 8 / 8, 1: 16 / 16, 2: 8 / 16)
     std::vector<mq::Problem> pre[3], dec[2][3];
@@ -253,25 +286,36 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         const int mode = p.a16 ? 1 : (p.o16 ? 2 : 0);
         if (is_decode(d)) {
             dec[p.bits == 8][mode].push_back(p);
-        } else if (wide && wide_eligible(d)) {
-            const mq::Widen16Job *job = nullptr;
-            for (const auto &j : pl.wide)
-                if (j.x == p.x && j.M == d.M && j.K == d.K && j.ldx == d.ldx) job = &j;
+        } else if (takes_wide(d)) {
             pre2.push_back(p);
-            pre2_x16.push_back(job->out);
-            pre2_rowsq.push_back(job->rowsq);
+            if (d.x16) {
+                pre2_x16.push_back(static_cast<const uint16_t *>(d.x16));
+                pre2_rowsq.push_back(d.xsq);
+            } else {
+                const mq::Widen16Job *job = nullptr;
+                for (const auto &j : pl.wide)
+                    if (j.x == p.x && j.M == d.M && j.K == d.K && j.ldx == d.ldx) job = &j;
+                pre2_x16.push_back(job->out);
+                pre2_rowsq.push_back(job->rowsq);
+            }
+            // the epilogue writes the f16 copy of y where its 4-byte stores apply
+            const bool fused = d.y16 && (reinterpret_cast<uintptr_t>(d.residual) & 3) == 0;
+            pre2_y16.push_back(fused ? static_cast<uint16_t *>(d.y16) : nullptr);
+            pre2_ysq.push_back(fused ? d.ysq : nullptr);
+            if (d.y16 && !fused) after.push_back(output_copy_job(d));
         } else {
             pre[mode].push_back(p);
+            if (d.y16) after.push_back(output_copy_job(d));
         }
     }
     int rc = MQ_OK;
     if (!pl.split.empty())
         rc = mq::launch_split16(pl.split.data(), (int)pl.split.size(), stream);
     if (rc == MQ_OK && !pre2.empty()) {
-        rc = mq::launch_widen16(pl.wide.data(), (int)pl.wide.size(), stream);
+        if (room) rc = mq::launch_widen16(pl.wide.data(), (int)pl.wide.size(), stream);
         if (rc == MQ_OK)
             rc = mq::launch_prefill2(pre2.data(), pre2_x16.data(), pre2_rowsq.data(),
-                                     (int)pre2.size(), stream);
+                                     pre2_y16.data(), pre2_ysq.data(), (int)pre2.size(), stream);
     }
     for (int mode = 0; mode < 3; ++mode)
         if (rc == MQ_OK && !pre[mode].empty())
@@ -280,6 +324,10 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         for (int a = 0; a < 3; ++a)
             if (rc == MQ_OK && !dec[b][a].empty())
                 rc = mq::launch_decode(dec[b][a].data(), (int)dec[b][a].size(), workspace, stream);
+    // f16 copies of outputs no epilogue wrote: the pre-pass on y, after everything
+    // that writes y (its row sums overwrite the caller's zeros)
+    if (rc == MQ_OK && !after.empty())
+        rc = mq::launch_widen16(after.data(), (int)after.size(), stream);
     return rc;
 }
 

@@ -117,8 +117,11 @@ constexpr int WIDEN16_MAX_JOBS = 64;
 int launch_widen16(const Widen16Job *jobs, int count, void *stream);
 // The 256-token prefill kernel: problems with 8-bit activations and output;
 // x16[i] / rowsq[i] are problem i's widened input and row sums of squares.
+// y16[i] / ysq[i] (may be null): problem i's output also written as f16 and
+// its row sums of squares added (the epilogue; y, the residual and ldy 4-byte
+// aligned).
 int launch_prefill2(const Problem *probs, const uint16_t *const *x16, const int32_t *const *rowsq,
-                    int count, void *stream);
+                    uint16_t *const *y16, int32_t *const *ysq, int count, void *stream);
 // wsq[n] = sum_k w[n][k]^2 of packed int8 / int4 weights (ldw bytes a row).
 int launch_weight_sq(const uint8_t *packed, int N, int K, int bits, int ldw, int32_t *wsq,
                      void *stream);

@@ -120,6 +120,8 @@ struct Params {
     CUtensorMap tmap_x[PREFILL_MAX_PROBLEMS];  // f16 [M][K] box 64 x 128 (128-byte swizzle)
     Problem p[PREFILL_MAX_PROBLEMS];           // tile_begin: first tile; tiles_m: token tiles
     const int32_t *rowsq[PREFILL_MAX_PROBLEMS];  // sum of squares of every token row
+    uint16_t *y16[PREFILL_MAX_PROBLEMS];         // or null: y also written as f16 [M][N]
+    int32_t *ysq[PREFILL_MAX_PROBLEMS];          // with y16: row sums of squares of y, added
     int count;
     int total_tiles;
     int npairs;
@@ -290,35 +292,58 @@ __device__ __forceinline__ void requant_pack32(const uint32_t (&f)[32], int32_t 
 // one 32-bit word.  The whole warp calls it (the shuffles); `nch` (0..4) is
 // the number of the group's channels below N; y0 / r0 point at token tok0 and
 // the group's first channel, and both, like ldy, are 4-byte aligned.
+// With y16 (chained layers): the same words also go out as f16 (8 bytes: four
+// channels of one token; y16 and ysq point at token tok0 and the group's
+// first channel / at token tok0, row pitch ldy16 elements), and each token's
+// sum of squares over the warp's 32 channels is added into ysq (dp4a over
+// the group's four channels, shuffles over the eight groups).
+template <bool CHAIN>
 __device__ __forceinline__ void store_words_v4(const uint32_t (&w)[TPT / 4], int8_t *y0,
                                                const int8_t *r0, size_t ldy, int ntok, int lane,
-                                               int nch) {
+                                               int nch, uint16_t *y16, int32_t *ysq,
+                                               size_t ldy16) {
     const int r = lane & 3;
     const uint32_t sel1 = (r & 1) ? 0x3715u : 0x6240u;
     const uint32_t sel2 = (r & 2) ? 0x3276u : 0x5410u;
+    // the bytes of this lane's group that are channels below N
+    const uint32_t valid = nch >= 4 ? 0xFFFFFFFFu : (nch <= 0 ? 0u : (1u << (8 * nch)) - 1u);
 #pragma unroll
     for (int q = 0; q < TPT / 4; ++q) {
         if (4 * q >= ntok) break;
         uint32_t v = prmt(w[q], __shfl_xor_sync(0xffffffffu, w[q], 1), sel1);
         v = prmt(v, __shfl_xor_sync(0xffffffffu, v, 2), sel2);
         const int tok = 4 * q + r;
-        if (tok < ntok && nch > 0) {
-            int8_t *yp = y0 + (size_t)tok * ldy;
-            if (r0) {
-                const int8_t *rp = r0 + (size_t)tok * ldy;
-                uint32_t res = 0;
-                if (nch == 4) {
-                    res = *reinterpret_cast<const uint32_t *>(rp);
-                } else {
-                    for (int c = 0; c < nch; ++c) res |= (uint32_t)(uint8_t)rp[c] << (8 * c);
-                }
-                v = __vaddss4(v, res);
+        const bool live = tok < ntok && nch > 0;
+        if (live && r0) {
+            const int8_t *rp = r0 + (size_t)tok * ldy;
+            uint32_t res = 0;
+            if (nch == 4) {
+                res = *reinterpret_cast<const uint32_t *>(rp);
+            } else {
+                for (int c = 0; c < nch; ++c) res |= (uint32_t)(uint8_t)rp[c] << (8 * c);
             }
+            v = __vaddss4(v, res);
+        }
+        if (live) {
+            int8_t *yp = y0 + (size_t)tok * ldy;
             if (nch == 4) {
                 *reinterpret_cast<uint32_t *>(yp) = v;
             } else {
                 for (int c = 0; c < nch; ++c) yp[c] = (int8_t)(v >> (8 * c));
             }
+        }
+        if (CHAIN && y16) {
+            const uint32_t vm = live ? v & valid : 0u;
+            if (live && nch == 4) {  // N % 16 == 0: a group is whole or past N
+                uint32_t h0, h1;
+                i8x4_to_f16x4(vm, h0, h1);
+                *reinterpret_cast<uint2 *>(y16 + (size_t)tok * ldy16) = make_uint2(h0, h1);
+            }
+            int sq = __dp4a((int)vm, (int)vm, 0);
+            sq += __shfl_xor_sync(0xffffffffu, sq, 4);
+            sq += __shfl_xor_sync(0xffffffffu, sq, 8);
+            sq += __shfl_xor_sync(0xffffffffu, sq, 16);
+            if (lane < 4 && tok < ntok) atomicAdd(ysq + tok, sq);
         }
     }
 }
@@ -343,7 +368,10 @@ __device__ __forceinline__ void store_words_b(const uint32_t (&w)[TPT / 4], int8
 
 // ZW: problems may have a weight zero point, folded into the widening of the
 // weights (w - zw); without it the widening offsets are immediate constants.
-template <bool ZW>
+// CHAIN: some problem's output also goes out as f16 with its row sums of
+// squares (a separate instantiation: the extra epilogue code slowed launches
+// that do not use it by ~5%).
+template <bool ZW, bool CHAIN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     prefill2_kernel(const __grid_constant__ Params P) {
     extern __shared__ uint8_t smem_raw[];
@@ -708,7 +736,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                 const int nch = max(0, min(4, p.N - chg));
                 int8_t *y0 = p.y + (size_t)tok0 * ldy + chg;
                 const int8_t *r0 = p.residual ? p.residual + (size_t)tok0 * ldy + chg : nullptr;
-                store_words_v4(w, y0, r0, ldy, ntok, lane, nch);
+                uint16_t *y16 = CHAIN ? P.y16[t.pi] : nullptr;
+                int32_t *ysq = y16 ? P.ysq[t.pi] + tok0 : nullptr;
+                if (y16) y16 += (size_t)tok0 * (size_t)p.N + chg;
+                store_words_v4<CHAIN>(w, y0, r0, ldy, ntok, lane, nch, y16, ysq, (size_t)p.N);
             } else if (ch_in) {
                 int8_t *yp = p.y + (size_t)tok0 * ldy + ch;
                 const int8_t *rp = p.residual ? p.residual + (size_t)tok0 * ldy + ch : nullptr;
@@ -814,7 +845,7 @@ int max_pairs(int dev) {
     cfg.blockDim = dim3(THREADS, 1, 1);
     cfg.dynamicSmemBytes = SMEM_BYTES;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, prefill2_kernel<false>, &cfg) == cudaSuccess &&
+    if (cudaOccupancyMaxActiveClusters(&clusters, prefill2_kernel<false, false>, &cfg) == cudaSuccess &&
         clusters > 0 && clusters < n)
         n = clusters;
     if (n > MAX_PAIRS) n = MAX_PAIRS;
@@ -923,13 +954,16 @@ bool prefill2_ready() {
     if (!(attr_done.load(std::memory_order_acquire) & (1ull << dev))) {
         const int smem = (int)SMEM_BYTES;
         const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
-        bool ok = cudaFuncSetAttribute(prefill2_kernel<false>, attr, smem) == cudaSuccess &&
-                  cudaFuncSetAttribute(prefill2_kernel<true>, attr, smem) == cudaSuccess;
+        bool ok = cudaFuncSetAttribute(prefill2_kernel<false, false>, attr, smem) == cudaSuccess &&
+                  cudaFuncSetAttribute(prefill2_kernel<true, false>, attr, smem) == cudaSuccess &&
+                  cudaFuncSetAttribute(prefill2_kernel<false, true>, attr, smem) == cudaSuccess &&
+                  cudaFuncSetAttribute(prefill2_kernel<true, true>, attr, smem) == cudaSuccess;
         // the register split of the warpgroups must fit what the launch gives
         // the CTA (see REG_SPLIT): a build that compiled to fewer registers per
         // thread is never launched (the 128-token kernel serves instead)
         for (const void *k :
-             {(const void *)prefill2_kernel<false>, (const void *)prefill2_kernel<true>}) {
+             {(const void *)prefill2_kernel<false, false>, (const void *)prefill2_kernel<true, false>,
+              (const void *)prefill2_kernel<false, true>, (const void *)prefill2_kernel<true, true>}) {
             cudaFuncAttributes fa{};
             ok = ok && cudaFuncGetAttributes(&fa, k) == cudaSuccess &&
                  fa.numRegs * THREADS >= REG_SPLIT;
@@ -945,7 +979,7 @@ bool prefill2_ready() {
 }
 
 int launch_prefill2(const Problem *probs, const uint16_t *const *x16, const int32_t *const *rowsq,
-                    int count, void *stream) {
+                    uint16_t *const *y16, int32_t *const *ysq, int count, void *stream) {
     using namespace prefill2;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MQ_ERR_CUDA;
@@ -955,9 +989,13 @@ int launch_prefill2(const Problem *probs, const uint16_t *const *x16, const int3
     if (pairs_max < 1) return MQ_ERR_CUDA;
     for (int begin = 0; begin < count; begin += PREFILL_MAX_PROBLEMS) {
         const int n = count - begin < PREFILL_MAX_PROBLEMS ? count - begin : PREFILL_MAX_PROBLEMS;
-        bool any_zw = false;
-        for (int i = begin; i < begin + n; ++i) any_zw = any_zw || probs[i].zw != nullptr;
-        auto kern = any_zw ? prefill2_kernel<true> : prefill2_kernel<false>;
+        bool any_zw = false, any_chain = false;
+        for (int i = begin; i < begin + n; ++i) {
+            any_zw = any_zw || probs[i].zw != nullptr;
+            any_chain = any_chain || (y16 && y16[i]);
+        }
+        auto kern = any_zw ? (any_chain ? prefill2_kernel<true, true> : prefill2_kernel<true, false>)
+                           : (any_chain ? prefill2_kernel<false, true> : prefill2_kernel<false, false>);
         Params P{};
         P.pre_w = 1;
         long long tiles = 0;
@@ -973,6 +1011,8 @@ int launch_prefill2(const Problem *probs, const uint16_t *const *x16, const int3
             Problem &q = P.p[i];
             q = probs[order[i]];
             P.rowsq[i] = rowsq[order[i]];
+            P.y16[i] = y16 ? y16[order[i]] : nullptr;
+            P.ysq[i] = y16 ? ysq[order[i]] : nullptr;
             if (q.wdynamic) P.pre_w = 0;
             q.tiles_m = (q.M + TN - 1) / TN;
             q.tile_begin = (int)tiles;

@@ -56,7 +56,8 @@ class LinearDesc(ctypes.Structure):
                 ("residual", _vp), ("zw", _vp), ("y", _vp), ("M", _i32), ("N", _i32), ("K", _i32),
                 ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32),
                 ("abits", _i32), ("obits", _i32), ("ldw", _i32),
-                ("wdynamic", _i32), ("wsq", _vp)]
+                ("wdynamic", _i32), ("wsq", _vp), ("y16", _vp), ("ysq", _vp), ("x16", _vp),
+                ("xsq", _vp)]
 
 
 lib.mq_status_string.argtypes = [_int]
@@ -336,13 +337,17 @@ def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, 
 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
               ldx=None, ldy=None, m=None, k=None, zw=None, abits=None, obits=None,
-              ldw: int = 0, wdynamic: bool = False, wsq=None) -> LinearDesc:
+              ldw: int = 0, wdynamic: bool = False, wsq=None, y16=None, ysq=None, x16=None,
+              xsq=None) -> LinearDesc:
     """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights;
     abits 16 (default: 16 for an int16 x) gives int16 activations and outputs;
     obits 16 with int8 x (default: 16 for an int16 y) an int16 output; `ldw`
     the bytes between weight rows (0: packed); `wdynamic` marks weights written
     by earlier work on the stream (read only after it completes); `wsq`
-    (device int32 [N], weight_sq_sums) the weights' sums of squares."""
+    (device int32 [N], weight_sq_sums) the weights' sums of squares; `y16` /
+    `ysq` (device f16 [M, N] / zero-filled int32 [M]) receive y as f16 and its
+    row sums of squares, `x16` / `xsq` pass those of an earlier call as this
+    call's x (chained layers, see mq.h)."""
     d = LinearDesc()
     if abits is None:
         abits = 16 if getattr(x, "element_size", lambda: 1)() == 2 else 8
@@ -356,6 +361,7 @@ def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
     d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
     d.zw = _ptr(zw)
     d.wsq = _ptr(wsq)
+    d.y16, d.ysq, d.x16, d.xsq = _ptr(y16), _ptr(ysq), _ptr(x16), _ptr(xsq)
     d.M = x.shape[0] if m is None else m
     d.K = x.shape[1] if k is None else k
     d.N = n

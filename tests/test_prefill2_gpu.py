@@ -210,3 +210,77 @@ def test_weight_norms_allow_one_chunk():
         ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
         assert lib.linear_batch([d], workspace=ws, ws_bytes=need) == 0
         assert_equal_int8(g.result(), want, f"wsq={with_wsq}")
+
+
+def _chain_pair(seed, m, k, n1, n2, residual):
+    """Two linears chained as layers are: A reads x, B reads A's output."""
+    a = synth.make_linear(0, 5, seed, "chainA", m, k, n1, 8)
+    if residual:
+        a.residual = np.random.default_rng(seed).integers(-128, 128, size=(m, n1)).astype(np.int8)
+    b = synth.make_linear(0, 6, seed, "chainB", m, n1, n2, 8)
+    return a, b
+
+
+@pytest.mark.parametrize("which", [0, 1, 2])   # default choice, 256-token forced, 128-token forced
+@pytest.mark.parametrize("residual", [False, True])
+def test_chained_f16_copies(which, residual):
+    # A writes y16 / ysq (fused in the 256-token epilogue, or by the pre-pass
+    # on y after the 128-token kernel); B reads them as x16 / xsq.  y16 is f16(y)
+    # and ysq the row sums of squares of y exactly, and B equals the oracle on y.
+    torch = torch_cuda()
+    lib = mq()
+    assert lib.test_prefill_kernel(which) == 0
+    a, b = _chain_pair(30 + which, 512, 2048, 1024, 768, residual)
+    ga = GpuLinear(a)
+    y16 = torch.full((a.M, a.N), 7.0, dtype=torch.float16, device="cuda")
+    ysq = torch.zeros(a.M, dtype=torch.int32, device="cuda")
+    da = lib.make_desc(ga.x, a.zx, ga.packed, ga.colsum, a.N, ga.m0, ga.shift, a.zy, ga.y, 8,
+                       residual=ga.residual, y16=y16, ysq=ysq)
+    need = lib.workspace_size_batch([da])
+    ws = torch.zeros(max(need, 16), dtype=torch.uint8, device="cuda")
+    assert lib.linear_batch([da], workspace=ws, ws_bytes=need) == 0
+    ya = ga.result()
+    assert_equal_int8(ya, oracle_y(a), "A")
+    assert np.array_equal(y16.cpu().numpy(), ya.astype(np.float16))
+    assert np.array_equal(ysq.cpu().numpy(), (ya.astype(np.int64) ** 2).sum(axis=1))
+    b.x = ya
+    gb = GpuLinear(b)
+    db = lib.make_desc(ga.y, b.zx, gb.packed, gb.colsum, b.N, gb.m0, gb.shift, b.zy, gb.y, 8,
+                       x16=y16, xsq=ysq)
+    need = lib.workspace_size_batch([db])
+    assert need == 0   # its only input comes widened: no pre-pass, no workspace
+    assert lib.linear_batch([db], workspace=None, ws_bytes=0) == 0
+    assert_equal_int8(gb.result(), oracle_y(b), "B")
+
+
+def test_chained_copy_of_a_small_output():
+    # an output below the 256-token kernel's limits (N = 128): its f16 copy comes
+    # from the pre-pass on y after the 128-token kernel
+    torch = torch_cuda()
+    lib = mq()
+    assert lib.test_prefill_kernel(0) == 0
+    a = synth.make_linear(0, 7, 0, "small", 300, 1024, 128, 8)
+    ga = GpuLinear(a)
+    y16 = torch.zeros((a.M, a.N), dtype=torch.float16, device="cuda")
+    ysq = torch.zeros(a.M, dtype=torch.int32, device="cuda")
+    da = lib.make_desc(ga.x, a.zx, ga.packed, ga.colsum, a.N, ga.m0, ga.shift, a.zy, ga.y, 8,
+                       y16=y16, ysq=ysq)
+    assert lib.linear_batch([da], workspace=None, ws_bytes=0) == 0
+    ya = ga.result()
+    assert np.array_equal(y16.cpu().numpy(), ya.astype(np.float16))
+    assert np.array_equal(ysq.cpu().numpy(), (ya.astype(np.int64) ** 2).sum(axis=1))
+
+
+def test_chained_fields_validated():
+    lib = mq()
+    torch = torch_cuda()
+    a = synth.make_linear(0, 8, 0, "val", 300, 1024, 264, 8)
+    ga = GpuLinear(a)
+    y16 = torch.zeros((a.M, a.N), dtype=torch.float16, device="cuda")
+    d = lib.make_desc(ga.x, a.zx, ga.packed, ga.colsum, a.N, ga.m0, ga.shift, a.zy, ga.y, 8,
+                      y16=y16)   # no ysq
+    assert lib.linear_batch([d]) == lib.MQ_ERR_INVALID_ARG
+    ysq = torch.zeros(a.M, dtype=torch.int32, device="cuda")
+    d = lib.make_desc(ga.x, a.zx, ga.packed, ga.colsum, a.N, ga.m0, ga.shift, a.zy, ga.y, 8,
+                      y16=y16, ysq=ysq)   # N = 264: not a multiple of 16
+    assert lib.linear_batch([d]) == lib.MQ_ERR_ALIGNMENT
