@@ -67,20 +67,21 @@ BLOCK_WORKLOAD = "tinyllama-1.1b-block-w8a8-prefill-m1024"
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the 256-token prefill kernel,
 # from one-pass ncu captures (`--profile block` / `--profile stack`, summaries under profiles/):
-# per launch on the config-1 block, and summed over the 45 launches of one headline-stack step.
+# per launch on the config-1 block, and summed over the 45 launches of one headline-stack step
+# (whose writes include the f16 copies of the chained outputs that leave L2 during the step).
 # ncu flushes the caches before every captured launch, so the f16 token copies that the pre-pass
 # has just written are read back from DRAM there (in the pipelined run they come from L2).
 # Valid only for the kernel sources they were taken on: reported as null once those change.
-PREFILL_TRAFFIC_BYTES = 66_789_547 + 1_169_152
+PREFILL_TRAFFIC_BYTES = 66_827_947 + 1_221_376
 PREFILL_TRAFFIC_SOURCES = ("mq_prefill2.cu", "mq_ptx.cuh", "mq_internal.h")
-PREFILL_TRAFFIC_SHA = "6f7381a3b710138c"
+PREFILL_TRAFFIC_SHA = "ae25ed65491297e2"
 
 
 def prefill_traffic():
     return PREFILL_TRAFFIC_BYTES if sources_sha() == PREFILL_TRAFFIC_SHA else None
 
 
-STACK_TRAFFIC_BYTES = 2_025_980_672 + 61_377_792
+STACK_TRAFFIC_BYTES = 2_029_162_240 + 332_227_840
 STACK_TRAFFIC_SHA = PREFILL_TRAFFIC_SHA
 
 
@@ -544,9 +545,10 @@ def run_weight_pipeline(mq, torch, reps: int = 5):
     colsum) over the TinyLlama block's seven f32 weight matrices (176 MB), in
     the paper's W8A8 setting (asymmetric per tensor, down per channel) and
     W4A8 (asymmetric per channel): microseconds per block and GB/s of f32
-    weights (each read twice: statistics, then codes).  Each call allocates
-    its outputs on the host side, so the timed steps are enqueued behind a
-    device sleep and the region measures the device, not the call rate."""
+    weights (each read twice: statistics, then codes), as one batched call
+    (three launches) and as seven per-linear calls.  Each call allocates its
+    outputs on the host side, so the timed steps are enqueued behind a device
+    sleep and the region measures the device, not the call rate."""
     g = torch.Generator(device="cuda")
     g.manual_seed(9)
     mats = [(torch.randn((n, k), device="cuda", generator=g) * 0.02,
@@ -559,21 +561,31 @@ def run_weight_pipeline(mq, torch, reps: int = 5):
         codes = [mq.MQ_WEIGHTS_ASYM_TENSOR if s_ == "asym_tensor" else mq.MQ_WEIGHTS_ASYM_CHANNEL
                  for s_ in schemes]
 
-        def block():
+        def per_linear():
             for (w, s_in), sc in zip(mats, codes):
                 mq.fold_quantize_pack(w, bits, sc, s_in)
-        block()
-        torch.cuda.synchronize()
-        torch.cuda._sleep(100_000_000)  # about 50 ms: the host enqueues every step meanwhile
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(reps):
+
+        def batched():
+            mq.fold_quantize_pack_batch([(w, bits, sc, s_in, None)
+                                         for (w, s_in), sc in zip(mats, codes)])
+
+        def timed(block):
             block()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        ms = e0.elapsed_time(e1) / reps
+            torch.cuda.synchronize()
+            torch.cuda._sleep(100_000_000)  # about 50 ms: the host enqueues every step meanwhile
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                block()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1) / reps
+
+        ms = timed(batched)
+        ms_each = timed(per_linear)
         out[f"w{bits}a8_block"] = {"us": round(ms * 1e3, 1),
-                                   "gbs_f32_weights": round(fbytes / (ms * 1e-3) / 1e9, 1)}
+                                   "gbs_f32_weights": round(fbytes / (ms * 1e-3) / 1e9, 1),
+                                   "per_linear_calls_us": round(ms_each * 1e3, 1)}
     del mats
     return out
 
@@ -1322,7 +1334,8 @@ def run_reference(args, dist: Dist):
 def run_profile_leg(mq, torch, dist, args):
     """One leg's timed loop alone, for a profiler (`--profile LEG`): the
     headline stack, the config-1 block, the config-2 decode block at M = 1,
-    or config 4's prefill step.  Prints the leg's time per step."""
+    config 4's prefill step, or config 4's decode step at M = 1 (block, then
+    head).  Prints the leg's time per step."""
     t0 = time.time()
     if args.profile == "stack":
         r = run_stack(mq, torch, dist, args.steps, args.warmup)
@@ -1333,6 +1346,9 @@ def run_profile_leg(mq, torch, dist, args):
     elif args.profile == "decode":
         r = run_decode(mq, torch, steps_per_m=args.steps, ms=(1,))
         per = r["m1"]["stream_us"] * 1e-3
+    elif args.profile == "gemma_decode":
+        r, _ = run_gemma_decode(mq, torch, reps=args.steps, block_layers=1)
+        per = r["step_us"] * 1e-3
     else:
         r, _ = run_gemma_prefill(mq, torch, steps=args.steps, check_rows=1)
         per = r["us_per_step"] * 1e-3
@@ -1346,7 +1362,7 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mq", "reference"], default="mq")
-    ap.add_argument("--profile", choices=["stack", "block", "decode", "gemma"], default=None,
+    ap.add_argument("--profile", choices=["stack", "block", "decode", "gemma", "gemma_decode"], default=None,
                     help="run only this leg's timed loop (for a profiler; no JSON line)")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -1435,7 +1451,8 @@ def main():
                      "unit": "TFLOP/s", "frac": round(kern_tflops / tc, 3),
                      "traffic": stack_traffic(),
                      "traffic_unit": "DRAM bytes per step (45 prefill2_kernel launches; ncu "
-                                     "flushes caches per launch, so the widened tokens count)",
+                                     "flushes caches per launch, so the f16 inputs are read "
+                                     "from DRAM)",
                      "kernel": "mq::prefill2::prefill2_kernel (45 launches a step; the first "
                                "after the pre-pass widen16_kernel that widens x_0, the rest "
                                "read the f16 copies the previous launches wrote)",
@@ -1470,7 +1487,8 @@ def main():
                                   "frac_hbm": round(attention16["gbs"] / hbm, 3)},
         "boundary_quantizers": {"unit": "GB/s of input + output bytes", **glue},
         "weight_pipeline": {"what": "fold of eq. 1 + quantize + pack + colsum, 7 linears, "
-                                    "176 MB of f32 weights", **wpipe},
+                                    "176 MB of f32 weights, one batched call (3 launches); "
+                                    "per_linear_calls_us: seven calls (14-20 launches)", **wpipe},
     }
     if rank == 0 and world == 1:
         line["cpu_baseline"], parity = cpu_baseline(st, checks=checks)

@@ -466,6 +466,32 @@ int mq_fold_quantize_pack(const float *w, int N, int K, const float *s_in, const
                           int32_t *zw, float *stats, void *stream);
 
 /*
+ * mq_fold_quantize_pack over up to MQ_FOLD_MAX_JOBS linears (e.g. the seven of
+ * one transformer block) in three launches instead of two or three per
+ * linear: the row statistics of every linear, the per-tensor reductions, then
+ * every linear's codes.  Each descriptor's fields are the arguments of
+ * mq_fold_quantize_pack, with the same requirements; every descriptor is
+ * checked before anything is launched.  Outputs (and the stats scratch) of
+ * different descriptors must not overlap.  The result is byte-identical to
+ * one mq_fold_quantize_pack call per descriptor.
+ * Errors: MQ_ERR_INVALID_ARG (also count < 0 or > MQ_FOLD_MAX_JOBS, descs NULL
+ * with count > 0), MQ_ERR_ALIGNMENT, MQ_ERR_CUDA.
+ */
+#define MQ_FOLD_MAX_JOBS 32
+typedef struct mq_fold_desc {
+    const float *w;
+    int32_t N, K;
+    const float *s_in, *s_out;
+    int32_t bits, scheme;
+    void *packed;
+    int32_t *colsum;
+    float *sw;
+    int32_t *zw;
+    float *stats;
+} mq_fold_desc;
+int mq_fold_quantize_pack_batch(const mq_fold_desc *descs, int count, void *stream);
+
+/*
  * The norm's affine before the first transformed linear absorbs S0^-1
  * (Figure 3): gamma_out[k] = gamma[k] / s[k], beta_out[k] = beta[k] / s[k],
  * f32.  Host arrays; beta and beta_out may be NULL (RMSNorm has no shift).

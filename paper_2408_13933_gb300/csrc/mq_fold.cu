@@ -11,11 +11,16 @@
 // (the _rn intrinsics keep the compiler from contracting them), so the codes
 // are the same on any correct implementation of the definition.
 //
-// Three kernels: per-row minima / maxima of w', for the per-tensor scheme a
-// one-CTA reduction of those to the tensor's, then quantization + packing +
-// colsum (w' is recomputed from w, which the first pass left in L2 for
-// matrices that fit).  The row kernels give each row one warp, so a CTA of
-// eight warps has eight rows in flight and the reductions are warp shuffles.
+// Three launches over a whole batch of linears (one call for a model block):
+// per-row minima / maxima of w', for the per-tensor scheme a one-CTA-per-
+// tensor reduction of those to the tensor's, then quantization + packing +
+// colsum, w' recomputed from w.  The last pass visits the rows in the reverse
+// order of the first, so it starts on the rows the first pass read last,
+// which are still in L2.  The later launches use programmatic dependent
+// launch: they start while the previous pass drains and wait for it before
+// reading its statistics.  The row kernels give each row one warp, so a CTA
+// of eight warps has eight rows in flight and the reductions are warp
+// shuffles.
 // When K is a multiple of 4 and the rows are 16-byte aligned, a lane loads
 // four weights (and four input scales) at a time, UNROLL such loads before
 // using them, and writes their codes as one 4-byte (int8) or 2-byte (int4)
@@ -117,6 +122,24 @@ struct Args {
                    // 2-byte (int4) aligned
 };
 
+// One launch's linears: job j's rows are CTAs block_begin[j] ..
+// block_begin[j + 1] - 1, ROWS rows each; tensor_jobs lists the per-tensor
+// jobs (pass 2 gives each one CTA).
+struct Batch {
+    Args job[FOLD_MAX_JOBS];
+    int block_begin[FOLD_MAX_JOBS + 1];
+    int tensor_jobs[FOLD_MAX_JOBS];
+    int count, ntensor;
+};
+
+// The job of row block `blk` and the first row of that block within the job.
+__device__ __forceinline__ int job_of(const Batch &B, int blk, int &row0) {
+    int j = 0;
+    while (j + 1 < B.count && blk >= B.block_begin[j + 1]) ++j;
+    row0 = (blk - B.block_begin[j]) * ROWS;
+    return j;
+}
+
 // Calls f(q, v) for every group q of four folded weights of row `row4` that
 // this lane owns (q = lane, lane + 32, ...), with the group's loads issued
 // UNROLL groups at a time.
@@ -145,10 +168,7 @@ __device__ __forceinline__ void for_each_four(const float4 *row4, const float4 *
 }
 
 // Pass 1: lo = min(min_k w'[n][k], 0), hi = max(max_k w'[n][k], 0) per row.
-__global__ void __launch_bounds__(THREADS) row_stats_kernel(const Args a) {
-    const int lane = threadIdx.x & 31;
-    const int n = blockIdx.x * ROWS + (threadIdx.x >> 5);
-    if (n >= a.N) return;
+__device__ __forceinline__ void row_stats(const Args &a, int n, int lane) {
     const float *row = a.w + (size_t)n * (size_t)a.K;
     const bool has_out = a.s_out != nullptr;
     const float so = has_out ? __ldg(a.s_out + n) : 1.0f;
@@ -175,9 +195,21 @@ __global__ void __launch_bounds__(THREADS) row_stats_kernel(const Args a) {
     }
 }
 
+__global__ void __launch_bounds__(THREADS) row_stats_kernel(const __grid_constant__ Batch B) {
+    griddep_launch_dependents();  // pass 2 / 3 wait for this grid before reading
+    int row0;
+    const int j = job_of(B, blockIdx.x, row0);
+    const Args a = B.job[j];
+    const int n = row0 + (threadIdx.x >> 5);
+    if (n < a.N) row_stats(a, n, threadIdx.x & 31);
+}
+
 // Pass 2 (per tensor): the tensor's lo / hi into stats[0], stats[1].
-__global__ void __launch_bounds__(THREADS) tensor_stats_kernel(const Args a) {
+__global__ void __launch_bounds__(THREADS) tensor_stats_kernel(const __grid_constant__ Batch B) {
     __shared__ float red[THREADS / 32];
+    griddep_launch_dependents();
+    const Args a = B.job[B.tensor_jobs[blockIdx.x]];
+    griddep_wait();  // the row statistics of pass 1
     float lo = 0.0f, hi = 0.0f;
     for (int n = threadIdx.x; n < a.N; n += THREADS) {
         lo = fminf(lo, a.stats[2 * n]);
@@ -192,10 +224,7 @@ __global__ void __launch_bounds__(THREADS) tensor_stats_kernel(const Args a) {
 }
 
 // Pass 3: scale and zero point of the row (or tensor), codes, packing, colsum.
-__global__ void __launch_bounds__(THREADS) quantize_pack_kernel(const Args a) {
-    const int lane = threadIdx.x & 31;
-    const int n = blockIdx.x * ROWS + (threadIdx.x >> 5);
-    if (n >= a.N) return;
+__device__ __forceinline__ void quantize_row(const Args &a, int n, int lane) {
     const float *row = a.w + (size_t)n * (size_t)a.K;
     const bool has_out = a.s_out != nullptr;
     const float so = has_out ? __ldg(a.s_out + n) : 1.0f;
@@ -270,27 +299,58 @@ __global__ void __launch_bounds__(THREADS) quantize_pack_kernel(const Args a) {
     }
 }
 
+// Row blocks in the reverse order of pass 1 (the last ones read are in L2).
+__global__ void __launch_bounds__(THREADS) quantize_pack_kernel(const __grid_constant__ Batch B) {
+    int row0;
+    const int j = job_of(B, (int)(gridDim.x - 1 - blockIdx.x), row0);
+    const Args a = B.job[j];
+    const int n = row0 + (threadIdx.x >> 5);
+    griddep_wait();  // the statistics of pass 1 (and 2)
+    if (n < a.N) quantize_row(a, n, threadIdx.x & 31);
+}
+
 }  // namespace fold
 
-// Arguments validated by mq_fold_quantize_pack (mq_host.cpp).
-int launch_fold(const float *w, int N, int K, const float *s_in, const float *s_out, int bits,
-                int scheme, void *packed, int32_t *colsum, float *sw, int32_t *zw, float *stats,
-                void *stream) {
+// Arguments validated by mq_fold_quantize_pack(_batch) (mq_host.cpp).
+int launch_fold(const FoldJob *jobs, int count, void *stream) {
     using namespace fold;
-    if (N == 0) return MQ_OK;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (count < 1 || count > FOLD_MAX_JOBS) return MQ_ERR_INVALID_ARG;
     const auto aligned = [](const void *p, uintptr_t b) {
         return (reinterpret_cast<uintptr_t>(p) & (b - 1)) == 0;
     };
-    const int vec = K % 4 == 0 && aligned(w, 16) && aligned(s_in, 16) &&
-                    aligned(packed, bits == 8 ? 4 : 2);
-    const Args a{w, s_in, s_out, N, K, bits, scheme, static_cast<uint8_t *>(packed),
-                 colsum, sw, zw, stats, vec};
-    const int blocks = N / ROWS + (N % ROWS != 0);
-    row_stats_kernel<<<blocks, THREADS, 0, s>>>(a);
-    if (scheme == 2) tensor_stats_kernel<<<1, THREADS, 0, s>>>(a);
-    quantize_pack_kernel<<<blocks, THREADS, 0, s>>>(a);
-    return cudaGetLastError() == cudaSuccess ? MQ_OK : MQ_ERR_CUDA;
+    Batch B{};
+    B.count = count;
+    int blocks = 0;
+    for (int j = 0; j < count; ++j) {
+        const FoldJob &f = jobs[j];
+        const int vec = f.K % 4 == 0 && aligned(f.w, 16) && aligned(f.s_in, 16) &&
+                        aligned(f.packed, f.bits == 8 ? 4 : 2);
+        B.job[j] = Args{f.w, f.s_in, f.s_out, f.N, f.K, f.bits, f.scheme,
+                        static_cast<uint8_t *>(f.packed), f.colsum, f.sw, f.zw, f.stats, vec};
+        B.block_begin[j] = blocks;
+        blocks += f.N / ROWS + (f.N % ROWS != 0);
+        if (f.scheme == 2 && f.N > 0) B.tensor_jobs[B.ntensor++] = j;
+    }
+    B.block_begin[count] = blocks;
+    if (blocks == 0) return MQ_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    auto launch = [&](void (*k)(Batch), int grid, bool pdl) {
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)grid, 1, 1);
+        cfg.blockDim = dim3(THREADS, 1, 1);
+        cfg.stream = s;
+        cfg.attrs = pdl ? attr : nullptr;
+        cfg.numAttrs = pdl ? 1 : 0;
+        return cudaLaunchKernelEx(&cfg, k, B) == cudaSuccess;
+    };
+    // pass 1 in plain stream order (w may be the previous kernel's output)
+    bool ok = launch(row_stats_kernel, blocks, false);
+    if (ok && B.ntensor) ok = launch(tensor_stats_kernel, B.ntensor, true);
+    if (ok) ok = launch(quantize_pack_kernel, blocks, true);
+    return ok ? MQ_OK : MQ_ERR_CUDA;
 }
 
 }  // namespace mq

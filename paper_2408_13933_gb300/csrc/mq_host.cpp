@@ -627,22 +627,45 @@ int mq_requantize(const void *q, int in_type, int64_t n, int32_t zx, int32_t M0,
     return mq::launch_glue(2, in_type, out_type, q, y, n, 0.0f, zx, zy, M0, shift, lo, hi, stream);
 }
 
+namespace {
+
+int check_fold(const mq_fold_desc &d) {
+    if (d.N < 0 || d.K < 0 || (d.bits != 8 && d.bits != 4) ||
+        d.scheme < MQ_WEIGHTS_SYM_CHANNEL || d.scheme > MQ_WEIGHTS_ASYM_TENSOR)
+        return MQ_ERR_INVALID_ARG;
+    if (d.bits == 4 && (d.K & 1)) return MQ_ERR_INVALID_ARG;
+    if (d.N == 0) return MQ_OK;
+    if (!d.colsum || !d.sw || !d.stats || (d.scheme != MQ_WEIGHTS_SYM_CHANNEL && !d.zw))
+        return MQ_ERR_INVALID_ARG;
+    if (d.K > 0 && (!d.w || !d.packed)) return MQ_ERR_INVALID_ARG;
+    if (!aligned_to(d.w, 4) || !aligned_to(d.s_in, 4) || !aligned_to(d.s_out, 4) ||
+        !aligned_to(d.colsum, 4) || !aligned_to(d.sw, 4) || !aligned_to(d.zw, 4) ||
+        !aligned_to(d.stats, 4))
+        return MQ_ERR_ALIGNMENT;
+    return MQ_OK;
+}
+
+}  // namespace
+
+int mq_fold_quantize_pack_batch(const mq_fold_desc *descs, int count, void *stream) {
+    if (count < 0 || count > MQ_FOLD_MAX_JOBS || (count > 0 && !descs)) return MQ_ERR_INVALID_ARG;
+    mq::FoldJob jobs[MQ_FOLD_MAX_JOBS];
+    int n = 0;
+    for (int i = 0; i < count; ++i) {
+        const mq_fold_desc &d = descs[i];
+        if (const int rc = check_fold(d)) return rc;
+        if (d.N == 0) continue;
+        jobs[n++] = mq::FoldJob{d.w,  d.N,      d.K,      d.s_in,   d.s_out, d.bits,
+                                d.scheme, d.packed, d.colsum, d.sw, d.zw,    d.stats};
+    }
+    return n ? mq::launch_fold(jobs, n, stream) : MQ_OK;
+}
+
 int mq_fold_quantize_pack(const float *w, int N, int K, const float *s_in, const float *s_out,
                           int bits, int scheme, void *packed, int32_t *colsum, float *sw,
                           int32_t *zw, float *stats, void *stream) {
-    if (N < 0 || K < 0 || (bits != 8 && bits != 4) || scheme < MQ_WEIGHTS_SYM_CHANNEL ||
-        scheme > MQ_WEIGHTS_ASYM_TENSOR)
-        return MQ_ERR_INVALID_ARG;
-    if (bits == 4 && (K & 1)) return MQ_ERR_INVALID_ARG;
-    if (N == 0) return MQ_OK;
-    if (!colsum || !sw || !stats || (scheme != MQ_WEIGHTS_SYM_CHANNEL && !zw))
-        return MQ_ERR_INVALID_ARG;
-    if (K > 0 && (!w || !packed)) return MQ_ERR_INVALID_ARG;
-    if (!aligned_to(w, 4) || !aligned_to(s_in, 4) || !aligned_to(s_out, 4) ||
-        !aligned_to(colsum, 4) || !aligned_to(sw, 4) || !aligned_to(zw, 4) || !aligned_to(stats, 4))
-        return MQ_ERR_ALIGNMENT;
-    return mq::launch_fold(w, N, K, s_in, s_out, bits, scheme, packed, colsum, sw, zw, stats,
-                           stream);
+    const mq_fold_desc d{w, N, K, s_in, s_out, bits, scheme, packed, colsum, sw, zw, stats};
+    return mq_fold_quantize_pack_batch(&d, 1, stream);
 }
 
 int mq_fold_norm(const float *gamma, const float *beta, const float *s, int K, float *gamma_out,

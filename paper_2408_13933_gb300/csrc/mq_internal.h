@@ -141,9 +141,20 @@ int launch_glue(int kind, int in_type, int out_type, const void *in, void *out, 
                 int32_t hi, void *stream);
 
 // Offline weight pipeline (mq_fold.cu): fold eq. 1 into f32 weights,
-// quantize by `scheme` (MQ_WEIGHTS_*), pack, colsum.
-int launch_fold(const float *w, int N, int K, const float *s_in, const float *s_out, int bits,
-                int scheme, void *packed, int32_t *colsum, float *sw, int32_t *zw, float *stats,
-                void *stream);
+// quantize by `scheme` (MQ_WEIGHTS_*), pack, colsum; one batch of linears in
+// three launches.
+constexpr int FOLD_MAX_JOBS = MQ_FOLD_MAX_JOBS;
+struct FoldJob {
+    const float *w;
+    int N, K;
+    const float *s_in, *s_out;
+    int bits, scheme;
+    void *packed;
+    int32_t *colsum;
+    float *sw;
+    int32_t *zw;
+    float *stats;
+};
+int launch_fold(const FoldJob *jobs, int count, void *stream);
 
 }  // namespace mq

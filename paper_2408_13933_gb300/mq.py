@@ -35,6 +35,7 @@ MQ_ERR_WORKSPACE = 7
 MQ_MAX_K = 65536
 MQ_MAX_K_ASYM8 = 32768
 MQ_MAX_BATCH = 256
+MQ_FOLD_MAX_JOBS = 32
 
 EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_weights",
             "mq_workspace_size", "mq_linear_w8a8", "mq_linear_w4a8", "mq_linear_batch",
@@ -43,7 +44,7 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm",
             "mq_row_sums", "mq_head_row_sums", "mq_transpose_i8", "mq_set_wait_limit_ns",
             "mq_test_skip_partials", "mq_test_decode_kernel", "mq_test_prefill_kernel",
-            "mq_weight_sq_sums"]
+            "mq_weight_sq_sums", "mq_fold_quantize_pack_batch"]
 MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
@@ -58,6 +59,13 @@ class LinearDesc(ctypes.Structure):
                 ("abits", _i32), ("obits", _i32), ("ldw", _i32),
                 ("wdynamic", _i32), ("wsq", _vp), ("y16", _vp), ("ysq", _vp), ("x16", _vp),
                 ("xsq", _vp)]
+
+
+class FoldDesc(ctypes.Structure):
+    """Mirror of mq_fold_desc."""
+    _fields_ = [("w", _vp), ("N", _i32), ("K", _i32), ("s_in", _vp), ("s_out", _vp),
+                ("bits", _i32), ("scheme", _i32), ("packed", _vp), ("colsum", _vp), ("sw", _vp),
+                ("zw", _vp), ("stats", _vp)]
 
 
 lib.mq_status_string.argtypes = [_int]
@@ -84,6 +92,7 @@ lib.mq_dequantize.argtypes = [_vp, _int, _i64, _f32, _i32, _vp, _vp]
 lib.mq_requantize.argtypes = [_vp, _int, _i64, _i32, _i32, _i32, _i32, _vp, _int, _vp]
 lib.mq_fold_quantize_pack.argtypes = [_vp, _int, _int, _vp, _vp, _int, _int, _vp, _vp, _vp, _vp,
                                       _vp, _vp]
+lib.mq_fold_quantize_pack_batch.argtypes = [ctypes.POINTER(FoldDesc), _int, _vp]
 lib.mq_fold_norm.argtypes = [_vp, _vp, _vp, _int, _vp, _vp]
 lib.mq_row_sums.argtypes = [_vp, _int, _int, _int, _vp, _vp]
 lib.mq_head_row_sums.argtypes = [_vp, _int, _int, _int, _int, _vp, _vp]
@@ -259,6 +268,31 @@ def fold_quantize_pack(w, bits: int, scheme: int, s_in=None, s_out=None, stream=
                                      _ptr(packed), _ptr(colsum), _ptr(sw), _ptr(zw), _ptr(stats),
                                      _stream(stream)), "mq_fold_quantize_pack")
     return (packed.view(n, packed.numel() // n) if n else packed), colsum, sw, zw
+
+
+def fold_quantize_pack_batch(jobs, stream=None):
+    """mq_fold_quantize_pack_batch: `jobs` is a list of (w, bits, scheme, s_in,
+    s_out) with w a CUDA f32 tensor [N, K]; returns one (packed, colsum, sw, zw)
+    per job, as fold_quantize_pack."""
+    import torch
+    outs, descs, keep = [], [], []
+    for w, bits, scheme, s_in, s_out in jobs:
+        n, k = w.shape
+        dev = w.device
+        packed = torch.empty(packed_size(n, k, bits), dtype=torch.uint8, device=dev)
+        colsum = torch.empty(n, dtype=torch.int32, device=dev)
+        sw = torch.empty(n, dtype=torch.float32, device=dev)
+        zw = (torch.empty(n, dtype=torch.int32, device=dev)
+              if scheme != MQ_WEIGHTS_SYM_CHANNEL else None)
+        stats = torch.empty(2 * max(n, 1), dtype=torch.float32, device=dev)
+        keep.append(stats)
+        descs.append(FoldDesc(_ptr(w), n, k, _ptr(s_in), _ptr(s_out), bits, scheme, _ptr(packed),
+                              _ptr(colsum), _ptr(sw), _ptr(zw), _ptr(stats)))
+        outs.append(((packed.view(n, packed.numel() // n) if n else packed), colsum, sw, zw))
+    arr = (FoldDesc * max(len(descs), 1))(*descs)
+    _check(lib.mq_fold_quantize_pack_batch(arr, len(descs), _stream(stream)),
+           "mq_fold_quantize_pack_batch")
+    return outs
 
 
 def fold_norm(gamma: np.ndarray, beta, s: np.ndarray):

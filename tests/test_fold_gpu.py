@@ -192,3 +192,67 @@ def test_folded_weights_drive_the_layer(bits, scheme):
     want = oracle.linear(x, zx, opk, bits, n, om0, osh, zy,
                          zw=ozw if scheme != 0 else None)
     assert_equal_int8(y.cpu().numpy(), want, f"folded layer bits={bits} scheme={scheme}")
+
+
+def test_fold_batch_mixed():
+    # one batched call over linears of every scheme, width and factor
+    # combination, with K not a multiple of 4, rows off the 16-byte boundary,
+    # N not a multiple of the eight rows of a CTA, an empty linear and the
+    # block's largest shape: every linear's bytes equal the oracle's (and so
+    # the per-linear entry point's)
+    torch = torch_cuda()
+    lib = mq()
+    specs = [  # (n, k, bits, scheme, factors)
+        (256, 2048, 8, 2, "both"), (37, 200, 4, 1, "in"), (5632, 2048, 8, 1, "out"),
+        (19, 202, 8, 0, "none"), (0, 64, 8, 2, "none"), (300, 5632, 4, 2, "both"),
+        (64, 1024, 4, 0, "in"), (129, 96, 8, 2, "out")]
+    jobs, wants, keep = [], [], []
+    for i, (n, k, bits, scheme, factors) in enumerate(specs):
+        w, s_in, s_out = _weights(500 + i, n, k)
+        si = s_in if factors in ("in", "both") else None
+        so = s_out if factors in ("out", "both") else None
+        if i == 3:  # off the 16-byte boundary
+            wbuf = torch.zeros(n * k + 1, dtype=torch.float32, device="cuda")
+            wbuf[1:] = torch.from_numpy(w.reshape(-1)).cuda()
+            wd = wbuf[1:].view(n, k)
+            keep.append(wbuf)
+        else:
+            wd = upload(w)
+        jobs.append((wd, bits, scheme, upload(si) if si is not None else None,
+                     upload(so) if so is not None else None))
+        wants.append(_want(w, si, so, bits, scheme) if n else None)
+    outs = lib.fold_quantize_pack_batch(jobs)
+    torch.cuda.synchronize()
+    for (n, k, bits, scheme, _), (packed, colsum, sw, zw), want in zip(specs, outs, wants):
+        if n == 0:
+            assert colsum.numel() == 0
+            continue
+        tag = f"batch job {n}x{k} bits={bits} scheme={scheme}"
+        assert np.array_equal(sw.cpu().numpy().view(np.uint32), want[2].view(np.uint32)), tag
+        assert np.array_equal(packed.cpu().numpy().reshape(want[0].shape), want[0]), tag
+        assert np.array_equal(colsum.cpu().numpy(), want[1]), tag
+        if scheme != 0:
+            assert np.array_equal(zw.cpu().numpy(), want[3]), tag
+
+
+def test_fold_batch_checks_every_descriptor_first():
+    # a bad descriptor anywhere fails the call before anything is launched
+    torch = torch_cuda()
+    lib = mq()
+    w = upload(_weights(7, 16, 64)[0])
+    colsum = torch.full((16,), -5, dtype=torch.int32, device="cuda")
+    sw = torch.zeros(16, dtype=torch.float32, device="cuda")
+    stats = torch.zeros(32, dtype=torch.float32, device="cuda")
+    packed = torch.zeros(16 * 64, dtype=torch.uint8, device="cuda")
+    ok = lib.FoldDesc(w.data_ptr(), 16, 64, None, None, 8, 0, packed.data_ptr(),
+                      colsum.data_ptr(), sw.data_ptr(), None, stats.data_ptr())
+    bad = lib.FoldDesc(w.data_ptr(), 16, 63, None, None, 4, 0, packed.data_ptr(),
+                       colsum.data_ptr(), sw.data_ptr(), None, stats.data_ptr())  # odd K, int4
+    arr = (lib.FoldDesc * 2)(ok, bad)
+    assert lib.lib.mq_fold_quantize_pack_batch(arr, 2, None) == lib.MQ_ERR_INVALID_ARG
+    torch.cuda.synchronize()
+    assert (colsum == -5).all(), "the good descriptor ran"
+    too_many = (lib.FoldDesc * (lib.MQ_FOLD_MAX_JOBS + 1))()
+    assert lib.lib.mq_fold_quantize_pack_batch(too_many, lib.MQ_FOLD_MAX_JOBS + 1, None) == \
+        lib.MQ_ERR_INVALID_ARG
+    assert lib.lib.mq_fold_quantize_pack_batch(None, 0, None) == 0

@@ -377,13 +377,17 @@ def test_o16_ldw_rowsums_transpose_validation(mq):
     assert t(None, 0, 8, 8, None, 8, None) == 0
 
 
-def test_descriptor_layout_matches_the_header(mq, tmp_path):
-    # the binding's ctypes struct against the C compiler's layout of mq_linear_desc
-    fields = [f[0] for f in mq.LinearDesc._fields_]
+@pytest.mark.parametrize("struct", ["LinearDesc", "FoldDesc"])
+def test_descriptor_layout_matches_the_header(mq, tmp_path, struct):
+    # the binding's ctypes structs against the C compiler's layouts of
+    # mq_linear_desc and mq_fold_desc
+    cls = getattr(mq, struct)
+    cname = {"LinearDesc": "mq_linear_desc", "FoldDesc": "mq_fold_desc"}[struct]
+    fields = [f[0] for f in cls._fields_]
     src = tmp_path / "layout.c"
-    body = "".join(f'    printf("{f} %zu\\n", offsetof(mq_linear_desc, {f}));\n' for f in fields)
+    body = "".join(f'    printf("{f} %zu\\n", offsetof({cname}, {f}));\n' for f in fields)
     src.write_text('#include <stddef.h>\n#include <stdio.h>\n#include "mq.h"\nint main(void) {\n'
-                   + body + '    printf("sizeof %zu\\n", sizeof(mq_linear_desc));\n    return 0;\n}\n')
+                   + body + f'    printf("sizeof %zu\\n", sizeof({cname}));\n    return 0;\n}}\n')
     exe = tmp_path / "layout"
     import subprocess
     subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o",
@@ -391,5 +395,5 @@ def test_descriptor_layout_matches_the_header(mq, tmp_path):
     out = dict(line.split() for line in subprocess.run([str(exe)], check=True, capture_output=True,
                                                        text=True).stdout.splitlines())
     for f in fields:
-        assert int(out[f]) == getattr(mq.LinearDesc, f).offset, f
-    assert int(out["sizeof"]) == ctypes.sizeof(mq.LinearDesc)
+        assert int(out[f]) == getattr(cls, f).offset, f
+    assert int(out["sizeof"]) == ctypes.sizeof(cls)
