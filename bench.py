@@ -710,7 +710,7 @@ def run_attention(mq, torch, reps: int = 60, check_rows: int = 4, bits16: bool =
     """Grouped-query attention's two integer matmuls of one TinyLlama layer at
     T = 1024 (the softmax between them is outside the integer layer): per step
     the key row sums of the 4 KV heads (one launch), S = Q K^T for 32 heads
-    (one batched call, one prefill launch, int16 scores), V^T of all heads
+    (one batched call, one token-major kernel launch, int16 scores), V^T of all heads
     (one transpose) and its row sums (one launch), and O = P V for 32 heads
     (one batched call).  Steps rotate over three
     layers' operands (about 300 MB, more than L2).  The host enqueues the timed

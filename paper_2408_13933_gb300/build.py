@@ -24,7 +24,7 @@ INCLUDE = os.path.join(ROOT, "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["mq_host.cpp", "mq_pack.cu", "mq_decode.cu", "mq_gemv.cu", "mq_prefill.cu", "mq_prefill2.cu",
-           "mq_noalloc.cu", "mq_glue.cu", "mq_fold.cu"]
+           "mq_noalloc.cu", "mq_glue.cu", "mq_fold.cu", "mq_tmajor.cu"]
 
 
 def nvcc() -> str:

@@ -10,6 +10,7 @@
 #include <vector>
 
 #include "mq_internal.h"
+#include "mq_tmajor.h"
 
 namespace mq {
 
@@ -19,12 +20,14 @@ std::atomic<uint64_t> g_wait_ns{DEFAULT_WAIT_NS};
 std::atomic<int> g_skip_cta{-1};
 std::atomic<int> g_decode_kernel{0};
 std::atomic<int> g_prefill_kernel{0};
+std::atomic<int> g_tmajor_kernel{0};
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_ns.load(std::memory_order_relaxed); }
 int test_skip_cta() { return g_skip_cta.load(std::memory_order_relaxed); }
 int test_decode_kernel() { return g_decode_kernel.load(std::memory_order_relaxed); }
 int test_prefill_kernel() { return g_prefill_kernel.load(std::memory_order_relaxed); }
+int test_tmajor_kernel() { return g_tmajor_kernel.load(std::memory_order_relaxed); }
 
 }  // namespace mq
 
@@ -262,6 +265,14 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
                 at + align1024(2 * (size_t)pl.wide[i].M * (size_t)pl.wide[i].K));
         }
     }
+    // the token-major kernel for short K (8-bit weights and activations; the
+    // attention scores Q K^T at head dimension K)
+    const int tmajor_mode = mq::test_tmajor_kernel();
+    auto takes_tmajor = [&](const mq::Problem &p) {
+        if (tmajor_mode == 2 || !mq::tmajor_suits(p)) return false;
+        return tmajor_mode == 1 || p.K <= 128;
+    };
+    std::vector<mq::Problem> tmaj[2];  // by o16
     std::vector<mq::Problem> pre2;
     std::vector<const uint16_t *> pre2_x16;
     std::vector<const int32_t *> pre2_rowsq;
@@ -286,6 +297,9 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         const int mode = p.a16 ? 1 : (p.o16 ? 2 : 0);
         if (is_decode(d)) {
             dec[p.bits == 8][mode].push_back(p);
+        } else if (takes_tmajor(p)) {
+            tmaj[p.o16 ? 1 : 0].push_back(p);
+            if (d.y16) after.push_back(output_copy_job(d));
         } else if (takes_wide(d)) {
             pre2.push_back(p);
             if (d.x16) {
@@ -317,6 +331,9 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
             rc = mq::launch_prefill2(pre2.data(), pre2_x16.data(), pre2_rowsq.data(),
                                      pre2_y16.data(), pre2_ysq.data(), (int)pre2.size(), stream);
     }
+    for (int o = 0; o < 2; ++o)
+        if (rc == MQ_OK && !tmaj[o].empty())
+            rc = mq::launch_tmajor(tmaj[o].data(), (int)tmaj[o].size(), stream);
     for (int mode = 0; mode < 3; ++mode)
         if (rc == MQ_OK && !pre[mode].empty())
             rc = mq::launch_prefill(pre[mode].data(), (int)pre[mode].size(), stream);
@@ -762,6 +779,12 @@ int mq_test_decode_kernel(int which) {
 int mq_test_prefill_kernel(int which) {
     if (which < 0 || which > 2) return MQ_ERR_INVALID_ARG;
     mq::g_prefill_kernel.store(which, std::memory_order_relaxed);
+    return MQ_OK;
+}
+
+int mq_test_tmajor_kernel(int which) {
+    if (which < 0 || which > 2) return MQ_ERR_INVALID_ARG;
+    mq::g_tmajor_kernel.store(which, std::memory_order_relaxed);
     return MQ_OK;
 }
 

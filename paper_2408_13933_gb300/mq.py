@@ -44,7 +44,7 @@ EXPORTED = ["mq_status_string", "mq_requant_params", "mq_packed_size", "mq_pack_
             "mq_dequantize", "mq_requantize", "mq_fold_quantize_pack", "mq_fold_norm",
             "mq_row_sums", "mq_head_row_sums", "mq_transpose_i8", "mq_set_wait_limit_ns",
             "mq_test_skip_partials", "mq_test_decode_kernel", "mq_test_prefill_kernel",
-            "mq_weight_sq_sums", "mq_fold_quantize_pack_batch"]
+            "mq_weight_sq_sums", "mq_fold_quantize_pack_batch", "mq_test_tmajor_kernel"]
 MQ_WEIGHTS_SYM_CHANNEL, MQ_WEIGHTS_ASYM_CHANNEL, MQ_WEIGHTS_ASYM_TENSOR = 0, 1, 2
 MQ_TYPE_F32, MQ_TYPE_F16, MQ_TYPE_BF16, MQ_TYPE_I8, MQ_TYPE_I16 = 0, 1, 2, 3, 4
 
@@ -101,6 +101,7 @@ lib.mq_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
 lib.mq_test_skip_partials.argtypes = [_int]
 lib.mq_test_decode_kernel.argtypes = [_int]
 lib.mq_test_prefill_kernel.argtypes = [_int]
+lib.mq_test_tmajor_kernel.argtypes = [_int]
 lib.mq_weight_sq_sums.argtypes = [_vp, _int, _int, _int, _int, _vp, _vp]
 for _f in EXPORTED:
     if _f != "mq_status_string":
@@ -447,3 +448,9 @@ def test_prefill_kernel(which: int) -> int:
     """mq_test_prefill_kernel (test hook): 0 by shape and workspace, 1 the
     256-token kernel whenever the workspace allows, 2 never."""
     return lib.mq_test_prefill_kernel(int(which))
+
+
+def test_tmajor_kernel(which: int) -> int:
+    """mq_test_tmajor_kernel (test hook): 0 the token-major kernel for K <= 128,
+    1 whenever it can serve a problem, 2 never."""
+    return lib.mq_test_tmajor_kernel(int(which))
