@@ -1334,8 +1334,9 @@ def run_reference(args, dist: Dist):
 def run_profile_leg(mq, torch, dist, args):
     """One leg's timed loop alone, for a profiler (`--profile LEG`): the
     headline stack, the config-1 block, the config-2 decode block at M = 1,
-    config 4's prefill step, or config 4's decode step at M = 1 (block, then
-    head).  Prints the leg's time per step."""
+    config 4's prefill step, config 4's decode step at M = 1 (block, then
+    head), or one TinyLlama layer's attention matmuls at T = 1024.  Prints the
+    leg's time per step."""
     t0 = time.time()
     if args.profile == "stack":
         r = run_stack(mq, torch, dist, args.steps, args.warmup)
@@ -1346,6 +1347,9 @@ def run_profile_leg(mq, torch, dist, args):
     elif args.profile == "decode":
         r = run_decode(mq, torch, steps_per_m=args.steps, ms=(1,))
         per = r["m1"]["stream_us"] * 1e-3
+    elif args.profile == "attention":
+        r, _ = run_attention(mq, torch, reps=args.steps, check_rows=1)
+        per = r["us_per_layer"] * 1e-3
     elif args.profile == "gemma_decode":
         r, _ = run_gemma_decode(mq, torch, reps=args.steps, block_layers=1)
         per = r["step_us"] * 1e-3
@@ -1362,7 +1366,7 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mq", "reference"], default="mq")
-    ap.add_argument("--profile", choices=["stack", "block", "decode", "gemma", "gemma_decode"], default=None,
+    ap.add_argument("--profile", choices=["stack", "block", "decode", "gemma", "gemma_decode", "attention"], default=None,
                     help="run only this leg's timed loop (for a profiler; no JSON line)")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -618,10 +618,10 @@ int mq_test_prefill_kernel(int which);
  * tensor-core MMA's M, 128 a tile; channels as its N) for prefill problems
  * with 8-bit activations and int8 weights, 16-byte aligned x and weights with
  * row pitches that are multiples of 16 bytes, and no residual with an int16
- * output.  0 (the initial state) takes it for such problems with K <= 128 (the
- * attention scores Q K^T at head dimension K), 1 for every such problem, 2
- * never.  All kernels are bit-exact; the hook lets the tests run each one on
- * any shape.
+ * output.  0 (the initial state) takes it for such problems with K <= 128 or
+ * N <= 64 (the attention matmuls: Q K^T at head dimension K, P V with head
+ * dimension N), 1 for every such problem, 2 never.  All kernels are
+ * bit-exact; the hook lets the tests run each one on any shape.
  * Errors: MQ_ERR_INVALID_ARG for values other than 0, 1, 2.
  */
 int mq_test_tmajor_kernel(int which);

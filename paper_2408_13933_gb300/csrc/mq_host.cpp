@@ -265,12 +265,13 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
                 at + align1024(2 * (size_t)pl.wide[i].M * (size_t)pl.wide[i].K));
         }
     }
-    // the token-major kernel for short K (8-bit weights and activations; the
-    // attention scores Q K^T at head dimension K)
+    // the token-major kernel for short K or few channels (8-bit weights and
+    // activations; the attention matmuls: Q K^T at head dimension K, P V with
+    // head dimension N)
     const int tmajor_mode = mq::test_tmajor_kernel();
     auto takes_tmajor = [&](const mq::Problem &p) {
         if (tmajor_mode == 2 || !mq::tmajor_suits(p)) return false;
-        return tmajor_mode == 1 || p.K <= 128;
+        return tmajor_mode == 1 || p.K <= 128 || p.N <= 64;
     };
     std::vector<mq::Problem> tmaj[2];  // by o16
     std::vector<mq::Problem> pre2;

@@ -1,10 +1,9 @@
 // mq_tmajor.cu -- the token-major tensor-core kernel: tokens are the MMA's M
 // (128 per tile) and output channels its N, the transpose of the prefill
-// kernels' roles.  It serves the shape those kernels are not built for: short
-// K, i.e. the attention scores of the integer block (Sec. 4.1; Q K^T at K =
-// head dim 64, int16 scores).  It runs any other int8 problem too (narrow
-// tiles of 64 channels over several exact runs), bit-exact, but the prefill
-// kernels are faster at long K (measured on P V: 56 against 40 us a layer).
+// kernels' roles.  It serves the shapes those kernels are not built for:
+// short K or few channels, i.e. the attention matmuls of the integer block
+// (Sec. 4.1; Q K^T at K = head dim 64 with int16 scores, P V with N = head
+// dim 64).
 //
 // Both zero points are folded into the widening: the tensor cores contract
 // x - zx and w - zw (f16 integers, |.| <= 255), so the accumulator is the
@@ -29,16 +28,17 @@
 //   F[b] in TMEM (two buffers) --8 epilogue warps--> y.
 //
 // Tile shapes: TN = 256 channels when K fits one exact run and N > 64 (the
-// epilogue streams each 32-column load out), else TN = 64 (with several runs
-// each epilogue thread keeps 32 running int32 sums across them).
+// epilogue requantizes each tile straight out of tensor memory), else TN = 64
+// (with several runs each epilogue thread keeps 64 running int32 sums).
 //
-// Warp roles (704 threads, one CTA per SM, persistent over a contiguous range
-// of tiles):
+// Warp roles (one CTA per SM, persistent over a contiguous range of tiles):
 //   warp 0      TMA producer (one thread)
 //   warp 1      tensor-memory allocation, MMA issue (one elected lane)
-//   warps 2-5   converters: widen one stage of x and w into an operand slot
-//   warps 6-21  epilogue: warp w drains TMEM lanes 32 (w % 4) .. + 31 (its
-//               tokens) and a quarter of a wide tile's columns
+//   then        converters: one group of four warps (wide tiles) or two
+//               taking alternate stages (narrow): widen a stage of x and w
+//               into an operand slot
+//   then        epilogue: 16 warps (wide) or 4 (narrow); each drains TMEM
+//               lanes 32 (w % 4) .. + 31 (its tokens) and 64 columns
 // Every mbarrier wait is bounded (mq_wait_parity); a timeout raises the CTA's
 // abort word and every role unwinds, waiting for issued MMAs and loads first.
 #include <cuda.h>
@@ -63,22 +63,34 @@ constexpr int TMT = 128;  // tokens per tile (MMA M)
 constexpr int TNW = 256;  // channels per wide tile (one exact run)
 constexpr int TNN = 64;   // channels per narrow tile (any K)
 constexpr int KS = 64;    // k per stage: one 128-byte f16 row
-constexpr int S8 = 2;     // staging stages
-constexpr int SF = 2;     // operand stages
 constexpr int TMA_WARP = 0;
 constexpr int MMA_WARP = 1;
 constexpr int CONV_WARP0 = 2;
-constexpr int GROUP_WARPS = 4;  // converter warps
+constexpr int GROUP_WARPS = 4;  // converter warps of one group
 constexpr int GROUP_THREADS = GROUP_WARPS * 32;
-constexpr int EPI_WARP0 = CONV_WARP0 + GROUP_WARPS;
-constexpr int EPI_WARPS = 16;
-constexpr int THREADS = (EPI_WARP0 + EPI_WARPS) * 32;
 constexpr int STX = TMT * KS;   // token staging bytes
-constexpr int STW = TNW * KS;   // weight staging bytes (narrow tiles use the first quarter)
 constexpr int OPA = TMT * 128;  // f16 token operand
-constexpr int OPB = TNW * 128;  // f16 weight operand
 constexpr int OUTB = 32 * 128;  // one 32 x 64 output block (int16; int8 uses half)
 constexpr uint32_t TMEM_COLS = 512;  // F[b] at column 256 b
+
+// The two tile shapes, each its own kernel.  Wide: 256 channels, one stage
+// per tile (the scores): a short pipeline, 16 epilogue warps for the
+// requantization.  Narrow: 64 channels over many stages (long K): six
+// staging stages, four operand slots and two converter groups taking
+// alternate stages (each group's waits and signals overlap the other's
+// widening), four epilogue warps.
+template <bool NARROW>
+struct Cfg {
+    static constexpr int TN = NARROW ? TNN : TNW;
+    static constexpr int S8 = NARROW ? 6 : 2;  // staging stages
+    static constexpr int SF = NARROW ? 4 : 2;  // operand slots
+    static constexpr int GROUPS = NARROW ? 2 : 1;
+    static constexpr int EPI_WARP0 = CONV_WARP0 + GROUPS * GROUP_WARPS;
+    static constexpr int EPI_WARPS = NARROW ? 4 : 16;
+    static constexpr int THREADS = (EPI_WARP0 + EPI_WARPS) * 32;
+    static constexpr int STW = TN * KS;   // weight staging bytes
+    static constexpr int OPB = TN * 128;  // f16 weight operand
+};
 
 // ----------------------------------------------------------------- PTX helpers
 __device__ __forceinline__ void tmem_alloc1(uint32_t *dst_smem, uint32_t ncols) {
@@ -163,18 +175,20 @@ struct Params {
     uint64_t wait_ns;
 };
 
+template <bool NARROW>
 struct Smem {
-    uint8_t opa[SF][OPA];  // 1024-byte aligned (the swizzle pattern follows address bits)
-    uint8_t opb[SF][OPB];
-    uint8_t out[EPI_WARPS][OUTB];  // per epilogue warp: a block of 32 tokens x 64 channels
+    using C = Cfg<NARROW>;
+    uint8_t opa[C::SF][OPA];  // 1024-byte aligned (the swizzle pattern follows address bits)
+    uint8_t opb[C::SF][C::OPB];
+    uint8_t out[C::EPI_WARPS][OUTB];  // per epilogue warp: a block of 32 tokens x 64 channels
     Problem prob[PREFILL_MAX_PROBLEMS];  // the problem table (parameter reads are slow)
     int tn[PREFILL_MAX_PROBLEMS], kpr[PREFILL_MAX_PROBLEMS], flags[PREFILL_MAX_PROBLEMS];
-    uint8_t stx[S8][STX];
-    uint8_t stw[S8][STW];
-    uint64_t ld_full[S8];
-    uint64_t ld_empty[S8];
-    uint64_t op_full[SF];
-    uint64_t op_empty[SF];
+    uint8_t stx[C::S8][STX];
+    uint8_t stw[C::S8][C::STW];
+    uint64_t ld_full[C::S8];
+    uint64_t ld_empty[C::S8];
+    uint64_t op_full[C::SF];
+    uint64_t op_empty[C::SF];
     uint64_t f_full[2];
     uint64_t f_empty[2];
     uint64_t done;
@@ -182,7 +196,10 @@ struct Smem {
     int abort;
 };
 
-constexpr size_t SMEM_BYTES = sizeof(Smem) + 1024;  // + alignment slack
+template <bool NARROW>
+constexpr size_t smem_bytes() {
+    return sizeof(Smem<NARROW>) + 1024;  // + alignment slack
+}
 
 struct Tile {
     int pi, tt, ct, tn;
@@ -190,7 +207,8 @@ struct Tile {
 };
 
 // The last problem whose first tile is <= tile.
-__device__ __forceinline__ int problem_of(const Smem &s, int count, int tile) {
+template <class S>
+__device__ __forceinline__ int problem_of(const S &s, int count, int tile) {
     int lo = 0, hi = count - 1;
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
@@ -202,7 +220,8 @@ __device__ __forceinline__ int problem_of(const Smem &s, int count, int tile) {
     return lo;
 }
 
-__device__ __forceinline__ Tile tile_of(const Smem &s, int count, int tile) {
+template <class S>
+__device__ __forceinline__ Tile tile_of(const S &s, int count, int tile) {
     Tile t;
     t.pi = problem_of(s, count, tile);
     const Problem &p = s.prob[t.pi];
@@ -215,8 +234,8 @@ __device__ __forceinline__ Tile tile_of(const Smem &s, int count, int tile) {
     return t;
 }
 
-__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, Smem &s,
-                                          const Params &P) {
+template <class S>
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, S &s, const Params &P) {
     bool ok = true;
     if ((threadIdx.x & 31) == 0) ok = mq_wait_parity(bar, parity, &s.abort, P.status, P.wait_ns);
     return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
@@ -394,11 +413,16 @@ __device__ __forceinline__ void flush_block(uint8_t *blk, const Problem &p, cons
     }
 }
 
-// O16: every problem of the launch has an int16 output (else int8).
-template <bool O16>
-__global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constant__ Params P) {
+// O16: every problem of the launch has an int16 output (else int8).  NARROW:
+// the narrow tile shape (every problem of the launch has it).
+template <bool O16, bool NARROW>
+__global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
+    tmajor_kernel(const __grid_constant__ Params P) {
+    using C = Cfg<NARROW>;
+    constexpr int S8 = C::S8, SF = C::SF, THREADS = C::THREADS;
+    constexpr int EPI_WARP0 = C::EPI_WARP0, EPI_WARPS = C::EPI_WARPS;
     extern __shared__ uint8_t smem_raw[];
-    Smem &s = *reinterpret_cast<Smem *>(
+    Smem<NARROW> &s = *reinterpret_cast<Smem<NARROW> *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -527,7 +551,8 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
     } else if (warp < EPI_WARP0) {
         // ------------------------------------------------------ converters
         griddep_wait();  // before reading the weight zero points
-        const int ct = threadIdx.x - CONV_WARP0 * 32;  // 0 .. 127
+        const int grp = (warp - CONV_WARP0) / GROUP_WARPS;  // stages it with it % GROUPS == grp
+        const int ct = threadIdx.x - (CONV_WARP0 + GROUP_WARPS * grp) * 32;  // 0 .. 127
         uint32_t it = 0;
         bool ok = true;
         for (int tile = tile0; ok && tile < tile1; ++tile) {
@@ -536,14 +561,15 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
             const uint32_t xoff = f16x2_i8_offset(p.zx);
             // the weight rows this thread widens: r = ct / 4 + 32 u
             const int wchunks = t.tn * (KS / 16);  // 16-byte chunks of the staged w
-            uint32_t woff[TNW / 32];
+            uint32_t woff[C::TN / 32];
 #pragma unroll
-            for (int u = 0; u < TNW / 32; ++u) {
+            for (int u = 0; u < C::TN / 32; ++u) {
                 const int ch = t.ct * t.tn + (ct >> 2) + 32 * u;
                 woff[u] = F16X2_1152;
                 if (p.zw && 32 * u < t.tn && ch < p.N) woff[u] = f16x2_i8_offset(__ldg(p.zw + ch));
             }
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+                if ((int)(it % C::GROUPS) != grp) continue;  // the other group's stage
                 const int s8 = it % S8, sf = it % SF;
                 if (!warp_wait(&s.ld_full[s8], (it / S8) & 1, s, P) ||
                     !warp_wait(&s.op_empty[sf], ((it / SF) & 1) ^ 1, s, P)) {
@@ -560,7 +586,7 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
                                 live < 0 ? 0 : (live > 16 ? 16 : live));
                 }
 #pragma unroll
-                for (int u = 0; u < (TNW * KS / 16) / GROUP_THREADS; ++u) {
+                for (int u = 0; u < (C::TN * KS / 16) / GROUP_THREADS; ++u) {
                     const int i = ct + GROUP_THREADS * u;
                     if (i < wchunks) widen_chunk(s.stw[s8] + 16 * i, s.opb[sf], i >> 2, i & 3, woff[u]);
                 }
@@ -575,34 +601,28 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
         if (!ok && lane == 0) s.abort = 1;
     } else {
         // ------------------------------------------------------ epilogue
-        // Warp w drains TMEM lanes 32 (w % 4) .. + 31 (its tokens) and
-        // quarter (w - EPI_WARP0) / 4 of a wide tile's 256 columns (two
-        // 32-column groups, one stored block of 64 channels); of a narrow
-        // tile's 64 columns the first two quarters take 32 each and the
-        // others only keep the accumulator handshake.
+        // Warp w drains TMEM lanes 32 (w % 4) .. + 31 (its tokens) and 64 of
+        // the tile's columns (a quarter of a wide tile, all of a narrow one):
+        // two 32-column groups, stored as one block of 32 tokens x 64 channels.
         griddep_wait();  // before the first global access (parameters, residual, y)
         const int ew = warp - EPI_WARP0;
         const int quad = warp & 3;  // TMEM lane quarter: tokens 32 quad .. + 31
-        const int colq = ew >> 2;   // column quarter
+        const int colq = ew >> 2;   // 64-column quarter of a wide tile (0 for narrow)
         uint8_t *blk = s.out[ew];
         uint32_t runs = 0;
         bool ok = true, pending = false;
         // this lane's channel's M0 / shift in each of the warp's two column
         // groups, loaded one tile ahead
         int32_t nm0[2], nsh[2];
-        auto first_channel = [&](const Tile &t) {
-            return t.ct * t.tn + (t.tn == TNW ? 64 * colq : 32 * colq);
-        };
         auto fetch = [&](int tile) {
             if (tile >= tile1) return;
             const Tile t = tile_of(s, P.count, tile);
             const Problem &p = s.prob[t.pi];
-            const int ng = t.tn == TNW ? 2 : (colq < 2 ? 1 : 0);
-            const int chw = first_channel(t);
+            const int chw = t.ct * C::TN + 64 * colq;
 #pragma unroll
             for (int u = 0; u < 2; ++u) {
                 const int ch = chw + 32 * u + lane;
-                const bool in = u < ng && ch < p.N;
+                const bool in = ch < p.N;
                 nm0[u] = in ? __ldg(p.M0 + ch) : 0;
                 nsh[u] = in ? __ldg(p.shift + ch) : 33;
             }
@@ -611,9 +631,7 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
         for (int tile = tile0; ok && tile < tile1; ++tile) {
             const Tile t = tile_of(s, P.count, tile);
             const Problem &p = s.prob[t.pi];
-            const bool wide = t.tn == TNW;
-            const int ng = wide ? 2 : (colq < 2 ? 1 : 0);  // 32-column groups of this warp
-            const int chw = first_channel(t);
+            const int chw = t.ct * C::TN + 64 * colq;  // first channel of this warp
             int32_t m0[2], sh[2];
             bool uni[2];
 #pragma unroll
@@ -622,7 +640,7 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
                 const int32_t a0 = __shfl_sync(0xffffffffu, m0[u], 0);
                 const int32_t s0 = __shfl_sync(0xffffffffu, sh[u], 0);
                 // lanes past N hold (0, 33): uniform if every live lane agrees
-                const bool live = u < ng && chw + 32 * u + lane < p.N;
+                const bool live = chw + 32 * u + lane < p.N;
                 uni[u] = __all_sync(0xffffffffu, !live || (m0[u] == a0 && sh[u] == s0));
             }
             fetch(tile + 1);  // the next tile's parameters, while this one runs
@@ -630,47 +648,45 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
             const int32_t zy = p.zy;
             const bool vec = (s.flags[t.pi] & 1) != 0;
             const bool by_tma = (s.flags[t.pi] & 2) != 0;
-            const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) +
-                                    (uint32_t)(wide ? 64 * colq : 32 * colq);
+            const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(64 * colq);
             const int nruns = (t.nkb + t.kpr - 1) / t.kpr;
-            if (ng > 0 && pending) {  // the block's previous TMA store has read it
+            const bool active = chw < p.N;  // any channel of this warp inside N
+            if (active && pending) {  // the block's previous TMA store has read it
                 if (lane == 0) store_wait_read0();
                 __syncwarp();
             }
-            if (nruns == 1) {
+            if (!NARROW || nruns == 1) {
                 const uint32_t b = runs & 1;
                 if (!warp_wait(&s.f_full[b], (runs >> 1) & 1, s, P)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
+                if (active) {
 #pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    if (u >= ng) break;
-                    int32_t a[32];
-                    {
-                        uint32_t f[32];
-                        tc_ld_32x32b_x32(t_lane + 256u * b + 32u * u, f);
-                        tc_wait_ld();
+                    for (int u = 0; u < 2; ++u) {
+                        int32_t a[32];
+                        {
+                            uint32_t f[32];
+                            tc_ld_32x32b_x32(t_lane + 256u * b + 32u * u, f);
+                            tc_wait_ld();
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) a[i] = f2i_exact(f[i]);
-                    }
-                    uint32_t w[16];
-                    requant32<O16>(a, m0[u], sh[u], uni[u], zy, w);
-                    if (wide)
+                            for (int i = 0; i < 32; ++i) a[i] = f2i_exact(f[i]);
+                        }
+                        uint32_t w[16];
+                        requant32<O16>(a, m0[u], sh[u], uni[u], zy, w);
                         stage32<O16, O16 ? 128 : 64>(blk, u, lane, w);
-                    else
-                        stage32<O16, O16 ? 64 : 32>(blk, 0, lane, w);
+                    }
                 }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&s.f_empty[b]);  // F[b] read: the MMAs may go on
                 ++runs;
             } else {
-                // several runs (narrow tile): 32 channels summed in int32
-                int32_t acc[32];
+                // several runs (narrow tiles): 64 channels summed in int32
+                int32_t acc[64];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) acc[i] = 0;
+                for (int i = 0; i < 64; ++i) acc[i] = 0;
                 for (int r = 0; r < nruns; ++r, ++runs) {
                     const uint32_t b = runs & 1;
                     if (!warp_wait(&s.f_full[b], (runs >> 1) & 1, s, P)) {
@@ -678,9 +694,9 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
                         break;
                     }
                     tc_fence_after();
-                    if (ng > 0) {
+                    if (active) {
 #pragma unroll
-                        for (int h = 0; h < 2; ++h) {  // two 16-column loads
+                        for (int h = 0; h < 4; ++h) {  // four 16-column loads
                             uint32_t f[16];
                             tc_ld_32x32b_x16(t_lane + 256u * b + 16u * h, f);
                             tc_wait_ld();
@@ -693,17 +709,20 @@ __global__ void __launch_bounds__(THREADS, 1) tmajor_kernel(const __grid_constan
                     if (lane == 0) mbar_arrive(&s.f_empty[b]);
                 }
                 if (!ok) break;
-                if (ng > 0) {
-                    uint32_t w[16];
-                    requant32<O16>(acc, m0[0], sh[0], uni[0], zy, w);
-                    stage32<O16, O16 ? 64 : 32>(blk, 0, lane, w);
+                if (active) {
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        int32_t a[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) a[i] = acc[32 * u + i];
+                        uint32_t w[16];
+                        requant32<O16>(a, m0[u], sh[u], uni[u], zy, w);
+                        stage32<O16, O16 ? 128 : 64>(blk, u, lane, w);
+                    }
                 }
             }
-            if (ng > 0) {
-                if (wide)
-                    flush_block<O16, O16 ? 128 : 64>(blk, p, &P.tmap_y[t.pi], tok0, chw, vec, by_tma, lane);
-                else
-                    flush_block<O16, O16 ? 64 : 32>(blk, p, &P.tmap_y[t.pi], tok0, chw, vec, by_tma, lane);
+            if (active) {
+                flush_block<O16, O16 ? 128 : 64>(blk, p, &P.tmap_y[t.pi], tok0, chw, vec, by_tma, lane);
                 pending = pending || by_tma;
             }
         }
@@ -756,16 +775,74 @@ bool tmajor_suits(const Problem &p) {
            p.ldw % 16 == 0 && !(p.o16 && p.residual);
 }
 
+namespace tmajor {
+
+// One launch of up to PREFILL_MAX_PROBLEMS problems of one tile shape.
+template <bool NARROW>
+int launch_group(const Problem *const *probs, int n, bool o16, int sms, cudaStream_t stream) {
+    const auto al16 = [](const void *v) { return (reinterpret_cast<uintptr_t>(v) & 15u) == 0; };
+    const int osz = o16 ? 2 : 1;
+    Params P{};
+    long long tiles = 0;
+    for (int i = 0; i < n; ++i) {
+        Problem &q = P.p[i];
+        q = *probs[i];
+        P.kpr[i] = run_stages(q);
+        P.tn[i] = Cfg<NARROW>::TN;
+        q.tiles_m = (q.M + TMT - 1) / TMT;
+        q.tile_begin = (int)tiles;
+        tiles += (long long)q.tiles_m * ((q.N + P.tn[i] - 1) / P.tn[i]);
+        if (!encode(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M, (uint64_t)q.ldx, KS, TMT, 1,
+                    CU_TENSOR_MAP_SWIZZLE_NONE) ||
+            !encode(&P.tmap_w[i], q.w, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldw, KS,
+                    (uint32_t)P.tn[i], 1, CU_TENSOR_MAP_SWIZZLE_NONE))
+            return MQ_ERR_CUDA;
+        // 16-byte stores where y's rows (and the residual's) allow them;
+        // without a residual, TMA stores of blocks of 32 tokens x 64 channels
+        // (rows of 128 or 64 bytes, swizzled to match)
+        P.vec[i] = al16(q.y) && ((size_t)q.ldy * osz) % 16 == 0 &&
+                   (!q.residual || al16(q.residual));
+        P.tma_y[i] = P.vec[i] && !q.residual;
+        if (P.tma_y[i] &&
+            !encode(&P.tmap_y[i], q.y, (uint64_t)q.N, (uint64_t)q.M, (uint64_t)q.ldy * osz, 64, 32,
+                    osz, o16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))
+            return MQ_ERR_CUDA;
+    }
+    if (tiles == 0) return MQ_OK;
+    if (tiles > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
+    P.count = n;
+    P.total_tiles = (int)tiles;
+    P.status = device_status_ptr();
+    P.wait_ns = wait_limit_ns();
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)(tiles < sms ? tiles : sms), 1, 1);
+    cfg.blockDim = dim3(Cfg<NARROW>::THREADS, 1, 1);
+    cfg.dynamicSmemBytes = smem_bytes<NARROW>();
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = o16 ? cudaLaunchKernelEx(&cfg, tmajor_kernel<true, NARROW>, P)
+                              : cudaLaunchKernelEx(&cfg, tmajor_kernel<false, NARROW>, P);
+    return e == cudaSuccess ? MQ_OK : MQ_ERR_CUDA;
+}
+
+}  // namespace tmajor
+
 int launch_tmajor(const Problem *probs, int count, void *stream) {
     using namespace tmajor;
     static std::atomic<uint64_t> attr_done{0};  // bit d: device d prepared
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MQ_ERR_CUDA;
     if (!(attr_done.load(std::memory_order_acquire) & (1ull << dev))) {
-        const int smem = (int)SMEM_BYTES;
         const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
-        if (cudaFuncSetAttribute(tmajor_kernel<false>, attr, smem) != cudaSuccess ||
-            cudaFuncSetAttribute(tmajor_kernel<true>, attr, smem) != cudaSuccess)
+        const int sw = (int)smem_bytes<false>(), sn = (int)smem_bytes<true>();
+        if (cudaFuncSetAttribute(tmajor_kernel<false, false>, attr, sw) != cudaSuccess ||
+            cudaFuncSetAttribute(tmajor_kernel<true, false>, attr, sw) != cudaSuccess ||
+            cudaFuncSetAttribute(tmajor_kernel<false, true>, attr, sn) != cudaSuccess ||
+            cudaFuncSetAttribute(tmajor_kernel<true, true>, attr, sn) != cudaSuccess)
             return MQ_ERR_CUDA;
         attr_done.fetch_or(1ull << dev, std::memory_order_release);
     }
@@ -773,62 +850,25 @@ int launch_tmajor(const Problem *probs, int count, void *stream) {
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return MQ_ERR_CUDA;
-    const auto al16 = [](const void *v) { return (reinterpret_cast<uintptr_t>(v) & 15u) == 0; };
-    for (int begin = 0; begin < count; begin += PREFILL_MAX_PROBLEMS) {
-        const int n = count - begin < PREFILL_MAX_PROBLEMS ? count - begin : PREFILL_MAX_PROBLEMS;
-        const bool o16 = probs[begin].o16 != 0;
-        const int osz = o16 ? 2 : 1;
-        Params P{};
-        long long tiles = 0;
-        for (int i = 0; i < n; ++i) {
-            Problem &q = P.p[i];
-            q = probs[begin + i];
-            P.kpr[i] = run_stages(q);
-            P.tn[i] = ((q.K + KS - 1) / KS <= P.kpr[i] && q.N > TNN) ? TNW : TNN;
-            q.tiles_m = (q.M + TMT - 1) / TMT;
-            q.tile_begin = (int)tiles;
-            tiles += (long long)q.tiles_m * ((q.N + P.tn[i] - 1) / P.tn[i]);
-            if (!encode(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M, (uint64_t)q.ldx, KS, TMT,
-                        1, CU_TENSOR_MAP_SWIZZLE_NONE) ||
-                !encode(&P.tmap_w[i], q.w, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldw, KS,
-                        (uint32_t)P.tn[i], 1, CU_TENSOR_MAP_SWIZZLE_NONE))
-                return MQ_ERR_CUDA;
-            // 16-byte stores where y's rows (and the residual's) allow them;
-            // without a residual, TMA stores of 32-token blocks of TN / 4
-            // channels (rows of 128, 64 or 32 bytes, swizzled to match)
-            P.vec[i] = al16(q.y) && ((size_t)q.ldy * osz) % 16 == 0 &&
-                       (!q.residual || al16(q.residual));
-            P.tma_y[i] = P.vec[i] && !q.residual;
-            if (P.tma_y[i]) {
-                const uint32_t cols = P.tn[i] == TNW ? 64u : 32u;
-                const uint32_t rowb = cols * (uint32_t)osz;
-                const CUtensorMapSwizzle swz = rowb == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
-                                               : rowb == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                                            : CU_TENSOR_MAP_SWIZZLE_32B;
-                if (!encode(&P.tmap_y[i], q.y, (uint64_t)q.N, (uint64_t)q.M,
-                            (uint64_t)q.ldy * osz, cols, 32, osz, swz))
-                    return MQ_ERR_CUDA;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const bool o16 = probs[0].o16 != 0;
+    // wide tiles where K fits one exact run and N > 64, narrow ones otherwise
+    for (int narrow = 0; narrow < 2; ++narrow) {
+        const Problem *list[PREFILL_MAX_PROBLEMS];
+        int n = 0;
+        for (int i = 0; i <= count; ++i) {
+            if (i < count) {
+                const Problem &q = probs[i];
+                const bool wide = (q.K + KS - 1) / KS <= run_stages(q) && q.N > TNN;
+                if (wide == (narrow == 0)) list[n++] = &q;
+            }
+            if (n == PREFILL_MAX_PROBLEMS || (i == count && n > 0)) {
+                const int rc = narrow ? launch_group<true>(list, n, o16, sms, st)
+                                      : launch_group<false>(list, n, o16, sms, st);
+                if (rc != MQ_OK) return rc;
+                n = 0;
             }
         }
-        if (tiles == 0) continue;
-        if (tiles > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
-        P.count = n;
-        P.total_tiles = (int)tiles;
-        P.status = device_status_ptr();
-        P.wait_ns = wait_limit_ns();
-        cudaLaunchConfig_t cfg{};
-        cfg.gridDim = dim3((unsigned)(tiles < sms ? tiles : sms), 1, 1);
-        cfg.blockDim = dim3(THREADS, 1, 1);
-        cfg.dynamicSmemBytes = SMEM_BYTES;
-        cfg.stream = static_cast<cudaStream_t>(stream);
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[0].val.programmaticStreamSerializationAllowed = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        const cudaError_t e = o16 ? cudaLaunchKernelEx(&cfg, tmajor_kernel<true>, P)
-                                  : cudaLaunchKernelEx(&cfg, tmajor_kernel<false>, P);
-        if (e != cudaSuccess) return MQ_ERR_CUDA;
     }
     return MQ_OK;
 }

@@ -451,6 +451,6 @@ def test_prefill_kernel(which: int) -> int:
 
 
 def test_tmajor_kernel(which: int) -> int:
-    """mq_test_tmajor_kernel (test hook): 0 the token-major kernel for K <= 128,
-    1 whenever it can serve a problem, 2 never."""
+    """mq_test_tmajor_kernel (test hook): 0 the token-major kernel for K <= 128
+    or N <= 64, 1 whenever it can serve a problem, 2 never."""
     return lib.mq_test_tmajor_kernel(int(which))

@@ -5,7 +5,7 @@ ones (64 channels, several runs with and without a weight zero point), int8
 output with and without the residual, int16 output, ragged tokens, channels
 and K, extreme codes at the exact-run bound, rows that take the scalar store
 path, a batch over more problems than one launch holds, and the automatic
-choice (K <= 128) against the other kernels' bytes."""
+choice (K <= 128 or N <= 64) against the other kernels' bytes."""
 import numpy as np
 import pytest
 
@@ -170,8 +170,8 @@ def test_tmajor_batch_over_two_launches():
 @pytest.mark.parametrize("shape", [(512, 1024, 64), (1024, 64, 1024), (300, 2048, 2048)],
                          ids=lambda s: "x".join(map(str, s)))
 def test_tmajor_choice_matches_other_kernels(shape):
-    # the automatic choice (the first shape takes the token-major kernel, the
-    # others not) gives the bytes the other kernels give
+    # the automatic choice (the first two shapes take the token-major kernel,
+    # the third not) gives the bytes the other kernels give
     lib = mq()
     m, n, k = shape
     outs = []
