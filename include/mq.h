@@ -290,6 +290,14 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
  * least that and a multiple of 16), so that a head's slice of a projection
  * output ([T][heads * d], one head's d columns) can serve as the weights
  * without a copy.
+ * Row sums derived by the call: in a descriptor with int8 weights, `colsum`
+ * may be NULL.  The token-major kernel (mq_test_tmajor_kernel) contracts
+ * x - zx and w - zw directly and needs no row sums; for a problem any other
+ * kernel serves, the call first computes colsum[n] = sum_k w[n][k] into its
+ * workspace (N * 4 bytes per distinct weight matrix, counted by
+ * mq_workspace_size_batch; rounded up to 128 bytes).  For weights written on
+ * the device every call (keys, V^T in attention) this replaces a separate
+ * row-sum launch.  The single-linear calls still require colsum.
  * Weights written on the device: the kernels read `packed` before waiting for
  * the previous kernel in the stream (see mq_linear_w8a8).  A descriptor whose
  * weights are produced by earlier work on the same stream (keys, or V^T from
@@ -300,7 +308,7 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
 typedef struct mq_linear_desc {
     const void *x;          /* int8 [M][ldx], or int16 with abits == 16 */
     const void *packed;
-    const int32_t *colsum;
+    const int32_t *colsum;  /* may be NULL with int8 weights (bits 8), see below */
     const int32_t *M0;
     const int32_t *shift;
     const int8_t *residual; /* may be NULL; int8 activations only */

@@ -68,7 +68,10 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     // 128 * 255 * 65536 < 2^31)
     if (d.zw && ab == 8 && d.bits == 8 && d.K > MQ_MAX_K_ASYM8) return MQ_ERR_K_OVERFLOW;
     if (d.M > 0 && d.N > 0) {
-        if (!d.colsum || !d.M0 || !d.shift || !d.y || d.ldy < d.N) return MQ_ERR_INVALID_ARG;
+        // colsum may be omitted with int8 weights: the call derives it (see
+        // batch_plan) or its kernel needs none
+        if ((!d.colsum && d.bits != 8) || !d.M0 || !d.shift || !d.y || d.ldy < d.N)
+            return MQ_ERR_INVALID_ARG;
         if (d.K > 0) {  // with K == 0 neither x nor the weights are read
             if (!d.x || !d.packed || d.ldx < d.K) return MQ_ERR_INVALID_ARG;
             const int kq = d.bits == 8 ? 16 : 32;  // k per 16-byte weight segment
@@ -148,6 +151,8 @@ struct Plan {
     bool any_decode = false;
     std::vector<mq::SplitJob> split;
     std::vector<size_t> split_off;
+    std::vector<mq::RowsumJob> csum;  // weight row sums of descriptors without colsum
+    std::vector<size_t> csum_off;
     std::vector<mq::Widen16Job> wide;
     std::vector<size_t> wide_off;  // f16 copy at wide_off, row sums at + align1024(2 M K)
     size_t required = 0;           // decode region + planes
@@ -179,6 +184,26 @@ mq::Widen16Job output_copy_job(const mq_linear_desc &d) {
     return j;
 }
 
+// Whether a prefill problem takes the token-major kernel (mq_tmajor.cu): short
+// K or few channels (8-bit weights and activations; the attention matmuls:
+// Q K^T at head dimension K, P V with head dimension N).
+bool routes_tmajor(const mq_linear_desc &d, const mq::Problem &p) {
+    if (is_decode(d)) return false;
+    const int mode = mq::test_tmajor_kernel();
+    if (mode == 2 || !mq::tmajor_suits(p)) return false;
+    return mode == 1 || p.K <= 128 || p.N <= 64;
+}
+
+// A descriptor without colsum whose kernel needs one: the call computes the
+// weights' row sums first (the token-major kernel folds both zero points into
+// its operands and reads no colsum).
+bool needs_row_sums(const mq_linear_desc &d) {
+    if (d.colsum || d.M <= 0 || d.N <= 0) return false;
+    mq::Problem p{};
+    if (check_desc(d, p) != MQ_OK) return false;
+    return !routes_tmajor(d, p);
+}
+
 Plan batch_plan(const mq_linear_desc *descs, int count) {
     Plan pl;
     size_t off = 0;
@@ -202,6 +227,21 @@ Plan batch_plan(const mq_linear_desc *descs, int count) {
         pl.split.push_back(j);
         pl.split_off.push_back(off);
         off += align128(2 * (size_t)d.M * (size_t)d.K);
+    }
+    for (int i = 0; i < count; ++i) {
+        const mq_linear_desc &d = descs[i];
+        if (!needs_row_sums(d)) continue;
+        const int ldw = d.ldw > 0 ? d.ldw : d.K;
+        if (find_job(pl.csum, d.packed, d.N, d.K, ldw) >= 0) continue;
+        off = align128(off);
+        mq::RowsumJob j{};
+        j.x = static_cast<const int8_t *>(d.packed);
+        j.M = d.N;
+        j.K = d.K;
+        j.ldx = ldw;
+        pl.csum.push_back(j);
+        pl.csum_off.push_back(off);
+        off += align128(4 * (size_t)d.N);
     }
     pl.required = (pl.any_decode ? mq::DECODE_WS_BYTES : 0) + off;
     size_t woff = 0;
@@ -243,6 +283,8 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
     uint8_t *region = static_cast<uint8_t *>(workspace) + (pl.any_decode ? mq::DECODE_WS_BYTES : 0);
     for (size_t i = 0; i < pl.split.size(); ++i)
         pl.split[i].out = reinterpret_cast<int8_t *>(region + pl.split_off[i]);
+    for (size_t i = 0; i < pl.csum.size(); ++i)
+        pl.csum[i].out = reinterpret_cast<int32_t *>(region + pl.csum_off[i]);
     // the 256-token kernel for problems whose f16 copy is given, and for the
     // others when the workspace has room for the widened inputs
     const bool room = !pl.wide.empty() && workspace && ws_bytes >= pl.bytes;
@@ -265,14 +307,6 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
                 at + align1024(2 * (size_t)pl.wide[i].M * (size_t)pl.wide[i].K));
         }
     }
-    // the token-major kernel for short K or few channels (8-bit weights and
-    // activations; the attention matmuls: Q K^T at head dimension K, P V with
-    // head dimension N)
-    const int tmajor_mode = mq::test_tmajor_kernel();
-    auto takes_tmajor = [&](const mq::Problem &p) {
-        if (tmajor_mode == 2 || !mq::tmajor_suits(p)) return false;
-        return tmajor_mode == 1 || p.K <= 128 || p.N <= 64;
-    };
     std::vector<mq::Problem> tmaj[2];  // by o16
     std::vector<mq::Problem> pre2;
     std::vector<const uint16_t *> pre2_x16;
@@ -295,10 +329,14 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
                 p.x = pl.split[find_job(pl.split, d.x, d.M, d.K, d.ldx)].out;
             }
         }
+        if (!p.colsum && needs_row_sums(d)) {  // the row sums computed first
+            const int ldw = d.ldw > 0 ? d.ldw : d.K;
+            p.colsum = pl.csum[find_job(pl.csum, d.packed, d.N, d.K, ldw)].out;
+        }
         const int mode = p.a16 ? 1 : (p.o16 ? 2 : 0);
         if (is_decode(d)) {
             dec[p.bits == 8][mode].push_back(p);
-        } else if (takes_tmajor(p)) {
+        } else if (routes_tmajor(d, p)) {
             tmaj[p.o16 ? 1 : 0].push_back(p);
             if (d.y16) after.push_back(output_copy_job(d));
         } else if (takes_wide(d)) {
@@ -324,7 +362,8 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         }
     }
     int rc = MQ_OK;
-    if (!pl.split.empty())
+    if (!pl.csum.empty()) rc = mq::launch_rowsum(pl.csum.data(), (int)pl.csum.size(), stream);
+    if (rc == MQ_OK && !pl.split.empty())
         rc = mq::launch_split16(pl.split.data(), (int)pl.split.size(), stream);
     if (rc == MQ_OK && !pre2.empty()) {
         if (room) rc = mq::launch_widen16(pl.wide.data(), (int)pl.wide.size(), stream);
@@ -352,6 +391,7 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
 int single(int bits, const int8_t *x, int M, int K, int ldx, int32_t zx, const void *packed,
            const int32_t *colsum, int N, const int32_t *M0, const int32_t *shift, int32_t zy,
            int8_t *y, int ldy, void *workspace, size_t ws_bytes, void *stream) {
+    if (!colsum && M > 0 && N > 0) return MQ_ERR_INVALID_ARG;  // required by the single calls
     mq_linear_desc d{};
     d.x = x;
     d.packed = packed;
@@ -376,6 +416,7 @@ int single(int bits, const int8_t *x, int M, int K, int ldx, int32_t zx, const v
 int single_a16(int bits, const int16_t *x, int M, int K, int ldx, int32_t zx, const void *packed,
                const int32_t *colsum, int N, const int32_t *M0, const int32_t *shift, int32_t zy,
                int16_t *y, int ldy, void *workspace, size_t ws_bytes, void *stream) {
+    if (!colsum && M > 0 && N > 0) return MQ_ERR_INVALID_ARG;  // required by the single calls
     mq_linear_desc d{};
     d.x = x;
     d.packed = packed;
@@ -510,7 +551,8 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed, int32
 int mq_workspace_size(int M, int N, int K, int bits, size_t *bytes) {
     if (!bytes || M < 0 || N < 0 || K < 0 || (bits != 8 && bits != 4)) return MQ_ERR_INVALID_ARG;
     mq_linear_desc d{};
-    d.x = reinterpret_cast<const void *>(16);  // a placeholder address: only sizes are planned
+    d.x = reinterpret_cast<const void *>(16);  // placeholder addresses: only sizes are planned
+    d.colsum = reinterpret_cast<const int32_t *>(16);
     d.M = M;
     d.N = N;
     d.K = K;
@@ -550,7 +592,8 @@ int mq_workspace_size_batch(const mq_linear_desc *descs, int count, size_t *byte
 int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes) {
     if (!bytes || M < 0 || N < 0 || K < 0 || (bits != 8 && bits != 4)) return MQ_ERR_INVALID_ARG;
     mq_linear_desc d{};
-    d.x = reinterpret_cast<const void *>(16);  // a placeholder address: only sizes are planned
+    d.x = reinterpret_cast<const void *>(16);  // placeholder addresses: only sizes are planned
+    d.colsum = reinterpret_cast<const int32_t *>(16);
     d.M = M;
     d.N = N;
     d.K = K;
