@@ -989,9 +989,11 @@ def stack_parity(st, rows):
 
 # --------------------------------------------------------------------------- config 0
 def run_single_linear(mq, torch, copies: int = 40, reps: int = 2000):
-    """Config 0: one W8A8 linear, M = 128, K = N = 2048 (1.07 G int8 ops, one
-    prefill launch), rotating over `copies` independent operand sets (180 MB
-    > L2): back to back, and with CUDA events around every launch."""
+    """Config 0: one W8A8 linear, M = 128, K = N = 2048 (1.07 G int8 ops; with
+    the workspace mq_workspace_size_batch asks for, split over K on the
+    token-major kernel plus one combine launch), rotating over `copies`
+    independent operand sets (180 MB > L2): back to back, and with CUDA events
+    around every call."""
     c = synth.make_linear(0, 0, 0, "cfg0", 128, 2048, 2048, 8)
     packed, colsum = mq.pack_weights(c.w, 8)
     m0, sh = mq.requant_params(c.sw, c.sx, c.sy)
@@ -1006,7 +1008,11 @@ def run_single_linear(mq, torch, copies: int = 40, reps: int = 2000):
                                                      c.zy, y, 8)))
     stream = torch.cuda.current_stream()
     sp = stream.cuda_stream
-    call = mq.lib.mq_linear_batch
+    wsn = mq.workspace_size_batch([sets[0][0]])
+    ws = torch.zeros(max(16, wsn), dtype=torch.uint8, device="cuda")
+    wsp = ws.data_ptr() if wsn else None
+    lib_call = mq.lib.mq_linear_batch
+    call = lambda a, n, _w, _b, s: lib_call(a, n, wsp, wsn, s)
     for i in range(2 * copies):
         assert call(sets[i % copies], 1, None, 0, sp) == 0
     torch.cuda.synchronize()
@@ -1032,6 +1038,7 @@ def run_single_linear(mq, torch, copies: int = 40, reps: int = 2000):
     check = ParityCheck("config0_single_linear_m128", "linear", c, 128, ys[0].cpu().numpy(),
                         threaded=True)
     return {"what": "one W8A8 linear, M = 128, K = N = 2048", "int8_ops": ops,
+            "workspace_bytes": wsn,
             "us_back_to_back": round(ms * 1e3, 2),
             "tops_back_to_back": round(ops / (ms * 1e-3) / 1e12, 1),
             "us_per_launch_events": round(kms * 1e3, 2),

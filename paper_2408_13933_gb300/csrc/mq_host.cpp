@@ -153,6 +153,11 @@ struct Plan {
     std::vector<size_t> split_off;
     std::vector<mq::RowsumJob> csum;  // weight row sums of descriptors without colsum
     std::vector<size_t> csum_off;
+    int ksplit = 0;                   // slices of K of the split problems (0: none)
+    std::vector<int> ks_idx;          // descriptors split over K
+    std::vector<size_t> ks_off;       // their int32 partial sums, from ks_at (1024-aligned)
+    size_t ks_at = 0;
+    size_t bytes_wide = 0;            // end of the widened inputs (or of the required part)
     std::vector<mq::Widen16Job> wide;
     std::vector<size_t> wide_off;  // f16 copy at wide_off, row sums at + align1024(2 M K)
     size_t required = 0;           // decode region + planes
@@ -202,6 +207,28 @@ bool needs_row_sums(const mq_linear_desc &d) {
     mq::Problem p{};
     if (check_desc(d, p) != MQ_OK) return false;
     return !routes_tmajor(d, p);
+}
+
+// SMs of the current device (cached per device; 0 if the query fails).
+int device_sms() {
+    static std::atomic<int> cached[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    int n = cached[dev].load(std::memory_order_relaxed);
+    if (n == 0 && cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+        cached[dev].store(n, std::memory_order_relaxed);
+    return n;
+}
+
+// A prefill problem that may be split over K: one that the 128-token kernel
+// would serve with few tiles (M < 256 or N < 256), 8-bit activations and
+// weights, long enough K, and a shape the token-major kernel can take.
+bool split_candidate(const mq_linear_desc &d) {
+    if (d.M <= 0 || d.N <= 0 || d.K < 512 || is_decode(d) || d.y16) return false;
+    if (abits_of(d) != 8 || d.bits != 8 || (d.M >= WIDE_MIN_M && d.N >= WIDE_MIN_N)) return false;
+    mq::Problem p{};
+    if (check_desc(d, p) != MQ_OK) return false;
+    return !routes_tmajor(d, p) && mq::tmajor_suits(p);
 }
 
 Plan batch_plan(const mq_linear_desc *descs, int count) {
@@ -264,6 +291,41 @@ Plan batch_plan(const mq_linear_desc *descs, int count) {
     }
     // + 1024: the region starts at the first 1024-byte boundary after wide_at()
     pl.bytes = pl.wide.empty() ? pl.required : wide_at(pl) + woff + 1024;
+    pl.bytes_wide = pl.bytes;
+    // Split K: prefill calls whose tiles would leave most SMs idle (one M = 128
+    // linear makes 8 pair tiles for 76 pairs) run their problems as S slices
+    // of K on the token-major kernel, each writing its raw int32 sums, then one
+    // combine launch requantizes.  S = SMs / (the token-major tiles of the
+    // call), at most 8, each slice at least 256 k; only with the choice of
+    // prefill kernel left automatic, and only when the workspace has room
+    // (optional, like the widened inputs).
+    if (mq::test_prefill_kernel() == 0) {
+        long long tiles = 0;
+        int kmin = 1 << 30;
+        for (int i = 0; i < count; ++i) {
+            const mq_linear_desc &d = descs[i];
+            if (!split_candidate(d)) continue;
+            tiles += (long long)((d.M + 127) / 128) * ((d.N + 63) / 64);
+            kmin = d.K < kmin ? d.K : kmin;
+            pl.ks_idx.push_back(i);
+        }
+        const int sms = device_sms();
+        long long S = tiles > 0 ? sms / tiles : 0;
+        if (S > 8) S = 8;
+        if (S > kmin / 256) S = kmin / 256;
+        if (S >= 2) {
+            pl.ksplit = (int)S;
+            pl.ks_at = pl.bytes > wide_at(pl) ? pl.bytes : wide_at(pl);
+            size_t o = 0;
+            for (int i : pl.ks_idx) {
+                pl.ks_off.push_back(o);
+                o += align1024((size_t)S * (size_t)descs[i].M * (size_t)descs[i].N * 4);
+            }
+            pl.bytes = pl.ks_at + o + 1024;
+        } else {
+            pl.ks_idx.clear();
+        }
+    }
     return pl;
 }
 
@@ -287,7 +349,11 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         pl.csum[i].out = reinterpret_cast<int32_t *>(region + pl.csum_off[i]);
     // the 256-token kernel for problems whose f16 copy is given, and for the
     // others when the workspace has room for the widened inputs
-    const bool room = !pl.wide.empty() && workspace && ws_bytes >= pl.bytes;
+    const bool room = !pl.wide.empty() && workspace && ws_bytes >= pl.bytes_wide;
+    const bool room_split = pl.ksplit > 0 && workspace && ws_bytes >= pl.bytes;
+    std::vector<mq::Problem> ksub;     // the slices of the split problems
+    std::vector<uint8_t> ksub_part;
+    std::vector<mq::ReduceJob> kred;   // their combines
     bool ready = false, ready_known = false;
     auto takes_wide = [&](const mq_linear_desc &d) {
         if (!wide_eligible(d) || !(d.x16 || room)) return false;
@@ -327,6 +393,46 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
                 p.ldx = d.ldx;
             } else {
                 p.x = pl.split[find_job(pl.split, d.x, d.M, d.K, d.ldx)].out;
+            }
+        }
+        if (room_split) {
+            int j = -1;
+            for (size_t u = 0; u < pl.ks_idx.size(); ++u)
+                if (pl.ks_idx[u] == i) j = (int)u;
+            if (j >= 0) {  // S slices of K, raw int32 sums into the workspace, then a combine
+                const uintptr_t base =
+                    (reinterpret_cast<uintptr_t>(workspace) + pl.ks_at + 1023) & ~(uintptr_t)1023;
+                int32_t *part = reinterpret_cast<int32_t *>(base + pl.ks_off[j]);
+                const size_t slice = (size_t)p.M * (size_t)p.N;
+                const int kl = ((p.K + pl.ksplit - 1) / pl.ksplit + 63) / 64 * 64;
+                int nslices = 0;
+                for (int k0 = 0; k0 < p.K; k0 += kl, ++nslices) {
+                    mq::Problem q = p;
+                    q.x = p.x + k0;
+                    q.w = p.w + k0;
+                    q.K = p.K - k0 < kl ? p.K - k0 : kl;
+                    q.y = reinterpret_cast<int8_t *>(part + (size_t)nslices * slice);
+                    q.ldy = p.N;
+                    q.residual = nullptr;
+                    q.o16 = 0;
+                    q.wsq = nullptr;
+                    ksub.push_back(q);
+                    ksub_part.push_back(1);
+                }
+                mq::ReduceJob r{};
+                r.part = part;
+                r.S = nslices;
+                r.M = p.M;
+                r.N = p.N;
+                r.M0 = p.M0;
+                r.shift = p.shift;
+                r.zy = p.zy;
+                r.residual = p.residual;
+                r.y = p.y;
+                r.ldy = p.ldy;
+                r.o16 = p.o16;
+                kred.push_back(r);
+                continue;
             }
         }
         if (!p.colsum && needs_row_sums(d)) {  // the row sums computed first
@@ -374,6 +480,10 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
     for (int o = 0; o < 2; ++o)
         if (rc == MQ_OK && !tmaj[o].empty())
             rc = mq::launch_tmajor(tmaj[o].data(), (int)tmaj[o].size(), stream);
+    if (rc == MQ_OK && !ksub.empty()) {
+        rc = mq::launch_tmajor(ksub.data(), (int)ksub.size(), stream, ksub_part.data());
+        if (rc == MQ_OK) rc = mq::launch_splitk_reduce(kred.data(), (int)kred.size(), stream);
+    }
     for (int mode = 0; mode < 3; ++mode)
         if (rc == MQ_OK && !pre[mode].empty())
             rc = mq::launch_prefill(pre[mode].data(), (int)pre[mode].size(), stream);

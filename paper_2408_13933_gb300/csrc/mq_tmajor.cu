@@ -169,6 +169,7 @@ struct Params {
     int kpr[PREFILL_MAX_PROBLEMS];              // stages per exact run
     int vec[PREFILL_MAX_PROBLEMS];              // y (and residual) rows allow 16-byte accesses
     int tma_y[PREFILL_MAX_PROBLEMS];            // y written by TMA stores (vec, no residual)
+    int part[PREFILL_MAX_PROBLEMS];             // y is int32 [M][ldy]: raw sums of a slice of K
     int count;
     int total_tiles;
     int *status;
@@ -413,6 +414,26 @@ __device__ __forceinline__ void flush_block(uint8_t *blk, const Problem &p, cons
     }
 }
 
+// A slice of split K: this lane's token's 32 raw sums (channels ch0 .. ch0 +
+// 31) into the int32 partial buffer y [M][ldy].
+__device__ __forceinline__ void store_part32(const int32_t *a, const Problem &p, int tok, int ch0) {
+    if (tok >= p.M) return;
+    int32_t *y = reinterpret_cast<int32_t *>(p.y) + (size_t)tok * (size_t)p.ldy + ch0;
+    const bool vec = (p.ldy & 3) == 0 && (reinterpret_cast<uintptr_t>(p.y) & 15) == 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const int ch = ch0 + 4 * j;
+        if (vec && ch + 4 <= p.N) {
+            *reinterpret_cast<int4 *>(y + 4 * j) =
+                make_int4(a[4 * j], a[4 * j + 1], a[4 * j + 2], a[4 * j + 3]);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                if (ch + e < p.N) y[4 * j + e] = a[4 * j + e];
+        }
+    }
+}
+
 // O16: every problem of the launch has an int16 output (else int8).  NARROW:
 // the narrow tile shape (every problem of the launch has it).
 template <bool O16, bool NARROW>
@@ -431,7 +452,7 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
         s.prob[i] = P.p[i];
         s.tn[i] = P.tn[i];
         s.kpr[i] = P.kpr[i];
-        s.flags[i] = (P.vec[i] ? 1 : 0) | (P.tma_y[i] ? 2 : 0);
+        s.flags[i] = (P.vec[i] ? 1 : 0) | (P.tma_y[i] ? 2 : 0) | (P.part[i] ? 4 : 0);
     }
     if (threadIdx.x == 0) {
         for (int i = 0; i < S8; ++i) {
@@ -648,6 +669,7 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
             const int32_t zy = p.zy;
             const bool vec = (s.flags[t.pi] & 1) != 0;
             const bool by_tma = (s.flags[t.pi] & 2) != 0;
+            const bool part = (s.flags[t.pi] & 4) != 0;  // raw int32 sums of a slice of K
             const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(64 * colq);
             const int nruns = (t.nkb + t.kpr - 1) / t.kpr;
             const bool active = chw < p.N;  // any channel of this warp inside N
@@ -672,6 +694,10 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                             tc_wait_ld();
 #pragma unroll
                             for (int i = 0; i < 32; ++i) a[i] = f2i_exact(f[i]);
+                        }
+                        if (part) {
+                            store_part32(a, p, tok0 + lane, chw + 32 * u);
+                            continue;
                         }
                         uint32_t w[16];
                         requant32<O16>(a, m0[u], sh[u], uni[u], zy, w);
@@ -709,7 +735,10 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                     if (lane == 0) mbar_arrive(&s.f_empty[b]);
                 }
                 if (!ok) break;
-                if (active) {
+                if (active && part) {
+                    store_part32(acc, p, tok0 + lane, chw);
+                    store_part32(acc + 32, p, tok0 + lane, chw + 32);
+                } else if (active) {
 #pragma unroll
                     for (int u = 0; u < 2; ++u) {
                         int32_t a[32];
@@ -721,7 +750,7 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                     }
                 }
             }
-            if (active) {
+            if (active && !part) {
                 flush_block<O16, O16 ? 128 : 64>(blk, p, &P.tmap_y[t.pi], tok0, chw, vec, by_tma, lane);
                 pending = pending || by_tma;
             }
@@ -779,7 +808,8 @@ namespace tmajor {
 
 // One launch of up to PREFILL_MAX_PROBLEMS problems of one tile shape.
 template <bool NARROW>
-int launch_group(const Problem *const *probs, int n, bool o16, int sms, cudaStream_t stream) {
+int launch_group(const Problem *const *probs, const bool *part, int n, bool o16, int sms,
+                 cudaStream_t stream) {
     const auto al16 = [](const void *v) { return (reinterpret_cast<uintptr_t>(v) & 15u) == 0; };
     const int osz = o16 ? 2 : 1;
     Params P{};
@@ -802,7 +832,8 @@ int launch_group(const Problem *const *probs, int n, bool o16, int sms, cudaStre
         // (rows of 128 or 64 bytes, swizzled to match)
         P.vec[i] = al16(q.y) && ((size_t)q.ldy * osz) % 16 == 0 &&
                    (!q.residual || al16(q.residual));
-        P.tma_y[i] = P.vec[i] && !q.residual;
+        P.part[i] = part[i] ? 1 : 0;
+        P.tma_y[i] = P.vec[i] && !q.residual && !part[i];
         if (P.tma_y[i] &&
             !encode(&P.tmap_y[i], q.y, (uint64_t)q.N, (uint64_t)q.M, (uint64_t)q.ldy * osz, 64, 32,
                     osz, o16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))
@@ -831,7 +862,7 @@ int launch_group(const Problem *const *probs, int n, bool o16, int sms, cudaStre
 
 }  // namespace tmajor
 
-int launch_tmajor(const Problem *probs, int count, void *stream) {
+int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *part) {
     using namespace tmajor;
     static std::atomic<uint64_t> attr_done{0};  // bit d: device d prepared
     int dev = 0;
@@ -855,19 +886,116 @@ int launch_tmajor(const Problem *probs, int count, void *stream) {
     // wide tiles where K fits one exact run and N > 64, narrow ones otherwise
     for (int narrow = 0; narrow < 2; ++narrow) {
         const Problem *list[PREFILL_MAX_PROBLEMS];
+        bool lpart[PREFILL_MAX_PROBLEMS];
         int n = 0;
         for (int i = 0; i <= count; ++i) {
             if (i < count) {
                 const Problem &q = probs[i];
                 const bool wide = (q.K + KS - 1) / KS <= run_stages(q) && q.N > TNN;
-                if (wide == (narrow == 0)) list[n++] = &q;
+                if (wide == (narrow == 0)) {
+                    lpart[n] = part && part[i];
+                    list[n++] = &q;
+                }
             }
             if (n == PREFILL_MAX_PROBLEMS || (i == count && n > 0)) {
-                const int rc = narrow ? launch_group<true>(list, n, o16, sms, st)
-                                      : launch_group<false>(list, n, o16, sms, st);
+                const int rc = narrow ? launch_group<true>(list, lpart, n, o16, sms, st)
+                                      : launch_group<false>(list, lpart, n, o16, sms, st);
                 if (rc != MQ_OK) return rc;
                 n = 0;
             }
+        }
+    }
+    return MQ_OK;
+}
+
+namespace tmajor {
+
+constexpr int REDUCE_THREADS = 256;
+
+struct ReduceParams {
+    ReduceJob job[REDUCE_MAX_JOBS];
+    int block_begin[REDUCE_MAX_JOBS + 1];
+    int count;
+};
+
+// y = requant(sum over the S slices of the int32 partial sums) (+ residual):
+// one thread per four consecutive outputs of a row.  The partial sums come
+// from the previous kernel in the stream, so nothing is read before
+// griddep_wait.
+template <bool O16>
+__global__ void __launch_bounds__(REDUCE_THREADS) reduce_kernel(const __grid_constant__ ReduceParams R) {
+    griddep_wait();
+    griddep_launch_dependents();
+    int j = 0;
+    while (j + 1 < R.count && (int)blockIdx.x >= R.block_begin[j + 1]) ++j;
+    const ReduceJob &q = R.job[j];
+    const int quads = (q.N + 3) >> 2;  // four-channel groups of a row
+    const int64_t e = (int64_t)(blockIdx.x - R.block_begin[j]) * REDUCE_THREADS + threadIdx.x;
+    if (e >= (int64_t)q.M * quads) return;
+    const int m = (int)(e / quads), n0 = 4 * (int)(e % quads);
+    const size_t slice = (size_t)q.M * (size_t)q.N;
+    const int32_t *src = q.part + (size_t)m * (size_t)q.N + n0;
+    int32_t acc[4] = {0, 0, 0, 0};
+    const bool vec = (q.N & 3) == 0 && n0 + 4 <= q.N;
+    for (int s = 0; s < q.S; ++s, src += slice) {
+        if (vec) {
+            const int4 v = __ldcg(reinterpret_cast<const int4 *>(src));
+            acc[0] += v.x, acc[1] += v.y, acc[2] += v.z, acc[3] += v.w;
+        } else {
+            for (int c = 0; c < 4; ++c)
+                if (n0 + c < q.N) acc[c] += __ldcg(src + c);
+        }
+    }
+    const size_t row = (size_t)m * (size_t)q.ldy;
+    for (int c = 0; c < 4; ++c) {
+        const int n = n0 + c;
+        if (n >= q.N) break;
+        const int32_t m0 = __ldg(q.M0 + n), sh = __ldg(q.shift + n);
+        if (O16) {
+            reinterpret_cast<int16_t *>(q.y)[row + n] =
+                (int16_t)mq_requant16((int64_t)acc[c], m0, sh, q.zy);
+        } else {
+            int32_t o = mq_requant(acc[c], m0, sh, q.zy);
+            if (q.residual) o = min(127, max(-128, o + (int32_t)q.residual[row + n]));
+            reinterpret_cast<int8_t *>(q.y)[row + n] = (int8_t)o;
+        }
+    }
+}
+
+}  // namespace tmajor
+
+int launch_splitk_reduce(const ReduceJob *jobs, int count, void *stream) {
+    using namespace tmajor;
+    for (int base = 0; base < count; base += REDUCE_MAX_JOBS) {
+        const int n = count - base < REDUCE_MAX_JOBS ? count - base : REDUCE_MAX_JOBS;
+        for (int o = 0; o < 2; ++o) {  // int8, then int16 outputs
+            ReduceParams R{};
+            int64_t blocks = 0;
+            int c = 0;
+            for (int i = 0; i < n; ++i) {
+                const ReduceJob &q = jobs[base + i];
+                if ((q.o16 != 0) != (o == 1) || q.M <= 0 || q.N <= 0) continue;
+                R.job[c] = q;
+                R.block_begin[c] = (int)blocks;
+                blocks += ((int64_t)q.M * ((q.N + 3) / 4) + REDUCE_THREADS - 1) / REDUCE_THREADS;
+                ++c;
+            }
+            if (c == 0) continue;
+            if (blocks > 0x7fffffffLL) return MQ_ERR_UNSUPPORTED_SHAPE;
+            R.block_begin[c] = (int)blocks;
+            R.count = c;
+            cudaLaunchConfig_t cfg{};
+            cfg.gridDim = dim3((unsigned)blocks, 1, 1);
+            cfg.blockDim = dim3(REDUCE_THREADS, 1, 1);
+            cfg.stream = static_cast<cudaStream_t>(stream);
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+            attr[0].val.programmaticStreamSerializationAllowed = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            const cudaError_t e = o ? cudaLaunchKernelEx(&cfg, reduce_kernel<true>, R)
+                                    : cudaLaunchKernelEx(&cfg, reduce_kernel<false>, R);
+            if (e != cudaSuccess) return MQ_ERR_CUDA;
         }
     }
     return MQ_OK;

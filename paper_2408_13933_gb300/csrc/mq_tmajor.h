@@ -11,8 +11,24 @@ namespace mq {
 // of 16 bytes, no residual with an int16 output.
 bool tmajor_suits(const Problem &p);
 // Launcher (asynchronous on `stream`; the problems of one call have the same
-// o16); returns MQ_OK or MQ_ERR_CUDA.
-int launch_tmajor(const Problem *probs, int count, void *stream);
+// o16); returns MQ_OK or MQ_ERR_CUDA.  part[i] nonzero (part may be null):
+// problem i is a slice of a split K whose y is an int32 [M][ldy] buffer of
+// its raw sums sum (x - zx)(w - zw), requantized later by launch_splitk_reduce.
+int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *part = nullptr);
+
+// One split problem's combine: y = requant(sum of the S slices' int32 sums,
+// part + s M N, s < S) with M0 / shift / zy (+ residual for int8 outputs).
+struct ReduceJob {
+    const int32_t *part;
+    int32_t S, M, N;
+    const int32_t *M0, *shift;
+    int32_t zy;
+    const int8_t *residual;
+    void *y;
+    int32_t ldy, o16;
+};
+constexpr int REDUCE_MAX_JOBS = 32;
+int launch_splitk_reduce(const ReduceJob *jobs, int count, void *stream);
 // Test hook (mq_test_tmajor_kernel): 0 takes the kernel for K <= 128 or
 // N <= 64, 1 whenever it can serve a problem, 2 never.
 int test_tmajor_kernel();
