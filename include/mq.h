@@ -108,13 +108,20 @@ int mq_pack_weights(const int8_t *w, int N, int K, int bits, void *packed,
  * its row sums of squares (4 M bytes), placed after the size of the decode
  * region, each rounded up to 1024 bytes, plus 1024 bytes of alignment slack.
  * That part is optional: a prefill call given less (even no workspace) runs
- * the 128-token kernel instead, bit-identical and slower.  Smaller M: 0.  For
- * mq_linear_batch use mq_workspace_size_batch.
+ * the 128-token kernel instead, bit-identical and slower.  Prefill shapes
+ * below that (M < 256 or N < 256, int8 weights, K >= 512) whose tiles would
+ * leave most SMs idle: room, also optional, for S slices' int32 partial sums
+ * (S M N 4 bytes, S = the SMs over the token-major kernel's tiles, at most 8,
+ * from the first 1024-byte boundary after the decode region's size, plus 1024
+ * bytes of slack): with it the call splits K over S launches' worth of tiles
+ * and combines them in one more launch, bit-identical (a forced prefill kernel,
+ * mq_test_prefill_kernel, never splits).  Otherwise 0.  For mq_linear_batch use
+ * mq_workspace_size_batch.
  * Workspace contract: device memory, 16-byte aligned, zero-filled before its
  * first use.  The decode region (the first mq_workspace_size(1, 1, 0, 4)
  * bytes) is left zero-filled again by every call that completes, so the
  * workspace can be reused by later calls on the same stream; the widened
- * inputs after it are scratch, overwritten by each call.  Calls that may run
+ * inputs and partial sums after it are scratch, overwritten by each call.  Calls that may run
  * concurrently (different streams) need different workspaces.  After
  * MQ_ERR_DEVICE_TIMEOUT the decode region must be zero-filled again.
  * Errors: MQ_ERR_INVALID_ARG.
@@ -375,11 +382,16 @@ typedef struct mq_linear_desc {
  * bytes) and row sums of squares (4 M bytes), each rounded up to 1024, placed
  * after the decode region's size, plus 1024 bytes of alignment slack; a call
  * given only the required part runs those descriptors on the 128-token
- * kernel.  0 when none applies.  The decode region (the first
+ * kernel.  The required part also holds, for descriptors without colsum that
+ * the token-major kernel does not serve, their weights' row sums (4 N bytes,
+ * rounded up to 128, per distinct weight matrix).  Last, optionally, the
+ * split-K partial sums of the call's small prefill descriptors (see
+ * mq_workspace_size; S is shared by the call, from all of them).  0 when none
+ * applies.  The decode region (the first
  * mq_workspace_size(1, 1, 0, 4) bytes) follows the contract of
  * mq_workspace_size: zero-filled before first use and left zero by every
- * call that completes; the plane and widened-input regions are scratch,
- * overwritten by each call.
+ * call that completes; the other regions are scratch, overwritten by each
+ * call.
  * Errors: MQ_ERR_INVALID_ARG (null pointers, count out of range, bad bits or
  * abits).
  */
