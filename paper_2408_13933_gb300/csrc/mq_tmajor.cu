@@ -134,12 +134,7 @@ __device__ __forceinline__ void tma_store_2d(const void *map, int x, int y, cons
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
 
-// Wait until at most one (zero) of this thread's bulk groups still reads
-// shared memory.
-__device__ __forceinline__ void store_wait_read1() {
-    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-}
-
+// Wait until none of this thread's bulk groups still reads shared memory.
 __device__ __forceinline__ void store_wait_read0() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
