@@ -8,10 +8,10 @@
 // Both zero points are folded into the widening: the tensor cores contract
 // x - zx and w - zw (f16 integers, |.| <= 255), so the accumulator is the
 // corrected sum itself and the epilogue only requantizes.  Each f32 run of
-// the contraction is exact: its partial sums stay below 2^22 (the run length
-// is 2^22 over the largest |x - zx| |w - zw|, in whole stages; one stage of
-// 64 k at the extremes), which also lets the epilogue convert them to int32
-// with an add instead of a conversion instruction.
+// the contraction is exact: its partial sums stay below 2^24 (narrow tiles)
+// or 2^22 (wide tiles, whose epilogue converts them to int32 with an add
+// instead of a conversion instruction); the run length is that bound over the
+// largest |x - zx| |w - zw|, in whole stages.
 //
 // A tile's accumulator lives in tensor memory with one token per lane, so an
 // epilogue thread holds 32 consecutive channels of one token after one
@@ -90,6 +90,12 @@ struct Cfg {
     static constexpr int THREADS = (EPI_WARP0 + EPI_WARPS) * 32;
     static constexpr int STW = TN * KS;   // weight staging bytes
     static constexpr int OPB = TN * 128;  // f16 weight operand
+    // accumulator buffers F[b] at tensor-memory column b TN: two wide ones;
+    // four narrow ones, so that the MMAs run ahead of the epilogue's drains
+    static constexpr int NF = NARROW ? 4 : 2;
+    // exact runs: partial sums below 2^22 for the wide epilogue's add-based
+    // conversion, below 2^24 (f32's exact integers) for the narrow one's
+    static constexpr int RUN_BITS = NARROW ? 24 : 22;
 };
 
 // ----------------------------------------------------------------- PTX helpers
@@ -185,8 +191,8 @@ struct Smem {
     uint64_t ld_empty[C::S8];
     uint64_t op_full[C::SF];
     uint64_t op_empty[C::SF];
-    uint64_t f_full[2];
-    uint64_t f_empty[2];
+    uint64_t f_full[C::NF];
+    uint64_t f_empty[C::NF];
     uint64_t done;
     uint32_t tmem_base;
     int abort;
@@ -458,7 +464,7 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
             mbar_init(&s.op_full[i], GROUP_WARPS);
             mbar_init(&s.op_empty[i], 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < C::NF; ++b) {
             mbar_init(&s.f_full[b], 1);
             mbar_init(&s.f_empty[b], EPI_WARPS);
         }
@@ -528,8 +534,8 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
             int kr = 0;  // stage within the exact run
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                 const bool run_start = kr == 0;
-                const uint32_t b = runs & 1;
-                if (run_start && !warp_wait(&s.f_empty[b], ((runs >> 1) & 1) ^ 1, s, P)) {
+                const uint32_t b = runs % C::NF;
+                if (run_start && !warp_wait(&s.f_empty[b], ((runs / C::NF) & 1) ^ 1, s, P)) {
                     ok = false;
                     break;
                 }
@@ -545,7 +551,7 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                     const uint64_t bd = smem_desc_sw128(smem_u32(s.opb[slot]));
 #pragma unroll
                     for (int j = 0; j < KS / 16; ++j)  // +32 B along K: +2 in the (addr >> 4) field
-                        mma_f16_ss(tmem + 256u * b, ad + 2 * j, bd + 2 * j, idesc,
+                        mma_f16_ss(tmem + (uint32_t)C::TN * b, ad + 2 * j, bd + 2 * j, idesc,
                                    (run_start && j == 0) ? 0u : 1u);
                     commit1(&s.op_empty[slot]);
                     if (run_end) commit1(&s.f_full[b]);
@@ -673,8 +679,8 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                 __syncwarp();
             }
             if (!NARROW || nruns == 1) {
-                const uint32_t b = runs & 1;
-                if (!warp_wait(&s.f_full[b], (runs >> 1) & 1, s, P)) {
+                const uint32_t b = runs % C::NF;
+                if (!warp_wait(&s.f_full[b], (runs / C::NF) & 1, s, P)) {
                     ok = false;
                     break;
                 }
@@ -685,10 +691,11 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                         int32_t a[32];
                         {
                             uint32_t f[32];
-                            tc_ld_32x32b_x32(t_lane + 256u * b + 32u * u, f);
+                            tc_ld_32x32b_x32(t_lane + (uint32_t)C::TN * b + 32u * u, f);
                             tc_wait_ld();
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) a[i] = f2i_exact(f[i]);
+                            for (int i = 0; i < 32; ++i)
+                                a[i] = NARROW ? __float2int_rn(__uint_as_float(f[i])) : f2i_exact(f[i]);
                         }
                         if (part) {
                             store_part32(a, p, tok0 + lane, chw + 32 * u);
@@ -709,8 +716,8 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
 #pragma unroll
                 for (int i = 0; i < 64; ++i) acc[i] = 0;
                 for (int r = 0; r < nruns; ++r, ++runs) {
-                    const uint32_t b = runs & 1;
-                    if (!warp_wait(&s.f_full[b], (runs >> 1) & 1, s, P)) {
+                    const uint32_t b = runs % C::NF;
+                    if (!warp_wait(&s.f_full[b], (runs / C::NF) & 1, s, P)) {
                         ok = false;
                         break;
                     }
@@ -719,10 +726,11 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
 #pragma unroll
                         for (int h = 0; h < 4; ++h) {  // four 16-column loads
                             uint32_t f[16];
-                            tc_ld_32x32b_x16(t_lane + 256u * b + 16u * h, f);
+                            tc_ld_32x32b_x16(t_lane + (uint32_t)C::TN * b + 16u * h, f);
                             tc_wait_ld();
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) acc[16 * h + i] += f2i_exact(f[i]);
+                            for (int i = 0; i < 16; ++i)
+                                acc[16 * h + i] += __float2int_rn(__uint_as_float(f[i]));
                         }
                     }
                     tc_fence_before();
@@ -781,12 +789,13 @@ bool encode(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows, ui
 
 // Stages per exact f32 run: the largest |x - zx| |w - zw| bounds every
 // product (x in [-128, 127]; w - zw in [-255, 255] with a per-channel zero
-// point, else w in [-128, 127]); the run keeps its partial sums below 2^22,
-// inside f32's exact integers and the range of f2i_exact.
-int run_stages(const Problem &p) {
+// point, else w in [-128, 127]); the run keeps its partial sums below
+// 2^run_bits: 2^22 inside the range of f2i_exact (wide tiles), 2^24 f32's
+// exact integers (narrow tiles, converted by cvt).
+int run_stages(const Problem &p, int run_bits) {
     const int64_t ax = p.zx >= 0 ? 128 + p.zx : 127 - p.zx;
     const int64_t aw = p.zw ? 255 : 128;
-    int64_t len = (((int64_t)1 << 22) - 1) / (ax * aw);
+    int64_t len = (((int64_t)1 << run_bits) - 1) / (ax * aw);
     len = len / KS;
     return len < 1 ? 1 : (int)len;
 }
@@ -812,7 +821,7 @@ int launch_group(const Problem *const *probs, const bool *part, int n, bool o16,
     for (int i = 0; i < n; ++i) {
         Problem &q = P.p[i];
         q = *probs[i];
-        P.kpr[i] = run_stages(q);
+        P.kpr[i] = run_stages(q, Cfg<NARROW>::RUN_BITS);
         P.tn[i] = Cfg<NARROW>::TN;
         q.tiles_m = (q.M + TMT - 1) / TMT;
         q.tile_begin = (int)tiles;
@@ -886,7 +895,7 @@ int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *
         for (int i = 0; i <= count; ++i) {
             if (i < count) {
                 const Problem &q = probs[i];
-                const bool wide = (q.K + KS - 1) / KS <= run_stages(q) && q.N > TNN;
+                const bool wide = (q.K + KS - 1) / KS <= run_stages(q, 22) && q.N > TNN;
                 if (wide == (narrow == 0)) {
                     lpart[n] = part && part[i];
                     list[n++] = &q;
