@@ -75,14 +75,15 @@ constexpr uint32_t TMEM_COLS = 512;  // F[b] at column 256 b
 
 // The two tile shapes, each its own kernel.  Wide: 256 channels, one stage
 // per tile (the scores): a short pipeline, 16 epilogue warps for the
-// requantization.  Narrow: 64 channels over many stages (long K): six
-// staging stages, four operand slots and two converter groups taking
-// alternate stages (each group's waits and signals overlap the other's
-// widening), four epilogue warps.
+// requantization.  Narrow: 64 channels over many stages (long K): eight
+// staging stages (the loads of P's 64-byte row segments take ~2 us to land),
+// four operand slots and two converter groups taking alternate stages (each
+// group's waits and signals overlap the other's widening), four epilogue
+// warps.
 template <bool NARROW>
 struct Cfg {
     static constexpr int TN = NARROW ? TNN : TNW;
-    static constexpr int S8 = NARROW ? 6 : 2;  // staging stages
+    static constexpr int S8 = NARROW ? 8 : 2;  // staging stages
     static constexpr int SF = NARROW ? 4 : 2;  // operand slots
     static constexpr int GROUPS = NARROW ? 2 : 1;
     static constexpr int EPI_WARP0 = CONV_WARP0 + GROUPS * GROUP_WARPS;
