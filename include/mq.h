@@ -385,7 +385,7 @@ typedef struct mq_linear_desc {
  * kernel.  The required part also holds, for descriptors without colsum that
  * the token-major kernel does not serve, their weights' row sums (4 N bytes,
  * rounded up to 128, per distinct weight matrix).  Last, optionally, the
- * split-K partial sums of the call's small prefill descriptors (see
+ * split-K partial sums, for a call made only of small prefill descriptors (see
  * mq_workspace_size; S is shared by the call, from all of them).  0 when none
  * applies.  The decode region (the first
  * mq_workspace_size(1, 1, 0, 4) bytes) follows the contract of

@@ -292,24 +292,29 @@ Plan batch_plan(const mq_linear_desc *descs, int count) {
     // + 1024: the region starts at the first 1024-byte boundary after wide_at()
     pl.bytes = pl.wide.empty() ? pl.required : wide_at(pl) + woff + 1024;
     pl.bytes_wide = pl.bytes;
-    // Split K: prefill calls whose tiles would leave most SMs idle (one M = 128
-    // linear makes 8 pair tiles for 76 pairs) run their problems as S slices
-    // of K on the token-major kernel, each writing its raw int32 sums, then one
-    // combine launch requantizes.  S = SMs / (the token-major tiles of the
-    // call), at most 8, each slice at least 256 k; only with the choice of
-    // prefill kernel left automatic, and only when the workspace has room
-    // (optional, like the widened inputs).
+    // Split K: a call made only of prefill problems whose tiles would leave
+    // most SMs idle (one M = 128 linear makes 8 pair tiles for 76 pairs) runs
+    // them as S slices of K on the token-major kernel, each writing its raw
+    // int32 sums, then one combine launch requantizes.  S = SMs / (the
+    // token-major tiles of the call), at most 8, each slice at least 256 k;
+    // only with the choice of prefill kernel left automatic, and only when the
+    // workspace has room (optional, like the widened inputs).
     if (mq::test_prefill_kernel() == 0) {
         long long tiles = 0;
         int kmin = 1 << 30;
+        bool all = true;  // only calls made of such problems alone
         for (int i = 0; i < count; ++i) {
             const mq_linear_desc &d = descs[i];
-            if (!split_candidate(d)) continue;
+            if (d.M <= 0 || d.N <= 0) continue;
+            if (!split_candidate(d)) {
+                all = false;
+                continue;
+            }
             tiles += (long long)((d.M + 127) / 128) * ((d.N + 63) / 64);
             kmin = d.K < kmin ? d.K : kmin;
             pl.ks_idx.push_back(i);
         }
-        const int sms = device_sms();
+        const int sms = all ? device_sms() : 0;
         long long S = tiles > 0 ? sms / tiles : 0;
         if (S > 8) S = 8;
         if (S > kmin / 256) S = kmin / 256;

@@ -838,7 +838,9 @@ int launch_group(const Problem *const *probs, const bool *part, int n, bool o16,
         P.vec[i] = al16(q.y) && ((size_t)q.ldy * osz) % 16 == 0 &&
                    (!q.residual || al16(q.residual));
         P.part[i] = part[i] ? 1 : 0;
-        P.tma_y[i] = P.vec[i] && !q.residual && !part[i];
+        // a TMA store clips the box at the tensor's edge only in whole 16-byte
+        // chunks of the inner dimension, so it serves rows of 16-byte multiples
+        P.tma_y[i] = P.vec[i] && !q.residual && !part[i] && ((size_t)q.N * osz) % 16 == 0;
         if (P.tma_y[i] &&
             !encode(&P.tmap_y[i], q.y, (uint64_t)q.N, (uint64_t)q.M, (uint64_t)q.ldy * osz, 64, 32,
                     osz, o16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))

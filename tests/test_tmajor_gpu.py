@@ -147,6 +147,20 @@ def test_tmajor_scalar_store_path(o16):
     assert (pad == 77).all(), "bytes past N written"
 
 
+@pytest.mark.parametrize("o16", [False, True], ids=["int8", "int16"])
+@pytest.mark.parametrize("n", [100, 50])
+def test_tmajor_row_tail_untouched(n, o16):
+    # N * size not a multiple of 16 with rows that are: the bytes between N
+    # and the row pitch stay untouched (a TMA store would clip only in whole
+    # 16-byte chunks, so such rows take the per-element tail)
+    m, k = 140, 256
+    pad = (-n) % 16 + 16
+    c = Case(61 + n, m, k, n, zw=True, o16=o16, pad_y=pad)
+    run([c])
+    assert_equal(c.got(), c.want(), f"tail n={n} o16={o16}")
+    assert (c.y.cpu().numpy()[:, n:] == 77).all(), "bytes past N written"
+
+
 @pytest.mark.parametrize("extreme", ["min", "max", "mixed"])
 @pytest.mark.parametrize("shape", [(130, 300, 1024), (70, 64, 2048)],
                          ids=lambda s: "x".join(map(str, s)))
