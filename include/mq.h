@@ -640,8 +640,9 @@ int mq_test_prefill_kernel(int which);
  * row pitches that are multiples of 16 bytes, and no residual with an int16
  * output.  0 (the initial state) takes it for such problems with K <= 128 or
  * N <= 64 (the attention matmuls: Q K^T at head dimension K, P V with head
- * dimension N), 1 for every such problem, 2 never.  All kernels are
- * bit-exact; the hook lets the tests run each one on any shape.
+ * dimension N) unless mq_test_prefill_kernel forces the 256-token kernel, 1
+ * for every such problem, 2 never.  All kernels are bit-exact; the hook lets
+ * the tests run each one on any shape.
  * Errors: MQ_ERR_INVALID_ARG for values other than 0, 1, 2.
  */
 int mq_test_tmajor_kernel(int which);

@@ -196,6 +196,8 @@ bool routes_tmajor(const mq_linear_desc &d, const mq::Problem &p) {
     if (is_decode(d)) return false;
     const int mode = mq::test_tmajor_kernel();
     if (mode == 2 || !mq::tmajor_suits(p)) return false;
+    // a forced 256-token kernel (test hook) comes before the automatic choice
+    if (mode == 0 && mq::test_prefill_kernel() == 1) return false;
     return mode == 1 || p.K <= 128 || p.N <= 64;
 }
 
