@@ -397,3 +397,45 @@ def test_descriptor_layout_matches_the_header(mq, tmp_path, struct):
     for f in fields:
         assert int(out[f]) == getattr(cls, f).offset, f
     assert int(out["sizeof"]) == ctypes.sizeof(cls)
+
+
+def test_colsum_optional_with_int8_weights(mq):
+    # colsum may be omitted with int8 weights: no workspace where the
+    # token-major kernel serves (it folds both zero points), the weights' row
+    # sums (4 N bytes, to 128, once per distinct weight matrix) elsewhere;
+    # int4 weights and the single-linear calls still require it
+    def no_colsum(d):
+        d.colsum = None
+        return d
+    short_k = no_colsum(_desc(mq, 300, 64, 200, 8, True))    # token-major: K <= 128
+    long_k = no_colsum(_desc(mq, 300, 512, 200, 8, True))    # 128-token kernel
+    assert mq.workspace_size_batch([short_k]) == 0
+    assert mq.workspace_size_batch([long_k]) == 4 * 200 + (-4 * 200) % 128
+    shared = no_colsum(_desc(mq, 100, 512, 200, 8, False))   # the same weights (FAKE)
+    assert mq.workspace_size_batch([long_k, shared]) == 4 * 200 + (-4 * 200) % 128
+    dec = mq.workspace_size(1, 1, 0, 4)
+    decode = no_colsum(_desc(mq, 4, 512, 200, 8, False))
+    assert mq.workspace_size_batch([decode]) == dec + 896
+    assert mq.test_tmajor_kernel(2) == 0                     # forbidden: row sums needed
+    try:
+        assert mq.workspace_size_batch([short_k]) == 896
+    finally:
+        assert mq.test_tmajor_kernel(0) == 0
+    # int4 weights without colsum: rejected before anything is launched
+    bad = (mq.LinearDesc * 1)(no_colsum(_desc(mq, 300, 512, 200, 4, False)))
+    assert mq.lib.mq_linear_batch(bad, 1, FAKE, 1 << 30, None) == mq.MQ_ERR_INVALID_ARG
+    # the single-linear calls: colsum required
+    assert mq.lib.mq_linear_w8a8(FAKE, 64, 512, 512, 0, FAKE, None, 32, FAKE, FAKE, 0, FAKE, 32,
+                                 FAKE, 1 << 30, None) == mq.MQ_ERR_INVALID_ARG
+
+
+def test_fold_batch_argument_checks_on_host(mq):
+    # count limits and an empty batch, before anything is launched
+    many = (mq.FoldDesc * (mq.MQ_FOLD_MAX_JOBS + 1))()
+    assert mq.lib.mq_fold_quantize_pack_batch(many, mq.MQ_FOLD_MAX_JOBS + 1, None) == \
+        mq.MQ_ERR_INVALID_ARG
+    assert mq.lib.mq_fold_quantize_pack_batch(None, 0, None) == 0
+    assert mq.lib.mq_fold_quantize_pack_batch(None, 1, None) == mq.MQ_ERR_INVALID_ARG
+    bad = mq.FoldDesc(FAKE, 16, 63, None, None, 4, 0, FAKE, FAKE, FAKE, None, FAKE)  # int4, odd K
+    assert mq.lib.mq_fold_quantize_pack_batch((mq.FoldDesc * 1)(bad), 1, None) == \
+        mq.MQ_ERR_INVALID_ARG
