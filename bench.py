@@ -611,8 +611,10 @@ class AttentionSet:
     """Device operands and batched descriptors of one layer's attention matmuls
     (TinyLlama: 32 query heads over 4 KV heads, head dim 64, T tokens):
     S_h = Q_h K_g^T (int8 in, int16 scores, keys as the weights read through a
-    row pitch, asymmetric per tensor: zw = zk) and O_h = P_h V_g (int8, V_g^T as
-    the weights, zw = zv), O written into head h's columns of [T][32 * 64].
+    row pitch, asymmetric per tensor: zw = zk) and O_h = P_h V_g (int8, V_g read
+    in place as transposed weights [T][64] through V's row pitch, zw = zv; in
+    the 16-bit setting V^T, made by one transpose launch), O written into head
+    h's columns of [T][32 * 64].
     Both read weights written on the device in the same stream (wdynamic), and
     leave the weights' row sums to the calls (colsum omitted: the token-major
     kernel needs none; the 16-bit setting's kernels get them computed inside
@@ -636,8 +638,9 @@ class AttentionSet:
         self.q, self.k, self.v, self.p = up(a.q), up(a.k), up(a.v), up(a.p)
         self.s = torch.empty((H, t, t), dtype=torch.int16, device=dev)
         self.o = torch.empty((t, H * D), dtype=torch.int16 if bits16 else torch.int8, device=dev)
-        # V^T of all heads at once [G d][T] (head g is rows g d .. g d + d - 1)
-        self.vt = torch.empty((G * D, t), dtype=torch.int8, device=dev)
+        # 16-bit setting: V^T of all heads at once [G d][T] (head g is rows g d ..
+        # g d + d - 1); with 8-bit P the token-major kernel reads V itself
+        self.vt = torch.empty((G * D, t), dtype=torch.int8, device=dev) if bits16 else None
         i32 = lambda n, v: up(np.full(n, v, np.int32))
         self.keep = [i32(t, self.M0_S), i32(t, self.SH_S), i32(t, a.zk),
                      i32(D, self.M0_O), i32(D, self.SH_O), i32(D, a.zv)]
@@ -646,10 +649,15 @@ class AttentionSet:
         ds = [mq.make_desc(self.q[:, h * D:(h + 1) * D], a.zq, self.k[:, (h // rep) * D:],
                            None, t, m0s, shs, self.ZY_S, self.s[h], 8, zw=zwk,
                            ldw=G * D, wdynamic=True) for h in range(H)]
-        vt_g = lambda g: self.vt[g * D:(g + 1) * D]
-        do = [mq.make_desc(self.p[h], a.zp, vt_g(h // rep), None, D, m0o, sho,
-                           self.ZY_O, self.o[:, h * D:(h + 1) * D], 8, zw=zwv, wdynamic=True)
-              for h in range(H)]
+        if bits16:
+            vt_g = lambda g: self.vt[g * D:(g + 1) * D]
+            do = [mq.make_desc(self.p[h], a.zp, vt_g(h // rep), None, D, m0o, sho,
+                               self.ZY_O, self.o[:, h * D:(h + 1) * D], 8, zw=zwv,
+                               wdynamic=True) for h in range(H)]
+        else:
+            do = [mq.make_desc(self.p[h], a.zp, self.v[:, (h // rep) * D:], None, D, m0o, sho,
+                               self.ZY_O, self.o[:, h * D:(h + 1) * D], 8, zw=zwv,
+                               ldw=G * D, wdynamic=True, wt=True) for h in range(H)]
         self.arr_s = (mq.LinearDesc * H)(*ds)
         self.arr_o = (mq.LinearDesc * H)(*do)
         self.ws_s_bytes = mq.workspace_size_batch(ds)
@@ -668,8 +676,9 @@ class AttentionSet:
             rcs.append(lib.mq_linear_batch(self.arr_s, H, self.ws_s.data_ptr(), self.ws_s_bytes,
                                            sp))
         if phase in ("all", "pv"):
-            rcs.append(lib.mq_transpose_i8(self.v.data_ptr(), t, G * D, G * D, self.vt.data_ptr(),
-                                           t, sp))
+            if self.vt is not None:
+                rcs.append(lib.mq_transpose_i8(self.v.data_ptr(), t, G * D, G * D,
+                                               self.vt.data_ptr(), t, sp))
             rcs.append(lib.mq_linear_batch(self.arr_o, H, self.ws_o.data_ptr(), self.ws_o_bytes,
                                            sp))
         if any(rcs):
@@ -706,9 +715,10 @@ def run_attention(mq, torch, reps: int = 60, check_rows: int = 4, bits16: bool =
     """Grouped-query attention's two integer matmuls of one TinyLlama layer at
     T = 1024 (the softmax between them is outside the integer layer): per step
     S = Q K^T for 32 heads (one batched call, one token-major kernel launch,
-    int16 scores, the keys' zero point folded in: no row sums), V^T of all heads
-    (one transpose), and O = P V for 32 heads (one batched call; in the 16-bit
-    setting each call also computes its weights' row sums).  Steps rotate over three
+    int16 scores, the keys' zero point folded in: no row sums) and O = P V for
+    32 heads (one batched call reading V in place; in the 16-bit setting V^T of
+    all heads by one transpose first, and each call also computes its weights'
+    row sums).  Steps rotate over three
     layers' operands (about 300 MB, more than L2).  The host enqueues the timed
     steps behind a device sleep, so the region measures the device, not the
     ctypes call rate; a second pass times the two phases alone."""
@@ -1361,6 +1371,8 @@ def run_profile_leg(mq, torch, dist, args):
         per = r["us_per_step"] * 1e-3
     print(f"profile leg {args.profile}: {per:.4f} ms per step ({time.time() - t0:.1f} s)",
           flush=True)
+    scalars = {k: v for k, v in r.items() if isinstance(v, (int, float, str))}
+    print(json.dumps(scalars), flush=True)
 
 
 def main():

@@ -305,6 +305,15 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
  * mq_workspace_size_batch; rounded up to 128 bytes).  For weights written on
  * the device every call (keys, V^T in attention) this replaces a separate
  * row-sum launch.  The single-linear calls still require colsum.
+ * Transposed weights (`wt`, int8 weights with 8-bit activations): `packed`
+ * holds w[n][k] at packed[k * ldw + n], i.e. an activation matrix [K][N] such
+ * as V in attention's P V (its head-g columns with ldw = the row pitch of V),
+ * read without a transpose.  Only the token-major kernel reads this layout:
+ * such a descriptor must be a prefill shape (M > 16) that kernel can serve (x
+ * and packed 16-byte aligned, ldx and ldw multiples of 16, no residual with an
+ * int16 output); otherwise, or with the token-major kernel forbidden
+ * (mq_test_tmajor_kernel), the call returns MQ_ERR_UNSUPPORTED_SHAPE before
+ * anything is launched.  colsum is not read (the kernel folds the zero points).
  * Weights written on the device: the kernels read `packed` before waiting for
  * the previous kernel in the stream (see mq_linear_w8a8).  A descriptor whose
  * weights are produced by earlier work on the same stream (keys, or V^T from
@@ -336,6 +345,8 @@ typedef struct mq_linear_desc {
     const void *x16;    /* may be NULL: device f16 [M][K], an f16 copy of x (a y16 of an earlier
                            call), see below */
     const int32_t *xsq; /* with x16: device int32 [M], sum_k x[m][k]^2 (that call's ysq) */
+    int32_t wt;         /* nonzero: packed holds the weights transposed, int8 [K][N] with
+                           `ldw` bytes between k-rows (0: N), see below */
 } mq_linear_desc;
 
 /*

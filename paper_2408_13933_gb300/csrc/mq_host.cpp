@@ -52,7 +52,10 @@ int check_desc(const mq_linear_desc &d, mq::Problem &out) {
     if (d.zx < zlo || d.zx > zhi || d.zy < ylo || d.zy > yhi) return MQ_ERR_INVALID_ARG;
     if (ab == 16 && d.residual) return MQ_ERR_INVALID_ARG;
     if (ob == 16 && d.residual) return MQ_ERR_INVALID_ARG;
-    const int64_t wrow = (int64_t)d.K * d.bits / 8;  // packed bytes of one weight row
+    // transposed weights: int8 [K][N] beside 8-bit activations
+    if (d.wt && (d.bits != 8 || ab != 8)) return MQ_ERR_INVALID_ARG;
+    // packed bytes of one weight row (of one k-row when transposed)
+    const int64_t wrow = d.wt ? (int64_t)d.N : (int64_t)d.K * d.bits / 8;
     if (d.ldw < 0 || (d.ldw > 0 && d.ldw < wrow)) return MQ_ERR_INVALID_ARG;
     if (d.ldw % 16 != 0) return MQ_ERR_ALIGNMENT;
     if (d.K > MQ_MAX_K) return MQ_ERR_K_OVERFLOW;
@@ -130,7 +133,7 @@ constexpr int WIDE_MIN_N = 256;
 // workspace has room for its widened input: a tensor-core shape with 8-bit
 // activations and output.
 bool wide_eligible(const mq_linear_desc &d) {
-    if (d.M <= 0 || d.N <= 0 || d.K <= 0 || is_decode(d)) return false;
+    if (d.M <= 0 || d.N <= 0 || d.K <= 0 || is_decode(d) || d.wt) return false;
     if (abits_of(d) != 8 || obits_of(d) != 8) return false;
     const int which = mq::test_prefill_kernel();
     if (which == 2) return false;
@@ -196,6 +199,7 @@ bool routes_tmajor(const mq_linear_desc &d, const mq::Problem &p) {
     if (is_decode(d)) return false;
     const int mode = mq::test_tmajor_kernel();
     if (mode == 2 || !mq::tmajor_suits(p)) return false;
+    if (d.wt) return true;  // transposed weights: this kernel alone reads them
     // a forced 256-token kernel (test hook) comes before the automatic choice
     if (mode == 0 && mq::test_prefill_kernel() == 1) return false;
     return mode == 1 || p.K <= 128 || p.N <= 64;
@@ -226,7 +230,7 @@ int device_sms() {
 // would serve with few tiles (M < 256 or N < 256), 8-bit activations and
 // weights, long enough K, and a shape the token-major kernel can take.
 bool split_candidate(const mq_linear_desc &d) {
-    if (d.M <= 0 || d.N <= 0 || d.K < 512 || is_decode(d) || d.y16) return false;
+    if (d.M <= 0 || d.N <= 0 || d.K < 512 || is_decode(d) || d.y16 || d.wt) return false;
     if (abits_of(d) != 8 || d.bits != 8 || (d.M >= WIDE_MIN_M && d.N >= WIDE_MIN_N)) return false;
     mq::Problem p{};
     if (check_desc(d, p) != MQ_OK) return false;
@@ -343,6 +347,10 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
     for (int i = 0; i < count; ++i) {
         const int rc = check_desc(descs[i], probs[i]);
         if (rc != MQ_OK) return rc;
+        // transposed weights are read by the token-major kernel alone
+        const mq_linear_desc &d = descs[i];
+        if (d.wt && d.M > 0 && d.N > 0 && d.K > 0 && !routes_tmajor(d, probs[i]))
+            return MQ_ERR_UNSUPPORTED_SHAPE;
     }
     // the decode kernel combines split 64-row units in the workspace, 16-bit
     // tensor-core descriptors read their int8 planes from there
@@ -381,6 +389,7 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
         }
     }
     std::vector<mq::Problem> tmaj[2];  // by o16
+    std::vector<uint8_t> tmaj_wt[2];   // their transposed-weights flags
     std::vector<mq::Problem> pre2;
     std::vector<const uint16_t *> pre2_x16;
     std::vector<const int32_t *> pre2_rowsq;
@@ -451,6 +460,7 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
             dec[p.bits == 8][mode].push_back(p);
         } else if (routes_tmajor(d, p)) {
             tmaj[p.o16 ? 1 : 0].push_back(p);
+            tmaj_wt[p.o16 ? 1 : 0].push_back(d.wt ? 1 : 0);
             if (d.y16) after.push_back(output_copy_job(d));
         } else if (takes_wide(d)) {
             pre2.push_back(p);
@@ -486,7 +496,8 @@ int run_batch(const mq_linear_desc *descs, int count, void *workspace, size_t ws
     }
     for (int o = 0; o < 2; ++o)
         if (rc == MQ_OK && !tmaj[o].empty())
-            rc = mq::launch_tmajor(tmaj[o].data(), (int)tmaj[o].size(), stream);
+            rc = mq::launch_tmajor(tmaj[o].data(), (int)tmaj[o].size(), stream, nullptr,
+                                   tmaj_wt[o].data());
     if (rc == MQ_OK && !ksub.empty()) {
         rc = mq::launch_tmajor(ksub.data(), (int)ksub.size(), stream, ksub_part.data());
         if (rc == MQ_OK) rc = mq::launch_splitk_reduce(kred.data(), (int)kred.size(), stream);

@@ -31,6 +31,12 @@
 // epilogue requantizes each tile straight out of tensor memory), else TN = 64
 // (with several runs each epilogue thread keeps 64 running int32 sums).
 //
+// Transposed weights (w stored [K][N], e.g. attention's V read in place for
+// P V): narrow tiles only.  TMA stages 64 k-rows x 64 channels; the
+// converters widen them row by row into an f16 tile with channels contiguous
+// (128-byte swizzled, N-major), which the MMA reads as an N-major B operand,
+// so no transpose is made anywhere.
+//
 // Warp roles (one CTA per SM, persistent over a contiguous range of tiles):
 //   warp 0      TMA producer (one thread)
 //   warp 1      tensor-memory allocation, MMA issue (one elected lane)
@@ -172,6 +178,8 @@ struct Params {
     int vec[PREFILL_MAX_PROBLEMS];              // y (and residual) rows allow 16-byte accesses
     int tma_y[PREFILL_MAX_PROBLEMS];            // y written by TMA stores (vec, no residual)
     int part[PREFILL_MAX_PROBLEMS];             // y is int32 [M][ldy]: raw sums of a slice of K
+    int wt[PREFILL_MAX_PROBLEMS];               // w stored [K][ldw] (narrow tiles); tmap_w: box
+                                                // 64 channels x 64 k
     int count;
     int total_tiles;
     int *status;
@@ -271,6 +279,49 @@ __device__ __forceinline__ void widen_chunk(const uint8_t *src, uint8_t *dst, in
     }
     *reinterpret_cast<uint4 *>(dst + sw128(r, 2 * c)) = make_uint4(h[0], h[1], h[2], h[3]);
     *reinterpret_cast<uint4 *>(dst + sw128(r, 2 * c + 1)) = make_uint4(h[4], h[5], h[6], h[7]);
+}
+
+// The weights' offsets of one staged [K][N] chunk (16 channels ch0 .. ch0 +
+// 15, one k): off[e] holds channels ch0 + 2e (low half) and ch0 + 2e + 1
+// (high half), 1152 + zw, or 1152 without a zero point or past N.
+template <int NOFF>
+__device__ __forceinline__ void wt_offsets(const Problem &p, int ch0, uint32_t (&off)[NOFF]) {
+    static_assert(NOFF >= 8, "eight channel pairs");
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        uint32_t lo = 0x6480u, hi = 0x6480u;
+        const int ch = ch0 + 2 * e;
+        if (p.zw && ch < p.N) lo = (uint32_t)(0x6480 + __ldg(p.zw + ch));
+        if (p.zw && ch + 1 < p.N) hi = (uint32_t)(0x6480 + __ldg(p.zw + ch + 1));
+        off[e] = (hi << 16) | lo;
+    }
+}
+
+// 16 int8 of one k (channels of one staged [K][N] chunk) -> 16 f16 (w - zw
+// per channel, offsets from wt_offsets) into chunks 2c and 2c + 1 of row r of
+// the N-major tile (the same 128-byte swizzle, rows now along k).
+template <int NOFF>
+__device__ __forceinline__ void widen_chunk_pairs(const uint8_t *src, uint8_t *dst, int r, int c,
+                                                  const uint32_t (&off)[NOFF]) {
+    const uint4 v = *reinterpret_cast<const uint4 *>(src);
+    const uint32_t q[4] = {v.x, v.y, v.z, v.w};
+    uint32_t h[8];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const uint32_t u = q[e] ^ 0x80808080u;
+        h[2 * e] = hsub2(prmt(u, 0x64646464u, 0x4140u), off[2 * e]);
+        h[2 * e + 1] = hsub2(prmt(u, 0x64646464u, 0x4342u), off[2 * e + 1]);
+    }
+    *reinterpret_cast<uint4 *>(dst + sw128(r, 2 * c)) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4 *>(dst + sw128(r, 2 * c + 1)) = make_uint4(h[4], h[5], h[6], h[7]);
+}
+
+// Shared-memory descriptor of an N-major operand in 128-byte swizzle atoms
+// (8 k-rows of 64 f16 channels, 1024 B): atoms along k 1024 B apart (the
+// stride field); along N (the leading field) there is one atom in a 64-channel
+// tile, given 1024 B as well.
+__device__ __forceinline__ uint64_t smem_desc_sw128_nmajor(uint32_t saddr) {
+    return (smem_desc_sw128(saddr) & ~(0x3FFFull << 16)) | ((uint64_t)(1024u >> 4) << 16);
 }
 
 // An f32 accumulator holding an integer v with |v| < 2^22 -> v: adding
@@ -454,7 +505,8 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
         s.prob[i] = P.p[i];
         s.tn[i] = P.tn[i];
         s.kpr[i] = P.kpr[i];
-        s.flags[i] = (P.vec[i] ? 1 : 0) | (P.tma_y[i] ? 2 : 0) | (P.part[i] ? 4 : 0);
+        s.flags[i] = (P.vec[i] ? 1 : 0) | (P.tma_y[i] ? 2 : 0) | (P.part[i] ? 4 : 0) |
+                     (NARROW && P.wt[i] ? 8 : 0);
     }
     if (threadIdx.x == 0) {
         for (int i = 0; i < S8; ++i) {
@@ -510,8 +562,12 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                     mbar_arrive_expect_tx(&s.ld_full[slot], bytes);
                     tma_load_2d(s.stx[slot], &P.tmap_x[t.pi], kb * KS, t.tt * TMT,
                                 &s.ld_full[slot]);
-                    tma_load_2d(s.stw[slot], &P.tmap_w[t.pi], kb * KS, t.ct * t.tn,
-                                &s.ld_full[slot]);
+                    if (s.flags[t.pi] & 8)  // [K][N]: x = channel, y = k
+                        tma_load_2d(s.stw[slot], &P.tmap_w[t.pi], t.ct * t.tn, kb * KS,
+                                    &s.ld_full[slot]);
+                    else
+                        tma_load_2d(s.stw[slot], &P.tmap_w[t.pi], kb * KS, t.ct * t.tn,
+                                    &s.ld_full[slot]);
                 }
             }
             if (!ok) {
@@ -531,7 +587,11 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
         bool ok = true;
         for (int tile = tile0; ok && tile < tile1; ++tile) {
             const Tile t = tile_of(s, P.count, tile);
-            const uint32_t idesc = idesc_f16_f32(TMT, t.tn);
+            const bool wt = (s.flags[t.pi] & 8) != 0;
+            // an N-major B (transposed weights): the "transpose B" bit; its
+            // 16-k steps are 16 rows of 128 bytes, 2048 B (+128 in addr >> 4)
+            const uint32_t idesc = idesc_f16_f32(TMT, t.tn) | (wt ? 1u << 16 : 0u);
+            const uint32_t bstep = wt ? 128u : 2u;
             int kr = 0;  // stage within the exact run
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                 const bool run_start = kr == 0;
@@ -549,10 +609,11 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                 const bool run_end = ++kr == t.kpr || kb + 1 == t.nkb;
                 if (elect_one()) {
                     const uint64_t ad = smem_desc_sw128(smem_u32(s.opa[slot]));
-                    const uint64_t bd = smem_desc_sw128(smem_u32(s.opb[slot]));
+                    const uint64_t bd = wt ? smem_desc_sw128_nmajor(smem_u32(s.opb[slot]))
+                                           : smem_desc_sw128(smem_u32(s.opb[slot]));
 #pragma unroll
                     for (int j = 0; j < KS / 16; ++j)  // +32 B along K: +2 in the (addr >> 4) field
-                        mma_f16_ss(tmem + (uint32_t)C::TN * b, ad + 2 * j, bd + 2 * j, idesc,
+                        mma_f16_ss(tmem + (uint32_t)C::TN * b, ad + 2 * j, bd + bstep * j, idesc,
                                    (run_start && j == 0) ? 0u : 1u);
                     commit1(&s.op_empty[slot]);
                     if (run_end) commit1(&s.f_full[b]);
@@ -584,12 +645,20 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
             const uint32_t xoff = f16x2_i8_offset(p.zx);
             // the weight rows this thread widens: r = ct / 4 + 32 u
             const int wchunks = t.tn * (KS / 16);  // 16-byte chunks of the staged w
-            uint32_t woff[C::TN / 32];
+            uint32_t woff[C::TN / 32 > 8 ? C::TN / 32 : 8];  // >= 8 for wt_offsets
+            const bool wt = NARROW && (s.flags[t.pi] & 8) != 0;
+            if (wt) {
+                // [K][N] staging: this thread's chunks are channels 16 (ct % 4) ..
+                // + 15 of every row; one offset per channel pair
+                wt_offsets(p, t.ct * t.tn + 16 * (ct & 3), woff);
+            } else {
 #pragma unroll
-            for (int u = 0; u < C::TN / 32; ++u) {
-                const int ch = t.ct * t.tn + (ct >> 2) + 32 * u;
-                woff[u] = F16X2_1152;
-                if (p.zw && 32 * u < t.tn && ch < p.N) woff[u] = f16x2_i8_offset(__ldg(p.zw + ch));
+                for (int u = 0; u < C::TN / 32; ++u) {
+                    const int ch = t.ct * t.tn + (ct >> 2) + 32 * u;
+                    woff[u] = F16X2_1152;
+                    if (p.zw && 32 * u < t.tn && ch < p.N)
+                        woff[u] = f16x2_i8_offset(__ldg(p.zw + ch));
+                }
             }
             for (int kb = 0; kb < t.nkb; ++kb, ++it) {
                 if ((int)(it % C::GROUPS) != grp) continue;  // the other group's stage
@@ -608,10 +677,21 @@ __global__ void __launch_bounds__(Cfg<NARROW>::THREADS, 1)
                     widen_chunk(s.stx[s8] + 16 * i, s.opa[sf], i >> 2, i & 3, xoff,
                                 live < 0 ? 0 : (live > 16 ? 16 : live));
                 }
+                if (wt) {
+                    // row r of the staging = k r, chunk c = channels 16 c .. + 15: the
+                    // f16 tile's row r, chunks 2c and 2c + 1 (N-major)
 #pragma unroll
-                for (int u = 0; u < (C::TN * KS / 16) / GROUP_THREADS; ++u) {
-                    const int i = ct + GROUP_THREADS * u;
-                    if (i < wchunks) widen_chunk(s.stw[s8] + 16 * i, s.opb[sf], i >> 2, i & 3, woff[u]);
+                    for (int u = 0; u < (C::TN * KS / 16) / GROUP_THREADS; ++u) {
+                        const int i = ct + GROUP_THREADS * u;
+                        widen_chunk_pairs(s.stw[s8] + 16 * i, s.opb[sf], i >> 2, i & 3, woff);
+                    }
+                } else {
+#pragma unroll
+                    for (int u = 0; u < (C::TN * KS / 16) / GROUP_THREADS; ++u) {
+                        const int i = ct + GROUP_THREADS * u;
+                        if (i < wchunks)
+                            widen_chunk(s.stw[s8] + 16 * i, s.opb[sf], i >> 2, i & 3, woff[u]);
+                    }
                 }
                 fence_proxy_async_smem();  // the f16 tiles, for the tensor core's reads
                 __syncwarp();
@@ -813,8 +893,8 @@ namespace tmajor {
 
 // One launch of up to PREFILL_MAX_PROBLEMS problems of one tile shape.
 template <bool NARROW>
-int launch_group(const Problem *const *probs, const bool *part, int n, bool o16, int sms,
-                 cudaStream_t stream) {
+int launch_group(const Problem *const *probs, const bool *part, const bool *wt, int n, bool o16,
+                 int sms, cudaStream_t stream) {
     const auto al16 = [](const void *v) { return (reinterpret_cast<uintptr_t>(v) & 15u) == 0; };
     const int osz = o16 ? 2 : 1;
     Params P{};
@@ -827,10 +907,17 @@ int launch_group(const Problem *const *probs, const bool *part, int n, bool o16,
         q.tiles_m = (q.M + TMT - 1) / TMT;
         q.tile_begin = (int)tiles;
         tiles += (long long)q.tiles_m * ((q.N + P.tn[i] - 1) / P.tn[i]);
+        P.wt[i] = NARROW && wt[i] ? 1 : 0;
+        if (!NARROW && wt[i]) return MQ_ERR_UNSUPPORTED_SHAPE;
+        const bool wmap = P.wt[i] ? encode(&P.tmap_w[i], q.w, (uint64_t)q.N, (uint64_t)q.K,
+                                           (uint64_t)q.ldw, (uint32_t)P.tn[i], KS, 1,
+                                           CU_TENSOR_MAP_SWIZZLE_NONE)
+                                  : encode(&P.tmap_w[i], q.w, (uint64_t)q.K, (uint64_t)q.N,
+                                           (uint64_t)q.ldw, KS, (uint32_t)P.tn[i], 1,
+                                           CU_TENSOR_MAP_SWIZZLE_NONE);
         if (!encode(&P.tmap_x[i], q.x, (uint64_t)q.K, (uint64_t)q.M, (uint64_t)q.ldx, KS, TMT, 1,
                     CU_TENSOR_MAP_SWIZZLE_NONE) ||
-            !encode(&P.tmap_w[i], q.w, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldw, KS,
-                    (uint32_t)P.tn[i], 1, CU_TENSOR_MAP_SWIZZLE_NONE))
+            !wmap)
             return MQ_ERR_CUDA;
         // 16-byte stores where y's rows (and the residual's) allow them;
         // without a residual, TMA stores of blocks of 32 tokens x 64 channels
@@ -869,7 +956,8 @@ int launch_group(const Problem *const *probs, const bool *part, int n, bool o16,
 
 }  // namespace tmajor
 
-int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *part) {
+int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *part,
+                  const uint8_t *wt) {
     using namespace tmajor;
     static std::atomic<uint64_t> attr_done{0};  // bit d: device d prepared
     int dev = 0;
@@ -891,22 +979,25 @@ int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const bool o16 = probs[0].o16 != 0;
     // wide tiles where K fits one exact run and N > 64, narrow ones otherwise
+    // (and for transposed weights)
     for (int narrow = 0; narrow < 2; ++narrow) {
         const Problem *list[PREFILL_MAX_PROBLEMS];
-        bool lpart[PREFILL_MAX_PROBLEMS];
+        bool lpart[PREFILL_MAX_PROBLEMS], lwt[PREFILL_MAX_PROBLEMS];
         int n = 0;
         for (int i = 0; i <= count; ++i) {
             if (i < count) {
                 const Problem &q = probs[i];
-                const bool wide = (q.K + KS - 1) / KS <= run_stages(q, 22) && q.N > TNN;
+                const bool t = wt && wt[i];
+                const bool wide = !t && (q.K + KS - 1) / KS <= run_stages(q, 22) && q.N > TNN;
                 if (wide == (narrow == 0)) {
                     lpart[n] = part && part[i];
+                    lwt[n] = t;
                     list[n++] = &q;
                 }
             }
             if (n == PREFILL_MAX_PROBLEMS || (i == count && n > 0)) {
-                const int rc = narrow ? launch_group<true>(list, lpart, n, o16, sms, st)
-                                      : launch_group<false>(list, lpart, n, o16, sms, st);
+                const int rc = narrow ? launch_group<true>(list, lpart, lwt, n, o16, sms, st)
+                                      : launch_group<false>(list, lpart, lwt, n, o16, sms, st);
                 if (rc != MQ_OK) return rc;
                 n = 0;
             }

@@ -14,7 +14,10 @@ bool tmajor_suits(const Problem &p);
 // o16); returns MQ_OK or MQ_ERR_CUDA.  part[i] nonzero (part may be null):
 // problem i is a slice of a split K whose y is an int32 [M][ldy] buffer of
 // its raw sums sum (x - zx)(w - zw), requantized later by launch_splitk_reduce.
-int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *part = nullptr);
+// wt[i] nonzero (wt may be null): problem i's w is stored transposed, int8
+// [K][N] with ldw bytes between k-rows (not with part).
+int launch_tmajor(const Problem *probs, int count, void *stream, const uint8_t *part = nullptr,
+                  const uint8_t *wt = nullptr);
 
 // One split problem's combine: y = requant(sum of the S slices' int32 sums,
 // part + s M N, s < S) with M0 / shift / zy (+ residual for int8 outputs).

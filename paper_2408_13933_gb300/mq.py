@@ -58,7 +58,7 @@ class LinearDesc(ctypes.Structure):
                 ("ldx", _i32), ("ldy", _i32), ("zx", _i32), ("zy", _i32), ("bits", _i32),
                 ("abits", _i32), ("obits", _i32), ("ldw", _i32),
                 ("wdynamic", _i32), ("wsq", _vp), ("y16", _vp), ("ysq", _vp), ("x16", _vp),
-                ("xsq", _vp)]
+                ("xsq", _vp), ("wt", _i32)]
 
 
 class FoldDesc(ctypes.Structure):
@@ -373,7 +373,7 @@ def linear_w4a8_noalloc(x, zx: int, packed, colsum, n: int, m0, shift, zy: int, 
 def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
               ldx=None, ldy=None, m=None, k=None, zw=None, abits=None, obits=None,
               ldw: int = 0, wdynamic: bool = False, wsq=None, y16=None, ysq=None, x16=None,
-              xsq=None) -> LinearDesc:
+              xsq=None, wt: bool = False) -> LinearDesc:
     """One mq_linear_desc; `zw` (device int32 [N]) gives asymmetric weights;
     abits 16 (default: 16 for an int16 x) gives int16 activations and outputs;
     obits 16 with int8 x (default: 16 for an int16 y) an int16 output; `ldw`
@@ -382,7 +382,8 @@ def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
     (device int32 [N], weight_sq_sums) the weights' sums of squares; `y16` /
     `ysq` (device f16 [M, N] / zero-filled int32 [M]) receive y as f16 and its
     row sums of squares, `x16` / `xsq` pass those of an earlier call as this
-    call's x (chained layers, see mq.h)."""
+    call's x (chained layers, see mq.h); `wt` says `packed` holds the weights
+    transposed, int8 [K][N] with `ldw` bytes between k-rows (see mq.h)."""
     d = LinearDesc()
     if abits is None:
         abits = 16 if getattr(x, "element_size", lambda: 1)() == 2 else 8
@@ -392,6 +393,7 @@ def make_desc(x, zx, packed, colsum, n, m0, shift, zy, y, bits, residual=None,
     d.obits = int(obits)
     d.ldw = int(ldw)
     d.wdynamic = int(bool(wdynamic))
+    d.wt = int(bool(wt))
     d.x, d.packed, d.colsum = _ptr(x), _ptr(packed), _ptr(colsum)
     d.M0, d.shift, d.residual, d.y = _ptr(m0), _ptr(shift), _ptr(residual), _ptr(y)
     d.zw = _ptr(zw)

@@ -2,7 +2,8 @@
 16-bit output (scores ahead of the 16-bit softmax), weights read through a
 row pitch (a head's slice of a projection output), row sums of activation
 matrices used as colsum, the int8 transpose, and grouped-query attention's
-Q K^T (int16 scores) and P V (int8) through the batch call."""
+Q K^T (int16 scores) and P V (int8) through the batch call, P V also with V
+read in place as transposed weights."""
 import numpy as np
 import pytest
 
@@ -210,6 +211,54 @@ def test_grouped_query_attention_matmuls(t_q):
                                  zw=np.full(D, zv, np.int32))
             assert_equal_int8(outs[r][:, h * D:(h + 1) * D].cpu().numpy(), want,
                               f"round {r} P V head {h}")
+
+
+@pytest.mark.parametrize("t_q", [200, 1024])
+def test_pv_reads_v_in_place(t_q):
+    # O_h = P_h V_g with V_g read where it lies ([T][G d], head g at columns
+    # g d, transposed weights through V's row pitch): no transpose, no row
+    # sums.  Three rounds rewrite the same V buffer on the stream just before
+    # each call (weights written on the device), all enqueued back to back.
+    torch = torch_cuda()
+    lib = mq()
+    rng = np.random.default_rng(23 + t_q)
+    T, H, G, D, R = 320, 8, 2, 64, 3
+    rep = H // G
+    i8 = lambda *s: rng.integers(-128, 128, size=s, dtype=np.int16).astype(np.int8)
+    vs, ps = [i8(T, G * D) for _ in range(R)], [i8(H, t_q, T) for _ in range(R)]
+    zp, zv = 9, -17
+    vds, pds = [upload(a) for a in vs], [upload(a) for a in ps]
+    m0o, sho, zyo = np.full(D, 1 << 30, np.int32), np.full(D, 40, np.int32), -3
+    dev = [upload(a) for a in (m0o, sho, np.full(D, zv, np.int32))]
+    m0od, shod, zwv = dev
+    vbuf = torch.empty((T, G * D), dtype=torch.int8, device="cuda")
+    outs = [torch.full((t_q, H * D), 9, dtype=torch.int8, device="cuda") for _ in range(R)]
+    keep = vds + pds + dev + [vbuf] + outs
+    arrs = []
+    for r in range(R):
+        do = [lib.make_desc(pds[r][h], zp, vbuf[:, (h // rep) * D:], None, D, m0od, shod, zyo,
+                            outs[r][:, h * D:(h + 1) * D], 8, zw=zwv, ldw=G * D,
+                            wdynamic=True, wt=True) for h in range(H)]
+        arrs.append((lib.LinearDesc * H)(*do))
+    need = lib.workspace_size_batch(list(arrs[0]))
+    assert need == 0
+    torch.cuda.synchronize()
+    sp = torch.cuda.current_stream().cuda_stream
+    for r in range(R):
+        vbuf.copy_(vds[r])
+        assert lib.lib.mq_linear_batch(arrs[r], H, None, 0, sp) == 0
+    torch.cuda.synchronize()
+    assert lib.check_device_status() == 0
+    for r in range(R):
+        for h in range(H):
+            g = h // rep
+            vtg = np.ascontiguousarray(vs[r][:, g * D:(g + 1) * D].T)
+            opk, _ = oracle.pack(vtg, 8)
+            want = oracle.linear(np.ascontiguousarray(ps[r][h]), zp, opk, 8, D, m0o, sho, zyo,
+                                 zw=np.full(D, zv, np.int32))
+            assert_equal_int8(outs[r][:, h * D:(h + 1) * D].cpu().numpy(), want,
+                              f"round {r} P V head {h}")
+    del keep
 
 
 @pytest.mark.parametrize("m", [3, 140])

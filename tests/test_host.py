@@ -429,6 +429,37 @@ def test_colsum_optional_with_int8_weights(mq):
                                  FAKE, 1 << 30, None) == mq.MQ_ERR_INVALID_ARG
 
 
+def test_transposed_weights_checks_on_host(mq):
+    # weights stored [K][N] (wt): int8 weights with 8-bit activations, k-rows
+    # of at least N bytes (16-byte multiples), prefill shapes the token-major
+    # kernel serves; every rejection happens before anything is launched, and
+    # such descriptors need neither row sums nor a widened input
+    def rc(d):
+        return mq.lib.mq_linear_batch((mq.LinearDesc * 1)(d), 1, FAKE, 1 << 30, None)
+
+    def wt(M=300, K=512, N=64, bits=8, **kw):
+        d = _desc(mq, M, K, N, bits, True)
+        d.colsum = None
+        d.wt = 1
+        for k, v in kw.items():
+            setattr(d, k, v)
+        return d
+    assert rc(wt(bits=4)) == mq.MQ_ERR_INVALID_ARG
+    assert rc(wt(abits=16)) == mq.MQ_ERR_INVALID_ARG
+    assert rc(wt(N=64, ldw=48)) == mq.MQ_ERR_INVALID_ARG          # ldw < N
+    assert rc(wt(ldw=72)) == mq.MQ_ERR_ALIGNMENT
+    assert rc(wt(M=4)) == mq.MQ_ERR_UNSUPPORTED_SHAPE             # decode shape
+    assert rc(wt(N=40)) == mq.MQ_ERR_UNSUPPORTED_SHAPE            # k-rows of 40 bytes
+    assert rc(wt(packed=FAKE + 8, ldw=64)) == mq.MQ_ERR_ALIGNMENT
+    assert mq.test_tmajor_kernel(2) == 0                          # kernel forbidden
+    try:
+        assert rc(wt()) == mq.MQ_ERR_UNSUPPORTED_SHAPE
+    finally:
+        assert mq.test_tmajor_kernel(0) == 0
+    assert mq.workspace_size_batch([wt(M=2048, K=2048, N=2048)]) == 0
+    assert mq.workspace_size_batch([wt(N=40, ldw=48)]) == 0
+
+
 def test_fold_batch_argument_checks_on_host(mq):
     # count limits and an empty batch, before anything is launched
     many = (mq.FoldDesc * (mq.MQ_FOLD_MAX_JOBS + 1))()

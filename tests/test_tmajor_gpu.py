@@ -4,8 +4,9 @@ shape by its test hook: wide tiles (one exact run, 256 channels) and narrow
 ones (64 channels, several runs with and without a weight zero point), int8
 output with and without the residual, int16 output, ragged tokens, channels
 and K, extreme codes at the exact-run bound, rows that take the scalar store
-path, a batch over more problems than one launch holds, and the automatic
-choice (K <= 128 or N <= 64) against the other kernels' bytes."""
+path, a batch over more problems than one launch holds, the automatic
+choice (K <= 128 or N <= 64) against the other kernels' bytes, and weights
+stored transposed ([K][N] inside wider rows, as attention's V)."""
 import numpy as np
 import pytest
 
@@ -196,3 +197,69 @@ def test_tmajor_choice_matches_other_kernels(shape):
         outs.append(c.got())
     assert_equal(outs[0], outs[1], f"auto vs never {shape}")
     assert_equal(outs[0], c.want(), f"oracle {shape}")
+
+
+class WtCase(Case):
+    """A Case whose weights are stored transposed: int8 [K][N] at column `col`
+    of rows `ldw` bytes apart (attention's V_g read in place), the other
+    columns holding codes the kernel must not read."""
+
+    def __init__(self, seed, m, k, n, ldw=None, col=0, **kw):
+        super().__init__(seed, m, k, n, **kw)
+        self.ldw = ldw or n
+        self.col = col
+        wt = np.full((k, self.ldw), 55, np.int8)
+        wt[:, col:col + n] = self.c.w.T
+        self.wt_dev = upload(wt)
+
+    def desc(self):
+        c = self.c
+        x, _, _, m0, sh = self.keep
+        return mq().make_desc(x, c.zx, self.wt_dev[:, self.col:], None, c.N, m0, sh, self.zy,
+                              self.y, 8, residual=self.dres, zw=self.dzw, ldw=self.ldw, wt=True)
+
+
+WT_SHAPES = [(200, 64, 1024, 64, 0),     # one narrow tile column, one run at its bound
+             (130, 96, 2048, 96, 0),     # ragged second channel tile, two runs
+             (40, 48, 3024, 48, 0),      # a ragged last stage
+             (300, 100, 320, 128, 0),    # ragged rows: N inside a 128-byte pitch
+             (1024, 64, 1024, 256, 64)]  # attention: V_1 of four KV heads
+
+
+@pytest.mark.parametrize("zw", [False, True], ids=["sym", "zw"])
+@pytest.mark.parametrize("shape", WT_SHAPES, ids=lambda s: "x".join(map(str, s)))
+def test_tmajor_transposed_weights(shape, zw):
+    m, n, k, ldw, col = shape
+    c = WtCase(3 * m + k, m, k, n, ldw=ldw, col=col, zw=zw)
+    run([c])
+    assert_equal(c.got(), c.want(), f"wt {shape} zw={zw}")
+
+
+@pytest.mark.parametrize("o16", [False, True], ids=["int8-residual", "int16"])
+def test_tmajor_transposed_weights_outputs(o16):
+    m, n, k = 256, 80, 1104
+    c = WtCase(17, m, k, n, ldw=96, zw=True, o16=o16, residual=not o16)
+    run([c])
+    assert_equal(c.got(), c.want(), f"wt outputs o16={o16}")
+
+
+@pytest.mark.parametrize("extreme", ["min", "max", "mixed"])
+def test_tmajor_transposed_weights_extreme(extreme):
+    m, n, k = 70, 64, 2048
+    c = WtCase(47, m, k, n, extreme=extreme)
+    run([c])
+    assert_equal(c.got(), c.want(), f"wt extreme {extreme}")
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_tmajor_transposed_weights_in_a_mixed_batch(mode):
+    # transposed and row-major weights in one call (one narrow launch holds
+    # both kinds, beside a wide one); with the automatic choice a transposed
+    # problem of long K and many channels still takes the token-major kernel
+    lib = mq()
+    assert lib.test_tmajor_kernel(mode) == 0
+    cases = [WtCase(71, 300, 512, 256, zw=True), Case(72, 200, 1024, 64, zw=True),
+             WtCase(73, 140, 640, 64, ldw=128, col=64), Case(74, 260, 64, 300)]
+    run(cases)
+    for i, c in enumerate(cases):
+        assert_equal(c.got(), c.want(), f"mixed batch problem {i} mode {mode}")
