@@ -305,15 +305,18 @@ int mq_workspace_size_a16(int M, int N, int K, int bits, size_t *bytes);
  * mq_workspace_size_batch; rounded up to 128 bytes).  For weights written on
  * the device every call (keys, V^T in attention) this replaces a separate
  * row-sum launch.  The single-linear calls still require colsum.
- * Transposed weights (`wt`, int8 weights with 8-bit activations): `packed`
- * holds w[n][k] at packed[k * ldw + n], i.e. an activation matrix [K][N] such
- * as V in attention's P V (its head-g columns with ldw = the row pitch of V),
- * read without a transpose.  Only the token-major kernel reads this layout:
- * such a descriptor must be a prefill shape (M > 16) that kernel can serve (x
- * and packed 16-byte aligned, ldx and ldw multiples of 16, no residual with an
- * int16 output); otherwise, or with the token-major kernel forbidden
- * (mq_test_tmajor_kernel), the call returns MQ_ERR_UNSUPPORTED_SHAPE before
- * anything is launched.  colsum is not read (the kernel folds the zero points).
+ * Transposed weights (`wt`, int8 weights with 8-bit activations, else
+ * MQ_ERR_INVALID_ARG): `packed` holds w[n][k] at packed[k * ldw + n], i.e. an
+ * activation matrix [K][N] such as V in attention's P V (its head-g columns
+ * with ldw = the row pitch of V), read without a transpose.  ldw is at least
+ * N (0 means N; smaller: MQ_ERR_INVALID_ARG) and, when given, a multiple of 16
+ * (else MQ_ERR_ALIGNMENT, as for unaligned x or packed).  Only the token-major
+ * kernel reads this layout: with K > 0 the descriptor must be a prefill shape
+ * (M > 16) that kernel can serve (rows of x and of packed 16-byte multiples, no
+ * residual with an int16 output); otherwise, or with the token-major kernel
+ * forbidden (mq_test_tmajor_kernel), the call returns MQ_ERR_UNSUPPORTED_SHAPE
+ * before anything is launched.  colsum is not read (the kernel folds the zero
+ * points).
  * Weights written on the device: the kernels read `packed` before waiting for
  * the previous kernel in the stream (see mq_linear_w8a8).  A descriptor whose
  * weights are produced by earlier work on the same stream (keys, or V^T from
